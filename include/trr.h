@@ -1,0 +1,177 @@
+/*
+ * trr.h - C ABI of the TriRoute serving hot path on GB300 (sm_103a).
+ *
+ * TriRoute (arxiv 2607.06601) routes every token, at every layer, with a policy
+ * pi_t = (a_t, e_t, b_t) (Sec. 3.1).  This library implements the inference-time
+ * consumer of two of its axes:
+ *   - a_t in {skip, local, full}: how much of the past the query reads
+ *     (Sec. 3.2(A), Eq. 2);
+ *   - b_t in {2, 4, 8, 16}: the bit-width at which the token's own K/V are written
+ *     to the cache for later queries (Sec. 3.2(C), Eq. 4; 16 = native bf16).
+ * At inference the decisions are hard (argmax), only the selected computation runs,
+ * and each token's KV is stored at its chosen width in a paged cache (Sec. 3.8).
+ * Sec. 7 names the two kernels a production system needs: mode-aware attention over
+ * ragged skip/local/full work, and a mixed-precision paged KV cache that groups tokens
+ * by precision.  Those are trr_decode_attn and trr_kv_append below.
+ *
+ * Conventions shared by every entry point
+ *   - Pointers marked "device" are CUDA device pointers on the current device; the
+ *     library never takes ownership of them.  "host" pointers are read before return.
+ *   - Every call is asynchronous and stream-ordered on `stream` (a cudaStream_t passed
+ *     as void*; NULL = legacy default stream).  No call synchronises the device except
+ *     trr_get_status and trr_destroy.
+ *   - Host-detectable errors (NULL pointers, sizes out of range, layer out of range)
+ *     return an error immediately and enqueue nothing.
+ *   - Device-detectable errors (see trr_kv_append / trr_decode_attn) are recorded in a
+ *     sticky device status word that keeps the FIRST error since it was last read;
+ *     trr_get_status reads and clears it.  No kernel traps or asserts.
+ *   - One stream at a time per cache: calls on the same cache must not overlap.
+ *
+ * Cache memory layout (fixed; the CPU oracle re-derives it independently)
+ *   class index c = 0,1,2,3 <-> b = 2,4,8,16.   P = page_size, d = head_dim,
+ *   G = group_size, Hkv = num_kv_heads, MP = ceil(max_context / P),
+ *   W32 = ceil(max_context / 32).
+ *   Metadata (int32 unless noted), all indexed [layer][seq]...:
+ *     last_pos  [L][S]          last position appended to (layer, seq), -1 if none
+ *     ntok      [L][S][4]       tokens of class c stored for (layer, seq)
+ *     presence  [L][S][W32] u32 bit (p % 32) of word p / 32 set <=> token p is stored
+ *     page_table[L][S][4][MP]   page ids of class c, in position order
+ *     page_first[L][S][4][MP]   position of the first token of each page
+ *     page_last [L][S][4][MP]   position of the last token of each page
+ *     next_page [4]             pages handed out so far per class (bump allocator)
+ *   Pools: class c holds pages_per_class[c] pages of PAGE_BYTES(b) bytes each:
+ *     HDR        = roundup(4 * P, 128)           header: int32 positions[P]
+ *     TOKB(b)    = 2*(d*b/8) + 2*(d/G)*4   (b < 16)  |  4*d   (b = 16)
+ *     SLICE(b)   = P * TOKB(b)                  one KV head of one page
+ *     PAGE_BYTES = roundup(HDR + Hkv * SLICE(b), 128)
+ *     head h starts at HDR + h * SLICE(b); inside it, for b < 16:
+ *       K codes [P][d*b/8] | V codes [P][d*b/8] | K sz [P][d/G][2] | V sz [P][d/G][2]
+ *     where sz = (scale, zero) as IEEE binary16, and for b = 16:
+ *       K [P][d] bf16 | V [P][d] bf16.
+ *   Code packing: element j of a head vector sits at byte floor(j*b/8), bit (j*b) % 8,
+ *   least significant bits first (2-bit codes 1,2,3,0 -> byte 0x39).
+ *   Page allocation: entries are taken in array order; an entry of class c whose
+ *   (layer, seq) has ntok % P == 0 opens page next_page[c]++ .
+ */
+#ifndef TRR_H
+#define TRR_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  TRR_OK = 0,
+  TRR_ERR_INVALID_ARG = 1,   /* bad pointer, size, enum value (bits, mode) or window */
+  TRR_ERR_OUT_OF_MEMORY = 2, /* cudaMalloc failed or caller pool too small */
+  TRR_ERR_OUT_OF_PAGES = 3,  /* a class pool is exhausted */
+  TRR_ERR_BAD_POSITION = 4,  /* position outside [0, max_context) or not increasing */
+  TRR_ERR_CUDA = 5,          /* a CUDA runtime call failed */
+  TRR_ERR_UNSUPPORTED = 6,   /* configuration outside the supported set */
+  TRR_ERR_BAD_VALUE = 7,     /* non-finite or |x| > 65504 value in a quantised group */
+  TRR_ERR_TIMEOUT = 8        /* a bounded wait inside a kernel gave up */
+} trr_status;
+
+enum { TRR_MODE_SKIP = 0, TRR_MODE_LOCAL = 1, TRR_MODE_FULL = 2 }; /* a_t, Eq. 2 */
+
+typedef struct trr_cache_config {
+  int32_t num_layers;      /* L >= 1 */
+  int32_t max_seqs;        /* S >= 1: sequence ids are 0 .. S-1 */
+  int32_t num_q_heads;     /* Hq, a multiple of num_kv_heads */
+  int32_t num_kv_heads;    /* Hkv >= 1 */
+  int32_t head_dim;        /* d: 64 or 128 */
+  int32_t group_size;      /* G: 32, 64 or 128 with G <= d (quantiser group along d) */
+  int32_t page_size;       /* P: 16, 32 or 64 tokens */
+  int32_t max_context;     /* positions are 0 .. max_context-1 */
+  int32_t pages_per_class[4]; /* pool capacity for b = 2, 4, 8, 16 */
+  int32_t max_append;      /* largest n accepted by trr_kv_append */
+  int32_t max_queries;     /* largest n accepted by trr_decode_attn */
+  int32_t split_bytes;     /* target KV bytes per split-K work item; 0 = 16384 */
+  int32_t skip_writes_kv;  /* 0: a skip token stores no KV (default); 1: it stores KV */
+  void* pool;              /* device memory of >= trr_cache_required_bytes, or NULL */
+  uint64_t pool_bytes;     /* size of `pool` (ignored when pool is NULL) */
+} trr_cache_config;
+
+typedef struct trr_cache trr_cache; /* opaque */
+
+/* Bytes of device memory a cache with this configuration needs (metadata, scratch
+ * and the four page pools).  Returns TRR_ERR_UNSUPPORTED / TRR_ERR_INVALID_ARG for a
+ * configuration outside the supported set. */
+trr_status trr_cache_required_bytes(const trr_cache_config* cfg, uint64_t* bytes);
+
+/* Create a cache on the current device.  With cfg->pool == NULL the library
+ * cudaMallocs the memory and frees it in trr_destroy; otherwise it carves everything
+ * out of the caller's buffer (>= trr_cache_required_bytes, 256-byte aligned), which
+ * must outlive the cache.  All metadata starts empty.  Synchronous. */
+trr_status trr_create_cache(const trr_cache_config* cfg, trr_cache** out);
+
+/* Quantise-on-write append (Sec. 3.2(C), Eq. 4; Sec. 3.8).
+ *   n entries, taken in array order; entry i is token positions[i] of sequence
+ *   seq_ids[i] at `layer`, with K/V rows k[i][Hkv][d], v[i][Hkv][d] (bf16, device,
+ *   contiguous), bit-width bits[i] in {2,4,8,16} and attention mode modes[i].
+ *   A skip token (modes[i] == 0) stores nothing unless skip_writes_kv == 1.
+ *   For b < 16 each group of G consecutive elements of a head vector is stored as
+ *     z = fp16(min x),  s = fp16(fl32(fl32(max x - min x) / (2^b - 1))),
+ *     c_j = clamp(rne(fl32(fl32(x_j - z) / s)), 0, 2^b - 1)   (c_j = 0 when s == 0)
+ *   with fl32 = IEEE binary32 round-to-nearest-even; b = 16 stores the bf16 bits.
+ *   seq_ids, positions, k, v, bits, modes: device arrays; 0 <= n <= max_append.
+ *   Device-detected errors: seq id out of range or bits/mode not allowed
+ *   (INVALID_ARG), a position outside [0, max_context) or not above the sequence's
+ *   last one (BAD_POSITION), a pool running out (OUT_OF_PAGES).  Any of these makes
+ *   the whole call a no-op and records the error of the lowest failing index.
+ *   A quantised group holding a non-finite value or |x| > 65504 is stored as zeros
+ *   and records BAD_VALUE; the rest of the call takes effect. */
+trr_status trr_kv_append(trr_cache* cache, int32_t layer, int32_t n,
+                         const int32_t* seq_ids, const int32_t* positions,
+                         const void* k_bf16, const void* v_bf16,
+                         const uint8_t* bits, const uint8_t* modes, void* stream);
+
+/* Mode-routed split-K decode attention over the mixed-precision cache (Eq. 2).
+ *   n queries; query i belongs to sequence seq_ids[i] at position t = q_positions[i],
+ *   has rows q[i][Hq][d] (bf16, device) and mode modes[i]:
+ *     skip : out row = 0
+ *     local: softmax attention over the stored tokens j with t-w+1 <= j <= t,
+ *            w = windows[i] (or window_scalar when windows == NULL), w >= 1
+ *     full : softmax attention over the stored tokens j <= t.
+ *   Query head h reads KV head h / (Hq / Hkv).  Scores are softmax_scale * q.k
+ *   (softmax_scale <= 0 means 1/sqrt(d)) with K/V dequantised as z + c*s; fp32
+ *   accumulation, bf16 (round-to-nearest-even) output out[i][Hq][d] (device).
+ *   A query with no stored token in range gets a zero row.
+ *   Device-detected errors (seq id, mode or window invalid: INVALID_ARG; position
+ *   outside [0, max_context): BAD_POSITION) zero that query's row and record the
+ *   error of the lowest failing index; other queries are computed.
+ *   seq_ids, q_positions, q, modes, windows, out: device; 0 <= n <= max_queries. */
+trr_status trr_decode_attn(trr_cache* cache, int32_t layer, int32_t n,
+                           const int32_t* seq_ids, const int32_t* q_positions,
+                           const void* q_bf16, const uint8_t* modes,
+                           const int32_t* windows, int32_t window_scalar,
+                           float softmax_scale, void* out_bf16, void* stream);
+
+/* Free library-owned memory (waits for the device first).  A caller pool is not
+ * freed.  NULL is accepted. */
+trr_status trr_destroy(trr_cache* cache);
+
+/* Read and clear the sticky device status (synchronises `stream`). */
+trr_status trr_get_status(trr_cache* cache, void* stream);
+
+/* Forget every sequence of every layer and return all pages to the pools
+ * (stream-ordered; metadata only, page bytes are not cleared). */
+trr_status trr_reset(trr_cache* cache, void* stream);
+
+/* Location of one layout region inside the cache's device memory, for inspection:
+ * 0 last_pos, 1 ntok, 2 presence, 3 page_table, 4 page_first, 5 page_last,
+ * 6 next_page, 7..10 pools of b = 2, 4, 8, 16.  *ptr is a device pointer. */
+trr_status trr_get_region(const trr_cache* cache, int32_t region, void** ptr,
+                          uint64_t* bytes);
+
+/* Number of SMs and kernels the last trr_decode_attn / trr_kv_append launched
+ * (host-side bookkeeping, no synchronisation). */
+int32_t trr_last_launch_count(const trr_cache* cache);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* TRR_H */

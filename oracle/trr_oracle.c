@@ -1,0 +1,551 @@
+/*
+ * trr_oracle.c - plain, slow, fp64 CPU oracle for the TriRoute serving path.
+ *
+ * TEST INFRASTRUCTURE ONLY.  Only tests/, __graft_entry__.smoke() and bench.py's
+ * cpu_baseline / reference leg load this file's library.  It shares no source, header,
+ * table or helper with the CUDA library; it re-derives the documented cache layout on
+ * its own.  Every step follows the paper in order, with no blocking or fusion:
+ *
+ *   - quantiser Q_b (Sec. 3.2(C), Eq. 4): z = min(x), s = (max(x) - min(x)) / (2^b - 1),
+ *     codes round((x - z) / s), stored code c dequantises to z + c*s; b = 16 keeps
+ *     the native value.  Readings where the paper is silent: min/max are taken per
+ *     group of G elements along the head dimension; s and z are stored as IEEE
+ *     binary16; s, the difference x - z and the quotient are each rounded to IEEE
+ *     binary32 (fl32) before round-half-to-even and a clamp to [0, 2^b - 1];
+ *     native precision is bf16.
+ *   - attention modes (Sec. 3.2(A), Eq. 2): skip -> 0; local -> softmax attention over
+ *     the last w positions t-w+1..t (w keys, the reading the cost model
+ *     kappa_local ~ 2 d min(t, w) of Sec. 3.5 and Appendix C fixes); full -> over
+ *     all positions <= t.  Only stored tokens take part.
+ *   - hard decisions at inference, KV stored at the chosen width, paged cache
+ *     (Sec. 3.8); grouping tokens by precision (Sec. 7) -> one width class per page.
+ *
+ * Floating point: fl32(op) is computed as a double operation followed by a cast to
+ * float.  For +, -, * and / of binary32 operands this double rounding is innocuous
+ * (53 >= 2*24 + 2), so it equals a single binary32 round-to-nearest-even.
+ * Attention is computed entirely in double.
+ *
+ * Parity status: every function here is pinned by tests (see tests/test_oracle_*.py).
+ */
+#include <fenv.h>
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#define ORC_OK 0
+#define ORC_INVALID_ARG 1
+#define ORC_OUT_OF_MEMORY 2
+#define ORC_OUT_OF_PAGES 3
+#define ORC_BAD_POSITION 4
+#define ORC_UNSUPPORTED 6
+#define ORC_BAD_VALUE 7
+
+static const int BITS_OF_CLASS[4] = {2, 4, 8, 16};
+
+typedef struct orc_cache {
+  int L, S, Hq, Hkv, d, G, P, maxctx, skip_writes_kv, no_pool;
+  int cap[4];
+  int MP, W32;
+  int32_t* last_pos;   /* [L][S] */
+  int32_t* ntok;       /* [L][S][4] */
+  uint32_t* presence;  /* [L][S][W32] */
+  int32_t* page_table; /* [L][S][4][MP] */
+  int32_t* page_first; /* [L][S][4][MP] */
+  int32_t* page_last;  /* [L][S][4][MP] */
+  int32_t next_page[4];
+  int64_t hdr, tokb[4], slice[4], page_bytes[4];
+  uint8_t* pool[4];
+} orc_cache;
+
+/* ------------------------------------------------------------------ numbers -- */
+
+double orc_bf16_to_double(uint16_t h) {
+  uint32_t u = (uint32_t)h << 16;
+  float f;
+  memcpy(&f, &u, 4);
+  return (double)f;
+}
+
+/* IEEE binary16: 1 sign, 5 exponent (bias 15), 10 fraction bits. */
+double orc_f16_to_double(uint16_t h) {
+  int sign = (h >> 15) & 1, e = (h >> 10) & 31, m = h & 1023;
+  double v;
+  if (e == 0)
+    v = ldexp((double)m, -24);
+  else if (e == 31)
+    v = m ? NAN : INFINITY;
+  else
+    v = ldexp((double)(1024 + m), e - 25);
+  return sign ? -v : v;
+}
+
+/* Round a finite double to the nearest binary16, ties to even. */
+uint16_t orc_double_to_f16(double x) {
+  uint16_t sign = (x < 0 || (x == 0 && signbit(x))) ? 0x8000 : 0;
+  double a = fabs(x);
+  if (a == 0) return sign;
+  if (a < ldexp(1.0, -14)) { /* subnormal range: quantum 2^-24 */
+    double r = nearbyint(ldexp(a, 24));
+    return (uint16_t)(sign | (uint16_t)r); /* r == 1024 encodes the smallest normal */
+  }
+  int E;
+  frexp(a, &E);                   /* a = f * 2^E, f in [0.5, 1) */
+  double r = nearbyint(ldexp(a, 11 - E)); /* significand scaled to [1024, 2048] */
+  if (r == 2048) { r = 1024; E += 1; }
+  int biased = (E - 1) + 15;
+  if (biased >= 31) return (uint16_t)(sign | 0x7C00); /* overflow -> inf */
+  return (uint16_t)(sign | (biased << 10) | ((int)r - 1024));
+}
+
+static double fl32(double x) { return (double)(float)x; }
+
+/* -------------------------------------------------------------- quantiser -- */
+
+/* Eq. 4 for one group of G bf16 values: writes binary16 bits of s and z and one
+ * unpacked code per element.  Returns 1 (and all zeros) when the group holds a
+ * non-finite value or one with |x| > 65504, which binary16 cannot carry. */
+int orc_quantize_group(const uint16_t* x, int G, int b, uint16_t* s16, uint16_t* z16,
+                       uint8_t* codes) {
+  int i;
+  double mn = INFINITY, mx = -INFINITY;
+  for (i = 0; i < G; i++) {
+    double xi = orc_bf16_to_double(x[i]);
+    if (!isfinite(xi) || fabs(xi) > 65504.0) {
+      *s16 = 0;
+      *z16 = 0;
+      memset(codes, 0, (size_t)G);
+      return 1;
+    }
+    if (xi < mn) mn = xi;
+    if (xi > mx) mx = xi;
+  }
+  int levels = (1 << b) - 1;
+  uint16_t zb = orc_double_to_f16(mn);                 /* z = min(x) */
+  double range = fl32(mx - mn);                         /* max(x) - min(x) */
+  uint16_t sb = orc_double_to_f16(fl32(range / (double)levels)); /* s */
+  double z = orc_f16_to_double(zb), s = orc_f16_to_double(sb);
+  for (i = 0; i < G; i++) {
+    int c = 0;
+    if (s != 0) {
+      double u = fl32(fl32(orc_bf16_to_double(x[i]) - z) / s); /* (x - z) / s */
+      double r = nearbyint(u);                                  /* round, ties even */
+      if (r < 0) r = 0;
+      if (r > levels) r = levels;
+      c = (int)r;
+    }
+    codes[i] = (uint8_t)c;
+  }
+  *s16 = sb;
+  *z16 = zb;
+  return 0;
+}
+
+/* Pack n codes of b bits, least significant bits first. */
+void orc_pack_codes(const uint8_t* codes, int n, int b, uint8_t* out) {
+  int j;
+  memset(out, 0, (size_t)(n * b / 8));
+  for (j = 0; j < n; j++) {
+    int bit = j * b;
+    out[bit / 8] |= (uint8_t)(codes[j] << (bit % 8));
+  }
+}
+
+static int unpack_code(const uint8_t* packed, int j, int b) {
+  int bit = j * b;
+  return (packed[bit / 8] >> (bit % 8)) & ((1 << b) - 1);
+}
+
+/* ------------------------------------------------------------------ layout -- */
+
+static int64_t roundup(int64_t x, int64_t a) { return (x + a - 1) / a * a; }
+
+static int class_of_bits(int b) {
+  int c;
+  for (c = 0; c < 4; c++)
+    if (BITS_OF_CLASS[c] == b) return c;
+  return -1;
+}
+
+static int64_t idx_ls(const orc_cache* o, int l, int s) { return (int64_t)l * o->S + s; }
+static int64_t idx_lsc(const orc_cache* o, int l, int s, int c) {
+  return idx_ls(o, l, s) * 4 + c;
+}
+static int64_t idx_pt(const orc_cache* o, int l, int s, int c, int k) {
+  return idx_lsc(o, l, s, c) * o->MP + k;
+}
+
+static uint8_t* page_ptr(const orc_cache* o, int c, int id) {
+  return o->pool[c] + (int64_t)id * o->page_bytes[c];
+}
+
+/* cfg: L, S, Hq, Hkv, d, G, P, max_context, cap[4], skip_writes_kv, no_pool.
+ * With no_pool = 1 only metadata and nothing of the page bytes is kept. */
+int orc_create(const int32_t* cfg, orc_cache** out) {
+  int c;
+  *out = NULL;
+  if (fegetround() != FE_TONEAREST) return ORC_UNSUPPORTED;
+  orc_cache* o = (orc_cache*)calloc(1, sizeof(orc_cache));
+  if (!o) return ORC_OUT_OF_MEMORY;
+  o->L = cfg[0]; o->S = cfg[1]; o->Hq = cfg[2]; o->Hkv = cfg[3];
+  o->d = cfg[4]; o->G = cfg[5]; o->P = cfg[6]; o->maxctx = cfg[7];
+  for (c = 0; c < 4; c++) o->cap[c] = cfg[8 + c];
+  o->skip_writes_kv = cfg[12];
+  o->no_pool = cfg[13];
+  if (o->L < 1 || o->S < 1 || o->Hkv < 1 || o->Hq < o->Hkv || o->Hq % o->Hkv ||
+      (o->d != 64 && o->d != 128) || (o->G != 32 && o->G != 64 && o->G != 128) ||
+      o->G > o->d || (o->P != 16 && o->P != 32 && o->P != 64) || o->maxctx < 1 ||
+      o->cap[0] < 0 || o->cap[1] < 0 || o->cap[2] < 0 || o->cap[3] < 0) {
+    free(o);
+    return ORC_UNSUPPORTED;
+  }
+  o->MP = (o->maxctx + o->P - 1) / o->P;
+  o->W32 = (o->maxctx + 31) / 32;
+  o->hdr = roundup(4 * (int64_t)o->P, 128);
+  for (c = 0; c < 4; c++) {
+    int b = BITS_OF_CLASS[c];
+    o->tokb[c] = b < 16 ? 2 * (o->d * b / 8) + 2 * (o->d / o->G) * 4 : 4 * o->d;
+    o->slice[c] = o->P * o->tokb[c];
+    o->page_bytes[c] = roundup(o->hdr + o->Hkv * o->slice[c], 128);
+  }
+  int64_t nls = (int64_t)o->L * o->S;
+  o->last_pos = (int32_t*)malloc(sizeof(int32_t) * nls);
+  o->ntok = (int32_t*)calloc((size_t)(nls * 4), sizeof(int32_t));
+  o->presence = (uint32_t*)calloc((size_t)(nls * o->W32), sizeof(uint32_t));
+  o->page_table = (int32_t*)malloc(sizeof(int32_t) * nls * 4 * o->MP);
+  o->page_first = (int32_t*)malloc(sizeof(int32_t) * nls * 4 * o->MP);
+  o->page_last = (int32_t*)malloc(sizeof(int32_t) * nls * 4 * o->MP);
+  int fail = !o->last_pos || !o->ntok || !o->presence || !o->page_table ||
+             !o->page_first || !o->page_last;
+  for (c = 0; c < 4 && !fail && !o->no_pool; c++) {
+    o->pool[c] = (uint8_t*)calloc((size_t)(o->cap[c] > 0 ? o->cap[c] : 1),
+                                  (size_t)o->page_bytes[c]);
+    if (!o->pool[c]) fail = 1;
+  }
+  *out = o;
+  if (fail) return ORC_OUT_OF_MEMORY;
+  int64_t i;
+  for (i = 0; i < nls; i++) o->last_pos[i] = -1;
+  for (i = 0; i < nls * 4 * o->MP; i++) {
+    o->page_table[i] = -1;
+    o->page_first[i] = -1;
+    o->page_last[i] = -1;
+  }
+  return ORC_OK;
+}
+
+void orc_destroy(orc_cache* o) {
+  int c;
+  if (!o) return;
+  free(o->last_pos); free(o->ntok); free(o->presence);
+  free(o->page_table); free(o->page_first); free(o->page_last);
+  for (c = 0; c < 4; c++) free(o->pool[c]);
+  free(o);
+}
+
+/* ------------------------------------------------------------------ append -- */
+
+/* Checks of one entry against the running state, in the documented order.
+ * tmp_last / tmp_ntok / tmp_next describe the cache as if earlier entries of this
+ * call had been applied. */
+static int check_entry(const orc_cache* o, int seq, int pos, int bits, int mode,
+                       const int32_t* tmp_last, const int32_t* tmp_ntok,
+                       const int32_t* tmp_next) {
+  if (seq < 0 || seq >= o->S) return ORC_INVALID_ARG;
+  int c = class_of_bits(bits);
+  if (c < 0) return ORC_INVALID_ARG;
+  if (mode < 0 || mode > 2) return ORC_INVALID_ARG;
+  if (pos < 0 || pos >= o->maxctx) return ORC_BAD_POSITION;
+  if (pos <= tmp_last[seq]) return ORC_BAD_POSITION;
+  if (mode == 0 && !o->skip_writes_kv) return ORC_OK;
+  if (tmp_ntok[seq * 4 + c] % o->P == 0 && tmp_next[c] >= o->cap[c]) return ORC_OUT_OF_PAGES;
+  return ORC_OK;
+}
+
+static void write_row(orc_cache* o, uint8_t* page, int c, int slot, int h,
+                      const uint16_t* krow, const uint16_t* vrow, int* bad) {
+  int b = BITS_OF_CLASS[c], d = o->d, G = o->G, P = o->P;
+  uint8_t* sl = page + o->hdr + (int64_t)h * o->slice[c];
+  if (b == 16) {
+    memcpy(sl + (int64_t)slot * d * 2, krow, (size_t)d * 2);
+    memcpy(sl + (int64_t)P * d * 2 + (int64_t)slot * d * 2, vrow, (size_t)d * 2);
+    return;
+  }
+  int rowb = d * b / 8, ng = d / G, which, g;
+  uint8_t codes[128];
+  for (which = 0; which < 2; which++) { /* 0 = K, 1 = V */
+    const uint16_t* x = which ? vrow : krow;
+    uint8_t* crow = sl + (int64_t)which * P * rowb + (int64_t)slot * rowb;
+    uint8_t* szrow = sl + 2 * (int64_t)P * rowb + (int64_t)which * P * ng * 4 +
+                     (int64_t)slot * ng * 4;
+    for (g = 0; g < ng; g++) {
+      uint16_t s16, z16;
+      *bad |= orc_quantize_group(x + g * G, G, b, &s16, &z16, codes);
+      orc_pack_codes(codes, G, b, crow + g * G * b / 8);
+      memcpy(szrow + g * 4, &s16, 2); /* little-endian host, as on the GPU */
+      memcpy(szrow + g * 4 + 2, &z16, 2);
+    }
+  }
+}
+
+int orc_append(orc_cache* o, int layer, int n, const int32_t* seq_ids,
+               const int32_t* positions, const uint16_t* k, const uint16_t* v,
+               const uint8_t* bits, const uint8_t* modes) {
+  int i, c;
+  if (layer < 0 || layer >= o->L || n < 0) return ORC_INVALID_ARG;
+  if (n == 0) return ORC_OK;
+  /* pass 1: validate every entry in order against a scratch copy of the state */
+  int32_t* tmp_last = (int32_t*)malloc(sizeof(int32_t) * o->S);
+  int32_t* tmp_ntok = (int32_t*)malloc(sizeof(int32_t) * o->S * 4);
+  int32_t tmp_next[4];
+  if (!tmp_last || !tmp_ntok) { free(tmp_last); free(tmp_ntok); return ORC_OUT_OF_MEMORY; }
+  memcpy(tmp_last, o->last_pos + idx_ls(o, layer, 0), sizeof(int32_t) * o->S);
+  memcpy(tmp_ntok, o->ntok + idx_lsc(o, layer, 0, 0), sizeof(int32_t) * o->S * 4);
+  memcpy(tmp_next, o->next_page, sizeof(tmp_next));
+  for (i = 0; i < n; i++) {
+    int e = check_entry(o, seq_ids[i], positions[i], bits[i], modes[i], tmp_last,
+                        tmp_ntok, tmp_next);
+    if (e != ORC_OK) { free(tmp_last); free(tmp_ntok); return e; }
+    tmp_last[seq_ids[i]] = positions[i];
+    if (modes[i] == 0 && !o->skip_writes_kv) continue;
+    c = class_of_bits(bits[i]);
+    if (tmp_ntok[seq_ids[i] * 4 + c] % o->P == 0) tmp_next[c]++;
+    tmp_ntok[seq_ids[i] * 4 + c]++;
+  }
+  free(tmp_last);
+  free(tmp_ntok);
+  /* pass 2: apply */
+  int bad = 0;
+  int64_t row = (int64_t)o->Hkv * o->d;
+  for (i = 0; i < n; i++) {
+    int s = seq_ids[i], pos = positions[i];
+    o->last_pos[idx_ls(o, layer, s)] = pos;
+    if (modes[i] == 0 && !o->skip_writes_kv) continue; /* skip: no KV entry */
+    c = class_of_bits(bits[i]);
+    int32_t* nt = &o->ntok[idx_lsc(o, layer, s, c)];
+    int kidx = *nt / o->P, slot = *nt % o->P;
+    if (slot == 0) {
+      o->page_table[idx_pt(o, layer, s, c, kidx)] = o->next_page[c]++;
+      o->page_first[idx_pt(o, layer, s, c, kidx)] = pos;
+    }
+    o->page_last[idx_pt(o, layer, s, c, kidx)] = pos;
+    (*nt)++;
+    o->presence[idx_ls(o, layer, s) * o->W32 + pos / 32] |= 1u << (pos % 32);
+    if (o->no_pool) continue;
+    uint8_t* page = page_ptr(o, c, o->page_table[idx_pt(o, layer, s, c, kidx)]);
+    int32_t p32 = pos;
+    memcpy(page + 4 * slot, &p32, 4);
+    int h;
+    for (h = 0; h < o->Hkv; h++)
+      write_row(o, page, c, slot, h, k + i * row + (int64_t)h * o->d,
+                v + i * row + (int64_t)h * o->d, &bad);
+  }
+  return bad ? ORC_BAD_VALUE : ORC_OK;
+}
+
+/* ---------------------------------------------------------------- dequant -- */
+
+/* Dequantised K and V (head h) of the token in `slot` of a class-c page. */
+static void dequant_slot(const orc_cache* o, const uint8_t* page, int c, int slot, int h,
+                         double* kout, double* vout) {
+  int b = BITS_OF_CLASS[c], d = o->d, G = o->G, P = o->P, j, which;
+  const uint8_t* sl = page + o->hdr + (int64_t)h * o->slice[c];
+  for (which = 0; which < 2; which++) {
+    double* outv = which ? vout : kout;
+    if (b == 16) {
+      const uint8_t* r = sl + (int64_t)which * P * d * 2 + (int64_t)slot * d * 2;
+      for (j = 0; j < d; j++) {
+        uint16_t h16;
+        memcpy(&h16, r + 2 * j, 2);
+        outv[j] = orc_bf16_to_double(h16);
+      }
+      continue;
+    }
+    int rowb = d * b / 8, ng = d / G;
+    const uint8_t* crow = sl + (int64_t)which * P * rowb + (int64_t)slot * rowb;
+    const uint8_t* szrow = sl + 2 * (int64_t)P * rowb + (int64_t)which * P * ng * 4 +
+                           (int64_t)slot * ng * 4;
+    for (j = 0; j < d; j++) {
+      uint16_t s16, z16;
+      memcpy(&s16, szrow + (j / G) * 4, 2);
+      memcpy(&z16, szrow + (j / G) * 4 + 2, 2);
+      outv[j] = orc_f16_to_double(z16) + unpack_code(crow, j, b) * orc_f16_to_double(s16);
+    }
+  }
+}
+
+static int tokens_in_page(const orc_cache* o, int layer, int s, int c, int kidx) {
+  int nt = o->ntok[idx_lsc(o, layer, s, c)];
+  int left = nt - kidx * o->P;
+  return left < o->P ? left : o->P;
+}
+
+static int32_t slot_position(const uint8_t* page, int slot) {
+  int32_t p;
+  memcpy(&p, page + 4 * slot, 4);
+  return p;
+}
+
+/* Dequantised K/V of position pos of (layer, seq), KV head h.  Returns the class index
+ * of the stored token, or -1 when the token is not stored. */
+int orc_dequant_token(const orc_cache* o, int layer, int s, int pos, int h, double* kout,
+                      double* vout) {
+  int c, kidx, slot;
+  if (o->no_pool) return -1;
+  for (c = 0; c < 4; c++) {
+    int np = (o->ntok[idx_lsc(o, layer, s, c)] + o->P - 1) / o->P;
+    for (kidx = 0; kidx < np; kidx++) {
+      const uint8_t* page = page_ptr(o, c, o->page_table[idx_pt(o, layer, s, c, kidx)]);
+      int fill = tokens_in_page(o, layer, s, c, kidx);
+      for (slot = 0; slot < fill; slot++)
+        if (slot_position(page, slot) == pos) {
+          dequant_slot(o, page, c, slot, h, kout, vout);
+          return c;
+        }
+    }
+  }
+  return -1;
+}
+
+/* --------------------------------------------------------------- attention -- */
+
+typedef struct { int c, kidx; } page_ref;
+
+static uint64_t lcg_next(uint64_t* st) {
+  *st = *st * 6364136223846793005ULL + 1442695040888963407ULL;
+  return *st >> 33;
+}
+
+/* Eq. 2 for every query; out is [n][Hq][d] doubles.  order_seed != 0 visits the pages
+ * (and the slots inside each page) in a pseudo-random order instead of page-table
+ * order, which must not change the result beyond fp64 rounding. */
+int orc_decode_attn(const orc_cache* o, int layer, int n, const int32_t* seq_ids,
+                    const int32_t* q_positions, const uint16_t* q, const uint8_t* modes,
+                    const int32_t* windows, int window_scalar, double scale,
+                    uint64_t order_seed, double* out) {
+  int i, h, j, status = ORC_OK;
+  if (layer < 0 || layer >= o->L || n < 0) return ORC_INVALID_ARG;
+  if (o->no_pool) return ORC_UNSUPPORTED;
+  int d = o->d, group = o->Hq / o->Hkv;
+  if (scale <= 0) scale = 1.0 / sqrt((double)d);
+  page_ref* refs = (page_ref*)malloc(sizeof(page_ref) * 4 * (o->MP + 1));
+  double* score = (double*)malloc(sizeof(double) * (o->maxctx + 1));
+  double* kv = (double*)malloc(sizeof(double) * 2 * d);
+  double* acc = (double*)malloc(sizeof(double) * d);
+  double* qd = (double*)malloc(sizeof(double) * d);
+  if (!refs || !score || !kv || !acc || !qd) {
+    free(refs); free(score); free(kv); free(acc); free(qd);
+    return ORC_OUT_OF_MEMORY;
+  }
+  for (i = 0; i < n; i++) {
+    double* orow = out + (int64_t)i * o->Hq * d;
+    int s = seq_ids[i], t = q_positions[i], mode = modes[i];
+    int w = windows ? windows[i] : window_scalar;
+    int err = ORC_OK;
+    if (s < 0 || s >= o->S || mode < 0 || mode > 2) err = ORC_INVALID_ARG;
+    else if (t < 0 || t >= o->maxctx) err = ORC_BAD_POSITION;
+    else if (mode == 1 && w < 1) err = ORC_INVALID_ARG;
+    for (j = 0; j < o->Hq * d; j++) orow[j] = 0.0;
+    if (err != ORC_OK) {
+      if (status == ORC_OK) status = err;
+      continue;
+    }
+    if (mode == 0) continue; /* Attn^skip = 0 */
+    int lo = mode == 2 ? 0 : (t - w + 1 > 0 ? t - w + 1 : 0);
+    /* the pages of this (layer, seq), all classes */
+    int nref = 0, c, kidx;
+    for (c = 0; c < 4; c++) {
+      int np = (o->ntok[idx_lsc(o, layer, s, c)] + o->P - 1) / o->P;
+      for (kidx = 0; kidx < np; kidx++) {
+        refs[nref].c = c;
+        refs[nref].kidx = kidx;
+        nref++;
+      }
+    }
+    uint64_t st = order_seed;
+    if (order_seed) { /* Fisher-Yates shuffle of the visiting order */
+      for (j = nref - 1; j > 0; j--) {
+        int r = (int)(lcg_next(&st) % (uint64_t)(j + 1));
+        page_ref tmp = refs[j];
+        refs[j] = refs[r];
+        refs[r] = tmp;
+      }
+    }
+    for (h = 0; h < o->Hq; h++) {
+      int kvh = h / group, r, nk = 0, slot;
+      for (j = 0; j < d; j++) qd[j] = orc_bf16_to_double(q[((int64_t)i * o->Hq + h) * d + j]);
+      /* pass 1: scores of the stored keys lo <= j <= t, and their maximum */
+      double mx = -INFINITY;
+      for (r = 0; r < nref; r++) {
+        int cc = refs[r].c, kk = refs[r].kidx;
+        const uint8_t* page = page_ptr(o, cc, o->page_table[idx_pt(o, layer, s, cc, kk)]);
+        int fill = tokens_in_page(o, layer, s, cc, kk);
+        for (slot = 0; slot < fill; slot++) {
+          int sl = order_seed ? fill - 1 - slot : slot;
+          int32_t pos = slot_position(page, sl);
+          if (pos < lo || pos > t) continue;
+          dequant_slot(o, page, cc, sl, kvh, kv, kv + d);
+          double dot = 0;
+          for (j = 0; j < d; j++) dot += qd[j] * kv[j];
+          score[nk] = scale * dot;
+          if (score[nk] > mx) mx = score[nk];
+          nk++;
+        }
+      }
+      if (nk == 0) continue; /* no stored token in range: zero row */
+      /* pass 2: softmax weights and the weighted sum of V */
+      double denom = 0;
+      for (j = 0; j < d; j++) acc[j] = 0;
+      nk = 0;
+      for (r = 0; r < nref; r++) {
+        int cc = refs[r].c, kk = refs[r].kidx;
+        const uint8_t* page = page_ptr(o, cc, o->page_table[idx_pt(o, layer, s, cc, kk)]);
+        int fill = tokens_in_page(o, layer, s, cc, kk);
+        for (slot = 0; slot < fill; slot++) {
+          int sl = order_seed ? fill - 1 - slot : slot;
+          int32_t pos = slot_position(page, sl);
+          if (pos < lo || pos > t) continue;
+          dequant_slot(o, page, cc, sl, kvh, kv, kv + d);
+          double p = exp(score[nk] - mx);
+          denom += p;
+          for (j = 0; j < d; j++) acc[j] += p * kv[d + j];
+          nk++;
+        }
+      }
+      for (j = 0; j < d; j++) orow[(int64_t)h * d + j] = acc[j] / denom;
+    }
+  }
+  free(refs); free(score); free(kv); free(acc); free(qd);
+  return status;
+}
+
+/* -------------------------------------------------------------- inspection -- */
+
+/* Region ids as in the library's documented layout: 0 last_pos, 1 ntok, 2 presence,
+ * 3 page_table, 4 page_first, 5 page_last, 6 next_page, 7..10 pools (b = 2,4,8,16).
+ * Returns the region's size in bytes and its host pointer. */
+int64_t orc_region(orc_cache* o, int id, void** ptr) {
+  int64_t nls = (int64_t)o->L * o->S;
+  switch (id) {
+    case 0: *ptr = o->last_pos; return 4 * nls;
+    case 1: *ptr = o->ntok; return 16 * nls;
+    case 2: *ptr = o->presence; return 4 * nls * o->W32;
+    case 3: *ptr = o->page_table; return 16 * nls * o->MP;
+    case 4: *ptr = o->page_first; return 16 * nls * o->MP;
+    case 5: *ptr = o->page_last; return 16 * nls * o->MP;
+    case 6: *ptr = o->next_page; return 16;
+    case 7: case 8: case 9: case 10:
+      *ptr = o->pool[id - 7];
+      return o->pool[id - 7] ? (int64_t)o->cap[id - 7] * o->page_bytes[id - 7] : 0;
+    default: *ptr = NULL; return -1;
+  }
+}
+
+/* Layout sizes: which = 0 header bytes, 1..4 slice bytes of class 0..3,
+ * 5..8 page bytes of class 0..3. */
+int64_t orc_layout(const orc_cache* o, int which) {
+  if (which == 0) return o->hdr;
+  if (which >= 1 && which <= 4) return o->slice[which - 1];
+  if (which >= 5 && which <= 8) return o->page_bytes[which - 5];
+  return -1;
+}
