@@ -59,6 +59,12 @@
 #include <stddef.h>
 #include <stdint.h>
 
+#if defined(__GNUC__)
+#define TRR_API __attribute__((visibility("default")))
+#else
+#define TRR_API
+#endif
+
 #ifdef __cplusplus
 extern "C" {
 #endif
@@ -100,13 +106,13 @@ typedef struct trr_cache trr_cache; /* opaque */
 /* Bytes of device memory a cache with this configuration needs (metadata, scratch
  * and the four page pools).  Returns TRR_ERR_UNSUPPORTED / TRR_ERR_INVALID_ARG for a
  * configuration outside the supported set. */
-trr_status trr_cache_required_bytes(const trr_cache_config* cfg, uint64_t* bytes);
+TRR_API trr_status trr_cache_required_bytes(const trr_cache_config* cfg, uint64_t* bytes);
 
 /* Create a cache on the current device.  With cfg->pool == NULL the library
  * cudaMallocs the memory and frees it in trr_destroy; otherwise it carves everything
  * out of the caller's buffer (>= trr_cache_required_bytes, 256-byte aligned), which
  * must outlive the cache.  All metadata starts empty.  Synchronous. */
-trr_status trr_create_cache(const trr_cache_config* cfg, trr_cache** out);
+TRR_API trr_status trr_create_cache(const trr_cache_config* cfg, trr_cache** out);
 
 /* Quantise-on-write append (Sec. 3.2(C), Eq. 4; Sec. 3.8).
  *   n entries, taken in array order; entry i is token positions[i] of sequence
@@ -124,7 +130,7 @@ trr_status trr_create_cache(const trr_cache_config* cfg, trr_cache** out);
  *   the whole call a no-op and records the error of the lowest failing index.
  *   A quantised group holding a non-finite value or |x| > 65504 is stored as zeros
  *   and records BAD_VALUE; the rest of the call takes effect. */
-trr_status trr_kv_append(trr_cache* cache, int32_t layer, int32_t n,
+TRR_API trr_status trr_kv_append(trr_cache* cache, int32_t layer, int32_t n,
                          const int32_t* seq_ids, const int32_t* positions,
                          const void* k_bf16, const void* v_bf16,
                          const uint8_t* bits, const uint8_t* modes, void* stream);
@@ -144,7 +150,7 @@ trr_status trr_kv_append(trr_cache* cache, int32_t layer, int32_t n,
  *   outside [0, max_context): BAD_POSITION) zero that query's row and record the
  *   error of the lowest failing index; other queries are computed.
  *   seq_ids, q_positions, q, modes, windows, out: device; 0 <= n <= max_queries. */
-trr_status trr_decode_attn(trr_cache* cache, int32_t layer, int32_t n,
+TRR_API trr_status trr_decode_attn(trr_cache* cache, int32_t layer, int32_t n,
                            const int32_t* seq_ids, const int32_t* q_positions,
                            const void* q_bf16, const uint8_t* modes,
                            const int32_t* windows, int32_t window_scalar,
@@ -152,24 +158,24 @@ trr_status trr_decode_attn(trr_cache* cache, int32_t layer, int32_t n,
 
 /* Free library-owned memory (waits for the device first).  A caller pool is not
  * freed.  NULL is accepted. */
-trr_status trr_destroy(trr_cache* cache);
+TRR_API trr_status trr_destroy(trr_cache* cache);
 
 /* Read and clear the sticky device status (synchronises `stream`). */
-trr_status trr_get_status(trr_cache* cache, void* stream);
+TRR_API trr_status trr_get_status(trr_cache* cache, void* stream);
 
 /* Forget every sequence of every layer and return all pages to the pools
  * (stream-ordered; metadata only, page bytes are not cleared). */
-trr_status trr_reset(trr_cache* cache, void* stream);
+TRR_API trr_status trr_reset(trr_cache* cache, void* stream);
 
 /* Location of one layout region inside the cache's device memory, for inspection:
  * 0 last_pos, 1 ntok, 2 presence, 3 page_table, 4 page_first, 5 page_last,
  * 6 next_page, 7..10 pools of b = 2, 4, 8, 16.  *ptr is a device pointer. */
-trr_status trr_get_region(const trr_cache* cache, int32_t region, void** ptr,
+TRR_API trr_status trr_get_region(const trr_cache* cache, int32_t region, void** ptr,
                           uint64_t* bytes);
 
 /* Number of SMs and kernels the last trr_decode_attn / trr_kv_append launched
  * (host-side bookkeeping, no synchronisation). */
-int32_t trr_last_launch_count(const trr_cache* cache);
+TRR_API int32_t trr_last_launch_count(const trr_cache* cache);
 
 #ifdef __cplusplus
 }

@@ -1,0 +1,245 @@
+// trr_append.cu - trr_kv_append: quantise-on-write into the width-class page pools.
+//
+// Two kernels per call:
+//   append_plan_kernel   one CTA, one thread per entry.  Validates every entry, ranks
+//                        it among the earlier entries of its (sequence, class), hands
+//                        out page ids in entry order, and commits the metadata only
+//                        when the whole call is valid (Sec. 3.8: each token's KV is
+//                        stored at its chosen width in a paged cache).
+//   append_write_kernel  one thread per (entry, KV head, K|V, group): the quantiser
+//                        Q_b of Sec. 3.2(C), Eq. 4, or a bf16 copy for b = 16.
+#include <climits>
+
+#include "trr_internal.cuh"
+
+namespace trr {
+
+__device__ __forceinline__ int class_of_bits(int b) {
+  return b == 2 ? 0 : b == 4 ? 1 : b == 8 ? 2 : b == 16 ? 3 : -1;
+}
+
+__global__ void __launch_bounds__(1024) append_plan_kernel(LayerArgs a, int n, const int32_t* __restrict__ seq_ids,
+                                                           const int32_t* __restrict__ positions,
+                                                           const uint8_t* __restrict__ bits,
+                                                           const uint8_t* __restrict__ modes) {
+  __shared__ int s_seq[1024];
+  __shared__ int s_pos[1024];
+  __shared__ int s_cls[1024];   // width class when the entry stores KV, else -1
+  __shared__ int s_open[1024];  // class of the page the entry opens, else -1
+  __shared__ int s_first_err;
+  __shared__ int s_nopen[kClasses];
+
+  const int e = threadIdx.x;
+  const bool act = e < n;
+  int seq = -1, pos = 0, c = -1, err = 0;
+  bool writes = false;
+  if (act) {
+    seq = seq_ids[e];
+    pos = positions[e];
+    const int m = modes[e];
+    if (seq < 0 || seq >= a.S) {
+      err = TRR_ERR_INVALID_ARG;
+    } else {
+      c = class_of_bits(bits[e]);
+      if (c < 0 || m > TRR_MODE_FULL) err = TRR_ERR_INVALID_ARG;
+      else if (pos < 0 || pos >= a.maxctx) err = TRR_ERR_BAD_POSITION;
+    }
+    writes = !err && (m != TRR_MODE_SKIP || a.skip_writes_kv);
+  }
+  s_seq[e] = (act && seq >= 0 && seq < a.S) ? seq : -1;
+  s_pos[e] = pos;
+  s_cls[e] = writes ? c : -1;
+  if (e == 0) s_first_err = INT_MAX;
+  if (e < kClasses) s_nopen[e] = 0;
+  __syncthreads();
+
+  // Earlier entries of the same sequence: the largest position and, per class, how
+  // many store KV.  Later ones: whether this entry is the sequence's / class's last.
+  int prev_max = -1, rank = 0;
+  bool later_seq = false, later_cls = false;
+  if (act && s_seq[e] >= 0) {
+    for (int j = 0; j < n; ++j) {
+      if (s_seq[j] != seq) continue;
+      if (j < e) {
+        prev_max = max(prev_max, s_pos[j]);
+        rank += (writes && s_cls[j] == c);
+      } else if (j > e) {
+        later_seq = true;
+        later_cls |= (writes && s_cls[j] == c);
+      }
+    }
+  }
+  int k = 0, slot = 0, kidx = 0;
+  bool opens = false;
+  if (act && !err && pos <= max(prev_max, a.last_pos[seq])) err = TRR_ERR_BAD_POSITION;
+  if (act && !err && writes) {
+    k = a.ntok[seq * 4 + c] + rank;
+    slot = k % a.P;
+    kidx = k / a.P;
+    opens = slot == 0;
+  }
+  s_open[e] = opens ? c : -1;
+  __syncthreads();
+
+  int pid = -1;
+  if (opens) {  // page ids in entry order: next_page + openers of this class before e
+    int before = 0;
+    for (int j = 0; j < e; ++j) before += (s_open[j] == c);
+    pid = a.ctrl[kNextPage + c] + before;
+    if (pid >= a.cap[c]) err = TRR_ERR_OUT_OF_PAGES;
+  }
+  if (act && err) atomicMin(&s_first_err, e);
+  __syncthreads();
+  if (s_first_err != INT_MAX) {  // the call is a no-op; record the lowest failing entry
+    if (e == s_first_err) set_status(a.ctrl, err);
+    if (e == 0) a.ctrl[kAppendOk] = 0;
+    return;
+  }
+
+  // Commit.  Openers first, so that later entries of the same page can read its id.
+  const int64_t row = (static_cast<int64_t>(seq) * 4 + c) * a.MP + kidx;
+  if (opens) {
+    a.pt[row] = pid;
+    a.pfirst[row] = pos;
+    atomicAdd(&s_nopen[c], 1);
+  }
+  __syncthreads();
+  if (act) {
+    AppendPlan p{-1, 0, 0, pos};
+    if (writes) {
+      if (!opens) pid = a.pt[row];
+      p.page = pid;
+      p.slot = slot;
+      p.cls = c;
+      if (!later_cls || slot == a.P - 1) a.plast[row] = pos;
+      if (!later_cls) a.ntok[seq * 4 + c] = k + 1;
+      reinterpret_cast<int32_t*>(a.pool[c] + pid * a.page_bytes[c])[slot] = pos;
+      atomicOr(&a.presence[static_cast<int64_t>(seq) * a.W32 + pos / 32], 1u << (pos % 32));
+    }
+    a.aplan[e] = p;
+    if (!later_seq) a.last_pos[seq] = pos;
+  }
+  __syncthreads();
+  if (e < kClasses) a.ctrl[kNextPage + e] += s_nopen[e];
+  if (e == 0) a.ctrl[kAppendOk] = 1;
+}
+
+__device__ __forceinline__ float bf16lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+
+// Eq. 4 on 32 consecutive values (one chunk of a group): codes packed LSB-first.
+template <int B>
+__device__ __forceinline__ void quantise_chunk(const uint4* src, float z, float s, uint32_t* dst) {
+  constexpr int levels = (1 << B) - 1;
+  constexpr int per_word = 32 / B;
+  uint32_t words[B];
+#pragma unroll
+  for (int w = 0; w < B; ++w) words[w] = 0;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const uint4 u = src[q];
+    const uint32_t wv[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int h = 0; h < 8; ++h) {
+      const float x = (h & 1) ? bf16hi(wv[h >> 1]) : bf16lo(wv[h >> 1]);
+      int code = 0;
+      if (s != 0.f) {
+        const float u32 = __fdiv_rn(__fsub_rn(x, z), s);
+        code = min(max(__float2int_rn(u32), 0), levels);
+      }
+      const int j = q * 8 + h;
+      words[j / per_word] |= static_cast<uint32_t>(code) << ((j % per_word) * B);
+    }
+  }
+#pragma unroll
+  for (int w = 0; w < B; ++w) dst[w] = words[w];
+}
+
+__global__ void __launch_bounds__(256) append_write_kernel(LayerArgs a, int n, const uint16_t* __restrict__ k,
+                                                           const uint16_t* __restrict__ v) {
+  if (a.ctrl[kAppendOk] == 0) return;
+  const int ng = a.d / a.G;
+  const int per_entry = a.Hkv * 2 * ng;
+  const int64_t gid = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (gid >= static_cast<int64_t>(n) * per_entry) return;
+  const int e = static_cast<int>(gid / per_entry);
+  const int r = static_cast<int>(gid % per_entry);
+  const int h = r / (2 * ng);
+  const int which = (r / ng) & 1;  // 0 = K, 1 = V
+  const int g = r % ng;
+  const AppendPlan p = a.aplan[e];
+  if (p.page < 0) return;
+  const int b = bits_of_class(p.cls);
+  const uint16_t* src = (which ? v : k) + (static_cast<int64_t>(e) * a.Hkv + h) * a.d + g * a.G;
+  uint8_t* sl = a.pool[p.cls] + p.page * a.page_bytes[p.cls] + a.hdr + static_cast<int64_t>(h) * a.slice[p.cls];
+  const uint4* s4 = reinterpret_cast<const uint4*>(src);
+  if (b == 16) {  // native precision: copy the bf16 bits
+    uint4* dst = reinterpret_cast<uint4*>(sl + static_cast<int64_t>(which) * a.P * a.d * 2 +
+                                          static_cast<int64_t>(p.slot) * a.d * 2 + g * a.G * 2);
+    for (int i = 0; i < a.G / 8; ++i) dst[i] = s4[i];
+    return;
+  }
+  // min / max of the group; values binary16 cannot carry make the group all zeros
+  float mn = __int_as_float(0x7f800000), mx = -mn;
+  bool bad = false;
+  for (int i = 0; i < a.G / 8; ++i) {
+    const uint4 u = s4[i];
+    const uint32_t wv[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int h2 = 0; h2 < 8; ++h2) {
+      const float x = (h2 & 1) ? bf16hi(wv[h2 >> 1]) : bf16lo(wv[h2 >> 1]);
+      bad |= !(fabsf(x) <= 65504.f);  // also true for NaN
+      mn = fminf(mn, x);
+      mx = fmaxf(mx, x);
+    }
+  }
+  const int rowb = a.d * b / 8;
+  uint32_t* codes = reinterpret_cast<uint32_t*>(sl + static_cast<int64_t>(which) * a.P * rowb +
+                                                static_cast<int64_t>(p.slot) * rowb + g * a.G * b / 8);
+  uint32_t* sz = reinterpret_cast<uint32_t*>(sl + 2 * static_cast<int64_t>(a.P) * rowb +
+                                             static_cast<int64_t>(which) * a.P * ng * 4 +
+                                             static_cast<int64_t>(p.slot) * ng * 4 + g * 4);
+  if (bad) {
+    for (int i = 0; i < a.G * b / 32; ++i) codes[i] = 0;
+    *sz = 0;
+    set_status(a.ctrl, TRR_ERR_BAD_VALUE);
+    return;
+  }
+  const __half z16 = __float2half_rn(mn);                                   // z = min(x)
+  const float levels = static_cast<float>((1 << b) - 1);
+  const __half s16 = __float2half_rn(__fdiv_rn(__fsub_rn(mx, mn), levels));  // s
+  const float z = __half2float(z16), s = __half2float(s16);
+  for (int q = 0; q < a.G / 32; ++q) {
+    uint32_t* dst = codes + q * b;  // 32 codes of b bits = b words
+    if (b == 2) quantise_chunk<2>(s4 + 4 * q, z, s, dst);
+    else if (b == 4) quantise_chunk<4>(s4 + 4 * q, z, s, dst);
+    else quantise_chunk<8>(s4 + 4 * q, z, s, dst);
+  }
+  *sz = static_cast<uint32_t>(__half_as_ushort(s16)) | (static_cast<uint32_t>(__half_as_ushort(z16)) << 16);
+}
+
+}  // namespace trr
+
+using namespace trr;
+
+extern "C" trr_status trr_kv_append(trr_cache* cache, int32_t layer, int32_t n, const int32_t* seq_ids,
+                                    const int32_t* positions, const void* k_bf16, const void* v_bf16,
+                                    const uint8_t* bits, const uint8_t* modes, void* stream) {
+  if (!cache) return TRR_ERR_INVALID_ARG;
+  const Layout& l = cache_layout(cache);
+  if (layer < 0 || layer >= l.L || n < 0 || n > l.max_append) return TRR_ERR_INVALID_ARG;
+  cache_set_launches(cache, 0);
+  if (n == 0) return TRR_OK;
+  if (!seq_ids || !positions || !k_bf16 || !v_bf16 || !bits || !modes) return TRR_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(k_bf16) | reinterpret_cast<uintptr_t>(v_bf16)) & 15)
+    return TRR_ERR_INVALID_ARG;  // rows are read 16 bytes at a time
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const LayerArgs a = layer_args(l, cache_views(cache), layer);
+  const int threads = (n + 31) / 32 * 32;
+  append_plan_kernel<<<1, threads, 0, s>>>(a, n, seq_ids, positions, bits, modes);
+  const int64_t work = static_cast<int64_t>(n) * l.Hkv * 2 * (l.d / l.G);
+  append_write_kernel<<<static_cast<unsigned>((work + 255) / 256), 256, 0, s>>>(
+      a, n, static_cast<const uint16_t*>(k_bf16), static_cast<const uint16_t*>(v_bf16));
+  cache_set_launches(cache, 2);
+  return cudaGetLastError() == cudaSuccess ? TRR_OK : TRR_ERR_CUDA;
+}

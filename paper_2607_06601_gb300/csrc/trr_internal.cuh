@@ -1,0 +1,172 @@
+// trr_internal.cuh - layout arithmetic, kernel argument blocks and PTX helpers shared
+// by the library's translation units (trr_cache.cu, trr_append.cu, trr_attn.cu).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <stdint.h>
+
+#include "../../include/trr.h"
+
+namespace trr {
+
+constexpr int kClasses = 4;
+__host__ __device__ constexpr int bits_of_class(int c) { return c == 0 ? 2 : c == 1 ? 4 : c == 2 ? 8 : 16; }
+
+// Control words (int32) at the start of the cache memory.
+enum Ctrl : int {
+  kStatus = 0,        // sticky first error since the last trr_get_status
+  kNextPage = 4,      // [4] pages handed out per class
+  kWorkCounter = 8,   // attention: next work item to hand out
+  kAppendOk = 10,     // append: 1 when the plan kernel committed the call
+  kFirstBadQuery = 12,// attention: lowest failing query index (INT_MAX = none)
+  kCtrlInts = 64
+};
+
+// Byte layout of one cache (see include/trr.h for the documented part).
+struct Layout {
+  int L, S, Hq, Hkv, d, G, P, maxctx, MP, W32;
+  int cap[kClasses];
+  int max_append, max_queries, split_bytes, skip_writes_kv;
+  int units;      // attention work units per query (one per query head)
+  int s_cap;      // most splits one (query, unit) is cut into
+  int64_t max_items;
+  int64_t hdr, tokb[kClasses], slice[kClasses], page_bytes[kClasses];
+  int64_t off_ctrl, off_last_pos, off_ntok, off_presence, off_pt, off_pfirst, off_plast;
+  int64_t off_aplan, off_qplan, off_cnt, off_part, off_pool[kClasses], total;
+};
+
+// Per-query plan written by the attention plan kernel.
+struct QueryPlan {
+  int seq, lo, hi, nsplit;      // key range [lo, hi]; nsplit = 0: nothing to do
+  int first[kClasses];          // first page (index in the class page list) in range
+  int npages[kClasses];         // pages in range
+  int ntok[kClasses];           // tokens of the class stored for the sequence
+  int err, pad0, pad1, pad2;
+};
+static_assert(sizeof(QueryPlan) == 80, "QueryPlan is 80 bytes");
+
+// Per-entry plan written by the append plan kernel.
+struct AppendPlan {
+  int page;   // page id, -1 = nothing stored
+  int slot;   // slot in the page
+  int cls;    // width class
+  int pos;    // position
+};
+
+struct Views {  // typed device pointers into the cache memory
+  int32_t* ctrl;
+  int32_t* last_pos;
+  int32_t* ntok;
+  uint32_t* presence;
+  int32_t* pt;
+  int32_t* pfirst;
+  int32_t* plast;
+  AppendPlan* aplan;
+  QueryPlan* qplan;
+  int32_t* cnt;
+  float* part;
+  uint8_t* pool[kClasses];
+};
+
+inline Views make_views(const Layout& l, void* base) {
+  uint8_t* b = static_cast<uint8_t*>(base);
+  Views v;
+  v.ctrl = reinterpret_cast<int32_t*>(b + l.off_ctrl);
+  v.last_pos = reinterpret_cast<int32_t*>(b + l.off_last_pos);
+  v.ntok = reinterpret_cast<int32_t*>(b + l.off_ntok);
+  v.presence = reinterpret_cast<uint32_t*>(b + l.off_presence);
+  v.pt = reinterpret_cast<int32_t*>(b + l.off_pt);
+  v.pfirst = reinterpret_cast<int32_t*>(b + l.off_pfirst);
+  v.plast = reinterpret_cast<int32_t*>(b + l.off_plast);
+  v.aplan = reinterpret_cast<AppendPlan*>(b + l.off_aplan);
+  v.qplan = reinterpret_cast<QueryPlan*>(b + l.off_qplan);
+  v.cnt = reinterpret_cast<int32_t*>(b + l.off_cnt);
+  v.part = reinterpret_cast<float*>(b + l.off_part);
+  for (int c = 0; c < kClasses; ++c) v.pool[c] = b + l.off_pool[c];
+  return v;
+}
+
+// Everything a kernel needs about one layer of one cache, passed by value.
+struct LayerArgs {
+  int layer, S, Hq, Hkv, d, G, P, maxctx, MP, W32, units, s_cap, split_bytes, skip_writes_kv;
+  int cap[kClasses];
+  int hdr;
+  int slice[kClasses];
+  int64_t page_bytes[kClasses];
+  int32_t* ctrl;
+  int32_t* last_pos;   // this layer: [S]
+  int32_t* ntok;       // this layer: [S][4]
+  uint32_t* presence;  // this layer: [S][W32]
+  int32_t* pt;         // this layer: [S][4][MP]
+  int32_t* pfirst;
+  int32_t* plast;
+  AppendPlan* aplan;
+  QueryPlan* qplan;
+  int32_t* cnt;
+  float* part;
+  uint8_t* pool[kClasses];
+};
+
+LayerArgs layer_args(const Layout& l, const Views& v, int layer);
+
+// Accessors of the opaque cache (defined in trr_cache.cu).
+const Layout& cache_layout(const trr_cache* c);
+const Views& cache_views(const trr_cache* c);
+int cache_num_sms(const trr_cache* c);
+void cache_set_launches(trr_cache* c, int n);
+
+// ------------------------------------------------------------------ PTX helpers --
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void fence_barrier_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+               : "memory");
+}
+
+// 1-D bulk copy global -> shared (this CTA), completion counted on `bar`.
+// dst, src 16-byte aligned; bytes a multiple of 16.
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cta.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          smem_u32(dst)),
+      "l"(src), "r"(bytes), "r"(smem_u32(bar))
+      : "memory");
+}
+
+// Bounded wait for phase `parity` of `bar`: returns false when it gave up.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint32_t max_tries = 1u << 22) {
+  uint32_t addr = smem_u32(bar);
+  for (uint32_t i = 0; i < max_tries; ++i) {
+    uint32_t done;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+        : "=r"(done)
+        : "r"(addr), "r"(parity)
+        : "memory");
+    if (done) return true;
+  }
+  return false;
+}
+
+__device__ __forceinline__ void set_status(int32_t* ctrl, int code) {
+  atomicCAS(ctrl + kStatus, 0, code);
+}
+
+}  // namespace trr
