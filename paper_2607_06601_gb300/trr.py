@@ -173,13 +173,13 @@ class Cache:
 
     def __init__(self, num_layers, max_seqs, num_q_heads, num_kv_heads, head_dim, group_size,
                  page_size, max_context, pages_per_class, max_append=1024, max_queries=1024,
-                 split_bytes=0, skip_writes_kv=0, device=None):
+                 split_bytes=0, skip_writes_kv=0, device=None, zero_pool=False):
         self.cfg = make_config(num_layers, max_seqs, num_q_heads, num_kv_heads, head_dim,
                                group_size, page_size, max_context, pages_per_class, max_append,
                                max_queries, split_bytes, skip_writes_kv)
         self.nbytes = trr_cache_required_bytes(self.cfg)
-        self.pool = torch.empty(self.nbytes, dtype=torch.uint8,
-                                device=device or torch.cuda.current_device())
+        alloc = torch.zeros if zero_pool else torch.empty
+        self.pool = alloc(self.nbytes, dtype=torch.uint8, device=device or torch.cuda.current_device())
         self.handle = trr_create_cache(self.cfg, self.pool)
         self.L, self.S, self.Hq, self.Hkv = num_layers, max_seqs, num_q_heads, num_kv_heads
         self.d, self.G, self.P, self.max_context = head_dim, group_size, page_size, max_context

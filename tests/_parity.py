@@ -28,8 +28,8 @@ class Pair:
                  max_queries=1024, split_bytes=0, oracle_pool=True):
         self.gpu = trr.Cache(L, S, Hq, Hkv, d, G, P, maxctx, caps, max_append=max_append,
                              max_queries=max_queries, split_bytes=split_bytes,
-                             skip_writes_kv=skip_writes_kv)
-        self.gpu.pool.zero_()   # unused slots read back as zeros, as the oracle's calloc
+                             skip_writes_kv=skip_writes_kv, zero_pool=True)
+        # zero_pool: unused slots read back as zeros, as the oracle's calloc
         self.orc = oracle.OracleCache(L, S, Hq, Hkv, d, G, P, maxctx, caps,
                                       skip_writes_kv=skip_writes_kv, no_pool=not oracle_pool)
         self.Hq, self.Hkv, self.d, self.P = Hq, Hkv, d, P
