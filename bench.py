@@ -1,0 +1,651 @@
+#!/usr/bin/env python
+"""Decode-attention effective HBM GB/s of the TriRoute serving path on GB300.
+
+One step = one decode step of the whole hot path for one batch: at every layer, the
+batch's new tokens are appended (quantise-on-write at each token's bit-width) and each
+token's query attends in its own mode (skip / local / full) over the mixed-precision
+paged cache.  Default workload: the 160M-scale decoder (12 layers, MHA 12 x 64,
+batch 32, 2048-token contexts, window 256, seeded bit / mode mixes).
+
+The cache holds R replicas of the batch (R * 32 sequences with their own seeded maps);
+step i serves replica i % R, so each sequence grows by at most 32 tokens over the run
+and consecutive steps never re-read the same cache lines (every step moves more bytes
+than L2 holds).  Steps are captured as CUDA graphs; the timed region replays K of them.
+
+value  = algorithmic attention bytes of the K steps / device time of the K steps
+         (codes + fp16 scale/zero + slot positions + page-table entries of the stored
+         keys in each non-skip query's range, plus Q and O rows)
+e2e    = the same, through the C ABI with host buffers: pinned H2D of every step's
+         inputs and D2H of every step's outputs inside the timed region
+roofline: the dominant kernel is the trr_decode_attn call (plan + attention kernel);
+         achieved = its algorithmic bytes per call / its average duration from CUDA
+         event nodes placed around each call in a second, instrumented replay.
+"""
+from __future__ import annotations
+
+import argparse
+import ctypes
+import json
+import math
+import os
+import statistics
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "decode-attention effective HBM GB/s and % of GB300 peak; attended KV tokens/s"
+UNIT = "GB/s"
+PAGE = 16
+BITS = (2, 4, 8, 16)
+
+
+# --------------------------------------------------------------------------- bytes --
+
+def token_bytes(d, G):
+    """Bytes of one stored token of one KV head (K + V) per width class."""
+    return [2 * (d * b // 8) + 2 * (d // G) * 4 for b in BITS[:3]] + [4 * d]
+
+
+class Accounting:
+    """Algorithmic bytes / attended keys of decode queries, from the seeded maps."""
+
+    def __init__(self, spec, d, G, Hq, Hkv, window, P=PAGE):
+        self.tokb = np.array(token_bytes(d, G), dtype=np.int64)
+        self.Hq, self.Hkv, self.d, self.window, self.P = Hq, Hkv, d, window, P
+
+    def query(self, bits_row, modes_row, t):
+        """(bytes, attended keys, pages) of one query at position t of one sequence
+        (the token at t already appended)."""
+        m = int(modes_row[t])
+        qo = 2 * self.Hq * self.d
+        if m == 0:
+            return qo // 2, 0, 0                      # only the zero O row is written
+        lo = 0 if m == 2 else max(0, t - self.window + 1)
+        stored = modes_row[:t + 1] != 0
+        b_row = bits_row[:t + 1]
+        total, keys, pages = 2 * qo, 0, 0
+        for c, b in enumerate(BITS):
+            sel = stored & (b_row == b)
+            before = int(np.count_nonzero(sel[:lo]))
+            n_in = int(np.count_nonzero(sel[lo:]))
+            if n_in:
+                i0, i1 = before, before + n_in
+                pages += (i1 - 1) // self.P - i0 // self.P + 1
+            keys += n_in
+            total += n_in * (int(self.tokb[c]) * self.Hkv + 4)
+        total += 4 * pages
+        return total, keys, pages
+
+
+# ------------------------------------------------------------------ clocks (NVML) --
+
+class ClockSampler:
+    """Samples SM clock and clock-event reasons of this GPU while running."""
+    REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown",
+               0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown"}
+
+    def __init__(self, uuid: str | None, period_s=0.002):
+        self.samples, self.reasons, self.max_mhz = [], set(), None
+        self.period, self.ok = period_s, False
+        self._stop = threading.Event()
+        try:
+            self.nv = ctypes.CDLL("libnvidia-ml.so.1")
+            if self.nv.nvmlInit_v2() != 0:
+                return
+            self.h = ctypes.c_void_p()
+            if uuid:
+                r = self.nv.nvmlDeviceGetHandleByUUID(uuid.encode(), ctypes.byref(self.h))
+            else:
+                r = self.nv.nvmlDeviceGetHandleByIndex_v2(0, ctypes.byref(self.h))
+            if r != 0:
+                return
+            mx = ctypes.c_uint()
+            if self.nv.nvmlDeviceGetMaxClockInfo(self.h, 1, ctypes.byref(mx)) == 0:
+                self.max_mhz = int(mx.value)
+            self.ok = True
+        except OSError:
+            pass
+
+    def _run(self):
+        clk, rs = ctypes.c_uint(), ctypes.c_ulonglong()
+        get_rs = getattr(self.nv, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+            self.nv.nvmlDeviceGetCurrentClocksThrottleReasons
+        while not self._stop.is_set():
+            if self.nv.nvmlDeviceGetClockInfo(self.h, 1, ctypes.byref(clk)) == 0:
+                self.samples.append(int(clk.value))
+            if get_rs(self.h, ctypes.byref(rs)) == 0:
+                for bit, name in self.REASONS.items():
+                    if rs.value & bit:
+                        self.reasons.add(name)
+            time.sleep(self.period)
+
+    def __enter__(self):
+        if self.ok:
+            self._t = threading.Thread(target=self._run, daemon=True)
+            self._t.start()
+        return self
+
+    def __exit__(self, *a):
+        if self.ok:
+            self._stop.set()
+            self._t.join()
+
+    def summary(self):
+        if not self.samples:
+            return {"sm_mhz": None, "sm_max_mhz": self.max_mhz, "reasons": sorted(self.reasons),
+                    "samples": 0}
+        return {"sm_mhz": float(statistics.median(self.samples)), "sm_max_mhz": self.max_mhz,
+                "reasons": sorted(self.reasons), "samples": len(self.samples)}
+
+
+# ------------------------------------------------------- CUDA event nodes (cudart) --
+
+class CudaRt:
+    """cudaEventRecordWithFlags(External) places timing events inside captured graphs."""
+
+    def __init__(self):
+        lib = None
+        for name in ("libcudart.so.13", "libcudart.so", "/usr/local/cuda/lib64/libcudart.so"):
+            try:
+                lib = ctypes.CDLL(name)
+                break
+            except OSError:
+                continue
+        if lib is None:
+            raise RuntimeError("libcudart not found")
+        self.lib = lib
+        lib.cudaEventCreateWithFlags.argtypes = [ctypes.POINTER(ctypes.c_void_p), ctypes.c_uint]
+        lib.cudaEventRecordWithFlags.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_uint]
+        lib.cudaEventElapsedTime.argtypes = [ctypes.POINTER(ctypes.c_float), ctypes.c_void_p, ctypes.c_void_p]
+        lib.cudaEventDestroy.argtypes = [ctypes.c_void_p]
+
+    def event(self):
+        e = ctypes.c_void_p()
+        assert self.lib.cudaEventCreateWithFlags(ctypes.byref(e), 0) == 0
+        return e
+
+    def record_external(self, ev, stream_handle):
+        assert self.lib.cudaEventRecordWithFlags(ev, ctypes.c_void_p(stream_handle), 1) == 0
+
+    def elapsed_ms(self, a, b):
+        ms = ctypes.c_float()
+        assert self.lib.cudaEventElapsedTime(ctypes.byref(ms), a, b) == 0
+        return float(ms.value)
+
+
+# ------------------------------------------------------------------- the workload --
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            pk = json.load(f)
+        return float(pk["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return 6800.0, "fallback"
+
+
+def ncu_traffic(workload):
+    """Per-launch DRAM bytes of the attention kernel from the committed ncu summary,
+    if it was taken on the current kernel source (else None)."""
+    import hashlib
+    src = os.path.join(ROOT, "paper_2607_06601_gb300", "csrc", "trr_attn.cu")
+    digest = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    path = os.path.join(ROOT, "profiles", f"attn_kernel_{workload}_traffic.txt")
+    try:
+        kv = dict(line.split(":", 1) for line in open(path) if ":" in line)
+    except OSError:
+        return None
+    if kv.get("source_sha256_16", "").strip() != digest:
+        return None
+    try:
+        return float(kv["dram_bytes_per_call"])
+    except (KeyError, ValueError):
+        return None
+
+
+def _mix(*xs):
+    """A deterministic 31-bit seed from small integers."""
+    h = 0x9E3779B9
+    for x in xs:
+        h = (h * 1000003 + int(x) + 1) & 0xFFFFFFFFFFFF
+    return h & 0x7FFFFFFF
+
+
+class Bench:
+    def __init__(self, args, rank=0, world=1):
+        import torch
+        from paper_2607_06601_gb300 import trr, workloads as wl
+        self.torch, self.trr, self.wl = torch, trr, wl
+        spec = wl.SPECS[args.workload]
+        if args.batch:
+            spec = spec.with_(batch=args.batch)
+        if args.layers:
+            spec = spec.with_(num_layers=args.layers)
+        # each rank serves its own batches (weak scaling): a rank-specific seed
+        self.spec = spec.with_(seed=spec.seed + 1000 * rank)
+        self.args, self.rank, self.world = args, rank, world
+        s = self.spec
+        self.L, self.B, self.Hq, self.Hkv, self.d, self.G = (
+            s.num_layers, s.batch, s.num_q_heads, s.num_kv_heads, s.head_dim, s.group_size)
+        self.window = s.window
+        self.e2e_warm, self.e2e_steps = 2, min(args.steps, 20)
+        self.total_steps = args.warmup + 2 * args.steps + self.e2e_warm + self.e2e_steps
+        self.grow = 32                                   # tokens a sequence may grow
+        self.R = max(1, math.ceil(self.total_steps / self.grow))
+        self.acct = Accounting(s, self.d, self.G, self.Hq, self.Hkv, self.window)
+        self.ctx = wl.contexts(s)                       # prebuilt context per sequence
+        self.maxctx = int(self.ctx.max()) + math.ceil(self.total_steps / self.R) + 1
+        self.dev = torch.device("cuda", torch.cuda.current_device())
+
+    # ---- maps
+    def maps(self, layer, r):
+        wl = self.wl
+        bits = np.empty((self.B, self.maxctx), dtype=np.uint8)
+        modes = np.empty((self.B, self.maxctx), dtype=np.uint8)
+        spec = self.spec.with_(contexts=("fixed", self.maxctx))
+        for s in range(self.B):
+            bits[s], modes[s] = wl.policy(spec, layer, r * self.B + s, self.maxctx)
+        return bits, modes
+
+    def setup(self):
+        torch, trr = self.torch, self.trr
+        L, B, R = self.L, self.B, self.R
+        S = R * B
+        self.all_maps = [[self.maps(l, r) for r in range(R)] for l in range(L)]
+        caps = np.zeros(4, dtype=np.int64)
+        for l in range(L):
+            for r in range(R):
+                bits, modes = self.all_maps[l][r]
+                for s in range(B):
+                    stored = modes[s] != 0
+                    for c, b in enumerate(BITS):
+                        caps[c] += -(-int(np.count_nonzero(stored & (bits[s] == b))) // PAGE) + 1
+        self.cache = trr.Cache(L, S, self.Hq, self.Hkv, self.d, self.G, PAGE, self.maxctx,
+                               [int(c) for c in caps], max_append=1024, max_queries=max(B, 64))
+        # prebuild every sequence's context (untimed), K/V drawn on the device
+        gen = torch.Generator(device=self.dev)
+        self.prebuild_calls = 0
+        for l in range(L):
+            chl = torch.tensor(self.wl.outlier_channels(self.spec, l), dtype=torch.long, device=self.dev)
+            bits_d = torch.from_numpy(np.concatenate([self.all_maps[l][r][0] for r in range(R)])).to(self.dev)
+            modes_d = torch.from_numpy(np.concatenate([self.all_maps[l][r][1] for r in range(R)])).to(self.dev)
+            ctx = np.tile(self.ctx, R)
+            for p0 in range(0, int(ctx.max()), max(1, 1024 // S)):
+                p1 = min(int(ctx.max()), p0 + max(1, 1024 // S))
+                pos = torch.arange(p0, p1, device=self.dev, dtype=torch.int32)
+                seqs = torch.arange(S, device=self.dev, dtype=torch.int32)
+                pp, ss = torch.meshgrid(pos, seqs, indexing="ij")
+                keep = pp < torch.from_numpy(ctx).to(self.dev)[ss.long()]
+                pp, ss = pp[keep].contiguous(), ss[keep].contiguous()
+                for e0 in range(0, pp.numel(), 1024):
+                    e1 = min(pp.numel(), e0 + 1024)
+                    sp, ps = ss[e0:e1].contiguous(), pp[e0:e1].contiguous()
+                    gen.manual_seed(_mix(self.spec.seed, 1, l, p0, e0))
+                    k, v = self._kv(e1 - e0, gen, chl)
+                    self.cache.append(l, sp, ps, k, v, bits_d[sp.long(), ps.long()].contiguous(),
+                                      modes_d[sp.long(), ps.long()].contiguous())
+                    self.prebuild_calls += 1
+        torch.cuda.synchronize()
+        st = self.cache.status()
+        if st != 0:
+            raise RuntimeError(f"cache build failed: status {st}")
+        self.prebuild_launches = 2 * self.prebuild_calls + 1  # + the status kernel
+        print(f"prebuild_launches={self.prebuild_launches}", file=sys.stderr, flush=True)
+        self.steps = [self._stage(i) for i in range(self.total_steps)]
+
+    def _kv(self, n, gen, ch):
+        torch = self.torch
+        shape = (n, self.Hkv * self.d)
+        k = torch.randn(shape, generator=gen, device=self.dev)
+        v = torch.randn(shape, generator=gen, device=self.dev)
+        if ch.numel():
+            k[:, ch] *= self.spec.outlier_scale
+            v[:, ch] *= self.spec.outlier_scale
+        return (k.view(n, self.Hkv, self.d).to(torch.bfloat16).contiguous(),
+                v.view(n, self.Hkv, self.d).to(torch.bfloat16).contiguous())
+
+    def _stage(self, i):
+        """Device inputs and host byte accounting of global step i."""
+        torch = self.torch
+        r, grow = i % self.R, i // self.R
+        gen = torch.Generator(device=self.dev)
+        layers = []
+        nbytes = keys = 0
+        for l in range(self.L):
+            bits, modes = self.all_maps[l][r]
+            pos = (self.ctx + grow).astype(np.int32)
+            seqs = (r * self.B + np.arange(self.B)).astype(np.int32)
+            b = bits[np.arange(self.B), pos]
+            m = modes[np.arange(self.B), pos]
+            gen.manual_seed(_mix(self.spec.seed, 2, i, l))
+            chl = torch.tensor(self.wl.outlier_channels(self.spec, l), dtype=torch.long, device=self.dev)
+            k, v = self._kv(self.B, gen, chl)
+            q = torch.randn((self.B, self.Hq, self.d), generator=gen, device=self.dev).to(torch.bfloat16)
+            for s in range(self.B):
+                nb, nk, _ = self.acct.query(bits[s], modes[s], int(pos[s]))
+                nbytes += nb
+                keys += nk
+            layers.append(dict(
+                seqs=torch.from_numpy(seqs).to(self.dev), pos=torch.from_numpy(pos).to(self.dev),
+                bits=torch.from_numpy(b).to(self.dev), modes=torch.from_numpy(m).to(self.dev),
+                k=k, v=v, q=q,
+                out=torch.empty((self.B, self.Hq, self.d), dtype=torch.bfloat16, device=self.dev)))
+        attn_bytes_per_layer = nbytes / self.L
+        return dict(layers=layers, bytes=nbytes, keys=keys, attn_bytes_per_layer=attn_bytes_per_layer)
+
+    # ---- one step through the C ABI
+    def run_step(self, st, events=None, stream=None):
+        c = self.cache
+        n = 0
+        for l, x in enumerate(st["layers"]):
+            c.append(l, x["seqs"], x["pos"], x["k"], x["v"], x["bits"], x["modes"], stream=stream)
+            n += c.launches()
+            if events is not None:
+                events[0](l)
+            c.decode_attn(l, x["seqs"], x["pos"], x["q"], x["modes"], window_scalar=self.window,
+                          out=x["out"], stream=stream)
+            n += c.launches()
+            if events is not None:
+                events[1](l)
+        return n
+
+    def capture(self, idx, instrument=None):
+        torch = self.torch
+        g = torch.cuda.CUDAGraph()
+        s = torch.cuda.Stream()
+        s.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(s):
+            with torch.cuda.graph(g, stream=s):
+                launches = self.run_step(self.steps[idx], instrument(idx, s) if instrument else None)
+        torch.cuda.current_stream().wait_stream(s)
+        return g, launches
+
+
+def run_gpu(args):
+    import torch
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl" if torch.distributed.is_nccl_available() else "gloo")
+    bench = Bench(args, rank, world)
+    bench.setup()
+    W, K = args.warmup, args.steps
+    rt = CudaRt()
+
+    # timed region: K plain step graphs
+    graphs = [bench.capture(i) for i in range(W + K)]
+    launches_per_step = graphs[0][1]
+    for i in range(W):
+        graphs[i][0].replay()
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    uuid = None
+    try:
+        uuid = str(torch.cuda.get_device_properties(local).uuid)
+        uuid = uuid if uuid.startswith("GPU-") else "GPU-" + uuid
+    except Exception:
+        pass
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(uuid) as clocks:
+        torch.cuda.synchronize()
+        t0.record()
+        for i in range(W, W + K):
+            graphs[i][0].replay()
+        t1.record()
+        torch.cuda.synchronize()
+    ms = t0.elapsed_time(t1)
+    if dist:
+        tt = torch.tensor([ms], dtype=torch.float64, device="cuda")
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms = float(tt.item())
+    step_bytes = sum(bench.steps[i]["bytes"] for i in range(W, W + K))
+    step_keys = sum(bench.steps[i]["keys"] for i in range(W, W + K))
+    del graphs
+
+    # attribution: the next K steps with event nodes around every trr_decode_attn call
+    evs = {}
+
+    def instrument(idx, s):
+        def before(l):
+            e = rt.event()
+            rt.record_external(e, s.cuda_stream)
+            evs[(idx, l, 0)] = e
+
+        def after(l):
+            e = rt.event()
+            rt.record_external(e, s.cuda_stream)
+            evs[(idx, l, 1)] = e
+        return before, after
+
+    base = W + K
+    igraphs = [bench.capture(i, instrument) for i in range(base, base + K)]
+    torch.cuda.synchronize()
+    for g, _ in igraphs:
+        g.replay()
+    torch.cuda.synchronize()
+    call_ms, call_bytes = [], []
+    for i in range(base, base + K):
+        for l in range(bench.L):
+            call_ms.append(rt.elapsed_ms(evs[(i, l, 0)], evs[(i, l, 1)]))
+            call_bytes.append(bench.steps[i]["attn_bytes_per_layer"])
+    del igraphs
+
+    # e2e: the public API with host buffers (pinned H2D inputs, D2H outputs per step)
+    e0 = base + K
+    host = []
+    for i in range(e0, e0 + bench.e2e_warm + bench.e2e_steps):
+        st = bench.steps[i]
+        hl = []
+        for x in st["layers"]:
+            hl.append({k: v.cpu().pin_memory() for k, v in x.items() if k != "out"})
+            hl[-1]["out"] = torch.empty_like(x["out"], device="cpu").pin_memory()
+        host.append(hl)
+    h2d = sum(v.numel() * v.element_size() for x in host[0] for k, v in x.items() if k != "out")
+    d2h = sum(x["out"].numel() * x["out"].element_size() for x in host[0])
+
+    def e2e_step(j):
+        st = bench.steps[e0 + j]
+        for x, hx in zip(st["layers"], host[j]):
+            for k in ("seqs", "pos", "bits", "modes", "k", "v", "q"):
+                x[k].copy_(hx[k], non_blocking=True)
+        bench.run_step(st)
+        for x, hx in zip(st["layers"], host[j]):
+            hx["out"].copy_(x["out"], non_blocking=True)
+
+    for j in range(bench.e2e_warm):
+        e2e_step(j)
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a0.record()
+    for j in range(bench.e2e_warm, bench.e2e_warm + bench.e2e_steps):
+        e2e_step(j)
+    a1.record()
+    torch.cuda.synchronize()
+    e2e_ms = a0.elapsed_time(a1)
+    e2e_bytes = sum(bench.steps[e0 + j]["bytes"] for j in range(bench.e2e_warm, bench.e2e_warm + bench.e2e_steps))
+    if dist:
+        tt = torch.tensor([e2e_ms], dtype=torch.float64, device="cuda")
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        e2e_ms = float(tt.item())
+    status = bench.cache.status()
+    if status != 0:
+        raise RuntimeError(f"device status {status} after the run")
+
+    peak, peak_kind = measured_peaks()
+    avg_bytes = float(np.mean(call_bytes))
+    avg_ms = float(np.mean(call_ms))
+    achieved = avg_bytes / (avg_ms * 1e-3) / 1e9
+    value = world * step_bytes / (ms * 1e-3) / 1e9
+    result = None
+    if rank == 0:
+        cpu = cpu_baseline(bench) if (world == 1 and not args.no_cpu_baseline) else None
+        result = {
+            "metric": METRIC, "value": round(value, 2), "unit": UNIT, "n_gpus": world,
+            "steps": K, "warmup": W, "ms_per_step": round(ms / K, 5), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": {
+                "workload": f"{bench.spec.name}: {bench.L} layers, MHA/GQA {bench.Hq}/{bench.Hkv} x {bench.d}, "
+                            f"batch {bench.B}/GPU, contexts {describe_ctx(bench)}, window {bench.window}, "
+                            f"group {bench.G}, page {PAGE}",
+                "kv_storage": "per-token 2/4/8-bit codes + fp16 scale/zero, or bf16; fp32 accumulation",
+                "global_batch": bench.B * world, "replicas": bench.R,
+                "l2": "inputs larger than L2: every step reads its replica's "
+                      f"{step_bytes / K / 1e6:.0f} MB, replicas rotate",
+                "parallelism": f"replicas{world}" if world > 1 else "single",
+                "bytes_per_step": int(step_bytes / K),
+            },
+            "kv_tokens_per_s": round(world * step_keys / (ms * 1e-3), 1),
+            "pct_of_8tbs": round(100 * value / world / 8000.0, 2),
+            "gpu_launches": launches_per_step * K,
+            "e2e": {"value": round(world * e2e_bytes / (e2e_ms * 1e-3) / 1e9, 2), "unit": UNIT,
+                    "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)},
+            "roofline": {"bound": "hbm", "achieved": round(achieved, 2), "peak": peak,
+                         "unit": "GB/s", "frac": round(achieved / peak, 4),
+                         "traffic": ncu_traffic(args.workload), "peak_kind": peak_kind,
+                         "kernel": "trr_decode_attn call (attn_plan_kernel + attn_kernel)",
+                         "bytes_per_call": round(avg_bytes), "us_per_call": round(avg_ms * 1e3, 3)},
+            "clocks": clocks.summary(),
+        }
+        if cpu is not None:
+            result["cpu_baseline"] = cpu
+    if dist:
+        dist.barrier()
+        dist.destroy_process_group()
+    return result
+
+
+def describe_ctx(bench):
+    c = bench.ctx
+    lo, hi = int(c.min()), int(c.max())
+    grow = math.ceil(bench.total_steps / bench.R)
+    base = f"{lo}" if lo == hi else f"{lo}-{hi}"
+    return f"{base} (+ up to {grow} decoded)"
+
+
+# ----------------------------------------------------------- the oracle on the CPU --
+
+def oracle_sample(spec, n_seqs, budget_s, window, layer=0):
+    """Time the CPU oracle's decode attention on a bounded sample of the workload:
+    layer 0, the first n_seqs sequences with their full prebuilt contexts, queries at
+    the last positions (each with its own mode), until budget_s of CPU time."""
+    import oracle
+    from paper_2607_06601_gb300 import workloads as wl
+    ctx = wl.contexts(spec)
+    n_seqs = min(n_seqs, spec.batch)
+    maxctx = int(ctx[:n_seqs].max())
+    caps = [n_seqs * (maxctx // PAGE + 2)] * 4
+    o = oracle.OracleCache(1, n_seqs, spec.num_q_heads, spec.num_kv_heads, spec.head_dim,
+                           spec.group_size, PAGE, maxctx, caps)
+    acct = Accounting(spec, spec.head_dim, spec.group_size, spec.num_q_heads, spec.num_kv_heads, window)
+    maps = []
+    for s in range(n_seqs):
+        n = int(ctx[s])
+        bits, modes = wl.policy(spec, layer, s, n)
+        q, k, v = wl.q_kv_fast(spec, layer, s, 0, n)
+        for p0 in range(0, n, 1024):
+            p1 = min(n, p0 + 1024)
+            assert o.append(0, [s] * (p1 - p0), np.arange(p0, p1), k[p0:p1], v[p0:p1], bits[p0:p1],
+                            modes[p0:p1]) == 0
+        maps.append((bits, modes, q))
+    spent, nbytes, keys, queries = 0.0, 0, 0, 0
+    t_start = time.perf_counter()
+    j = 0
+    while spent < budget_s and j < 4096:
+        s = j % n_seqs
+        t = int(ctx[s]) - 1 - (j // n_seqs)
+        bits, modes, q = maps[s]
+        c0 = time.process_time()
+        st, _ = o.decode_attn(0, [s], [t], q[t:t + 1], [modes[t]], window_scalar=window)
+        spent += time.process_time() - c0
+        assert st == 0
+        nb, nk, _ = acct.query(bits, modes, t)
+        nbytes += nb
+        keys += nk
+        queries += 1
+        j += 1
+    wall = time.perf_counter() - t_start
+    return nbytes, keys, queries, spent, wall
+
+
+def cpu_baseline(bench):
+    nbytes, keys, queries, spent, wall = oracle_sample(bench.spec, 4, 15.0, bench.window)
+    return {"value": round(nbytes / spent / 1e9, 4), "unit": UNIT, "cores": 1, "kind": "oracle",
+            "kv_tokens_per_s": round(keys / spent, 1),
+            "sample": f"{queries} decode queries (layer 0, sequences 0-3 at their last positions, "
+                      f"seeded modes), single-threaded fp64 C oracle, {spent:.1f} s CPU"}
+
+
+def run_reference(args):
+    """The reference arm: the CPU oracle as it stands, on the same metric and workload."""
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return None
+    from paper_2607_06601_gb300 import workloads as wl
+    import oracle
+    oracle.build()
+    spec = wl.SPECS[args.workload]
+    if args.batch:
+        spec = spec.with_(batch=args.batch)
+    per_step = max(0.5, min(5.0, 150.0 / max(1, args.steps + args.warmup)))
+    for _ in range(args.warmup):
+        oracle_sample(spec, 1, per_step / 4, spec.window)
+    tot_b = tot_k = 0
+    tot_t = 0.0
+    for _ in range(args.steps):
+        nb, nk, nq, spent, _ = oracle_sample(spec, 2, per_step, spec.window)
+        tot_b += nb
+        tot_k += nk
+        tot_t += spent
+    value = tot_b / tot_t / 1e9
+    return {
+        "impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": UNIT,
+        "n_gpus": int(os.environ.get("WORLD_SIZE", "1")), "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(1e3 * tot_t / max(1, args.steps), 3), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": f"{spec.name} (same maps and shapes as the GPU arm), oracle sample per step"},
+        "kv_tokens_per_s": round(tot_k / tot_t, 1),
+        "cpu_baseline": {"value": round(value, 4), "unit": UNIT, "cores": 1, "kind": "oracle",
+                         "sample": "each step: decode queries of sequences 0-1 at their last positions, "
+                                   f"layer 0, about {per_step:.1f} s of single-threaded CPU"},
+        "e2e": {"value": round(value, 4), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=100)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="160m", choices=["tiny", "160m", "1p3b", "gqa_long", "sweep"])
+    ap.add_argument("--batch", type=int, default=0)
+    ap.add_argument("--layers", type=int, default=0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be at least 3")
+    if args.impl == "reference":
+        res = run_reference(args)
+    else:
+        import __graft_entry__
+        __graft_entry__.build()
+        res = run_gpu(args)
+    if res is not None:
+        print(json.dumps(res), flush=True)
+
+
+if __name__ == "__main__":
+    main()

@@ -478,9 +478,14 @@ __global__ void __launch_bounds__(256, 1) attn_kernel(const AttnKernelArgs ka) {
   }
 }
 
-template <int D>
-static cudaError_t configure(int smem) {
-  return cudaFuncSetAttribute(attn_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+constexpr int kAttnSmemLimit = 200 * 1024;  // dynamic shared memory of one attention CTA
+
+// Done once per cache at creation, so that calls stay legal inside stream capture.
+cudaError_t attn_configure() {
+  cudaError_t e = cudaFuncSetAttribute(attn_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, kAttnSmemLimit);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(attn_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, kAttnSmemLimit);
+  return e;
 }
 
 }  // namespace trr
@@ -514,12 +519,10 @@ extern "C" trr_status trr_decode_attn(trr_cache* cache, int32_t layer, int32_t n
   ka.slot_bytes = static_cast<int>(l.slice[3]);
   ka.base_bytes = ((n + 1) * 4 + 127) / 128 * 128;
   const int per_warp = ka.ns * (ka.slot_bytes + 4 * l.P + 8);
-  const int budget = 200 * 1024 - ka.base_bytes;
+  const int budget = kAttnSmemLimit - ka.base_bytes;
   const int nwarps = std::min(8, budget / per_warp);
   if (nwarps < 1) return TRR_ERR_UNSUPPORTED;
   const int smem = ka.base_bytes + nwarps * per_warp;
-  const cudaError_t ce = l.d == 64 ? configure<64>(smem) : configure<128>(smem);
-  if (ce != cudaSuccess) return TRR_ERR_CUDA;
   const int grid = cache_num_sms(cache);
   if (l.d == 64)
     attn_kernel<64><<<grid, nwarps * 32, smem, s>>>(ka);

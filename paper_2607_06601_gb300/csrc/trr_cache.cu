@@ -177,6 +177,11 @@ extern "C" trr_status trr_create_cache(const trr_cache_config* cfg, trr_cache** 
     }
     c->owned = true;
   }
+  if (attn_configure() != cudaSuccess) {
+    if (c->owned) cudaFree(c->base);
+    delete c;
+    return TRR_ERR_CUDA;
+  }
   c->views = make_views(l, c->base);
   c->last_launches = 0;
   st = clear_metadata(c, nullptr);

@@ -117,6 +117,9 @@ const Views& cache_views(const trr_cache* c);
 int cache_num_sms(const trr_cache* c);
 void cache_set_launches(trr_cache* c, int n);
 
+// One-time kernel attribute setup (defined in trr_attn.cu).
+cudaError_t attn_configure();
+
 // ------------------------------------------------------------------ PTX helpers --
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
