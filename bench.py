@@ -267,7 +267,8 @@ class Bench:
                     for c, b in enumerate(BITS):
                         caps[c] += -(-int(np.count_nonzero(stored & (bits[s] == b))) // PAGE) + 1
         self.cache = trr.Cache(L, S, self.Hq, self.Hkv, self.d, self.G, PAGE, self.maxctx,
-                               [int(c) for c in caps], max_append=1024, max_queries=max(B, 64))
+                               [int(c) for c in caps], max_append=1024, max_queries=max(B, 64),
+                               split_bytes=self.args.split_bytes)
         # prebuild every sequence's context (untimed), K/V drawn on the device
         gen = torch.Generator(device=self.dev)
         self.prebuild_calls = 0
@@ -506,6 +507,7 @@ def run_gpu(args):
                       f"{step_bytes / K / 1e6:.0f} MB, replicas rotate",
                 "parallelism": f"replicas{world}" if world > 1 else "single",
                 "bytes_per_step": int(step_bytes / K),
+                "split_bytes": args.split_bytes or "default",
             },
             "kv_tokens_per_s": round(world * step_keys / (ms * 1e-3), 1),
             "pct_of_8tbs": round(100 * value / world / 8000.0, 2),
@@ -634,6 +636,8 @@ def main():
     ap.add_argument("--batch", type=int, default=0)
     ap.add_argument("--layers", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--split-bytes", type=int, default=0,
+                    help="target KV bytes per split-K work item (0: the library default)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")

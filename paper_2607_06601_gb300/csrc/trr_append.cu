@@ -29,6 +29,8 @@ __global__ void __launch_bounds__(1024) append_plan_kernel(LayerArgs a, int n, c
   __shared__ int s_first_err;
   __shared__ int s_nopen[kClasses];
 
+  pdl_wait();
+  pdl_trigger();
   const int e = threadIdx.x;
   const bool act = e < n;
   int seq = -1, pos = 0, c = -1, err = 0;
@@ -157,6 +159,8 @@ __device__ __forceinline__ void quantise_chunk(const uint4* src, float z, float 
 
 __global__ void __launch_bounds__(256) append_write_kernel(LayerArgs a, int n, const uint16_t* __restrict__ k,
                                                            const uint16_t* __restrict__ v) {
+  pdl_wait();
+  pdl_trigger();
   if (a.ctrl[kAppendOk] == 0) return;
   const int ng = a.d / a.G;
   const int per_entry = a.Hkv * 2 * ng;
@@ -236,10 +240,11 @@ extern "C" trr_status trr_kv_append(trr_cache* cache, int32_t layer, int32_t n, 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const LayerArgs a = layer_args(l, cache_views(cache), layer);
   const int threads = (n + 31) / 32 * 32;
-  append_plan_kernel<<<1, threads, 0, s>>>(a, n, seq_ids, positions, bits, modes);
+  cudaError_t e = launch_pdl(append_plan_kernel, dim3(1), dim3(threads), 0, s, a, n, seq_ids, positions, bits, modes);
+  if (e != cudaSuccess) return TRR_ERR_CUDA;
   const int64_t work = static_cast<int64_t>(n) * l.Hkv * 2 * (l.d / l.G);
-  append_write_kernel<<<static_cast<unsigned>((work + 255) / 256), 256, 0, s>>>(
-      a, n, static_cast<const uint16_t*>(k_bf16), static_cast<const uint16_t*>(v_bf16));
+  e = launch_pdl(append_write_kernel, dim3(static_cast<unsigned>((work + 255) / 256)), dim3(256), 0, s, a, n,
+                 static_cast<const uint16_t*>(k_bf16), static_cast<const uint16_t*>(v_bf16));
   cache_set_launches(cache, 2);
-  return cudaGetLastError() == cudaSuccess ? TRR_OK : TRR_ERR_CUDA;
+  return e == cudaSuccess ? TRR_OK : TRR_ERR_CUDA;
 }

@@ -1,20 +1,29 @@
 // trr_attn.cu - trr_decode_attn: mode-routed split-K decode attention over the
 // mixed-precision paged cache (Sec. 3.2(A), Eq. 2; Sec. 3.8; Sec. 7).
 //
-// Two kernels per call:
+// Two kernels per call, chained with programmatic dependent launch:
 //   attn_plan_kernel  one warp per query.  Key range by mode (full: [0, t]; local:
-//                     [t-w+1, t]; skip: none), the pages of each width class that
-//                     intersect it (found from each page's first/last position), and
-//                     the number of split-K work items from the bytes in range.  Skip
+//                     [t-w+1, t]; skip: none); for each width class the pages that
+//                     intersect it, found by a 32-way search over the pages'
+//                     first / last positions (all classes and both ends at once); the
+//                     number of split-K work items from the bytes in range.  Skip
 //                     queries and empty ranges get their zero rows here.
-//   attn_kernel       persistent, one CTA per SM, every warp an independent worker.
-//                     A warp takes one (query, head, split) item at a time, streams its
-//                     pages through a private ring of shared-memory slots filled by 1-D
-//                     bulk copies (cp.async.bulk + mbarrier), dequantises in registers
-//                     (k = z + c*s folded as s*sum(q*c) + z*sum(q)), runs an online
-//                     softmax per lane, merges lanes with shuffles, and either writes
-//                     the bf16 row (one split) or a partial; the last split to finish
-//                     merges the partials (no waiting: an atomic arrival counter).
+//   attn_kernel       persistent, two CTAs per SM, every warp an independent worker.
+//                     Work items (query, head, split) are dealt round-robin.  A warp
+//                     streams the pages of its items through a private 3-slot ring of
+//                     shared memory filled by 1-D bulk copies (cp.async.bulk +
+//                     mbarrier), with the query row riding on the first copy of each
+//                     item, so items follow each other without a pipeline drain.
+//                     Lane pair (key, half) of a 64-wide head (four lanes for 128)
+//                     dequantises in registers and keeps its own online softmax;
+//                     lanes merge with shuffles; one split writes the bf16 row, several
+//                     write fp32 partials and the last to arrive merges them.
+//
+// Dequantisation: k = z + c*s, so q.k = s * sum(q_i c_i) + z * sum(q_i).  A code is
+// masked in place (no shift) and its bits read as a binary32 subnormal, c * 2^(e-149)
+// where e is its bit offset; the query is pre-scaled per width class by 2^(100-e) so
+// that q_i * x_i = q_i c_i 2^-49 exactly as an fp32 product.  V is accumulated in a
+// domain scaled by 2^-49 with the per-offset factor folded into the key's weight.
 #include <algorithm>
 #include <climits>
 
@@ -23,15 +32,77 @@
 namespace trr {
 
 #define kNegInf (-__int_as_float(0x7f800000))
+constexpr float kTau = 8.f;    // lazy rescale threshold (log2 units)
+
+
+// ----------------------------------------------------------------------- plan --
+
+// Count of k in [0, n) with arr[k] < x (arr increasing), searched by the whole warp.
+// The first round probes the last 32 entries: decode queries look at the end of the
+// page lists, so that round almost always settles it.  Otherwise 32 probes per round
+// narrow the rest.  Every search of the call advances in the same round.
+template <int NS>
+__device__ __forceinline__ void warp_count_below(const int* const (&arr)[NS], const int (&n)[NS],
+                                                 const int (&x)[NS], int (&out)[NS], int lane) {
+  int lo[NS], hi[NS];
+  {
+    int v[NS], idx[NS];
+#pragma unroll
+    for (int i = 0; i < NS; ++i) {
+      idx[i] = max(0, n[i] - 32) + lane;
+      v[i] = idx[i] < n[i] ? arr[i][idx[i]] : INT_MAX;
+    }
+#pragma unroll
+    for (int i = 0; i < NS; ++i) {
+      const unsigned below = __ballot_sync(0xffffffffu, idx[i] < n[i] && v[i] < x[i]);
+      const int base = max(0, n[i] - 32);
+      if (n[i] <= 32 || (below & 1u)) {  // arr[base] < x: everything before it is too
+        lo[i] = hi[i] = base + __popc(below);
+      } else {
+        lo[i] = 0;
+        hi[i] = base;
+      }
+    }
+  }
+  for (int round = 0; round < 6; ++round) {
+    int v[NS], idx[NS], step[NS];
+    bool any = false;
+#pragma unroll
+    for (int i = 0; i < NS; ++i) {
+      const int span = hi[i] - lo[i];
+      step[i] = span <= 32 ? 1 : (span + 31) / 32;
+      idx[i] = lo[i] + lane * step[i];
+      v[i] = (span > 0 && idx[i] < hi[i]) ? arr[i][idx[i]] : INT_MAX;
+      any |= span > 0;
+    }
+    if (!any) break;
+#pragma unroll
+    for (int i = 0; i < NS; ++i) {
+      const int span = hi[i] - lo[i];
+      const int cnt = __popc(__ballot_sync(0xffffffffu, idx[i] < hi[i] && v[i] < x[i]));
+      if (span <= 0) continue;
+      if (span <= 32 || cnt == 0) {
+        lo[i] = hi[i] = lo[i] + (span <= 32 ? cnt : 0);
+      } else {
+        const int last = lo[i] + (cnt - 1) * step[i];  // last probe below x
+        hi[i] = min(hi[i], lo[i] + cnt * step[i]);
+        lo[i] = last + 1;
+      }
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < NS; ++i) out[i] = lo[i];
+}
 
 __global__ void __launch_bounds__(256) attn_plan_kernel(LayerArgs a, int n, const int32_t* __restrict__ seq_ids,
                                                         const int32_t* __restrict__ q_positions,
                                                         const uint8_t* __restrict__ modes,
                                                         const int32_t* __restrict__ windows, int window_scalar,
                                                         uint16_t* __restrict__ out) {
+  pdl_wait();
+  pdl_trigger();
   const int lane = threadIdx.x & 31;
   const int qi = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-  if (blockIdx.x == 0 && threadIdx.x == 0) a.ctrl[kWorkCounter] = 0;
   if (qi >= n) return;
   const int seq = seq_ids[qi], t = q_positions[qi], mode = modes[qi];
   const int w = windows ? windows[qi] : window_scalar;
@@ -47,65 +118,159 @@ __global__ void __launch_bounds__(256) attn_plan_kernel(LayerArgs a, int n, cons
   qp.lo = 0;
   qp.hi = t;
   qp.pad0 = qp.pad1 = qp.pad2 = 0;
-  int64_t bytes = 0;
+#pragma unroll
+  for (int c = 0; c < kClasses; ++c) qp.first[c] = qp.npages[c] = qp.ntok[c] = 0;
   int total_pages = 0;
-  for (int c = 0; c < kClasses; ++c) {
-    qp.first[c] = 0;
-    qp.npages[c] = 0;
-    qp.ntok[c] = 0;
-  }
   if (!err && mode != TRR_MODE_SKIP) {
     const int lo = mode == TRR_MODE_FULL ? 0 : max(0, t - w + 1);
     qp.lo = lo;
+    const int* arr[2 * kClasses];
+    int np[2 * kClasses], x[2 * kClasses], cnt[2 * kClasses];
+#pragma unroll
     for (int c = 0; c < kClasses; ++c) {
       const int nt = a.ntok[seq * 4 + c];
-      const int np = (nt + a.P - 1) / a.P;
-      const int64_t row = static_cast<int64_t>(seq * 4 + c) * a.MP;
-      int below = 0, upto = 0;  // pages ending before lo; pages starting at or before t
-      for (int base = 0; base < np; base += 32) {
-        const int kk = base + lane;
-        const bool in = kk < np;
-        const int pl = in ? a.plast[row + kk] : INT_MAX;
-        const int pf = in ? a.pfirst[row + kk] : INT_MAX;
-        below += __popc(__ballot_sync(0xffffffffu, in && pl < lo));
-        upto += __popc(__ballot_sync(0xffffffffu, in && pf <= t));
-      }
       qp.ntok[c] = nt;
-      qp.first[c] = below;
-      qp.npages[c] = max(0, upto - below);
+      const int64_t row = static_cast<int64_t>(seq * 4 + c) * a.MP;
+      arr[c] = a.plast + row;                 // pages ending before lo
+      np[c] = lo > 0 ? (nt + a.P - 1) / a.P : 0;
+      x[c] = lo;
+      arr[kClasses + c] = a.pfirst + row;     // pages starting at or before t
+      np[kClasses + c] = (nt + a.P - 1) / a.P;
+      x[kClasses + c] = t + 1;
+    }
+    warp_count_below<2 * kClasses>(arr, np, x, cnt, lane);
+    int64_t bytes = 0;
+#pragma unroll
+    for (int c = 0; c < kClasses; ++c) {
+      qp.first[c] = cnt[c];
+      qp.npages[c] = max(0, cnt[kClasses + c] - cnt[c]);
       bytes += static_cast<int64_t>(qp.npages[c]) * a.slice[c];
       total_pages += qp.npages[c];
     }
     if (bytes > 0) {
-      int64_t ns = (bytes + a.split_bytes - 1) / a.split_bytes;
+      int64_t ns = max((bytes + a.split_bytes - 1) / a.split_bytes,
+                       static_cast<int64_t>((total_pages + kDescMaxPages - 1) / kDescMaxPages));
       ns = min(ns, static_cast<int64_t>(a.s_cap));
       qp.nsplit = static_cast<int>(min(ns, static_cast<int64_t>(total_pages)));
     }
   }
-  if (lane == 0) a.qplan[qi] = qp;
+  if (lane < 20) reinterpret_cast<int*>(a.qplan + qi)[lane] = reinterpret_cast<const int*>(&qp)[lane];
   if (qp.nsplit == 0) {  // skip, invalid or nothing stored in range: a zero row
     uint4* o = reinterpret_cast<uint4*>(out + static_cast<int64_t>(qi) * a.Hq * a.d);
     const int n16 = a.Hq * a.d / 8;
     for (int i = lane; i < n16; i += 32) o[i] = make_uint4(0, 0, 0, 0);
+    if (err && lane == 0) atomicMin(&a.ctrl[kFirstBadQuery], qi);
+    return;
   }
-  if (err && lane == 0) atomicMin(&a.ctrl[kFirstBadQuery], qi);
+  // Descriptors: one per split, at consecutive indices taken from a shared counter.
+  // Split sp of class c takes the class's pages [first + sp*np/ns, first + (sp+1)*np/ns).
+  const int ns = qp.nsplit;
+  int base = 0;
+  if (lane == 0) base = atomicAdd(&a.ctrl[kDescCounter], ns);
+  base = __shfl_sync(0xffffffffu, base, 0);
+  SplitDesc* dsc = a.desc + base;
+  auto bnd = [&](int c, int sp) { return static_cast<int>(static_cast<int64_t>(sp) * qp.npages[c] / ns); };
+  for (int sp = lane; sp < ns; sp += 32) {
+    int T = 0;
+#pragma unroll
+    for (int c = 0; c < kClasses; ++c) T += bnd(c, sp + 1) - bnd(c, sp);
+    int* h = &dsc[sp].qi;
+    h[0] = qi; h[1] = seq; h[2] = qp.lo; h[3] = qp.hi; h[4] = ns; h[5] = sp; h[6] = T; h[7] = base;
+  }
+  const int c1 = qp.npages[0], c2 = c1 + qp.npages[1], c3 = c2 + qp.npages[2];
+  constexpr int kBatch = 8;  // page ids loaded before any descriptor store
+  for (int f0 = 0; f0 < total_pages; f0 += 32 * kBatch) {
+    int id[kBatch], cls[kBatch], kid[kBatch];
+#pragma unroll
+    for (int b = 0; b < kBatch; ++b) {
+      const int f = f0 + 32 * b + lane;
+      const int c = (f >= c1) + (f >= c2) + (f >= c3);
+      const int local = f - (c == 0 ? 0 : c == 1 ? c1 : c == 2 ? c2 : c3);
+      cls[b] = c;
+      kid[b] = qp.first[c] + local;
+      id[b] = f < total_pages ? a.pt[static_cast<int64_t>(seq * 4 + c) * a.MP + kid[b]] : -1;
+    }
+#pragma unroll
+    for (int b = 0; b < kBatch; ++b) {
+      const int f = f0 + 32 * b + lane;
+      if (f >= total_pages) break;
+      const int c = cls[b];
+      const int local = kid[b] - qp.first[c];
+      const int np = qp.npages[c];
+      const int sp = static_cast<int>((static_cast<int64_t>(local + 1) * ns - 1) / np);
+      int pos = local - bnd(c, sp);
+      for (int c0 = 0; c0 < c; ++c0) pos += bnd(c0, sp + 1) - bnd(c0, sp);
+      const int fill = min(a.P, qp.ntok[c] - kid[b] * a.P);
+      dsc[sp].page[pos] = id[b];
+      dsc[sp].meta[pos] = c | (fill << 8);
+    }
+  }
 }
+
+// ------------------------------------------------------------------ dequant --
 
 __device__ __forceinline__ float bf_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 
-// State of one lane: an online softmax over its keys (log2 domain) and the weighted
-// sum of V over its 32 dimensions.  zacc collects p*z, the zero-point part of V.
+// exact 2^e, -126 <= e <= 127 (folds to a constant for constant e)
+__device__ __forceinline__ float pow2f(int e) { return __int_as_float((127 + e) << 23); }
+
+// Bit offset of element i (of a lane's 32) inside the word it is extracted from.
+__host__ __device__ constexpr int ex_of(int B, int i) {
+  return B == 2 ? ((i % 16) < 11 ? 2 * (i % 16) : 2 * (i % 16 - 11))
+                : B == 4 ? ((i % 8) < 5 ? 4 * (i % 8) : 4 * (i % 8 - 5)) : 0;
+}
+// Pre-scale exponent of the query in class B.
+__host__ __device__ constexpr int qe_of(int B, int i) { return B == 16 ? 0 : 100 - ex_of(B, i); }
+
+// Element i as c * 2^(ex-149): the code left in place, read as a subnormal.
+template <int B>
+__device__ __forceinline__ float code_at(const uint32_t* w, const uint32_t* h, int i) {
+  if (B == 2) {
+    const int j = i % 16;
+    return __uint_as_float(j < 11 ? (w[i / 16] & (3u << (2 * j))) : (h[i / 16] & (3u << (2 * (j - 11)))));
+  } else if (B == 4) {
+    const int j = i % 8;
+    return __uint_as_float(j < 5 ? (w[i / 8] & (15u << (4 * j))) : (h[i / 8] & (15u << (4 * (j - 5)))));
+  } else {
+    return __uint_as_float(__byte_perm(w[i / 4], 0u, 0x4440u | (i % 4)));
+  }
+}
+template <int B>
+__device__ __forceinline__ void high_parts(const uint32_t* w, uint32_t* h) {
+  constexpr int sh = B == 2 ? 22 : B == 4 ? 20 : 16;
+#pragma unroll
+  for (int k = 0; k < B; ++k) h[k] = w[k] >> sh;
+}
+
+template <int BFROM, int BTO>
+__device__ __forceinline__ void rescale_q(float (&qp)[32]) {
+#pragma unroll
+  for (int i = 0; i < 32; ++i) qp[i] *= pow2f(qe_of(BTO, i) - qe_of(BFROM, i));
+}
+
+// qp from the domain of class `from` to that of class `to` (from < to, or from = 16).
+__device__ __forceinline__ void rescale_q_dyn(float (&qp)[32], int from, int to) {
+  switch (from * 4 + to) {
+    case 1: rescale_q<2, 4>(qp); break;
+    case 2: rescale_q<2, 8>(qp); break;
+    case 3: rescale_q<2, 16>(qp); break;
+    case 6: rescale_q<4, 8>(qp); break;
+    case 7: rescale_q<4, 16>(qp); break;
+    case 11: rescale_q<8, 16>(qp); break;
+    case 12: rescale_q<16, 2>(qp); break;
+    case 13: rescale_q<16, 4>(qp); break;
+    case 14: rescale_q<16, 8>(qp); break;
+    default: break;
+  }
+}
+
 struct LaneState {
-  float m, l, zacc;
-  float acc[32];
+  float m, l, zacc;  // running max (log2), sum of weights, sum of p*z (V zero points)
+  float acc[32];     // sum of p*v over the lane's 32 dims, scaled by 2^-49
 };
 
-// Lazy rescaling: the running maximum moves only when a score exceeds it by more than
-// kTau (log2 units), so p = 2^(score - m) stays below 2^kTau.
-constexpr float kTau = 8.f;
-
-__device__ __forceinline__ void softmax_step(LaneState& st, float score, float& p) {
+__device__ __forceinline__ float softmax_step(LaneState& st, float score) {
   if (score > st.m + kTau) {
     const float alpha = exp2f(st.m - score);  // 0 when m = -inf
 #pragma unroll
@@ -114,17 +279,18 @@ __device__ __forceinline__ void softmax_step(LaneState& st, float score, float& 
     st.zacc *= alpha;
     st.m = score;
   }
-  p = exp2f(score - st.m);
+  const float p = exp2f(score - st.m);
   st.l += p;
+  return p;
 }
 
-// One page of width class B in shared memory.  Lane -> (key kl, 32-dim part).
+// One page of width class B in shared memory; lane -> (key kl, 32-dim part).
 template <int D, int B>
 __device__ __forceinline__ void consume_page(const uint8_t* sl, const int* spos, int P, int G, int fill,
-                                             int lo, int hi, const float (&qf)[32], float sumq,
+                                             int lo, int hi, const float (&qp)[32], float sumq,
                                              LaneState& st, int lane) {
-  constexpr int LPK = D / 32;   // lanes per key
-  constexpr int KPI = 32 / LPK; // keys per pass
+  constexpr int LPK = D / 32;
+  constexpr int KPI = 32 / LPK;
   const int part = lane % LPK, kl = lane / LPK;
   const int ng = D / G;
   const int grp = part * 32 / G;
@@ -132,85 +298,81 @@ __device__ __forceinline__ void consume_page(const uint8_t* sl, const int* spos,
     const int key = it * KPI + kl;
     const int pos = spos[key];
     const bool valid = key < fill && pos >= lo && pos <= hi;
-    float dot = 0.f;
+    float dot;
     if (B == 16) {
-      const uint4* kp = reinterpret_cast<const uint4*>(sl + (static_cast<int64_t>(key) * D + part * 32) * 2);
-      float d0 = 0.f, d1 = 0.f;
+      const uint4* kp = reinterpret_cast<const uint4*>(sl + (key * D + part * 32) * 2);
+      float d[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
         const uint4 u = kp[q];
-        d0 = fmaf(qf[8 * q + 0], bf_lo(u.x), d0);
-        d1 = fmaf(qf[8 * q + 1], bf_hi(u.x), d1);
-        d0 = fmaf(qf[8 * q + 2], bf_lo(u.y), d0);
-        d1 = fmaf(qf[8 * q + 3], bf_hi(u.y), d1);
-        d0 = fmaf(qf[8 * q + 4], bf_lo(u.z), d0);
-        d1 = fmaf(qf[8 * q + 5], bf_hi(u.z), d1);
-        d0 = fmaf(qf[8 * q + 6], bf_lo(u.w), d0);
-        d1 = fmaf(qf[8 * q + 7], bf_hi(u.w), d1);
+        d[0] = fmaf(qp[8 * q + 0], bf_lo(u.x), d[0]);
+        d[1] = fmaf(qp[8 * q + 1], bf_hi(u.x), d[1]);
+        d[2] = fmaf(qp[8 * q + 2], bf_lo(u.y), d[2]);
+        d[3] = fmaf(qp[8 * q + 3], bf_hi(u.y), d[3]);
+        d[0] = fmaf(qp[8 * q + 4], bf_lo(u.z), d[0]);
+        d[1] = fmaf(qp[8 * q + 5], bf_hi(u.z), d[1]);
+        d[2] = fmaf(qp[8 * q + 6], bf_lo(u.w), d[2]);
+        d[3] = fmaf(qp[8 * q + 7], bf_hi(u.w), d[3]);
       }
-      dot = d0 + d1;
+      dot = (d[0] + d[1]) + (d[2] + d[3]);
     } else {
       constexpr int rowb = D * B / 8;
-      constexpr int WORDS = B;  // 32 codes of B bits
-      constexpr int PER = 32 / B;
+      uint32_t w[B], h[B];
       const uint32_t* kc = reinterpret_cast<const uint32_t*>(sl + key * rowb + part * 4 * B);
-      uint32_t wv[WORDS];
 #pragma unroll
-      for (int w = 0; w < WORDS; ++w) wv[w] = kc[w];
+      for (int k = 0; k < B; ++k) w[k] = kc[k];
+      if (B != 8) high_parts<B>(w, h);
       const uint32_t szw = *reinterpret_cast<const uint32_t*>(sl + 2 * P * rowb + (key * ng + grp) * 4);
+      float d[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int i = 0; i < 32; ++i) d[i & 3] = fmaf(qp[i], code_at<B>(w, h, i), d[i & 3]);
       const float s = __half2float(__ushort_as_half(static_cast<unsigned short>(szw & 0xFFFF)));
       const float z = __half2float(__ushort_as_half(static_cast<unsigned short>(szw >> 16)));
-      float d0 = 0.f, d1 = 0.f;
-#pragma unroll
-      for (int j = 0; j < 32; ++j) {
-        const float cf = static_cast<float>((wv[j / PER] >> ((j % PER) * B)) & ((1u << B) - 1));
-        if (j & 1) d1 = fmaf(qf[j], cf, d1);
-        else d0 = fmaf(qf[j], cf, d0);
-      }
-      dot = fmaf(s, d0 + d1, z * sumq);
+      dot = fmaf(s * pow2f(49), (d[0] + d[1]) + (d[2] + d[3]), z * sumq);
     }
 #pragma unroll
     for (int o = 1; o < LPK; o <<= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
     if (valid) {
-      float p;
-      softmax_step(st, dot, p);
+      const float p = softmax_step(st, dot);
       if (B == 16) {
-        const uint4* vp =
-            reinterpret_cast<const uint4*>(sl + (static_cast<int64_t>(P) * D + key * D + part * 32) * 2);
+        const uint4* vp = reinterpret_cast<const uint4*>(sl + (P * D + key * D + part * 32) * 2);
+        const float wv = p * pow2f(-49);
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
           const uint4 u = vp[q];
-          st.acc[8 * q + 0] = fmaf(p, bf_lo(u.x), st.acc[8 * q + 0]);
-          st.acc[8 * q + 1] = fmaf(p, bf_hi(u.x), st.acc[8 * q + 1]);
-          st.acc[8 * q + 2] = fmaf(p, bf_lo(u.y), st.acc[8 * q + 2]);
-          st.acc[8 * q + 3] = fmaf(p, bf_hi(u.y), st.acc[8 * q + 3]);
-          st.acc[8 * q + 4] = fmaf(p, bf_lo(u.z), st.acc[8 * q + 4]);
-          st.acc[8 * q + 5] = fmaf(p, bf_hi(u.z), st.acc[8 * q + 5]);
-          st.acc[8 * q + 6] = fmaf(p, bf_lo(u.w), st.acc[8 * q + 6]);
-          st.acc[8 * q + 7] = fmaf(p, bf_hi(u.w), st.acc[8 * q + 7]);
+          st.acc[8 * q + 0] = fmaf(wv, bf_lo(u.x), st.acc[8 * q + 0]);
+          st.acc[8 * q + 1] = fmaf(wv, bf_hi(u.x), st.acc[8 * q + 1]);
+          st.acc[8 * q + 2] = fmaf(wv, bf_lo(u.y), st.acc[8 * q + 2]);
+          st.acc[8 * q + 3] = fmaf(wv, bf_hi(u.y), st.acc[8 * q + 3]);
+          st.acc[8 * q + 4] = fmaf(wv, bf_lo(u.z), st.acc[8 * q + 4]);
+          st.acc[8 * q + 5] = fmaf(wv, bf_hi(u.z), st.acc[8 * q + 5]);
+          st.acc[8 * q + 6] = fmaf(wv, bf_lo(u.w), st.acc[8 * q + 6]);
+          st.acc[8 * q + 7] = fmaf(wv, bf_hi(u.w), st.acc[8 * q + 7]);
         }
       } else {
         constexpr int rowb = D * B / 8;
-        constexpr int PER = 32 / B;
+        uint32_t w[B], h[B];
         const uint32_t* vc = reinterpret_cast<const uint32_t*>(sl + P * rowb + key * rowb + part * 4 * B);
-        uint32_t wv[B];
 #pragma unroll
-        for (int w = 0; w < B; ++w) wv[w] = vc[w];
+        for (int k = 0; k < B; ++k) w[k] = vc[k];
+        if (B != 8) high_parts<B>(w, h);
         const uint32_t szw =
             *reinterpret_cast<const uint32_t*>(sl + 2 * P * rowb + P * ng * 4 + (key * ng + grp) * 4);
         const float s = __half2float(__ushort_as_half(static_cast<unsigned short>(szw & 0xFFFF)));
         const float z = __half2float(__ushort_as_half(static_cast<unsigned short>(szw >> 16)));
-        const float ps = p * s;
+        const float wb = p * s * pow2f(100);
 #pragma unroll
-        for (int j = 0; j < 32; ++j) {
-          const float cf = static_cast<float>((wv[j / PER] >> ((j % PER) * B)) & ((1u << B) - 1));
-          st.acc[j] = fmaf(ps, cf, st.acc[j]);
-        }
+        for (int i = 0; i < 32; ++i)
+          st.acc[i] = fmaf(wb * pow2f(-ex_of(B, i)), code_at<B>(w, h, i), st.acc[i]);
         st.zacc = fmaf(p, z, st.zacc);
       }
     }
   }
 }
+
+// -------------------------------------------------------------------- kernel --
+
+constexpr int kSlots = 8;  // pages a warp may have in flight (one mbarrier each)
 
 struct AttnKernelArgs {
   LayerArgs a;
@@ -218,50 +380,71 @@ struct AttnKernelArgs {
   const uint16_t* q;
   uint16_t* out;
   float qscale;      // softmax scale * log2(e)
-  int ns;            // ring slots per warp
-  int slot_bytes;    // bytes of one slot (the largest slice)
-  int base_bytes;    // shared bytes of the item-base table
+  int ring_bytes;    // bytes of one warp's ring of shared memory
 };
 
+// Per-slot record the producer writes for the consumer.
+struct SlotInfo {
+  int cls, fill, lo, hi;
+  int flags;   // 1 first page of its item, 2 last page, 4 no page (item without pages)
+  int item, qi, qh;
+  int nsplit, off, qoff, span;  // ring offsets of the page and the query row; bytes to release
+  int base, pad0, pad1, pad2;   // descriptor index of the query's split 0
+};
+
+// Producer-side description of the item being issued.
+struct ProdItem {
+  int item, qi, qh, kvh, nsplit, T, lo, hi, base, pad0, pad1, pad2;
+};
+static_assert(sizeof(SlotInfo) % 16 == 0 && sizeof(ProdItem) % 16 == 0, "16-byte multiples");
+
+// Shared-memory carve-up of one attention CTA; every region starts 16-byte aligned
+// (mbarriers need 8, bulk-copy destinations 16).
+__host__ __device__ constexpr int align16(int x) { return (x + 15) & ~15; }
+struct AttnSmem {
+  int rings, infos, items, bars, total;
+  __host__ __device__ AttnSmem(int nwarps, int ring_bytes)
+      : rings(0),
+        infos(align16(nwarps * ring_bytes)),
+        items(infos + align16(nwarps * kSlots * static_cast<int>(sizeof(SlotInfo)))),
+        bars(items + align16(nwarps * static_cast<int>(sizeof(ProdItem)))),
+        total(bars + align16(nwarps * kSlots * 8)) {}
+};
+
+// The last warp of the grid to finish resets the descriptor counter for the next call
+// (every warp has read it by then); no warp waits for another.
+__device__ __forceinline__ void finish_warp(int32_t* ctrl, int warps, int lane) {
+  if (lane == 0) {
+    __threadfence();
+    if (atomicAdd(ctrl + kDoneWarps, 1) == warps - 1) {
+      ctrl[kDescCounter] = 0;
+      ctrl[kDoneWarps] = 0;
+    }
+  }
+}
+
 template <int D>
-__global__ void __launch_bounds__(256, 1) attn_kernel(const AttnKernelArgs ka) {
-  constexpr int LPK = D / 32;
+__global__ void __launch_bounds__(256, 2) attn_kernel(const AttnKernelArgs ka) {
+  constexpr int LPK = D / 32;  // lanes per key
+  constexpr int DPL = D / 32;  // dimensions per lane after the merge
   const LayerArgs& a = ka.a;
   extern __shared__ __align__(128) uint8_t smem[];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
-  const int n = ka.n;
-  int* s_base = reinterpret_cast<int*>(smem);  // [n + 1] first item of each query
-  uint8_t* slots = smem + ka.base_bytes + static_cast<int64_t>(warp) * ka.ns * ka.slot_bytes;
-  int* wpos = reinterpret_cast<int*>(smem + ka.base_bytes + static_cast<int64_t>(nwarps) * ka.ns * ka.slot_bytes) +
-              warp * ka.ns * a.P;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + ka.base_bytes +
-                                               static_cast<int64_t>(nwarps) * ka.ns * (ka.slot_bytes + 4 * a.P)) +
-                   warp * ka.ns;
+  const int qrow = D * 2;  // bytes of one query row
+  const int R = ka.ring_bytes;
+  const AttnSmem lay(nwarps, R);  // [rings][slot infos][producer items][mbarriers]
+  uint8_t* ring = smem + lay.rings + warp * R;
+  SlotInfo* sinfo = reinterpret_cast<SlotInfo*>(smem + lay.infos) + warp * kSlots;
+  ProdItem* pi = reinterpret_cast<ProdItem*>(smem + lay.items) + warp;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + lay.bars) + warp * kSlots;
 
-  // item bases: exclusive scan of nsplit * units over the queries
-  {
-    __shared__ int s_warp_sum[32];
-    const int per = (n + blockDim.x - 1) / blockDim.x;
-    const int i0 = threadIdx.x * per;
-    int sum = 0;
-    for (int i = i0; i < min(n, i0 + per); ++i) sum += a.qplan[i].nsplit * a.units;
-    int incl = sum;
+  if (lane == 0) {
 #pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const int y = __shfl_up_sync(0xffffffffu, incl, o);
-      if (lane >= o) incl += y;
-    }
-    if (lane == 31) s_warp_sum[warp] = incl;
-    __syncthreads();
-    int woff = 0;
-    for (int w = 0; w < warp; ++w) woff += s_warp_sum[w];
-    int run = woff + incl - sum;
-    for (int i = i0; i < min(n, i0 + per); ++i) {
-      s_base[i] = run;
-      run += a.qplan[i].nsplit * a.units;
-    }
-    if (threadIdx.x == blockDim.x - 1) s_base[n] = woff + incl;
+    for (int i = 0; i < kSlots; ++i) mbar_init(&bars[i], 1);
+    fence_barrier_init();
   }
+  pdl_wait();
+  pdl_trigger();
   if (blockIdx.x == 0 && threadIdx.x == 0) {  // status of the lowest invalid query
     const int bad = a.ctrl[kFirstBadQuery];
     if (bad != INT_MAX) {
@@ -269,139 +452,186 @@ __global__ void __launch_bounds__(256, 1) attn_kernel(const AttnKernelArgs ka) {
       a.ctrl[kFirstBadQuery] = INT_MAX;
     }
   }
-  if (lane == 0) {
-    for (int i = 0; i < ka.ns; ++i) mbar_init(&bars[i], 1);
-    fence_barrier_init();
-  }
-  __syncthreads();
-  const int total = s_base[n];
+  // work items: (descriptor, query head) pairs, descriptors in the plan's order
+  const int total = *reinterpret_cast<volatile int*>(a.ctrl + kDescCounter) * a.units;
   const int group = a.Hq / a.Hkv;
-  uint32_t gcount = 0;  // pages this warp has consumed so far (slot ring position)
+  const int wstride = gridDim.x * nwarps;
 
-  for (;;) {
-    int item = 0;
-    if (lane == 0) item = atomicAdd(&a.ctrl[kWorkCounter], 1);
-    item = __shfl_sync(0xffffffffu, item, 0);
-    if (item >= total) break;
-    int qlo = 0, qhi = n - 1;  // the query whose items contain `item`
-    while (qlo < qhi) {
-      const int mid = (qlo + qhi + 1) >> 1;
-      if (s_base[mid] <= item) qlo = mid;
-      else qhi = mid - 1;
-    }
-    const int qi = qlo;
-    const QueryPlan& qp = a.qplan[qi];
-    const int nsplit = qp.nsplit, seq = qp.seq, lo = qp.lo, hi = qp.hi;
-    const int local = item - s_base[qi];
-    const int unit = local / nsplit, split = local % nsplit;
-    const int qh = unit, kvh = qh / group;
-    int cb[kClasses], cum[kClasses + 1], ntk[kClasses];
-    cum[0] = 0;
-#pragma unroll
-    for (int c = 0; c < kClasses; ++c) {
-      const int np = qp.npages[c];
-      cb[c] = qp.first[c] + static_cast<int>(static_cast<int64_t>(split) * np / nsplit);
-      const int ce = qp.first[c] + static_cast<int>(static_cast<int64_t>(split + 1) * np / nsplit);
-      cum[c + 1] = cum[c] + (ce - cb[c]);
-      ntk[c] = qp.ntok[c];
-    }
-    const int T = cum[kClasses];
-    const int64_t ptrow = static_cast<int64_t>(seq) * 4 * a.MP;
+  // ------------------------------------------------------------ producer --
+  // Items are dealt round-robin.  The descriptor of the producer's next item is
+  // prefetched one item ahead (three words per lane), so starting an item costs no
+  // global round trip.
+  int next_item = blockIdx.x * nwarps + warp;
+  int nd0 = 0, nd1 = 0, nd2 = 0;       // prefetched descriptor: page ids, class|fill, header
+  int wid = -1, wmeta = 0;             // the producer's item: page id / class|fill of page `lane`
+  int pf = 0, pT = 0;                  // next page of the producer's item, its page count
+  bool pvalid = false;
+  uint32_t issued = 0, consumed = 0;   // pages issued / consumed by this warp
+  int head = 0, used = 0;              // ring: next free offset, bytes held
 
-    // query: this lane's 32 dimensions, scaled into the log2 domain
-    const int part = lane % LPK;
-    float qf[32];
-    float sumq = 0.f;
-    {
-      const uint4* qp4 = reinterpret_cast<const uint4*>(ka.q + (static_cast<int64_t>(qi) * a.Hq + qh) * D + part * 32);
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const uint4 u = qp4[q];
-        qf[8 * q + 0] = bf_lo(u.x) * ka.qscale;
-        qf[8 * q + 1] = bf_hi(u.x) * ka.qscale;
-        qf[8 * q + 2] = bf_lo(u.y) * ka.qscale;
-        qf[8 * q + 3] = bf_hi(u.y) * ka.qscale;
-        qf[8 * q + 4] = bf_lo(u.z) * ka.qscale;
-        qf[8 * q + 5] = bf_hi(u.z) * ka.qscale;
-        qf[8 * q + 6] = bf_lo(u.w) * ka.qscale;
-        qf[8 * q + 7] = bf_hi(u.w) * ka.qscale;
-      }
-#pragma unroll
-      for (int j = 0; j < 32; ++j) sumq += qf[j];
+  auto prefetch = [&](int item) {
+    if (item >= total) return;
+    const int* d = reinterpret_cast<const int*>(a.desc + item / a.units);
+    nd0 = d[lane];
+    nd1 = d[32 + lane];
+    nd2 = lane < 8 ? d[64 + lane] : 0;
+  };
+  auto start_item = [&]() -> bool {
+    if (next_item >= total) return false;
+    const int item = next_item;
+    wid = nd0;
+    wmeta = nd1;
+    const int qi = __shfl_sync(0xffffffffu, nd2, 0);
+    const int lo = __shfl_sync(0xffffffffu, nd2, 2), hi = __shfl_sync(0xffffffffu, nd2, 3);
+    const int nsplit = __shfl_sync(0xffffffffu, nd2, 4);
+    pT = __shfl_sync(0xffffffffu, nd2, 6);
+    const int unit = item - (item / a.units) * a.units;
+    const int base = __shfl_sync(0xffffffffu, nd2, 7);
+    next_item += wstride;
+    prefetch(next_item);
+    if (lane == 0) {
+      ProdItem t;
+      t.item = item; t.qi = qi; t.qh = unit; t.kvh = unit / group; t.nsplit = nsplit;
+      t.T = pT; t.lo = lo; t.hi = hi; t.base = base;
+      *pi = t;
     }
-    LaneState st;
-    st.m = kNegInf;
-    st.l = 0.f;
-    st.zacc = 0.f;
-#pragma unroll
-    for (int j = 0; j < 32; ++j) st.acc[j] = 0.f;
-
-    // page ids of flat pages [wbase, wbase + 32), one per lane
-    auto class_of_flat = [&](int f) { return (f >= cum[1]) + (f >= cum[2]) + (f >= cum[3]); };
-    int wbase = 0, wid = -1;
-    auto load_window = [&](int base) {
-      const int f = base + lane;
-      wid = -1;
-      if (f < T) {
-        const int c = class_of_flat(f);
-        wid = a.pt[ptrow + c * a.MP + cb[c] + (f - cum[c])];
-      }
-    };
-    load_window(0);
-    auto issue = [&](int f) {  // warp-uniform: start the copy of flat page f
-      if (f - wbase >= 32) {
-        wbase += 32;
-        load_window(wbase);
-      }
-      const int c = class_of_flat(f);
-      const int id = __shfl_sync(0xffffffffu, wid, f - wbase);
-      const uint32_t slot = (gcount + f) % ka.ns;
-      if (lane == 0) {
+    __syncwarp();
+    pf = 0;
+    return true;
+  };
+  // start the copy of the producer's next page if a slot and ring space are free
+  auto try_issue = [&]() -> bool {
+    if (!pvalid) {
+      pvalid = start_item();
+      if (!pvalid) return false;
+    }
+    if (issued - consumed >= kSlots) return false;
+    const bool first = pf == 0;
+    int c = 0, fill = 0, id = -1, bytes_page = 0;
+    if (pT > 0) {
+      id = __shfl_sync(0xffffffffu, wid, pf);
+      const int m = __shfl_sync(0xffffffffu, wmeta, pf);
+      c = m & 255;
+      fill = m >> 8;
+      bytes_page = a.slice[c] + 4 * a.P;
+    }
+    const int need = bytes_page + (first ? qrow : 0);
+    if (used == 0) head = 0;  // an empty ring can start anywhere
+    int off = head, waste = 0;
+    if (off + need > R) {
+      waste = R - off;
+      off = 0;
+    }
+    if (used + waste + need > R) return false;
+    head = off + need;
+    used += waste + need;
+    const uint32_t slot = issued % kSlots;
+    if (lane == 0) {
+      const ProdItem& it = *pi;
+      SlotInfo si;
+      si.cls = c;
+      si.fill = fill;
+      si.lo = it.lo;
+      si.hi = it.hi;
+      si.flags = (first ? 1 : 0) | (pf + 1 >= pT ? 2 : 0) | (pT == 0 ? 4 : 0);
+      si.item = it.item;
+      si.qi = it.qi;
+      si.qh = it.qh;
+      si.nsplit = it.nsplit;
+      si.off = off;
+      si.qoff = off + bytes_page;
+      si.span = waste + need;
+      si.base = it.base;
+      si.pad0 = si.pad1 = si.pad2 = 0;
+      sinfo[slot] = si;
+      fence_proxy_async_smem();
+      mbar_arrive_expect_tx(&bars[slot], need);
+      if (pT > 0) {
         const uint8_t* page = a.pool[c] + static_cast<int64_t>(id) * a.page_bytes[c];
-        fence_proxy_async_smem();
-        mbar_arrive_expect_tx(&bars[slot], a.slice[c] + 4 * a.P);
-        bulk_g2s(slots + slot * ka.slot_bytes, page + a.hdr + static_cast<int64_t>(kvh) * a.slice[c], a.slice[c],
+        bulk_g2s(ring + off, page + a.hdr + static_cast<int64_t>(it.kvh) * a.slice[c], a.slice[c], &bars[slot]);
+        bulk_g2s(ring + off + a.slice[c], page, 4 * a.P, &bars[slot]);
+      }
+      if (first)
+        bulk_g2s(ring + off + bytes_page, ka.q + (static_cast<int64_t>(it.qi) * a.Hq + it.qh) * D, qrow,
                  &bars[slot]);
-        bulk_g2s(wpos + slot * a.P, page, 4 * a.P, &bars[slot]);
-      }
-    };
-    const int pre = min(T, ka.ns);
-    for (int f = 0; f < pre; ++f) issue(f);
-    bool timed_out = false;
-    for (int f = 0; f < T; ++f) {
-      const uint32_t g = gcount + f;
-      const uint32_t slot = g % ka.ns;
-      const bool arrived = mbar_wait(&bars[slot], (g / ka.ns) & 1);
-      if (!__all_sync(0xffffffffu, arrived)) {  // give up together, never half a warp
-        timed_out = true;
-        // wait (bounded) for the copies still in flight, then give up on this kernel
-        for (int r = f + 1; r < min(T, f + ka.ns); ++r) {
-          const uint32_t g2 = gcount + r;
-          mbar_wait(&bars[g2 % ka.ns], (g2 / ka.ns) & 1);
-        }
-        break;
-      }
-      const int c = class_of_flat(f);
-      const int kidx = cb[c] + (f - cum[c]);
-      const int fill = min(a.P, ntk[c] - kidx * a.P);
-      const uint8_t* sl = slots + slot * ka.slot_bytes;
-      const int* sp = wpos + slot * a.P;
-      switch (c) {
-        case 0: consume_page<D, 2>(sl, sp, a.P, a.G, fill, lo, hi, qf, sumq, st, lane); break;
-        case 1: consume_page<D, 4>(sl, sp, a.P, a.G, fill, lo, hi, qf, sumq, st, lane); break;
-        case 2: consume_page<D, 8>(sl, sp, a.P, a.G, fill, lo, hi, qf, sumq, st, lane); break;
-        default: consume_page<D, 16>(sl, sp, a.P, a.G, fill, lo, hi, qf, sumq, st, lane); break;
-      }
-      __syncwarp();
-      if (f + ka.ns < T) issue(f + ka.ns);
     }
-    if (timed_out) {
+    __syncwarp();
+    ++issued;
+    ++pf;
+    if (pf >= pT) pvalid = false;
+    return true;
+  };
+
+  prefetch(next_item);
+  while (try_issue()) {
+  }
+
+  // ------------------------------------------------------------ consumer --
+  const int part = lane % LPK, kl = lane / LPK;
+  LaneState st;
+  float qp[32];
+  float sumq = 0.f;
+  int cur_cls = 3;
+  st.m = kNegInf;
+  st.l = 0.f;
+  st.zacc = 0.f;
+  while (consumed < issued) {
+    const uint32_t g = consumed;
+    const uint32_t slot = g % kSlots;
+    const bool arrived = mbar_wait(&bars[slot], (g / kSlots) & 1);
+    if (!__all_sync(0xffffffffu, arrived)) {  // give up together, never half a warp
+      for (uint32_t r = g + 1; r < issued; ++r) mbar_wait(&bars[r % kSlots], (r / kSlots) & 1);
       if (lane == 0) set_status(a.ctrl, TRR_ERR_TIMEOUT);
+      finish_warp(a.ctrl, gridDim.x * nwarps, lane);
       return;
     }
-    gcount += T;
+    const SlotInfo si = sinfo[slot];
+    if (si.flags & 1) {  // first page of an item: query row and a fresh state
+      const uint4* q4 = reinterpret_cast<const uint4*>(ring + si.qoff + part * 64);
+      sumq = 0.f;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const uint4 u = q4[q];
+        const uint32_t wv[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int h = 0; h < 4; ++h) {
+          qp[8 * q + 2 * h] = bf_lo(wv[h]) * ka.qscale;
+          qp[8 * q + 2 * h + 1] = bf_hi(wv[h]) * ka.qscale;
+        }
+      }
+#pragma unroll
+      for (int j = 0; j < 32; ++j) sumq += qp[j];
+      cur_cls = 3;  // the neutral scale is class 16's
+      st.m = kNegInf;
+      st.l = 0.f;
+      st.zacc = 0.f;
+#pragma unroll
+      for (int j = 0; j < 32; ++j) st.acc[j] = 0.f;
+    }
+    if (!(si.flags & 4)) {
+      if (si.cls != cur_cls) {
+        rescale_q_dyn(qp, cur_cls, si.cls);
+        cur_cls = si.cls;
+      }
+      const uint8_t* sl = ring + si.off;
+      const int* sp = reinterpret_cast<const int*>(ring + si.off + a.slice[si.cls]);
+      switch (si.cls) {
+        case 0: consume_page<D, 2>(sl, sp, a.P, a.G, si.fill, si.lo, si.hi, qp, sumq, st, lane); break;
+        case 1: consume_page<D, 4>(sl, sp, a.P, a.G, si.fill, si.lo, si.hi, qp, sumq, st, lane); break;
+        case 2: consume_page<D, 8>(sl, sp, a.P, a.G, si.fill, si.lo, si.hi, qp, sumq, st, lane); break;
+        default: consume_page<D, 16>(sl, sp, a.P, a.G, si.fill, si.lo, si.hi, qp, sumq, st, lane); break;
+      }
+    }
+    __syncwarp();
+    used -= si.span;  // release the slot's ring bytes, refill
+    consumed = g + 1;
+    while (try_issue()) {
+    }
+    if (!(si.flags & 2)) continue;
 
-    // merge the lanes that share a part: max, rescale, sum
+    // ---- last page of the item: merge the lanes that share a part.  Rescale to the
+    // common maximum, then reduce-scatter over the key lanes: each halving step keeps
+    // half of the 32 dims and sends the other half to the partner lane.
     float M = st.m;
 #pragma unroll
     for (int o = LPK; o < 32; o <<= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
@@ -410,61 +640,60 @@ __global__ void __launch_bounds__(256, 1) attn_kernel(const AttnKernelArgs ka) {
 #pragma unroll
     for (int o = LPK; o < 32; o <<= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
 #pragma unroll
-    for (int j = 0; j < 32; ++j) {
-      float x = (st.acc[j] + st.zacc) * f;
+    for (int j = 0; j < 32; ++j) st.acc[j] = fmaf(st.acc[j], pow2f(49), st.zacc) * f;
 #pragma unroll
-      for (int o = LPK; o < 32; o <<= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
-      st.acc[j] = x;
-    }
-    const int64_t orow = (static_cast<int64_t>(qi) * a.Hq + qh) * D;
-    if (nsplit == 1) {
-      if (lane < LPK) {
-        const float inv = L > 0.f ? 1.f / L : 0.f;
-        uint4* o4 = reinterpret_cast<uint4*>(ka.out + orow + part * 32);
+    for (int width = 16, o = 16; o >= LPK; width >>= 1, o >>= 1) {
+      const bool upper = lane & o;
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          uint32_t w[4];
-#pragma unroll
-          for (int h = 0; h < 4; ++h) {
-            const __nv_bfloat162 b2 = __floats2bfloat162_rn(st.acc[8 * q + 2 * h] * inv, st.acc[8 * q + 2 * h + 1] * inv);
-            w[h] = *reinterpret_cast<const uint32_t*>(&b2);
-          }
-          o4[q] = make_uint4(w[0], w[1], w[2], w[3]);
+      for (int i = 0; i < 16; ++i) {
+        if (i < width) {
+          const float keep = upper ? st.acc[width + i] : st.acc[i];
+          const float give = upper ? st.acc[i] : st.acc[width + i];
+          st.acc[i] = keep + __shfl_xor_sync(0xffffffffu, give, o);
         }
       }
+    }
+    // lane (kl, part) now holds dims part*32 + DPL*kl .. + DPL-1 in acc[0 .. DPL-1]
+    const int64_t orow = (static_cast<int64_t>(si.qi) * a.Hq + si.qh) * D;
+    const int dim0 = part * 32 + DPL * kl;
+    if (si.nsplit == 1) {
+      const float inv = L > 0.f ? 1.f / L : 0.f;
+#pragma unroll
+      for (int j = 0; j < DPL; j += 2)
+        *reinterpret_cast<__nv_bfloat162*>(ka.out + orow + dim0 + j) =
+            __floats2bfloat162_rn(st.acc[j] * inv, st.acc[j + 1] * inv);
       continue;
     }
-    // several splits: store this one's partial, the last to arrive merges them all
-    const int first_item = s_base[qi] + unit * nsplit;
-    float* pp = a.part + static_cast<int64_t>(item) * (D + 4);
-    if (lane < LPK) {
-      float4* p4 = reinterpret_cast<float4*>(pp + part * 32);
+    // several splits: store this one's partial (at the item's index), the last to
+    // arrive merges them all; split s of this query head is item (base + s)*units + unit
+    const int unit = si.qh;
+    const int split0 = si.base;
+    float* pp = a.part + static_cast<int64_t>(si.item) * (D + 4);
 #pragma unroll
-      for (int q = 0; q < 8; ++q) p4[q] = make_float4(st.acc[4 * q], st.acc[4 * q + 1], st.acc[4 * q + 2], st.acc[4 * q + 3]);
-      if (lane == 0) {
-        pp[D] = M;
-        pp[D + 1] = L;
-      }
-    }
+    for (int j = 0; j < DPL; j += 2) *reinterpret_cast<float2*>(pp + dim0 + j) = make_float2(st.acc[j], st.acc[j + 1]);
+    if (lane == 0) *reinterpret_cast<float2*>(pp + D) = make_float2(M, L);
     __threadfence();
     __syncwarp();
     int last = 0;
-    int32_t* counter = a.cnt + static_cast<int64_t>(qi) * a.units + unit;
-    if (lane == 0) last = atomicAdd(counter, 1) == nsplit - 1;
+    int32_t* counter = a.cnt + static_cast<int64_t>(si.qi) * a.units + unit;
+    if (lane == 0) last = atomicAdd(counter, 1) == si.nsplit - 1;
     last = __shfl_sync(0xffffffffu, last, 0);
     if (!last) continue;
     __threadfence();
-    constexpr int DPL = D / 32;  // dimensions per lane in the merge
     float Mx = kNegInf;
-    for (int s = 0; s < nsplit; ++s) Mx = fmaxf(Mx, __ldcg(a.part + static_cast<int64_t>(first_item + s) * (D + 4) + D));
+    for (int s = lane; s < si.nsplit; s += 32)
+      Mx = fmaxf(Mx, __ldcg(a.part + (static_cast<int64_t>(split0 + s) * a.units + unit) * (D + 4) + D));
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) Mx = fmaxf(Mx, __shfl_xor_sync(0xffffffffu, Mx, o));
     float Ls = 0.f, o[DPL];
 #pragma unroll
     for (int j = 0; j < DPL; ++j) o[j] = 0.f;
-    for (int s = 0; s < nsplit; ++s) {
-      const float* ps = a.part + static_cast<int64_t>(first_item + s) * (D + 4);
-      const float ms = __ldcg(ps + D);
-      const float wgt = (ms == kNegInf) ? 0.f : exp2f(ms - Mx);
-      Ls = fmaf(wgt, __ldcg(ps + D + 1), Ls);
+#pragma unroll 4
+    for (int s = 0; s < si.nsplit; ++s) {
+      const float* ps = a.part + (static_cast<int64_t>(split0 + s) * a.units + unit) * (D + 4);
+      const float2 ml = __ldcg(reinterpret_cast<const float2*>(ps + D));
+      const float wgt = (ml.x == kNegInf) ? 0.f : exp2f(ml.x - Mx);
+      Ls = fmaf(wgt, ml.y, Ls);
 #pragma unroll
       for (int j = 0; j < DPL; ++j) o[j] = fmaf(wgt, __ldcg(ps + lane * DPL + j), o[j]);
     }
@@ -476,9 +705,10 @@ __global__ void __launch_bounds__(256, 1) attn_kernel(const AttnKernelArgs ka) {
     }
     if (lane == 0) *counter = 0;
   }
+  finish_warp(a.ctrl, gridDim.x * nwarps, lane);
 }
 
-constexpr int kAttnSmemLimit = 200 * 1024;  // dynamic shared memory of one attention CTA
+constexpr int kAttnSmemLimit = 110 * 1024;  // dynamic shared memory of one attention CTA
 
 // Done once per cache at creation, so that calls stay legal inside stream capture.
 cudaError_t attn_configure() {
@@ -506,8 +736,9 @@ extern "C" trr_status trr_decode_attn(trr_cache* cache, int32_t layer, int32_t n
     return TRR_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const LayerArgs a = layer_args(l, cache_views(cache), layer);
-  attn_plan_kernel<<<(n + 7) / 8, 256, 0, s>>>(a, n, seq_ids, q_positions, modes, windows, window_scalar,
-                                               static_cast<uint16_t*>(out_bf16));
+  cudaError_t e = launch_pdl(attn_plan_kernel, dim3((n + 7) / 8), dim3(256), 0, s, a, n, seq_ids, q_positions,
+                             modes, windows, window_scalar, static_cast<uint16_t*>(out_bf16));
+  if (e != cudaSuccess) return TRR_ERR_CUDA;
   AttnKernelArgs ka;
   ka.a = a;
   ka.n = n;
@@ -515,19 +746,18 @@ extern "C" trr_status trr_decode_attn(trr_cache* cache, int32_t layer, int32_t n
   ka.out = static_cast<uint16_t*>(out_bf16);
   const float scale = softmax_scale > 0.f ? softmax_scale : 1.f / sqrtf(static_cast<float>(l.d));
   ka.qscale = scale * 1.4426950408889634f;
-  ka.ns = 4;
-  ka.slot_bytes = static_cast<int>(l.slice[3]);
-  ka.base_bytes = ((n + 1) * 4 + 127) / 128 * 128;
-  const int per_warp = ka.ns * (ka.slot_bytes + 4 * l.P + 8);
-  const int budget = kAttnSmemLimit - ka.base_bytes;
-  const int nwarps = std::min(8, budget / per_warp);
+  // a ring holds at least one page of the widest class with its positions and a query row
+  const int widest = static_cast<int>(l.slice[3]) + 4 * l.P + 2 * l.d;
+  ka.ring_bytes = std::max(12 * 1024, (widest + 127) / 128 * 128);
+  int nwarps = 8;
+  while (nwarps > 0 && AttnSmem(nwarps, ka.ring_bytes).total > kAttnSmemLimit) --nwarps;
   if (nwarps < 1) return TRR_ERR_UNSUPPORTED;
-  const int smem = ka.base_bytes + nwarps * per_warp;
-  const int grid = cache_num_sms(cache);
+  const int smem = AttnSmem(nwarps, ka.ring_bytes).total;
+  const int grid = 2 * cache_num_sms(cache);
   if (l.d == 64)
-    attn_kernel<64><<<grid, nwarps * 32, smem, s>>>(ka);
+    e = launch_pdl(attn_kernel<64>, dim3(grid), dim3(nwarps * 32), static_cast<size_t>(smem), s, ka);
   else
-    attn_kernel<128><<<grid, nwarps * 32, smem, s>>>(ka);
+    e = launch_pdl(attn_kernel<128>, dim3(grid), dim3(nwarps * 32), static_cast<size_t>(smem), s, ka);
   cache_set_launches(cache, 2);
-  return cudaGetLastError() == cudaSuccess ? TRR_OK : TRR_ERR_CUDA;
+  return e == cudaSuccess ? TRR_OK : TRR_ERR_CUDA;
 }

@@ -36,6 +36,7 @@ LayerArgs layer_args(const Layout& l, const Views& v, int layer) {
   a.plast = v.plast + ls * 4 * l.MP;
   a.aplan = v.aplan;
   a.qplan = v.qplan;
+  a.desc = v.desc;
   a.cnt = v.cnt;
   a.part = v.part;
   return a;
@@ -78,8 +79,12 @@ static trr_status make_layout(const trr_cache_config* c, Layout* l) {
     l->page_bytes[k] = roundup(l->hdr + l->Hkv * l->slice[k], 128);
   }
   l->units = l->Hq;
+  // splits per query: enough for split_bytes each even if every token were bf16, and
+  // enough to keep each split within kDescMaxPages pages (+ one partial page per class)
   const int64_t most = static_cast<int64_t>(l->maxctx) * l->tokb[3];
-  l->s_cap = static_cast<int>(std::min<int64_t>(128, std::max<int64_t>(1, (most + l->split_bytes - 1) / l->split_bytes)));
+  const int64_t by_bytes = (most + l->split_bytes - 1) / l->split_bytes;
+  const int64_t by_pages = (l->MP + kClasses + kDescMaxPages - 1) / kDescMaxPages;
+  l->s_cap = static_cast<int>(std::max<int64_t>(1, std::max(by_bytes, by_pages)));
   l->max_items = static_cast<int64_t>(l->max_queries) * l->units * l->s_cap;
 
   const int64_t nls = static_cast<int64_t>(l->L) * l->S;
@@ -98,6 +103,7 @@ static trr_status make_layout(const trr_cache_config* c, Layout* l) {
   l->off_plast = take(16 * nls * l->MP);
   l->off_aplan = take(static_cast<int64_t>(sizeof(AppendPlan)) * l->max_append);
   l->off_qplan = take(static_cast<int64_t>(sizeof(QueryPlan)) * l->max_queries);
+  l->off_desc = take(static_cast<int64_t>(sizeof(SplitDesc)) * l->max_queries * l->s_cap);
   l->off_cnt = take(4 * static_cast<int64_t>(l->max_queries) * l->units);
   l->off_part = take(4 * l->max_items * (l->Hq / l->units) * (l->d + 4));
   for (int k = 0; k < kClasses; ++k) l->off_pool[k] = take(l->cap[k] * l->page_bytes[k]);

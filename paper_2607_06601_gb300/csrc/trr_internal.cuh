@@ -21,6 +21,8 @@ enum Ctrl : int {
   kWorkCounter = 8,   // attention: next work item to hand out
   kAppendOk = 10,     // append: 1 when the plan kernel committed the call
   kFirstBadQuery = 12,// attention: lowest failing query index (INT_MAX = none)
+  kDescCounter = 13,  // attention: split descriptors handed out by the plan kernel
+  kDoneWarps = 14,    // attention: warps finished (the last one resets the two counters)
   kCtrlInts = 64
 };
 
@@ -34,7 +36,7 @@ struct Layout {
   int64_t max_items;
   int64_t hdr, tokb[kClasses], slice[kClasses], page_bytes[kClasses];
   int64_t off_ctrl, off_last_pos, off_ntok, off_presence, off_pt, off_pfirst, off_plast;
-  int64_t off_aplan, off_qplan, off_cnt, off_part, off_pool[kClasses], total;
+  int64_t off_aplan, off_qplan, off_desc, off_cnt, off_part, off_pool[kClasses], total;
 };
 
 // Per-query plan written by the attention plan kernel.
@@ -46,6 +48,19 @@ struct QueryPlan {
   int err, pad0, pad1, pad2;
 };
 static_assert(sizeof(QueryPlan) == 80, "QueryPlan is 80 bytes");
+
+// One split-K work unit of one query, written by the attention plan kernel: the ids
+// of its pages (at most kDescPages, in class-then-position order), each page's width
+// class and token count, and the query's key range.  Laid out so that a warp loads it
+// with three coalesced words per lane.
+constexpr int kDescPages = 32;
+constexpr int kDescMaxPages = 28;  // splits are sized to hold at most this many pages, + 4
+struct SplitDesc {
+  int page[kDescPages];
+  int meta[kDescPages];  // class | fill << 8
+  int qi, seq, lo, hi, nsplit, split, T, base;  // base: descriptor index of split 0
+};
+static_assert(sizeof(SplitDesc) == 288, "SplitDesc is 288 bytes");
 
 // Per-entry plan written by the append plan kernel.
 struct AppendPlan {
@@ -65,6 +80,7 @@ struct Views {  // typed device pointers into the cache memory
   int32_t* plast;
   AppendPlan* aplan;
   QueryPlan* qplan;
+  SplitDesc* desc;
   int32_t* cnt;
   float* part;
   uint8_t* pool[kClasses];
@@ -82,6 +98,7 @@ inline Views make_views(const Layout& l, void* base) {
   v.plast = reinterpret_cast<int32_t*>(b + l.off_plast);
   v.aplan = reinterpret_cast<AppendPlan*>(b + l.off_aplan);
   v.qplan = reinterpret_cast<QueryPlan*>(b + l.off_qplan);
+  v.desc = reinterpret_cast<SplitDesc*>(b + l.off_desc);
   v.cnt = reinterpret_cast<int32_t*>(b + l.off_cnt);
   v.part = reinterpret_cast<float*>(b + l.off_part);
   for (int c = 0; c < kClasses; ++c) v.pool[c] = b + l.off_pool[c];
@@ -104,6 +121,7 @@ struct LayerArgs {
   int32_t* plast;
   AppendPlan* aplan;
   QueryPlan* qplan;
+  SplitDesc* desc;     // [max_queries][s_cap]
   int32_t* cnt;
   float* part;
   uint8_t* pool[kClasses];
@@ -153,15 +171,17 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
       : "memory");
 }
 
-// Bounded wait for phase `parity` of `bar`: returns false when it gave up.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint32_t max_tries = 1u << 22) {
+// Bounded wait for phase `parity` of `bar`: returns false when it gave up.  Each try
+// parks the thread until the phase completes or about 20 us pass, so a waiting warp
+// does not take issue slots; at most max_tries tries (about a second).
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint32_t max_tries = 50000) {
   uint32_t addr = smem_u32(bar);
   for (uint32_t i = 0; i < max_tries; ++i) {
     uint32_t done;
     asm volatile(
-        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n selp.u32 %0, 1, 0, p;\n}"
         : "=r"(done)
-        : "r"(addr), "r"(parity)
+        : "r"(addr), "r"(parity), "r"(20000)
         : "memory");
     if (done) return true;
   }
@@ -170,6 +190,29 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint32
 
 __device__ __forceinline__ void set_status(int32_t* ctrl, int code) {
   atomicCAS(ctrl + kStatus, 0, code);
+}
+
+// Programmatic dependent launch: a kernel launched with launch_pdl may start while the
+// previous kernel of the stream is still running; it must call pdl_wait() before it
+// touches memory that kernel writes, and calls pdl_trigger() to let its own successor
+// start early.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+template <typename... Args>
+inline cudaError_t launch_pdl(void (*kern)(Args...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                              Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, args...);
 }
 
 }  // namespace trr
