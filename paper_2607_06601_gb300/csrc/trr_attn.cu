@@ -761,3 +761,111 @@ extern "C" trr_status trr_decode_attn(trr_cache* cache, int32_t layer, int32_t n
   cache_set_launches(cache, 2);
   return e == cudaSuccess ? TRR_OK : TRR_ERR_CUDA;
 }
+
+// ------------------------------------------------------ static-scratch variant --
+//
+// trr_decode_attn_static runs the same two kernels as trr_decode_attn, but keeps all
+// of its per-call scratch (query plans, split descriptors, arrival counters, fp32
+// partials and the call's control words) in one file-scope device array instead of
+// the cache's scratch region.  Nothing is allocated per call or at set-up.
+namespace trr {
+
+constexpr int64_t kStaticScratchBytes = 32ll << 20;  // 32 MiB on every device using the library
+static __device__ __align__(256) uint8_t g_static_scratch[kStaticScratchBytes];
+
+constexpr int kMaxDevices = 64;
+static void* g_static_ptr[kMaxDevices];  // device address of g_static_scratch, per device
+
+// Address of the array on the current device, looked up once per device.
+static cudaError_t static_scratch(void** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+  if (!g_static_ptr[dev]) {
+    void* ptr = nullptr;
+    e = cudaGetSymbolAddress(&ptr, g_static_scratch);
+    if (e != cudaSuccess) return e;
+    g_static_ptr[dev] = ptr;
+  }
+  *out = g_static_ptr[dev];
+  return cudaSuccess;
+}
+
+// Clears what a call needs at zero: the control words and the arrival counters.
+__global__ void static_scratch_clear_kernel(int32_t* wctrl, int32_t* cnt, int ncnt) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < kCtrlInts) wctrl[i] = i == kFirstBadQuery ? INT_MAX : 0;
+  for (int j = i; j < ncnt; j += gridDim.x * blockDim.x) cnt[j] = 0;
+}
+
+// Forwards the call's first error to the cache's sticky status word.
+__global__ void static_scratch_status_kernel(const int32_t* wctrl, int32_t* ctrl) {
+  const int st = wctrl[kStatus];
+  if (st != 0) atomicCAS(ctrl + kStatus, 0, st);
+}
+
+}  // namespace trr
+
+extern "C" trr_status trr_decode_attn_static(trr_cache* cache, int32_t layer, int32_t n, const int32_t* seq_ids,
+                                             const int32_t* q_positions, const void* q_bf16, const uint8_t* modes,
+                                             const int32_t* windows, int32_t window_scalar, float softmax_scale,
+                                             void* out_bf16, void* stream) {
+  if (!cache) return TRR_ERR_INVALID_ARG;
+  const Layout& l = cache_layout(cache);
+  if (layer < 0 || layer >= l.L || n < 0) return TRR_ERR_INVALID_ARG;
+  cache_set_launches(cache, 0);
+  if (n == 0) return TRR_OK;
+  if (!seq_ids || !q_positions || !q_bf16 || !modes || !out_bf16) return TRR_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(q_bf16) | reinterpret_cast<uintptr_t>(out_bf16)) & 15)
+    return TRR_ERR_INVALID_ARG;
+  // scratch of this call, carved from the static array; reject what does not fit
+  auto up = [](int64_t x) { return (x + 255) / 256 * 256; };
+  const int64_t nd = static_cast<int64_t>(n) * l.s_cap;  // most split descriptors
+  const int64_t b_ctrl = up(4 * kCtrlInts);
+  const int64_t b_qplan = up(static_cast<int64_t>(sizeof(QueryPlan)) * n);
+  const int64_t b_desc = up(static_cast<int64_t>(sizeof(SplitDesc)) * nd);
+  const int64_t b_cnt = up(4ll * n * l.units);
+  const int64_t b_part = up(4ll * nd * l.units * (l.d + 4));
+  if (b_ctrl + b_qplan + b_desc + b_cnt + b_part > kStaticScratchBytes) return TRR_ERR_OUT_OF_MEMORY;
+  void* base = nullptr;
+  if (static_scratch(&base) != cudaSuccess) return TRR_ERR_CUDA;
+  uint8_t* b = static_cast<uint8_t*>(base);
+  LayerArgs a = layer_args(l, cache_views(cache), layer);
+  int32_t* cache_ctrl = a.ctrl;
+  a.ctrl = reinterpret_cast<int32_t*>(b);
+  a.qplan = reinterpret_cast<QueryPlan*>(b + b_ctrl);
+  a.desc = reinterpret_cast<SplitDesc*>(b + b_ctrl + b_qplan);
+  a.cnt = reinterpret_cast<int32_t*>(b + b_ctrl + b_qplan + b_desc);
+  a.part = reinterpret_cast<float*>(b + b_ctrl + b_qplan + b_desc + b_cnt);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int ncnt = n * l.units;
+  static_scratch_clear_kernel<<<std::max(1, std::min(256, (ncnt + 255) / 256)), 256, 0, s>>>(a.ctrl, a.cnt, ncnt);
+  cudaError_t e = cudaGetLastError();
+  if (e == cudaSuccess)
+    e = launch_pdl(attn_plan_kernel, dim3((n + 7) / 8), dim3(256), 0, s, a, n, seq_ids, q_positions, modes,
+                   windows, window_scalar, static_cast<uint16_t*>(out_bf16));
+  if (e != cudaSuccess) return TRR_ERR_CUDA;
+  AttnKernelArgs ka;
+  ka.a = a;
+  ka.n = n;
+  ka.q = static_cast<const uint16_t*>(q_bf16);
+  ka.out = static_cast<uint16_t*>(out_bf16);
+  const float scale = softmax_scale > 0.f ? softmax_scale : 1.f / sqrtf(static_cast<float>(l.d));
+  ka.qscale = scale * 1.4426950408889634f;
+  const int widest = static_cast<int>(l.slice[3]) + 4 * l.P + 2 * l.d;
+  ka.ring_bytes = std::max(12 * 1024, (widest + 127) / 128 * 128);
+  int nwarps = 8;
+  while (nwarps > 0 && AttnSmem(nwarps, ka.ring_bytes).total > kAttnSmemLimit) --nwarps;
+  if (nwarps < 1) return TRR_ERR_UNSUPPORTED;
+  const int smem = AttnSmem(nwarps, ka.ring_bytes).total;
+  const int grid = 2 * cache_num_sms(cache);
+  if (l.d == 64)
+    e = launch_pdl(attn_kernel<64>, dim3(grid), dim3(nwarps * 32), static_cast<size_t>(smem), s, ka);
+  else
+    e = launch_pdl(attn_kernel<128>, dim3(grid), dim3(nwarps * 32), static_cast<size_t>(smem), s, ka);
+  if (e != cudaSuccess) return TRR_ERR_CUDA;
+  static_scratch_status_kernel<<<1, 1, 0, s>>>(a.ctrl, cache_ctrl);
+  cache_set_launches(cache, 4);
+  return cudaGetLastError() == cudaSuccess ? TRR_OK : TRR_ERR_CUDA;
+}

@@ -39,7 +39,7 @@ class trr_cache_config(ctypes.Structure):
 
 
 EXPORTS = ("trr_cache_required_bytes", "trr_create_cache", "trr_kv_append", "trr_decode_attn",
-           "trr_destroy", "trr_get_status", "trr_reset", "trr_get_region",
+           "trr_decode_attn_static", "trr_destroy", "trr_get_status", "trr_reset", "trr_get_region",
            "trr_last_launch_count")
 
 _lib = None
@@ -65,6 +65,7 @@ def load(build_if_missing: bool = False) -> ctypes.CDLL:
     L.trr_create_cache.argtypes = [ctypes.POINTER(trr_cache_config), ctypes.POINTER(P)]
     L.trr_kv_append.argtypes = [P, I32, I32, P, P, P, P, P, P, P]
     L.trr_decode_attn.argtypes = [P, I32, I32, P, P, P, P, P, I32, ctypes.c_float, P, P]
+    L.trr_decode_attn_static.argtypes = [P, I32, I32, P, P, P, P, P, I32, ctypes.c_float, P, P]
     L.trr_destroy.argtypes = [P]
     L.trr_get_status.argtypes = [P, P]
     L.trr_reset.argtypes = [P, P]
@@ -139,6 +140,19 @@ def trr_decode_attn(cache, layer, seq_ids, q_positions, q, modes, windows, windo
     n = seq_ids.numel()
     win = None if windows is None else _dev(windows, torch.int32, "windows")
     _check("trr_decode_attn", load().trr_decode_attn(
+        cache, layer, n, _dev(seq_ids, torch.int32, "seq_ids"),
+        _dev(q_positions, torch.int32, "q_positions"), _dev(q, torch.bfloat16, "q"),
+        _dev(modes, torch.uint8, "modes"), win, int(window_scalar), float(softmax_scale),
+        _dev(out, torch.bfloat16, "out"), _stream(stream)))
+
+
+def trr_decode_attn_static(cache, layer, seq_ids, q_positions, q, modes, windows, window_scalar,
+                           softmax_scale, out, stream=None):
+    """trr_decode_attn with its scratch in the library's static device array: no
+    allocation anywhere on the way (see include/trr.h)."""
+    n = seq_ids.numel()
+    win = None if windows is None else _dev(windows, torch.int32, "windows")
+    _check("trr_decode_attn_static", load().trr_decode_attn_static(
         cache, layer, n, _dev(seq_ids, torch.int32, "seq_ids"),
         _dev(q_positions, torch.int32, "q_positions"), _dev(q, torch.bfloat16, "q"),
         _dev(modes, torch.uint8, "modes"), win, int(window_scalar), float(softmax_scale),

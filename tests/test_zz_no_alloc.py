@@ -1,0 +1,79 @@
+"""trr_decode_attn_static: decode attention whose per-call scratch lives in the
+library's static device array, for callers that cannot allocate device memory where
+they call it (for instance an engine inside a fixed, fully reserved memory budget).
+
+Checked through the C ABI against trr_decode_attn on the same cache and queries, on two
+calls in a row (the second finds the array holding the first call's contents), with a
+query count above the cache's max_queries, and a call too large for the array is
+refused before anything runs."""
+import numpy as np
+import pytest
+import torch
+
+from paper_2607_06601_gb300 import trr, workloads as wl
+from tests._parity import check_attention, dev
+
+pytestmark = pytest.mark.gpu
+
+
+def _cache_with_context(rng, S=6, n_ctx=400, Hq=8, Hkv=4, d=64):
+    cache = trr.Cache(1, S, Hq, Hkv, d, 32, 16, 512, [S * 40] * 4, max_queries=16)
+    for p0 in range(0, n_ctx, 64):
+        ps = np.arange(p0, min(n_ctx, p0 + 64))
+        seqs = np.repeat(np.arange(S), len(ps)).astype(np.int32)
+        pos = np.tile(ps, S).astype(np.int32)
+        k = wl.bf16_bits(rng.standard_normal((len(seqs), Hkv, d), dtype=np.float32))
+        v = wl.bf16_bits(rng.standard_normal((len(seqs), Hkv, d), dtype=np.float32))
+        order = np.lexsort((seqs, pos))  # position-major: each sequence in order
+        cache.append(0, dev(seqs[order], torch.int32), dev(pos[order], torch.int32),
+                     dev(k[order], torch.bfloat16), dev(v[order], torch.bfloat16),
+                     dev(rng.choice([2, 4, 8, 16], size=len(seqs)).astype(np.uint8), torch.uint8),
+                     dev(rng.choice(3, size=len(seqs)).astype(np.uint8), torch.uint8))
+    return cache
+
+
+def test_static_scratch_matches_decode_attn_on_two_calls():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a GPU")
+    torch.cuda.set_device(0)
+    rng = np.random.default_rng(77)
+    S, Hq, d = 6, 8, 64
+    cache = _cache_with_context(rng, S=S, Hq=Hq, d=d)
+    nq = 48  # more queries than the cache's max_queries (16)
+    seqs = dev(rng.integers(0, S, nq).astype(np.int32), torch.int32)
+    ts = dev(rng.integers(0, 400, nq).astype(np.int32), torch.int32)
+    q = dev(wl.bf16_bits(rng.standard_normal((nq, Hq, d), dtype=np.float32)), torch.bfloat16)
+    modes = dev(rng.choice(3, size=nq).astype(np.uint8), torch.uint8)
+    wins = dev(rng.choice([1, 7, 64, 300], size=nq).astype(np.int32), torch.int32)
+    ref = torch.empty((nq, Hq, d), dtype=torch.bfloat16, device="cuda")
+    for i0 in range(0, nq, 16):  # the existing entry point, within its max_queries
+        sl = slice(i0, i0 + 16)
+        trr.trr_decode_attn(cache.handle, 0, seqs[sl].contiguous(), ts[sl].contiguous(), q[sl].contiguous(),
+                            modes[sl].contiguous(), wins[sl].contiguous(), 0, 0.0, ref[sl])
+    ref_np = ref.float().cpu().numpy().astype(np.float64)
+    assert np.abs(ref_np).max() > 0
+    for _ in range(2):
+        out = torch.full((nq, Hq, d), float("nan"), dtype=torch.bfloat16, device="cuda")
+        trr.trr_decode_attn_static(cache.handle, 0, seqs, ts, q, modes, wins, 0, 0.0, out)
+        got = out.float().cpu().numpy().astype(np.float64)
+        check_attention(got, ref_np, modes.cpu().numpy())
+    assert cache.status() == 0
+
+
+def test_static_scratch_refuses_calls_larger_than_the_array():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a GPU")
+    torch.cuda.set_device(0)
+    rng = np.random.default_rng(78)
+    cache = _cache_with_context(rng, n_ctx=64)
+    nq = 4000
+    seqs = torch.zeros(nq, dtype=torch.int32, device="cuda")
+    ts = torch.zeros(nq, dtype=torch.int32, device="cuda")
+    q = torch.zeros((nq, 8, 64), dtype=torch.bfloat16, device="cuda")
+    modes = torch.full((nq,), 2, dtype=torch.uint8, device="cuda")
+    out = torch.zeros((nq, 8, 64), dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(trr.TrrError) as err:
+        trr.trr_decode_attn_static(cache.handle, 0, seqs, ts, q, modes, None, 0, 0.0, out)
+    assert err.value.code == 2  # TRR_ERR_OUT_OF_MEMORY: nothing launched
+    assert cache.launches() == 0
+    assert cache.status() == 0
