@@ -40,7 +40,7 @@ sys.path.insert(0, ROOT)
 
 METRIC = "decode-attention effective HBM GB/s and % of GB300 peak; attended KV tokens/s"
 UNIT = "GB/s"
-PAGE = 16
+PAGE = 32  # default page size (tokens); --page-size overrides
 BITS = (2, 4, 8, 16)
 
 
@@ -238,7 +238,8 @@ class Bench:
         self.total_steps = args.warmup + 2 * args.steps + self.e2e_warm + self.e2e_steps
         self.grow = 32                                   # tokens a sequence may grow
         self.R = max(1, math.ceil(self.total_steps / self.grow))
-        self.acct = Accounting(s, self.d, self.G, self.Hq, self.Hkv, self.window)
+        self.P = args.page_size or PAGE
+        self.acct = Accounting(s, self.d, self.G, self.Hq, self.Hkv, self.window, self.P)
         self.ctx = wl.contexts(s)                       # prebuilt context per sequence
         self.maxctx = int(self.ctx.max()) + math.ceil(self.total_steps / self.R) + 1
         self.dev = torch.device("cuda", torch.cuda.current_device())
@@ -265,8 +266,8 @@ class Bench:
                 for s in range(B):
                     stored = modes[s] != 0
                     for c, b in enumerate(BITS):
-                        caps[c] += -(-int(np.count_nonzero(stored & (bits[s] == b))) // PAGE) + 1
-        self.cache = trr.Cache(L, S, self.Hq, self.Hkv, self.d, self.G, PAGE, self.maxctx,
+                        caps[c] += -(-int(np.count_nonzero(stored & (bits[s] == b))) // self.P) + 1
+        self.cache = trr.Cache(L, S, self.Hq, self.Hkv, self.d, self.G, self.P, self.maxctx,
                                [int(c) for c in caps], max_append=1024, max_queries=max(B, 64),
                                split_bytes=self.args.split_bytes)
         # prebuild every sequence's context (untimed), K/V drawn on the device
@@ -500,7 +501,7 @@ def run_gpu(args):
             "config": {
                 "workload": f"{bench.spec.name}: {bench.L} layers, MHA/GQA {bench.Hq}/{bench.Hkv} x {bench.d}, "
                             f"batch {bench.B}/GPU, contexts {describe_ctx(bench)}, window {bench.window}, "
-                            f"group {bench.G}, page {PAGE}",
+                            f"group {bench.G}, page {bench.P}",
                 "kv_storage": "per-token 2/4/8-bit codes + fp16 scale/zero, or bf16; fp32 accumulation",
                 "global_batch": bench.B * world, "replicas": bench.R,
                 "l2": "inputs larger than L2: every step reads its replica's "
@@ -636,6 +637,8 @@ def main():
     ap.add_argument("--batch", type=int, default=0)
     ap.add_argument("--layers", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--page-size", type=int, default=0, choices=[0, 16, 32, 64],
+                    help="tokens per cache page (0: 32)")
     ap.add_argument("--split-bytes", type=int, default=0,
                     help="target KV bytes per split-K work item (0: the library default)")
     args = ap.parse_args()

@@ -117,13 +117,15 @@ __global__ void __launch_bounds__(256) attn_plan_kernel(LayerArgs a, int n, cons
   qp.nsplit = 0;
   qp.lo = 0;
   qp.hi = t;
-  qp.pad0 = qp.pad1 = qp.pad2 = 0;
+  qp.base = qp.pad1 = qp.pad2 = 0;
 #pragma unroll
   for (int c = 0; c < kClasses; ++c) qp.first[c] = qp.npages[c] = qp.ntok[c] = 0;
   int total_pages = 0;
+  bool upper_mask = false;  // the query sits before the sequence's last stored position
   if (!err && mode != TRR_MODE_SKIP) {
     const int lo = mode == TRR_MODE_FULL ? 0 : max(0, t - w + 1);
     qp.lo = lo;
+    upper_mask = t < a.last_pos[seq];
     const int* arr[2 * kClasses];
     int np[2 * kClasses], x[2 * kClasses], cnt[2 * kClasses];
 #pragma unroll
@@ -154,8 +156,8 @@ __global__ void __launch_bounds__(256) attn_plan_kernel(LayerArgs a, int n, cons
       qp.nsplit = static_cast<int>(min(ns, static_cast<int64_t>(total_pages)));
     }
   }
-  if (lane < 20) reinterpret_cast<int*>(a.qplan + qi)[lane] = reinterpret_cast<const int*>(&qp)[lane];
   if (qp.nsplit == 0) {  // skip, invalid or nothing stored in range: a zero row
+    if (lane < 20) reinterpret_cast<int*>(a.qplan + qi)[lane] = reinterpret_cast<const int*>(&qp)[lane];
     uint4* o = reinterpret_cast<uint4*>(out + static_cast<int64_t>(qi) * a.Hq * a.d);
     const int n16 = a.Hq * a.d / 8;
     for (int i = lane; i < n16; i += 32) o[i] = make_uint4(0, 0, 0, 0);
@@ -165,22 +167,10 @@ __global__ void __launch_bounds__(256) attn_plan_kernel(LayerArgs a, int n, cons
   // Descriptors: one per split, at consecutive indices taken from a shared counter.
   // Split sp of class c takes the class's pages [first + sp*np/ns, first + (sp+1)*np/ns).
   const int ns = qp.nsplit;
-  int base = 0;
-  if (lane == 0) base = atomicAdd(&a.ctrl[kDescCounter], ns);
-  base = __shfl_sync(0xffffffffu, base, 0);
-  SplitDesc* dsc = a.desc + base;
-  auto bnd = [&](int c, int sp) { return static_cast<int>(static_cast<int64_t>(sp) * qp.npages[c] / ns); };
-  for (int sp = lane; sp < ns; sp += 32) {
-    int T = 0;
-#pragma unroll
-    for (int c = 0; c < kClasses; ++c) T += bnd(c, sp + 1) - bnd(c, sp);
-    int* h = &dsc[sp].qi;
-    h[0] = qi; h[1] = seq; h[2] = qp.lo; h[3] = qp.hi; h[4] = ns; h[5] = sp; h[6] = T; h[7] = base;
-  }
   const int c1 = qp.npages[0], c2 = c1 + qp.npages[1], c3 = c2 + qp.npages[2];
   constexpr int kBatch = 8;  // page ids loaded before any descriptor store
-  for (int f0 = 0; f0 < total_pages; f0 += 32 * kBatch) {
-    int id[kBatch], cls[kBatch], kid[kBatch];
+  int id[kBatch], cls[kBatch], kid[kBatch];
+  auto load_batch = [&](int f0) {
 #pragma unroll
     for (int b = 0; b < kBatch; ++b) {
       const int f = f0 + 32 * b + lane;
@@ -190,6 +180,24 @@ __global__ void __launch_bounds__(256) attn_plan_kernel(LayerArgs a, int n, cons
       kid[b] = qp.first[c] + local;
       id[b] = f < total_pages ? a.pt[static_cast<int64_t>(seq * 4 + c) * a.MP + kid[b]] : -1;
     }
+  };
+  load_batch(0);  // in flight together with the counter atomic
+  int base = 0;
+  if (lane == 0) base = atomicAdd(&a.ctrl[kDescCounter], ns);
+  base = __shfl_sync(0xffffffffu, base, 0);
+  qp.base = base;
+  if (lane < 20) reinterpret_cast<int*>(a.qplan + qi)[lane] = reinterpret_cast<const int*>(&qp)[lane];
+  SplitDesc* dsc = a.desc + base;
+  auto bnd = [&](int c, int sp) { return static_cast<int>(static_cast<int64_t>(sp) * qp.npages[c] / ns); };
+  for (int sp = lane; sp < ns; sp += 32) {
+    int T = 0;
+#pragma unroll
+    for (int c = 0; c < kClasses; ++c) T += bnd(c, sp + 1) - bnd(c, sp);
+    int* h = &dsc[sp].qi;
+    h[0] = qi; h[1] = seq; h[2] = qp.lo; h[3] = qp.hi; h[4] = ns; h[5] = sp; h[6] = T; h[7] = base;
+  }
+  for (int f0 = 0; f0 < total_pages; f0 += 32 * kBatch) {
+    if (f0 > 0) load_batch(f0);
 #pragma unroll
     for (int b = 0; b < kBatch; ++b) {
       const int f = f0 + 32 * b + lane;
@@ -201,8 +209,12 @@ __global__ void __launch_bounds__(256) attn_plan_kernel(LayerArgs a, int n, cons
       int pos = local - bnd(c, sp);
       for (int c0 = 0; c0 < c; ++c0) pos += bnd(c0, sp + 1) - bnd(c0, sp);
       const int fill = min(a.P, qp.ntok[c] - kid[b] * a.P);
+      // slot positions are needed on a page that may hold keys outside [lo, t]: the
+      // first page of a window that starts after 0, the last one when t is not the
+      // sequence's last stored position
+      const bool mask = (qp.lo > 0 && local == 0) || (upper_mask && local == np - 1);
       dsc[sp].page[pos] = id[b];
-      dsc[sp].meta[pos] = c | (fill << 8);
+      dsc[sp].meta[pos] = c | (fill << 2) | (mask ? 512 : 0);
     }
   }
 }
@@ -236,6 +248,16 @@ __device__ __forceinline__ float code_at(const uint32_t* w, const uint32_t* h, i
     return __uint_as_float(__byte_perm(w[i / 4], 0u, 0x4440u | (i % 4)));
   }
 }
+// d = a * b + c on two fp32 lanes at once (packed fp32 FMA).
+__device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) {
+  float2 d;
+  asm("{\n .reg .b64 ra, rb, rc, rd;\n mov.b64 ra, {%2, %3};\n mov.b64 rb, {%4, %5};\n"
+      " mov.b64 rc, {%6, %7};\n fma.rn.f32x2 rd, ra, rb, rc;\n mov.b64 {%0, %1}, rd;\n}"
+      : "=f"(d.x), "=f"(d.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+  return d;
+}
+
 template <int B>
 __device__ __forceinline__ void high_parts(const uint32_t* w, uint32_t* h) {
   constexpr int sh = B == 2 ? 22 : B == 4 ? 20 : 16;
@@ -284,7 +306,8 @@ __device__ __forceinline__ float softmax_step(LaneState& st, float score) {
   return p;
 }
 
-// One page of width class B in shared memory; lane -> (key kl, 32-dim part).
+// One page of width class B in shared memory; lane -> (key kl, 32-dim part).  Keys
+// past `fill` are empty slots; with `spos` set, keys outside [lo, hi] are masked too.
 template <int D, int B>
 __device__ __forceinline__ void consume_page(const uint8_t* sl, const int* spos, int P, int G, int fill,
                                              int lo, int hi, const float (&qp)[32], float sumq,
@@ -296,8 +319,11 @@ __device__ __forceinline__ void consume_page(const uint8_t* sl, const int* spos,
   const int grp = part * 32 / G;
   for (int it = 0; it < P / KPI; ++it) {
     const int key = it * KPI + kl;
-    const int pos = spos[key];
-    const bool valid = key < fill && pos >= lo && pos <= hi;
+    bool valid = key < fill;
+    if (spos) {
+      const int pos = spos[key];
+      valid = valid && pos >= lo && pos <= hi;
+    }
     float dot;
     if (B == 16) {
       const uint4* kp = reinterpret_cast<const uint4*>(sl + (key * D + part * 32) * 2);
@@ -323,12 +349,14 @@ __device__ __forceinline__ void consume_page(const uint8_t* sl, const int* spos,
       for (int k = 0; k < B; ++k) w[k] = kc[k];
       if (B != 8) high_parts<B>(w, h);
       const uint32_t szw = *reinterpret_cast<const uint32_t*>(sl + 2 * P * rowb + (key * ng + grp) * 4);
-      float d[4] = {0.f, 0.f, 0.f, 0.f};
+      float2 d2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
 #pragma unroll
-      for (int i = 0; i < 32; ++i) d[i & 3] = fmaf(qp[i], code_at<B>(w, h, i), d[i & 3]);
+      for (int i = 0; i < 16; ++i)
+        d2[i & 1] = ffma2(make_float2(qp[2 * i], qp[2 * i + 1]),
+                          make_float2(code_at<B>(w, h, 2 * i), code_at<B>(w, h, 2 * i + 1)), d2[i & 1]);
       const float s = __half2float(__ushort_as_half(static_cast<unsigned short>(szw & 0xFFFF)));
       const float z = __half2float(__ushort_as_half(static_cast<unsigned short>(szw >> 16)));
-      dot = fmaf(s * pow2f(49), (d[0] + d[1]) + (d[2] + d[3]), z * sumq);
+      dot = fmaf(s * pow2f(49), (d2[0].x + d2[0].y) + (d2[1].x + d2[1].y), z * sumq);
     }
 #pragma unroll
     for (int o = 1; o < LPK; o <<= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
@@ -376,52 +404,36 @@ constexpr int kSlots = 8;  // pages a warp may have in flight (one mbarrier each
 
 struct AttnKernelArgs {
   LayerArgs a;
-  int n;
   const uint16_t* q;
   uint16_t* out;
   float qscale;      // softmax scale * log2(e)
   int ring_bytes;    // bytes of one warp's ring of shared memory
+  int max_desc;      // capacity of the descriptor array
 };
 
-// Per-slot record the producer writes for the consumer.
-struct SlotInfo {
-  int cls, fill, lo, hi;
-  int flags;   // 1 first page of its item, 2 last page, 4 no page (item without pages)
-  int item, qi, qh;
-  int nsplit, off, qoff, span;  // ring offsets of the page and the query row; bytes to release
-  int base, pad0, pad1, pad2;   // descriptor index of the query's split 0
+// Per-page record the producer writes for the consumer (two 16-byte words).
+struct SlotRec {
+  int meta;   // class | fill << 2 | mask << 9 | flags << 10 (1 first, 2 last, 4 no page)
+  int off;    // ring offset of the page's slice (then its positions when masked, then
+              // the query row on the first page of an item)
+  int span;   // ring bytes to release after the page
+  int lo;     // key range [lo, hi] of the item's query
+  int hi, item, qi, qh;
+  int nsplit, pad0, pad1, pad2;
 };
-
-// Producer-side description of the item being issued.
-struct ProdItem {
-  int item, qi, qh, kvh, nsplit, T, lo, hi, base, pad0, pad1, pad2;
-};
-static_assert(sizeof(SlotInfo) % 16 == 0 && sizeof(ProdItem) % 16 == 0, "16-byte multiples");
+static_assert(sizeof(SlotRec) == 48, "SlotRec is three 16-byte words");
 
 // Shared-memory carve-up of one attention CTA; every region starts 16-byte aligned
 // (mbarriers need 8, bulk-copy destinations 16).
 __host__ __device__ constexpr int align16(int x) { return (x + 15) & ~15; }
 struct AttnSmem {
-  int rings, infos, items, bars, total;
+  int rings, recs, bars, total;
   __host__ __device__ AttnSmem(int nwarps, int ring_bytes)
       : rings(0),
-        infos(align16(nwarps * ring_bytes)),
-        items(infos + align16(nwarps * kSlots * static_cast<int>(sizeof(SlotInfo)))),
-        bars(items + align16(nwarps * static_cast<int>(sizeof(ProdItem)))),
+        recs(align16(nwarps * ring_bytes)),
+        bars(recs + align16(nwarps * kSlots * static_cast<int>(sizeof(SlotRec)))),
         total(bars + align16(nwarps * kSlots * 8)) {}
 };
-
-// The last warp of the grid to finish resets the descriptor counter for the next call
-// (every warp has read it by then); no warp waits for another.
-__device__ __forceinline__ void finish_warp(int32_t* ctrl, int warps, int lane) {
-  if (lane == 0) {
-    __threadfence();
-    if (atomicAdd(ctrl + kDoneWarps, 1) == warps - 1) {
-      ctrl[kDescCounter] = 0;
-      ctrl[kDoneWarps] = 0;
-    }
-  }
-}
 
 template <int D>
 __global__ void __launch_bounds__(256, 2) attn_kernel(const AttnKernelArgs ka) {
@@ -432,10 +444,9 @@ __global__ void __launch_bounds__(256, 2) attn_kernel(const AttnKernelArgs ka) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
   const int qrow = D * 2;  // bytes of one query row
   const int R = ka.ring_bytes;
-  const AttnSmem lay(nwarps, R);  // [rings][slot infos][producer items][mbarriers]
+  const AttnSmem lay(nwarps, R);  // [rings][slot records][mbarriers]
   uint8_t* ring = smem + lay.rings + warp * R;
-  SlotInfo* sinfo = reinterpret_cast<SlotInfo*>(smem + lay.infos) + warp * kSlots;
-  ProdItem* pi = reinterpret_cast<ProdItem*>(smem + lay.items) + warp;
+  SlotRec* recs = reinterpret_cast<SlotRec*>(smem + lay.recs) + warp * kSlots;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + lay.bars) + warp * kSlots;
 
   if (lane == 0) {
@@ -445,6 +456,24 @@ __global__ void __launch_bounds__(256, 2) attn_kernel(const AttnKernelArgs ka) {
   }
   pdl_wait();
   pdl_trigger();
+  const int group = a.Hq / a.Hkv;
+  const int wstride = gridDim.x * nwarps;
+
+  // ------------------------------------------------------------ producer --
+  // Work items are (descriptor, query head) pairs dealt round-robin.  The descriptor of
+  // the producer's next item is prefetched one item ahead (three words per lane).
+  int next_item = blockIdx.x * nwarps + warp;
+  int nd0 = 0, nd1 = 0, nd2 = 0;       // prefetched descriptor: page ids, metas, header
+  auto prefetch = [&](int item) {
+    const int d = item / a.units;
+    if (d >= ka.max_desc) return;  // past any descriptor the plan can write
+    const int* dp = reinterpret_cast<const int*>(a.desc + d);
+    nd0 = dp[lane];
+    nd1 = dp[32 + lane];
+    nd2 = lane < 8 ? dp[64 + lane] : 0;
+  };
+  prefetch(next_item);  // in flight together with the descriptor count
+  const int total = *reinterpret_cast<volatile int*>(a.ctrl + kDescCounter) * a.units;
   if (blockIdx.x == 0 && threadIdx.x == 0) {  // status of the lowest invalid query
     const int bad = a.ctrl[kFirstBadQuery];
     if (bad != INT_MAX) {
@@ -452,54 +481,32 @@ __global__ void __launch_bounds__(256, 2) attn_kernel(const AttnKernelArgs ka) {
       a.ctrl[kFirstBadQuery] = INT_MAX;
     }
   }
-  // work items: (descriptor, query head) pairs, descriptors in the plan's order
-  const int total = *reinterpret_cast<volatile int*>(a.ctrl + kDescCounter) * a.units;
-  const int group = a.Hq / a.Hkv;
-  const int wstride = gridDim.x * nwarps;
 
-  // ------------------------------------------------------------ producer --
-  // Items are dealt round-robin.  The descriptor of the producer's next item is
-  // prefetched one item ahead (three words per lane), so starting an item costs no
-  // global round trip.
-  int next_item = blockIdx.x * nwarps + warp;
-  int nd0 = 0, nd1 = 0, nd2 = 0;       // prefetched descriptor: page ids, class|fill, header
-  int wid = -1, wmeta = 0;             // the producer's item: page id / class|fill of page `lane`
-  int pf = 0, pT = 0;                  // next page of the producer's item, its page count
+  int wid = -1, wmeta = 0;             // the producer's item: page id / meta of page `lane`
+  int p_item = 0, p_qi = 0, p_qh = 0, p_kvh = 0, p_nsplit = 0, p_T = 0, p_lo = 0, p_hi = 0;
+  int pf = 0;                          // next page of the producer's item
   bool pvalid = false;
   uint32_t issued = 0, consumed = 0;   // pages issued / consumed by this warp
   int head = 0, used = 0;              // ring: next free offset, bytes held
 
-  auto prefetch = [&](int item) {
-    if (item >= total) return;
-    const int* d = reinterpret_cast<const int*>(a.desc + item / a.units);
-    nd0 = d[lane];
-    nd1 = d[32 + lane];
-    nd2 = lane < 8 ? d[64 + lane] : 0;
-  };
   auto start_item = [&]() -> bool {
     if (next_item >= total) return false;
-    const int item = next_item;
+    p_item = next_item;
     wid = nd0;
     wmeta = nd1;
-    const int qi = __shfl_sync(0xffffffffu, nd2, 0);
-    const int lo = __shfl_sync(0xffffffffu, nd2, 2), hi = __shfl_sync(0xffffffffu, nd2, 3);
-    const int nsplit = __shfl_sync(0xffffffffu, nd2, 4);
-    pT = __shfl_sync(0xffffffffu, nd2, 6);
-    const int unit = item - (item / a.units) * a.units;
-    const int base = __shfl_sync(0xffffffffu, nd2, 7);
+    p_qi = __shfl_sync(0xffffffffu, nd2, 0);
+    p_lo = __shfl_sync(0xffffffffu, nd2, 2);
+    p_hi = __shfl_sync(0xffffffffu, nd2, 3);
+    p_nsplit = __shfl_sync(0xffffffffu, nd2, 4);
+    p_T = __shfl_sync(0xffffffffu, nd2, 6);
+    p_qh = p_item - (p_item / a.units) * a.units;
+    p_kvh = p_qh / group;
     next_item += wstride;
-    prefetch(next_item);
-    if (lane == 0) {
-      ProdItem t;
-      t.item = item; t.qi = qi; t.qh = unit; t.kvh = unit / group; t.nsplit = nsplit;
-      t.T = pT; t.lo = lo; t.hi = hi; t.base = base;
-      *pi = t;
-    }
-    __syncwarp();
+    if (next_item < total) prefetch(next_item);
     pf = 0;
     return true;
   };
-  // start the copy of the producer's next page if a slot and ring space are free
+  // start the copies of the producer's next page if a slot and ring space are free
   auto try_issue = [&]() -> bool {
     if (!pvalid) {
       pvalid = start_item();
@@ -507,13 +514,11 @@ __global__ void __launch_bounds__(256, 2) attn_kernel(const AttnKernelArgs ka) {
     }
     if (issued - consumed >= kSlots) return false;
     const bool first = pf == 0;
-    int c = 0, fill = 0, id = -1, bytes_page = 0;
-    if (pT > 0) {
+    int meta = 0, id = -1, bytes_page = 0;
+    if (p_T > 0) {
       id = __shfl_sync(0xffffffffu, wid, pf);
-      const int m = __shfl_sync(0xffffffffu, wmeta, pf);
-      c = m & 255;
-      fill = m >> 8;
-      bytes_page = a.slice[c] + 4 * a.P;
+      meta = __shfl_sync(0xffffffffu, wmeta, pf);
+      bytes_page = a.slice[meta & 3] + ((meta & 512) ? 4 * a.P : 0);
     }
     const int need = bytes_page + (first ? qrow : 0);
     if (used == 0) head = 0;  // an empty ring can start anywhere
@@ -526,43 +531,33 @@ __global__ void __launch_bounds__(256, 2) attn_kernel(const AttnKernelArgs ka) {
     head = off + need;
     used += waste + need;
     const uint32_t slot = issued % kSlots;
+    const int flags = (first ? 1 : 0) | (pf + 1 >= p_T ? 2 : 0) | (p_T == 0 ? 4 : 0);
+    // The record, then the arrival.  The ring is written only by bulk copies; the warp's
+    // earlier reads of these bytes have completed (their values were consumed), and the
+    // record reaches the consumer through the mbarrier's release / acquire, so no proxy
+    // fence is needed here.
     if (lane == 0) {
-      const ProdItem& it = *pi;
-      SlotInfo si;
-      si.cls = c;
-      si.fill = fill;
-      si.lo = it.lo;
-      si.hi = it.hi;
-      si.flags = (first ? 1 : 0) | (pf + 1 >= pT ? 2 : 0) | (pT == 0 ? 4 : 0);
-      si.item = it.item;
-      si.qi = it.qi;
-      si.qh = it.qh;
-      si.nsplit = it.nsplit;
-      si.off = off;
-      si.qoff = off + bytes_page;
-      si.span = waste + need;
-      si.base = it.base;
-      si.pad0 = si.pad1 = si.pad2 = 0;
-      sinfo[slot] = si;
-      fence_proxy_async_smem();
+      int4* rp = reinterpret_cast<int4*>(recs + slot);
+      rp[0] = make_int4(meta | (flags << 10), off, waste + need, p_lo);
+      rp[1] = make_int4(p_hi, p_item, p_qi, p_qh);
+      rp[2] = make_int4(p_nsplit, 0, 0, 0);
       mbar_arrive_expect_tx(&bars[slot], need);
-      if (pT > 0) {
+      const int c = meta & 3;
+      if (p_T > 0) {
         const uint8_t* page = a.pool[c] + static_cast<int64_t>(id) * a.page_bytes[c];
-        bulk_g2s(ring + off, page + a.hdr + static_cast<int64_t>(it.kvh) * a.slice[c], a.slice[c], &bars[slot]);
-        bulk_g2s(ring + off + a.slice[c], page, 4 * a.P, &bars[slot]);
+        bulk_g2s(ring + off, page + a.hdr + static_cast<int64_t>(p_kvh) * a.slice[c], a.slice[c], &bars[slot]);
+        if (meta & 512) bulk_g2s(ring + off + a.slice[c], page, 4 * a.P, &bars[slot]);
       }
       if (first)
-        bulk_g2s(ring + off + bytes_page, ka.q + (static_cast<int64_t>(it.qi) * a.Hq + it.qh) * D, qrow,
-                 &bars[slot]);
+        bulk_g2s(ring + off + bytes_page, ka.q + (static_cast<int64_t>(p_qi) * a.Hq + p_qh) * D, qrow, &bars[slot]);
     }
     __syncwarp();
     ++issued;
     ++pf;
-    if (pf >= pT) pvalid = false;
+    if (pf >= p_T) pvalid = false;
     return true;
   };
 
-  prefetch(next_item);
   while (try_issue()) {
   }
 
@@ -572,6 +567,7 @@ __global__ void __launch_bounds__(256, 2) attn_kernel(const AttnKernelArgs ka) {
   float qp[32];
   float sumq = 0.f;
   int cur_cls = 3;
+  int c_lo = 0, c_hi = 0;  // key range of the consumer's item
   st.m = kNegInf;
   st.l = 0.f;
   st.zacc = 0.f;
@@ -582,12 +578,15 @@ __global__ void __launch_bounds__(256, 2) attn_kernel(const AttnKernelArgs ka) {
     if (!__all_sync(0xffffffffu, arrived)) {  // give up together, never half a warp
       for (uint32_t r = g + 1; r < issued; ++r) mbar_wait(&bars[r % kSlots], (r / kSlots) & 1);
       if (lane == 0) set_status(a.ctrl, TRR_ERR_TIMEOUT);
-      finish_warp(a.ctrl, gridDim.x * nwarps, lane);
       return;
     }
-    const SlotInfo si = sinfo[slot];
-    if (si.flags & 1) {  // first page of an item: query row and a fresh state
-      const uint4* q4 = reinterpret_cast<const uint4*>(ring + si.qoff + part * 64);
+    const int4 r0 = *reinterpret_cast<const int4*>(recs + slot);
+    const int meta = r0.x, flags = meta >> 10;
+    if (flags & 1) {  // first page of an item: query row, key range and a fresh state
+      c_lo = r0.w;
+      c_hi = reinterpret_cast<const int*>(recs + slot)[4];
+      const int qoff = r0.y + ((flags & 4) ? 0 : a.slice[meta & 3] + ((meta & 512) ? 4 * a.P : 0));
+      const uint4* q4 = reinterpret_cast<const uint4*>(ring + qoff + part * 64);
       sumq = 0.f;
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
@@ -608,30 +607,34 @@ __global__ void __launch_bounds__(256, 2) attn_kernel(const AttnKernelArgs ka) {
 #pragma unroll
       for (int j = 0; j < 32; ++j) st.acc[j] = 0.f;
     }
-    if (!(si.flags & 4)) {
-      if (si.cls != cur_cls) {
-        rescale_q_dyn(qp, cur_cls, si.cls);
-        cur_cls = si.cls;
+    if (!(flags & 4)) {
+      const int cls = meta & 3, fill = (meta >> 2) & 127;
+      if (cls != cur_cls) {
+        rescale_q_dyn(qp, cur_cls, cls);
+        cur_cls = cls;
       }
-      const uint8_t* sl = ring + si.off;
-      const int* sp = reinterpret_cast<const int*>(ring + si.off + a.slice[si.cls]);
-      switch (si.cls) {
-        case 0: consume_page<D, 2>(sl, sp, a.P, a.G, si.fill, si.lo, si.hi, qp, sumq, st, lane); break;
-        case 1: consume_page<D, 4>(sl, sp, a.P, a.G, si.fill, si.lo, si.hi, qp, sumq, st, lane); break;
-        case 2: consume_page<D, 8>(sl, sp, a.P, a.G, si.fill, si.lo, si.hi, qp, sumq, st, lane); break;
-        default: consume_page<D, 16>(sl, sp, a.P, a.G, si.fill, si.lo, si.hi, qp, sumq, st, lane); break;
+      const uint8_t* sl = ring + r0.y;
+      const int* sp = (meta & 512) ? reinterpret_cast<const int*>(ring + r0.y + a.slice[cls]) : nullptr;
+      switch (cls) {
+        case 0: consume_page<D, 2>(sl, sp, a.P, a.G, fill, c_lo, c_hi, qp, sumq, st, lane); break;
+        case 1: consume_page<D, 4>(sl, sp, a.P, a.G, fill, c_lo, c_hi, qp, sumq, st, lane); break;
+        case 2: consume_page<D, 8>(sl, sp, a.P, a.G, fill, c_lo, c_hi, qp, sumq, st, lane); break;
+        default: consume_page<D, 16>(sl, sp, a.P, a.G, fill, c_lo, c_hi, qp, sumq, st, lane); break;
       }
     }
     __syncwarp();
-    used -= si.span;  // release the slot's ring bytes, refill
+    used -= r0.z;  // release the slot's ring bytes, refill
     consumed = g + 1;
     while (try_issue()) {
     }
-    if (!(si.flags & 2)) continue;
+    if (!(flags & 2)) continue;
 
     // ---- last page of the item: merge the lanes that share a part.  Rescale to the
     // common maximum, then reduce-scatter over the key lanes: each halving step keeps
     // half of the 32 dims and sends the other half to the partner lane.
+    const int4 r1 = *reinterpret_cast<const int4*>(reinterpret_cast<const int*>(recs + slot) + 4);
+    const int item = r1.y, qi = r1.z, qh = r1.w;
+    const int nsplit = reinterpret_cast<const int*>(recs + slot)[8];
     float M = st.m;
 #pragma unroll
     for (int o = LPK; o < 32; o <<= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
@@ -654,58 +657,62 @@ __global__ void __launch_bounds__(256, 2) attn_kernel(const AttnKernelArgs ka) {
       }
     }
     // lane (kl, part) now holds dims part*32 + DPL*kl .. + DPL-1 in acc[0 .. DPL-1]
-    const int64_t orow = (static_cast<int64_t>(si.qi) * a.Hq + si.qh) * D;
     const int dim0 = part * 32 + DPL * kl;
-    if (si.nsplit == 1) {
+    if (nsplit == 1) {
+      const int64_t orow = (static_cast<int64_t>(qi) * a.Hq + qh) * D;
       const float inv = L > 0.f ? 1.f / L : 0.f;
 #pragma unroll
       for (int j = 0; j < DPL; j += 2)
         *reinterpret_cast<__nv_bfloat162*>(ka.out + orow + dim0 + j) =
             __floats2bfloat162_rn(st.acc[j] * inv, st.acc[j + 1] * inv);
-      continue;
+    } else {  // a partial at the item's index; attn_combine_kernel merges the splits
+      float* pp = a.part + static_cast<int64_t>(item) * (D + 4);
+#pragma unroll
+      for (int j = 0; j < DPL; j += 2)
+        *reinterpret_cast<float2*>(pp + dim0 + j) = make_float2(st.acc[j], st.acc[j + 1]);
+      if (lane == 0) *reinterpret_cast<float2*>(pp + D) = make_float2(M, L);
     }
-    // several splits: store this one's partial (at the item's index), the last to
-    // arrive merges them all; split s of this query head is item (base + s)*units + unit
-    const int unit = si.qh;
-    const int split0 = si.base;
-    float* pp = a.part + static_cast<int64_t>(si.item) * (D + 4);
-#pragma unroll
-    for (int j = 0; j < DPL; j += 2) *reinterpret_cast<float2*>(pp + dim0 + j) = make_float2(st.acc[j], st.acc[j + 1]);
-    if (lane == 0) *reinterpret_cast<float2*>(pp + D) = make_float2(M, L);
-    __threadfence();
-    __syncwarp();
-    int last = 0;
-    int32_t* counter = a.cnt + static_cast<int64_t>(si.qi) * a.units + unit;
-    if (lane == 0) last = atomicAdd(counter, 1) == si.nsplit - 1;
-    last = __shfl_sync(0xffffffffu, last, 0);
-    if (!last) continue;
-    __threadfence();
-    float Mx = kNegInf;
-    for (int s = lane; s < si.nsplit; s += 32)
-      Mx = fmaxf(Mx, __ldcg(a.part + (static_cast<int64_t>(split0 + s) * a.units + unit) * (D + 4) + D));
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) Mx = fmaxf(Mx, __shfl_xor_sync(0xffffffffu, Mx, o));
-    float Ls = 0.f, o[DPL];
-#pragma unroll
-    for (int j = 0; j < DPL; ++j) o[j] = 0.f;
-#pragma unroll 4
-    for (int s = 0; s < si.nsplit; ++s) {
-      const float* ps = a.part + (static_cast<int64_t>(split0 + s) * a.units + unit) * (D + 4);
-      const float2 ml = __ldcg(reinterpret_cast<const float2*>(ps + D));
-      const float wgt = (ml.x == kNegInf) ? 0.f : exp2f(ml.x - Mx);
-      Ls = fmaf(wgt, ml.y, Ls);
-#pragma unroll
-      for (int j = 0; j < DPL; ++j) o[j] = fmaf(wgt, __ldcg(ps + lane * DPL + j), o[j]);
-    }
-    const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
-#pragma unroll
-    for (int j = 0; j < DPL; j += 2) {
-      const __nv_bfloat162 b2 = __floats2bfloat162_rn(o[j] * inv, o[j + 1] * inv);
-      *reinterpret_cast<__nv_bfloat162*>(ka.out + orow + lane * DPL + j) = b2;
-    }
-    if (lane == 0) *counter = 0;
   }
-  finish_warp(a.ctrl, gridDim.x * nwarps, lane);
+}
+
+// One warp per (query, query head) with several splits: merge the fp32 partials of
+// splits 0..nsplit-1 (items (base + s) * units + head) into the bf16 row.  Block 0 also
+// resets the descriptor counter for the next call.
+template <int D>
+__global__ void __launch_bounds__(256) attn_combine_kernel(LayerArgs a, int n, uint16_t* __restrict__ out) {
+  constexpr int DPL = D / 32;
+  pdl_wait();
+  pdl_trigger();
+  if (blockIdx.x == 0 && threadIdx.x == 0) a.ctrl[kDescCounter] = 0;
+  const int lane = threadIdx.x & 31;
+  const int w = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (w >= n * a.units) return;
+  const int qi = w / a.units, qh = w - qi * a.units;
+  const int nsplit = a.qplan[qi].nsplit, base = a.qplan[qi].base;
+  if (nsplit <= 1) return;
+  float Mx = kNegInf;
+  for (int s = lane; s < nsplit; s += 32)
+    Mx = fmaxf(Mx, a.part[(static_cast<int64_t>(base + s) * a.units + qh) * (D + 4) + D]);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) Mx = fmaxf(Mx, __shfl_xor_sync(0xffffffffu, Mx, o));
+  float Ls = 0.f, o[DPL];
+#pragma unroll
+  for (int j = 0; j < DPL; ++j) o[j] = 0.f;
+#pragma unroll 4
+  for (int s = 0; s < nsplit; ++s) {
+    const float* ps = a.part + (static_cast<int64_t>(base + s) * a.units + qh) * (D + 4);
+    const float2 ml = *reinterpret_cast<const float2*>(ps + D);
+    const float wgt = (ml.x == kNegInf) ? 0.f : exp2f(ml.x - Mx);
+    Ls = fmaf(wgt, ml.y, Ls);
+#pragma unroll
+    for (int j = 0; j < DPL; ++j) o[j] = fmaf(wgt, ps[lane * DPL + j], o[j]);
+  }
+  const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
+  const int64_t orow = (static_cast<int64_t>(qi) * a.Hq + qh) * D;
+#pragma unroll
+  for (int j = 0; j < DPL; j += 2)
+    *reinterpret_cast<__nv_bfloat162*>(out + orow + lane * DPL + j) =
+        __floats2bfloat162_rn(o[j] * inv, o[j + 1] * inv);
 }
 
 constexpr int kAttnSmemLimit = 110 * 1024;  // dynamic shared memory of one attention CTA
@@ -715,6 +722,42 @@ cudaError_t attn_configure() {
   cudaError_t e = cudaFuncSetAttribute(attn_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, kAttnSmemLimit);
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(attn_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, kAttnSmemLimit);
+  return e;
+}
+
+// The three launches of one attention call (plan, attention, combine) with the given
+// scratch views in `a`.
+static cudaError_t launch_attention(const Layout& l, const LayerArgs& a, int num_sms, int n,
+                                    const int32_t* seq_ids, const int32_t* q_positions, const void* q_bf16,
+                                    const uint8_t* modes, const int32_t* windows, int window_scalar,
+                                    float softmax_scale, void* out_bf16, int64_t max_desc, cudaStream_t s) {
+  cudaError_t e = launch_pdl(attn_plan_kernel, dim3((n + 7) / 8), dim3(256), 0, s, a, n, seq_ids, q_positions,
+                             modes, windows, window_scalar, static_cast<uint16_t*>(out_bf16));
+  if (e != cudaSuccess) return e;
+  AttnKernelArgs ka;
+  ka.a = a;
+  ka.q = static_cast<const uint16_t*>(q_bf16);
+  ka.out = static_cast<uint16_t*>(out_bf16);
+  const float scale = softmax_scale > 0.f ? softmax_scale : 1.f / sqrtf(static_cast<float>(l.d));
+  ka.qscale = scale * 1.4426950408889634f;
+  // a ring holds at least one page of the widest class with its positions and a query row
+  const int widest = static_cast<int>(l.slice[3]) + 4 * l.P + 2 * l.d;
+  ka.ring_bytes = std::max(12 * 1024, (widest + 127) / 128 * 128);
+  ka.max_desc = static_cast<int>(std::min<int64_t>(max_desc, INT_MAX));
+  int nwarps = 8;
+  while (nwarps > 0 && AttnSmem(nwarps, ka.ring_bytes).total > kAttnSmemLimit) --nwarps;
+  if (nwarps < 1) return cudaErrorInvalidConfiguration;
+  const int smem = AttnSmem(nwarps, ka.ring_bytes).total;
+  if (l.d == 64)
+    e = launch_pdl(attn_kernel<64>, dim3(2 * num_sms), dim3(nwarps * 32), static_cast<size_t>(smem), s, ka);
+  else
+    e = launch_pdl(attn_kernel<128>, dim3(2 * num_sms), dim3(nwarps * 32), static_cast<size_t>(smem), s, ka);
+  if (e != cudaSuccess) return e;
+  const int cw = n * l.units;
+  if (l.d == 64)
+    e = launch_pdl(attn_combine_kernel<64>, dim3((cw + 7) / 8), dim3(256), 0, s, a, n, static_cast<uint16_t*>(out_bf16));
+  else
+    e = launch_pdl(attn_combine_kernel<128>, dim3((cw + 7) / 8), dim3(256), 0, s, a, n, static_cast<uint16_t*>(out_bf16));
   return e;
 }
 
@@ -734,31 +777,12 @@ extern "C" trr_status trr_decode_attn(trr_cache* cache, int32_t layer, int32_t n
   if (!seq_ids || !q_positions || !q_bf16 || !modes || !out_bf16) return TRR_ERR_INVALID_ARG;
   if ((reinterpret_cast<uintptr_t>(q_bf16) | reinterpret_cast<uintptr_t>(out_bf16)) & 15)
     return TRR_ERR_INVALID_ARG;
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
   const LayerArgs a = layer_args(l, cache_views(cache), layer);
-  cudaError_t e = launch_pdl(attn_plan_kernel, dim3((n + 7) / 8), dim3(256), 0, s, a, n, seq_ids, q_positions,
-                             modes, windows, window_scalar, static_cast<uint16_t*>(out_bf16));
-  if (e != cudaSuccess) return TRR_ERR_CUDA;
-  AttnKernelArgs ka;
-  ka.a = a;
-  ka.n = n;
-  ka.q = static_cast<const uint16_t*>(q_bf16);
-  ka.out = static_cast<uint16_t*>(out_bf16);
-  const float scale = softmax_scale > 0.f ? softmax_scale : 1.f / sqrtf(static_cast<float>(l.d));
-  ka.qscale = scale * 1.4426950408889634f;
-  // a ring holds at least one page of the widest class with its positions and a query row
-  const int widest = static_cast<int>(l.slice[3]) + 4 * l.P + 2 * l.d;
-  ka.ring_bytes = std::max(12 * 1024, (widest + 127) / 128 * 128);
-  int nwarps = 8;
-  while (nwarps > 0 && AttnSmem(nwarps, ka.ring_bytes).total > kAttnSmemLimit) --nwarps;
-  if (nwarps < 1) return TRR_ERR_UNSUPPORTED;
-  const int smem = AttnSmem(nwarps, ka.ring_bytes).total;
-  const int grid = 2 * cache_num_sms(cache);
-  if (l.d == 64)
-    e = launch_pdl(attn_kernel<64>, dim3(grid), dim3(nwarps * 32), static_cast<size_t>(smem), s, ka);
-  else
-    e = launch_pdl(attn_kernel<128>, dim3(grid), dim3(nwarps * 32), static_cast<size_t>(smem), s, ka);
-  cache_set_launches(cache, 2);
+  const cudaError_t e = launch_attention(l, a, cache_num_sms(cache), n, seq_ids, q_positions, q_bf16, modes,
+                                         windows, window_scalar, softmax_scale, out_bf16,
+                                         static_cast<int64_t>(l.max_queries) * l.s_cap,
+                                         static_cast<cudaStream_t>(stream));
+  cache_set_launches(cache, 3);
   return e == cudaSuccess ? TRR_OK : TRR_ERR_CUDA;
 }
 
@@ -843,29 +867,10 @@ extern "C" trr_status trr_decode_attn_static(trr_cache* cache, int32_t layer, in
   static_scratch_clear_kernel<<<std::max(1, std::min(256, (ncnt + 255) / 256)), 256, 0, s>>>(a.ctrl, a.cnt, ncnt);
   cudaError_t e = cudaGetLastError();
   if (e == cudaSuccess)
-    e = launch_pdl(attn_plan_kernel, dim3((n + 7) / 8), dim3(256), 0, s, a, n, seq_ids, q_positions, modes,
-                   windows, window_scalar, static_cast<uint16_t*>(out_bf16));
-  if (e != cudaSuccess) return TRR_ERR_CUDA;
-  AttnKernelArgs ka;
-  ka.a = a;
-  ka.n = n;
-  ka.q = static_cast<const uint16_t*>(q_bf16);
-  ka.out = static_cast<uint16_t*>(out_bf16);
-  const float scale = softmax_scale > 0.f ? softmax_scale : 1.f / sqrtf(static_cast<float>(l.d));
-  ka.qscale = scale * 1.4426950408889634f;
-  const int widest = static_cast<int>(l.slice[3]) + 4 * l.P + 2 * l.d;
-  ka.ring_bytes = std::max(12 * 1024, (widest + 127) / 128 * 128);
-  int nwarps = 8;
-  while (nwarps > 0 && AttnSmem(nwarps, ka.ring_bytes).total > kAttnSmemLimit) --nwarps;
-  if (nwarps < 1) return TRR_ERR_UNSUPPORTED;
-  const int smem = AttnSmem(nwarps, ka.ring_bytes).total;
-  const int grid = 2 * cache_num_sms(cache);
-  if (l.d == 64)
-    e = launch_pdl(attn_kernel<64>, dim3(grid), dim3(nwarps * 32), static_cast<size_t>(smem), s, ka);
-  else
-    e = launch_pdl(attn_kernel<128>, dim3(grid), dim3(nwarps * 32), static_cast<size_t>(smem), s, ka);
+    e = launch_attention(l, a, cache_num_sms(cache), n, seq_ids, q_positions, q_bf16, modes, windows,
+                         window_scalar, softmax_scale, out_bf16, nd, s);
   if (e != cudaSuccess) return TRR_ERR_CUDA;
   static_scratch_status_kernel<<<1, 1, 0, s>>>(a.ctrl, cache_ctrl);
-  cache_set_launches(cache, 4);
+  cache_set_launches(cache, 5);
   return cudaGetLastError() == cudaSuccess ? TRR_OK : TRR_ERR_CUDA;
 }

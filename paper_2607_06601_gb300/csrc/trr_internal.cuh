@@ -45,7 +45,7 @@ struct QueryPlan {
   int first[kClasses];          // first page (index in the class page list) in range
   int npages[kClasses];         // pages in range
   int ntok[kClasses];           // tokens of the class stored for the sequence
-  int err, pad0, pad1, pad2;
+  int err, base, pad1, pad2;    // base: descriptor index of split 0
 };
 static_assert(sizeof(QueryPlan) == 80, "QueryPlan is 80 bytes");
 
@@ -57,7 +57,7 @@ constexpr int kDescPages = 32;
 constexpr int kDescMaxPages = 28;  // splits are sized to hold at most this many pages, + 4
 struct SplitDesc {
   int page[kDescPages];
-  int meta[kDescPages];  // class | fill << 8
+  int meta[kDescPages];  // class | fill << 2 | (slot positions needed) << 9
   int qi, seq, lo, hi, nsplit, split, T, base;  // base: descriptor index of split 0
 };
 static_assert(sizeof(SplitDesc) == 288, "SplitDesc is 288 bytes");
