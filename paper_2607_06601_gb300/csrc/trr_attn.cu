@@ -258,6 +258,23 @@ __device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) {
   return d;
 }
 
+// The B words of 32 B-bit codes at a 4B-byte aligned address, in as few shared loads
+// as possible (one 8- or 16-byte load per row part keeps the warp's request
+// conflict-free).
+template <int B>
+__device__ __forceinline__ void load_codes(const uint8_t* p, uint32_t* w) {
+  if (B == 2) {
+    const uint2 u = *reinterpret_cast<const uint2*>(p);
+    w[0] = u.x; w[1] = u.y;
+  } else {
+#pragma unroll
+    for (int k = 0; k < B; k += 4) {
+      const uint4 u = *reinterpret_cast<const uint4*>(p + 4 * k);
+      w[k] = u.x; w[k + 1] = u.y; w[k + 2] = u.z; w[k + 3] = u.w;
+    }
+  }
+}
+
 template <int B>
 __device__ __forceinline__ void high_parts(const uint32_t* w, uint32_t* h) {
   constexpr int sh = B == 2 ? 22 : B == 4 ? 20 : 16;
@@ -271,20 +288,45 @@ __device__ __forceinline__ void rescale_q(float (&qp)[32]) {
   for (int i = 0; i < 32; ++i) qp[i] *= pow2f(qe_of(BTO, i) - qe_of(BFROM, i));
 }
 
+// V is accumulated as acc_i * 2^(ex_i(B) - 49) while class B's pages are consumed
+// (B = 16: ex = 0), so that every element of a key takes the same weight p*s*2^100.
+template <int BFROM, int BTO>
+__device__ __forceinline__ void rescale_acc(float (&acc)[32]) {
+#pragma unroll
+  for (int i = 0; i < 32; ++i) acc[i] *= pow2f((BTO == 16 ? 0 : ex_of(BTO, i)) - (BFROM == 16 ? 0 : ex_of(BFROM, i)));
+}
+
 // qp from the domain of class `from` to that of class `to` (from < to, or from = 16).
-__device__ __forceinline__ void rescale_q_dyn(float (&qp)[32], int from, int to) {
+__device__ __forceinline__ void rescale_dyn(float (&qp)[32], float (&acc)[32], int from, int to) {
   switch (from * 4 + to) {
-    case 1: rescale_q<2, 4>(qp); break;
-    case 2: rescale_q<2, 8>(qp); break;
-    case 3: rescale_q<2, 16>(qp); break;
-    case 6: rescale_q<4, 8>(qp); break;
-    case 7: rescale_q<4, 16>(qp); break;
-    case 11: rescale_q<8, 16>(qp); break;
-    case 12: rescale_q<16, 2>(qp); break;
-    case 13: rescale_q<16, 4>(qp); break;
-    case 14: rescale_q<16, 8>(qp); break;
+    case 1: rescale_q<2, 4>(qp); rescale_acc<2, 4>(acc); break;
+    case 2: rescale_q<2, 8>(qp); rescale_acc<2, 8>(acc); break;
+    case 3: rescale_q<2, 16>(qp); rescale_acc<2, 16>(acc); break;
+    case 6: rescale_q<4, 8>(qp); rescale_acc<4, 8>(acc); break;
+    case 7: rescale_q<4, 16>(qp); rescale_acc<4, 16>(acc); break;
+    case 11: rescale_q<8, 16>(qp); rescale_acc<8, 16>(acc); break;
+    case 12: rescale_q<16, 2>(qp); rescale_acc<16, 2>(acc); break;
+    case 13: rescale_q<16, 4>(qp); rescale_acc<16, 4>(acc); break;
+    case 14: rescale_q<16, 8>(qp); rescale_acc<16, 8>(acc); break;
     default: break;
   }
+}
+// acc from class `from`'s domain back to class 16's (the common one of the merge)
+__device__ __forceinline__ void acc_to_neutral(float (&acc)[32], int from) {
+  switch (from) {
+    case 0: rescale_acc<2, 16>(acc); break;
+    case 1: rescale_acc<4, 16>(acc); break;
+    case 2: rescale_acc<8, 16>(acc); break;
+    default: break;
+  }
+}
+
+// 2^x with the hardware approximation (relative error about 2^-22; results below the
+// binary32 normal range flush to zero, far below a softmax sum's resolution).
+__device__ __forceinline__ float fast_exp2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
 }
 
 struct LaneState {
@@ -294,14 +336,14 @@ struct LaneState {
 
 __device__ __forceinline__ float softmax_step(LaneState& st, float score) {
   if (score > st.m + kTau) {
-    const float alpha = exp2f(st.m - score);  // 0 when m = -inf
+    const float alpha = fast_exp2(st.m - score);  // 0 when m = -inf
 #pragma unroll
     for (int j = 0; j < 32; ++j) st.acc[j] *= alpha;
     st.l *= alpha;
     st.zacc *= alpha;
     st.m = score;
   }
-  const float p = exp2f(score - st.m);
+  const float p = fast_exp2(score - st.m);
   st.l += p;
   return p;
 }
@@ -344,9 +386,7 @@ __device__ __forceinline__ void consume_page(const uint8_t* sl, const int* spos,
     } else {
       constexpr int rowb = D * B / 8;
       uint32_t w[B], h[B];
-      const uint32_t* kc = reinterpret_cast<const uint32_t*>(sl + key * rowb + part * 4 * B);
-#pragma unroll
-      for (int k = 0; k < B; ++k) w[k] = kc[k];
+      load_codes<B>(sl + key * rowb + part * 4 * B, w);
       if (B != 8) high_parts<B>(w, h);
       const uint32_t szw = *reinterpret_cast<const uint32_t*>(sl + 2 * P * rowb + (key * ng + grp) * 4);
       float2 d2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
@@ -354,9 +394,8 @@ __device__ __forceinline__ void consume_page(const uint8_t* sl, const int* spos,
       for (int i = 0; i < 16; ++i)
         d2[i & 1] = ffma2(make_float2(qp[2 * i], qp[2 * i + 1]),
                           make_float2(code_at<B>(w, h, 2 * i), code_at<B>(w, h, 2 * i + 1)), d2[i & 1]);
-      const float s = __half2float(__ushort_as_half(static_cast<unsigned short>(szw & 0xFFFF)));
-      const float z = __half2float(__ushort_as_half(static_cast<unsigned short>(szw >> 16)));
-      dot = fmaf(s * pow2f(49), (d2[0].x + d2[0].y) + (d2[1].x + d2[1].y), z * sumq);
+      const float2 sz = __half22float2(*reinterpret_cast<const __half2*>(&szw));  // (s, z)
+      dot = fmaf(sz.x * pow2f(49), (d2[0].x + d2[0].y) + (d2[1].x + d2[1].y), sz.y * sumq);
     }
 #pragma unroll
     for (int o = 1; o < LPK; o <<= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
@@ -365,34 +404,37 @@ __device__ __forceinline__ void consume_page(const uint8_t* sl, const int* spos,
       if (B == 16) {
         const uint4* vp = reinterpret_cast<const uint4*>(sl + (P * D + key * D + part * 32) * 2);
         const float wv = p * pow2f(-49);
+        const float2 w2 = make_float2(wv, wv);
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
           const uint4 u = vp[q];
-          st.acc[8 * q + 0] = fmaf(wv, bf_lo(u.x), st.acc[8 * q + 0]);
-          st.acc[8 * q + 1] = fmaf(wv, bf_hi(u.x), st.acc[8 * q + 1]);
-          st.acc[8 * q + 2] = fmaf(wv, bf_lo(u.y), st.acc[8 * q + 2]);
-          st.acc[8 * q + 3] = fmaf(wv, bf_hi(u.y), st.acc[8 * q + 3]);
-          st.acc[8 * q + 4] = fmaf(wv, bf_lo(u.z), st.acc[8 * q + 4]);
-          st.acc[8 * q + 5] = fmaf(wv, bf_hi(u.z), st.acc[8 * q + 5]);
-          st.acc[8 * q + 6] = fmaf(wv, bf_lo(u.w), st.acc[8 * q + 6]);
-          st.acc[8 * q + 7] = fmaf(wv, bf_hi(u.w), st.acc[8 * q + 7]);
+          const uint32_t uw[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+          for (int h = 0; h < 4; ++h) {
+            const int i = 8 * q + 2 * h;
+            const float2 r = ffma2(w2, make_float2(bf_lo(uw[h]), bf_hi(uw[h])), make_float2(st.acc[i], st.acc[i + 1]));
+            st.acc[i] = r.x;
+            st.acc[i + 1] = r.y;
+          }
         }
       } else {
         constexpr int rowb = D * B / 8;
         uint32_t w[B], h[B];
-        const uint32_t* vc = reinterpret_cast<const uint32_t*>(sl + P * rowb + key * rowb + part * 4 * B);
-#pragma unroll
-        for (int k = 0; k < B; ++k) w[k] = vc[k];
+        load_codes<B>(sl + P * rowb + key * rowb + part * 4 * B, w);
         if (B != 8) high_parts<B>(w, h);
         const uint32_t szw =
             *reinterpret_cast<const uint32_t*>(sl + 2 * P * rowb + P * ng * 4 + (key * ng + grp) * 4);
-        const float s = __half2float(__ushort_as_half(static_cast<unsigned short>(szw & 0xFFFF)));
-        const float z = __half2float(__ushort_as_half(static_cast<unsigned short>(szw >> 16)));
-        const float wb = p * s * pow2f(100);
+        const float2 sz = __half22float2(*reinterpret_cast<const __half2*>(&szw));  // (s, z)
+        const float wb = p * sz.x * pow2f(100);
+        const float2 w2 = make_float2(wb, wb);
 #pragma unroll
-        for (int i = 0; i < 32; ++i)
-          st.acc[i] = fmaf(wb * pow2f(-ex_of(B, i)), code_at<B>(w, h, i), st.acc[i]);
-        st.zacc = fmaf(p, z, st.zacc);
+        for (int i = 0; i < 32; i += 2) {
+          const float2 r = ffma2(w2, make_float2(code_at<B>(w, h, i), code_at<B>(w, h, i + 1)),
+                                 make_float2(st.acc[i], st.acc[i + 1]));
+          st.acc[i] = r.x;
+          st.acc[i + 1] = r.y;
+        }
+        st.zacc = fmaf(p, sz.y, st.zacc);
       }
     }
   }
@@ -610,7 +652,7 @@ __global__ void __launch_bounds__(256, 2) attn_kernel(const AttnKernelArgs ka) {
     if (!(flags & 4)) {
       const int cls = meta & 3, fill = (meta >> 2) & 127;
       if (cls != cur_cls) {
-        rescale_q_dyn(qp, cur_cls, cls);
+        rescale_dyn(qp, st.acc, cur_cls, cls);
         cur_cls = cls;
       }
       const uint8_t* sl = ring + r0.y;
@@ -635,10 +677,11 @@ __global__ void __launch_bounds__(256, 2) attn_kernel(const AttnKernelArgs ka) {
     const int4 r1 = *reinterpret_cast<const int4*>(reinterpret_cast<const int*>(recs + slot) + 4);
     const int item = r1.y, qi = r1.z, qh = r1.w;
     const int nsplit = reinterpret_cast<const int*>(recs + slot)[8];
+    acc_to_neutral(st.acc, cur_cls);
     float M = st.m;
 #pragma unroll
     for (int o = LPK; o < 32; o <<= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-    const float f = (st.m == kNegInf) ? 0.f : exp2f(st.m - M);
+    const float f = (st.m == kNegInf) ? 0.f : fast_exp2(st.m - M);
     float L = st.l * f;
 #pragma unroll
     for (int o = LPK; o < 32; o <<= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
