@@ -121,8 +121,9 @@ TRR_API trr_status trr_create_cache(const trr_cache_config* cfg, trr_cache** out
  *   A skip token (modes[i] == 0) stores nothing unless skip_writes_kv == 1.
  *   For b < 16 each group of G consecutive elements of a head vector is stored as
  *     z = fp16(min x),  s = fp16(fl32(fl32(max x - min x) / (2^b - 1))),
- *     c_j = clamp(rne(fl32(fl32(x_j - z) / s)), 0, 2^b - 1)   (c_j = 0 when s == 0)
- *   with fl32 = IEEE binary32 round-to-nearest-even; b = 16 stores the bf16 bits.
+ *     c_j = clamp(rne((x_j - z) / s), 0, 2^b - 1)   (c_j = 0 when s == 0)
+ *   with fl32 = IEEE binary32 round-to-nearest-even and rne taken on the EXACT quotient
+ *   (c_j is the nearest level z + c*s, ties to the even c); b = 16 stores the bf16 bits.
  *   seq_ids, positions, k, v, bits, modes: device arrays; 0 <= n <= max_append.
  *   Device-detected errors: seq id out of range or bits/mode not allowed
  *   (INVALID_ARG), a position outside [0, max_context) or not above the sequence's

@@ -10,8 +10,9 @@
  *     codes round((x - z) / s), stored code c dequantises to z + c*s; b = 16 keeps
  *     the native value.  Readings where the paper is silent: min/max are taken per
  *     group of G elements along the head dimension; s and z are stored as IEEE
- *     binary16; s, the difference x - z and the quotient are each rounded to IEEE
- *     binary32 (fl32) before round-half-to-even and a clamp to [0, 2^b - 1];
+ *     binary16, s computed as fp16(fl32(fl32(max - min) / (2^b - 1))); the code is
+ *     round-half-to-even of the EXACT quotient (x - z) / s, clamped to [0, 2^b - 1],
+ *     i.e. the index of the nearest of the levels z + c*s, ties to the even index;
  *     native precision is bf16.
  *   - attention modes (Sec. 3.2(A), Eq. 2): skip -> 0; local -> softmax attention over
  *     the last w positions t-w+1..t (w keys, the reading the cost model
@@ -126,13 +127,20 @@ int orc_quantize_group(const uint16_t* x, int G, int b, uint16_t* s16, uint16_t*
   uint16_t sb = orc_double_to_f16(fl32(range / (double)levels)); /* s */
   double z = orc_f16_to_double(zb), s = orc_f16_to_double(sb);
   for (i = 0; i < G; i++) {
+    /* round((x - z) / s) on the exact quotient, clamped to the levels: walk up the
+     * levels z + c*s while x lies above the midpoint between level c and level c+1
+     * (or on it with c odd, so that a tie ends on the even level).  The midpoint
+     * z + (c + 1/2) s is exact in double: z and s are binary16, so it is a multiple
+     * of 2^-25 below 2^18.  x is a bf16 value, exact in double, so every comparison is
+     * exact.  With s = 0 every level is z and the code is 0. */
+    double xi = orc_bf16_to_double(x[i]);
     int c = 0;
     if (s != 0) {
-      double u = fl32(fl32(orc_bf16_to_double(x[i]) - z) / s); /* (x - z) / s */
-      double r = nearbyint(u);                                  /* round, ties even */
-      if (r < 0) r = 0;
-      if (r > levels) r = levels;
-      c = (int)r;
+      while (c < levels) {
+        double mid = z + ((double)c + 0.5) * s;
+        if (xi > mid || (xi == mid && (c & 1))) c++;
+        else break;
+      }
     }
     codes[i] = (uint8_t)c;
   }

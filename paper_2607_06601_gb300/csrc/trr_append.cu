@@ -129,6 +129,24 @@ __global__ void __launch_bounds__(1024) append_plan_kernel(LayerArgs a, int n, c
 __device__ __forceinline__ float bf16lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 
+// round((x - z) / s) of Eq. 4 on the exact quotient, ties to even, clamped to [0, levels].
+// u = fl32(fl32(x - z) / s) is within 2^-22 |u| of the exact quotient (two binary32
+// roundings), so rint(u) is exact unless u lies that close to a half-way point c + 1/2.
+// There the midpoint z + (c + 1/2) s is formed in binary64, where it is exact (z and s
+// are binary16: a multiple of 2^-25 below 2^18), and compared with x (a bf16 value).
+// Only half-way points inside [0, levels] matter: the clamp settles the others.
+__device__ __forceinline__ int code_of(float x, float z, float s, int levels) {
+  const float u = __fdiv_rn(__fsub_rn(x, z), s);
+  const float fl = floorf(u);
+  if (fabsf(__fsub_rn(u, fl + 0.5f)) <= fabsf(u) * 0x1p-21f && fl >= 0.f && fl < static_cast<float>(levels)) {
+    const double mid = __dadd_rn(static_cast<double>(z), __dmul_rn(static_cast<double>(fl) + 0.5, static_cast<double>(s)));
+    const double xd = static_cast<double>(x);
+    const int c = static_cast<int>(fl);
+    return (xd > mid || (xd == mid && (c & 1))) ? c + 1 : c;
+  }
+  return min(max(__float2int_rn(u), 0), levels);
+}
+
 // Eq. 4 on 32 consecutive values (one chunk of a group): codes packed LSB-first.
 template <int B>
 __device__ __forceinline__ void quantise_chunk(const uint4* src, float z, float s, uint32_t* dst) {
@@ -144,11 +162,7 @@ __device__ __forceinline__ void quantise_chunk(const uint4* src, float z, float 
 #pragma unroll
     for (int h = 0; h < 8; ++h) {
       const float x = (h & 1) ? bf16hi(wv[h >> 1]) : bf16lo(wv[h >> 1]);
-      int code = 0;
-      if (s != 0.f) {
-        const float u32 = __fdiv_rn(__fsub_rn(x, z), s);
-        code = min(max(__float2int_rn(u32), 0), levels);
-      }
+      const int code = s != 0.f ? code_of(x, z, s, levels) : 0;
       const int j = q * 8 + h;
       words[j / per_word] |= static_cast<uint32_t>(code) << ((j % per_word) * B);
     }

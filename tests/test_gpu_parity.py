@@ -187,6 +187,39 @@ def test_edge_cases_and_error_contract():
     pair.check_regions()
 
 
+def test_append_rounds_the_exact_quotient_near_half_way_points():
+    """Groups built so that (x - z) / s lies on, or within 2^-60 of, a half-way point c + 1/2
+    (z = -(c + 1/2), s = 1, x = 0 or +-tiny), mixed with groups of small integers and
+    quarter-integers that put exact ties everywhere: the codes must follow the exact
+    quotient, bit for bit with the oracle."""
+    rng = np.random.default_rng(21)
+    d, G, Hkv = 64, 32, 2
+    tiny = 2.0 ** -60
+    rows, bits = [], []
+    for b, cs in ((2, range(3)), (4, range(15)), (8, [127])):
+        levels = (1 << b) - 1
+        for c in cs:
+            tok = np.empty((Hkv, d), dtype=np.float32)
+            for h in range(Hkv):
+                for g in range(d // G):
+                    grp = rng.choice([tiny, -tiny, 0.0, -0.0, 2.0 ** -100, -(2.0 ** -126)], size=G)
+                    at = rng.choice(G, size=2, replace=False)
+                    grp[at[0]], grp[at[1]] = -(c + 0.5), levels - c - 0.5
+                    tok[h, g * G:(g + 1) * G] = grp
+            rows.append(tok)
+            bits.append(b)
+    for _ in range(24):
+        b = int(rng.choice([2, 4, 8]))
+        rows.append((rng.integers(-40, 40, size=(Hkv, d)) / rng.choice([1, 2, 4])).astype(np.float32))
+        bits.append(b)
+    n = len(rows)
+    K = wl.bf16_bits(np.stack(rows))
+    V = wl.bf16_bits(-np.stack(rows[::-1]))
+    pair = Pair(1, 1, 2, Hkv, d, G, 16, 128, [8, 8, 8, 8], max_append=128)
+    pair.append(0, [0] * n, list(range(n)), K, V, bits, [FULL] * n)
+    pair.check_regions()
+
+
 def test_skip_writes_kv_variant():
     rng = np.random.default_rng(8)
     pair, ent, bits, modes = _random_setup(rng, 64, 32, 16, 2, 2, [50, 200], skip_writes_kv=1)

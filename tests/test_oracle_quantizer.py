@@ -2,6 +2,8 @@
 facts that do not come from the oracle itself: numpy's IEEE conversions, the exact
 nearest-level definition enumerated over all 2^b levels, the closed-form error bound,
 hand-packed bytes, and special cases with known answers."""
+from fractions import Fraction
+
 import numpy as np
 import pytest
 
@@ -53,6 +55,17 @@ def test_pack_hand_examples():
     assert oracle.pack_codes([7, 200, 255, 0], 8) == bytes([7, 200, 255, 0])
 
 
+def _exact_nearest_ok(x, z, s, c, levels):
+    xf, zf, sf = Fraction(x), Fraction(z), Fraction(s)
+    d = abs(xf - (zf + c * sf))
+    for nb in (c - 1, c + 1):
+        if 0 <= nb <= levels:
+            dn = abs(xf - (zf + nb * sf))
+            if dn < d or (dn == d and c % 2 == 1):
+                return False
+    return True
+
+
 def _groups(rng, G, count):
     out = [rng.standard_normal(G).astype(np.float32) for _ in range(count)]
     out += [(rng.standard_normal(G) * 8).astype(np.float32) for _ in range(count // 4)]
@@ -65,9 +78,9 @@ def _groups(rng, G, count):
 @pytest.mark.parametrize("b", [2, 4, 8])
 @pytest.mark.parametrize("G", [32, 64, 128])
 def test_quantizer_nearest_level_and_bound(b, G):
-    """codes are a nearest level z + c*s (all 2^b levels enumerated), except that a
-    quotient within binary32 rounding of a half-way point may go either way; every
-    element meets the closed-form bound of Eq. 4 with binary16 s and z."""
+    """codes are the nearest level z + c*s (all 2^b levels enumerated), ties to the even
+    code, decided in exact rational arithmetic; every element meets the closed-form bound
+    of Eq. 4 with binary16 s and z."""
     rng = np.random.default_rng(1000 * b + G)
     levels = (1 << b) - 1
     for xb in _groups(rng, G, 60):
@@ -89,10 +102,11 @@ def test_quantizer_nearest_level_and_bound(b, G):
         dist = np.abs(x[:, None] - lv[None, :])
         best = dist.min(axis=1)
         chosen = dist[np.arange(G), codes]
-        u = (x - z) / s
-        near_tie = np.abs(np.abs(u - np.floor(u)) - 0.5) < 1e-5
-        ok = (chosen <= best * (1 + 1e-12) + 1e-300) | near_tie
-        assert ok.all()
+        assert (chosen <= best * (1 + 1e-9) + 1e-300).all()
+        # exactly: |x - level| is convex in the code, so the chosen code beats both
+        # neighbours (strictly, or equal with the chosen code even)
+        for xi, c in zip(x, codes):
+            assert _exact_nearest_ok(xi, z, s, int(c), levels), (xi, z, s, c)
         xhat = z + codes * s
         bound = max(s / 2 * (1 + 1e-5), z - mn, mx - lv[-1], 0.0)
         assert (np.abs(x - xhat) <= bound + 1e-300).all()
@@ -116,6 +130,29 @@ def test_quantizer_special_cases():
     vals = np.array([0, 3, 0.5, 1.5, 2.5, 1, 2, 3] * 4, dtype=np.float32)
     s16, z16, codes, _ = oracle.quantize_group(bf16_bits(vals), 2)
     assert list(codes[:8]) == [0, 3, 0, 2, 2, 1, 2, 3]
+
+
+def test_quantizer_rounds_the_exact_quotient():
+    """Near a half-way point the code follows the exact quotient (x - z) / s, not a
+    rounded one: with z = -2.5 and s = 1, x = +-2^-60 gives quotients 2.5 +- 2^-60, which
+    round to 3 and 2, although binary32 (or binary64) arithmetic would see a tie at 2.5."""
+    tiny = 2.0 ** -60
+    vals = np.array([-2.5, 0.5, tiny, -tiny, 0.0, 2.0 ** -30, -(2.0 ** -30), 0.5] * 4, dtype=np.float32)
+    s16, z16, codes, bad = oracle.quantize_group(bf16_bits(vals), 2)
+    assert not bad
+    assert float(np.uint16(s16).view(np.float16)) == 1.0
+    assert float(np.uint16(z16).view(np.float16)) == -2.5
+    assert list(codes[:8]) == [0, 3, 3, 2, 2, 3, 2, 3]
+    # the same at every half-way point c + 1/2 that bf16 inputs can put a tie on:
+    # z = -(c + 1/2), s = 1, x in {+tiny, -tiny, 0}
+    for b, cs in ((2, range(3)), (4, range(15)), (8, [127])):
+        levels = (1 << b) - 1
+        for c in cs:
+            grp = np.array([-(c + 0.5), levels - c - 0.5] + [tiny, -tiny, 0.0] * 10, dtype=np.float32)
+            s16, z16, codes, bad = oracle.quantize_group(bf16_bits(grp), b)
+            assert float(np.uint16(s16).view(np.float16)) == 1.0
+            assert float(np.uint16(z16).view(np.float16)) == -(c + 0.5)
+            assert list(codes[2:5]) == [c + 1, c, c + (c % 2)], (b, c)
 
 
 def test_quantizer_rejects_unrepresentable_values():
