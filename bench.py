@@ -209,6 +209,26 @@ def ncu_traffic(workload):
         return None
 
 
+def rank_spec(spec, rank):
+    """Each rank serves its own batches (weak scaling): a rank-specific seed."""
+    return spec.with_(seed=spec.seed + 1000 * rank)
+
+
+def across_ranks(dist, device, ms, *units):
+    """The job's time and work over one process per GPU: the MAX of the ranks' timed
+    milliseconds and the SUM of their work units (bytes, keys).  No data-path
+    collective exists; this is bookkeeping after the timed region."""
+    if dist is None:
+        return (float(ms), *[float(u) for u in units])
+    import torch
+    t = torch.tensor([float(ms)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    u = torch.tensor([float(x) for x in units], dtype=torch.float64, device=device)
+    if len(units):
+        dist.all_reduce(u, op=dist.ReduceOp.SUM)
+    return (float(t.item()), *[float(x) for x in u.tolist()])
+
+
 def _mix(*xs):
     """A deterministic 31-bit seed from small integers."""
     h = 0x9E3779B9
@@ -227,8 +247,7 @@ class Bench:
             spec = spec.with_(batch=args.batch)
         if args.layers:
             spec = spec.with_(num_layers=args.layers)
-        # each rank serves its own batches (weak scaling): a rank-specific seed
-        self.spec = spec.with_(seed=spec.seed + 1000 * rank)
+        self.spec = rank_spec(spec, rank)
         self.args, self.rank, self.world = args, rank, world
         s = self.spec
         self.L, self.B, self.Hq, self.Hkv, self.d, self.G = (
@@ -407,12 +426,10 @@ def run_gpu(args):
         t1.record()
         torch.cuda.synchronize()
     ms = t0.elapsed_time(t1)
-    if dist:
-        tt = torch.tensor([ms], dtype=torch.float64, device="cuda")
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms = float(tt.item())
     step_bytes = sum(bench.steps[i]["bytes"] for i in range(W, W + K))
     step_keys = sum(bench.steps[i]["keys"] for i in range(W, W + K))
+    rank_bytes = step_bytes
+    ms, job_bytes, job_keys = across_ranks(dist, "cuda", ms, step_bytes, step_keys)
     del graphs
 
     # attribution: the next K steps with event nodes around every trr_decode_attn call
@@ -478,10 +495,7 @@ def run_gpu(args):
     torch.cuda.synchronize()
     e2e_ms = a0.elapsed_time(a1)
     e2e_bytes = sum(bench.steps[e0 + j]["bytes"] for j in range(bench.e2e_warm, bench.e2e_warm + bench.e2e_steps))
-    if dist:
-        tt = torch.tensor([e2e_ms], dtype=torch.float64, device="cuda")
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        e2e_ms = float(tt.item())
+    e2e_ms, e2e_bytes = across_ranks(dist, "cuda", e2e_ms, e2e_bytes)
     status = bench.cache.status()
     if status != 0:
         raise RuntimeError(f"device status {status} after the run")
@@ -490,7 +504,7 @@ def run_gpu(args):
     avg_bytes = float(np.mean(call_bytes))
     avg_ms = float(np.mean(call_ms))
     achieved = avg_bytes / (avg_ms * 1e-3) / 1e9
-    value = world * step_bytes / (ms * 1e-3) / 1e9
+    value = job_bytes / (ms * 1e-3) / 1e9
     result = None
     if rank == 0:
         cpu = cpu_baseline(bench) if (world == 1 and not args.no_cpu_baseline) else None
@@ -505,15 +519,15 @@ def run_gpu(args):
                 "kv_storage": "per-token 2/4/8-bit codes + fp16 scale/zero, or bf16; fp32 accumulation",
                 "global_batch": bench.B * world, "replicas": bench.R,
                 "l2": "inputs larger than L2: every step reads its replica's "
-                      f"{step_bytes / K / 1e6:.0f} MB, replicas rotate",
+                      f"{rank_bytes / K / 1e6:.0f} MB, replicas rotate",
                 "parallelism": f"replicas{world}" if world > 1 else "single",
-                "bytes_per_step": int(step_bytes / K),
+                "bytes_per_step": int(job_bytes / K),
                 "split_bytes": args.split_bytes or "default",
             },
-            "kv_tokens_per_s": round(world * step_keys / (ms * 1e-3), 1),
+            "kv_tokens_per_s": round(job_keys / (ms * 1e-3), 1),
             "pct_of_8tbs": round(100 * value / world / 8000.0, 2),
             "gpu_launches": launches_per_step * K,
-            "e2e": {"value": round(world * e2e_bytes / (e2e_ms * 1e-3) / 1e9, 2), "unit": UNIT,
+            "e2e": {"value": round(e2e_bytes / (e2e_ms * 1e-3) / 1e9, 2), "unit": UNIT,
                     "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)},
             "roofline": {"bound": "hbm", "achieved": round(achieved, 2), "peak": peak,
                          "unit": "GB/s", "frac": round(achieved / peak, 4),
