@@ -17,7 +17,7 @@ value  = algorithmic attention bytes of the K steps / device time of the K steps
          keys in each non-skip query's range, plus Q and O rows)
 e2e    = the same, through the C ABI with host buffers: pinned H2D of every step's
          inputs and D2H of every step's outputs inside the timed region
-roofline: the dominant kernel is the trr_decode_attn call (plan + attention kernel);
+roofline: the dominant kernel is the trr_decode_attn call (one attention kernel);
          achieved = its algorithmic bytes per call / its average duration from CUDA
          event nodes placed around each call in a second, instrumented replay.
 """
@@ -532,7 +532,7 @@ def run_gpu(args):
             "roofline": {"bound": "hbm", "achieved": round(achieved, 2), "peak": peak,
                          "unit": "GB/s", "frac": round(achieved / peak, 4),
                          "traffic": ncu_traffic(args.workload), "peak_kind": peak_kind,
-                         "kernel": "trr_decode_attn call (attn_plan_kernel + attn_kernel)",
+                         "kernel": "trr_decode_attn call (attn_kernel, one launch)",
                          "bytes_per_call": round(avg_bytes), "us_per_call": round(avg_ms * 1e3, 3)},
             "clocks": clocks.summary(),
         }

@@ -1,23 +1,24 @@
 // trr_attn.cu - trr_decode_attn: mode-routed split-K decode attention over the
 // mixed-precision paged cache (Sec. 3.2(A), Eq. 2; Sec. 3.8; Sec. 7).
 //
-// Two kernels per call, chained with programmatic dependent launch:
-//   attn_plan_kernel  one warp per query.  Key range by mode (full: [0, t]; local:
-//                     [t-w+1, t]; skip: none); for each width class the pages that
-//                     intersect it, found by a 32-way search over the pages'
-//                     first / last positions (all classes and both ends at once); the
-//                     number of split-K work items from the bytes in range.  Skip
-//                     queries and empty ranges get their zero rows here.
-//   attn_kernel       persistent, two CTAs per SM, every warp an independent worker.
-//                     Work items (query, head, split) are dealt round-robin.  A warp
-//                     streams the pages of its items through a private 3-slot ring of
-//                     shared memory filled by 1-D bulk copies (cp.async.bulk +
-//                     mbarrier), with the query row riding on the first copy of each
-//                     item, so items follow each other without a pipeline drain.
-//                     Lane pair (key, half) of a 64-wide head (four lanes for 128)
-//                     dequantises in registers and keeps its own online softmax;
-//                     lanes merge with shuffles; one split writes the bf16 row, several
-//                     write fp32 partials and the last to arrive merges them.
+// One persistent kernel per call (two CTAs per SM, every warp an independent worker):
+//   1. Every CTA cuts the call into work units: query q gets ns_q splits from the
+//      length of its key range (full: [0, t]; local: [t-w+1, t]; skip or invalid: one
+//      unit that writes the zero row) and a prefix sum numbers the units.  The same
+//      deterministic computation in every CTA takes the place of a planning kernel.
+//   2. Work items (unit, query head) are dealt round-robin to the warps.  A warp plans
+//      its item itself: the sequence's per-class token counts, a 32-way search of the
+//      pages' first / last positions at window edges, and the split's share of every
+//      class's pages in range (one page id per lane).  It streams those pages' slices
+//      of the head through a private ring of shared memory filled by 1-D bulk copies
+//      (cp.async.bulk + mbarrier), the query row riding on the first copy of each
+//      item, so items follow each other without a pipeline drain.  Lane pair (key,
+//      half) of a 64-wide head (four lanes for 128) dequantises in registers and keeps
+//      its own online softmax; lanes merge with shuffles.
+//   3. A query with one split gets its bf16 row from that item.  Otherwise each split
+//      writes an fp32 partial and counts its arrival; the last split of the (query,
+//      head) to arrive merges the partials, writes the row and resets the counter.
+//   4. The last CTA to finish records the error of the lowest failing query.
 //
 // Dequantisation: k = z + c*s, so q.k = s * sum(q_i c_i) + z * sum(q_i).  A code is
 // masked in place (no shift) and its bits read as a binary32 subnormal, c * 2^(e-149)
@@ -37,186 +38,52 @@ constexpr float kTau = 8.f;    // lazy rescale threshold (log2 units)
 
 // ----------------------------------------------------------------------- plan --
 
-// Count of k in [0, n) with arr[k] < x (arr increasing), searched by the whole warp.
-// The first round probes the last 32 entries: decode queries look at the end of the
-// page lists, so that round almost always settles it.  Otherwise 32 probes per round
-// narrow the rest.  Every search of the call advances in the same round.
+// For NS increasing arrays arr_i = base + i * stride of n[i] entries: the count of
+// entries below x, searched by the whole warp.  The first round probes the last 32
+// entries: decode queries look at the end of the page lists, so that round almost always
+// settles it.  Otherwise 32 probes per round narrow the rest.  Every search advances in
+// the same round.
 template <int NS>
-__device__ __forceinline__ void warp_count_below(const int* const (&arr)[NS], const int (&n)[NS],
-                                                 const int (&x)[NS], int (&out)[NS], int lane) {
+__device__ __forceinline__ void warp_count_below(const int* base, int64_t stride, const int (&n)[NS], int x,
+                                                 int (&out)[NS], int lane) {
   int lo[NS], hi[NS];
-  {
-    int v[NS], idx[NS];
 #pragma unroll
-    for (int i = 0; i < NS; ++i) {
-      idx[i] = max(0, n[i] - 32) + lane;
-      v[i] = idx[i] < n[i] ? arr[i][idx[i]] : INT_MAX;
-    }
-#pragma unroll
-    for (int i = 0; i < NS; ++i) {
-      const unsigned below = __ballot_sync(0xffffffffu, idx[i] < n[i] && v[i] < x[i]);
-      const int base = max(0, n[i] - 32);
-      if (n[i] <= 32 || (below & 1u)) {  // arr[base] < x: everything before it is too
-        lo[i] = hi[i] = base + __popc(below);
-      } else {
-        lo[i] = 0;
-        hi[i] = base;
-      }
+  for (int i = 0; i < NS; ++i) {
+    const int idx = max(0, n[i] - 32) + lane;
+    const int v = idx < n[i] ? base[i * stride + idx] : INT_MAX;
+    const unsigned below = __ballot_sync(0xffffffffu, idx < n[i] && v < x);
+    const int b = max(0, n[i] - 32);
+    if (n[i] <= 32 || (below & 1u)) {  // arr[b] < x: everything before it is too
+      lo[i] = hi[i] = b + __popc(below);
+    } else {
+      lo[i] = 0;
+      hi[i] = b;
     }
   }
   for (int round = 0; round < 6; ++round) {
-    int v[NS], idx[NS], step[NS];
     bool any = false;
 #pragma unroll
-    for (int i = 0; i < NS; ++i) {
-      const int span = hi[i] - lo[i];
-      step[i] = span <= 32 ? 1 : (span + 31) / 32;
-      idx[i] = lo[i] + lane * step[i];
-      v[i] = (span > 0 && idx[i] < hi[i]) ? arr[i][idx[i]] : INT_MAX;
-      any |= span > 0;
-    }
+    for (int i = 0; i < NS; ++i) any |= hi[i] > lo[i];
     if (!any) break;
 #pragma unroll
     for (int i = 0; i < NS; ++i) {
       const int span = hi[i] - lo[i];
-      const int cnt = __popc(__ballot_sync(0xffffffffu, idx[i] < hi[i] && v[i] < x[i]));
+      const int step = span <= 32 ? 1 : (span + 31) / 32;
+      const int idx = lo[i] + lane * step;
+      const int v = (span > 0 && idx < hi[i]) ? base[i * stride + idx] : INT_MAX;
+      const int cnt = __popc(__ballot_sync(0xffffffffu, idx < hi[i] && v < x));
       if (span <= 0) continue;
       if (span <= 32 || cnt == 0) {
         lo[i] = hi[i] = lo[i] + (span <= 32 ? cnt : 0);
       } else {
-        const int last = lo[i] + (cnt - 1) * step[i];  // last probe below x
-        hi[i] = min(hi[i], lo[i] + cnt * step[i]);
+        const int last = lo[i] + (cnt - 1) * step;  // last probe below x
+        hi[i] = min(hi[i], lo[i] + cnt * step);
         lo[i] = last + 1;
       }
     }
   }
 #pragma unroll
   for (int i = 0; i < NS; ++i) out[i] = lo[i];
-}
-
-__global__ void __launch_bounds__(256) attn_plan_kernel(LayerArgs a, int n, const int32_t* __restrict__ seq_ids,
-                                                        const int32_t* __restrict__ q_positions,
-                                                        const uint8_t* __restrict__ modes,
-                                                        const int32_t* __restrict__ windows, int window_scalar,
-                                                        uint16_t* __restrict__ out) {
-  pdl_wait();
-  pdl_trigger();
-  const int lane = threadIdx.x & 31;
-  const int qi = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-  if (qi >= n) return;
-  const int seq = seq_ids[qi], t = q_positions[qi], mode = modes[qi];
-  const int w = windows ? windows[qi] : window_scalar;
-  int err = 0;
-  if (seq < 0 || seq >= a.S || mode > TRR_MODE_FULL) err = TRR_ERR_INVALID_ARG;
-  else if (t < 0 || t >= a.maxctx) err = TRR_ERR_BAD_POSITION;
-  else if (mode == TRR_MODE_LOCAL && w < 1) err = TRR_ERR_INVALID_ARG;
-
-  QueryPlan qp;
-  qp.seq = seq;
-  qp.err = err;
-  qp.nsplit = 0;
-  qp.lo = 0;
-  qp.hi = t;
-  qp.base = qp.pad1 = qp.pad2 = 0;
-#pragma unroll
-  for (int c = 0; c < kClasses; ++c) qp.first[c] = qp.npages[c] = qp.ntok[c] = 0;
-  int total_pages = 0;
-  bool upper_mask = false;  // the query sits before the sequence's last stored position
-  if (!err && mode != TRR_MODE_SKIP) {
-    const int lo = mode == TRR_MODE_FULL ? 0 : max(0, t - w + 1);
-    qp.lo = lo;
-    upper_mask = t < a.last_pos[seq];
-    const int* arr[2 * kClasses];
-    int np[2 * kClasses], x[2 * kClasses], cnt[2 * kClasses];
-#pragma unroll
-    for (int c = 0; c < kClasses; ++c) {
-      const int nt = a.ntok[seq * 4 + c];
-      qp.ntok[c] = nt;
-      const int64_t row = static_cast<int64_t>(seq * 4 + c) * a.MP;
-      arr[c] = a.plast + row;                 // pages ending before lo
-      np[c] = lo > 0 ? (nt + a.P - 1) / a.P : 0;
-      x[c] = lo;
-      arr[kClasses + c] = a.pfirst + row;     // pages starting at or before t
-      np[kClasses + c] = (nt + a.P - 1) / a.P;
-      x[kClasses + c] = t + 1;
-    }
-    warp_count_below<2 * kClasses>(arr, np, x, cnt, lane);
-    int64_t bytes = 0;
-#pragma unroll
-    for (int c = 0; c < kClasses; ++c) {
-      qp.first[c] = cnt[c];
-      qp.npages[c] = max(0, cnt[kClasses + c] - cnt[c]);
-      bytes += static_cast<int64_t>(qp.npages[c]) * a.slice[c];
-      total_pages += qp.npages[c];
-    }
-    if (bytes > 0) {
-      int64_t ns = max((bytes + a.split_bytes - 1) / a.split_bytes,
-                       static_cast<int64_t>((total_pages + kDescMaxPages - 1) / kDescMaxPages));
-      ns = min(ns, static_cast<int64_t>(a.s_cap));
-      qp.nsplit = static_cast<int>(min(ns, static_cast<int64_t>(total_pages)));
-    }
-  }
-  if (qp.nsplit == 0) {  // skip, invalid or nothing stored in range: a zero row
-    if (lane < 20) reinterpret_cast<int*>(a.qplan + qi)[lane] = reinterpret_cast<const int*>(&qp)[lane];
-    uint4* o = reinterpret_cast<uint4*>(out + static_cast<int64_t>(qi) * a.Hq * a.d);
-    const int n16 = a.Hq * a.d / 8;
-    for (int i = lane; i < n16; i += 32) o[i] = make_uint4(0, 0, 0, 0);
-    if (err && lane == 0) atomicMin(&a.ctrl[kFirstBadQuery], qi);
-    return;
-  }
-  // Descriptors: one per split, at consecutive indices taken from a shared counter.
-  // Split sp of class c takes the class's pages [first + sp*np/ns, first + (sp+1)*np/ns).
-  const int ns = qp.nsplit;
-  const int c1 = qp.npages[0], c2 = c1 + qp.npages[1], c3 = c2 + qp.npages[2];
-  constexpr int kBatch = 8;  // page ids loaded before any descriptor store
-  int id[kBatch], cls[kBatch], kid[kBatch];
-  auto load_batch = [&](int f0) {
-#pragma unroll
-    for (int b = 0; b < kBatch; ++b) {
-      const int f = f0 + 32 * b + lane;
-      const int c = (f >= c1) + (f >= c2) + (f >= c3);
-      const int local = f - (c == 0 ? 0 : c == 1 ? c1 : c == 2 ? c2 : c3);
-      cls[b] = c;
-      kid[b] = qp.first[c] + local;
-      id[b] = f < total_pages ? a.pt[static_cast<int64_t>(seq * 4 + c) * a.MP + kid[b]] : -1;
-    }
-  };
-  load_batch(0);  // in flight together with the counter atomic
-  int base = 0;
-  if (lane == 0) base = atomicAdd(&a.ctrl[kDescCounter], ns);
-  base = __shfl_sync(0xffffffffu, base, 0);
-  qp.base = base;
-  if (lane < 20) reinterpret_cast<int*>(a.qplan + qi)[lane] = reinterpret_cast<const int*>(&qp)[lane];
-  SplitDesc* dsc = a.desc + base;
-  auto bnd = [&](int c, int sp) { return static_cast<int>(static_cast<int64_t>(sp) * qp.npages[c] / ns); };
-  for (int sp = lane; sp < ns; sp += 32) {
-    int T = 0;
-#pragma unroll
-    for (int c = 0; c < kClasses; ++c) T += bnd(c, sp + 1) - bnd(c, sp);
-    int* h = &dsc[sp].qi;
-    h[0] = qi; h[1] = seq; h[2] = qp.lo; h[3] = qp.hi; h[4] = ns; h[5] = sp; h[6] = T; h[7] = base;
-  }
-  for (int f0 = 0; f0 < total_pages; f0 += 32 * kBatch) {
-    if (f0 > 0) load_batch(f0);
-#pragma unroll
-    for (int b = 0; b < kBatch; ++b) {
-      const int f = f0 + 32 * b + lane;
-      if (f >= total_pages) break;
-      const int c = cls[b];
-      const int local = kid[b] - qp.first[c];
-      const int np = qp.npages[c];
-      const int sp = static_cast<int>((static_cast<int64_t>(local + 1) * ns - 1) / np);
-      int pos = local - bnd(c, sp);
-      for (int c0 = 0; c0 < c; ++c0) pos += bnd(c0, sp + 1) - bnd(c0, sp);
-      const int fill = min(a.P, qp.ntok[c] - kid[b] * a.P);
-      // slot positions are needed on a page that may hold keys outside [lo, t]: the
-      // first page of a window that starts after 0, the last one when t is not the
-      // sequence's last stored position
-      const bool mask = (qp.lo > 0 && local == 0) || (upper_mask && local == np - 1);
-      dsc[sp].page[pos] = id[b];
-      dsc[sp].meta[pos] = c | (fill << 2) | (mask ? 512 : 0);
-    }
-  }
 }
 
 // ------------------------------------------------------------------ dequant --
@@ -442,18 +309,38 @@ __device__ __forceinline__ void consume_page(const uint8_t* sl, const int* spos,
 
 // -------------------------------------------------------------------- kernel --
 
-constexpr int kSlots = 8;  // pages a warp may have in flight (one mbarrier each)
+constexpr int kSlots = 8;          // pages a warp may have in flight (one mbarrier each)
+constexpr int kItemsPerWarp = 3;   // splits are made small enough for about this many
+                                   // items per warp (never below the cache's pos_split)
 
 struct AttnKernelArgs {
   LayerArgs a;
+  int n;                       // queries of the call
+  const int32_t* seq_ids;
+  const int32_t* q_positions;
+  const uint8_t* modes;
+  const int32_t* windows;      // per-query windows, or null: window_scalar
+  int window_scalar;
   const uint16_t* q;
   uint16_t* out;
   float qscale;      // softmax scale * log2(e)
   int ring_bytes;    // bytes of one warp's ring of shared memory
-  int max_desc;      // capacity of the descriptor array
 };
 
-// Per-page record the producer writes for the consumer (two 16-byte words).
+// Error of a query's arguments, 0 when it is valid.
+__device__ __forceinline__ int query_error(const LayerArgs& a, int seq, int t, int mode, int w) {
+  if (seq < 0 || seq >= a.S || mode > TRR_MODE_FULL) return TRR_ERR_INVALID_ARG;
+  if (t < 0 || t >= a.maxctx) return TRR_ERR_BAD_POSITION;
+  if (mode == TRR_MODE_LOCAL && w < 1) return TRR_ERR_INVALID_ARG;
+  return 0;
+}
+
+// Key positions in range (Eq. 2): full [0, t]; local the last w positions up to t.
+__device__ __forceinline__ int query_range(int t, int mode, int w) {
+  return mode == TRR_MODE_FULL ? t + 1 : mode == TRR_MODE_LOCAL ? min(w, t + 1) : 0;
+}
+
+// Per-page record the producer writes for the consumer (three 16-byte words).
 struct SlotRec {
   int meta;   // class | fill << 2 | mask << 9 | flags << 10 (1 first, 2 last, 4 no page)
   int off;    // ring offset of the page's slice (then its positions when masked, then
@@ -461,35 +348,123 @@ struct SlotRec {
   int span;   // ring bytes to release after the page
   int lo;     // key range [lo, hi] of the item's query
   int hi, item, qi, qh;
-  int nsplit, pad0, pad1, pad2;
+  int nsplit, base, pad0, pad1;  // base: unit index of split 0 of the item's query
 };
 static_assert(sizeof(SlotRec) == 48, "SlotRec is three 16-byte words");
 
 // Shared-memory carve-up of one attention CTA; every region starts 16-byte aligned
 // (mbarriers need 8, bulk-copy destinations 16).
 __host__ __device__ constexpr int align16(int x) { return (x + 15) & ~15; }
+constexpr int kWarpWords = 16;  // per-warp shared words: [0, 8) item plan, [8, 14) merge
 struct AttnSmem {
-  int rings, recs, bars, total;
-  __host__ __device__ AttnSmem(int nwarps, int ring_bytes)
+  int rings, recs, bars, words, pre, red, total;
+  __host__ __device__ AttnSmem(int nwarps, int ring_bytes, int n)
       : rings(0),
         recs(align16(nwarps * ring_bytes)),
         bars(recs + align16(nwarps * kSlots * static_cast<int>(sizeof(SlotRec)))),
-        total(bars + align16(nwarps * kSlots * 8)) {}
+        words(bars + align16(nwarps * kSlots * 8)),
+        pre(words + nwarps * kWarpWords * 4),
+        red(pre + align16(4 * (n + 1))),
+        total(red + 16 * 8) {}
 };
 
+// The plan of one work item as the producer needs it: lane j holds page j's id and meta
+// in registers; the item's fields sit in the warp's shared words (written by lane 0):
+// [0] lo [1] hi [2] item [3] query [4] query head [5] splits [6] unit of split 0 [7] KV head.
 template <int D>
-__global__ void __launch_bounds__(256, 2) attn_kernel(const AttnKernelArgs ka) {
+__device__ __forceinline__ int plan_next_item(const AttnKernelArgs& ka, const int* pre, int n, int wstride, int lane,
+                                           int* next_item, int* wplan, int& wid, int& wmeta) {
+  const LayerArgs& a = ka.a;
+  const int total = pre[n] * a.Hq;
+  while (*next_item < total) {
+    const int i = *next_item;
+    *next_item += wstride;
+    const int u = i / a.Hq, h = i - u * a.Hq;
+    int lo_q = 0, hi_q = n;  // the query of unit u: pre[q] <= u < pre[q + 1]
+    while (hi_q - lo_q > 1) {
+      const int mid = (lo_q + hi_q) >> 1;
+      if (pre[mid] <= u) lo_q = mid;
+      else hi_q = mid;
+    }
+    const int q = lo_q, sp = u - pre[q], ns = pre[q + 1] - pre[q];
+    const int seq = ka.seq_ids[q], t = ka.q_positions[q], mode = ka.modes[q];
+    const int w = ka.windows ? ka.windows[q] : ka.window_scalar;
+    const int err = query_error(a, seq, t, mode, w);
+    if (err || mode == TRR_MODE_SKIP) {  // a zero row; the error of the lowest query
+      uint4* o = reinterpret_cast<uint4*>(ka.out + (static_cast<int64_t>(q) * a.Hq + h) * D);
+      if (lane < D / 8) o[lane] = make_uint4(0, 0, 0, 0);
+      if (err && h == 0 && lane == 0) atomicMin(&a.ctrl[kFirstBadQuery], q * 16 + err);
+      continue;
+    }
+    const int lo = mode == TRR_MODE_FULL ? 0 : max(0, t - w + 1);
+    // per class: pages ending before lo, pages starting at or before t
+    int nt[kClasses];
+#pragma unroll
+    for (int c = 0; c < kClasses; ++c) nt[c] = a.ntok[seq * 4 + c];
+    const bool upper_mask = t < a.last_pos[seq];  // keys after t may be stored
+    int pages[kClasses], first[kClasses], end[kClasses];
+#pragma unroll
+    for (int c = 0; c < kClasses; ++c) {
+      pages[c] = (nt[c] + a.P - 1) / a.P;
+      first[c] = 0;
+      end[c] = pages[c];
+    }
+    const int64_t row0 = static_cast<int64_t>(seq) * 4 * a.MP;
+    if (lo > 0) warp_count_below<kClasses>(a.plast + row0, a.MP, pages, lo, first, lane);
+    if (upper_mask) warp_count_below<kClasses>(a.pfirst + row0, a.MP, pages, t + 1, end, lane);
+    // this split's share of each class's pages in range, then one page per lane
+    int beg[kClasses], tc[kClasses], npr[kClasses];
+    int T = 0;
+#pragma unroll
+    for (int c = 0; c < kClasses; ++c) {
+      npr[c] = max(0, end[c] - first[c]);
+      beg[c] = first[c] + static_cast<int>(static_cast<int64_t>(sp) * npr[c] / ns);
+      tc[c] = first[c] + static_cast<int>(static_cast<int64_t>(sp + 1) * npr[c] / ns) - beg[c];
+      T += tc[c];
+    }
+    T = min(T, kItemMaxPages + kClasses);  // the split bound keeps T within this
+    wid = -1;
+    wmeta = 0;
+    if (lane < T) {
+      const int t1 = tc[0], t2 = t1 + tc[1], t3 = t2 + tc[2];
+      const int c = (lane >= t1) + (lane >= t2) + (lane >= t3);
+      auto pick = [c](const int (&v)[kClasses]) { return c == 0 ? v[0] : c == 1 ? v[1] : c == 2 ? v[2] : v[3]; };
+      const int kid = pick(beg) + lane - (c == 0 ? 0 : c == 1 ? t1 : c == 2 ? t2 : t3);
+      const int f = pick(first);
+      wid = a.pt[static_cast<int64_t>(seq * 4 + c) * a.MP + kid];
+      const int fill = min(a.P, pick(nt) - kid * a.P);
+      // slot positions are needed on a page that may hold keys outside [lo, t]
+      const bool mask = (lo > 0 && kid == f) || (upper_mask && kid == f + pick(npr) - 1);
+      wmeta = c | (fill << 2) | (mask ? 512 : 0);
+    }
+    if (lane == 0) {
+      reinterpret_cast<int4*>(wplan)[0] = make_int4(lo, t, i, q);
+      reinterpret_cast<int4*>(wplan)[1] = make_int4(h, ns, pre[q], h / (a.Hq / a.Hkv));
+    }
+    __syncwarp();
+    return T;
+  }
+  return -1;
+}
+
+template <int D>
+__global__ void __launch_bounds__(256, 2) attn_kernel(const __grid_constant__ AttnKernelArgs ka) {
   constexpr int LPK = D / 32;  // lanes per key
   constexpr int DPL = D / 32;  // dimensions per lane after the merge
   const LayerArgs& a = ka.a;
   extern __shared__ __align__(128) uint8_t smem[];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+  const int n = ka.n;
   const int qrow = D * 2;  // bytes of one query row
   const int R = ka.ring_bytes;
-  const AttnSmem lay(nwarps, R);  // [rings][slot records][mbarriers]
+  const AttnSmem lay(nwarps, R, n);  // [rings][slot records][mbarriers][unit prefix][scratch]
   uint8_t* ring = smem + lay.rings + warp * R;
   SlotRec* recs = reinterpret_cast<SlotRec*>(smem + lay.recs) + warp * kSlots;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + lay.bars) + warp * kSlots;
+  int* pre = reinterpret_cast<int*>(smem + lay.pre);
+  int* wplan = reinterpret_cast<int*>(smem + lay.words) + warp * kWarpWords;
+  int* wmerge = wplan + 8;
+  long long* red = reinterpret_cast<long long*>(smem + lay.red);
 
   if (lane == 0) {
 #pragma unroll
@@ -498,55 +473,69 @@ __global__ void __launch_bounds__(256, 2) attn_kernel(const AttnKernelArgs ka) {
   }
   pdl_wait();
   pdl_trigger();
-  const int group = a.Hq / a.Hkv;
+
+  // ---------------------------------------------------------- work units --
+  // Every CTA computes the same split of the call: query q gets ns_q splits from its key
+  // range; pre[q] numbers its first unit, pre[n] counts them all.
+  long long rsum = 0;
+  for (int q = threadIdx.x; q < n; q += blockDim.x) {
+    const int seq = ka.seq_ids[q], t = ka.q_positions[q], mode = ka.modes[q];
+    const int w = ka.windows ? ka.windows[q] : ka.window_scalar;
+    const int r = query_error(a, seq, t, mode, w) ? 0 : query_range(t, mode, w);
+    pre[q] = r;
+    rsum += r;
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) rsum += __shfl_xor_sync(0xffffffffu, rsum, o);
+  if (lane == 0) red[warp] = rsum;
+  __syncthreads();
+  rsum = 0;
+  for (int k = 0; k < nwarps; ++k) rsum += red[k];
+  // splits small enough for about kItemsPerWarp items per warp, never below pos_split
+  const long long want = static_cast<long long>(gridDim.x) * nwarps * kItemsPerWarp;
+  const long long by_work = (rsum * a.Hq + want - 1) / want;
+  const int pos_split = static_cast<int>(max(static_cast<long long>(a.pos_split), min(by_work, 1ll << 30)));
+  {
+    const int chunk = (n + blockDim.x - 1) / blockDim.x;
+    const int q0 = min(n, static_cast<int>(threadIdx.x) * chunk), q1 = min(n, q0 + chunk);
+    int mine = 0;
+    for (int q = q0; q < q1; ++q) mine += splits_of(pre[q], pos_split, a.P, a.s_cap);
+    int incl = mine;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int v = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += v;
+    }
+    __syncthreads();  // every read of red above is done
+    if (lane == 31) red[8 + warp] = incl;
+    __syncthreads();
+    int off = incl - mine;
+    for (int k = 0; k < warp; ++k) off += static_cast<int>(red[8 + k]);
+    for (int q = q0; q < q1; ++q) {
+      const int ns = splits_of(pre[q], pos_split, a.P, a.s_cap);
+      pre[q] = off;
+      off += ns;
+    }
+    if (threadIdx.x == blockDim.x - 1) pre[n] = off;
+    __syncthreads();
+  }
   const int wstride = gridDim.x * nwarps;
 
   // ------------------------------------------------------------ producer --
-  // Work items are (descriptor, query head) pairs dealt round-robin.  The descriptor of
-  // the producer's next item is prefetched one item ahead (three words per lane).
+  // Items are dealt round-robin; consecutive warps take consecutive heads of one unit,
+  // so the planning loads of a unit mostly hit in L1.
   int next_item = blockIdx.x * nwarps + warp;
-  int nd0 = 0, nd1 = 0, nd2 = 0;       // prefetched descriptor: page ids, metas, header
-  auto prefetch = [&](int item) {
-    const int d = item / a.units;
-    if (d >= ka.max_desc) return;  // past any descriptor the plan can write
-    const int* dp = reinterpret_cast<const int*>(a.desc + d);
-    nd0 = dp[lane];
-    nd1 = dp[32 + lane];
-    nd2 = lane < 8 ? dp[64 + lane] : 0;
-  };
-  prefetch(next_item);  // in flight together with the descriptor count
-  const int total = *reinterpret_cast<volatile int*>(a.ctrl + kDescCounter) * a.units;
-  if (blockIdx.x == 0 && threadIdx.x == 0) {  // status of the lowest invalid query
-    const int bad = a.ctrl[kFirstBadQuery];
-    if (bad != INT_MAX) {
-      set_status(a.ctrl, a.qplan[bad].err);
-      a.ctrl[kFirstBadQuery] = INT_MAX;
-    }
-  }
-
   int wid = -1, wmeta = 0;             // the producer's item: page id / meta of page `lane`
-  int p_item = 0, p_qi = 0, p_qh = 0, p_kvh = 0, p_nsplit = 0, p_T = 0, p_lo = 0, p_hi = 0;
+  int p_T = 0;                         // pages of the producer's item
   int pf = 0;                          // next page of the producer's item
   bool pvalid = false;
   uint32_t issued = 0, consumed = 0;   // pages issued / consumed by this warp
   int head = 0, used = 0;              // ring: next free offset, bytes held
 
   auto start_item = [&]() -> bool {
-    if (next_item >= total) return false;
-    p_item = next_item;
-    wid = nd0;
-    wmeta = nd1;
-    p_qi = __shfl_sync(0xffffffffu, nd2, 0);
-    p_lo = __shfl_sync(0xffffffffu, nd2, 2);
-    p_hi = __shfl_sync(0xffffffffu, nd2, 3);
-    p_nsplit = __shfl_sync(0xffffffffu, nd2, 4);
-    p_T = __shfl_sync(0xffffffffu, nd2, 6);
-    p_qh = p_item - (p_item / a.units) * a.units;
-    p_kvh = p_qh / group;
-    next_item += wstride;
-    if (next_item < total) prefetch(next_item);
+    p_T = plan_next_item<D>(ka, pre, n, wstride, lane, &next_item, wplan, wid, wmeta);
     pf = 0;
-    return true;
+    return p_T >= 0;
   };
   // start the copies of the producer's next page if a slot and ring space are free
   auto try_issue = [&]() -> bool {
@@ -579,19 +568,21 @@ __global__ void __launch_bounds__(256, 2) attn_kernel(const AttnKernelArgs ka) {
     // record reaches the consumer through the mbarrier's release / acquire, so no proxy
     // fence is needed here.
     if (lane == 0) {
+      const int4 pa = reinterpret_cast<const int4*>(wplan)[0];  // lo, hi, item, query
+      const int4 pb = reinterpret_cast<const int4*>(wplan)[1];  // head, splits, base, KV head
       int4* rp = reinterpret_cast<int4*>(recs + slot);
-      rp[0] = make_int4(meta | (flags << 10), off, waste + need, p_lo);
-      rp[1] = make_int4(p_hi, p_item, p_qi, p_qh);
-      rp[2] = make_int4(p_nsplit, 0, 0, 0);
+      rp[0] = make_int4(meta | (flags << 10), off, waste + need, pa.x);
+      rp[1] = make_int4(pa.y, pa.z, pa.w, pb.x);
+      rp[2] = make_int4(pb.y, pb.z, 0, 0);
       mbar_arrive_expect_tx(&bars[slot], need);
       const int c = meta & 3;
       if (p_T > 0) {
         const uint8_t* page = a.pool[c] + static_cast<int64_t>(id) * a.page_bytes[c];
-        bulk_g2s(ring + off, page + a.hdr + static_cast<int64_t>(p_kvh) * a.slice[c], a.slice[c], &bars[slot]);
+        bulk_g2s(ring + off, page + a.hdr + static_cast<int64_t>(pb.w) * a.slice[c], a.slice[c], &bars[slot]);
         if (meta & 512) bulk_g2s(ring + off + a.slice[c], page, 4 * a.P, &bars[slot]);
       }
       if (first)
-        bulk_g2s(ring + off + bytes_page, ka.q + (static_cast<int64_t>(p_qi) * a.Hq + p_qh) * D, qrow, &bars[slot]);
+        bulk_g2s(ring + off + bytes_page, ka.q + (static_cast<int64_t>(pa.w) * a.Hq + pb.x) * D, qrow, &bars[slot]);
     }
     __syncwarp();
     ++issued;
@@ -600,33 +591,117 @@ __global__ void __launch_bounds__(256, 2) attn_kernel(const AttnKernelArgs ka) {
     return true;
   };
 
-  while (try_issue()) {
-  }
-
   // ------------------------------------------------------------ consumer --
   const int part = lane % LPK, kl = lane / LPK;
   LaneState st;
   float qp[32];
   float sumq = 0.f;
   int cur_cls = 3;
-  int c_lo = 0, c_hi = 0;  // key range of the consumer's item
   st.m = kNegInf;
   st.l = 0.f;
   st.zacc = 0.f;
-  while (consumed < issued) {
+  // The merge of an item's lanes and splits, once its last page is consumed.
+  bool merge_pending = false;
+  auto merge_item = [&]() {
+    const int4 mr = reinterpret_cast<const int4*>(wmerge)[0];  // item, query, head, splits
+    const int m_item = mr.x, m_qi = mr.y, m_qh = mr.z, m_nsplit = mr.w, m_base = wmerge[4];
+    // merge the lanes that share a part.  Rescale to the common maximum, then
+    // reduce-scatter over the key lanes: each halving step keeps half of the 32 dims
+    // and sends the other half to the partner lane.
+    acc_to_neutral(st.acc, cur_cls);
+    float M = st.m;
+#pragma unroll
+    for (int o = LPK; o < 32; o <<= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+    const float f = (st.m == kNegInf) ? 0.f : fast_exp2(st.m - M);
+    float L = st.l * f;
+#pragma unroll
+    for (int o = LPK; o < 32; o <<= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
+#pragma unroll
+    for (int j = 0; j < 32; ++j) st.acc[j] = fmaf(st.acc[j], pow2f(49), st.zacc) * f;
+#pragma unroll
+    for (int width = 16, o = 16; o >= LPK; width >>= 1, o >>= 1) {
+      const bool upper = lane & o;
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        if (i < width) {
+          const float keep = upper ? st.acc[width + i] : st.acc[i];
+          const float give = upper ? st.acc[i] : st.acc[width + i];
+          st.acc[i] = keep + __shfl_xor_sync(0xffffffffu, give, o);
+        }
+      }
+    }
+    // lane (kl, part) now holds dims part*32 + DPL*kl .. + DPL-1 in acc[0 .. DPL-1]
+    const int dim0 = part * 32 + DPL * kl;
+    const int64_t orow = (static_cast<int64_t>(m_qi) * a.Hq + m_qh) * D;
+    if (m_nsplit == 1) {
+      const float inv = L > 0.f ? 1.f / L : 0.f;
+#pragma unroll
+      for (int j = 0; j < DPL; j += 2)
+        *reinterpret_cast<__nv_bfloat162*>(ka.out + orow + dim0 + j) =
+            __floats2bfloat162_rn(st.acc[j] * inv, st.acc[j + 1] * inv);
+      return;
+    }
+    // a partial at the item's index; the last split of (query, head) to arrive merges
+    float* pp = a.part + static_cast<int64_t>(m_item) * (D + 4);
+#pragma unroll
+    for (int j = 0; j < DPL; j += 2)
+      *reinterpret_cast<float2*>(pp + dim0 + j) = make_float2(st.acc[j], st.acc[j + 1]);
+    if (lane == 0) *reinterpret_cast<float2*>(pp + D) = make_float2(M, L);
+    __threadfence();
+    __syncwarp();
+    int arrivals = 0;
+    int* counter = a.cnt + static_cast<int64_t>(m_qi) * a.Hq + m_qh;
+    if (lane == 0) arrivals = atomicAdd(counter, 1);
+    arrivals = __shfl_sync(0xffffffffu, arrivals, 0);
+    if (arrivals != m_nsplit - 1) return;
+    __threadfence();
+    const float* p0 = a.part + (static_cast<int64_t>(m_base) * a.Hq + m_qh) * (D + 4);
+    const int64_t sstride = static_cast<int64_t>(a.Hq) * (D + 4);
+    float Mx = kNegInf;
+    for (int s = lane; s < m_nsplit; s += 32) Mx = fmaxf(Mx, __ldcg(p0 + s * sstride + D));
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) Mx = fmaxf(Mx, __shfl_xor_sync(0xffffffffu, Mx, o));
+    float Ls = 0.f, acc_o[DPL];
+#pragma unroll
+    for (int j = 0; j < DPL; ++j) acc_o[j] = 0.f;
+#pragma unroll 4
+    for (int s = 0; s < m_nsplit; ++s) {
+      const float* ps = p0 + s * sstride;
+      const float2 ml = __ldcg(reinterpret_cast<const float2*>(ps + D));
+      const float wgt = (ml.x == kNegInf) ? 0.f : fast_exp2(ml.x - Mx);
+      Ls = fmaf(wgt, ml.y, Ls);
+#pragma unroll
+      for (int j = 0; j < DPL; ++j) acc_o[j] = fmaf(wgt, __ldcg(ps + lane * DPL + j), acc_o[j]);
+    }
+    const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
+#pragma unroll
+    for (int j = 0; j < DPL; j += 2)
+      *reinterpret_cast<__nv_bfloat162*>(ka.out + orow + lane * DPL + j) =
+          __floats2bfloat162_rn(acc_o[j] * inv, acc_o[j + 1] * inv);
+    if (lane == 0) *counter = 0;  // ready for the next call
+  };
+
+  for (;;) {
+    // refill first, so that the next item's copies fly while this one merges; the one
+    // place the producer plans items
+    while (try_issue()) {
+    }
+    if (merge_pending) {
+      merge_pending = false;
+      merge_item();
+    }
+    if (consumed == issued) break;
     const uint32_t g = consumed;
     const uint32_t slot = g % kSlots;
     const bool arrived = mbar_wait(&bars[slot], (g / kSlots) & 1);
     if (!__all_sync(0xffffffffu, arrived)) {  // give up together, never half a warp
       for (uint32_t r = g + 1; r < issued; ++r) mbar_wait(&bars[r % kSlots], (r / kSlots) & 1);
       if (lane == 0) set_status(a.ctrl, TRR_ERR_TIMEOUT);
-      return;
+      break;
     }
     const int4 r0 = *reinterpret_cast<const int4*>(recs + slot);
     const int meta = r0.x, flags = meta >> 10;
-    if (flags & 1) {  // first page of an item: query row, key range and a fresh state
-      c_lo = r0.w;
-      c_hi = reinterpret_cast<const int*>(recs + slot)[4];
+    if (flags & 1) {  // first page of an item: query row and a fresh state
       const int qoff = r0.y + ((flags & 4) ? 0 : a.slice[meta & 3] + ((meta & 512) ? 4 * a.P : 0));
       const uint4* q4 = reinterpret_cast<const uint4*>(ring + qoff + part * 64);
       sumq = 0.f;
@@ -657,6 +732,7 @@ __global__ void __launch_bounds__(256, 2) attn_kernel(const AttnKernelArgs ka) {
       }
       const uint8_t* sl = ring + r0.y;
       const int* sp = (meta & 512) ? reinterpret_cast<const int*>(ring + r0.y + a.slice[cls]) : nullptr;
+      const int c_lo = r0.w, c_hi = reinterpret_cast<const int*>(recs + slot)[4];  // key range
       switch (cls) {
         case 0: consume_page<D, 2>(sl, sp, a.P, a.G, fill, c_lo, c_hi, qp, sumq, st, lane); break;
         case 1: consume_page<D, 4>(sl, sp, a.P, a.G, fill, c_lo, c_hi, qp, sumq, st, lane); break;
@@ -664,101 +740,33 @@ __global__ void __launch_bounds__(256, 2) attn_kernel(const AttnKernelArgs ka) {
         default: consume_page<D, 16>(sl, sp, a.P, a.G, fill, c_lo, c_hi, qp, sumq, st, lane); break;
       }
     }
-    __syncwarp();
-    used -= r0.z;  // release the slot's ring bytes, refill
-    consumed = g + 1;
-    while (try_issue()) {
-    }
-    if (!(flags & 2)) continue;
-
-    // ---- last page of the item: merge the lanes that share a part.  Rescale to the
-    // common maximum, then reduce-scatter over the key lanes: each halving step keeps
-    // half of the 32 dims and sends the other half to the partner lane.
-    const int4 r1 = *reinterpret_cast<const int4*>(reinterpret_cast<const int*>(recs + slot) + 4);
-    const int item = r1.y, qi = r1.z, qh = r1.w;
-    const int nsplit = reinterpret_cast<const int*>(recs + slot)[8];
-    acc_to_neutral(st.acc, cur_cls);
-    float M = st.m;
-#pragma unroll
-    for (int o = LPK; o < 32; o <<= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-    const float f = (st.m == kNegInf) ? 0.f : fast_exp2(st.m - M);
-    float L = st.l * f;
-#pragma unroll
-    for (int o = LPK; o < 32; o <<= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
-#pragma unroll
-    for (int j = 0; j < 32; ++j) st.acc[j] = fmaf(st.acc[j], pow2f(49), st.zacc) * f;
-#pragma unroll
-    for (int width = 16, o = 16; o >= LPK; width >>= 1, o >>= 1) {
-      const bool upper = lane & o;
-#pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        if (i < width) {
-          const float keep = upper ? st.acc[width + i] : st.acc[i];
-          const float give = upper ? st.acc[i] : st.acc[width + i];
-          st.acc[i] = keep + __shfl_xor_sync(0xffffffffu, give, o);
-        }
+    if (flags & 2) {  // last page of the item: its merge follows the refill
+      if (lane == 0) {
+        const int* rw = reinterpret_cast<const int*>(recs + slot);
+        reinterpret_cast<int4*>(wmerge)[0] = make_int4(rw[5], rw[6], rw[7], rw[8]);
+        wmerge[4] = rw[9];
       }
+      merge_pending = true;
     }
-    // lane (kl, part) now holds dims part*32 + DPL*kl .. + DPL-1 in acc[0 .. DPL-1]
-    const int dim0 = part * 32 + DPL * kl;
-    if (nsplit == 1) {
-      const int64_t orow = (static_cast<int64_t>(qi) * a.Hq + qh) * D;
-      const float inv = L > 0.f ? 1.f / L : 0.f;
-#pragma unroll
-      for (int j = 0; j < DPL; j += 2)
-        *reinterpret_cast<__nv_bfloat162*>(ka.out + orow + dim0 + j) =
-            __floats2bfloat162_rn(st.acc[j] * inv, st.acc[j + 1] * inv);
-    } else {  // a partial at the item's index; attn_combine_kernel merges the splits
-      float* pp = a.part + static_cast<int64_t>(item) * (D + 4);
-#pragma unroll
-      for (int j = 0; j < DPL; j += 2)
-        *reinterpret_cast<float2*>(pp + dim0 + j) = make_float2(st.acc[j], st.acc[j + 1]);
-      if (lane == 0) *reinterpret_cast<float2*>(pp + D) = make_float2(M, L);
+    __syncwarp();
+    used -= r0.z;  // release the slot's ring bytes (the record is read)
+    consumed = g + 1;
+  }
+
+  // The last CTA to finish records the error of the lowest failing query.
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    __threadfence();
+    if (atomicAdd(&a.ctrl[kDoneCtas], 1) == static_cast<int>(gridDim.x) - 1) {
+      __threadfence();
+      const int bad = atomicExch(&a.ctrl[kFirstBadQuery], INT_MAX);
+      if (bad != INT_MAX) set_status(a.ctrl, bad & 15);
+      atomicExch(&a.ctrl[kDoneCtas], 0);
     }
   }
 }
 
-// One warp per (query, query head) with several splits: merge the fp32 partials of
-// splits 0..nsplit-1 (items (base + s) * units + head) into the bf16 row.  Block 0 also
-// resets the descriptor counter for the next call.
-template <int D>
-__global__ void __launch_bounds__(256) attn_combine_kernel(LayerArgs a, int n, uint16_t* __restrict__ out) {
-  constexpr int DPL = D / 32;
-  pdl_wait();
-  pdl_trigger();
-  if (blockIdx.x == 0 && threadIdx.x == 0) a.ctrl[kDescCounter] = 0;
-  const int lane = threadIdx.x & 31;
-  const int w = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-  if (w >= n * a.units) return;
-  const int qi = w / a.units, qh = w - qi * a.units;
-  const int nsplit = a.qplan[qi].nsplit, base = a.qplan[qi].base;
-  if (nsplit <= 1) return;
-  float Mx = kNegInf;
-  for (int s = lane; s < nsplit; s += 32)
-    Mx = fmaxf(Mx, a.part[(static_cast<int64_t>(base + s) * a.units + qh) * (D + 4) + D]);
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) Mx = fmaxf(Mx, __shfl_xor_sync(0xffffffffu, Mx, o));
-  float Ls = 0.f, o[DPL];
-#pragma unroll
-  for (int j = 0; j < DPL; ++j) o[j] = 0.f;
-#pragma unroll 4
-  for (int s = 0; s < nsplit; ++s) {
-    const float* ps = a.part + (static_cast<int64_t>(base + s) * a.units + qh) * (D + 4);
-    const float2 ml = *reinterpret_cast<const float2*>(ps + D);
-    const float wgt = (ml.x == kNegInf) ? 0.f : exp2f(ml.x - Mx);
-    Ls = fmaf(wgt, ml.y, Ls);
-#pragma unroll
-    for (int j = 0; j < DPL; ++j) o[j] = fmaf(wgt, ps[lane * DPL + j], o[j]);
-  }
-  const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
-  const int64_t orow = (static_cast<int64_t>(qi) * a.Hq + qh) * D;
-#pragma unroll
-  for (int j = 0; j < DPL; j += 2)
-    *reinterpret_cast<__nv_bfloat162*>(out + orow + lane * DPL + j) =
-        __floats2bfloat162_rn(o[j] * inv, o[j + 1] * inv);
-}
-
-constexpr int kAttnSmemLimit = 110 * 1024;  // dynamic shared memory of one attention CTA
+constexpr int kAttnSmemLimit = 113 * 1024;  // dynamic shared memory of one attention CTA
 
 // Done once per cache at creation, so that calls stay legal inside stream capture.
 cudaError_t attn_configure() {
@@ -768,40 +776,38 @@ cudaError_t attn_configure() {
   return e;
 }
 
-// The three launches of one attention call (plan, attention, combine) with the given
-// scratch views in `a`.
+// The one launch of an attention call with the given scratch views in `a`.
 static cudaError_t launch_attention(const Layout& l, const LayerArgs& a, int num_sms, int n,
                                     const int32_t* seq_ids, const int32_t* q_positions, const void* q_bf16,
                                     const uint8_t* modes, const int32_t* windows, int window_scalar,
-                                    float softmax_scale, void* out_bf16, int64_t max_desc, cudaStream_t s) {
-  cudaError_t e = launch_pdl(attn_plan_kernel, dim3((n + 7) / 8), dim3(256), 0, s, a, n, seq_ids, q_positions,
-                             modes, windows, window_scalar, static_cast<uint16_t*>(out_bf16));
-  if (e != cudaSuccess) return e;
+                                    float softmax_scale, void* out_bf16, cudaStream_t s) {
   AttnKernelArgs ka;
   ka.a = a;
+  ka.n = n;
+  ka.seq_ids = seq_ids;
+  ka.q_positions = q_positions;
+  ka.modes = modes;
+  ka.windows = windows;
+  ka.window_scalar = window_scalar;
   ka.q = static_cast<const uint16_t*>(q_bf16);
   ka.out = static_cast<uint16_t*>(out_bf16);
   const float scale = softmax_scale > 0.f ? softmax_scale : 1.f / sqrtf(static_cast<float>(l.d));
   ka.qscale = scale * 1.4426950408889634f;
-  // a ring holds at least one page of the widest class with its positions and a query row
-  const int widest = static_cast<int>(l.slice[3]) + 4 * l.P + 2 * l.d;
-  ka.ring_bytes = std::max(12 * 1024, (widest + 127) / 128 * 128);
-  ka.max_desc = static_cast<int>(std::min<int64_t>(max_desc, INT_MAX));
-  int nwarps = 8;
-  while (nwarps > 0 && AttnSmem(nwarps, ka.ring_bytes).total > kAttnSmemLimit) --nwarps;
+  // a ring holds at least one page of the widest class with its positions and a query
+  // row; up to 12 KB when shared memory allows
+  const int widest = (static_cast<int>(l.slice[3]) + 4 * l.P + 2 * l.d + 127) / 128 * 128;
+  int nwarps = 8, ring = 0;
+  for (; nwarps > 0; --nwarps) {
+    const int fixed = AttnSmem(nwarps, 0, n).total;
+    ring = std::min(std::max(12 * 1024, widest), (kAttnSmemLimit - fixed) / nwarps / 128 * 128);
+    if (ring >= widest) break;
+  }
   if (nwarps < 1) return cudaErrorInvalidConfiguration;
-  const int smem = AttnSmem(nwarps, ka.ring_bytes).total;
+  ka.ring_bytes = ring;
+  const int smem = AttnSmem(nwarps, ring, n).total;
   if (l.d == 64)
-    e = launch_pdl(attn_kernel<64>, dim3(2 * num_sms), dim3(nwarps * 32), static_cast<size_t>(smem), s, ka);
-  else
-    e = launch_pdl(attn_kernel<128>, dim3(2 * num_sms), dim3(nwarps * 32), static_cast<size_t>(smem), s, ka);
-  if (e != cudaSuccess) return e;
-  const int cw = n * l.units;
-  if (l.d == 64)
-    e = launch_pdl(attn_combine_kernel<64>, dim3((cw + 7) / 8), dim3(256), 0, s, a, n, static_cast<uint16_t*>(out_bf16));
-  else
-    e = launch_pdl(attn_combine_kernel<128>, dim3((cw + 7) / 8), dim3(256), 0, s, a, n, static_cast<uint16_t*>(out_bf16));
-  return e;
+    return launch_pdl(attn_kernel<64>, dim3(2 * num_sms), dim3(nwarps * 32), static_cast<size_t>(smem), s, ka);
+  return launch_pdl(attn_kernel<128>, dim3(2 * num_sms), dim3(nwarps * 32), static_cast<size_t>(smem), s, ka);
 }
 
 }  // namespace trr
@@ -823,18 +829,17 @@ extern "C" trr_status trr_decode_attn(trr_cache* cache, int32_t layer, int32_t n
   const LayerArgs a = layer_args(l, cache_views(cache), layer);
   const cudaError_t e = launch_attention(l, a, cache_num_sms(cache), n, seq_ids, q_positions, q_bf16, modes,
                                          windows, window_scalar, softmax_scale, out_bf16,
-                                         static_cast<int64_t>(l.max_queries) * l.s_cap,
                                          static_cast<cudaStream_t>(stream));
-  cache_set_launches(cache, 3);
+  cache_set_launches(cache, 1);
   return e == cudaSuccess ? TRR_OK : TRR_ERR_CUDA;
 }
 
 // ------------------------------------------------------ static-scratch variant --
 //
-// trr_decode_attn_static runs the same two kernels as trr_decode_attn, but keeps all
-// of its per-call scratch (query plans, split descriptors, arrival counters, fp32
-// partials and the call's control words) in one file-scope device array instead of
-// the cache's scratch region.  Nothing is allocated per call or at set-up.
+// trr_decode_attn_static runs the same kernel as trr_decode_attn, but keeps all of its
+// per-call scratch (arrival counters, fp32 partials and the call's control words) in one
+// file-scope device array instead of the cache's scratch region.  Nothing is allocated
+// per call or at set-up.
 namespace trr {
 
 constexpr int64_t kStaticScratchBytes = 32ll << 20;  // 32 MiB on every device using the library
@@ -888,32 +893,27 @@ extern "C" trr_status trr_decode_attn_static(trr_cache* cache, int32_t layer, in
     return TRR_ERR_INVALID_ARG;
   // scratch of this call, carved from the static array; reject what does not fit
   auto up = [](int64_t x) { return (x + 255) / 256 * 256; };
-  const int64_t nd = static_cast<int64_t>(n) * l.s_cap;  // most split descriptors
   const int64_t b_ctrl = up(4 * kCtrlInts);
-  const int64_t b_qplan = up(static_cast<int64_t>(sizeof(QueryPlan)) * n);
-  const int64_t b_desc = up(static_cast<int64_t>(sizeof(SplitDesc)) * nd);
   const int64_t b_cnt = up(4ll * n * l.units);
-  const int64_t b_part = up(4ll * nd * l.units * (l.d + 4));
-  if (b_ctrl + b_qplan + b_desc + b_cnt + b_part > kStaticScratchBytes) return TRR_ERR_OUT_OF_MEMORY;
+  const int64_t b_part = up(4ll * n * l.s_cap * l.units * (l.d + 4));
+  if (b_ctrl + b_cnt + b_part > kStaticScratchBytes) return TRR_ERR_OUT_OF_MEMORY;
   void* base = nullptr;
   if (static_scratch(&base) != cudaSuccess) return TRR_ERR_CUDA;
   uint8_t* b = static_cast<uint8_t*>(base);
   LayerArgs a = layer_args(l, cache_views(cache), layer);
   int32_t* cache_ctrl = a.ctrl;
   a.ctrl = reinterpret_cast<int32_t*>(b);
-  a.qplan = reinterpret_cast<QueryPlan*>(b + b_ctrl);
-  a.desc = reinterpret_cast<SplitDesc*>(b + b_ctrl + b_qplan);
-  a.cnt = reinterpret_cast<int32_t*>(b + b_ctrl + b_qplan + b_desc);
-  a.part = reinterpret_cast<float*>(b + b_ctrl + b_qplan + b_desc + b_cnt);
+  a.cnt = reinterpret_cast<int32_t*>(b + b_ctrl);
+  a.part = reinterpret_cast<float*>(b + b_ctrl + b_cnt);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const int ncnt = n * l.units;
   static_scratch_clear_kernel<<<std::max(1, std::min(256, (ncnt + 255) / 256)), 256, 0, s>>>(a.ctrl, a.cnt, ncnt);
   cudaError_t e = cudaGetLastError();
   if (e == cudaSuccess)
     e = launch_attention(l, a, cache_num_sms(cache), n, seq_ids, q_positions, q_bf16, modes, windows,
-                         window_scalar, softmax_scale, out_bf16, nd, s);
+                         window_scalar, softmax_scale, out_bf16, s);
   if (e != cudaSuccess) return TRR_ERR_CUDA;
   static_scratch_status_kernel<<<1, 1, 0, s>>>(a.ctrl, cache_ctrl);
-  cache_set_launches(cache, 5);
+  cache_set_launches(cache, 3);
   return cudaGetLastError() == cudaSuccess ? TRR_OK : TRR_ERR_CUDA;
 }

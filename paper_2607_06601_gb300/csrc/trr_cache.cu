@@ -17,7 +17,8 @@ LayerArgs layer_args(const Layout& l, const Views& v, int layer) {
   LayerArgs a;
   a.layer = layer;
   a.S = l.S; a.Hq = l.Hq; a.Hkv = l.Hkv; a.d = l.d; a.G = l.G; a.P = l.P;
-  a.maxctx = l.maxctx; a.MP = l.MP; a.W32 = l.W32; a.units = l.units; a.s_cap = l.s_cap;
+  a.maxctx = l.maxctx; a.MP = l.MP; a.W32 = l.W32; a.units = l.units; a.pos_split = l.pos_split;
+  a.s_cap = l.s_cap;
   a.split_bytes = l.split_bytes; a.skip_writes_kv = l.skip_writes_kv;
   a.hdr = static_cast<int>(l.hdr);
   for (int c = 0; c < kClasses; ++c) {
@@ -35,8 +36,6 @@ LayerArgs layer_args(const Layout& l, const Views& v, int layer) {
   a.pfirst = v.pfirst + ls * 4 * l.MP;
   a.plast = v.plast + ls * 4 * l.MP;
   a.aplan = v.aplan;
-  a.qplan = v.qplan;
-  a.desc = v.desc;
   a.cnt = v.cnt;
   a.part = v.part;
   return a;
@@ -79,12 +78,11 @@ static trr_status make_layout(const trr_cache_config* c, Layout* l) {
     l->page_bytes[k] = roundup(l->hdr + l->Hkv * l->slice[k], 128);
   }
   l->units = l->Hq;
-  // splits per query: enough for split_bytes each even if every token were bf16, and
-  // enough to keep each split within kDescMaxPages pages (+ one partial page per class)
-  const int64_t most = static_cast<int64_t>(l->maxctx) * l->tokb[3];
-  const int64_t by_bytes = (most + l->split_bytes - 1) / l->split_bytes;
-  const int64_t by_pages = (l->MP + kClasses + kDescMaxPages - 1) / kDescMaxPages;
-  l->s_cap = static_cast<int>(std::max<int64_t>(1, std::max(by_bytes, by_pages)));
+  // splits per query: at least pos_split key positions each (split_bytes of 8-bit
+  // tokens), and few enough pages per split for any range up to max_context
+  l->pos_split = static_cast<int>(std::max<int64_t>(l->P, l->split_bytes / l->tokb[2]));
+  l->s_cap = 1 << 30;
+  l->s_cap = std::max(splits_of(l->maxctx, l->pos_split, l->P, l->s_cap), 1);
   l->max_items = static_cast<int64_t>(l->max_queries) * l->units * l->s_cap;
 
   const int64_t nls = static_cast<int64_t>(l->L) * l->S;
@@ -102,8 +100,6 @@ static trr_status make_layout(const trr_cache_config* c, Layout* l) {
   l->off_pfirst = take(16 * nls * l->MP);
   l->off_plast = take(16 * nls * l->MP);
   l->off_aplan = take(static_cast<int64_t>(sizeof(AppendPlan)) * l->max_append);
-  l->off_qplan = take(static_cast<int64_t>(sizeof(QueryPlan)) * l->max_queries);
-  l->off_desc = take(static_cast<int64_t>(sizeof(SplitDesc)) * l->max_queries * l->s_cap);
   l->off_cnt = take(4 * static_cast<int64_t>(l->max_queries) * l->units);
   l->off_part = take(4 * l->max_items * (l->Hq / l->units) * (l->d + 4));
   for (int k = 0; k < kClasses; ++k) l->off_pool[k] = take(l->cap[k] * l->page_bytes[k]);

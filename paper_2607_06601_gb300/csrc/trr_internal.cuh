@@ -18,49 +18,41 @@ __host__ __device__ constexpr int bits_of_class(int c) { return c == 0 ? 2 : c =
 enum Ctrl : int {
   kStatus = 0,        // sticky first error since the last trr_get_status
   kNextPage = 4,      // [4] pages handed out per class
-  kWorkCounter = 8,   // attention: next work item to hand out
   kAppendOk = 10,     // append: 1 when the plan kernel committed the call
-  kFirstBadQuery = 12,// attention: lowest failing query index (INT_MAX = none)
-  kDescCounter = 13,  // attention: split descriptors handed out by the plan kernel
-  kDoneWarps = 14,    // attention: warps finished (the last one resets the two counters)
+  kFirstBadQuery = 12,// attention: min of (query index * 16 + error) over failing queries
+                      // (INT_MAX = none)
+  kDoneCtas = 14,     // attention: CTAs finished (the last one records the status)
   kCtrlInts = 64
 };
+
+// Splits of one attention work unit are sized to hold at most this many pages (+ one
+// partial page per class), so that a warp holds an item's page ids one per lane.
+constexpr int kItemMaxPages = 28;
 
 // Byte layout of one cache (see include/trr.h for the documented part).
 struct Layout {
   int L, S, Hq, Hkv, d, G, P, maxctx, MP, W32;
   int cap[kClasses];
   int max_append, max_queries, split_bytes, skip_writes_kv;
-  int units;      // attention work units per query (one per query head)
-  int s_cap;      // most splits one (query, unit) is cut into
+  int units;      // attention work units per query split (one per query head)
+  int pos_split;  // key positions per split at least (split_bytes of 8-bit tokens)
+  int s_cap;      // most splits one query is cut into
   int64_t max_items;
   int64_t hdr, tokb[kClasses], slice[kClasses], page_bytes[kClasses];
   int64_t off_ctrl, off_last_pos, off_ntok, off_presence, off_pt, off_pfirst, off_plast;
-  int64_t off_aplan, off_qplan, off_desc, off_cnt, off_part, off_pool[kClasses], total;
+  int64_t off_aplan, off_cnt, off_part, off_pool[kClasses], total;
 };
 
-// Per-query plan written by the attention plan kernel.
-struct QueryPlan {
-  int seq, lo, hi, nsplit;      // key range [lo, hi]; nsplit = 0: nothing to do
-  int first[kClasses];          // first page (index in the class page list) in range
-  int npages[kClasses];         // pages in range
-  int ntok[kClasses];           // tokens of the class stored for the sequence
-  int err, base, pad1, pad2;    // base: descriptor index of split 0
-};
-static_assert(sizeof(QueryPlan) == 80, "QueryPlan is 80 bytes");
-
-// One split-K work unit of one query, written by the attention plan kernel: the ids
-// of its pages (at most kDescPages, in class-then-position order), each page's width
-// class and token count, and the query's key range.  Laid out so that a warp loads it
-// with three coalesced words per lane.
-constexpr int kDescPages = 32;
-constexpr int kDescMaxPages = 28;  // splits are sized to hold at most this many pages, + 4
-struct SplitDesc {
-  int page[kDescPages];
-  int meta[kDescPages];  // class | fill << 2 | (slot positions needed) << 9
-  int qi, seq, lo, hi, nsplit, split, T, base;  // base: descriptor index of split 0
-};
-static_assert(sizeof(SplitDesc) == 288, "SplitDesc is 288 bytes");
+// Splits of a query whose key range spans `range` positions: at least pos_split
+// positions each, enough that no split holds more than kItemMaxPages + 4 pages, at most
+// s_cap (which covers the page bound for any range up to max_context).
+__host__ __device__ inline int splits_of(int range, int pos_split, int P, int s_cap) {
+  if (range <= 0) return 1;
+  const int by_len = (range + pos_split - 1) / pos_split;
+  const int by_pages = ((range + P - 1) / P + 2 * kClasses + kItemMaxPages - 1) / kItemMaxPages;
+  const int ns = by_len > by_pages ? by_len : by_pages;
+  return ns < s_cap ? ns : s_cap;
+}
 
 // Per-entry plan written by the append plan kernel.
 struct AppendPlan {
@@ -79,8 +71,6 @@ struct Views {  // typed device pointers into the cache memory
   int32_t* pfirst;
   int32_t* plast;
   AppendPlan* aplan;
-  QueryPlan* qplan;
-  SplitDesc* desc;
   int32_t* cnt;
   float* part;
   uint8_t* pool[kClasses];
@@ -97,8 +87,6 @@ inline Views make_views(const Layout& l, void* base) {
   v.pfirst = reinterpret_cast<int32_t*>(b + l.off_pfirst);
   v.plast = reinterpret_cast<int32_t*>(b + l.off_plast);
   v.aplan = reinterpret_cast<AppendPlan*>(b + l.off_aplan);
-  v.qplan = reinterpret_cast<QueryPlan*>(b + l.off_qplan);
-  v.desc = reinterpret_cast<SplitDesc*>(b + l.off_desc);
   v.cnt = reinterpret_cast<int32_t*>(b + l.off_cnt);
   v.part = reinterpret_cast<float*>(b + l.off_part);
   for (int c = 0; c < kClasses; ++c) v.pool[c] = b + l.off_pool[c];
@@ -107,7 +95,7 @@ inline Views make_views(const Layout& l, void* base) {
 
 // Everything a kernel needs about one layer of one cache, passed by value.
 struct LayerArgs {
-  int layer, S, Hq, Hkv, d, G, P, maxctx, MP, W32, units, s_cap, split_bytes, skip_writes_kv;
+  int layer, S, Hq, Hkv, d, G, P, maxctx, MP, W32, units, pos_split, s_cap, split_bytes, skip_writes_kv;
   int cap[kClasses];
   int hdr;
   int slice[kClasses];
@@ -120,10 +108,8 @@ struct LayerArgs {
   int32_t* pfirst;
   int32_t* plast;
   AppendPlan* aplan;
-  QueryPlan* qplan;
-  SplitDesc* desc;     // [max_queries][s_cap]
-  int32_t* cnt;
-  float* part;
+  int32_t* cnt;        // [max_queries][Hq] split arrivals (zero between calls)
+  float* part;         // [max_queries * s_cap * Hq][d + 4] fp32 partials: acc, M, L
   uint8_t* pool[kClasses];
 };
 
