@@ -1,6 +1,7 @@
 // trr_append.cu - trr_kv_append: quantise-on-write into the width-class page pools.
 //
-// Two kernels per call:
+// Calls of up to 256 entries (decode steps) run as one kernel, append_fused_kernel
+// (below); larger ones as two:
 //   append_plan_kernel   one CTA, one thread per entry.  Validates every entry, ranks
 //                        it among the earlier entries of its (sequence, class), hands
 //                        out page ids in entry order, and commits the metadata only
@@ -130,13 +131,14 @@ __device__ __forceinline__ float bf16lo(uint32_t w) { return __uint_as_float(w <
 __device__ __forceinline__ float bf16hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 
 // round((x - z) / s) of Eq. 4 on the exact quotient, ties to even, clamped to [0, levels].
-// u = fl32(fl32(x - z) / s) is within 2^-22 |u| of the exact quotient (two binary32
-// roundings), so rint(u) is exact unless u lies that close to a half-way point c + 1/2.
-// There the midpoint z + (c + 1/2) s is formed in binary64, where it is exact (z and s
-// are binary16: a multiple of 2^-25 below 2^18), and compared with x (a bf16 value).
-// Only half-way points inside [0, levels] matter: the clamp settles the others.
-__device__ __forceinline__ int code_of(float x, float z, float s, int levels) {
-  const float u = __fdiv_rn(__fsub_rn(x, z), s);
+// u = fl32(fl32(x - z) * rs) with rs = fl32(1 / s) is within 3 binary32 roundings, under
+// 2^-21 |u|, of the exact quotient, so rint(u) is exact unless u lies that close to a
+// half-way point c + 1/2.  There the midpoint z + (c + 1/2) s is formed in binary64,
+// where it is exact (z and s are binary16: a multiple of 2^-25 below 2^18), and compared
+// with x (a bf16 value).  Only half-way points inside [0, levels] matter: the clamp
+// settles the others.
+__device__ __forceinline__ int code_of(float x, float z, float s, float rs, int levels) {
+  const float u = __fmul_rn(__fsub_rn(x, z), rs);
   const float fl = floorf(u);
   if (fabsf(__fsub_rn(u, fl + 0.5f)) <= fabsf(u) * 0x1p-21f && fl >= 0.f && fl < static_cast<float>(levels)) {
     const double mid = __dadd_rn(static_cast<double>(z), __dmul_rn(static_cast<double>(fl) + 0.5, static_cast<double>(s)));
@@ -149,7 +151,7 @@ __device__ __forceinline__ int code_of(float x, float z, float s, int levels) {
 
 // Eq. 4 on 32 consecutive values (one chunk of a group): codes packed LSB-first.
 template <int B>
-__device__ __forceinline__ void quantise_chunk(const uint4* src, float z, float s, uint32_t* dst) {
+__device__ __forceinline__ void quantise_chunk(const uint4* src, float z, float s, float rs, uint32_t* dst) {
   constexpr int levels = (1 << B) - 1;
   constexpr int per_word = 32 / B;
   uint32_t words[B];
@@ -162,7 +164,7 @@ __device__ __forceinline__ void quantise_chunk(const uint4* src, float z, float 
 #pragma unroll
     for (int h = 0; h < 8; ++h) {
       const float x = (h & 1) ? bf16hi(wv[h >> 1]) : bf16lo(wv[h >> 1]);
-      const int code = s != 0.f ? code_of(x, z, s, levels) : 0;
+      const int code = s != 0.f ? code_of(x, z, s, rs, levels) : 0;
       const int j = q * 8 + h;
       words[j / per_word] |= static_cast<uint32_t>(code) << ((j % per_word) * B);
     }
@@ -226,14 +228,237 @@ __global__ void __launch_bounds__(256) append_write_kernel(LayerArgs a, int n, c
   const __half z16 = __float2half_rn(mn);                                   // z = min(x)
   const float levels = static_cast<float>((1 << b) - 1);
   const __half s16 = __float2half_rn(__fdiv_rn(__fsub_rn(mx, mn), levels));  // s
-  const float z = __half2float(z16), s = __half2float(s16);
+  const float z = __half2float(z16), s = __half2float(s16), rs = __frcp_rn(s);
   for (int q = 0; q < a.G / 32; ++q) {
     uint32_t* dst = codes + q * b;  // 32 codes of b bits = b words
-    if (b == 2) quantise_chunk<2>(s4 + 4 * q, z, s, dst);
-    else if (b == 4) quantise_chunk<4>(s4 + 4 * q, z, s, dst);
-    else quantise_chunk<8>(s4 + 4 * q, z, s, dst);
+    if (b == 2) quantise_chunk<2>(s4 + 4 * q, z, s, rs, dst);
+    else if (b == 4) quantise_chunk<4>(s4 + 4 * q, z, s, rs, dst);
+    else quantise_chunk<8>(s4 + 4 * q, z, s, rs, dst);
   }
   *sz = static_cast<uint32_t>(__half_as_ushort(s16)) | (static_cast<uint32_t>(__half_as_ushort(z16)) << 16);
+}
+
+// ------------------------------------------------------------ one-kernel append --
+//
+// For calls of up to kFusedMax entries (a decode step) one kernel does the whole append.
+// Every CTA plans every entry (the same deterministic plan as append_plan_kernel, from
+// the metadata as the call found it), each warp quantises one (entry, KV head, K|V) row,
+// and the last CTA to finish commits the metadata: no CTA reads metadata after the
+// commit, since every other CTA has finished by then.
+
+constexpr int kFusedMax = 256;
+
+// One row of d values (entry, KV head, K or V) by a warp: lane l holds values
+// EPL*l .. EPL*l + EPL-1; a group's min / max by shuffles over its G/EPL lanes; codes
+// packed LSB-first and gathered into 32-bit words by OR over the lanes of each word.
+template <int D>
+__device__ __forceinline__ void quantise_row(const uint16_t* src, uint8_t* codes_row, uint32_t* sz_row, int b, int G,
+                                             int lane, int32_t* ctrl) {
+  constexpr int EPL = D / 32;
+  float x[EPL];
+  if (EPL == 2) {
+    const uint32_t w = reinterpret_cast<const uint32_t*>(src)[lane];
+    x[0] = bf16lo(w);
+    x[1] = bf16hi(w);
+  } else {
+    const uint2 w = reinterpret_cast<const uint2*>(src)[lane];
+    x[0] = bf16lo(w.x);
+    x[1] = bf16hi(w.x);
+    x[EPL > 2 ? 2 : 0] = bf16lo(w.y);
+    x[EPL > 3 ? 3 : 0] = bf16hi(w.y);
+  }
+  const int GL = G / EPL;  // lanes of one group
+  float mn = x[0], mx = x[0];
+  bool bad = false;
+#pragma unroll
+  for (int i = 0; i < EPL; ++i) {
+    bad |= !(fabsf(x[i]) <= 65504.f);  // also true for NaN
+    mn = fminf(mn, x[i]);
+    mx = fmaxf(mx, x[i]);
+  }
+  for (int o = 1; o < GL; o <<= 1) {
+    mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, o));
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    bad |= __shfl_xor_sync(0xffffffffu, static_cast<int>(bad), o) != 0;
+  }
+  const int levels = (1 << b) - 1;
+  uint32_t val = 0, szw = 0;
+  if (!bad) {
+    const __half z16 = __float2half_rn(mn);                                                    // z = min(x)
+    const __half s16 = __float2half_rn(__fdiv_rn(__fsub_rn(mx, mn), static_cast<float>(levels)));  // s
+    const float z = __half2float(z16), s = __half2float(s16), rs = __frcp_rn(s);
+#pragma unroll
+    for (int i = 0; i < EPL; ++i)
+      val |= static_cast<uint32_t>(s != 0.f ? code_of(x[i], z, s, rs, levels) : 0) << (i * b);
+    szw = static_cast<uint32_t>(__half_as_ushort(s16)) | (static_cast<uint32_t>(__half_as_ushort(z16)) << 16);
+  } else if (lane % GL == 0) {
+    set_status(ctrl, TRR_ERR_BAD_VALUE);
+  }
+  const int LPW = 32 / (EPL * b);  // lanes sharing one 32-bit word of codes
+  val <<= (lane % LPW) * EPL * b;
+  for (int o = 1; o < LPW; o <<= 1) val |= __shfl_xor_sync(0xffffffffu, val, o);
+  if (lane % LPW == 0) reinterpret_cast<uint32_t*>(codes_row)[lane / LPW] = val;
+  if (lane % GL == 0) sz_row[lane / GL] = szw;
+}
+
+template <int D>
+__global__ void __launch_bounds__(256) append_fused_kernel(LayerArgs a, int n, const int32_t* __restrict__ seq_ids,
+                                                           const int32_t* __restrict__ positions,
+                                                           const uint8_t* __restrict__ bits,
+                                                           const uint8_t* __restrict__ modes,
+                                                           const uint16_t* __restrict__ k,
+                                                           const uint16_t* __restrict__ v) {
+  __shared__ int s_seq[kFusedMax];
+  __shared__ int s_pos[kFusedMax];
+  __shared__ int s_cls[kFusedMax];   // width class when the entry stores KV, else -1
+  __shared__ int s_k[kFusedMax];     // token index in the (sequence, class) list
+  __shared__ int s_pid[kFusedMax];   // page of the token (openers: the new page)
+  __shared__ int s_wopen[8][kClasses];
+  __shared__ int s_next[kClasses];
+  __shared__ int s_first_err;
+  __shared__ int s_last;
+
+  pdl_wait();
+  pdl_trigger();
+  const int e = threadIdx.x, lane = e & 31, warp = e >> 5;
+  const bool act = e < n;
+  int seq = -1, pos = 0, c = -1, err = 0;
+  bool writes = false;
+  if (act) {
+    seq = seq_ids[e];
+    pos = positions[e];
+    const int m = modes[e];
+    if (seq < 0 || seq >= a.S) {
+      err = TRR_ERR_INVALID_ARG;
+    } else {
+      c = class_of_bits(bits[e]);
+      if (c < 0 || m > TRR_MODE_FULL) err = TRR_ERR_INVALID_ARG;
+      else if (pos < 0 || pos >= a.maxctx) err = TRR_ERR_BAD_POSITION;
+    }
+    writes = !err && (m != TRR_MODE_SKIP || a.skip_writes_kv);
+  }
+  s_seq[e] = (act && seq >= 0 && seq < a.S) ? seq : -1;
+  s_pos[e] = pos;
+  s_cls[e] = writes ? c : -1;
+  if (e < kClasses) s_next[e] = a.ctrl[kNextPage + e];
+  if (e == 0) s_first_err = INT_MAX;
+  __syncthreads();
+
+  // earlier entries of the same sequence: the largest position and, per class, how many
+  // store KV; later ones: whether this entry is the sequence's / class's last
+  int prev_max = -1, rank = 0;
+  bool later_seq = false, later_cls = false;
+  if (act && s_seq[e] >= 0) {
+    for (int j = 0; j < n; ++j) {
+      if (s_seq[j] != seq) continue;
+      if (j < e) {
+        prev_max = max(prev_max, s_pos[j]);
+        rank += (writes && s_cls[j] == c);
+      } else if (j > e) {
+        later_seq = true;
+        later_cls |= (writes && s_cls[j] == c);
+      }
+    }
+  }
+  int tok = 0, nt_old = 0;
+  bool opens = false;
+  if (act && !err) {
+    if (pos <= max(prev_max, a.last_pos[seq])) err = TRR_ERR_BAD_POSITION;
+    if (writes) {
+      nt_old = a.ntok[seq * 4 + c];
+      tok = nt_old + rank;
+      opens = tok % a.P == 0;
+    }
+  }
+  // page ids in entry order: next_page + openers of the same class before e
+  int before = 0;
+#pragma unroll
+  for (int cc = 0; cc < kClasses; ++cc) {
+    const unsigned bal = __ballot_sync(0xffffffffu, !err && opens && c == cc);
+    if (lane == 0) s_wopen[warp][cc] = __popc(bal);
+    if (c == cc) before = __popc(bal & ((1u << lane) - 1u));
+  }
+  __syncthreads();
+  int pid = -1;
+  if (opens) {
+    for (int w = 0; w < warp; ++w) before += s_wopen[w][c];
+    pid = s_next[c] + before;
+    if (pid >= a.cap[c]) err = TRR_ERR_OUT_OF_PAGES;
+  }
+  if (act && err) atomicMin(&s_first_err, e);
+  s_k[e] = tok;
+  s_pid[e] = pid;
+  __syncthreads();
+  if (s_first_err != INT_MAX) {  // the call is a no-op; record the lowest failing entry
+    if (blockIdx.x == 0 && e == s_first_err) set_status(a.ctrl, err);
+    return;
+  }
+  const int kidx = tok / a.P;
+  const int64_t prow = (static_cast<int64_t>(seq) * 4 + c) * a.MP + kidx;
+  if (writes && !opens) {  // a page opened earlier: by a previous call, or by this one
+    if (kidx * a.P < nt_old) {
+      pid = a.pt[prow];
+    } else {
+      for (int j = 0; j < e; ++j)
+        if (s_seq[j] == seq && s_cls[j] == c && s_k[j] == kidx * a.P) pid = s_pid[j];
+    }
+    s_pid[e] = pid;
+  }
+  __syncthreads();
+
+  // this warp's row: (entry, KV head, K|V)
+  const int row = blockIdx.x * (blockDim.x >> 5) + warp;
+  if (row < n * a.Hkv * 2) {
+    const int re = row / (2 * a.Hkv), h = (row >> 1) % a.Hkv, which = row & 1;
+    const int rc = s_cls[re];
+    if (rc >= 0) {
+      const int b = bits_of_class(rc), slot = s_k[re] % a.P;
+      const uint16_t* src = (which ? v : k) + (static_cast<int64_t>(re) * a.Hkv + h) * D;
+      uint8_t* sl = a.pool[rc] + static_cast<int64_t>(s_pid[re]) * a.page_bytes[rc] + a.hdr +
+                    static_cast<int64_t>(h) * a.slice[rc];
+      if (b == 16) {
+        uint32_t* dst = reinterpret_cast<uint32_t*>(sl + (static_cast<int64_t>(which) * a.P + slot) * D * 2);
+        if (D == 64) dst[lane] = reinterpret_cast<const uint32_t*>(src)[lane];
+        else reinterpret_cast<uint2*>(dst)[lane] = reinterpret_cast<const uint2*>(src)[lane];
+      } else {
+        const int rowb = D * b / 8, ng = D / a.G;
+        uint8_t* codes_row = sl + (static_cast<int64_t>(which) * a.P + slot) * rowb;
+        uint32_t* sz_row = reinterpret_cast<uint32_t*>(sl + 2 * static_cast<int64_t>(a.P) * rowb +
+                                                      (static_cast<int64_t>(which) * a.P + slot) * ng * 4);
+        quantise_row<D>(src, codes_row, sz_row, b, a.G, lane, a.ctrl);
+      }
+    }
+  }
+
+  // the last CTA to finish commits the metadata of every entry
+  __syncthreads();
+  if (e == 0) {
+    __threadfence();
+    s_last = atomicAdd(&a.ctrl[kAppendDone], 1) == static_cast<int>(gridDim.x) - 1;
+  }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  if (act) {
+    if (writes) {
+      const int slot = tok % a.P;
+      if (opens) {
+        a.pt[prow] = pid;
+        a.pfirst[prow] = pos;
+      }
+      if (!later_cls || slot == a.P - 1) a.plast[prow] = pos;
+      if (!later_cls) a.ntok[seq * 4 + c] = tok + 1;
+      reinterpret_cast<int32_t*>(a.pool[c] + static_cast<int64_t>(pid) * a.page_bytes[c])[slot] = pos;
+      atomicOr(&a.presence[static_cast<int64_t>(seq) * a.W32 + pos / 32], 1u << (pos % 32));
+    }
+    if (!later_seq) a.last_pos[seq] = pos;
+  }
+  if (e < kClasses) {
+    int opened = 0;
+    for (int w = 0; w < 8; ++w) opened += s_wopen[w][e];
+    a.ctrl[kNextPage + e] = s_next[e] + opened;
+  }
+  if (e == 0) a.ctrl[kAppendDone] = 0;
 }
 
 }  // namespace trr
@@ -253,6 +478,16 @@ extern "C" trr_status trr_kv_append(trr_cache* cache, int32_t layer, int32_t n, 
     return TRR_ERR_INVALID_ARG;  // rows are read 16 bytes at a time
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const LayerArgs a = layer_args(l, cache_views(cache), layer);
+  if (n <= kFusedMax) {  // one kernel: 256 threads plan, one warp per (entry, head, K|V) row
+    const unsigned blocks = static_cast<unsigned>((static_cast<int64_t>(n) * l.Hkv * 2 + 7) / 8);
+    const cudaError_t e =
+        l.d == 64 ? launch_pdl(append_fused_kernel<64>, dim3(blocks), dim3(256), 0, s, a, n, seq_ids, positions, bits,
+                               modes, static_cast<const uint16_t*>(k_bf16), static_cast<const uint16_t*>(v_bf16))
+                  : launch_pdl(append_fused_kernel<128>, dim3(blocks), dim3(256), 0, s, a, n, seq_ids, positions,
+                               bits, modes, static_cast<const uint16_t*>(k_bf16), static_cast<const uint16_t*>(v_bf16));
+    cache_set_launches(cache, 1);
+    return e == cudaSuccess ? TRR_OK : TRR_ERR_CUDA;
+  }
   const int threads = (n + 31) / 32 * 32;
   cudaError_t e = launch_pdl(append_plan_kernel, dim3(1), dim3(threads), 0, s, a, n, seq_ids, positions, bits, modes);
   if (e != cudaSuccess) return TRR_ERR_CUDA;

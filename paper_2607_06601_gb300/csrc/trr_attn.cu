@@ -188,6 +188,14 @@ __device__ __forceinline__ void acc_to_neutral(float (&acc)[32], int from) {
   }
 }
 
+// atomic add with release (of what this thread has seen written) and acquire (of what
+// the threads that released the same counter wrote) at GPU scope
+__device__ __forceinline__ int atom_add_acq_rel(int* p, int v) {
+  int old;
+  asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+  return old;
+}
+
 // 2^x with the hardware approximation (relative error about 2^-22; results below the
 // binary32 normal range flush to zero, far below a softmax sum's resolution).
 __device__ __forceinline__ float fast_exp2(float x) {
@@ -410,6 +418,14 @@ __device__ __forceinline__ int plan_next_item(const AttnKernelArgs& ka, const in
       end[c] = pages[c];
     }
     const int64_t row0 = static_cast<int64_t>(seq) * 4 * a.MP;
+    // a window's pages are almost always among the last 32 of each class: their ids are
+    // loaded together with the search's first probes
+    int tb[kClasses], ptail[kClasses];
+#pragma unroll
+    for (int c = 0; c < kClasses; ++c) {
+      tb[c] = max(0, pages[c] - 32);
+      ptail[c] = (lo > 0 && tb[c] + lane < pages[c]) ? a.pt[row0 + c * a.MP + tb[c] + lane] : -1;
+    }
     if (lo > 0) warp_count_below<kClasses>(a.plast + row0, a.MP, pages, lo, first, lane);
     if (upper_mask) warp_count_below<kClasses>(a.pfirst + row0, a.MP, pages, t + 1, end, lane);
     // this split's share of each class's pages in range, then one page per lane
@@ -425,13 +441,19 @@ __device__ __forceinline__ int plan_next_item(const AttnKernelArgs& ka, const in
     T = min(T, kItemMaxPages + kClasses);  // the split bound keeps T within this
     wid = -1;
     wmeta = 0;
+    const int t1 = tc[0], t2 = t1 + tc[1], t3 = t2 + tc[2];
+    const int c = (lane >= t1) + (lane >= t2) + (lane >= t3);
+    auto pick = [c](const int (&v)[kClasses]) { return c == 0 ? v[0] : c == 1 ? v[1] : c == 2 ? v[2] : v[3]; };
+    const int kid = pick(beg) + lane - (c == 0 ? 0 : c == 1 ? t1 : c == 2 ? t2 : t3);
+    int from_tail = -1;
+#pragma unroll
+    for (int cc = 0; cc < kClasses; ++cc) {
+      const int v = __shfl_sync(0xffffffffu, ptail[cc], (kid - tb[cc]) & 31);
+      if (c == cc && kid >= tb[cc]) from_tail = v;
+    }
     if (lane < T) {
-      const int t1 = tc[0], t2 = t1 + tc[1], t3 = t2 + tc[2];
-      const int c = (lane >= t1) + (lane >= t2) + (lane >= t3);
-      auto pick = [c](const int (&v)[kClasses]) { return c == 0 ? v[0] : c == 1 ? v[1] : c == 2 ? v[2] : v[3]; };
-      const int kid = pick(beg) + lane - (c == 0 ? 0 : c == 1 ? t1 : c == 2 ? t2 : t3);
       const int f = pick(first);
-      wid = a.pt[static_cast<int64_t>(seq * 4 + c) * a.MP + kid];
+      wid = from_tail >= 0 ? from_tail : a.pt[static_cast<int64_t>(seq * 4 + c) * a.MP + kid];
       const int fill = min(a.P, pick(nt) - kid * a.P);
       // slot positions are needed on a page that may hold keys outside [lo, t]
       const bool mask = (lo > 0 && kid == f) || (upper_mask && kid == f + pick(npr) - 1);
@@ -647,14 +669,15 @@ __global__ void __launch_bounds__(256, 2) attn_kernel(const __grid_constant__ At
     for (int j = 0; j < DPL; j += 2)
       *reinterpret_cast<float2*>(pp + dim0 + j) = make_float2(st.acc[j], st.acc[j + 1]);
     if (lane == 0) *reinterpret_cast<float2*>(pp + D) = make_float2(M, L);
-    __threadfence();
+    // the warp's partial stores happen before lane 0's release; the last arriver's
+    // acquire happens before its lanes read the other splits' partials
     __syncwarp();
     int arrivals = 0;
     int* counter = a.cnt + static_cast<int64_t>(m_qi) * a.Hq + m_qh;
-    if (lane == 0) arrivals = atomicAdd(counter, 1);
+    if (lane == 0) arrivals = atom_add_acq_rel(counter, 1);
+    __syncwarp();
     arrivals = __shfl_sync(0xffffffffu, arrivals, 0);
     if (arrivals != m_nsplit - 1) return;
-    __threadfence();
     const float* p0 = a.part + (static_cast<int64_t>(m_base) * a.Hq + m_qh) * (D + 4);
     const int64_t sstride = static_cast<int64_t>(a.Hq) * (D + 4);
     float Mx = kNegInf;

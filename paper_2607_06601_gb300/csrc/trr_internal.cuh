@@ -19,6 +19,7 @@ enum Ctrl : int {
   kStatus = 0,        // sticky first error since the last trr_get_status
   kNextPage = 4,      // [4] pages handed out per class
   kAppendOk = 10,     // append: 1 when the plan kernel committed the call
+  kAppendDone = 11,   // one-kernel append: CTAs finished (the last one commits)
   kFirstBadQuery = 12,// attention: min of (query index * 16 + error) over failing queries
                       // (INT_MAX = none)
   kDoneCtas = 14,     // attention: CTAs finished (the last one records the status)
