@@ -115,7 +115,10 @@ __global__ void __launch_bounds__(1024) append_plan_kernel(LayerArgs a, int n, c
       p.slot = slot;
       p.cls = c;
       if (!later_cls || slot == a.P - 1) a.plast[row] = pos;
-      if (!later_cls) a.ntok[seq * 4 + c] = k + 1;
+      if (!later_cls) {
+        a.ntok[seq * 4 + c] = k + 1;
+        a.lastpg[seq * 4 + c] = pid;
+      }
       reinterpret_cast<int32_t*>(a.pool[c] + pid * a.page_bytes[c])[slot] = pos;
       atomicOr(&a.presence[static_cast<int64_t>(seq) * a.W32 + pos / 32], 1u << (pos % 32));
     }
@@ -252,16 +255,14 @@ constexpr int kFusedMax = 256;
 // EPL*l .. EPL*l + EPL-1; a group's min / max by shuffles over its G/EPL lanes; codes
 // packed LSB-first and gathered into 32-bit words by OR over the lanes of each word.
 template <int D>
-__device__ __forceinline__ void quantise_row(const uint16_t* src, uint8_t* codes_row, uint32_t* sz_row, int b, int G,
+__device__ __forceinline__ void quantise_row(const uint2 w, uint8_t* codes_row, uint32_t* sz_row, int b, int G,
                                              int lane, int32_t* ctrl) {
   constexpr int EPL = D / 32;
   float x[EPL];
   if (EPL == 2) {
-    const uint32_t w = reinterpret_cast<const uint32_t*>(src)[lane];
-    x[0] = bf16lo(w);
-    x[1] = bf16hi(w);
+    x[0] = bf16lo(w.x);
+    x[1] = bf16hi(w.x);
   } else {
-    const uint2 w = reinterpret_cast<const uint2*>(src)[lane];
     x[0] = bf16lo(w.x);
     x[1] = bf16hi(w.x);
     x[EPL > 2 ? 2 : 0] = bf16lo(w.y);
@@ -322,6 +323,16 @@ __global__ void __launch_bounds__(256) append_fused_kernel(LayerArgs a, int n, c
   pdl_trigger();
   const int e = threadIdx.x, lane = e & 31, warp = e >> 5;
   const bool act = e < n;
+  // this warp's row (entry, KV head, K|V), loaded while the entries are planned
+  const int row = blockIdx.x * (blockDim.x >> 5) + warp;
+  const bool has_row = row < n * a.Hkv * 2;
+  const int re = row / (2 * a.Hkv), rh = (row >> 1) % a.Hkv, which = row & 1;
+  uint2 raw = make_uint2(0, 0);
+  if (has_row) {
+    const uint16_t* src = (which ? v : k) + (static_cast<int64_t>(re) * a.Hkv + rh) * D;
+    if (D == 64) raw.x = reinterpret_cast<const uint32_t*>(src)[lane];
+    else raw = reinterpret_cast<const uint2*>(src)[lane];
+  }
   int seq = -1, pos = 0, c = -1, err = 0;
   bool writes = false;
   if (act) {
@@ -360,12 +371,16 @@ __global__ void __launch_bounds__(256) append_fused_kernel(LayerArgs a, int n, c
       }
     }
   }
-  int tok = 0, nt_old = 0;
+  int tok = 0, nt_old = 0, last_page = -1;
   bool opens = false;
   if (act && !err) {
-    if (pos <= max(prev_max, a.last_pos[seq])) err = TRR_ERR_BAD_POSITION;
+    const int lp = a.last_pos[seq];
     if (writes) {
       nt_old = a.ntok[seq * 4 + c];
+      last_page = a.lastpg[seq * 4 + c];
+    }
+    if (pos <= max(prev_max, lp)) err = TRR_ERR_BAD_POSITION;
+    if (writes) {
       tok = nt_old + rank;
       opens = tok % a.P == 0;
     }
@@ -395,9 +410,10 @@ __global__ void __launch_bounds__(256) append_fused_kernel(LayerArgs a, int n, c
   }
   const int kidx = tok / a.P;
   const int64_t prow = (static_cast<int64_t>(seq) * 4 + c) * a.MP + kidx;
-  if (writes && !opens) {  // a page opened earlier: by a previous call, or by this one
+  if (writes && !opens) {  // a page opened earlier: by a previous call (then the class's
+                           // last page), or by an earlier entry of this call
     if (kidx * a.P < nt_old) {
-      pid = a.pt[prow];
+      pid = last_page;
     } else {
       for (int j = 0; j < e; ++j)
         if (s_seq[j] == seq && s_cls[j] == c && s_k[j] == kidx * a.P) pid = s_pid[j];
@@ -406,39 +422,32 @@ __global__ void __launch_bounds__(256) append_fused_kernel(LayerArgs a, int n, c
   }
   __syncthreads();
 
-  // this warp's row: (entry, KV head, K|V)
-  const int row = blockIdx.x * (blockDim.x >> 5) + warp;
-  if (row < n * a.Hkv * 2) {
-    const int re = row / (2 * a.Hkv), h = (row >> 1) % a.Hkv, which = row & 1;
+  if (has_row) {
     const int rc = s_cls[re];
     if (rc >= 0) {
       const int b = bits_of_class(rc), slot = s_k[re] % a.P;
-      const uint16_t* src = (which ? v : k) + (static_cast<int64_t>(re) * a.Hkv + h) * D;
       uint8_t* sl = a.pool[rc] + static_cast<int64_t>(s_pid[re]) * a.page_bytes[rc] + a.hdr +
-                    static_cast<int64_t>(h) * a.slice[rc];
+                    static_cast<int64_t>(rh) * a.slice[rc];
       if (b == 16) {
         uint32_t* dst = reinterpret_cast<uint32_t*>(sl + (static_cast<int64_t>(which) * a.P + slot) * D * 2);
-        if (D == 64) dst[lane] = reinterpret_cast<const uint32_t*>(src)[lane];
-        else reinterpret_cast<uint2*>(dst)[lane] = reinterpret_cast<const uint2*>(src)[lane];
+        if (D == 64) dst[lane] = raw.x;
+        else reinterpret_cast<uint2*>(dst)[lane] = raw;
       } else {
         const int rowb = D * b / 8, ng = D / a.G;
         uint8_t* codes_row = sl + (static_cast<int64_t>(which) * a.P + slot) * rowb;
         uint32_t* sz_row = reinterpret_cast<uint32_t*>(sl + 2 * static_cast<int64_t>(a.P) * rowb +
                                                       (static_cast<int64_t>(which) * a.P + slot) * ng * 4);
-        quantise_row<D>(src, codes_row, sz_row, b, a.G, lane, a.ctrl);
+        quantise_row<D>(raw, codes_row, sz_row, b, a.G, lane, a.ctrl);
       }
     }
   }
 
-  // the last CTA to finish commits the metadata of every entry
+  // the last CTA to finish commits the metadata of every entry: its acquire follows the
+  // release of every other CTA, after all of their reads of the old metadata
   __syncthreads();
-  if (e == 0) {
-    __threadfence();
-    s_last = atomicAdd(&a.ctrl[kAppendDone], 1) == static_cast<int>(gridDim.x) - 1;
-  }
+  if (e == 0) s_last = atom_add_acq_rel(&a.ctrl[kAppendDone], 1) == static_cast<int>(gridDim.x) - 1;
   __syncthreads();
   if (!s_last) return;
-  __threadfence();
   if (act) {
     if (writes) {
       const int slot = tok % a.P;
@@ -447,7 +456,10 @@ __global__ void __launch_bounds__(256) append_fused_kernel(LayerArgs a, int n, c
         a.pfirst[prow] = pos;
       }
       if (!later_cls || slot == a.P - 1) a.plast[prow] = pos;
-      if (!later_cls) a.ntok[seq * 4 + c] = tok + 1;
+      if (!later_cls) {
+        a.ntok[seq * 4 + c] = tok + 1;
+        a.lastpg[seq * 4 + c] = pid;
+      }
       reinterpret_cast<int32_t*>(a.pool[c] + static_cast<int64_t>(pid) * a.page_bytes[c])[slot] = pos;
       atomicOr(&a.presence[static_cast<int64_t>(seq) * a.W32 + pos / 32], 1u << (pos % 32));
     }

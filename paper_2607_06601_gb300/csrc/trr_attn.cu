@@ -115,32 +115,8 @@ __device__ __forceinline__ float code_at(const uint32_t* w, const uint32_t* h, i
     return __uint_as_float(__byte_perm(w[i / 4], 0u, 0x4440u | (i % 4)));
   }
 }
-// d = a * b + c on two fp32 lanes at once (packed fp32 FMA).
-__device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) {
-  float2 d;
-  asm("{\n .reg .b64 ra, rb, rc, rd;\n mov.b64 ra, {%2, %3};\n mov.b64 rb, {%4, %5};\n"
-      " mov.b64 rc, {%6, %7};\n fma.rn.f32x2 rd, ra, rb, rc;\n mov.b64 {%0, %1}, rd;\n}"
-      : "=f"(d.x), "=f"(d.y)
-      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
-  return d;
-}
-
-// The B words of 32 B-bit codes at a 4B-byte aligned address, in as few shared loads
-// as possible (one 8- or 16-byte load per row part keeps the warp's request
-// conflict-free).
-template <int B>
-__device__ __forceinline__ void load_codes(const uint8_t* p, uint32_t* w) {
-  if (B == 2) {
-    const uint2 u = *reinterpret_cast<const uint2*>(p);
-    w[0] = u.x; w[1] = u.y;
-  } else {
-#pragma unroll
-    for (int k = 0; k < B; k += 4) {
-      const uint4 u = *reinterpret_cast<const uint4*>(p + 4 * k);
-      w[k] = u.x; w[k + 1] = u.y; w[k + 2] = u.z; w[k + 3] = u.w;
-    }
-  }
-}
+// d = a * b + c on two fp32 lanes at once (packed fp32 FMA, round to nearest).
+__device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) { return __ffma2_rn(a, b, c); }
 
 template <int B>
 __device__ __forceinline__ void high_parts(const uint32_t* w, uint32_t* h) {
@@ -149,10 +125,19 @@ __device__ __forceinline__ void high_parts(const uint32_t* w, uint32_t* h) {
   for (int k = 0; k < B; ++k) h[k] = w[k] >> sh;
 }
 
+// x *= f on pairs of fp32 lanes (packed multiply)
+__device__ __forceinline__ void fmul2_inplace(float& x0, float& x1, float f0, float f1) {
+  const float2 r = __fmul2_rn(make_float2(x0, x1), make_float2(f0, f1));
+  x0 = r.x;
+  x1 = r.y;
+}
+
 template <int BFROM, int BTO>
 __device__ __forceinline__ void rescale_q(float (&qp)[32]) {
 #pragma unroll
-  for (int i = 0; i < 32; ++i) qp[i] *= pow2f(qe_of(BTO, i) - qe_of(BFROM, i));
+  for (int i = 0; i < 32; i += 2)
+    fmul2_inplace(qp[i], qp[i + 1], pow2f(qe_of(BTO, i) - qe_of(BFROM, i)),
+                  pow2f(qe_of(BTO, i + 1) - qe_of(BFROM, i + 1)));
 }
 
 // V is accumulated as acc_i * 2^(ex_i(B) - 49) while class B's pages are consumed
@@ -160,7 +145,10 @@ __device__ __forceinline__ void rescale_q(float (&qp)[32]) {
 template <int BFROM, int BTO>
 __device__ __forceinline__ void rescale_acc(float (&acc)[32]) {
 #pragma unroll
-  for (int i = 0; i < 32; ++i) acc[i] *= pow2f((BTO == 16 ? 0 : ex_of(BTO, i)) - (BFROM == 16 ? 0 : ex_of(BFROM, i)));
+  for (int i = 0; i < 32; i += 2)
+    fmul2_inplace(acc[i], acc[i + 1],
+                  pow2f((BTO == 16 ? 0 : ex_of(BTO, i)) - (BFROM == 16 ? 0 : ex_of(BFROM, i))),
+                  pow2f((BTO == 16 ? 0 : ex_of(BTO, i + 1)) - (BFROM == 16 ? 0 : ex_of(BFROM, i + 1))));
 }
 
 // qp from the domain of class `from` to that of class `to` (from < to, or from = 16).
@@ -186,14 +174,6 @@ __device__ __forceinline__ void acc_to_neutral(float (&acc)[32], int from) {
     case 2: rescale_acc<8, 16>(acc); break;
     default: break;
   }
-}
-
-// atomic add with release (of what this thread has seen written) and acquire (of what
-// the threads that released the same counter wrote) at GPU scope
-__device__ __forceinline__ int atom_add_acq_rel(int* p, int v) {
-  int old;
-  asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
-  return old;
 }
 
 // 2^x with the hardware approximation (relative error about 2^-22; results below the
@@ -223,47 +203,82 @@ __device__ __forceinline__ float softmax_step(LaneState& st, float score) {
   return p;
 }
 
-// One page of width class B in shared memory; lane -> (key kl, 32-dim part).  Keys
-// past `fill` are empty slots; with `spos` set, keys outside [lo, hi] are masked too.
-template <int D, int B>
-__device__ __forceinline__ void consume_page(const uint8_t* sl, const int* spos, int P, int G, int fill,
-                                             int lo, int hi, const float (&qp)[32], float sumq,
-                                             LaneState& st, int lane) {
+// Shared-memory loads at 32-bit shared addresses.  Volatile: they stay after the
+// mbarrier wait that makes the bytes valid.
+__device__ __forceinline__ uint4 lds128(uint32_t a) {
+  uint4 v;
+  asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a));
+  return v;
+}
+__device__ __forceinline__ uint2 lds64(uint32_t a) {
+  uint2 v;
+  asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(a));
+  return v;
+}
+__device__ __forceinline__ uint32_t lds32(uint32_t a) {
+  uint32_t v;
+  asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(a));
+  return v;
+}
+
+// The B words of 32 B-bit codes at shared address a (4B-byte aligned), in as few loads as
+// possible (one 8- or 16-byte load per row part keeps the warp's request conflict-free).
+template <int B>
+__device__ __forceinline__ void lds_codes(uint32_t a, uint32_t* w) {
+  if (B == 2) {
+    const uint2 u = lds64(a);
+    w[0] = u.x; w[1] = u.y;
+  } else {
+#pragma unroll
+    for (int k = 0; k < B; k += 4) {
+      const uint4 u = lds128(a + 4 * k);
+      w[k] = u.x; w[k + 1] = u.y; w[k + 2] = u.z; w[k + 3] = u.w;
+    }
+  }
+}
+
+// One page of width class B (P = NIT * keys per iteration tokens) at shared address s0;
+// lane -> (key kl, 32-dim part).  Keys past `fill` are empty slots; with positions at
+// spos (masked pages), keys outside [lo, hi] are masked too.
+template <int D, int B, int NIT>
+__device__ __forceinline__ void consume_page(uint32_t s0, uint32_t spos, bool masked, int G, int fill, int lo,
+                                             int hi, const float (&qp)[32], float sumq, LaneState& st, int lane) {
   constexpr int LPK = D / 32;
   constexpr int KPI = 32 / LPK;
+  constexpr int P = NIT * KPI;
+  constexpr int rowb = B == 16 ? 2 * D : D * B / 8;  // bytes of one key's row of K (or V)
   const int part = lane % LPK, kl = lane / LPK;
   const int ng = D / G;
   const int grp = part * 32 / G;
-  for (int it = 0; it < P / KPI; ++it) {
+  const uint32_t krow = s0 + kl * rowb + part * (B == 16 ? 64 : 4 * B);   // this lane's K bytes, key kl
+  const uint32_t ksz = s0 + 2 * P * rowb + (kl * ng + grp) * 4;           // its (s, z), key kl
+  const uint32_t szstep = KPI * ng * 4;
+#pragma unroll
+  for (int it = 0; it < NIT; ++it) {
     const int key = it * KPI + kl;
     bool valid = key < fill;
-    if (spos) {
-      const int pos = spos[key];
+    if (masked) {
+      const int pos = static_cast<int>(lds32(spos + 4 * key));
       valid = valid && pos >= lo && pos <= hi;
     }
+    const uint32_t ka = krow + it * KPI * rowb, va = ka + P * rowb;
     float dot;
     if (B == 16) {
-      const uint4* kp = reinterpret_cast<const uint4*>(sl + (key * D + part * 32) * 2);
-      float d[4] = {0.f, 0.f, 0.f, 0.f};
+      float2 d2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
-        const uint4 u = kp[q];
-        d[0] = fmaf(qp[8 * q + 0], bf_lo(u.x), d[0]);
-        d[1] = fmaf(qp[8 * q + 1], bf_hi(u.x), d[1]);
-        d[2] = fmaf(qp[8 * q + 2], bf_lo(u.y), d[2]);
-        d[3] = fmaf(qp[8 * q + 3], bf_hi(u.y), d[3]);
-        d[0] = fmaf(qp[8 * q + 4], bf_lo(u.z), d[0]);
-        d[1] = fmaf(qp[8 * q + 5], bf_hi(u.z), d[1]);
-        d[2] = fmaf(qp[8 * q + 6], bf_lo(u.w), d[2]);
-        d[3] = fmaf(qp[8 * q + 7], bf_hi(u.w), d[3]);
+        const uint4 u = lds128(ka + 16 * q);
+        d2[0] = ffma2(make_float2(qp[8 * q + 0], qp[8 * q + 1]), make_float2(bf_lo(u.x), bf_hi(u.x)), d2[0]);
+        d2[1] = ffma2(make_float2(qp[8 * q + 2], qp[8 * q + 3]), make_float2(bf_lo(u.y), bf_hi(u.y)), d2[1]);
+        d2[0] = ffma2(make_float2(qp[8 * q + 4], qp[8 * q + 5]), make_float2(bf_lo(u.z), bf_hi(u.z)), d2[0]);
+        d2[1] = ffma2(make_float2(qp[8 * q + 6], qp[8 * q + 7]), make_float2(bf_lo(u.w), bf_hi(u.w)), d2[1]);
       }
-      dot = (d[0] + d[1]) + (d[2] + d[3]);
+      dot = (d2[0].x + d2[0].y) + (d2[1].x + d2[1].y);
     } else {
-      constexpr int rowb = D * B / 8;
       uint32_t w[B], h[B];
-      load_codes<B>(sl + key * rowb + part * 4 * B, w);
+      lds_codes<B>(ka, w);
       if (B != 8) high_parts<B>(w, h);
-      const uint32_t szw = *reinterpret_cast<const uint32_t*>(sl + 2 * P * rowb + (key * ng + grp) * 4);
+      const uint32_t szw = lds32(ksz + it * szstep);
       float2 d2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
 #pragma unroll
       for (int i = 0; i < 16; ++i)
@@ -277,12 +292,11 @@ __device__ __forceinline__ void consume_page(const uint8_t* sl, const int* spos,
     if (valid) {
       const float p = softmax_step(st, dot);
       if (B == 16) {
-        const uint4* vp = reinterpret_cast<const uint4*>(sl + (P * D + key * D + part * 32) * 2);
         const float wv = p * pow2f(-49);
         const float2 w2 = make_float2(wv, wv);
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
-          const uint4 u = vp[q];
+          const uint4 u = lds128(va + 16 * q);
           const uint32_t uw[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
           for (int h = 0; h < 4; ++h) {
@@ -293,12 +307,10 @@ __device__ __forceinline__ void consume_page(const uint8_t* sl, const int* spos,
           }
         }
       } else {
-        constexpr int rowb = D * B / 8;
         uint32_t w[B], h[B];
-        load_codes<B>(sl + P * rowb + key * rowb + part * 4 * B, w);
+        lds_codes<B>(va, w);
         if (B != 8) high_parts<B>(w, h);
-        const uint32_t szw =
-            *reinterpret_cast<const uint32_t*>(sl + 2 * P * rowb + P * ng * 4 + (key * ng + grp) * 4);
+        const uint32_t szw = lds32(ksz + it * szstep + P * ng * 4);
         const float2 sz = __half22float2(*reinterpret_cast<const __half2*>(&szw));  // (s, z)
         const float wb = p * sz.x * pow2f(100);
         const float2 w2 = make_float2(wb, wb);
@@ -313,6 +325,18 @@ __device__ __forceinline__ void consume_page(const uint8_t* sl, const int* spos,
       }
     }
   }
+}
+
+// consume_page for the class and page size of the call
+template <int D, int B>
+__device__ __forceinline__ void consume_page_p(int P, uint32_t s0, uint32_t spos, bool masked, int G, int fill,
+                                               int lo, int hi, const float (&qp)[32], float sumq, LaneState& st,
+                                               int lane) {
+  // pages of 16, 32 or 64 tokens: 1, 2 or 4 iterations of 16 keys (d = 64), 2, 4 or 8 of 8
+  constexpr int KPI = 32 / (D / 32);
+  if (P == 16) consume_page<D, B, 16 / KPI>(s0, spos, masked, G, fill, lo, hi, qp, sumq, st, lane);
+  else if (P == 32) consume_page<D, B, 32 / KPI>(s0, spos, masked, G, fill, lo, hi, qp, sumq, st, lane);
+  else consume_page<D, B, 64 / KPI>(s0, spos, masked, G, fill, lo, hi, qp, sumq, st, lane);
 }
 
 // -------------------------------------------------------------------- kernel --
@@ -348,28 +372,26 @@ __device__ __forceinline__ int query_range(int t, int mode, int w) {
   return mode == TRR_MODE_FULL ? t + 1 : mode == TRR_MODE_LOCAL ? min(w, t + 1) : 0;
 }
 
-// Per-page record the producer writes for the consumer (three 16-byte words).
-struct SlotRec {
-  int meta;   // class | fill << 2 | mask << 9 | flags << 10 (1 first, 2 last, 4 no page)
-  int off;    // ring offset of the page's slice (then its positions when masked, then
-              // the query row on the first page of an item)
-  int span;   // ring bytes to release after the page
-  int lo;     // key range [lo, hi] of the item's query
-  int hi, item, qi, qh;
-  int nsplit, base, pad0, pad1;  // base: unit index of split 0 of the item's query
-};
-static_assert(sizeof(SlotRec) == 48, "SlotRec is three 16-byte words");
+// Per-page record the producer writes for the consumer: meta = class | fill << 2 |
+// mask << 9 | flags << 10 (1 first, 2 last, 4 no page) | item entry << 13, the ring
+// offset of the page's slice (then its positions when masked, then the query row on the
+// first page of an item) and the ring bytes to release after the page.  The item's own
+// fields sit once in the warp's item table (kItemSlots entries of 8 words: lo, hi, item,
+// query, head, splits, unit of split 0, KV head); an entry is rewritten only after every
+// record of its previous item has been consumed (at most kSlots records are in flight).
+constexpr int kItemSlots = 8;
+static_assert(kItemSlots >= kSlots, "an item entry outlives the records in flight");
 
 // Shared-memory carve-up of one attention CTA; every region starts 16-byte aligned
 // (mbarriers need 8, bulk-copy destinations 16).
 __host__ __device__ constexpr int align16(int x) { return (x + 15) & ~15; }
-constexpr int kWarpWords = 16;  // per-warp shared words: [0, 8) item plan, [8, 14) merge
+constexpr int kWarpWords = kItemSlots * 8 + 8;  // per-warp shared words: item table, merge
 struct AttnSmem {
   int rings, recs, bars, words, pre, red, total;
   __host__ __device__ AttnSmem(int nwarps, int ring_bytes, int n)
       : rings(0),
         recs(align16(nwarps * ring_bytes)),
-        bars(recs + align16(nwarps * kSlots * static_cast<int>(sizeof(SlotRec)))),
+        bars(recs + align16(nwarps * kSlots * 16)),
         words(bars + align16(nwarps * kSlots * 8)),
         pre(words + nwarps * kWarpWords * 4),
         red(pre + align16(4 * (n + 1))),
@@ -381,7 +403,7 @@ struct AttnSmem {
 // [0] lo [1] hi [2] item [3] query [4] query head [5] splits [6] unit of split 0 [7] KV head.
 template <int D>
 __device__ __forceinline__ int plan_next_item(const AttnKernelArgs& ka, const int* pre, int n, int wstride, int lane,
-                                           int* next_item, int* wplan, int& wid, int& wmeta) {
+                                           int* next_item, int* wplan, int& wid, int& wmeta, int& kvh) {
   const LayerArgs& a = ka.a;
   const int total = pre[n] * a.Hq;
   while (*next_item < total) {
@@ -429,13 +451,16 @@ __device__ __forceinline__ int plan_next_item(const AttnKernelArgs& ka, const in
     if (lo > 0) warp_count_below<kClasses>(a.plast + row0, a.MP, pages, lo, first, lane);
     if (upper_mask) warp_count_below<kClasses>(a.pfirst + row0, a.MP, pages, t + 1, end, lane);
     // this split's share of each class's pages in range, then one page per lane
+    // split sp of ns takes np / ns pages of the class, one more when sp < np % ns
     int beg[kClasses], tc[kClasses], npr[kClasses];
     int T = 0;
 #pragma unroll
     for (int c = 0; c < kClasses; ++c) {
       npr[c] = max(0, end[c] - first[c]);
-      beg[c] = first[c] + static_cast<int>(static_cast<int64_t>(sp) * npr[c] / ns);
-      tc[c] = first[c] + static_cast<int>(static_cast<int64_t>(sp + 1) * npr[c] / ns) - beg[c];
+      const unsigned each = static_cast<unsigned>(npr[c]) / static_cast<unsigned>(ns);
+      const int extra = npr[c] - static_cast<int>(each) * ns;
+      beg[c] = first[c] + sp * static_cast<int>(each) + min(sp, extra);
+      tc[c] = static_cast<int>(each) + (sp < extra ? 1 : 0);
       T += tc[c];
     }
     T = min(T, kItemMaxPages + kClasses);  // the split bound keeps T within this
@@ -459,9 +484,10 @@ __device__ __forceinline__ int plan_next_item(const AttnKernelArgs& ka, const in
       const bool mask = (lo > 0 && kid == f) || (upper_mask && kid == f + pick(npr) - 1);
       wmeta = c | (fill << 2) | (mask ? 512 : 0);
     }
+    kvh = h / (a.Hq / a.Hkv);
     if (lane == 0) {
       reinterpret_cast<int4*>(wplan)[0] = make_int4(lo, t, i, q);
-      reinterpret_cast<int4*>(wplan)[1] = make_int4(h, ns, pre[q], h / (a.Hq / a.Hkv));
+      reinterpret_cast<int4*>(wplan)[1] = make_int4(h, ns, pre[q], kvh);
     }
     __syncwarp();
     return T;
@@ -481,11 +507,11 @@ __global__ void __launch_bounds__(256, 2) attn_kernel(const __grid_constant__ At
   const int R = ka.ring_bytes;
   const AttnSmem lay(nwarps, R, n);  // [rings][slot records][mbarriers][unit prefix][scratch]
   uint8_t* ring = smem + lay.rings + warp * R;
-  SlotRec* recs = reinterpret_cast<SlotRec*>(smem + lay.recs) + warp * kSlots;
+  int4* recs = reinterpret_cast<int4*>(smem + lay.recs) + warp * kSlots;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + lay.bars) + warp * kSlots;
   int* pre = reinterpret_cast<int*>(smem + lay.pre);
-  int* wplan = reinterpret_cast<int*>(smem + lay.words) + warp * kWarpWords;
-  int* wmerge = wplan + 8;
+  int* witems = reinterpret_cast<int*>(smem + lay.words) + warp * kWarpWords;  // item table
+  int* wmerge = witems + kItemSlots * 8;
   long long* red = reinterpret_cast<long long*>(smem + lay.red);
 
   if (lane == 0) {
@@ -514,9 +540,11 @@ __global__ void __launch_bounds__(256, 2) attn_kernel(const __grid_constant__ At
   rsum = 0;
   for (int k = 0; k < nwarps; ++k) rsum += red[k];
   // splits small enough for about kItemsPerWarp items per warp, never below pos_split
-  const long long want = static_cast<long long>(gridDim.x) * nwarps * kItemsPerWarp;
-  const long long by_work = (rsum * a.Hq + want - 1) / want;
-  const int pos_split = static_cast<int>(max(static_cast<long long>(a.pos_split), min(by_work, 1ll << 30)));
+  // (binary32 arithmetic: the same result in every CTA, and it only sizes the splits)
+  const float want = static_cast<float>(gridDim.x * nwarps * kItemsPerWarp);
+  const float by_work = ceilf(static_cast<float>(rsum) * static_cast<float>(a.Hq) / want);
+  const int pos_split = by_work > static_cast<float>(a.pos_split) ? static_cast<int>(fminf(by_work, 1073741824.f))
+                                                                   : a.pos_split;
   {
     const int chunk = (n + blockDim.x - 1) / blockDim.x;
     const int q0 = min(n, static_cast<int>(threadIdx.x) * chunk), q1 = min(n, q0 + chunk);
@@ -549,23 +577,29 @@ __global__ void __launch_bounds__(256, 2) attn_kernel(const __grid_constant__ At
   int next_item = blockIdx.x * nwarps + warp;
   int wid = -1, wmeta = 0;             // the producer's item: page id / meta of page `lane`
   int p_T = 0;                         // pages of the producer's item
+  int p_kvh = 0;                       // its KV head
   int pf = 0;                          // next page of the producer's item
   bool pvalid = false;
   uint32_t issued = 0, consumed = 0;   // pages issued / consumed by this warp
+  uint32_t started = 0;                // items started by this warp (item table index)
   int head = 0, used = 0;              // ring: next free offset, bytes held
 
   auto start_item = [&]() -> bool {
-    p_T = plan_next_item<D>(ka, pre, n, wstride, lane, &next_item, wplan, wid, wmeta);
+    p_T = plan_next_item<D>(ka, pre, n, wstride, lane, &next_item, witems + (started % kItemSlots) * 8, wid,
+                            wmeta, p_kvh);
     pf = 0;
-    return p_T >= 0;
+    if (p_T < 0) return false;
+    ++started;
+    return true;
   };
   // start the copies of the producer's next page if a slot and ring space are free
   auto try_issue = [&]() -> bool {
+    if (issued - consumed >= kSlots) return false;  // first: an item entry is reused only
+                                                    // once fewer records are in flight
     if (!pvalid) {
       pvalid = start_item();
       if (!pvalid) return false;
     }
-    if (issued - consumed >= kSlots) return false;
     const bool first = pf == 0;
     int meta = 0, id = -1, bytes_page = 0;
     if (p_T > 0) {
@@ -590,21 +624,19 @@ __global__ void __launch_bounds__(256, 2) attn_kernel(const __grid_constant__ At
     // record reaches the consumer through the mbarrier's release / acquire, so no proxy
     // fence is needed here.
     if (lane == 0) {
-      const int4 pa = reinterpret_cast<const int4*>(wplan)[0];  // lo, hi, item, query
-      const int4 pb = reinterpret_cast<const int4*>(wplan)[1];  // head, splits, base, KV head
-      int4* rp = reinterpret_cast<int4*>(recs + slot);
-      rp[0] = make_int4(meta | (flags << 10), off, waste + need, pa.x);
-      rp[1] = make_int4(pa.y, pa.z, pa.w, pb.x);
-      rp[2] = make_int4(pb.y, pb.z, 0, 0);
+      const int entry = (started - 1) % kItemSlots;
+      recs[slot] = make_int4(meta | (flags << 10) | (entry << 13), off, waste + need, 0);
       mbar_arrive_expect_tx(&bars[slot], need);
       const int c = meta & 3;
       if (p_T > 0) {
         const uint8_t* page = a.pool[c] + static_cast<int64_t>(id) * a.page_bytes[c];
-        bulk_g2s(ring + off, page + a.hdr + static_cast<int64_t>(pb.w) * a.slice[c], a.slice[c], &bars[slot]);
+        bulk_g2s(ring + off, page + a.hdr + static_cast<int64_t>(p_kvh) * a.slice[c], a.slice[c], &bars[slot]);
         if (meta & 512) bulk_g2s(ring + off + a.slice[c], page, 4 * a.P, &bars[slot]);
       }
-      if (first)
-        bulk_g2s(ring + off + bytes_page, ka.q + (static_cast<int64_t>(pa.w) * a.Hq + pb.x) * D, qrow, &bars[slot]);
+      if (first) {
+        const int* it = witems + entry * 8;
+        bulk_g2s(ring + off + bytes_page, ka.q + (static_cast<int64_t>(it[3]) * a.Hq + it[4]) * D, qrow, &bars[slot]);
+      }
     }
     __syncwarp();
     ++issued;
@@ -638,8 +670,15 @@ __global__ void __launch_bounds__(256, 2) attn_kernel(const __grid_constant__ At
     float L = st.l * f;
 #pragma unroll
     for (int o = LPK; o < 32; o <<= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
+    {
+      const float2 s49 = make_float2(pow2f(49) * f, pow2f(49) * f), zf = make_float2(st.zacc * f, st.zacc * f);
 #pragma unroll
-    for (int j = 0; j < 32; ++j) st.acc[j] = fmaf(st.acc[j], pow2f(49), st.zacc) * f;
+      for (int j = 0; j < 32; j += 2) {
+        const float2 r = __ffma2_rn(make_float2(st.acc[j], st.acc[j + 1]), s49, zf);
+        st.acc[j] = r.x;
+        st.acc[j + 1] = r.y;
+      }
+    }
 #pragma unroll
     for (int width = 16, o = 16; o >= LPK; width >>= 1, o >>= 1) {
       const bool upper = lane & o;
@@ -722,24 +761,27 @@ __global__ void __launch_bounds__(256, 2) attn_kernel(const __grid_constant__ At
       if (lane == 0) set_status(a.ctrl, TRR_ERR_TIMEOUT);
       break;
     }
-    const int4 r0 = *reinterpret_cast<const int4*>(recs + slot);
-    const int meta = r0.x, flags = meta >> 10;
+    const int4 r0 = recs[slot];
+    const int meta = r0.x, flags = (meta >> 10) & 7;
+    const int* item_words = witems + (meta >> 13) * 8;  // lo, hi, item, query, head, splits, base
     if (flags & 1) {  // first page of an item: query row and a fresh state
       const int qoff = r0.y + ((flags & 4) ? 0 : a.slice[meta & 3] + ((meta & 512) ? 4 * a.P : 0));
-      const uint4* q4 = reinterpret_cast<const uint4*>(ring + qoff + part * 64);
-      sumq = 0.f;
+      const uint32_t qa = smem_u32(ring + qoff + part * 64);
+      const float2 qs2 = make_float2(ka.qscale, ka.qscale);
+      float2 sq2 = make_float2(0.f, 0.f);
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
-        const uint4 u = q4[q];
+        const uint4 u = lds128(qa + 16 * q);
         const uint32_t wv[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
         for (int h = 0; h < 4; ++h) {
-          qp[8 * q + 2 * h] = bf_lo(wv[h]) * ka.qscale;
-          qp[8 * q + 2 * h + 1] = bf_hi(wv[h]) * ka.qscale;
+          const float2 r = __fmul2_rn(make_float2(bf_lo(wv[h]), bf_hi(wv[h])), qs2);
+          qp[8 * q + 2 * h] = r.x;
+          qp[8 * q + 2 * h + 1] = r.y;
+          sq2 = __fadd2_rn(sq2, r);
         }
       }
-#pragma unroll
-      for (int j = 0; j < 32; ++j) sumq += qp[j];
+      sumq = sq2.x + sq2.y;
       cur_cls = 3;  // the neutral scale is class 16's
       st.m = kNegInf;
       st.l = 0.f;
@@ -753,21 +795,21 @@ __global__ void __launch_bounds__(256, 2) attn_kernel(const __grid_constant__ At
         rescale_dyn(qp, st.acc, cur_cls, cls);
         cur_cls = cls;
       }
-      const uint8_t* sl = ring + r0.y;
-      const int* sp = (meta & 512) ? reinterpret_cast<const int*>(ring + r0.y + a.slice[cls]) : nullptr;
-      const int c_lo = r0.w, c_hi = reinterpret_cast<const int*>(recs + slot)[4];  // key range
+      const uint32_t s0 = smem_u32(ring + r0.y);
+      const uint32_t sp = s0 + a.slice[cls];  // slot positions, on masked pages
+      const bool masked = meta & 512;
+      const int c_lo = item_words[0], c_hi = item_words[1];  // key range
       switch (cls) {
-        case 0: consume_page<D, 2>(sl, sp, a.P, a.G, fill, c_lo, c_hi, qp, sumq, st, lane); break;
-        case 1: consume_page<D, 4>(sl, sp, a.P, a.G, fill, c_lo, c_hi, qp, sumq, st, lane); break;
-        case 2: consume_page<D, 8>(sl, sp, a.P, a.G, fill, c_lo, c_hi, qp, sumq, st, lane); break;
-        default: consume_page<D, 16>(sl, sp, a.P, a.G, fill, c_lo, c_hi, qp, sumq, st, lane); break;
+        case 0: consume_page_p<D, 2>(a.P, s0, sp, masked, a.G, fill, c_lo, c_hi, qp, sumq, st, lane); break;
+        case 1: consume_page_p<D, 4>(a.P, s0, sp, masked, a.G, fill, c_lo, c_hi, qp, sumq, st, lane); break;
+        case 2: consume_page_p<D, 8>(a.P, s0, sp, masked, a.G, fill, c_lo, c_hi, qp, sumq, st, lane); break;
+        default: consume_page_p<D, 16>(a.P, s0, sp, masked, a.G, fill, c_lo, c_hi, qp, sumq, st, lane); break;
       }
     }
     if (flags & 2) {  // last page of the item: its merge follows the refill
       if (lane == 0) {
-        const int* rw = reinterpret_cast<const int*>(recs + slot);
-        reinterpret_cast<int4*>(wmerge)[0] = make_int4(rw[5], rw[6], rw[7], rw[8]);
-        wmerge[4] = rw[9];
+        reinterpret_cast<int4*>(wmerge)[0] = make_int4(item_words[2], item_words[3], item_words[4], item_words[5]);
+        wmerge[4] = item_words[6];
       }
       merge_pending = true;
     }

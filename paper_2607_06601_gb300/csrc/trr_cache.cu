@@ -35,6 +35,7 @@ LayerArgs layer_args(const Layout& l, const Views& v, int layer) {
   a.pt = v.pt + ls * 4 * l.MP;
   a.pfirst = v.pfirst + ls * 4 * l.MP;
   a.plast = v.plast + ls * 4 * l.MP;
+  a.lastpg = v.lastpg + ls * 4;
   a.aplan = v.aplan;
   a.cnt = v.cnt;
   a.part = v.part;
@@ -99,6 +100,7 @@ static trr_status make_layout(const trr_cache_config* c, Layout* l) {
   l->off_pt = take(16 * nls * l->MP);
   l->off_pfirst = take(16 * nls * l->MP);
   l->off_plast = take(16 * nls * l->MP);
+  l->off_lastpg = take(16 * nls);
   l->off_aplan = take(static_cast<int64_t>(sizeof(AppendPlan)) * l->max_append);
   l->off_cnt = take(4 * static_cast<int64_t>(l->max_queries) * l->units);
   l->off_part = take(4 * l->max_items * (l->Hq / l->units) * (l->d + 4));
@@ -145,6 +147,7 @@ static trr_status clear_metadata(trr_cache* c, cudaStream_t s) {
   ok = ok && cudaMemsetAsync(b + l.off_ntok, 0, 16 * nls, s) == cudaSuccess;
   ok = ok && cudaMemsetAsync(b + l.off_presence, 0, 4 * nls * l.W32, s) == cudaSuccess;
   ok = ok && cudaMemsetAsync(b + l.off_pt, 0xFF, 3 * (l.off_pfirst - l.off_pt), s) == cudaSuccess;
+  ok = ok && cudaMemsetAsync(b + l.off_lastpg, 0xFF, 16 * nls, s) == cudaSuccess;
   ok = ok && cudaMemsetAsync(b + l.off_cnt, 0, 4 * static_cast<int64_t>(l.max_queries) * l.units, s) == cudaSuccess;
   return ok ? TRR_OK : TRR_ERR_CUDA;
 }

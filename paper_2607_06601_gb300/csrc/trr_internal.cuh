@@ -40,7 +40,7 @@ struct Layout {
   int s_cap;      // most splits one query is cut into
   int64_t max_items;
   int64_t hdr, tokb[kClasses], slice[kClasses], page_bytes[kClasses];
-  int64_t off_ctrl, off_last_pos, off_ntok, off_presence, off_pt, off_pfirst, off_plast;
+  int64_t off_ctrl, off_last_pos, off_ntok, off_presence, off_pt, off_pfirst, off_plast, off_lastpg;
   int64_t off_aplan, off_cnt, off_part, off_pool[kClasses], total;
 };
 
@@ -71,6 +71,7 @@ struct Views {  // typed device pointers into the cache memory
   int32_t* pt;
   int32_t* pfirst;
   int32_t* plast;
+  int32_t* lastpg;
   AppendPlan* aplan;
   int32_t* cnt;
   float* part;
@@ -87,6 +88,7 @@ inline Views make_views(const Layout& l, void* base) {
   v.pt = reinterpret_cast<int32_t*>(b + l.off_pt);
   v.pfirst = reinterpret_cast<int32_t*>(b + l.off_pfirst);
   v.plast = reinterpret_cast<int32_t*>(b + l.off_plast);
+  v.lastpg = reinterpret_cast<int32_t*>(b + l.off_lastpg);
   v.aplan = reinterpret_cast<AppendPlan*>(b + l.off_aplan);
   v.cnt = reinterpret_cast<int32_t*>(b + l.off_cnt);
   v.part = reinterpret_cast<float*>(b + l.off_part);
@@ -108,6 +110,7 @@ struct LayerArgs {
   int32_t* pt;         // this layer: [S][4][MP]
   int32_t* pfirst;
   int32_t* plast;
+  int32_t* lastpg;     // this layer: [S][4] id of the page holding token ntok-1 (internal)
   AppendPlan* aplan;
   int32_t* cnt;        // [max_queries][Hq] split arrivals (zero between calls)
   float* part;         // [max_queries * s_cap * Hq][d + 4] fp32 partials: acc, M, L
@@ -173,6 +176,14 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint32
     if (done) return true;
   }
   return false;
+}
+
+// atomic add with release (of what this thread has seen written) and acquire (of what
+// the threads that released the same counter wrote) at GPU scope
+__device__ __forceinline__ int atom_add_acq_rel(int* p, int v) {
+  int old;
+  asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+  return old;
 }
 
 __device__ __forceinline__ void set_status(int32_t* ctrl, int code) {
