@@ -190,12 +190,20 @@ def measured_peaks():
         return 6800.0, "fallback"
 
 
+def kernel_source_digest():
+    """sha256 (16 hex digits) of the sources that decide what the attention kernel does:
+    the kernel, the cache layout and the shared header."""
+    import hashlib
+    h = hashlib.sha256()
+    for f in ("trr_attn.cu", "trr_cache.cu", "trr_internal.cuh"):
+        h.update(open(os.path.join(ROOT, "paper_2607_06601_gb300", "csrc", f), "rb").read())
+    return h.hexdigest()[:16]
+
+
 def ncu_traffic(workload):
     """Per-launch DRAM bytes of the attention kernel from the committed ncu summary,
-    if it was taken on the current kernel source (else None)."""
-    import hashlib
-    src = os.path.join(ROOT, "paper_2607_06601_gb300", "csrc", "trr_attn.cu")
-    digest = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    if it was taken on the current kernel sources (else None)."""
+    digest = kernel_source_digest()
     path = os.path.join(ROOT, "profiles", f"attn_kernel_{workload}_traffic.txt")
     try:
         kv = dict(line.split(":", 1) for line in open(path) if ":" in line)

@@ -95,7 +95,7 @@ typedef struct trr_cache_config {
   int32_t pages_per_class[4]; /* pool capacity for b = 2, 4, 8, 16 */
   int32_t max_append;      /* largest n accepted by trr_kv_append */
   int32_t max_queries;     /* largest n accepted by trr_decode_attn */
-  int32_t split_bytes;     /* target KV bytes per split-K work item; 0 = 16384 */
+  int32_t split_bytes;     /* least KV bytes (of 8-bit tokens) per split-K work item; 0 = 24576 */
   int32_t skip_writes_kv;  /* 0: a skip token stores no KV (default); 1: it stores KV */
   void* pool;              /* device memory of >= trr_cache_required_bytes, or NULL */
   uint64_t pool_bytes;     /* size of `pool` (ignored when pool is NULL) */

@@ -253,7 +253,7 @@ __device__ __forceinline__ void consume_page(uint32_t s0, uint32_t spos, bool ma
   const uint32_t krow = s0 + kl * rowb + part * (B == 16 ? 64 : 4 * B);   // this lane's K bytes, key kl
   const uint32_t ksz = s0 + 2 * P * rowb + (kl * ng + grp) * 4;           // its (s, z), key kl
   const uint32_t szstep = KPI * ng * 4;
-#pragma unroll
+#pragma unroll 4
   for (int it = 0; it < NIT; ++it) {
     const int key = it * KPI + kl;
     bool valid = key < fill;
@@ -325,18 +325,6 @@ __device__ __forceinline__ void consume_page(uint32_t s0, uint32_t spos, bool ma
       }
     }
   }
-}
-
-// consume_page for the class and page size of the call
-template <int D, int B>
-__device__ __forceinline__ void consume_page_p(int P, uint32_t s0, uint32_t spos, bool masked, int G, int fill,
-                                               int lo, int hi, const float (&qp)[32], float sumq, LaneState& st,
-                                               int lane) {
-  // pages of 16, 32 or 64 tokens: 1, 2 or 4 iterations of 16 keys (d = 64), 2, 4 or 8 of 8
-  constexpr int KPI = 32 / (D / 32);
-  if (P == 16) consume_page<D, B, 16 / KPI>(s0, spos, masked, G, fill, lo, hi, qp, sumq, st, lane);
-  else if (P == 32) consume_page<D, B, 32 / KPI>(s0, spos, masked, G, fill, lo, hi, qp, sumq, st, lane);
-  else consume_page<D, B, 64 / KPI>(s0, spos, masked, G, fill, lo, hi, qp, sumq, st, lane);
 }
 
 // -------------------------------------------------------------------- kernel --
@@ -495,9 +483,10 @@ __device__ __forceinline__ int plan_next_item(const AttnKernelArgs& ka, const in
   return -1;
 }
 
-template <int D>
+template <int D, int P>
 __global__ void __launch_bounds__(256, 2) attn_kernel(const __grid_constant__ AttnKernelArgs ka) {
   constexpr int LPK = D / 32;  // lanes per key
+  constexpr int KPI = 32 / LPK;  // keys per warp iteration
   constexpr int DPL = D / 32;  // dimensions per lane after the merge
   const LayerArgs& a = ka.a;
   extern __shared__ __align__(128) uint8_t smem[];
@@ -605,7 +594,7 @@ __global__ void __launch_bounds__(256, 2) attn_kernel(const __grid_constant__ At
     if (p_T > 0) {
       id = __shfl_sync(0xffffffffu, wid, pf);
       meta = __shfl_sync(0xffffffffu, wmeta, pf);
-      bytes_page = a.slice[meta & 3] + ((meta & 512) ? 4 * a.P : 0);
+      bytes_page = a.slice[meta & 3] + ((meta & 512) ? 4 * P : 0);
     }
     const int need = bytes_page + (first ? qrow : 0);
     if (used == 0) head = 0;  // an empty ring can start anywhere
@@ -631,7 +620,7 @@ __global__ void __launch_bounds__(256, 2) attn_kernel(const __grid_constant__ At
       if (p_T > 0) {
         const uint8_t* page = a.pool[c] + static_cast<int64_t>(id) * a.page_bytes[c];
         bulk_g2s(ring + off, page + a.hdr + static_cast<int64_t>(p_kvh) * a.slice[c], a.slice[c], &bars[slot]);
-        if (meta & 512) bulk_g2s(ring + off + a.slice[c], page, 4 * a.P, &bars[slot]);
+        if (meta & 512) bulk_g2s(ring + off + a.slice[c], page, 4 * P, &bars[slot]);
       }
       if (first) {
         const int* it = witems + entry * 8;
@@ -765,7 +754,7 @@ __global__ void __launch_bounds__(256, 2) attn_kernel(const __grid_constant__ At
     const int meta = r0.x, flags = (meta >> 10) & 7;
     const int* item_words = witems + (meta >> 13) * 8;  // lo, hi, item, query, head, splits, base
     if (flags & 1) {  // first page of an item: query row and a fresh state
-      const int qoff = r0.y + ((flags & 4) ? 0 : a.slice[meta & 3] + ((meta & 512) ? 4 * a.P : 0));
+      const int qoff = r0.y + ((flags & 4) ? 0 : a.slice[meta & 3] + ((meta & 512) ? 4 * P : 0));
       const uint32_t qa = smem_u32(ring + qoff + part * 64);
       const float2 qs2 = make_float2(ka.qscale, ka.qscale);
       float2 sq2 = make_float2(0.f, 0.f);
@@ -800,10 +789,10 @@ __global__ void __launch_bounds__(256, 2) attn_kernel(const __grid_constant__ At
       const bool masked = meta & 512;
       const int c_lo = item_words[0], c_hi = item_words[1];  // key range
       switch (cls) {
-        case 0: consume_page_p<D, 2>(a.P, s0, sp, masked, a.G, fill, c_lo, c_hi, qp, sumq, st, lane); break;
-        case 1: consume_page_p<D, 4>(a.P, s0, sp, masked, a.G, fill, c_lo, c_hi, qp, sumq, st, lane); break;
-        case 2: consume_page_p<D, 8>(a.P, s0, sp, masked, a.G, fill, c_lo, c_hi, qp, sumq, st, lane); break;
-        default: consume_page_p<D, 16>(a.P, s0, sp, masked, a.G, fill, c_lo, c_hi, qp, sumq, st, lane); break;
+        case 0: consume_page<D, 2, P / KPI>(s0, sp, masked, a.G, fill, c_lo, c_hi, qp, sumq, st, lane); break;
+        case 1: consume_page<D, 4, P / KPI>(s0, sp, masked, a.G, fill, c_lo, c_hi, qp, sumq, st, lane); break;
+        case 2: consume_page<D, 8, P / KPI>(s0, sp, masked, a.G, fill, c_lo, c_hi, qp, sumq, st, lane); break;
+        default: consume_page<D, 16, P / KPI>(s0, sp, masked, a.G, fill, c_lo, c_hi, qp, sumq, st, lane); break;
       }
     }
     if (flags & 2) {  // last page of the item: its merge follows the refill
@@ -835,10 +824,15 @@ constexpr int kAttnSmemLimit = 113 * 1024;  // dynamic shared memory of one atte
 
 // Done once per cache at creation, so that calls stay legal inside stream capture.
 cudaError_t attn_configure() {
-  cudaError_t e = cudaFuncSetAttribute(attn_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, kAttnSmemLimit);
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(attn_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, kAttnSmemLimit);
-  return e;
+  const void* kernels[] = {
+      reinterpret_cast<const void*>(attn_kernel<64, 16>), reinterpret_cast<const void*>(attn_kernel<64, 32>),
+      reinterpret_cast<const void*>(attn_kernel<64, 64>), reinterpret_cast<const void*>(attn_kernel<128, 16>),
+      reinterpret_cast<const void*>(attn_kernel<128, 32>), reinterpret_cast<const void*>(attn_kernel<128, 64>)};
+  for (const void* k : kernels) {
+    const cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, kAttnSmemLimit);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
 }
 
 // The one launch of an attention call with the given scratch views in `a`.
@@ -870,9 +864,18 @@ static cudaError_t launch_attention(const Layout& l, const LayerArgs& a, int num
   if (nwarps < 1) return cudaErrorInvalidConfiguration;
   ka.ring_bytes = ring;
   const int smem = AttnSmem(nwarps, ring, n).total;
-  if (l.d == 64)
-    return launch_pdl(attn_kernel<64>, dim3(2 * num_sms), dim3(nwarps * 32), static_cast<size_t>(smem), s, ka);
-  return launch_pdl(attn_kernel<128>, dim3(2 * num_sms), dim3(nwarps * 32), static_cast<size_t>(smem), s, ka);
+  // one kernel per head size and page size: the page loop unrolls, and a kernel's code
+  // holds only the four width classes it can meet
+  const dim3 grid(2 * num_sms), block(nwarps * 32);
+  const size_t sm = static_cast<size_t>(smem);
+  if (l.d == 64) {
+    if (l.P == 16) return launch_pdl(attn_kernel<64, 16>, grid, block, sm, s, ka);
+    if (l.P == 32) return launch_pdl(attn_kernel<64, 32>, grid, block, sm, s, ka);
+    return launch_pdl(attn_kernel<64, 64>, grid, block, sm, s, ka);
+  }
+  if (l.P == 16) return launch_pdl(attn_kernel<128, 16>, grid, block, sm, s, ka);
+  if (l.P == 32) return launch_pdl(attn_kernel<128, 32>, grid, block, sm, s, ka);
+  return launch_pdl(attn_kernel<128, 64>, grid, block, sm, s, ka);
 }
 
 }  // namespace trr

@@ -69,7 +69,7 @@ static trr_status make_layout(const trr_cache_config* c, Layout* l) {
   for (int k = 0; k < kClasses; ++k) l->cap[k] = c->pages_per_class[k];
   l->max_append = c->max_append;
   l->max_queries = c->max_queries;
-  l->split_bytes = c->split_bytes ? c->split_bytes : 16384;
+  l->split_bytes = c->split_bytes ? c->split_bytes : 24576;
   l->skip_writes_kv = c->skip_writes_kv;
   l->hdr = roundup(4 * static_cast<int64_t>(l->P), 128);
   for (int k = 0; k < kClasses; ++k) {
