@@ -253,7 +253,7 @@ __device__ __forceinline__ void consume_page(uint32_t s0, uint32_t spos, bool ma
   const uint32_t krow = s0 + kl * rowb + part * (B == 16 ? 64 : 4 * B);   // this lane's K bytes, key kl
   const uint32_t ksz = s0 + 2 * P * rowb + (kl * ng + grp) * 4;           // its (s, z), key kl
   const uint32_t szstep = KPI * ng * 4;
-#pragma unroll 4
+#pragma unroll 1
   for (int it = 0; it < NIT; ++it) {
     const int key = it * KPI + kl;
     bool valid = key < fill;
