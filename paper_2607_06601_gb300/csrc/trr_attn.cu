@@ -240,12 +240,83 @@ __device__ __forceinline__ void lds_codes(uint32_t a, uint32_t* w) {
 // One page of width class B (P = NIT * keys per iteration tokens) at shared address s0;
 // lane -> (key kl, 32-dim part).  Keys past `fill` are empty slots; with positions at
 // spos (masked pages), keys outside [lo, hi] are masked too.
+// q.k of one key at shared address ka (this lane's 32 dims) in class B, with its (s, z)
+// word at kszaddr for B < 16: s * sum(q_i c_i) + z * sum(q_i) in the domain of qp.
+template <int B>
+__device__ __forceinline__ float k_dot(uint32_t ka, uint32_t kszaddr, const float (&qp)[32], float sumq) {
+  float2 d2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+  if (B == 16) {
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const uint4 u = lds128(ka + 16 * q);
+      d2[0] = ffma2(make_float2(qp[8 * q + 0], qp[8 * q + 1]), make_float2(bf_lo(u.x), bf_hi(u.x)), d2[0]);
+      d2[1] = ffma2(make_float2(qp[8 * q + 2], qp[8 * q + 3]), make_float2(bf_lo(u.y), bf_hi(u.y)), d2[1]);
+      d2[0] = ffma2(make_float2(qp[8 * q + 4], qp[8 * q + 5]), make_float2(bf_lo(u.z), bf_hi(u.z)), d2[0]);
+      d2[1] = ffma2(make_float2(qp[8 * q + 6], qp[8 * q + 7]), make_float2(bf_lo(u.w), bf_hi(u.w)), d2[1]);
+    }
+    return (d2[0].x + d2[0].y) + (d2[1].x + d2[1].y);
+  }
+  uint32_t w[B], h[B];
+  lds_codes<B>(ka, w);
+  if (B != 8) high_parts<B>(w, h);
+  const uint32_t szw = lds32(kszaddr);
+#pragma unroll
+  for (int i = 0; i < 16; ++i)
+    d2[i & 1] = ffma2(make_float2(qp[2 * i], qp[2 * i + 1]),
+                      make_float2(code_at<B>(w, h, 2 * i), code_at<B>(w, h, 2 * i + 1)), d2[i & 1]);
+  const float2 sz = __half22float2(*reinterpret_cast<const __half2*>(&szw));  // (s, z)
+  return fmaf(sz.x * pow2f(49), (d2[0].x + d2[0].y) + (d2[1].x + d2[1].y), sz.y * sumq);
+}
+
+// acc += p * v for one key's V at shared address va (this lane's 32 dims) in class B,
+// with its (s, z) word at vszaddr for B < 16.
+template <int B>
+__device__ __forceinline__ void v_acc(uint32_t va, uint32_t vszaddr, float p, LaneState& st) {
+  if (B == 16) {
+    const float wv = p * pow2f(-49);
+    const float2 w2 = make_float2(wv, wv);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const uint4 u = lds128(va + 16 * q);
+      const uint32_t uw[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+      for (int h = 0; h < 4; ++h) {
+        const int i = 8 * q + 2 * h;
+        const float2 r = ffma2(w2, make_float2(bf_lo(uw[h]), bf_hi(uw[h])), make_float2(st.acc[i], st.acc[i + 1]));
+        st.acc[i] = r.x;
+        st.acc[i + 1] = r.y;
+      }
+    }
+    return;
+  }
+  uint32_t w[B], h[B];
+  lds_codes<B>(va, w);
+  if (B != 8) high_parts<B>(w, h);
+  const uint32_t szw = lds32(vszaddr);
+  const float2 sz = __half22float2(*reinterpret_cast<const __half2*>(&szw));  // (s, z)
+  const float wb = p * sz.x * pow2f(100);
+  const float2 w2 = make_float2(wb, wb);
+#pragma unroll
+  for (int i = 0; i < 32; i += 2) {
+    const float2 r = ffma2(w2, make_float2(code_at<B>(w, h, i), code_at<B>(w, h, i + 1)),
+                           make_float2(st.acc[i], st.acc[i + 1]));
+    st.acc[i] = r.x;
+    st.acc[i + 1] = r.y;
+  }
+  st.zacc = fmaf(p, sz.y, st.zacc);
+}
+
+// One page of width class B (P = NIT * keys per iteration tokens) at shared address s0;
+// lane -> (key kl, 32-dim part), and two keys per lane per iteration (kl and kl + KPI)
+// when NIT is even, so that their dependency chains overlap.  Keys past `fill` are
+// empty slots; with positions at spos (masked pages), keys outside [lo, hi] are masked.
 template <int D, int B, int NIT>
 __device__ __forceinline__ void consume_page(uint32_t s0, uint32_t spos, bool masked, int G, int fill, int lo,
                                              int hi, const float (&qp)[32], float sumq, LaneState& st, int lane) {
   constexpr int LPK = D / 32;
   constexpr int KPI = 32 / LPK;
   constexpr int P = NIT * KPI;
+  constexpr int KP = NIT % 2 == 0 ? 2 : 1;  // keys per lane per iteration
   constexpr int rowb = B == 16 ? 2 * D : D * B / 8;  // bytes of one key's row of K (or V)
   const int part = lane % LPK, kl = lane / LPK;
   const int ng = D / G;
@@ -254,84 +325,79 @@ __device__ __forceinline__ void consume_page(uint32_t s0, uint32_t spos, bool ma
   const uint32_t ksz = s0 + 2 * P * rowb + (kl * ng + grp) * 4;           // its (s, z), key kl
   const uint32_t szstep = KPI * ng * 4;
 #pragma unroll 1
-  for (int it = 0; it < NIT; ++it) {
-    const int key = it * KPI + kl;
-    bool valid = key < fill;
-    if (masked) {
-      const int pos = static_cast<int>(lds32(spos + 4 * key));
-      valid = valid && pos >= lo && pos <= hi;
-    }
-    const uint32_t ka = krow + it * KPI * rowb, va = ka + P * rowb;
-    float dot;
-    if (B == 16) {
-      float2 d2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+  for (int it = 0; it < NIT; it += KP) {
+    bool valid[KP];
+    float dot[KP];
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const uint4 u = lds128(ka + 16 * q);
-        d2[0] = ffma2(make_float2(qp[8 * q + 0], qp[8 * q + 1]), make_float2(bf_lo(u.x), bf_hi(u.x)), d2[0]);
-        d2[1] = ffma2(make_float2(qp[8 * q + 2], qp[8 * q + 3]), make_float2(bf_lo(u.y), bf_hi(u.y)), d2[1]);
-        d2[0] = ffma2(make_float2(qp[8 * q + 4], qp[8 * q + 5]), make_float2(bf_lo(u.z), bf_hi(u.z)), d2[0]);
-        d2[1] = ffma2(make_float2(qp[8 * q + 6], qp[8 * q + 7]), make_float2(bf_lo(u.w), bf_hi(u.w)), d2[1]);
+    for (int k = 0; k < KP; ++k) {
+      const int key = (it + k) * KPI + kl;
+      valid[k] = key < fill;
+      if (masked) {
+        const int pos = static_cast<int>(lds32(spos + 4 * key));
+        valid[k] = valid[k] && pos >= lo && pos <= hi;
       }
-      dot = (d2[0].x + d2[0].y) + (d2[1].x + d2[1].y);
-    } else {
-      uint32_t w[B], h[B];
-      lds_codes<B>(ka, w);
-      if (B != 8) high_parts<B>(w, h);
-      const uint32_t szw = lds32(ksz + it * szstep);
-      float2 d2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
-#pragma unroll
-      for (int i = 0; i < 16; ++i)
-        d2[i & 1] = ffma2(make_float2(qp[2 * i], qp[2 * i + 1]),
-                          make_float2(code_at<B>(w, h, 2 * i), code_at<B>(w, h, 2 * i + 1)), d2[i & 1]);
-      const float2 sz = __half22float2(*reinterpret_cast<const __half2*>(&szw));  // (s, z)
-      dot = fmaf(sz.x * pow2f(49), (d2[0].x + d2[0].y) + (d2[1].x + d2[1].y), sz.y * sumq);
+      dot[k] = k_dot<B>(krow + (it + k) * KPI * rowb, ksz + (it + k) * szstep, qp, sumq);
     }
 #pragma unroll
-    for (int o = 1; o < LPK; o <<= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
-    if (valid) {
-      const float p = softmax_step(st, dot);
-      if (B == 16) {
-        const float wv = p * pow2f(-49);
-        const float2 w2 = make_float2(wv, wv);
+    for (int k = 0; k < KP; ++k) {
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const uint4 u = lds128(va + 16 * q);
-          const uint32_t uw[4] = {u.x, u.y, u.z, u.w};
+      for (int o = 1; o < LPK; o <<= 1) dot[k] += __shfl_xor_sync(0xffffffffu, dot[k], o);
+    }
+    // online softmax over the lane's keys: one lazy rescale for both
+    float top = kNegInf;
 #pragma unroll
-          for (int h = 0; h < 4; ++h) {
-            const int i = 8 * q + 2 * h;
-            const float2 r = ffma2(w2, make_float2(bf_lo(uw[h]), bf_hi(uw[h])), make_float2(st.acc[i], st.acc[i + 1]));
-            st.acc[i] = r.x;
-            st.acc[i + 1] = r.y;
-          }
-        }
-      } else {
-        uint32_t w[B], h[B];
-        lds_codes<B>(va, w);
-        if (B != 8) high_parts<B>(w, h);
-        const uint32_t szw = lds32(ksz + it * szstep + P * ng * 4);
-        const float2 sz = __half22float2(*reinterpret_cast<const __half2*>(&szw));  // (s, z)
-        const float wb = p * sz.x * pow2f(100);
-        const float2 w2 = make_float2(wb, wb);
+    for (int k = 0; k < KP; ++k)
+      if (valid[k]) top = fmaxf(top, dot[k]);
+    if (top > st.m + kTau) {
+      const float alpha = fast_exp2(st.m - top);  // 0 when m = -inf
 #pragma unroll
-        for (int i = 0; i < 32; i += 2) {
-          const float2 r = ffma2(w2, make_float2(code_at<B>(w, h, i), code_at<B>(w, h, i + 1)),
-                                 make_float2(st.acc[i], st.acc[i + 1]));
-          st.acc[i] = r.x;
-          st.acc[i + 1] = r.y;
-        }
-        st.zacc = fmaf(p, sz.y, st.zacc);
+      for (int j = 0; j < 32; ++j) st.acc[j] *= alpha;
+      st.l *= alpha;
+      st.zacc *= alpha;
+      st.m = top;
+    }
+#pragma unroll
+    for (int k = 0; k < KP; ++k) {
+      if (valid[k]) {
+        const float p = fast_exp2(dot[k] - st.m);
+        st.l += p;
+        const uint32_t va = krow + (it + k) * KPI * rowb + P * rowb;
+        v_acc<B>(va, ksz + (it + k) * szstep + P * ng * 4, p, st);
       }
     }
   }
 }
 
 // -------------------------------------------------------------------- kernel --
+//
+// One CTA = one producer warp + kNcw consumer warps.  A work unit is (query, split,
+// block of query heads).  The producer plans each unit once (the key range, every
+// class's pages in range, the split's share) and streams it through the CTA's ring of
+// shared memory as stages: the unit's query rows, then for every page the slices of
+// the KV heads the block reads, with the page's slot positions when the page straddles
+// the key range.  Consumers read the stages in order and release each one.
 
-constexpr int kSlots = 8;          // pages a warp may have in flight (one mbarrier each)
-constexpr int kItemsPerWarp = 3;   // splits are made small enough for about this many
-                                   // items per warp (never below the cache's pos_split)
+constexpr int kNcw = 4;           // consumer warps per CTA
+constexpr int kStages = 16;       // stage records a CTA may have in flight
+constexpr int kUnitsPerCta = 3;   // units per CTA of a large call, at most
+constexpr float kMinUnitPositions = 512.f;  // key positions of a large call's unit, at least
+constexpr int kCtasPerSm = 3;
+
+// Stage record, three int4 words written by the producer before it arrives on the
+// stage's full barrier:
+//   a = {meta, ring offset of the stage's bytes, query, lo}
+//   b = {hi (= t), split, splits, unit number of split 0}
+//   c = {first KV slice of the stage (block-relative), KV slices in it, ring offset of
+//        the page's slot positions or -1, 0}
+// meta = class | fill << 2 | flags | head block << 16.
+enum : int {
+  kMask = 1 << 9,     // the page may hold keys outside [lo, hi]: positions follow the slices
+  kFirst = 1 << 10,   // first stage of a unit (its query rows)
+  kLast = 1 << 11,    // last stage of a unit
+  kNoPage = 1 << 12,  // the unit has no page in range
+  kEnd = 1 << 13,     // no more units
+  kQRows = 1 << 14    // the stage holds the unit's query rows
+};
 
 struct AttnKernelArgs {
   LayerArgs a;
@@ -344,7 +410,9 @@ struct AttnKernelArgs {
   const uint16_t* q;
   uint16_t* out;
   float qscale;      // softmax scale * log2(e)
-  int ring_bytes;    // bytes of one warp's ring of shared memory
+  int ring_bytes;    // bytes of the CTA's ring of shared memory
+  int hpu;           // query heads per work unit
+  int scr_floats;    // per-consumer-warp scratch (floats) of the tensor-core path
 };
 
 // Error of a query's arguments, 0 when it is valid.
@@ -360,160 +428,113 @@ __device__ __forceinline__ int query_range(int t, int mode, int w) {
   return mode == TRR_MODE_FULL ? t + 1 : mode == TRR_MODE_LOCAL ? min(w, t + 1) : 0;
 }
 
-// Per-page record the producer writes for the consumer: meta = class | fill << 2 |
-// mask << 9 | flags << 10 (1 first, 2 last, 4 no page) | item entry << 13, the ring
-// offset of the page's slice (then its positions when masked, then the query row on the
-// first page of an item) and the ring bytes to release after the page.  The item's own
-// fields sit once in the warp's item table (kItemSlots entries of 8 words: lo, hi, item,
-// query, head, splits, unit of split 0, KV head); an entry is rewritten only after every
-// record of its previous item has been consumed (at most kSlots records are in flight).
-constexpr int kItemSlots = 8;
-static_assert(kItemSlots >= kSlots, "an item entry outlives the records in flight");
-
 // Shared-memory carve-up of one attention CTA; every region starts 16-byte aligned
 // (mbarriers need 8, bulk-copy destinations 16).
 __host__ __device__ constexpr int align16(int x) { return (x + 15) & ~15; }
-constexpr int kWarpWords = kItemSlots * 8 + 8;  // per-warp shared words: item table, merge
 struct AttnSmem {
-  int rings, recs, bars, words, pre, red, total;
-  __host__ __device__ AttnSmem(int nwarps, int ring_bytes, int n)
-      : rings(0),
-        recs(align16(nwarps * ring_bytes)),
-        bars(recs + align16(nwarps * kSlots * 16)),
-        words(bars + align16(nwarps * kSlots * 8)),
-        pre(words + nwarps * kWarpWords * 4),
+  int ring, recs, sbytes, full, empty, scr, pre, red, flag, total;
+  __host__ __device__ AttnSmem(int ring_bytes, int n, int scr_floats)
+      : ring(0),
+        recs(align16(ring_bytes)),
+        sbytes(recs + kStages * 48),
+        full(sbytes + align16(kStages * 4)),
+        empty(full + kStages * 8),
+        scr(empty + kStages * 8),
+        pre(scr + align16(kNcw * scr_floats * 4)),
         red(pre + align16(4 * (n + 1))),
-        total(red + 16 * 8) {}
+        flag(red + 16 * 8),
+        total(flag + 16) {}
 };
 
-// The plan of one work item as the producer needs it: lane j holds page j's id and meta
-// in registers; the item's fields sit in the warp's shared words (written by lane 0):
-// [0] lo [1] hi [2] item [3] query [4] query head [5] splits [6] unit of split 0 [7] KV head.
-template <int D>
-__device__ __forceinline__ int plan_next_item(const AttnKernelArgs& ka, const int* pre, int n, int wstride, int lane,
-                                           int* next_item, int* wplan, int& wid, int& wmeta, int& kvh) {
-  const LayerArgs& a = ka.a;
-  const int total = pre[n] * a.Hq;
-  while (*next_item < total) {
-    const int i = *next_item;
-    *next_item += wstride;
-    const int u = i / a.Hq, h = i - u * a.Hq;
-    int lo_q = 0, hi_q = n;  // the query of unit u: pre[q] <= u < pre[q + 1]
-    while (hi_q - lo_q > 1) {
-      const int mid = (lo_q + hi_q) >> 1;
-      if (pre[mid] <= u) lo_q = mid;
-      else hi_q = mid;
-    }
-    const int q = lo_q, sp = u - pre[q], ns = pre[q + 1] - pre[q];
-    const int seq = ka.seq_ids[q], t = ka.q_positions[q], mode = ka.modes[q];
-    const int w = ka.windows ? ka.windows[q] : ka.window_scalar;
-    const int err = query_error(a, seq, t, mode, w);
-    if (err || mode == TRR_MODE_SKIP) {  // a zero row; the error of the lowest query
-      uint4* o = reinterpret_cast<uint4*>(ka.out + (static_cast<int64_t>(q) * a.Hq + h) * D);
-      if (lane < D / 8) o[lane] = make_uint4(0, 0, 0, 0);
-      if (err && h == 0 && lane == 0) atomicMin(&a.ctrl[kFirstBadQuery], q * 16 + err);
-      continue;
-    }
-    const int lo = mode == TRR_MODE_FULL ? 0 : max(0, t - w + 1);
-    // per class: pages ending before lo, pages starting at or before t
-    int nt[kClasses];
-#pragma unroll
-    for (int c = 0; c < kClasses; ++c) nt[c] = a.ntok[seq * 4 + c];
-    const bool upper_mask = t < a.last_pos[seq];  // keys after t may be stored
-    int pages[kClasses], first[kClasses], end[kClasses];
-#pragma unroll
-    for (int c = 0; c < kClasses; ++c) {
-      pages[c] = (nt[c] + a.P - 1) / a.P;
-      first[c] = 0;
-      end[c] = pages[c];
-    }
-    const int64_t row0 = static_cast<int64_t>(seq) * 4 * a.MP;
-    // a window's pages are almost always among the last 32 of each class: their ids are
-    // loaded together with the search's first probes
-    int tb[kClasses], ptail[kClasses];
-#pragma unroll
-    for (int c = 0; c < kClasses; ++c) {
-      tb[c] = max(0, pages[c] - 32);
-      ptail[c] = (lo > 0 && tb[c] + lane < pages[c]) ? a.pt[row0 + c * a.MP + tb[c] + lane] : -1;
-    }
-    if (lo > 0) warp_count_below<kClasses>(a.plast + row0, a.MP, pages, lo, first, lane);
-    if (upper_mask) warp_count_below<kClasses>(a.pfirst + row0, a.MP, pages, t + 1, end, lane);
-    // this split's share of each class's pages in range, then one page per lane
-    // split sp of ns takes np / ns pages of the class, one more when sp < np % ns
-    int beg[kClasses], tc[kClasses], npr[kClasses];
-    int T = 0;
-#pragma unroll
-    for (int c = 0; c < kClasses; ++c) {
-      npr[c] = max(0, end[c] - first[c]);
-      const unsigned each = static_cast<unsigned>(npr[c]) / static_cast<unsigned>(ns);
-      const int extra = npr[c] - static_cast<int>(each) * ns;
-      beg[c] = first[c] + sp * static_cast<int>(each) + min(sp, extra);
-      tc[c] = static_cast<int>(each) + (sp < extra ? 1 : 0);
-      T += tc[c];
-    }
-    T = min(T, kItemMaxPages + kClasses);  // the split bound keeps T within this
-    wid = -1;
-    wmeta = 0;
-    const int t1 = tc[0], t2 = t1 + tc[1], t3 = t2 + tc[2];
-    const int c = (lane >= t1) + (lane >= t2) + (lane >= t3);
-    auto pick = [c](const int (&v)[kClasses]) { return c == 0 ? v[0] : c == 1 ? v[1] : c == 2 ? v[2] : v[3]; };
-    const int kid = pick(beg) + lane - (c == 0 ? 0 : c == 1 ? t1 : c == 2 ? t2 : t3);
-    int from_tail = -1;
-#pragma unroll
-    for (int cc = 0; cc < kClasses; ++cc) {
-      const int v = __shfl_sync(0xffffffffu, ptail[cc], (kid - tb[cc]) & 31);
-      if (c == cc && kid >= tb[cc]) from_tail = v;
-    }
-    if (lane < T) {
-      const int f = pick(first);
-      wid = from_tail >= 0 ? from_tail : a.pt[static_cast<int64_t>(seq * 4 + c) * a.MP + kid];
-      const int fill = min(a.P, pick(nt) - kid * a.P);
-      // slot positions are needed on a page that may hold keys outside [lo, t]
-      const bool mask = (lo > 0 && kid == f) || (upper_mask && kid == f + pick(npr) - 1);
-      wmeta = c | (fill << 2) | (mask ? 512 : 0);
-    }
-    kvh = h / (a.Hq / a.Hkv);
-    if (lane == 0) {
-      reinterpret_cast<int4*>(wplan)[0] = make_int4(lo, t, i, q);
-      reinterpret_cast<int4*>(wplan)[1] = make_int4(h, ns, pre[q], kvh);
-    }
-    __syncwarp();
-    return T;
+// Bounded wait that also gives up once *abort is set (by a warp that gave up).
+__device__ __forceinline__ bool mbar_wait_or(uint64_t* bar, uint32_t parity, volatile int* abort) {
+  const uint32_t addr = smem_u32(bar);
+  for (uint32_t i = 0; i < 50000; ++i) {
+    uint32_t done;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n selp.u32 %0, 1, 0, p;\n}"
+        : "=r"(done)
+        : "r"(addr), "r"(parity), "r"(20000)
+        : "memory");
+    if (done) return true;
+    if (*abort) return false;
   }
-  return -1;
+  return false;
 }
 
-template <int D, int P>
-__global__ void __launch_bounds__(256, 2) attn_kernel(const __grid_constant__ AttnKernelArgs ka) {
-  constexpr int LPK = D / 32;  // lanes per key
-  constexpr int KPI = 32 / LPK;  // keys per warp iteration
-  constexpr int DPL = D / 32;  // dimensions per lane after the merge
-  const LayerArgs& a = ka.a;
-  extern __shared__ __align__(128) uint8_t smem[];
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
-  const int n = ka.n;
-  const int qrow = D * 2;  // bytes of one query row
-  const int R = ka.ring_bytes;
-  const AttnSmem lay(nwarps, R, n);  // [rings][slot records][mbarriers][unit prefix][scratch]
-  uint8_t* ring = smem + lay.rings + warp * R;
-  int4* recs = reinterpret_cast<int4*>(smem + lay.recs) + warp * kSlots;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + lay.bars) + warp * kSlots;
-  int* pre = reinterpret_cast<int*>(smem + lay.pre);
-  int* witems = reinterpret_cast<int*>(smem + lay.words) + warp * kWarpWords;  // item table
-  int* wmerge = witems + kItemSlots * 8;
-  long long* red = reinterpret_cast<long long*>(smem + lay.red);
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
 
-  if (lane == 0) {
+// Pages of split sp (of ns) of a query of sequence seq over key positions [lo, t]:
+// returns their number T (<= kItemMaxPages + 4); lane j < T gets page j's id in wid and
+// class | fill << 2 | kMask in wmeta.  Pages are listed class by class, each class's in
+// position order; split sp of ns takes np / ns of a class's np pages in range, one more
+// when sp < np % ns.
+__device__ __forceinline__ int plan_split(const LayerArgs& a, int P, int seq, int lo, int t, int sp, int ns,
+                                          int lane, int& wid, int& wmeta) {
+  int nt[kClasses];
 #pragma unroll
-    for (int i = 0; i < kSlots; ++i) mbar_init(&bars[i], 1);
-    fence_barrier_init();
+  for (int c = 0; c < kClasses; ++c) nt[c] = a.ntok[seq * 4 + c];
+  const bool upper_mask = t < a.last_pos[seq];  // keys after t may be stored
+  int pages[kClasses], first[kClasses], end[kClasses];
+#pragma unroll
+  for (int c = 0; c < kClasses; ++c) {
+    pages[c] = (nt[c] + P - 1) / P;
+    first[c] = 0;
+    end[c] = pages[c];
   }
-  pdl_wait();
-  pdl_trigger();
+  const int64_t row0 = static_cast<int64_t>(seq) * 4 * a.MP;
+  // a window's pages are almost always among the last 32 of each class: their ids are
+  // loaded together with the search's first probes
+  int tb[kClasses], ptail[kClasses];
+#pragma unroll
+  for (int c = 0; c < kClasses; ++c) {
+    tb[c] = max(0, pages[c] - 32);
+    ptail[c] = tb[c] + lane < pages[c] ? a.pt[row0 + c * a.MP + tb[c] + lane] : -1;
+  }
+  if (lo > 0) warp_count_below<kClasses>(a.plast + row0, a.MP, pages, lo, first, lane);
+  if (upper_mask) warp_count_below<kClasses>(a.pfirst + row0, a.MP, pages, t + 1, end, lane);
+  int beg[kClasses], tc[kClasses], npr[kClasses];
+  int T = 0;
+#pragma unroll
+  for (int c = 0; c < kClasses; ++c) {
+    npr[c] = max(0, end[c] - first[c]);
+    const unsigned each = static_cast<unsigned>(npr[c]) / static_cast<unsigned>(ns);
+    const int extra = npr[c] - static_cast<int>(each) * ns;
+    beg[c] = first[c] + sp * static_cast<int>(each) + min(sp, extra);
+    tc[c] = static_cast<int>(each) + (sp < extra ? 1 : 0);
+    T += tc[c];
+  }
+  T = min(T, kItemMaxPages + kClasses);  // the split bound keeps T within this
+  wid = -1;
+  wmeta = 0;
+  const int t1 = tc[0], t2 = t1 + tc[1], t3 = t2 + tc[2];
+  const int c = (lane >= t1) + (lane >= t2) + (lane >= t3);
+  auto pick = [c](const int (&v)[kClasses]) { return c == 0 ? v[0] : c == 1 ? v[1] : c == 2 ? v[2] : v[3]; };
+  const int kid = pick(beg) + lane - (c == 0 ? 0 : c == 1 ? t1 : c == 2 ? t2 : t3);
+  int from_tail = -1;
+#pragma unroll
+  for (int cc = 0; cc < kClasses; ++cc) {
+    const int v = __shfl_sync(0xffffffffu, ptail[cc], (kid - tb[cc]) & 31);
+    if (c == cc && kid >= tb[cc]) from_tail = v;
+  }
+  if (lane < T) {
+    const int f = pick(first);
+    wid = from_tail >= 0 ? from_tail : a.pt[static_cast<int64_t>(seq * 4 + c) * a.MP + kid];
+    const int fill = min(P, pick(nt) - kid * P);
+    // slot positions are needed on a page that may hold keys outside [lo, t]
+    const bool mask = (lo > 0 && kid == f) || (upper_mask && kid == f + pick(npr) - 1);
+    wmeta = c | (fill << 2) | (mask ? kMask : 0);
+  }
+  return T;
+}
 
-  // ---------------------------------------------------------- work units --
-  // Every CTA computes the same split of the call: query q gets ns_q splits from its key
-  // range; pre[q] numbers its first unit, pre[n] counts them all.
+// The work units of a call, computed the same way by every CTA: query q gets ns_q
+// splits from its key range; pre[q] numbers its first split, pre[n] counts them all.
+__device__ __forceinline__ void plan_units(const AttnKernelArgs& ka, int P, int NQB, int* pre, long long* red) {
+  const LayerArgs& a = ka.a;
+  const int n = ka.n, lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
   long long rsum = 0;
   for (int q = threadIdx.x; q < n; q += blockDim.x) {
     const int seq = ka.seq_ids[q], t = ka.q_positions[q], mode = ka.modes[q];
@@ -528,114 +549,339 @@ __global__ void __launch_bounds__(256, 2) attn_kernel(const __grid_constant__ At
   __syncthreads();
   rsum = 0;
   for (int k = 0; k < nwarps; ++k) rsum += red[k];
-  // splits small enough for about kItemsPerWarp items per warp, never below pos_split
-  // (binary32 arithmetic: the same result in every CTA, and it only sizes the splits)
-  const float want = static_cast<float>(gridDim.x * nwarps * kItemsPerWarp);
-  const float by_work = ceilf(static_cast<float>(rsum) * static_cast<float>(a.Hq) / want);
+  // Split size: a small call gets about one unit per CTA (its units are latency-bound
+  // chains, and a second unit on a CTA doubles the call); a large one up to
+  // kUnitsPerCta per CTA, each of at least kMinUnitPositions positions per head block
+  // (the producer plans the next unit while the consumers work on this one); never
+  // below pos_split.  Binary32 arithmetic: the same result in every CTA, and it only
+  // sizes the splits.
+  const float ctas = static_cast<float>(gridDim.x);
+  const float rs = static_cast<float>(rsum) * static_cast<float>(NQB);
+  const float want = fmaxf(0.8f * ctas, fminf(static_cast<float>(kUnitsPerCta) * ctas, rs / kMinUnitPositions));
+  const float by_work = ceilf(rs / want);
   const int pos_split = by_work > static_cast<float>(a.pos_split) ? static_cast<int>(fminf(by_work, 1073741824.f))
                                                                    : a.pos_split;
-  {
-    const int chunk = (n + blockDim.x - 1) / blockDim.x;
-    const int q0 = min(n, static_cast<int>(threadIdx.x) * chunk), q1 = min(n, q0 + chunk);
-    int mine = 0;
-    for (int q = q0; q < q1; ++q) mine += splits_of(pre[q], pos_split, a.P, a.s_cap);
-    int incl = mine;
+  const int chunk = (n + blockDim.x - 1) / blockDim.x;
+  const int q0 = min(n, static_cast<int>(threadIdx.x) * chunk), q1 = min(n, q0 + chunk);
+  int mine = 0;
+  for (int q = q0; q < q1; ++q) mine += splits_of(pre[q], pos_split, P, a.s_cap);
+  int incl = mine;
 #pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const int v = __shfl_up_sync(0xffffffffu, incl, o);
-      if (lane >= o) incl += v;
-    }
-    __syncthreads();  // every read of red above is done
-    if (lane == 31) red[8 + warp] = incl;
-    __syncthreads();
-    int off = incl - mine;
-    for (int k = 0; k < warp; ++k) off += static_cast<int>(red[8 + k]);
-    for (int q = q0; q < q1; ++q) {
-      const int ns = splits_of(pre[q], pos_split, a.P, a.s_cap);
-      pre[q] = off;
-      off += ns;
-    }
-    if (threadIdx.x == blockDim.x - 1) pre[n] = off;
-    __syncthreads();
+  for (int o = 1; o < 32; o <<= 1) {
+    const int v = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += v;
   }
-  const int wstride = gridDim.x * nwarps;
+  __syncthreads();  // every read of red above is done
+  if (lane == 31) red[8 + warp] = incl;
+  __syncthreads();
+  int off = incl - mine;
+  for (int k = 0; k < warp; ++k) off += static_cast<int>(red[8 + k]);
+  for (int q = q0; q < q1; ++q) {
+    const int ns = splits_of(pre[q], pos_split, P, a.s_cap);
+    pre[q] = off;
+    off += ns;
+  }
+  if (threadIdx.x == blockDim.x - 1) pre[n] = off;
+  __syncthreads();
+}
 
-  // ------------------------------------------------------------ producer --
-  // Items are dealt round-robin; consecutive warps take consecutive heads of one unit,
-  // so the planning loads of a unit mostly hit in L1.
-  int next_item = blockIdx.x * nwarps + warp;
-  int wid = -1, wmeta = 0;             // the producer's item: page id / meta of page `lane`
-  int p_T = 0;                         // pages of the producer's item
-  int p_kvh = 0;                       // its KV head
-  int pf = 0;                          // next page of the producer's item
-  bool pvalid = false;
-  uint32_t issued = 0, consumed = 0;   // pages issued / consumed by this warp
-  uint32_t started = 0;                // items started by this warp (item table index)
-  int head = 0, used = 0;              // ring: next free offset, bytes held
+// Everything the producer and consumers of one CTA share.
+struct CtaRing {
+  uint8_t* ring;
+  int4* recs;
+  int* sbytes;
+  uint64_t* full;
+  uint64_t* empty;
+  volatile int* abort_flag;
+  int R;
+};
 
-  auto start_item = [&]() -> bool {
-    p_T = plan_next_item<D>(ka, pre, n, wstride, lane, &next_item, witems + (started % kItemSlots) * 8, wid,
-                            wmeta, p_kvh);
-    pf = 0;
-    if (p_T < 0) return false;
-    ++started;
+// The producer warp: takes units (the CTA's own first, then from a call-wide counter),
+// plans each and pushes its stages; ends with an end record.
+template <int D>
+__device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, int NQB, const int* pre,
+                                             const CtaRing& cr, int lane) {
+  const LayerArgs& a = ka.a;
+  const int n = ka.n, g = a.Hq / a.Hkv, R = cr.R;
+  const int total = pre[n] * NQB;
+  uint32_t pushed = 0, released = 0;  // stages pushed / seen released by the consumers
+  int rhead = 0, rused = 0;           // ring: next free offset, bytes held
+  bool ok = true;
+  // wait for the oldest stage in flight to be released and take back its bytes
+  auto release_one = [&]() -> bool {
+    const uint32_t slot = released % kStages;
+    if (!mbar_wait_or(&cr.empty[slot], (released / kStages) & 1, cr.abort_flag)) return false;
+    rused -= cr.sbytes[slot];
+    ++released;
     return true;
   };
-  // start the copies of the producer's next page if a slot and ring space are free
-  auto try_issue = [&]() -> bool {
-    if (issued - consumed >= kSlots) return false;  // first: an item entry is reused only
-                                                    // once fewer records are in flight
-    if (!pvalid) {
-      pvalid = start_item();
-      if (!pvalid) return false;
+  // a slot and `need` contiguous ring bytes; -1 when a wait gave up
+  auto reserve = [&](int need, int& taken) -> int {
+    for (;;) {
+      if (pushed - released < static_cast<uint32_t>(kStages)) {
+        if (rused == 0) rhead = 0;  // an empty ring can start anywhere
+        int off = rhead, waste = 0;
+        if (off + need > R) {
+          waste = R - off;
+          off = 0;
+        }
+        if (rused + waste + need <= R) {
+          rhead = off + need;
+          rused += waste + need;
+          taken = waste + need;
+          return off;
+        }
+      }
+      if (pushed == released || !release_one()) return -1;
     }
-    const bool first = pf == 0;
-    int meta = 0, id = -1, bytes_page = 0;
-    if (p_T > 0) {
-      id = __shfl_sync(0xffffffffu, wid, pf);
-      meta = __shfl_sync(0xffffffffu, wmeta, pf);
-      bytes_page = a.slice[meta & 3] + ((meta & 512) ? 4 * P : 0);
-    }
-    const int need = bytes_page + (first ? qrow : 0);
-    if (used == 0) head = 0;  // an empty ring can start anywhere
-    int off = head, waste = 0;
-    if (off + need > R) {
-      waste = R - off;
-      off = 0;
-    }
-    if (used + waste + need > R) return false;
-    head = off + need;
-    used += waste + need;
-    const uint32_t slot = issued % kSlots;
-    const int flags = (first ? 1 : 0) | (pf + 1 >= p_T ? 2 : 0) | (p_T == 0 ? 4 : 0);
-    // The record, then the arrival.  The ring is written only by bulk copies; the warp's
-    // earlier reads of these bytes have completed (their values were consumed), and the
-    // record reaches the consumer through the mbarrier's release / acquire, so no proxy
-    // fence is needed here.
+  };
+  // the record of the stage taking slot pushed % kStages, then its arrival with the
+  // bytes its copies will bring (the copies follow, issued by lane 0)
+  auto push = [&](int4 ra, int4 rb, int4 rc, int taken, int tx) -> uint32_t {
+    const uint32_t slot = pushed % kStages;
     if (lane == 0) {
-      const int entry = (started - 1) % kItemSlots;
-      recs[slot] = make_int4(meta | (flags << 10) | (entry << 13), off, waste + need, 0);
-      mbar_arrive_expect_tx(&bars[slot], need);
-      const int c = meta & 3;
-      if (p_T > 0) {
+      cr.recs[slot * 3 + 0] = ra;
+      cr.recs[slot * 3 + 1] = rb;
+      cr.recs[slot * 3 + 2] = rc;
+      cr.sbytes[slot] = taken;
+      mbar_arrive_expect_tx(&cr.full[slot], static_cast<uint32_t>(tx));
+    }
+    ++pushed;
+    return slot;
+  };
+
+  int u = blockIdx.x;  // the first unit is the CTA's own; later ones come from the counter
+  while (u < total) {
+    int u_next = 0;
+    if (lane == 0) u_next = static_cast<int>(gridDim.x) + atomicAdd(&a.ctrl[kNextUnit], 1);  // used last
+    const int un = u / NQB, qb = u - un * NQB;
+    int lo_q = 0, hi_q = n;  // the query of split un: pre[q] <= un < pre[q + 1]
+    while (hi_q - lo_q > 1) {
+      const int mid = (lo_q + hi_q) >> 1;
+      if (pre[mid] <= un) lo_q = mid;
+      else hi_q = mid;
+    }
+    const int q = lo_q, sp = un - pre[q], ns = pre[q + 1] - pre[q];
+    const int seq = ka.seq_ids[q], t = ka.q_positions[q], mode = ka.modes[q];
+    const int w = ka.windows ? ka.windows[q] : ka.window_scalar;
+    const int err = query_error(a, seq, t, mode, w);
+    const int h0 = qb * ka.hpu, nh = min(ka.hpu, a.Hq - h0);
+    if (err || mode == TRR_MODE_SKIP) {  // zero rows; the error of the lowest query
+      uint4* o = reinterpret_cast<uint4*>(ka.out + (static_cast<int64_t>(q) * a.Hq + h0) * D);
+      for (int i = lane; i < nh * D / 8; i += 32) o[i] = make_uint4(0, 0, 0, 0);
+      if (err && qb == 0 && lane == 0) atomicMin(&a.ctrl[kFirstBadQuery], q * 16 + err);
+    } else {
+      const int lo = mode == TRR_MODE_FULL ? 0 : max(0, t - w + 1);
+      int wid, wmeta;
+      const int T = plan_split(a, P, seq, lo, t, sp, ns, lane, wid, wmeta);
+      const int kv0 = h0 / g, nkv = (h0 + nh - 1) / g - kv0 + 1;
+      const int4 rb = make_int4(t, sp, ns, pre[q]);
+      {  // the unit's query rows
+        const int need = nh * D * 2;
+        int taken = 0;
+        const int off = reserve(need, taken);
+        if (off < 0) {
+          ok = false;
+          break;
+        }
+        const int meta = kQRows | kFirst | (T == 0 ? (kLast | kNoPage) : 0) | (qb << 16);
+        const uint32_t slot = push(make_int4(meta, off, q, lo), rb, make_int4(0, 0, -1, 0), taken, need);
+        if (lane == 0)
+          bulk_g2s(cr.ring + off, ka.q + (static_cast<int64_t>(q) * a.Hq + h0) * D, need, &cr.full[slot]);
+      }
+      for (int j = 0; j < T && ok; ++j) {
+        const int id = __shfl_sync(0xffffffffu, wid, j);
+        const int pm = __shfl_sync(0xffffffffu, wmeta, j);
+        const int c = pm & 3, slice = a.slice[c];
+        const int posb = (pm & kMask) ? 4 * P : 0;
+        const int maxk = max(1, (R / 2 - posb) / slice);  // KV slices per stage
         const uint8_t* page = a.pool[c] + static_cast<int64_t>(id) * a.page_bytes[c];
-        bulk_g2s(ring + off, page + a.hdr + static_cast<int64_t>(p_kvh) * a.slice[c], a.slice[c], &bars[slot]);
-        if (meta & 512) bulk_g2s(ring + off + a.slice[c], page, 4 * P, &bars[slot]);
+        for (int k0 = 0; k0 < nkv; k0 += maxk) {
+          const int nk = min(maxk, nkv - k0);
+          const int need = nk * slice + posb;
+          int taken = 0;
+          const int off = reserve(need, taken);
+          if (off < 0) {
+            ok = false;
+            break;
+          }
+          const bool last = j == T - 1 && k0 + nk >= nkv;
+          const int meta = pm | (last ? kLast : 0) | (qb << 16);
+          const uint32_t slot =
+              push(make_int4(meta, off, q, lo), rb, make_int4(k0, nk, posb ? off + nk * slice : -1, 0), taken, need);
+          if (lane == 0) {
+            bulk_g2s(cr.ring + off, page + a.hdr + static_cast<int64_t>(kv0 + k0) * slice, nk * slice, &cr.full[slot]);
+            if (posb) bulk_g2s(cr.ring + off + nk * slice, page, posb, &cr.full[slot]);
+          }
+        }
       }
-      if (first) {
-        const int* it = witems + entry * 8;
-        bulk_g2s(ring + off + bytes_page, ka.q + (static_cast<int64_t>(it[3]) * a.Hq + it[4]) * D, qrow, &bars[slot]);
-      }
+      if (!ok) break;
     }
     __syncwarp();
-    ++issued;
-    ++pf;
-    if (pf >= p_T) pvalid = false;
-    return true;
-  };
+    u = __shfl_sync(0xffffffffu, u_next, 0);
+  }
+  if (ok) {
+    int taken = 0;
+    if (reserve(0, taken) < 0) ok = false;
+    else push(make_int4(kEnd, 0, 0, 0), make_int4(0, 0, 0, 0), make_int4(0, 0, -1, 0), taken, 0);
+  }
+  if (!ok) {  // a wait gave up: stop the consumers, then let every copy in flight land
+    if (lane == 0) {
+      *cr.abort_flag = 1;
+      set_status(a.ctrl, TRR_ERR_TIMEOUT);
+    }
+    for (uint32_t s = released; s < pushed; ++s) mbar_wait(&cr.full[s % kStages], (s / kStages) & 1);
+  }
+}
 
-  // ------------------------------------------------------------ consumer --
+// Merges `count` partial rows at p0, p0 + stride, ...: the common maximum Mx, the
+// weighted sum of L and the weighted rows (lane holds dims lane * DPL ..).
+template <int D>
+__device__ __forceinline__ void merge_partials(const float* p0, int64_t stride, int count, int lane, float& Mx,
+                                               float& Ls, float (&acc_o)[D / 32]) {
+  constexpr int DPL = D / 32;
+  Mx = kNegInf;
+  for (int s = lane; s < count; s += 32) Mx = fmaxf(Mx, __ldcg(p0 + s * stride + D));
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) Mx = fmaxf(Mx, __shfl_xor_sync(0xffffffffu, Mx, o));
+  Ls = 0.f;
+#pragma unroll
+  for (int j = 0; j < DPL; ++j) acc_o[j] = 0.f;
+  for (int s0 = 0; s0 < count; s0 += 32) {
+    float wl = 0.f;  // lane s: weight of row s0 + s
+    if (s0 + lane < count) {
+      const float2 ml = __ldcg(reinterpret_cast<const float2*>(p0 + (s0 + lane) * stride + D));
+      wl = (ml.x == kNegInf) ? 0.f : fast_exp2(ml.x - Mx);
+      Ls = fmaf(wl, ml.y, Ls);
+    }
+    const int cnt = min(32, count - s0);
+#pragma unroll 8
+    for (int s = 0; s < cnt; ++s) {
+      const float wgt = __shfl_sync(0xffffffffu, wl, s);
+      const float* ps = p0 + (s0 + s) * stride + lane * DPL;
+#pragma unroll
+      for (int j = 0; j < DPL; ++j) acc_o[j] = fmaf(wgt, __ldcg(ps + j), acc_o[j]);
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) Ls += __shfl_xor_sync(0xffffffffu, Ls, o);
+}
+
+// Counts this warp's arrival on *counter (release of its partial stores, acquire of
+// the others'); true for the last of `expected` arrivals, which resets the counter.
+__device__ __forceinline__ bool arrive_last(int* counter, int expected, int lane) {
+  __syncwarp();
+  int arrivals = 0;
+  if (lane == 0) arrivals = atom_add_acq_rel(counter, 1);
+  __syncwarp();
+  arrivals = __shfl_sync(0xffffffffu, arrivals, 0);
+  if (arrivals != expected - 1) return false;
+  if (lane == 0) *counter = 0;  // ready for the next call
+  return true;
+}
+
+// A (query, head) row at its end: lane holds DPL consecutive dims from dim0 of the
+// unnormalised sum acc = sum_j p_j v_j (weights relative to max M, log2 domain) and the
+// row's weight sum L.  One split: the bf16 row.  Otherwise the split's fp32 partial,
+// merged in two levels: the last split of each group of kMergeGroup to arrive folds the
+// group into the group's first partial, and the last group to arrive merges the groups
+// into the row (one level when nsplit <= kMergeGroup).
+template <int D>
+__device__ __forceinline__ void store_or_merge(const AttnKernelArgs& ka, const float* v, int dim0, float M, float L,
+                                               int sp, int qi, int qh, int nsplit, int base, int lane) {
+  constexpr int DPL = D / 32;
+  const LayerArgs& a = ka.a;
+  const int64_t orow = (static_cast<int64_t>(qi) * a.Hq + qh) * D;
+  if (nsplit == 1) {
+    const float inv = L > 0.f ? 1.f / L : 0.f;
+#pragma unroll
+    for (int j = 0; j < DPL; j += 2)
+      *reinterpret_cast<__nv_bfloat162*>(ka.out + orow + dim0 + j) = __floats2bfloat162_rn(v[j] * inv, v[j + 1] * inv);
+    return;
+  }
+  const int64_t sstride = static_cast<int64_t>(a.Hq) * (D + 4);
+  float* p0 = a.part + (static_cast<int64_t>(base) * a.Hq + qh) * (D + 4);  // split 0's partial
+  float* pp = p0 + sp * sstride;
+#pragma unroll
+  for (int j = 0; j < DPL; j += 2) *reinterpret_cast<float2*>(pp + dim0 + j) = make_float2(v[j], v[j + 1]);
+  if (lane == 0) *reinterpret_cast<float2*>(pp + D) = make_float2(M, L);
+  int* counters = a.cnt + (static_cast<int64_t>(qi) * a.Hq + qh) * a.cnt_stride;
+  float Mx, Ls, acc_o[DPL];
+  int ngroups = nsplit, gstride = 1;
+  if (nsplit > kMergeGroup) {
+    const int gr = sp / kMergeGroup, g0 = gr * kMergeGroup, gn = min(kMergeGroup, nsplit - g0);
+    if (!arrive_last(counters + 1 + gr, gn, lane)) return;
+    float* pg = p0 + g0 * sstride;
+    merge_partials<D>(pg, sstride, gn, lane, Mx, Ls, acc_o);
+    __syncwarp();  // every lane has read the group's rows before the first is overwritten
+#pragma unroll
+    for (int j = 0; j < DPL; ++j) __stcg(pg + lane * DPL + j, acc_o[j]);
+    if (lane == 0) __stcg(reinterpret_cast<float2*>(pg + D), make_float2(Mx, Ls));
+    ngroups = (nsplit + kMergeGroup - 1) / kMergeGroup;
+    gstride = kMergeGroup;
+  }
+  if (!arrive_last(counters, ngroups, lane)) return;
+  merge_partials<D>(p0, sstride * gstride, ngroups, lane, Mx, Ls, acc_o);
+  const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
+#pragma unroll
+  for (int j = 0; j < DPL; j += 2)
+    *reinterpret_cast<__nv_bfloat162*>(ka.out + orow + lane * DPL + j) =
+        __floats2bfloat162_rn(acc_o[j] * inv, acc_o[j + 1] * inv);
+}
+
+// ------------------------------------------------- CUDA-core consumer (MHA) --
+// Warp cw computes query head (block * kNcw + cw): lane pair (key, half) of a 64-wide
+// head (four lanes for 128) dequantises in registers and keeps its own online softmax.
+
+// The end of a unit for a CUDA-core consumer: merge the lanes' states, then store.
+template <int D>
+__device__ __forceinline__ void finish_unit(const AttnKernelArgs& ka, LaneState& st, int cur_cls, int sp, int qi,
+                                            int qh, int nsplit, int base, int lane) {
+  constexpr int LPK = D / 32;  // lanes per key
+  constexpr int DPL = D / 32;  // dimensions per lane after the merge
   const int part = lane % LPK, kl = lane / LPK;
+  // rescale to the common maximum, then reduce-scatter over the key lanes: each
+  // halving step keeps half of the 32 dims and sends the other half to the partner
+  acc_to_neutral(st.acc, cur_cls);
+  float M = st.m;
+#pragma unroll
+  for (int o = LPK; o < 32; o <<= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+  const float f = (st.m == kNegInf) ? 0.f : fast_exp2(st.m - M);
+  float L = st.l * f;
+#pragma unroll
+  for (int o = LPK; o < 32; o <<= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
+  {
+    const float2 s49 = make_float2(pow2f(49) * f, pow2f(49) * f), zf = make_float2(st.zacc * f, st.zacc * f);
+#pragma unroll
+    for (int j = 0; j < 32; j += 2) {
+      const float2 r = __ffma2_rn(make_float2(st.acc[j], st.acc[j + 1]), s49, zf);
+      st.acc[j] = r.x;
+      st.acc[j + 1] = r.y;
+    }
+  }
+#pragma unroll
+  for (int width = 16, o = 16; o >= LPK; width >>= 1, o >>= 1) {
+    const bool upper = lane & o;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      if (i < width) {
+        const float keep = upper ? st.acc[width + i] : st.acc[i];
+        const float give = upper ? st.acc[i] : st.acc[width + i];
+        st.acc[i] = keep + __shfl_xor_sync(0xffffffffu, give, o);
+      }
+    }
+  }
+  // lane (kl, part) now holds dims part*32 + DPL*kl .. + DPL-1 in acc[0 .. DPL-1]
+  store_or_merge<D>(ka, st.acc, part * 32 + DPL * kl, M, L, sp, qi, qh, nsplit, base, lane);
+}
+
+template <int D, int P>
+__device__ __forceinline__ void run_consumer_cc(const AttnKernelArgs& ka, const CtaRing& cr, int cw, int lane) {
+  constexpr int LPK = D / 32;    // lanes per key
+  constexpr int KPI = 32 / LPK;  // keys per warp iteration
+  const LayerArgs& a = ka.a;
+  const int g = a.Hq / a.Hkv;
+  const int part = lane % LPK;
   LaneState st;
   float qp[32];
   float sumq = 0.f;
@@ -643,171 +889,616 @@ __global__ void __launch_bounds__(256, 2) attn_kernel(const __grid_constant__ At
   st.m = kNegInf;
   st.l = 0.f;
   st.zacc = 0.f;
-  // The merge of an item's lanes and splits, once its last page is consumed.
-  bool merge_pending = false;
-  auto merge_item = [&]() {
-    const int4 mr = reinterpret_cast<const int4*>(wmerge)[0];  // item, query, head, splits
-    const int m_item = mr.x, m_qi = mr.y, m_qh = mr.z, m_nsplit = mr.w, m_base = wmerge[4];
-    // merge the lanes that share a part.  Rescale to the common maximum, then
-    // reduce-scatter over the key lanes: each halving step keeps half of the 32 dims
-    // and sends the other half to the partner lane.
-    acc_to_neutral(st.acc, cur_cls);
-    float M = st.m;
 #pragma unroll
-    for (int o = LPK; o < 32; o <<= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-    const float f = (st.m == kNegInf) ? 0.f : fast_exp2(st.m - M);
-    float L = st.l * f;
-#pragma unroll
-    for (int o = LPK; o < 32; o <<= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
-    {
-      const float2 s49 = make_float2(pow2f(49) * f, pow2f(49) * f), zf = make_float2(st.zacc * f, st.zacc * f);
-#pragma unroll
-      for (int j = 0; j < 32; j += 2) {
-        const float2 r = __ffma2_rn(make_float2(st.acc[j], st.acc[j + 1]), s49, zf);
-        st.acc[j] = r.x;
-        st.acc[j + 1] = r.y;
-      }
-    }
-#pragma unroll
-    for (int width = 16, o = 16; o >= LPK; width >>= 1, o >>= 1) {
-      const bool upper = lane & o;
-#pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        if (i < width) {
-          const float keep = upper ? st.acc[width + i] : st.acc[i];
-          const float give = upper ? st.acc[i] : st.acc[width + i];
-          st.acc[i] = keep + __shfl_xor_sync(0xffffffffu, give, o);
-        }
-      }
-    }
-    // lane (kl, part) now holds dims part*32 + DPL*kl .. + DPL-1 in acc[0 .. DPL-1]
-    const int dim0 = part * 32 + DPL * kl;
-    const int64_t orow = (static_cast<int64_t>(m_qi) * a.Hq + m_qh) * D;
-    if (m_nsplit == 1) {
-      const float inv = L > 0.f ? 1.f / L : 0.f;
-#pragma unroll
-      for (int j = 0; j < DPL; j += 2)
-        *reinterpret_cast<__nv_bfloat162*>(ka.out + orow + dim0 + j) =
-            __floats2bfloat162_rn(st.acc[j] * inv, st.acc[j + 1] * inv);
-      return;
-    }
-    // a partial at the item's index; the last split of (query, head) to arrive merges
-    float* pp = a.part + static_cast<int64_t>(m_item) * (D + 4);
-#pragma unroll
-    for (int j = 0; j < DPL; j += 2)
-      *reinterpret_cast<float2*>(pp + dim0 + j) = make_float2(st.acc[j], st.acc[j + 1]);
-    if (lane == 0) *reinterpret_cast<float2*>(pp + D) = make_float2(M, L);
-    // the warp's partial stores happen before lane 0's release; the last arriver's
-    // acquire happens before its lanes read the other splits' partials
-    __syncwarp();
-    int arrivals = 0;
-    int* counter = a.cnt + static_cast<int64_t>(m_qi) * a.Hq + m_qh;
-    if (lane == 0) arrivals = atom_add_acq_rel(counter, 1);
-    __syncwarp();
-    arrivals = __shfl_sync(0xffffffffu, arrivals, 0);
-    if (arrivals != m_nsplit - 1) return;
-    const float* p0 = a.part + (static_cast<int64_t>(m_base) * a.Hq + m_qh) * (D + 4);
-    const int64_t sstride = static_cast<int64_t>(a.Hq) * (D + 4);
-    float Mx = kNegInf;
-    for (int s = lane; s < m_nsplit; s += 32) Mx = fmaxf(Mx, __ldcg(p0 + s * sstride + D));
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) Mx = fmaxf(Mx, __shfl_xor_sync(0xffffffffu, Mx, o));
-    float Ls = 0.f, acc_o[DPL];
-#pragma unroll
-    for (int j = 0; j < DPL; ++j) acc_o[j] = 0.f;
-#pragma unroll 4
-    for (int s = 0; s < m_nsplit; ++s) {
-      const float* ps = p0 + s * sstride;
-      const float2 ml = __ldcg(reinterpret_cast<const float2*>(ps + D));
-      const float wgt = (ml.x == kNegInf) ? 0.f : fast_exp2(ml.x - Mx);
-      Ls = fmaf(wgt, ml.y, Ls);
-#pragma unroll
-      for (int j = 0; j < DPL; ++j) acc_o[j] = fmaf(wgt, __ldcg(ps + lane * DPL + j), acc_o[j]);
-    }
-    const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
-#pragma unroll
-    for (int j = 0; j < DPL; j += 2)
-      *reinterpret_cast<__nv_bfloat162*>(ka.out + orow + lane * DPL + j) =
-          __floats2bfloat162_rn(acc_o[j] * inv, acc_o[j + 1] * inv);
-    if (lane == 0) *counter = 0;  // ready for the next call
-  };
-
-  for (;;) {
-    // refill first, so that the next item's copies fly while this one merges; the one
-    // place the producer plans items
-    while (try_issue()) {
-    }
-    if (merge_pending) {
-      merge_pending = false;
-      merge_item();
-    }
-    if (consumed == issued) break;
-    const uint32_t g = consumed;
-    const uint32_t slot = g % kSlots;
-    const bool arrived = mbar_wait(&bars[slot], (g / kSlots) & 1);
+  for (int j = 0; j < 32; ++j) st.acc[j] = 0.f;
+  // the current unit
+  int u_q = 0, u_h = 0, u_kvi = 0, u_lo = 0, u_hi = 0, u_sp = 0, u_ns = 1, u_base = 0;
+  bool active = false;
+  for (uint32_t s = 0;; ++s) {
+    const uint32_t slot = s % kStages;
+    const bool arrived = mbar_wait_or(&cr.full[slot], (s / kStages) & 1, cr.abort_flag);
     if (!__all_sync(0xffffffffu, arrived)) {  // give up together, never half a warp
-      for (uint32_t r = g + 1; r < issued; ++r) mbar_wait(&bars[r % kSlots], (r / kSlots) & 1);
-      if (lane == 0) set_status(a.ctrl, TRR_ERR_TIMEOUT);
+      if (lane == 0) {
+        *cr.abort_flag = 1;
+        set_status(a.ctrl, TRR_ERR_TIMEOUT);
+      }
       break;
     }
-    const int4 r0 = recs[slot];
-    const int meta = r0.x, flags = (meta >> 10) & 7;
-    const int* item_words = witems + (meta >> 13) * 8;  // lo, hi, item, query, head, splits, base
-    if (flags & 1) {  // first page of an item: query row and a fresh state
-      const int qoff = r0.y + ((flags & 4) ? 0 : a.slice[meta & 3] + ((meta & 512) ? 4 * P : 0));
-      const uint32_t qa = smem_u32(ring + qoff + part * 64);
-      const float2 qs2 = make_float2(ka.qscale, ka.qscale);
-      float2 sq2 = make_float2(0.f, 0.f);
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const uint4 u = lds128(qa + 16 * q);
-        const uint32_t wv[4] = {u.x, u.y, u.z, u.w};
-#pragma unroll
-        for (int h = 0; h < 4; ++h) {
-          const float2 r = __fmul2_rn(make_float2(bf_lo(wv[h]), bf_hi(wv[h])), qs2);
-          qp[8 * q + 2 * h] = r.x;
-          qp[8 * q + 2 * h + 1] = r.y;
-          sq2 = __fadd2_rn(sq2, r);
-        }
-      }
-      sumq = sq2.x + sq2.y;
+    const int4 ra = cr.recs[slot * 3 + 0];
+    const int meta = ra.x;
+    if (meta & kEnd) break;
+    if (meta & kQRows) {
+      const int4 rb = cr.recs[slot * 3 + 1];
+      const int qb = meta >> 16;
+      u_h = qb * kNcw + cw;
+      active = u_h < a.Hq;
+      u_kvi = u_h / g - (qb * kNcw) / g;
+      u_q = ra.z;
+      u_lo = ra.w;
+      u_hi = rb.x;
+      u_sp = rb.y;
+      u_ns = rb.z;
+      u_base = rb.w;
       cur_cls = 3;  // the neutral scale is class 16's
       st.m = kNegInf;
       st.l = 0.f;
       st.zacc = 0.f;
 #pragma unroll
       for (int j = 0; j < 32; ++j) st.acc[j] = 0.f;
-    }
-    if (!(flags & 4)) {
-      const int cls = meta & 3, fill = (meta >> 2) & 127;
-      if (cls != cur_cls) {
-        rescale_dyn(qp, st.acc, cur_cls, cls);
-        cur_cls = cls;
+      if (active && !(meta & kNoPage)) {
+        const uint32_t qa = smem_u32(cr.ring + ra.y + cw * D * 2 + part * 64);
+        const float2 qs2 = make_float2(ka.qscale, ka.qscale);
+        float2 sq2 = make_float2(0.f, 0.f);
+#pragma unroll
+        for (int qq = 0; qq < 4; ++qq) {
+          const uint4 uq = lds128(qa + 16 * qq);
+          const uint32_t wv[4] = {uq.x, uq.y, uq.z, uq.w};
+#pragma unroll
+          for (int h = 0; h < 4; ++h) {
+            const float2 r = __fmul2_rn(make_float2(bf_lo(wv[h]), bf_hi(wv[h])), qs2);
+            qp[8 * qq + 2 * h] = r.x;
+            qp[8 * qq + 2 * h + 1] = r.y;
+            sq2 = __fadd2_rn(sq2, r);
+          }
+        }
+        sumq = sq2.x + sq2.y;
       }
-      const uint32_t s0 = smem_u32(ring + r0.y);
-      const uint32_t sp = s0 + a.slice[cls];  // slot positions, on masked pages
-      const bool masked = meta & 512;
-      const int c_lo = item_words[0], c_hi = item_words[1];  // key range
-      switch (cls) {
-        case 0: consume_page<D, 2, P / KPI>(s0, sp, masked, a.G, fill, c_lo, c_hi, qp, sumq, st, lane); break;
-        case 1: consume_page<D, 4, P / KPI>(s0, sp, masked, a.G, fill, c_lo, c_hi, qp, sumq, st, lane); break;
-        case 2: consume_page<D, 8, P / KPI>(s0, sp, masked, a.G, fill, c_lo, c_hi, qp, sumq, st, lane); break;
-        default: consume_page<D, 16, P / KPI>(s0, sp, masked, a.G, fill, c_lo, c_hi, qp, sumq, st, lane); break;
+    } else if (active) {
+      const int4 rc = cr.recs[slot * 3 + 2];
+      if (u_kvi >= rc.x && u_kvi < rc.x + rc.y) {
+        const int cls = meta & 3, fill = (meta >> 2) & 127;
+        if (cls != cur_cls) {
+          rescale_dyn(qp, st.acc, cur_cls, cls);
+          cur_cls = cls;
+        }
+        const uint32_t s0 = smem_u32(cr.ring + ra.y + (u_kvi - rc.x) * a.slice[cls]);
+        const bool masked = meta & kMask;
+        const uint32_t sp = masked ? smem_u32(cr.ring + rc.z) : s0;
+        switch (cls) {
+          case 0: consume_page<D, 2, P / KPI>(s0, sp, masked, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
+          case 1: consume_page<D, 4, P / KPI>(s0, sp, masked, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
+          case 2: consume_page<D, 8, P / KPI>(s0, sp, masked, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
+          default: consume_page<D, 16, P / KPI>(s0, sp, masked, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
+        }
       }
-    }
-    if (flags & 2) {  // last page of the item: its merge follows the refill
-      if (lane == 0) {
-        reinterpret_cast<int4*>(wmerge)[0] = make_int4(item_words[2], item_words[3], item_words[4], item_words[5]);
-        wmerge[4] = item_words[6];
-      }
-      merge_pending = true;
     }
     __syncwarp();
-    used -= r0.z;  // release the slot's ring bytes (the record is read)
-    consumed = g + 1;
+    if (lane == 0) mbar_arrive(&cr.empty[slot]);  // the stage's bytes are read
+    if ((meta & kLast) && active)
+      finish_unit<D>(ka, st, cur_cls, u_sp, u_q, u_h, u_ns, u_base, lane);
   }
+}
 
-  // The last CTA to finish records the error of the lowest failing query.
+// ------------------------------------------------ tensor-core consumer (GQA) --
+//
+// Warp cw computes the g query heads of KV head (block * kNcw + cw) with mma.sync
+// m16n8k16 (f16 or bf16 operands, f32 accumulation).  Thread (gid, tig) = (lane / 4,
+// lane % 4) as in the PTX fragment layouts.
+//
+// q.k: D_s[key][col] = sum_k A[key][k] B[k][col] with A the K codes of 16 keys and B
+// the query rows, column col = (head r, quantiser group gi) = (col / NG, col % NG)
+// holding head r's query on group gi's dimensions (zero elsewhere), so every column
+// gets its own group sum and s, z apply per group.  A code is masked in place and
+// read as an f16 subnormal c * 2^(pos - 24) (pos = its bit offset in the 16-bit half);
+// the query is pre-scaled by 2^(smax - pos) in f16 so that every product carries the
+// same factor 2^(smax - 24).  Width 16 uses bf16 operands (the query is bf16 already).
+//
+// P.V: O^T[dim][col] = sum_k V^T[dim][key] W[key][col] with W = p * s (f16; bf16 hi
+// and lo parts for width 16, whose values are raw bf16).  Pairs along keys for the A
+// operand come from byte permutes of two keys' code words.  Each accumulator row keeps
+// its class's factor 2^(pos - 24) until the class changes.
+
+__device__ __forceinline__ void mma_f16(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                        uint32_t b0, uint32_t b1) {
+  asm("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ void mma_bf16(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                         uint32_t b0, uint32_t b1) {
+  asm("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+template <int B>
+__device__ __forceinline__ void mma_cls(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                        uint32_t b0, uint32_t b1) {
+  if (B == 16) mma_bf16(c, a0, a1, a2, a3, b0, b1);
+  else mma_f16(c, a0, a1, a2, a3, b0, b1);
+}
+
+__device__ __forceinline__ uint32_t pack_f16x2(float lo, float hi) {
+  const __half2 h = __floats2half2_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t*>(&h);
+}
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t*>(&h);
+}
+
+// K side: pair i of a thread's D/4 dims of one key, as an A-operand word.
+template <int B>
+__device__ __forceinline__ uint32_t k_pair(const uint32_t* kw, int i) {
+  if (B == 16) return kw[i];
+  if (B == 8) return __byte_perm(kw[i >> 1], 0u, (i & 1) ? 0x4342 : 0x4140);
+  if (B == 4) {
+    const int k = i & 3;
+    const uint32_t w = k < 2 ? kw[i >> 2] : (kw[i >> 2] >> 8);
+    return w & ((k & 1) ? 0x00F000F0u : 0x000F000Fu);
+  }
+  const int k = i & 7;
+  const uint32_t w = k < 5 ? kw[i >> 3] : (kw[i >> 3] >> 10);
+  return w & (0x00030003u << (2 * (k < 5 ? k : k - 5)));
+}
+// the two dims (relative to the thread's first) of K pair i and their bit offset
+template <int B> __host__ __device__ constexpr int kp_lo(int i) {
+  return B >= 8 ? 2 * i : B == 4 ? 8 * (i / 4) + i % 4 : 16 * (i / 8) + i % 8;
+}
+template <int B> __host__ __device__ constexpr int kp_hi(int i) {
+  return B >= 8 ? 2 * i + 1 : B == 4 ? 8 * (i / 4) + i % 4 + 4 : 16 * (i / 8) + 8 + i % 8;
+}
+template <int B> __host__ __device__ constexpr int kp_pos(int i) {
+  return B >= 8 ? 0 : B == 4 ? 4 * (i % 2) : 2 * ((i % 8) < 5 ? i % 8 : i % 8 - 5);
+}
+template <int B> __host__ __device__ constexpr int smax_of() { return B == 2 ? 8 : B == 4 ? 4 : 0; }
+
+// V side: dim j of the thread's D/8 dims for keys (a, b) as an A-operand word (key a
+// in the low half).
+template <int B>
+__device__ __forceinline__ uint32_t v_pair(const uint32_t* wa, const uint32_t* wb, int j) {
+  if (B == 16) return __byte_perm(wa[j >> 1], wb[j >> 1], (j & 1) ? 0x7632 : 0x5410);
+  if (B == 8) {
+    const int k = j & 3;
+    const uint32_t x = __byte_perm(wa[j >> 2], wb[j >> 2], k < 2 ? 0x5140 : 0x7362);
+    return __byte_perm(x, 0u, (k & 1) ? 0x4342 : 0x4140);
+  }
+  if (B == 4) {
+    const int k = j & 7;
+    uint32_t x = __byte_perm(wa[j >> 3], wb[j >> 3], k < 4 ? 0x5410 : 0x7632);
+    if ((k & 3) >= 2) x >>= 8;
+    return x & ((k & 1) ? 0x00F000F0u : 0x000F000Fu);
+  }
+  const int k = j & 15, kk = k & 7;
+  uint32_t x = __byte_perm(wa[j >> 4], wb[j >> 4], k < 8 ? 0x5410 : 0x7632);
+  if (kk >= 5) x >>= 10;
+  return x & (0x00030003u << (2 * (kk < 5 ? kk : kk - 5)));
+}
+// log2 of the factor a V accumulator row carries in class index c (dim j of the
+// thread's D/8): 2^(pos - 24) for codes, 1 for bf16
+__host__ __device__ constexpr int vfac_log2(int c, int j) {
+  return c == 3 ? 0 : c == 2 ? -24 : c == 1 ? 4 * (j & 1) - 24 : 2 * ((j & 7) < 5 ? (j & 7) : (j & 7) - 5) - 24;
+}
+
+// Loads `nw` 32-bit words from shared address a (16-byte loads where aligned).
+template <int NW>
+__device__ __forceinline__ void lds_words(uint32_t a, uint32_t* w) {
+  if (NW % 4 == 0) {
+#pragma unroll
+    for (int k = 0; k < NW; k += 4) {
+      const uint4 u = lds128(a + 4 * k);
+      w[k] = u.x; w[k + 1] = u.y; w[k + 2] = u.z; w[k + 3] = u.w;
+    }
+  } else if (NW == 2) {
+    const uint2 u = lds64(a);
+    w[0] = u.x; w[1] = u.y;
+  } else {
+    w[0] = lds32(a);
+  }
+}
+
+template <int D, int NG>
+struct MmaState {
+  static constexpr int NP = D / 8;   // K pairs per thread and key
+  static constexpr int MT = D / 16;  // m-tiles of P.V
+  uint32_t qraw[NP];  // bf16 query of the thread's B column on its D/4 dims
+  uint32_t kb[NP];    // the q.k B operand in the current class
+  float qsum[2];      // qscale * sum of the query over (head, group) of the thread's two columns
+  float m[2], l[2], zacc[2];
+  float acc[MT][4];
+  float escale;       // 2^-E: the query pre-scale keeping f16 values in range
+  int E;
+};
+
+template <int D, int NG, int B>
+__device__ __forceinline__ void mma_build_kb(MmaState<D, NG>& ms) {
+  constexpr int NP = D / 8;
+  if (B == 16) {
+#pragma unroll
+    for (int i = 0; i < NP; ++i) ms.kb[i] = ms.qraw[i];
+  } else {
+#pragma unroll
+    for (int i = 0; i < NP; ++i) {
+      const int lo = kp_lo<B>(i), hi = kp_hi<B>(i);
+      const float f = pow2f(smax_of<B>() - kp_pos<B>(i)) * ms.escale;
+      const float ql = (lo & 1) ? bf_hi(ms.qraw[lo >> 1]) : bf_lo(ms.qraw[lo >> 1]);
+      const float qh = (hi & 1) ? bf_hi(ms.qraw[hi >> 1]) : bf_lo(ms.qraw[hi >> 1]);
+      ms.kb[i] = pack_f16x2(ql * f, qh * f);
+    }
+  }
+}
+
+// class index from -> to: new B operand, accumulator rows to the new class's factors
+template <int D, int NG>
+__device__ __forceinline__ void mma_switch(MmaState<D, NG>& ms, int from, int to) {
+  switch (to) {
+    case 0: mma_build_kb<D, NG, 2>(ms); break;
+    case 1: mma_build_kb<D, NG, 4>(ms); break;
+    case 2: mma_build_kb<D, NG, 8>(ms); break;
+    default: mma_build_kb<D, NG, 16>(ms); break;
+  }
+#pragma unroll
+  for (int t = 0; t < D / 16; ++t) {
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      const int j = 2 * t + r;
+      const float f = __int_as_float((127 + vfac_log2(to, j) - vfac_log2(from, j)) << 23);
+      ms.acc[t][2 * r] *= f;
+      ms.acc[t][2 * r + 1] *= f;
+    }
+  }
+}
+
+// One page of class B: keys in chunks of 16.
+template <int D, int NG, int B>
+__device__ __forceinline__ void mma_page(MmaState<D, NG>& ms, uint32_t s0, uint32_t spos, bool masked, int P, int fill,
+                                         int lo, int hi, float qscale, const bool (&col_ok)[2],
+                                         const int (&col_gi)[2], int lane) {
+  constexpr int KS = D / 16, MT = D / 16;
+  constexpr int rowb = B == 16 ? 2 * D : D * B / 8;  // bytes of one key's K (or V) row
+  constexpr int KW = D * B / 128;                    // K words per thread and key (D/4 dims)
+  constexpr int VB = D * B / 64;                     // V bytes per thread and key (D/8 dims)
+  constexpr int VW = VB >= 4 ? VB / 4 : 1;           // V words loaded per key
+  const int gid = lane >> 2, tig = lane & 3;
+  const uint32_t kbase = s0, vbase = s0 + P * rowb;
+  const uint32_t kszb = s0 + 2 * P * rowb, vszb = kszb + P * NG * 4;
+  const float kfac = __int_as_float((127 + 24 - smax_of<B>() + ms.E) << 23) * qscale;
+  const uint32_t wsel = (gid & 1) ? 0x7632u : 0x5410u;  // the W half of this thread's B column
+#pragma unroll 1
+  for (int c0 = 0; c0 < fill; c0 += 16) {
+    // ------------------------------------------------ scores of keys c0+gid, c0+gid+8
+    const int k1 = c0 + gid, k2 = k1 + 8;
+    uint32_t kw1[KW], kw2[KW];
+    lds_words<KW>(kbase + k1 * rowb + tig * (KW * 4), kw1);
+    lds_words<KW>(kbase + k2 * rowb + tig * (KW * 4), kw2);
+    float ca[4] = {0.f, 0.f, 0.f, 0.f}, cb[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int s = 0; s < KS; ++s) {
+      if (s & 1)
+        mma_cls<B>(cb, k_pair<B>(kw1, 2 * s), k_pair<B>(kw2, 2 * s), k_pair<B>(kw1, 2 * s + 1),
+                   k_pair<B>(kw2, 2 * s + 1), ms.kb[2 * s], ms.kb[2 * s + 1]);
+      else
+        mma_cls<B>(ca, k_pair<B>(kw1, 2 * s), k_pair<B>(kw2, 2 * s), k_pair<B>(kw1, 2 * s + 1),
+                   k_pair<B>(kw2, 2 * s + 1), ms.kb[2 * s], ms.kb[2 * s + 1]);
+    }
+    bool v1 = k1 < fill, v2 = k2 < fill;
+    if (masked) {
+      const int p1 = static_cast<int>(lds32(spos + 4 * k1)), p2 = static_cast<int>(lds32(spos + 4 * k2));
+      v1 = v1 && p1 >= lo && p1 <= hi;
+      v2 = v2 && p2 >= lo && p2 <= hi;
+    }
+    // column partial scores cp[key][j] (log2 units)
+    float cp[2][2];
+    float2 vsz[2][2];  // V (s, z) of the thread's two keys for its two columns' groups
+#pragma unroll
+    for (int kk = 0; kk < 2; ++kk) {
+      const int key = kk ? k2 : k1;
+#pragma unroll
+      for (int j = 0; j < 2; ++j) {
+        const float cv = ca[2 * kk + j] + cb[2 * kk + j];
+        if (B == 16) {
+          cp[kk][j] = cv * qscale;
+        } else {
+          const uint32_t szw = lds32(kszb + (key * NG + col_gi[j]) * 4);
+          const float2 sz = __half22float2(*reinterpret_cast<const __half2*>(&szw));
+          cp[kk][j] = fmaf(sz.x * kfac, cv, sz.y * ms.qsum[j]);
+        }
+      }
+      if (B != 16) {
+#pragma unroll
+        for (int j = 0; j < 2; ++j) {
+          const uint32_t szw = lds32(vszb + (key * NG + col_gi[j]) * 4);
+          vsz[kk][j] = __half22float2(*reinterpret_cast<const __half2*>(&szw));
+        }
+      }
+    }
+    if (B != 16) {  // a slot past the fill or outside the range may hold any bytes
+#pragma unroll
+      for (int j = 0; j < 2; ++j) {
+        if (!v1) vsz[0][j] = make_float2(0.f, 0.f);
+        if (!v2) vsz[1][j] = make_float2(0.f, 0.f);
+      }
+    }
+    // head scores per column slot
+    float sc[2][2];
+#pragma unroll
+    for (int kk = 0; kk < 2; ++kk) {
+      if (NG == 1) {
+        sc[kk][0] = cp[kk][0];
+        sc[kk][1] = cp[kk][1];
+      } else {
+        float h = cp[kk][0] + cp[kk][1];
+        if (NG == 4) h += __shfl_xor_sync(0xffffffffu, h, 1);
+        sc[kk][0] = sc[kk][1] = h;
+      }
+      const bool vk = kk ? v2 : v1;
+#pragma unroll
+      for (int j = 0; j < 2; ++j)
+        if (!(vk && col_ok[j])) sc[kk][j] = kNegInf;
+    }
+    // online softmax per slot (the running max is shared by the key lanes: p <= 1)
+    float p[2][2];
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      if (NG > 1 && j == 1) {
+        p[0][1] = p[0][0];
+        p[1][1] = p[1][0];
+        continue;
+      }
+      float mx = fmaxf(sc[0][j], sc[1][j]);
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 8));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
+      if (mx > ms.m[j]) {
+        const float alpha = fast_exp2(ms.m[j] - mx);
+        ms.m[j] = mx;
+        const int j1 = NG > 1 ? 1 : j;  // both slots hold one head when NG > 1
+#pragma unroll
+        for (int jj = j; jj <= j1; ++jj) {
+          ms.l[jj] *= alpha;
+          ms.zacc[jj] *= alpha;
+#pragma unroll
+          for (int t = 0; t < MT; ++t) {
+            ms.acc[t][jj] *= alpha;
+            ms.acc[t][jj + 2] *= alpha;
+          }
+        }
+        if (NG > 1) ms.m[1] = mx;
+      }
+      p[0][j] = fast_exp2(sc[0][j] - ms.m[j]);
+      p[1][j] = fast_exp2(sc[1][j] - ms.m[j]);
+    }
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      ms.l[j] += p[0][j] + p[1][j];
+      if (B != 16) ms.zacc[j] = fmaf(p[0][j], vsz[0][j].y, fmaf(p[1][j], vsz[1][j].y, ms.zacc[j]));
+    }
+    // ------------------------------------------------ P.V
+    // W of the thread's keys (gid, gid + 8) x columns (2 tig, 2 tig + 1), then the
+    // B operand of column gid, keys (2 tig, 2 tig + 1) and (2 tig + 8, 2 tig + 9)
+    const int src0 = 8 * tig + (gid >> 1), src1 = src0 + 4;
+    uint32_t b0, b1, bl0 = 0, bl1 = 0;
+    if (B == 16) {
+      const uint32_t h1 = pack_bf16x2(p[0][0], p[0][1]), h2 = pack_bf16x2(p[1][0], p[1][1]);
+      const uint32_t l1 = pack_bf16x2(p[0][0] - bf_lo(h1), p[0][1] - bf_hi(h1));
+      const uint32_t l2 = pack_bf16x2(p[1][0] - bf_lo(h2), p[1][1] - bf_hi(h2));
+      b0 = __byte_perm(__shfl_sync(0xffffffffu, h1, src0), __shfl_sync(0xffffffffu, h1, src1), wsel);
+      b1 = __byte_perm(__shfl_sync(0xffffffffu, h2, src0), __shfl_sync(0xffffffffu, h2, src1), wsel);
+      bl0 = __byte_perm(__shfl_sync(0xffffffffu, l1, src0), __shfl_sync(0xffffffffu, l1, src1), wsel);
+      bl1 = __byte_perm(__shfl_sync(0xffffffffu, l2, src0), __shfl_sync(0xffffffffu, l2, src1), wsel);
+    } else {
+      const uint32_t x1 = pack_f16x2(p[0][0] * vsz[0][0].x, p[0][1] * vsz[0][1].x);
+      const uint32_t x2 = pack_f16x2(p[1][0] * vsz[1][0].x, p[1][1] * vsz[1][1].x);
+      b0 = __byte_perm(__shfl_sync(0xffffffffu, x1, src0), __shfl_sync(0xffffffffu, x1, src1), wsel);
+      b1 = __byte_perm(__shfl_sync(0xffffffffu, x2, src0), __shfl_sync(0xffffffffu, x2, src1), wsel);
+    }
+    // V codes of keys (2 tig, 2 tig + 1) and (2 tig + 8, 2 tig + 9) on dims gid * D/8 ..
+    const int ka0 = c0 + 2 * tig;
+    const uint32_t voff = vbase + (VB >= 4 ? gid * VB : (gid * VB) & ~3);
+    uint32_t wa0[VW], wb0[VW], wa1[VW], wb1[VW];
+    lds_words<VW>(voff + ka0 * rowb, wa0);
+    lds_words<VW>(voff + (ka0 + 1) * rowb, wb0);
+    lds_words<VW>(voff + (ka0 + 8) * rowb, wa1);
+    lds_words<VW>(voff + (ka0 + 9) * rowb, wb1);
+    if (VB < 4) {  // two bytes per key: this thread's half of the word
+      const int sh = ((gid * VB) & 3) * 8;
+      wa0[0] >>= sh; wb0[0] >>= sh; wa1[0] >>= sh; wb1[0] >>= sh;
+    }
+    uint32_t m0 = 0xffffffffu, m1 = 0xffffffffu;  // bf16 values of keys out of range read as 0
+    if (B == 16) {
+      const uint32_t bal1 = __ballot_sync(0xffffffffu, v1), bal2 = __ballot_sync(0xffffffffu, v2);
+      m0 = ((bal1 >> (8 * tig)) & 1 ? 0x0000ffffu : 0u) | ((bal1 >> (8 * tig + 4)) & 1 ? 0xffff0000u : 0u);
+      m1 = ((bal2 >> (8 * tig)) & 1 ? 0x0000ffffu : 0u) | ((bal2 >> (8 * tig + 4)) & 1 ? 0xffff0000u : 0u);
+    }
+#pragma unroll
+    for (int t = 0; t < MT; ++t) {
+      const uint32_t a0 = v_pair<B>(wa0, wb0, 2 * t) & m0, a1 = v_pair<B>(wa0, wb0, 2 * t + 1) & m0;
+      const uint32_t a2 = v_pair<B>(wa1, wb1, 2 * t) & m1, a3 = v_pair<B>(wa1, wb1, 2 * t + 1) & m1;
+      mma_cls<B>(ms.acc[t], a0, a1, a2, a3, b0, b1);
+      if (B == 16) mma_bf16(ms.acc[t], a0, a1, a2, a3, bl0, bl1);
+    }
+  }
+}
+
+// The end of a unit for a tensor-core consumer: per head, the row into the warp's
+// scratch, then stored or merged like a CUDA-core row.
+template <int D, int NG>
+__device__ __forceinline__ void mma_finish(const AttnKernelArgs& ka, MmaState<D, NG>& ms, int cur_cls, int kv, int qi,
+                                           int sp, int ns, int base, const bool (&col_ok)[2], const int (&col_r)[2],
+                                           const int (&col_gi)[2], float* scr, int lane) {
+  constexpr int G = D / NG, DPL = D / 32, MT = D / 16, DV = D / 8;
+  const LayerArgs& a = ka.a;
+  const int g = a.Hq / a.Hkv;
+  const int gid = lane >> 2;
+#pragma unroll
+  for (int j = 0; j < 2; ++j) {
+#pragma unroll
+    for (int o = 4; o < 32; o <<= 1) {
+      ms.l[j] += __shfl_xor_sync(0xffffffffu, ms.l[j], o);
+      ms.zacc[j] += __shfl_xor_sync(0xffffffffu, ms.zacc[j], o);
+    }
+  }
+#pragma unroll
+  for (int t = 0; t < MT; ++t) {
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      const int jd = 2 * t + r, dim = gid * DV + jd;
+      const float inv = __int_as_float((127 - vfac_log2(cur_cls, jd)) << 23);
+#pragma unroll
+      for (int j = 0; j < 2; ++j)
+        if (col_ok[j] && dim / G == col_gi[j]) scr[col_r[j] * (D + 4) + dim] = fmaf(ms.acc[t][2 * r + j], inv, ms.zacc[j]);
+    }
+  }
+  if (gid == 0) {
+#pragma unroll
+    for (int j = 0; j < 2; ++j)
+      if (col_ok[j] && col_gi[j] == 0) {
+        scr[col_r[j] * (D + 4) + D] = ms.m[j];
+        scr[col_r[j] * (D + 4) + D + 1] = ms.l[j];
+      }
+  }
+  __syncwarp();
+  for (int r = 0; r < g; ++r) {
+    const float* row = scr + r * (D + 4);
+    float v[DPL];
+#pragma unroll
+    for (int j = 0; j < DPL; ++j) v[j] = row[lane * DPL + j];
+    const int qh = kv * g + r;
+    store_or_merge<D>(ka, v, lane * DPL, row[D], row[D + 1], sp, qi, qh, ns, base, lane);
+  }
+  __syncwarp();
+}
+
+template <int D, int NG>
+__device__ __forceinline__ void run_consumer_mma(const AttnKernelArgs& ka, const CtaRing& cr, int P, int cw, int lane,
+                                                 float* scr) {
+  constexpr int NP = D / 8, MT = D / 16, G = D / NG;
+  const LayerArgs& a = ka.a;
+  const int g = a.Hq / a.Hkv;
+  const int gid = lane >> 2, tig = lane & 3;
+  // the B column of q.k this thread holds, and its two accumulator columns
+  const int brow_r = gid / NG, brow_gi = gid % NG;
+  const bool b_ok = brow_r < g && (tig * (D / 4)) / G == brow_gi;
+  bool col_ok[2];
+  int col_r[2], col_gi[2];
+#pragma unroll
+  for (int j = 0; j < 2; ++j) {
+    const int c = 2 * tig + j;
+    col_r[j] = c / NG;
+    col_gi[j] = c % NG;
+    col_ok[j] = col_r[j] < g;
+  }
+  MmaState<D, NG> ms;
+  int cur_cls = 3;
+  int u_q = 0, u_kv = 0, u_lo = 0, u_hi = 0, u_sp = 0, u_ns = 1, u_base = 0;
+  bool active = false;
+  for (uint32_t s = 0;; ++s) {
+    const uint32_t slot = s % kStages;
+    const bool arrived = mbar_wait_or(&cr.full[slot], (s / kStages) & 1, cr.abort_flag);
+    if (!__all_sync(0xffffffffu, arrived)) {  // give up together, never half a warp
+      if (lane == 0) {
+        *cr.abort_flag = 1;
+        set_status(a.ctrl, TRR_ERR_TIMEOUT);
+      }
+      break;
+    }
+    const int4 ra = cr.recs[slot * 3 + 0];
+    const int meta = ra.x;
+    if (meta & kEnd) break;
+    if (meta & kQRows) {
+      const int4 rb = cr.recs[slot * 3 + 1];
+      const int qb = meta >> 16;
+      u_kv = qb * kNcw + cw;
+      active = u_kv < a.Hkv;
+      u_q = ra.z;
+      u_lo = ra.w;
+      u_hi = rb.x;
+      u_sp = rb.y;
+      u_ns = rb.z;
+      u_base = rb.w;
+      cur_cls = 3;
+#pragma unroll
+      for (int j = 0; j < 2; ++j) {
+        ms.m[j] = -1e30f;
+        ms.l[j] = 0.f;
+        ms.zacc[j] = 0.f;
+        ms.qsum[j] = 0.f;
+      }
+#pragma unroll
+      for (int t = 0; t < MT; ++t) ms.acc[t][0] = ms.acc[t][1] = ms.acc[t][2] = ms.acc[t][3] = 0.f;
+      if (active && !(meta & kNoPage)) {
+        // head brow_r's query on the thread's D/4 dims, zero outside its group
+        const uint32_t qa = smem_u32(cr.ring + ra.y + ((cw * g + min(brow_r, g - 1)) * D + tig * (D / 4)) * 2);
+        lds_words<NP>(qa, ms.qraw);
+        float qmax = 0.f, qs = 0.f;
+#pragma unroll
+        for (int i = 0; i < NP; ++i) {
+          if (!b_ok) ms.qraw[i] = 0u;
+          const float x0 = bf_lo(ms.qraw[i]), x1 = bf_hi(ms.qraw[i]);
+          qmax = fmaxf(qmax, fmaxf(fabsf(x0), fabsf(x1)));
+          qs += x0 + x1;
+        }
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) qmax = fmaxf(qmax, __shfl_xor_sync(0xffffffffu, qmax, o));
+        qs += __shfl_xor_sync(0xffffffffu, qs, 1);
+        qs += __shfl_xor_sync(0xffffffffu, qs, 2);
+        // qs: this B column's (head, group) sum; the accumulator columns 2 tig, 2 tig + 1
+        // are the B columns of lanes 4 (2 tig) and 4 (2 tig + 1)
+        ms.qsum[0] = __shfl_sync(0xffffffffu, qs, 8 * tig) * ka.qscale;
+        ms.qsum[1] = __shfl_sync(0xffffffffu, qs, 8 * tig + 4) * ka.qscale;
+        const int ex = static_cast<int>((__float_as_uint(qmax) >> 23) & 0xff) - 127;
+        ms.E = min(100, max(0, ex - 6));
+        ms.escale = __int_as_float((127 - ms.E) << 23);
+        mma_build_kb<D, NG, 16>(ms);
+      }
+    } else if (active) {
+      const int4 rc = cr.recs[slot * 3 + 2];
+      if (cw >= rc.x && cw < rc.x + rc.y) {
+        const int cls = meta & 3, fill = (meta >> 2) & 127;
+        if (cls != cur_cls) {
+          mma_switch<D, NG>(ms, cur_cls, cls);
+          cur_cls = cls;
+        }
+        const uint32_t s0 = smem_u32(cr.ring + ra.y + (cw - rc.x) * a.slice[cls]);
+        const bool masked = meta & kMask;
+        const uint32_t sp = masked ? smem_u32(cr.ring + rc.z) : s0;
+        switch (cls) {
+          case 0: mma_page<D, NG, 2>(ms, s0, sp, masked, P, fill, u_lo, u_hi, ka.qscale, col_ok, col_gi, lane); break;
+          case 1: mma_page<D, NG, 4>(ms, s0, sp, masked, P, fill, u_lo, u_hi, ka.qscale, col_ok, col_gi, lane); break;
+          case 2: mma_page<D, NG, 8>(ms, s0, sp, masked, P, fill, u_lo, u_hi, ka.qscale, col_ok, col_gi, lane); break;
+          default: mma_page<D, NG, 16>(ms, s0, sp, masked, P, fill, u_lo, u_hi, ka.qscale, col_ok, col_gi, lane); break;
+        }
+      }
+    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&cr.empty[slot]);  // the stage's bytes are read
+    if ((meta & kLast) && active)
+      mma_finish<D, NG>(ka, ms, cur_cls, u_kv, u_q, u_sp, u_ns, u_base, col_ok, col_r, col_gi, scr, lane);
+  }
+}
+
+// ---------------------------------------------------------------- kernels --
+
+// The prologue every attention kernel shares: barriers, the dependency on the previous
+// kernel, the call's work units.
+__device__ __forceinline__ CtaRing attn_prologue(const AttnKernelArgs& ka, uint8_t* smem, int P, int NQB, int*& pre) {
+  const AttnSmem lay(ka.ring_bytes, ka.n, ka.scr_floats);
+  CtaRing cr;
+  cr.ring = smem + lay.ring;
+  cr.recs = reinterpret_cast<int4*>(smem + lay.recs);
+  cr.sbytes = reinterpret_cast<int*>(smem + lay.sbytes);
+  cr.full = reinterpret_cast<uint64_t*>(smem + lay.full);
+  cr.empty = reinterpret_cast<uint64_t*>(smem + lay.empty);
+  cr.abort_flag = reinterpret_cast<volatile int*>(smem + lay.flag);
+  cr.R = ka.ring_bytes;
+  pre = reinterpret_cast<int*>(smem + lay.pre);
+  if (threadIdx.x == 0) {
+#pragma unroll 1
+    for (int i = 0; i < kStages; ++i) {
+      mbar_init(&cr.full[i], 1);
+      mbar_init(&cr.empty[i], kNcw);
+    }
+    *cr.abort_flag = 0;
+    fence_barrier_init();
+  }
+  pdl_wait();
+  pdl_trigger();
+  plan_units(ka, P, NQB, pre, reinterpret_cast<long long*>(smem + lay.red));
+  return cr;
+}
+
+// The epilogue: the last CTA to finish records the error of the lowest failing query
+// and readies the call's counters for the next call.
+__device__ __forceinline__ void attn_epilogue(const LayerArgs& a) {
   __syncthreads();
   if (threadIdx.x == 0) {
     __threadfence();
@@ -815,24 +1506,78 @@ __global__ void __launch_bounds__(256, 2) attn_kernel(const __grid_constant__ At
       __threadfence();
       const int bad = atomicExch(&a.ctrl[kFirstBadQuery], INT_MAX);
       if (bad != INT_MAX) set_status(a.ctrl, bad & 15);
+      atomicExch(&a.ctrl[kNextUnit], 0);
       atomicExch(&a.ctrl[kDoneCtas], 0);
     }
   }
 }
 
-constexpr int kAttnSmemLimit = 113 * 1024;  // dynamic shared memory of one attention CTA
+// CUDA-core path: units of kNcw query heads, one per consumer warp.
+template <int D, int P>
+__global__ void __launch_bounds__(32 * (kNcw + 1), kCtasPerSm) attn_kernel(const __grid_constant__ AttnKernelArgs ka) {
+  extern __shared__ __align__(128) uint8_t smem[];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int NQB = (ka.a.Hq + ka.hpu - 1) / ka.hpu;
+  int* pre;
+  const CtaRing cr = attn_prologue(ka, smem, P, NQB, pre);
+  if (warp == 0) run_producer<D>(ka, P, NQB, pre, cr, lane);
+  else run_consumer_cc<D, P>(ka, cr, warp - 1, lane);
+  attn_epilogue(ka.a);
+}
+
+// Tensor-core path: units of kNcw KV heads with all their query heads.
+template <int D, int NG>
+__global__ void __launch_bounds__(32 * (kNcw + 1), kCtasPerSm) attn_mma_kernel(const __grid_constant__ AttnKernelArgs ka) {
+  extern __shared__ __align__(128) uint8_t smem[];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int NQB = (ka.a.Hq + ka.hpu - 1) / ka.hpu;
+  const int P = ka.a.P;
+  int* pre;
+  const CtaRing cr = attn_prologue(ka, smem, P, NQB, pre);
+  if (warp == 0) {
+    run_producer<D>(ka, P, NQB, pre, cr, lane);
+  } else {
+    const AttnSmem lay(ka.ring_bytes, ka.n, ka.scr_floats);
+    float* scr = reinterpret_cast<float*>(smem + lay.scr) + (warp - 1) * ka.scr_floats;
+    run_consumer_mma<D, NG>(ka, cr, P, warp - 1, lane, scr);
+  }
+  attn_epilogue(ka.a);
+}
+
+constexpr int kAttnSmemLimit = 72 * 1024;  // dynamic shared memory of one attention CTA
 
 // Done once per cache at creation, so that calls stay legal inside stream capture.
 cudaError_t attn_configure() {
   const void* kernels[] = {
-      reinterpret_cast<const void*>(attn_kernel<64, 16>), reinterpret_cast<const void*>(attn_kernel<64, 32>),
-      reinterpret_cast<const void*>(attn_kernel<64, 64>), reinterpret_cast<const void*>(attn_kernel<128, 16>),
-      reinterpret_cast<const void*>(attn_kernel<128, 32>), reinterpret_cast<const void*>(attn_kernel<128, 64>)};
+      reinterpret_cast<const void*>(attn_kernel<64, 16>),     reinterpret_cast<const void*>(attn_kernel<64, 32>),
+      reinterpret_cast<const void*>(attn_kernel<64, 64>),     reinterpret_cast<const void*>(attn_kernel<128, 16>),
+      reinterpret_cast<const void*>(attn_kernel<128, 32>),    reinterpret_cast<const void*>(attn_kernel<128, 64>),
+      reinterpret_cast<const void*>(attn_mma_kernel<64, 1>),  reinterpret_cast<const void*>(attn_mma_kernel<64, 2>),
+      reinterpret_cast<const void*>(attn_mma_kernel<128, 1>), reinterpret_cast<const void*>(attn_mma_kernel<128, 2>),
+      reinterpret_cast<const void*>(attn_mma_kernel<128, 4>)};
   for (const void* k : kernels) {
     const cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, kAttnSmemLimit);
     if (e != cudaSuccess) return e;
   }
   return cudaSuccess;
+}
+
+// The tensor-core path serves query groups (g >= 2) whose (head, group) columns fit
+// one 8-wide mma tile.
+static bool use_mma(const Layout& l) {
+  const int g = l.Hq / l.Hkv, ng = l.d / l.G;
+  return g >= 2 && g * ng <= 8;
+}
+
+// Ring bytes an attention call with n queries gets, or -1 when one stage of the
+// widest page (one KV slice, its positions) or of the query rows would not fit.
+static int attn_ring_bytes(const Layout& l, int n, int hpu, int scr_floats) {
+  const int fixed = AttnSmem(0, n, scr_floats).total;
+  const int ring = (kAttnSmemLimit - fixed) / 128 * 128;
+  const int widest = static_cast<int>(l.slice[3]) + 4 * l.P;
+  const int qrows = hpu * 2 * l.d;
+  if (ring < std::max(widest, qrows)) return -1;
+  return ring;
 }
 
 // The one launch of an attention call with the given scratch views in `a`.
@@ -852,22 +1597,27 @@ static cudaError_t launch_attention(const Layout& l, const LayerArgs& a, int num
   ka.out = static_cast<uint16_t*>(out_bf16);
   const float scale = softmax_scale > 0.f ? softmax_scale : 1.f / sqrtf(static_cast<float>(l.d));
   ka.qscale = scale * 1.4426950408889634f;
-  // a ring holds at least one page of the widest class with its positions and a query
-  // row; up to 12 KB when shared memory allows
-  const int widest = (static_cast<int>(l.slice[3]) + 4 * l.P + 2 * l.d + 127) / 128 * 128;
-  int nwarps = 8, ring = 0;
-  for (; nwarps > 0; --nwarps) {
-    const int fixed = AttnSmem(nwarps, 0, n).total;
-    ring = std::min(std::max(12 * 1024, widest), (kAttnSmemLimit - fixed) / nwarps / 128 * 128);
-    if (ring >= widest) break;
-  }
-  if (nwarps < 1) return cudaErrorInvalidConfiguration;
+  const bool mma = use_mma(l);
+  const int g = l.Hq / l.Hkv;
+  ka.hpu = mma ? kNcw * g : kNcw;
+  ka.scr_floats = mma ? g * (l.d + 4) : 0;
+  const int ring = attn_ring_bytes(l, n, ka.hpu, ka.scr_floats);
+  if (ring < 0) return cudaErrorInvalidConfiguration;
   ka.ring_bytes = ring;
-  const int smem = AttnSmem(nwarps, ring, n).total;
+  const size_t sm = static_cast<size_t>(AttnSmem(ring, n, ka.scr_floats).total);
+  const dim3 grid(kCtasPerSm * num_sms), block(32 * (kNcw + 1));
+  if (mma) {
+    const int ng = l.d / l.G;
+    if (l.d == 64) {
+      if (ng == 1) return launch_pdl(attn_mma_kernel<64, 1>, grid, block, sm, s, ka);
+      return launch_pdl(attn_mma_kernel<64, 2>, grid, block, sm, s, ka);
+    }
+    if (ng == 1) return launch_pdl(attn_mma_kernel<128, 1>, grid, block, sm, s, ka);
+    if (ng == 2) return launch_pdl(attn_mma_kernel<128, 2>, grid, block, sm, s, ka);
+    return launch_pdl(attn_mma_kernel<128, 4>, grid, block, sm, s, ka);
+  }
   // one kernel per head size and page size: the page loop unrolls, and a kernel's code
   // holds only the four width classes it can meet
-  const dim3 grid(2 * num_sms), block(nwarps * 32);
-  const size_t sm = static_cast<size_t>(smem);
   if (l.d == 64) {
     if (l.P == 16) return launch_pdl(attn_kernel<64, 16>, grid, block, sm, s, ka);
     if (l.P == 32) return launch_pdl(attn_kernel<64, 32>, grid, block, sm, s, ka);
@@ -962,7 +1712,7 @@ extern "C" trr_status trr_decode_attn_static(trr_cache* cache, int32_t layer, in
   // scratch of this call, carved from the static array; reject what does not fit
   auto up = [](int64_t x) { return (x + 255) / 256 * 256; };
   const int64_t b_ctrl = up(4 * kCtrlInts);
-  const int64_t b_cnt = up(4ll * n * l.units);
+  const int64_t b_cnt = up(4ll * n * l.units * l.cnt_stride);
   const int64_t b_part = up(4ll * n * l.s_cap * l.units * (l.d + 4));
   if (b_ctrl + b_cnt + b_part > kStaticScratchBytes) return TRR_ERR_OUT_OF_MEMORY;
   void* base = nullptr;
@@ -974,7 +1724,7 @@ extern "C" trr_status trr_decode_attn_static(trr_cache* cache, int32_t layer, in
   a.cnt = reinterpret_cast<int32_t*>(b + b_ctrl);
   a.part = reinterpret_cast<float*>(b + b_ctrl + b_cnt);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const int ncnt = n * l.units;
+  const int ncnt = n * l.units * l.cnt_stride;
   static_scratch_clear_kernel<<<std::max(1, std::min(256, (ncnt + 255) / 256)), 256, 0, s>>>(a.ctrl, a.cnt, ncnt);
   cudaError_t e = cudaGetLastError();
   if (e == cudaSuccess)

@@ -23,12 +23,17 @@ enum Ctrl : int {
   kFirstBadQuery = 12,// attention: min of (query index * 16 + error) over failing queries
                       // (INT_MAX = none)
   kDoneCtas = 14,     // attention: CTAs finished (the last one records the status)
+  kNextUnit = 15,     // attention: next work unit to hand out
   kCtrlInts = 64
 };
 
 // Splits of one attention work unit are sized to hold at most this many pages (+ one
 // partial page per class), so that a warp holds an item's page ids one per lane.
 constexpr int kItemMaxPages = 28;
+
+// Split partials are merged in groups of this many (then the groups): a query with
+// ns splits per head has 1 + ceil(ns / kMergeGroup) arrival counters per head.
+constexpr int kMergeGroup = 8;
 
 // Byte layout of one cache (see include/trr.h for the documented part).
 struct Layout {
@@ -38,6 +43,7 @@ struct Layout {
   int units;      // attention work units per query split (one per query head)
   int pos_split;  // key positions per split at least (split_bytes of 8-bit tokens)
   int s_cap;      // most splits one query is cut into
+  int cnt_stride; // arrival counters per (query, head): 1 + ceil(s_cap / kMergeGroup)
   int64_t max_items;
   int64_t hdr, tokb[kClasses], slice[kClasses], page_bytes[kClasses];
   int64_t off_ctrl, off_last_pos, off_ntok, off_presence, off_pt, off_pfirst, off_plast, off_lastpg;
@@ -98,7 +104,7 @@ inline Views make_views(const Layout& l, void* base) {
 
 // Everything a kernel needs about one layer of one cache, passed by value.
 struct LayerArgs {
-  int layer, S, Hq, Hkv, d, G, P, maxctx, MP, W32, units, pos_split, s_cap, split_bytes, skip_writes_kv;
+  int layer, S, Hq, Hkv, d, G, P, maxctx, MP, W32, units, pos_split, s_cap, cnt_stride, split_bytes, skip_writes_kv;
   int cap[kClasses];
   int hdr;
   int slice[kClasses];
@@ -112,7 +118,7 @@ struct LayerArgs {
   int32_t* plast;
   int32_t* lastpg;     // this layer: [S][4] id of the page holding token ntok-1 (internal)
   AppendPlan* aplan;
-  int32_t* cnt;        // [max_queries][Hq] split arrivals (zero between calls)
+  int32_t* cnt;        // [max_queries][Hq][cnt_stride] split arrivals (zero between calls)
   float* part;         // [max_queries * s_cap * Hq][d + 4] fp32 partials: acc, M, L
   uint8_t* pool[kClasses];
 };
