@@ -1,30 +1,38 @@
 // trr_attn.cu - trr_decode_attn: mode-routed split-K decode attention over the
 // mixed-precision paged cache (Sec. 3.2(A), Eq. 2; Sec. 3.8; Sec. 7).
 //
-// One persistent kernel per call (two CTAs per SM, every warp an independent worker):
+// One persistent kernel per call: three CTAs per SM, each one producer warp and four
+// consumer warps around a ring of shared memory.
 //   1. Every CTA cuts the call into work units: query q gets ns_q splits from the
 //      length of its key range (full: [0, t]; local: [t-w+1, t]; skip or invalid: one
-//      unit that writes the zero row) and a prefix sum numbers the units.  The same
-//      deterministic computation in every CTA takes the place of a planning kernel.
-//   2. Work items (unit, query head) are dealt round-robin to the warps.  A warp plans
-//      its item itself: the sequence's per-class token counts, a 32-way search of the
-//      pages' first / last positions at window edges, and the split's share of every
-//      class's pages in range (one page id per lane).  It streams those pages' slices
-//      of the head through a private ring of shared memory filled by 1-D bulk copies
-//      (cp.async.bulk + mbarrier), the query row riding on the first copy of each
-//      item, so items follow each other without a pipeline drain.  Lane pair (key,
-//      half) of a 64-wide head (four lanes for 128) dequantises in registers and keeps
-//      its own online softmax; lanes merge with shuffles.
-//   3. A query with one split gets its bf16 row from that item.  Otherwise each split
-//      writes an fp32 partial and counts its arrival; the last split of the (query,
-//      head) to arrive merges the partials, writes the row and resets the counter.
-//   4. The last CTA to finish records the error of the lowest failing query.
+//      split that writes the zero rows), and a unit is a split and a block of query
+//      heads.  The same deterministic computation in every CTA takes the place of a
+//      planning kernel.  Splits are sized for about one unit per CTA on a small call
+//      and up to three on a large one.
+//   2. The producer warp takes units (its CTA's own first, then from a call-wide
+//      counter) and plans each once: the sequence's per-class token counts, a 32-way
+//      search of the pages' first / last positions at window edges, the split's share
+//      of every class's pages in range.  It pushes the unit through the ring as stages
+//      filled by 1-D bulk copies (cp.async.bulk + mbarrier): the block's query rows,
+//      then per page the slices of the KV heads the block reads (slot positions too
+//      when the page straddles the key range).
+//   3. Consumer warps read the stages in order and release each one.  Two consumers:
+//        - CUDA cores (one query head per warp; MHA and wide query groups): lane pair
+//          (key, half) of a 64-wide head (four lanes for 128) dequantises in registers
+//          and keeps its own online softmax; lanes merge with shuffles;
+//        - tensor cores (one KV head and its whole query group per warp, g >= 2 with
+//          g * d/G <= 8): q.k and P.V as mma.sync m16n8k16 with f32 accumulation.
+//   4. A query with one split gets its bf16 rows from that unit.  Otherwise each split
+//      writes fp32 partials; partials merge in two levels (groups of kMergeGroup, then
+//      the groups), each by the last arrival, which resets its counter.
+//   5. The last CTA to finish records the error of the lowest failing query.
 //
-// Dequantisation: k = z + c*s, so q.k = s * sum(q_i c_i) + z * sum(q_i).  A code is
-// masked in place (no shift) and its bits read as a binary32 subnormal, c * 2^(e-149)
-// where e is its bit offset; the query is pre-scaled per width class by 2^(100-e) so
-// that q_i * x_i = q_i c_i 2^-49 exactly as an fp32 product.  V is accumulated in a
-// domain scaled by 2^-49 with the per-offset factor folded into the key's weight.
+// CUDA-core dequantisation: k = z + c*s, so q.k = s * sum(q_i c_i) + z * sum(q_i).  A
+// code is masked in place (no shift) and its bits read as a binary32 subnormal,
+// c * 2^(e-149) where e is its bit offset; the query is pre-scaled per width class by
+// 2^(100-e) so that q_i * x_i = q_i c_i 2^-49 exactly as an fp32 product.  V is
+// accumulated in a domain scaled by 2^-49 with the per-offset factor folded into the
+// key's weight.
 #include <algorithm>
 #include <climits>
 
@@ -188,20 +196,6 @@ struct LaneState {
   float m, l, zacc;  // running max (log2), sum of weights, sum of p*z (V zero points)
   float acc[32];     // sum of p*v over the lane's 32 dims, scaled by 2^-49
 };
-
-__device__ __forceinline__ float softmax_step(LaneState& st, float score) {
-  if (score > st.m + kTau) {
-    const float alpha = fast_exp2(st.m - score);  // 0 when m = -inf
-#pragma unroll
-    for (int j = 0; j < 32; ++j) st.acc[j] *= alpha;
-    st.l *= alpha;
-    st.zacc *= alpha;
-    st.m = score;
-  }
-  const float p = fast_exp2(score - st.m);
-  st.l += p;
-  return p;
-}
 
 // Shared-memory loads at 32-bit shared addresses.  Volatile: they stay after the
 // mbarrier wait that makes the bytes valid.
@@ -410,6 +404,7 @@ struct AttnKernelArgs {
   const uint16_t* q;
   uint16_t* out;
   float qscale;      // softmax scale * log2(e)
+  int q0;            // index of the launch's first query in the call (error reports)
   int ring_bytes;    // bytes of the CTA's ring of shared memory
   int hpu;           // query heads per work unit
   int scr_floats;    // per-consumer-warp scratch (floats) of the tensor-core path
@@ -432,7 +427,7 @@ __device__ __forceinline__ int query_range(int t, int mode, int w) {
 // (mbarriers need 8, bulk-copy destinations 16).
 __host__ __device__ constexpr int align16(int x) { return (x + 15) & ~15; }
 struct AttnSmem {
-  int ring, recs, sbytes, full, empty, scr, pre, red, flag, total;
+  int ring, recs, sbytes, full, empty, scr, pre, perm, info, red, flag, total;
   __host__ __device__ AttnSmem(int ring_bytes, int n, int scr_floats)
       : ring(0),
         recs(align16(ring_bytes)),
@@ -441,8 +436,10 @@ struct AttnSmem {
         empty(full + kStages * 8),
         scr(empty + kStages * 8),
         pre(scr + align16(kNcw * scr_floats * 4)),
-        red(pre + align16(4 * (n + 1))),
-        flag(red + 16 * 8),
+        perm(pre + align16(4 * (n + 1))),
+        info(perm + align16(4 * n)),
+        red(info + align16(4 * n)),
+        flag(red + 64 * 4),
         total(flag + 16) {}
 };
 
@@ -530,25 +527,32 @@ __device__ __forceinline__ int plan_split(const LayerArgs& a, int P, int seq, in
   return T;
 }
 
-// The work units of a call, computed the same way by every CTA: query q gets ns_q
-// splits from its key range; pre[q] numbers its first split, pre[n] counts them all.
-__device__ __forceinline__ void plan_units(const AttnKernelArgs& ka, int P, int NQB, int* pre, long long* red) {
+// The work units of a launch, computed the same way by every CTA: query q gets ns_q
+// splits from its key range.  Units are numbered largest first (queries in full mode,
+// then local, then skip or invalid ones, each group in query order), so that the last
+// units handed out are the small ones: query perm[k] is the k-th in that order, its
+// splits are units pre[k] .. pre[k + 1] - 1, and pre[n] counts them all.
+__device__ __forceinline__ void plan_units(const AttnKernelArgs& ka, int P, int NQB, int* pre, int* perm, int* info,
+                                           int* red) {
   const LayerArgs& a = ka.a;
   const int n = ka.n, lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
   long long rsum = 0;
   for (int q = threadIdx.x; q < n; q += blockDim.x) {
     const int seq = ka.seq_ids[q], t = ka.q_positions[q], mode = ka.modes[q];
     const int w = ka.windows ? ka.windows[q] : ka.window_scalar;
-    const int r = query_error(a, seq, t, mode, w) ? 0 : query_range(t, mode, w);
-    pre[q] = r;
+    const bool bad = query_error(a, seq, t, mode, w) != 0;
+    const int r = bad ? 0 : query_range(t, mode, w);
+    const int cls = bad ? 2 : mode == TRR_MODE_FULL ? 0 : mode == TRR_MODE_LOCAL ? 1 : 2;
+    info[q] = r | (cls << 29);  // r <= max_context <= 2^24
     rsum += r;
   }
+  long long* red64 = reinterpret_cast<long long*>(red);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) rsum += __shfl_xor_sync(0xffffffffu, rsum, o);
-  if (lane == 0) red[warp] = rsum;
+  if (lane == 0) red64[warp] = rsum;
   __syncthreads();
   rsum = 0;
-  for (int k = 0; k < nwarps; ++k) rsum += red[k];
+  for (int k = 0; k < nwarps; ++k) rsum += red64[k];
   // Split size: a small call gets about one unit per CTA (its units are latency-bound
   // chains, and a second unit on a CTA doubles the call); a large one up to
   // kUnitsPerCta per CTA, each of at least kMinUnitPositions positions per head block
@@ -561,28 +565,62 @@ __device__ __forceinline__ void plan_units(const AttnKernelArgs& ka, int P, int 
   const float by_work = ceilf(rs / want);
   const int pos_split = by_work > static_cast<float>(a.pos_split) ? static_cast<int>(fminf(by_work, 1073741824.f))
                                                                    : a.pos_split;
+  // per class, this thread's queries and splits (a contiguous chunk of queries)
   const int chunk = (n + blockDim.x - 1) / blockDim.x;
   const int q0 = min(n, static_cast<int>(threadIdx.x) * chunk), q1 = min(n, q0 + chunk);
-  int mine = 0;
-  for (int q = q0; q < q1; ++q) mine += splits_of(pre[q], pos_split, P, a.s_cap);
-  int incl = mine;
+  int v[6] = {0, 0, 0, 0, 0, 0};  // queries of class 0, 1, 2, then their splits
+  for (int q = q0; q < q1; ++q) {
+    const int i = info[q], c = i >> 29;
+    v[c] += 1;
+    v[3 + c] += splits_of(i & 0x1fffffff, pos_split, P, a.s_cap);
+  }
+  // exclusive scan over the threads, and the totals
+  int incl[6];
 #pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const int v = __shfl_up_sync(0xffffffffu, incl, o);
-    if (lane >= o) incl += v;
+  for (int j = 0; j < 6; ++j) {
+    incl[j] = v[j];
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int x = __shfl_up_sync(0xffffffffu, incl[j], o);
+      if (lane >= o) incl[j] += x;
+    }
   }
   __syncthreads();  // every read of red above is done
-  if (lane == 31) red[8 + warp] = incl;
-  __syncthreads();
-  int off = incl - mine;
-  for (int k = 0; k < warp; ++k) off += static_cast<int>(red[8 + k]);
-  for (int q = q0; q < q1; ++q) {
-    const int ns = splits_of(pre[q], pos_split, P, a.s_cap);
-    pre[q] = off;
-    off += ns;
+  if (lane == 31) {
+#pragma unroll
+    for (int j = 0; j < 6; ++j) red[16 + warp * 6 + j] = incl[j];
   }
-  if (threadIdx.x == blockDim.x - 1) pre[n] = off;
   __syncthreads();
+  int off[6], tot[6];
+#pragma unroll
+  for (int j = 0; j < 6; ++j) {
+    off[j] = incl[j] - v[j];
+    tot[j] = 0;
+    for (int k = 0; k < nwarps; ++k) {
+      const int x = red[16 + k * 6 + j];
+      if (k < warp) off[j] += x;
+      tot[j] += x;
+    }
+  }
+  // class c's ranks and units follow those of the classes before it
+  off[1] += tot[0];
+  off[2] += tot[0] + tot[1];
+  off[4] += tot[3];
+  off[5] += tot[3] + tot[4];
+  for (int q = q0; q < q1; ++q) {
+    const int i = info[q], c = i >> 29;
+    const int ns = splits_of(i & 0x1fffffff, pos_split, P, a.s_cap);
+    const int k = c == 0 ? off[0]++ : c == 1 ? off[1]++ : off[2]++;
+    perm[k] = q;
+    if (c == 0) { pre[k] = off[3]; off[3] += ns; }
+    else if (c == 1) { pre[k] = off[4]; off[4] += ns; }
+    else { pre[k] = off[5]; off[5] += ns; }
+  }
+  if (threadIdx.x == 0) pre[n] = tot[3] + tot[4] + tot[5];
+  __syncthreads();
+  if (blockIdx.x == 0) {  // each query's first partial and splits, for the combine kernel
+    for (int k = threadIdx.x; k < n; k += blockDim.x) a.qtab[perm[k]] = make_int2(pre[k], pre[k + 1] - pre[k]);
+  }
 }
 
 // Everything the producer and consumers of one CTA share.
@@ -600,7 +638,7 @@ struct CtaRing {
 // plans each and pushes its stages; ends with an end record.
 template <int D>
 __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, int NQB, const int* pre,
-                                             const CtaRing& cr, int lane) {
+                                             const int* perm, const CtaRing& cr, int lane) {
   const LayerArgs& a = ka.a;
   const int n = ka.n, g = a.Hq / a.Hkv, R = cr.R;
   const int total = pre[n] * NQB;
@@ -655,13 +693,13 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
     int u_next = 0;
     if (lane == 0) u_next = static_cast<int>(gridDim.x) + atomicAdd(&a.ctrl[kNextUnit], 1);  // used last
     const int un = u / NQB, qb = u - un * NQB;
-    int lo_q = 0, hi_q = n;  // the query of split un: pre[q] <= un < pre[q + 1]
-    while (hi_q - lo_q > 1) {
-      const int mid = (lo_q + hi_q) >> 1;
-      if (pre[mid] <= un) lo_q = mid;
-      else hi_q = mid;
+    int lo_k = 0, hi_k = n;  // the query of split un: pre[k] <= un < pre[k + 1]
+    while (hi_k - lo_k > 1) {
+      const int mid = (lo_k + hi_k) >> 1;
+      if (pre[mid] <= un) lo_k = mid;
+      else hi_k = mid;
     }
-    const int q = lo_q, sp = un - pre[q], ns = pre[q + 1] - pre[q];
+    const int q = perm[lo_k], sp = un - pre[lo_k], ns = pre[lo_k + 1] - pre[lo_k];
     const int seq = ka.seq_ids[q], t = ka.q_positions[q], mode = ka.modes[q];
     const int w = ka.windows ? ka.windows[q] : ka.window_scalar;
     const int err = query_error(a, seq, t, mode, w);
@@ -669,13 +707,13 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
     if (err || mode == TRR_MODE_SKIP) {  // zero rows; the error of the lowest query
       uint4* o = reinterpret_cast<uint4*>(ka.out + (static_cast<int64_t>(q) * a.Hq + h0) * D);
       for (int i = lane; i < nh * D / 8; i += 32) o[i] = make_uint4(0, 0, 0, 0);
-      if (err && qb == 0 && lane == 0) atomicMin(&a.ctrl[kFirstBadQuery], q * 16 + err);
+      if (err && qb == 0 && lane == 0) atomicMin(&a.ctrl[kFirstBadQuery], (ka.q0 + q) * 16 + err);
     } else {
       const int lo = mode == TRR_MODE_FULL ? 0 : max(0, t - w + 1);
       int wid, wmeta;
       const int T = plan_split(a, P, seq, lo, t, sp, ns, lane, wid, wmeta);
       const int kv0 = h0 / g, nkv = (h0 + nh - 1) / g - kv0 + 1;
-      const int4 rb = make_int4(t, sp, ns, pre[q]);
+      const int4 rb = make_int4(t, sp, ns, pre[lo_k]);
       {  // the unit's query rows
         const int need = nh * D * 2;
         int taken = 0;
@@ -689,13 +727,22 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
         if (lane == 0)
           bulk_g2s(cr.ring + off, ka.q + (static_cast<int64_t>(q) * a.Hq + h0) * D, need, &cr.full[slot]);
       }
+      // every page's copy, worked out once per unit (lane j: page j), so that a push
+      // is a few shuffles and the copy
+      uint64_t pg_src = 0;  // the page
+      int pg_geo = 0;       // slice bytes | KV slices per stage << 20
+      if (lane < T) {
+        const int c = wmeta & 3, slice = a.slice[c];
+        const int posb = (wmeta & kMask) ? 4 * P : 0;
+        pg_src = reinterpret_cast<uint64_t>(a.pool[c] + static_cast<int64_t>(wid) * a.page_bytes[c]);
+        pg_geo = slice | (max(1, (R / 2 - posb) / slice) << 20);
+      }
       for (int j = 0; j < T && ok; ++j) {
-        const int id = __shfl_sync(0xffffffffu, wid, j);
+        const uint8_t* page = reinterpret_cast<const uint8_t*>(__shfl_sync(0xffffffffu, pg_src, j));
+        const int geo = __shfl_sync(0xffffffffu, pg_geo, j);
         const int pm = __shfl_sync(0xffffffffu, wmeta, j);
-        const int c = pm & 3, slice = a.slice[c];
+        const int slice = geo & 0xfffff, maxk = geo >> 20;
         const int posb = (pm & kMask) ? 4 * P : 0;
-        const int maxk = max(1, (R / 2 - posb) / slice);  // KV slices per stage
-        const uint8_t* page = a.pool[c] + static_cast<int64_t>(id) * a.page_bytes[c];
         for (int k0 = 0; k0 < nkv; k0 += maxk) {
           const int nk = min(maxk, nkv - k0);
           const int need = nk * slice + posb;
@@ -734,99 +781,27 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
   }
 }
 
-// Merges `count` partial rows at p0, p0 + stride, ...: the common maximum Mx, the
-// weighted sum of L and the weighted rows (lane holds dims lane * DPL ..).
-template <int D>
-__device__ __forceinline__ void merge_partials(const float* p0, int64_t stride, int count, int lane, float& Mx,
-                                               float& Ls, float (&acc_o)[D / 32]) {
-  constexpr int DPL = D / 32;
-  Mx = kNegInf;
-  for (int s = lane; s < count; s += 32) Mx = fmaxf(Mx, __ldcg(p0 + s * stride + D));
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) Mx = fmaxf(Mx, __shfl_xor_sync(0xffffffffu, Mx, o));
-  Ls = 0.f;
-#pragma unroll
-  for (int j = 0; j < DPL; ++j) acc_o[j] = 0.f;
-  for (int s0 = 0; s0 < count; s0 += 32) {
-    float wl = 0.f;  // lane s: weight of row s0 + s
-    if (s0 + lane < count) {
-      const float2 ml = __ldcg(reinterpret_cast<const float2*>(p0 + (s0 + lane) * stride + D));
-      wl = (ml.x == kNegInf) ? 0.f : fast_exp2(ml.x - Mx);
-      Ls = fmaf(wl, ml.y, Ls);
-    }
-    const int cnt = min(32, count - s0);
-#pragma unroll 8
-    for (int s = 0; s < cnt; ++s) {
-      const float wgt = __shfl_sync(0xffffffffu, wl, s);
-      const float* ps = p0 + (s0 + s) * stride + lane * DPL;
-#pragma unroll
-      for (int j = 0; j < DPL; ++j) acc_o[j] = fmaf(wgt, __ldcg(ps + j), acc_o[j]);
-    }
-  }
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) Ls += __shfl_xor_sync(0xffffffffu, Ls, o);
-}
-
-// Counts this warp's arrival on *counter (release of its partial stores, acquire of
-// the others'); true for the last of `expected` arrivals, which resets the counter.
-__device__ __forceinline__ bool arrive_last(int* counter, int expected, int lane) {
-  __syncwarp();
-  int arrivals = 0;
-  if (lane == 0) arrivals = atom_add_acq_rel(counter, 1);
-  __syncwarp();
-  arrivals = __shfl_sync(0xffffffffu, arrivals, 0);
-  if (arrivals != expected - 1) return false;
-  if (lane == 0) *counter = 0;  // ready for the next call
-  return true;
-}
-
 // A (query, head) row at its end: lane holds DPL consecutive dims from dim0 of the
 // unnormalised sum acc = sum_j p_j v_j (weights relative to max M, log2 domain) and the
-// row's weight sum L.  One split: the bf16 row.  Otherwise the split's fp32 partial,
-// merged in two levels: the last split of each group of kMergeGroup to arrive folds the
-// group into the group's first partial, and the last group to arrive merges the groups
-// into the row (one level when nsplit <= kMergeGroup).
+// row's weight sum L.  One split: the bf16 row.  Otherwise the split's fp32 partial
+// (acc, M, L), which the combine kernel merges with the query's other splits.
 template <int D>
-__device__ __forceinline__ void store_or_merge(const AttnKernelArgs& ka, const float* v, int dim0, float M, float L,
-                                               int sp, int qi, int qh, int nsplit, int base, int lane) {
+__device__ __forceinline__ void store_row(const AttnKernelArgs& ka, const float* v, int dim0, float M, float L, int sp,
+                                          int qi, int qh, int nsplit, int base, int lane) {
   constexpr int DPL = D / 32;
   const LayerArgs& a = ka.a;
-  const int64_t orow = (static_cast<int64_t>(qi) * a.Hq + qh) * D;
   if (nsplit == 1) {
+    const int64_t orow = (static_cast<int64_t>(qi) * a.Hq + qh) * D;
     const float inv = L > 0.f ? 1.f / L : 0.f;
 #pragma unroll
     for (int j = 0; j < DPL; j += 2)
       *reinterpret_cast<__nv_bfloat162*>(ka.out + orow + dim0 + j) = __floats2bfloat162_rn(v[j] * inv, v[j + 1] * inv);
     return;
   }
-  const int64_t sstride = static_cast<int64_t>(a.Hq) * (D + 4);
-  float* p0 = a.part + (static_cast<int64_t>(base) * a.Hq + qh) * (D + 4);  // split 0's partial
-  float* pp = p0 + sp * sstride;
+  float* pp = a.part + ((static_cast<int64_t>(base) + sp) * a.Hq + qh) * (D + 4);
 #pragma unroll
-  for (int j = 0; j < DPL; j += 2) *reinterpret_cast<float2*>(pp + dim0 + j) = make_float2(v[j], v[j + 1]);
-  if (lane == 0) *reinterpret_cast<float2*>(pp + D) = make_float2(M, L);
-  int* counters = a.cnt + (static_cast<int64_t>(qi) * a.Hq + qh) * a.cnt_stride;
-  float Mx, Ls, acc_o[DPL];
-  int ngroups = nsplit, gstride = 1;
-  if (nsplit > kMergeGroup) {
-    const int gr = sp / kMergeGroup, g0 = gr * kMergeGroup, gn = min(kMergeGroup, nsplit - g0);
-    if (!arrive_last(counters + 1 + gr, gn, lane)) return;
-    float* pg = p0 + g0 * sstride;
-    merge_partials<D>(pg, sstride, gn, lane, Mx, Ls, acc_o);
-    __syncwarp();  // every lane has read the group's rows before the first is overwritten
-#pragma unroll
-    for (int j = 0; j < DPL; ++j) __stcg(pg + lane * DPL + j, acc_o[j]);
-    if (lane == 0) __stcg(reinterpret_cast<float2*>(pg + D), make_float2(Mx, Ls));
-    ngroups = (nsplit + kMergeGroup - 1) / kMergeGroup;
-    gstride = kMergeGroup;
-  }
-  if (!arrive_last(counters, ngroups, lane)) return;
-  merge_partials<D>(p0, sstride * gstride, ngroups, lane, Mx, Ls, acc_o);
-  const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
-#pragma unroll
-  for (int j = 0; j < DPL; j += 2)
-    *reinterpret_cast<__nv_bfloat162*>(ka.out + orow + lane * DPL + j) =
-        __floats2bfloat162_rn(acc_o[j] * inv, acc_o[j + 1] * inv);
+  for (int j = 0; j < DPL; j += 2) __stcg(reinterpret_cast<float2*>(pp + dim0 + j), make_float2(v[j], v[j + 1]));
+  if (lane == 0) __stcg(reinterpret_cast<float2*>(pp + D), make_float2(M, L));
 }
 
 // ------------------------------------------------- CUDA-core consumer (MHA) --
@@ -872,7 +847,7 @@ __device__ __forceinline__ void finish_unit(const AttnKernelArgs& ka, LaneState&
     }
   }
   // lane (kl, part) now holds dims part*32 + DPL*kl .. + DPL-1 in acc[0 .. DPL-1]
-  store_or_merge<D>(ka, st.acc, part * 32 + DPL * kl, M, L, sp, qi, qh, nsplit, base, lane);
+  store_row<D>(ka, st.acc, part * 32 + DPL * kl, M, L, sp, qi, qh, nsplit, base, lane);
 }
 
 template <int D, int P>
@@ -1353,7 +1328,7 @@ __device__ __forceinline__ void mma_finish(const AttnKernelArgs& ka, MmaState<D,
 #pragma unroll
     for (int j = 0; j < DPL; ++j) v[j] = row[lane * DPL + j];
     const int qh = kv * g + r;
-    store_or_merge<D>(ka, v, lane * DPL, row[D], row[D + 1], sp, qi, qh, ns, base, lane);
+    store_row<D>(ka, v, lane * DPL, row[D], row[D + 1], sp, qi, qh, ns, base, lane);
   }
   __syncwarp();
 }
@@ -1470,7 +1445,8 @@ __device__ __forceinline__ void run_consumer_mma(const AttnKernelArgs& ka, const
 
 // The prologue every attention kernel shares: barriers, the dependency on the previous
 // kernel, the call's work units.
-__device__ __forceinline__ CtaRing attn_prologue(const AttnKernelArgs& ka, uint8_t* smem, int P, int NQB, int*& pre) {
+__device__ __forceinline__ CtaRing attn_prologue(const AttnKernelArgs& ka, uint8_t* smem, int P, int NQB, int*& pre,
+                                                 int*& perm) {
   const AttnSmem lay(ka.ring_bytes, ka.n, ka.scr_floats);
   CtaRing cr;
   cr.ring = smem + lay.ring;
@@ -1481,6 +1457,7 @@ __device__ __forceinline__ CtaRing attn_prologue(const AttnKernelArgs& ka, uint8
   cr.abort_flag = reinterpret_cast<volatile int*>(smem + lay.flag);
   cr.R = ka.ring_bytes;
   pre = reinterpret_cast<int*>(smem + lay.pre);
+  perm = reinterpret_cast<int*>(smem + lay.perm);
   if (threadIdx.x == 0) {
 #pragma unroll 1
     for (int i = 0; i < kStages; ++i) {
@@ -1492,7 +1469,7 @@ __device__ __forceinline__ CtaRing attn_prologue(const AttnKernelArgs& ka, uint8
   }
   pdl_wait();
   pdl_trigger();
-  plan_units(ka, P, NQB, pre, reinterpret_cast<long long*>(smem + lay.red));
+  plan_units(ka, P, NQB, pre, perm, reinterpret_cast<int*>(smem + lay.info), reinterpret_cast<int*>(smem + lay.red));
   return cr;
 }
 
@@ -1518,9 +1495,9 @@ __global__ void __launch_bounds__(32 * (kNcw + 1), kCtasPerSm) attn_kernel(const
   extern __shared__ __align__(128) uint8_t smem[];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int NQB = (ka.a.Hq + ka.hpu - 1) / ka.hpu;
-  int* pre;
-  const CtaRing cr = attn_prologue(ka, smem, P, NQB, pre);
-  if (warp == 0) run_producer<D>(ka, P, NQB, pre, cr, lane);
+  int *pre, *perm;
+  const CtaRing cr = attn_prologue(ka, smem, P, NQB, pre, perm);
+  if (warp == 0) run_producer<D>(ka, P, NQB, pre, perm, cr, lane);
   else run_consumer_cc<D, P>(ka, cr, warp - 1, lane);
   attn_epilogue(ka.a);
 }
@@ -1532,16 +1509,99 @@ __global__ void __launch_bounds__(32 * (kNcw + 1), kCtasPerSm) attn_mma_kernel(c
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int NQB = (ka.a.Hq + ka.hpu - 1) / ka.hpu;
   const int P = ka.a.P;
-  int* pre;
-  const CtaRing cr = attn_prologue(ka, smem, P, NQB, pre);
+  int *pre, *perm;
+  const CtaRing cr = attn_prologue(ka, smem, P, NQB, pre, perm);
   if (warp == 0) {
-    run_producer<D>(ka, P, NQB, pre, cr, lane);
+    run_producer<D>(ka, P, NQB, pre, perm, cr, lane);
   } else {
     const AttnSmem lay(ka.ring_bytes, ka.n, ka.scr_floats);
     float* scr = reinterpret_cast<float*>(smem + lay.scr) + (warp - 1) * ka.scr_floats;
     run_consumer_mma<D, NG>(ka, cr, P, warp - 1, lane, scr);
   }
   attn_epilogue(ka.a);
+}
+
+// ------------------------------------------------------------------ combine --
+// Merges the split partials of every (query, head) of a launch whose query has more
+// than one split: one CTA of kCombineWarps warps per (query, head); warp w folds splits
+// w, w + kCombineWarps, ... over its own maximum, then warp 0 folds the warps and
+// writes the bf16 row.  Chained after the attention kernel (programmatic dependent
+// launch): it reads nothing before that kernel has finished.
+constexpr int kCombineWarps = 4;
+
+struct CombineArgs {
+  const float* part;  // [units][Hq][D + 4] partials of the launch
+  const int2* qtab;   // [n] first partial and splits of each query
+  uint16_t* out;      // [n][Hq][D] bf16 rows of the launch
+  int Hq;
+};
+
+template <int D>
+__global__ void __launch_bounds__(32 * kCombineWarps) attn_combine_kernel(const __grid_constant__ CombineArgs ca) {
+  constexpr int DPL = D / 32;
+  __shared__ float sacc[kCombineWarps][D];
+  __shared__ float sml[kCombineWarps][2];
+  pdl_wait();
+  pdl_trigger();
+  const int qi = blockIdx.x / ca.Hq, qh = blockIdx.x - qi * ca.Hq;
+  const int2 e = ca.qtab[qi];
+  if (e.y <= 1) return;  // written by the attention kernel
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int64_t stride = static_cast<int64_t>(ca.Hq) * (D + 4);
+  const float* p0 = ca.part + (static_cast<int64_t>(e.x) * ca.Hq + qh) * (D + 4) + warp * stride;
+  const int64_t wstride = stride * kCombineWarps;  // between this warp's splits
+  const int cnt = (e.y - warp + kCombineWarps - 1) / kCombineWarps;
+  float Mx = kNegInf;
+  for (int s = lane; s < cnt; s += 32) Mx = fmaxf(Mx, __ldcg(p0 + s * wstride + D));
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) Mx = fmaxf(Mx, __shfl_xor_sync(0xffffffffu, Mx, o));
+  float Ls = 0.f, acc[DPL];
+#pragma unroll
+  for (int j = 0; j < DPL; ++j) acc[j] = 0.f;
+  for (int s0 = 0; s0 < cnt; s0 += 32) {
+    float wl = 0.f;  // lane s: weight of split s0 + s of this warp
+    if (s0 + lane < cnt) {
+      const float2 ml = __ldcg(reinterpret_cast<const float2*>(p0 + (s0 + lane) * wstride + D));
+      wl = (ml.x == kNegInf) ? 0.f : fast_exp2(ml.x - Mx);
+      Ls = fmaf(wl, ml.y, Ls);
+    }
+    const int m = min(32, cnt - s0);
+#pragma unroll 8
+    for (int s = 0; s < m; ++s) {
+      const float wgt = __shfl_sync(0xffffffffu, wl, s);
+      const float* ps = p0 + (s0 + s) * wstride + lane * DPL;
+#pragma unroll
+      for (int j = 0; j < DPL; ++j) acc[j] = fmaf(wgt, __ldcg(ps + j), acc[j]);
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) Ls += __shfl_xor_sync(0xffffffffu, Ls, o);
+#pragma unroll
+  for (int j = 0; j < DPL; ++j) sacc[warp][lane * DPL + j] = acc[j];
+  if (lane == 0) {
+    sml[warp][0] = Mx;
+    sml[warp][1] = Ls;
+  }
+  __syncthreads();
+  if (warp != 0) return;
+  float M = kNegInf;
+#pragma unroll
+  for (int w = 0; w < kCombineWarps; ++w) M = fmaxf(M, sml[w][0]);
+  float L = 0.f, o[DPL];
+#pragma unroll
+  for (int j = 0; j < DPL; ++j) o[j] = 0.f;
+#pragma unroll
+  for (int w = 0; w < kCombineWarps; ++w) {
+    const float f = sml[w][0] == kNegInf ? 0.f : fast_exp2(sml[w][0] - M);
+    L = fmaf(f, sml[w][1], L);
+#pragma unroll
+    for (int j = 0; j < DPL; ++j) o[j] = fmaf(f, sacc[w][lane * DPL + j], o[j]);
+  }
+  const float inv = L > 0.f ? 1.f / L : 0.f;
+  uint16_t* orow = ca.out + (static_cast<int64_t>(qi) * ca.Hq + qh) * D + lane * DPL;
+#pragma unroll
+  for (int j = 0; j < DPL; j += 2)
+    *reinterpret_cast<__nv_bfloat162*>(orow + j) = __floats2bfloat162_rn(o[j] * inv, o[j + 1] * inv);
 }
 
 constexpr int kAttnSmemLimit = 72 * 1024;  // dynamic shared memory of one attention CTA
@@ -1580,52 +1640,81 @@ static int attn_ring_bytes(const Layout& l, int n, int hpu, int scr_floats) {
   return ring;
 }
 
-// The one launch of an attention call with the given scratch views in `a`.
+// Queries per launch: their unit tables live in the CTAs' shared memory; a call with
+// more queries is cut into launches of this many, chained on the stream.
+constexpr int kMaxLaunchQueries = 1024;
+
+static cudaError_t launch_one(const Layout& l, const AttnKernelArgs& ka, int num_sms, cudaStream_t s) {
+  const bool mma = use_mma(l);
+  const int ring = attn_ring_bytes(l, ka.n, ka.hpu, ka.scr_floats);
+  if (ring < 0) return cudaErrorInvalidConfiguration;
+  AttnKernelArgs k = ka;
+  k.ring_bytes = ring;
+  const size_t sm = static_cast<size_t>(AttnSmem(ring, k.n, k.scr_floats).total);
+  const dim3 grid(kCtasPerSm * num_sms), block(32 * (kNcw + 1));
+  if (mma) {
+    const int ng = l.d / l.G;
+    if (l.d == 64) {
+      if (ng == 1) return launch_pdl(attn_mma_kernel<64, 1>, grid, block, sm, s, k);
+      return launch_pdl(attn_mma_kernel<64, 2>, grid, block, sm, s, k);
+    }
+    if (ng == 1) return launch_pdl(attn_mma_kernel<128, 1>, grid, block, sm, s, k);
+    if (ng == 2) return launch_pdl(attn_mma_kernel<128, 2>, grid, block, sm, s, k);
+    return launch_pdl(attn_mma_kernel<128, 4>, grid, block, sm, s, k);
+  }
+  // one kernel per head size and page size: the page loop unrolls, and a kernel's code
+  // holds only the four width classes it can meet
+  if (l.d == 64) {
+    if (l.P == 16) return launch_pdl(attn_kernel<64, 16>, grid, block, sm, s, k);
+    if (l.P == 32) return launch_pdl(attn_kernel<64, 32>, grid, block, sm, s, k);
+    return launch_pdl(attn_kernel<64, 64>, grid, block, sm, s, k);
+  }
+  if (l.P == 16) return launch_pdl(attn_kernel<128, 16>, grid, block, sm, s, k);
+  if (l.P == 32) return launch_pdl(attn_kernel<128, 32>, grid, block, sm, s, k);
+  return launch_pdl(attn_kernel<128, 64>, grid, block, sm, s, k);
+}
+
+// The launches of an attention call with the given scratch views in `a`; *launches
+// counts them.
 static cudaError_t launch_attention(const Layout& l, const LayerArgs& a, int num_sms, int n,
                                     const int32_t* seq_ids, const int32_t* q_positions, const void* q_bf16,
                                     const uint8_t* modes, const int32_t* windows, int window_scalar,
-                                    float softmax_scale, void* out_bf16, cudaStream_t s) {
+                                    float softmax_scale, void* out_bf16, cudaStream_t s, int* launches) {
+  *launches = 0;
   AttnKernelArgs ka;
   ka.a = a;
-  ka.n = n;
-  ka.seq_ids = seq_ids;
-  ka.q_positions = q_positions;
-  ka.modes = modes;
-  ka.windows = windows;
   ka.window_scalar = window_scalar;
-  ka.q = static_cast<const uint16_t*>(q_bf16);
-  ka.out = static_cast<uint16_t*>(out_bf16);
   const float scale = softmax_scale > 0.f ? softmax_scale : 1.f / sqrtf(static_cast<float>(l.d));
   ka.qscale = scale * 1.4426950408889634f;
   const bool mma = use_mma(l);
   const int g = l.Hq / l.Hkv;
   ka.hpu = mma ? kNcw * g : kNcw;
   ka.scr_floats = mma ? g * (l.d + 4) : 0;
-  const int ring = attn_ring_bytes(l, n, ka.hpu, ka.scr_floats);
-  if (ring < 0) return cudaErrorInvalidConfiguration;
-  ka.ring_bytes = ring;
-  const size_t sm = static_cast<size_t>(AttnSmem(ring, n, ka.scr_floats).total);
-  const dim3 grid(kCtasPerSm * num_sms), block(32 * (kNcw + 1));
-  if (mma) {
-    const int ng = l.d / l.G;
-    if (l.d == 64) {
-      if (ng == 1) return launch_pdl(attn_mma_kernel<64, 1>, grid, block, sm, s, ka);
-      return launch_pdl(attn_mma_kernel<64, 2>, grid, block, sm, s, ka);
-    }
-    if (ng == 1) return launch_pdl(attn_mma_kernel<128, 1>, grid, block, sm, s, ka);
-    if (ng == 2) return launch_pdl(attn_mma_kernel<128, 2>, grid, block, sm, s, ka);
-    return launch_pdl(attn_mma_kernel<128, 4>, grid, block, sm, s, ka);
+  const int64_t row = static_cast<int64_t>(l.Hq) * l.d;  // bf16 elements per query
+  for (int q0 = 0; q0 < n; q0 += kMaxLaunchQueries) {
+    ka.n = std::min(kMaxLaunchQueries, n - q0);
+    ka.q0 = q0;
+    ka.seq_ids = seq_ids + q0;
+    ka.q_positions = q_positions + q0;
+    ka.modes = modes + q0;
+    ka.windows = windows ? windows + q0 : nullptr;
+    ka.q = static_cast<const uint16_t*>(q_bf16) + q0 * row;
+    ka.out = static_cast<uint16_t*>(out_bf16) + q0 * row;
+    ka.a.qtab = a.qtab + q0;
+    cudaError_t e = launch_one(l, ka, num_sms, s);
+    if (e != cudaSuccess) return e;
+    CombineArgs ca;
+    ca.part = a.part;
+    ca.qtab = ka.a.qtab;
+    ca.out = ka.out;
+    ca.Hq = l.Hq;
+    const dim3 cgrid(ka.n * l.Hq), cblock(32 * kCombineWarps);
+    e = l.d == 64 ? launch_pdl(attn_combine_kernel<64>, cgrid, cblock, 0, s, ca)
+                  : launch_pdl(attn_combine_kernel<128>, cgrid, cblock, 0, s, ca);
+    if (e != cudaSuccess) return e;
+    *launches += 2;
   }
-  // one kernel per head size and page size: the page loop unrolls, and a kernel's code
-  // holds only the four width classes it can meet
-  if (l.d == 64) {
-    if (l.P == 16) return launch_pdl(attn_kernel<64, 16>, grid, block, sm, s, ka);
-    if (l.P == 32) return launch_pdl(attn_kernel<64, 32>, grid, block, sm, s, ka);
-    return launch_pdl(attn_kernel<64, 64>, grid, block, sm, s, ka);
-  }
-  if (l.P == 16) return launch_pdl(attn_kernel<128, 16>, grid, block, sm, s, ka);
-  if (l.P == 32) return launch_pdl(attn_kernel<128, 32>, grid, block, sm, s, ka);
-  return launch_pdl(attn_kernel<128, 64>, grid, block, sm, s, ka);
+  return cudaSuccess;
 }
 
 }  // namespace trr
@@ -1645,17 +1734,18 @@ extern "C" trr_status trr_decode_attn(trr_cache* cache, int32_t layer, int32_t n
   if ((reinterpret_cast<uintptr_t>(q_bf16) | reinterpret_cast<uintptr_t>(out_bf16)) & 15)
     return TRR_ERR_INVALID_ARG;
   const LayerArgs a = layer_args(l, cache_views(cache), layer);
+  int launches = 0;
   const cudaError_t e = launch_attention(l, a, cache_num_sms(cache), n, seq_ids, q_positions, q_bf16, modes,
                                          windows, window_scalar, softmax_scale, out_bf16,
-                                         static_cast<cudaStream_t>(stream));
-  cache_set_launches(cache, 1);
+                                         static_cast<cudaStream_t>(stream), &launches);
+  cache_set_launches(cache, launches);
   return e == cudaSuccess ? TRR_OK : TRR_ERR_CUDA;
 }
 
 // ------------------------------------------------------ static-scratch variant --
 //
-// trr_decode_attn_static runs the same kernel as trr_decode_attn, but keeps all of its
-// per-call scratch (arrival counters, fp32 partials and the call's control words) in one
+// trr_decode_attn_static runs the same kernels as trr_decode_attn, but keeps all of its
+// per-call scratch (the query table, fp32 partials and the call's control words) in one
 // file-scope device array instead of the cache's scratch region.  Nothing is allocated
 // per call or at set-up.
 namespace trr {
@@ -1682,11 +1772,10 @@ static cudaError_t static_scratch(void** out) {
   return cudaSuccess;
 }
 
-// Clears what a call needs at zero: the control words and the arrival counters.
-__global__ void static_scratch_clear_kernel(int32_t* wctrl, int32_t* cnt, int ncnt) {
-  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+// Clears what a call needs at zero: the control words.
+__global__ void static_scratch_clear_kernel(int32_t* wctrl) {
+  const int i = threadIdx.x;
   if (i < kCtrlInts) wctrl[i] = i == kFirstBadQuery ? INT_MAX : 0;
-  for (int j = i; j < ncnt; j += gridDim.x * blockDim.x) cnt[j] = 0;
 }
 
 // Forwards the call's first error to the cache's sticky status word.
@@ -1712,26 +1801,26 @@ extern "C" trr_status trr_decode_attn_static(trr_cache* cache, int32_t layer, in
   // scratch of this call, carved from the static array; reject what does not fit
   auto up = [](int64_t x) { return (x + 255) / 256 * 256; };
   const int64_t b_ctrl = up(4 * kCtrlInts);
-  const int64_t b_cnt = up(4ll * n * l.units * l.cnt_stride);
+  const int64_t b_qtab = up(8ll * n);
   const int64_t b_part = up(4ll * n * l.s_cap * l.units * (l.d + 4));
-  if (b_ctrl + b_cnt + b_part > kStaticScratchBytes) return TRR_ERR_OUT_OF_MEMORY;
+  if (b_ctrl + b_qtab + b_part > kStaticScratchBytes) return TRR_ERR_OUT_OF_MEMORY;
   void* base = nullptr;
   if (static_scratch(&base) != cudaSuccess) return TRR_ERR_CUDA;
   uint8_t* b = static_cast<uint8_t*>(base);
   LayerArgs a = layer_args(l, cache_views(cache), layer);
   int32_t* cache_ctrl = a.ctrl;
   a.ctrl = reinterpret_cast<int32_t*>(b);
-  a.cnt = reinterpret_cast<int32_t*>(b + b_ctrl);
-  a.part = reinterpret_cast<float*>(b + b_ctrl + b_cnt);
+  a.qtab = reinterpret_cast<int2*>(b + b_ctrl);
+  a.part = reinterpret_cast<float*>(b + b_ctrl + b_qtab);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const int ncnt = n * l.units * l.cnt_stride;
-  static_scratch_clear_kernel<<<std::max(1, std::min(256, (ncnt + 255) / 256)), 256, 0, s>>>(a.ctrl, a.cnt, ncnt);
+  static_scratch_clear_kernel<<<1, kCtrlInts, 0, s>>>(a.ctrl);
   cudaError_t e = cudaGetLastError();
+  int launches = 0;
   if (e == cudaSuccess)
     e = launch_attention(l, a, cache_num_sms(cache), n, seq_ids, q_positions, q_bf16, modes, windows,
-                         window_scalar, softmax_scale, out_bf16, s);
+                         window_scalar, softmax_scale, out_bf16, s, &launches);
   if (e != cudaSuccess) return TRR_ERR_CUDA;
   static_scratch_status_kernel<<<1, 1, 0, s>>>(a.ctrl, cache_ctrl);
-  cache_set_launches(cache, 3);
+  cache_set_launches(cache, launches + 2);
   return cudaGetLastError() == cudaSuccess ? TRR_OK : TRR_ERR_CUDA;
 }

@@ -19,7 +19,6 @@ LayerArgs layer_args(const Layout& l, const Views& v, int layer) {
   a.S = l.S; a.Hq = l.Hq; a.Hkv = l.Hkv; a.d = l.d; a.G = l.G; a.P = l.P;
   a.maxctx = l.maxctx; a.MP = l.MP; a.W32 = l.W32; a.units = l.units; a.pos_split = l.pos_split;
   a.s_cap = l.s_cap;
-  a.cnt_stride = l.cnt_stride;
   a.split_bytes = l.split_bytes; a.skip_writes_kv = l.skip_writes_kv;
   a.hdr = static_cast<int>(l.hdr);
   for (int c = 0; c < kClasses; ++c) {
@@ -38,7 +37,7 @@ LayerArgs layer_args(const Layout& l, const Views& v, int layer) {
   a.plast = v.plast + ls * 4 * l.MP;
   a.lastpg = v.lastpg + ls * 4;
   a.aplan = v.aplan;
-  a.cnt = v.cnt;
+  a.qtab = v.qtab;
   a.part = v.part;
   return a;
 }
@@ -85,7 +84,6 @@ static trr_status make_layout(const trr_cache_config* c, Layout* l) {
   l->pos_split = static_cast<int>(std::max<int64_t>(l->P, l->split_bytes / l->tokb[2]));
   l->s_cap = 1 << 30;
   l->s_cap = std::max(splits_of(l->maxctx, l->pos_split, l->P, l->s_cap), 1);
-  l->cnt_stride = 1 + (l->s_cap + kMergeGroup - 1) / kMergeGroup;
   l->max_items = static_cast<int64_t>(l->max_queries) * l->units * l->s_cap;
 
   const int64_t nls = static_cast<int64_t>(l->L) * l->S;
@@ -104,7 +102,7 @@ static trr_status make_layout(const trr_cache_config* c, Layout* l) {
   l->off_plast = take(16 * nls * l->MP);
   l->off_lastpg = take(16 * nls);
   l->off_aplan = take(static_cast<int64_t>(sizeof(AppendPlan)) * l->max_append);
-  l->off_cnt = take(4 * static_cast<int64_t>(l->max_queries) * l->units * l->cnt_stride);
+  l->off_qtab = take(8 * static_cast<int64_t>(l->max_queries));
   l->off_part = take(4 * l->max_items * (l->Hq / l->units) * (l->d + 4));
   for (int k = 0; k < kClasses; ++k) l->off_pool[k] = take(l->cap[k] * l->page_bytes[k]);
   l->total = off;
@@ -150,8 +148,6 @@ static trr_status clear_metadata(trr_cache* c, cudaStream_t s) {
   ok = ok && cudaMemsetAsync(b + l.off_presence, 0, 4 * nls * l.W32, s) == cudaSuccess;
   ok = ok && cudaMemsetAsync(b + l.off_pt, 0xFF, 3 * (l.off_pfirst - l.off_pt), s) == cudaSuccess;
   ok = ok && cudaMemsetAsync(b + l.off_lastpg, 0xFF, 16 * nls, s) == cudaSuccess;
-  ok = ok && cudaMemsetAsync(b + l.off_cnt, 0, 4 * static_cast<int64_t>(l.max_queries) * l.units * l.cnt_stride, s) ==
-                  cudaSuccess;
   return ok ? TRR_OK : TRR_ERR_CUDA;
 }
 

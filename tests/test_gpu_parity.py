@@ -63,12 +63,12 @@ CONFIGS = [  # d, G, P, Hq, Hkv
 
 
 def _random_setup(rng, d, G, P, Hq, Hkv, ctxs, bits_p=(0.25, 0.25, 0.25, 0.25),
-                  modes_p=(0.2, 0.4, 0.4), skip_writes_kv=0, per_call=1024, split_bytes=0):
+                  modes_p=(0.2, 0.4, 0.4), skip_writes_kv=0, per_call=1024, split_bytes=0, max_queries=1024):
     S = len(ctxs)
     maxctx = max(ctxs) + 8
     caps = [S * (maxctx // P + 2)] * 4
     pair = Pair(1, S, Hq, Hkv, d, G, P, maxctx, caps, skip_writes_kv=skip_writes_kv,
-                split_bytes=split_bytes)
+                split_bytes=split_bytes, max_queries=max_queries)
     ent = [(s, p) for p in range(max(ctxs)) for s in range(S) if p < ctxs[s]]
     bits = {(s, p): int(rng.choice([2, 4, 8, 16], p=bits_p)) for s, p in ent}
     modes = {(s, p): int(rng.choice(3, p=modes_p)) for s, p in ent}
@@ -111,6 +111,27 @@ def test_many_splits_and_small_split_bytes():
     for _ in range(3):  # repeated calls reuse the arrival counters
         pair.attend(0, [0, 1, 2, 0, 1, 2], [899, 1499, 39, 500, 1000, 20],
                     q, [FULL, FULL, FULL, LOCAL, LOCAL, LOCAL], window_scalar=300)
+
+
+def test_calls_above_one_launch_of_queries_and_an_error_in_the_second():
+    """More queries than one launch takes (1024): the call runs as several launches,
+    each with its own work units and merges, and an invalid query in the second one is
+    reported with its index in the whole call (the lowest failing index)."""
+    rng = np.random.default_rng(31)
+    ctxs = [70, 260, 130, 33]
+    for Hq, Hkv in ((4, 4), (8, 2)):  # CUDA-core and tensor-core consumers
+        pair, ent, _, _ = _random_setup(rng, 64, 32, 16, Hq, Hkv, ctxs, split_bytes=1024, max_queries=2048)
+        nq = 1100
+        seqs = rng.integers(0, len(ctxs), nq)
+        ts = np.array([rng.integers(0, ctxs[s]) for s in seqs])
+        ms = rng.choice(3, size=nq)
+        ws = rng.choice([1, 5, 40, 300], size=nq)
+        q = wl.bf16_bits(rng.standard_normal((nq, Hq, 64), dtype=np.float32))
+        pair.attend(0, seqs, ts, q, ms, windows=ws)
+        bad = ms.copy()
+        bad[1050] = 7  # not a mode
+        got, ref = pair.attend(0, seqs, ts, q, bad, windows=ws, expect=1)
+        assert (got[1050] == 0).all()
 
 
 def test_bulk_append_with_repeated_sequences_equals_incremental():
