@@ -160,16 +160,16 @@ TRR_API trr_status trr_decode_attn(trr_cache* cache, int32_t layer, int32_t n,
 /* trr_decode_attn without any per-call scratch in the cache's memory (this entry point
  * has no counterpart in the paper; it serves callers that cannot allocate).
  *   Same arguments, results and error contract as trr_decode_attn, but its scratch
- *   (control words, the per-query split table, fp32 partials) lives in one
+ *   (control words, split arrival counters, fp32 partials) lives in one
  *   32 MiB array that the library declares as a static device variable: every GPU that
  *   loads the library holds it until the process exits, and no call allocates device
  *   memory.  This is for callers that must not call cudaMalloc at the point of the
  *   call, such as an engine running inside a fixed, fully reserved memory budget, and
  *   that need more queries per call than the cache's max_queries scratch was sized
  *   for: n is bounded by the array instead of by max_queries.
- *   The call needs 256 + 8 * n + n * Hq * S_cap * (4*d + 16) bytes (plus 256-byte
- *   rounding per region), with S_cap the most splits per query of this cache; a call
- *   above 32 MiB returns TRR_ERR_OUT_OF_MEMORY and launches nothing.
+ *   The call needs 256 + n * Hq * (4 * (1 + ceil(S_cap / 8)) + S_cap * (4*d + 16))
+ *   bytes (plus 256-byte rounding per region), with S_cap the most splits per query of
+ *   this cache; a call above 32 MiB returns TRR_ERR_OUT_OF_MEMORY and launches nothing.
  *   The first call on a device looks up the array's device address (once per device,
  *   with that device current); make that first call before any stream capture.
  *   Every call clears what must start at zero and then overwrites the array, so calls

@@ -102,7 +102,7 @@ __device__ __forceinline__ float bf_hi(uint32_t w) { return __uint_as_float(w & 
 // exact 2^e, -126 <= e <= 127 (folds to a constant for constant e)
 __device__ __forceinline__ float pow2f(int e) { return __int_as_float((127 + e) << 23); }
 
-// Bit offset of element i (of a lane's 32) inside the word it is extracted from.
+// Bit offset of element i (of a lane's 16 or 32) inside the word it is extracted from.
 __host__ __device__ constexpr int ex_of(int B, int i) {
   return B == 2 ? ((i % 16) < 11 ? 2 * (i % 16) : 2 * (i % 16 - 11))
                 : B == 4 ? ((i % 8) < 5 ? 4 * (i % 8) : 4 * (i % 8 - 5)) : 0;
@@ -126,11 +126,12 @@ __device__ __forceinline__ float code_at(const uint32_t* w, const uint32_t* h, i
 // d = a * b + c on two fp32 lanes at once (packed fp32 FMA, round to nearest).
 __device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) { return __ffma2_rn(a, b, c); }
 
-template <int B>
+// The words' high parts (codes past the binary32 mantissa, shifted down); NW words.
+template <int B, int NW>
 __device__ __forceinline__ void high_parts(const uint32_t* w, uint32_t* h) {
   constexpr int sh = B == 2 ? 22 : B == 4 ? 20 : 16;
 #pragma unroll
-  for (int k = 0; k < B; ++k) h[k] = w[k] >> sh;
+  for (int k = 0; k < NW; ++k) h[k] = w[k] >> sh;
 }
 
 // x *= f on pairs of fp32 lanes (packed multiply)
@@ -140,27 +141,28 @@ __device__ __forceinline__ void fmul2_inplace(float& x0, float& x1, float f0, fl
   x1 = r.y;
 }
 
-template <int BFROM, int BTO>
-__device__ __forceinline__ void rescale_q(float (&qp)[32]) {
+template <int BFROM, int BTO, int E>
+__device__ __forceinline__ void rescale_q(float (&qp)[E]) {
 #pragma unroll
-  for (int i = 0; i < 32; i += 2)
+  for (int i = 0; i < E; i += 2)
     fmul2_inplace(qp[i], qp[i + 1], pow2f(qe_of(BTO, i) - qe_of(BFROM, i)),
                   pow2f(qe_of(BTO, i + 1) - qe_of(BFROM, i + 1)));
 }
 
 // V is accumulated as acc_i * 2^(ex_i(B) - 49) while class B's pages are consumed
 // (B = 16: ex = 0), so that every element of a key takes the same weight p*s*2^100.
-template <int BFROM, int BTO>
-__device__ __forceinline__ void rescale_acc(float (&acc)[32]) {
+template <int BFROM, int BTO, int E>
+__device__ __forceinline__ void rescale_acc(float (&acc)[E]) {
 #pragma unroll
-  for (int i = 0; i < 32; i += 2)
+  for (int i = 0; i < E; i += 2)
     fmul2_inplace(acc[i], acc[i + 1],
                   pow2f((BTO == 16 ? 0 : ex_of(BTO, i)) - (BFROM == 16 ? 0 : ex_of(BFROM, i))),
                   pow2f((BTO == 16 ? 0 : ex_of(BTO, i + 1)) - (BFROM == 16 ? 0 : ex_of(BFROM, i + 1))));
 }
 
 // qp from the domain of class `from` to that of class `to` (from < to, or from = 16).
-__device__ __forceinline__ void rescale_dyn(float (&qp)[32], float (&acc)[32], int from, int to) {
+template <int E>
+__device__ __forceinline__ void rescale_dyn(float (&qp)[E], float (&acc)[E], int from, int to) {
   switch (from * 4 + to) {
     case 1: rescale_q<2, 4>(qp); rescale_acc<2, 4>(acc); break;
     case 2: rescale_q<2, 8>(qp); rescale_acc<2, 8>(acc); break;
@@ -175,7 +177,8 @@ __device__ __forceinline__ void rescale_dyn(float (&qp)[32], float (&acc)[32], i
   }
 }
 // acc from class `from`'s domain back to class 16's (the common one of the merge)
-__device__ __forceinline__ void acc_to_neutral(float (&acc)[32], int from) {
+template <int E>
+__device__ __forceinline__ void acc_to_neutral(float (&acc)[E], int from) {
   switch (from) {
     case 0: rescale_acc<2, 16>(acc); break;
     case 1: rescale_acc<4, 16>(acc); break;
@@ -192,9 +195,10 @@ __device__ __forceinline__ float fast_exp2(float x) {
   return y;
 }
 
+template <int E>
 struct LaneState {
   float m, l, zacc;  // running max (log2), sum of weights, sum of p*z (V zero points)
-  float acc[32];     // sum of p*v over the lane's 32 dims, scaled by 2^-49
+  float acc[E];      // sum of p*v over the lane's E dims, scaled by 2^-49
 };
 
 // Shared-memory loads at 32-bit shared addresses.  Volatile: they stay after the
@@ -215,16 +219,19 @@ __device__ __forceinline__ uint32_t lds32(uint32_t a) {
   return v;
 }
 
-// The B words of 32 B-bit codes at shared address a (4B-byte aligned), in as few loads as
-// possible (one 8- or 16-byte load per row part keeps the warp's request conflict-free).
-template <int B>
+// The NW words of a lane's codes at shared address a (4 NW-byte aligned), in as few
+// loads as possible (one 4-, 8- or 16-byte load per row part keeps the warp's request
+// conflict-free).
+template <int NW>
 __device__ __forceinline__ void lds_codes(uint32_t a, uint32_t* w) {
-  if (B == 2) {
+  if (NW == 1) {
+    w[0] = lds32(a);
+  } else if (NW == 2) {
     const uint2 u = lds64(a);
     w[0] = u.x; w[1] = u.y;
   } else {
 #pragma unroll
-    for (int k = 0; k < B; k += 4) {
+    for (int k = 0; k < NW; k += 4) {
       const uint4 u = lds128(a + 4 * k);
       w[k] = u.x; w[k + 1] = u.y; w[k + 2] = u.z; w[k + 3] = u.w;
     }
@@ -234,14 +241,14 @@ __device__ __forceinline__ void lds_codes(uint32_t a, uint32_t* w) {
 // One page of width class B (P = NIT * keys per iteration tokens) at shared address s0;
 // lane -> (key kl, 32-dim part).  Keys past `fill` are empty slots; with positions at
 // spos (masked pages), keys outside [lo, hi] are masked too.
-// q.k of one key at shared address ka (this lane's 32 dims) in class B, with its (s, z)
+// q.k of one key at shared address ka (this lane's E dims) in class B, with its (s, z)
 // word at kszaddr for B < 16: s * sum(q_i c_i) + z * sum(q_i) in the domain of qp.
-template <int B>
-__device__ __forceinline__ float k_dot(uint32_t ka, uint32_t kszaddr, const float (&qp)[32], float sumq) {
+template <int B, int E>
+__device__ __forceinline__ float k_dot(uint32_t ka, uint32_t kszaddr, const float (&qp)[E], float sumq) {
   float2 d2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
   if (B == 16) {
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
+    for (int q = 0; q < E / 8; ++q) {
       const uint4 u = lds128(ka + 16 * q);
       d2[0] = ffma2(make_float2(qp[8 * q + 0], qp[8 * q + 1]), make_float2(bf_lo(u.x), bf_hi(u.x)), d2[0]);
       d2[1] = ffma2(make_float2(qp[8 * q + 2], qp[8 * q + 3]), make_float2(bf_lo(u.y), bf_hi(u.y)), d2[1]);
@@ -250,27 +257,28 @@ __device__ __forceinline__ float k_dot(uint32_t ka, uint32_t kszaddr, const floa
     }
     return (d2[0].x + d2[0].y) + (d2[1].x + d2[1].y);
   }
-  uint32_t w[B], h[B];
-  lds_codes<B>(ka, w);
-  if (B != 8) high_parts<B>(w, h);
+  constexpr int NW = E * B / 32;
+  uint32_t w[NW], h[NW];
+  lds_codes<NW>(ka, w);
+  if (B != 8) high_parts<B, NW>(w, h);
   const uint32_t szw = lds32(kszaddr);
 #pragma unroll
-  for (int i = 0; i < 16; ++i)
+  for (int i = 0; i < E / 2; ++i)
     d2[i & 1] = ffma2(make_float2(qp[2 * i], qp[2 * i + 1]),
                       make_float2(code_at<B>(w, h, 2 * i), code_at<B>(w, h, 2 * i + 1)), d2[i & 1]);
   const float2 sz = __half22float2(*reinterpret_cast<const __half2*>(&szw));  // (s, z)
   return fmaf(sz.x * pow2f(49), (d2[0].x + d2[0].y) + (d2[1].x + d2[1].y), sz.y * sumq);
 }
 
-// acc += p * v for one key's V at shared address va (this lane's 32 dims) in class B,
+// acc += p * v for one key's V at shared address va (this lane's E dims) in class B,
 // with its (s, z) word at vszaddr for B < 16.
-template <int B>
-__device__ __forceinline__ void v_acc(uint32_t va, uint32_t vszaddr, float p, LaneState& st) {
+template <int B, int E>
+__device__ __forceinline__ void v_acc(uint32_t va, uint32_t vszaddr, float p, LaneState<E>& st) {
   if (B == 16) {
     const float wv = p * pow2f(-49);
     const float2 w2 = make_float2(wv, wv);
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
+    for (int q = 0; q < E / 8; ++q) {
       const uint4 u = lds128(va + 16 * q);
       const uint32_t uw[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
@@ -283,15 +291,16 @@ __device__ __forceinline__ void v_acc(uint32_t va, uint32_t vszaddr, float p, La
     }
     return;
   }
-  uint32_t w[B], h[B];
-  lds_codes<B>(va, w);
-  if (B != 8) high_parts<B>(w, h);
+  constexpr int NW = E * B / 32;
+  uint32_t w[NW], h[NW];
+  lds_codes<NW>(va, w);
+  if (B != 8) high_parts<B, NW>(w, h);
   const uint32_t szw = lds32(vszaddr);
   const float2 sz = __half22float2(*reinterpret_cast<const __half2*>(&szw));  // (s, z)
   const float wb = p * sz.x * pow2f(100);
   const float2 w2 = make_float2(wb, wb);
 #pragma unroll
-  for (int i = 0; i < 32; i += 2) {
+  for (int i = 0; i < E; i += 2) {
     const float2 r = ffma2(w2, make_float2(code_at<B>(w, h, i), code_at<B>(w, h, i + 1)),
                            make_float2(st.acc[i], st.acc[i + 1]));
     st.acc[i] = r.x;
@@ -301,22 +310,22 @@ __device__ __forceinline__ void v_acc(uint32_t va, uint32_t vszaddr, float p, La
 }
 
 // One page of width class B (P = NIT * keys per iteration tokens) at shared address s0;
-// lane -> (key kl, 32-dim part), and two keys per lane per iteration (kl and kl + KPI)
+// lane -> (key kl, E-dim part), and two keys per lane per iteration (kl and kl + KPI)
 // when NIT is even, so that their dependency chains overlap.  Keys past `fill` are
 // empty slots; with positions at spos (masked pages), keys outside [lo, hi] are masked.
-template <int D, int B, int NIT>
+template <int D, int B, int NIT, int E>
 __device__ __forceinline__ void consume_page(uint32_t s0, uint32_t spos, bool masked, int G, int fill, int lo,
-                                             int hi, const float (&qp)[32], float sumq, LaneState& st, int lane) {
-  constexpr int LPK = D / 32;
+                                             int hi, const float (&qp)[E], float sumq, LaneState<E>& st, int lane) {
+  constexpr int LPK = D / E;
   constexpr int KPI = 32 / LPK;
   constexpr int P = NIT * KPI;
   constexpr int KP = NIT % 2 == 0 ? 2 : 1;  // keys per lane per iteration
   constexpr int rowb = B == 16 ? 2 * D : D * B / 8;  // bytes of one key's row of K (or V)
   const int part = lane % LPK, kl = lane / LPK;
   const int ng = D / G;
-  const int grp = part * 32 / G;
-  const uint32_t krow = s0 + kl * rowb + part * (B == 16 ? 64 : 4 * B);   // this lane's K bytes, key kl
-  const uint32_t ksz = s0 + 2 * P * rowb + (kl * ng + grp) * 4;           // its (s, z), key kl
+  const int grp = part * E / G;
+  const uint32_t krow = s0 + kl * rowb + part * (E * B / 8);   // this lane's K bytes, key kl
+  const uint32_t ksz = s0 + 2 * P * rowb + (kl * ng + grp) * 4;  // its (s, z), key kl
   const uint32_t szstep = KPI * ng * 4;
 #pragma unroll 1
   for (int it = 0; it < NIT; it += KP) {
@@ -330,7 +339,7 @@ __device__ __forceinline__ void consume_page(uint32_t s0, uint32_t spos, bool ma
         const int pos = static_cast<int>(lds32(spos + 4 * key));
         valid[k] = valid[k] && pos >= lo && pos <= hi;
       }
-      dot[k] = k_dot<B>(krow + (it + k) * KPI * rowb, ksz + (it + k) * szstep, qp, sumq);
+      dot[k] = k_dot<B, E>(krow + (it + k) * KPI * rowb, ksz + (it + k) * szstep, qp, sumq);
     }
 #pragma unroll
     for (int k = 0; k < KP; ++k) {
@@ -345,7 +354,7 @@ __device__ __forceinline__ void consume_page(uint32_t s0, uint32_t spos, bool ma
     if (top > st.m + kTau) {
       const float alpha = fast_exp2(st.m - top);  // 0 when m = -inf
 #pragma unroll
-      for (int j = 0; j < 32; ++j) st.acc[j] *= alpha;
+      for (int j = 0; j < E; ++j) st.acc[j] *= alpha;
       st.l *= alpha;
       st.zacc *= alpha;
       st.m = top;
@@ -356,7 +365,7 @@ __device__ __forceinline__ void consume_page(uint32_t s0, uint32_t spos, bool ma
         const float p = fast_exp2(dot[k] - st.m);
         st.l += p;
         const uint32_t va = krow + (it + k) * KPI * rowb + P * rowb;
-        v_acc<B>(va, ksz + (it + k) * szstep + P * ng * 4, p, st);
+        v_acc<B, E>(va, ksz + (it + k) * szstep + P * ng * 4, p, st);
       }
     }
   }
@@ -375,7 +384,16 @@ constexpr int kNcw = 4;           // consumer warps per CTA
 constexpr int kStages = 16;       // stage records a CTA may have in flight
 constexpr int kUnitsPerCta = 3;   // units per CTA of a large call, at most
 constexpr float kMinUnitPositions = 512.f;  // key positions of a large call's unit, at least
-constexpr int kCtasPerSm = 3;
+constexpr int kCtasPerSm = 3;     // CTAs per SM
+
+// Dims per lane of the CUDA-core consumer (E = 16 would use four lanes per key at d = 64
+// and half the registers, but it issues twice the instructions per key), and its CTAs
+// per SM.
+__host__ __device__ constexpr int cc_elems(int) { return 32; }
+__host__ __device__ constexpr int cc_ctas_per_sm(int) { return kCtasPerSm; }
+// dynamic shared memory of one attention CTA with `ctas` CTAs per SM (228 KB per SM,
+// 1 KB of it reserved per CTA)
+__host__ __device__ constexpr int attn_smem_limit(int ctas) { return ctas >= 5 ? 44 * 1024 : 72 * 1024; }
 
 // Stage record, three int4 words written by the producer before it arrives on the
 // stage's full barrier:
@@ -427,7 +445,7 @@ __device__ __forceinline__ int query_range(int t, int mode, int w) {
 // (mbarriers need 8, bulk-copy destinations 16).
 __host__ __device__ constexpr int align16(int x) { return (x + 15) & ~15; }
 struct AttnSmem {
-  int ring, recs, sbytes, full, empty, scr, pre, perm, info, red, flag, total;
+  int ring, recs, sbytes, full, empty, scr, pre, red, flag, total;
   __host__ __device__ AttnSmem(int ring_bytes, int n, int scr_floats)
       : ring(0),
         recs(align16(ring_bytes)),
@@ -436,10 +454,8 @@ struct AttnSmem {
         empty(full + kStages * 8),
         scr(empty + kStages * 8),
         pre(scr + align16(kNcw * scr_floats * 4)),
-        perm(pre + align16(4 * (n + 1))),
-        info(perm + align16(4 * n)),
-        red(info + align16(4 * n)),
-        flag(red + 64 * 4),
+        red(pre + align16(4 * (n + 1))),
+        flag(red + 16 * 8),
         total(flag + 16) {}
 };
 
@@ -527,32 +543,25 @@ __device__ __forceinline__ int plan_split(const LayerArgs& a, int P, int seq, in
   return T;
 }
 
-// The work units of a launch, computed the same way by every CTA: query q gets ns_q
-// splits from its key range.  Units are numbered largest first (queries in full mode,
-// then local, then skip or invalid ones, each group in query order), so that the last
-// units handed out are the small ones: query perm[k] is the k-th in that order, its
-// splits are units pre[k] .. pre[k + 1] - 1, and pre[n] counts them all.
-__device__ __forceinline__ void plan_units(const AttnKernelArgs& ka, int P, int NQB, int* pre, int* perm, int* info,
-                                           int* red) {
+// The work units of a call, computed the same way by every CTA: query q gets ns_q
+// splits from its key range; pre[q] numbers its first split, pre[n] counts them all.
+__device__ __forceinline__ void plan_units(const AttnKernelArgs& ka, int P, int NQB, int* pre, long long* red) {
   const LayerArgs& a = ka.a;
   const int n = ka.n, lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
   long long rsum = 0;
   for (int q = threadIdx.x; q < n; q += blockDim.x) {
     const int seq = ka.seq_ids[q], t = ka.q_positions[q], mode = ka.modes[q];
     const int w = ka.windows ? ka.windows[q] : ka.window_scalar;
-    const bool bad = query_error(a, seq, t, mode, w) != 0;
-    const int r = bad ? 0 : query_range(t, mode, w);
-    const int cls = bad ? 2 : mode == TRR_MODE_FULL ? 0 : mode == TRR_MODE_LOCAL ? 1 : 2;
-    info[q] = r | (cls << 29);  // r <= max_context <= 2^24
+    const int r = query_error(a, seq, t, mode, w) ? 0 : query_range(t, mode, w);
+    pre[q] = r;
     rsum += r;
   }
-  long long* red64 = reinterpret_cast<long long*>(red);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) rsum += __shfl_xor_sync(0xffffffffu, rsum, o);
-  if (lane == 0) red64[warp] = rsum;
+  if (lane == 0) red[warp] = rsum;
   __syncthreads();
   rsum = 0;
-  for (int k = 0; k < nwarps; ++k) rsum += red64[k];
+  for (int k = 0; k < nwarps; ++k) rsum += red[k];
   // Split size: a small call gets about one unit per CTA (its units are latency-bound
   // chains, and a second unit on a CTA doubles the call); a large one up to
   // kUnitsPerCta per CTA, each of at least kMinUnitPositions positions per head block
@@ -565,62 +574,28 @@ __device__ __forceinline__ void plan_units(const AttnKernelArgs& ka, int P, int 
   const float by_work = ceilf(rs / want);
   const int pos_split = by_work > static_cast<float>(a.pos_split) ? static_cast<int>(fminf(by_work, 1073741824.f))
                                                                    : a.pos_split;
-  // per class, this thread's queries and splits (a contiguous chunk of queries)
   const int chunk = (n + blockDim.x - 1) / blockDim.x;
   const int q0 = min(n, static_cast<int>(threadIdx.x) * chunk), q1 = min(n, q0 + chunk);
-  int v[6] = {0, 0, 0, 0, 0, 0};  // queries of class 0, 1, 2, then their splits
-  for (int q = q0; q < q1; ++q) {
-    const int i = info[q], c = i >> 29;
-    v[c] += 1;
-    v[3 + c] += splits_of(i & 0x1fffffff, pos_split, P, a.s_cap);
-  }
-  // exclusive scan over the threads, and the totals
-  int incl[6];
+  int mine = 0;
+  for (int q = q0; q < q1; ++q) mine += splits_of(pre[q], pos_split, P, a.s_cap);
+  int incl = mine;
 #pragma unroll
-  for (int j = 0; j < 6; ++j) {
-    incl[j] = v[j];
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const int x = __shfl_up_sync(0xffffffffu, incl[j], o);
-      if (lane >= o) incl[j] += x;
-    }
+  for (int o = 1; o < 32; o <<= 1) {
+    const int v = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += v;
   }
   __syncthreads();  // every read of red above is done
-  if (lane == 31) {
-#pragma unroll
-    for (int j = 0; j < 6; ++j) red[16 + warp * 6 + j] = incl[j];
-  }
+  if (lane == 31) red[8 + warp] = incl;
   __syncthreads();
-  int off[6], tot[6];
-#pragma unroll
-  for (int j = 0; j < 6; ++j) {
-    off[j] = incl[j] - v[j];
-    tot[j] = 0;
-    for (int k = 0; k < nwarps; ++k) {
-      const int x = red[16 + k * 6 + j];
-      if (k < warp) off[j] += x;
-      tot[j] += x;
-    }
-  }
-  // class c's ranks and units follow those of the classes before it
-  off[1] += tot[0];
-  off[2] += tot[0] + tot[1];
-  off[4] += tot[3];
-  off[5] += tot[3] + tot[4];
+  int off = incl - mine;
+  for (int k = 0; k < warp; ++k) off += static_cast<int>(red[8 + k]);
   for (int q = q0; q < q1; ++q) {
-    const int i = info[q], c = i >> 29;
-    const int ns = splits_of(i & 0x1fffffff, pos_split, P, a.s_cap);
-    const int k = c == 0 ? off[0]++ : c == 1 ? off[1]++ : off[2]++;
-    perm[k] = q;
-    if (c == 0) { pre[k] = off[3]; off[3] += ns; }
-    else if (c == 1) { pre[k] = off[4]; off[4] += ns; }
-    else { pre[k] = off[5]; off[5] += ns; }
+    const int ns = splits_of(pre[q], pos_split, P, a.s_cap);
+    pre[q] = off;
+    off += ns;
   }
-  if (threadIdx.x == 0) pre[n] = tot[3] + tot[4] + tot[5];
+  if (threadIdx.x == blockDim.x - 1) pre[n] = off;
   __syncthreads();
-  if (blockIdx.x == 0) {  // each query's first partial and splits, for the combine kernel
-    for (int k = threadIdx.x; k < n; k += blockDim.x) a.qtab[perm[k]] = make_int2(pre[k], pre[k + 1] - pre[k]);
-  }
 }
 
 // Everything the producer and consumers of one CTA share.
@@ -638,7 +613,7 @@ struct CtaRing {
 // plans each and pushes its stages; ends with an end record.
 template <int D>
 __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, int NQB, const int* pre,
-                                             const int* perm, const CtaRing& cr, int lane) {
+                                             const CtaRing& cr, int lane) {
   const LayerArgs& a = ka.a;
   const int n = ka.n, g = a.Hq / a.Hkv, R = cr.R;
   const int total = pre[n] * NQB;
@@ -693,13 +668,13 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
     int u_next = 0;
     if (lane == 0) u_next = static_cast<int>(gridDim.x) + atomicAdd(&a.ctrl[kNextUnit], 1);  // used last
     const int un = u / NQB, qb = u - un * NQB;
-    int lo_k = 0, hi_k = n;  // the query of split un: pre[k] <= un < pre[k + 1]
-    while (hi_k - lo_k > 1) {
-      const int mid = (lo_k + hi_k) >> 1;
-      if (pre[mid] <= un) lo_k = mid;
-      else hi_k = mid;
+    int lo_q = 0, hi_q = n;  // the query of split un: pre[q] <= un < pre[q + 1]
+    while (hi_q - lo_q > 1) {
+      const int mid = (lo_q + hi_q) >> 1;
+      if (pre[mid] <= un) lo_q = mid;
+      else hi_q = mid;
     }
-    const int q = perm[lo_k], sp = un - pre[lo_k], ns = pre[lo_k + 1] - pre[lo_k];
+    const int q = lo_q, sp = un - pre[q], ns = pre[q + 1] - pre[q];
     const int seq = ka.seq_ids[q], t = ka.q_positions[q], mode = ka.modes[q];
     const int w = ka.windows ? ka.windows[q] : ka.window_scalar;
     const int err = query_error(a, seq, t, mode, w);
@@ -713,7 +688,7 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
       int wid, wmeta;
       const int T = plan_split(a, P, seq, lo, t, sp, ns, lane, wid, wmeta);
       const int kv0 = h0 / g, nkv = (h0 + nh - 1) / g - kv0 + 1;
-      const int4 rb = make_int4(t, sp, ns, pre[lo_k]);
+      const int4 rb = make_int4(t, sp, ns, pre[q]);
       {  // the unit's query rows
         const int need = nh * D * 2;
         int taken = 0;
@@ -781,27 +756,99 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
   }
 }
 
+// Merges `count` partial rows at p0, p0 + stride, ...: the common maximum Mx, the
+// weighted sum of L and the weighted rows (lane holds dims lane * DPL ..).
+template <int D>
+__device__ __forceinline__ void merge_partials(const float* p0, int64_t stride, int count, int lane, float& Mx,
+                                               float& Ls, float (&acc_o)[D / 32]) {
+  constexpr int DPL = D / 32;
+  Mx = kNegInf;
+  for (int s = lane; s < count; s += 32) Mx = fmaxf(Mx, __ldcg(p0 + s * stride + D));
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) Mx = fmaxf(Mx, __shfl_xor_sync(0xffffffffu, Mx, o));
+  Ls = 0.f;
+#pragma unroll
+  for (int j = 0; j < DPL; ++j) acc_o[j] = 0.f;
+  for (int s0 = 0; s0 < count; s0 += 32) {
+    float wl = 0.f;  // lane s: weight of row s0 + s
+    if (s0 + lane < count) {
+      const float2 ml = __ldcg(reinterpret_cast<const float2*>(p0 + (s0 + lane) * stride + D));
+      wl = (ml.x == kNegInf) ? 0.f : fast_exp2(ml.x - Mx);
+      Ls = fmaf(wl, ml.y, Ls);
+    }
+    const int cnt = min(32, count - s0);
+#pragma unroll 8
+    for (int s = 0; s < cnt; ++s) {
+      const float wgt = __shfl_sync(0xffffffffu, wl, s);
+      const float* ps = p0 + (s0 + s) * stride + lane * DPL;
+#pragma unroll
+      for (int j = 0; j < DPL; ++j) acc_o[j] = fmaf(wgt, __ldcg(ps + j), acc_o[j]);
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) Ls += __shfl_xor_sync(0xffffffffu, Ls, o);
+}
+
+// Counts this warp's arrival on *counter (release of its partial stores, acquire of
+// the others'); true for the last of `expected` arrivals, which resets the counter.
+__device__ __forceinline__ bool arrive_last(int* counter, int expected, int lane) {
+  __syncwarp();
+  int arrivals = 0;
+  if (lane == 0) arrivals = atom_add_acq_rel(counter, 1);
+  __syncwarp();
+  arrivals = __shfl_sync(0xffffffffu, arrivals, 0);
+  if (arrivals != expected - 1) return false;
+  if (lane == 0) *counter = 0;  // ready for the next call
+  return true;
+}
+
 // A (query, head) row at its end: lane holds DPL consecutive dims from dim0 of the
 // unnormalised sum acc = sum_j p_j v_j (weights relative to max M, log2 domain) and the
-// row's weight sum L.  One split: the bf16 row.  Otherwise the split's fp32 partial
-// (acc, M, L), which the combine kernel merges with the query's other splits.
+// row's weight sum L.  One split: the bf16 row.  Otherwise the split's fp32 partial,
+// merged in two levels: the last split of each group of kMergeGroup to arrive folds the
+// group into the group's first partial, and the last group to arrive merges the groups
+// into the row (one level when nsplit <= kMergeGroup).
 template <int D>
-__device__ __forceinline__ void store_row(const AttnKernelArgs& ka, const float* v, int dim0, float M, float L, int sp,
-                                          int qi, int qh, int nsplit, int base, int lane) {
+__device__ __forceinline__ void store_or_merge(const AttnKernelArgs& ka, const float* v, int dim0, float M, float L,
+                                               int sp, int qi, int qh, int nsplit, int base, int lane) {
   constexpr int DPL = D / 32;
   const LayerArgs& a = ka.a;
+  const int64_t orow = (static_cast<int64_t>(qi) * a.Hq + qh) * D;
   if (nsplit == 1) {
-    const int64_t orow = (static_cast<int64_t>(qi) * a.Hq + qh) * D;
     const float inv = L > 0.f ? 1.f / L : 0.f;
 #pragma unroll
     for (int j = 0; j < DPL; j += 2)
       *reinterpret_cast<__nv_bfloat162*>(ka.out + orow + dim0 + j) = __floats2bfloat162_rn(v[j] * inv, v[j + 1] * inv);
     return;
   }
-  float* pp = a.part + ((static_cast<int64_t>(base) + sp) * a.Hq + qh) * (D + 4);
+  const int64_t sstride = static_cast<int64_t>(a.Hq) * (D + 4);
+  float* p0 = a.part + (static_cast<int64_t>(base) * a.Hq + qh) * (D + 4);  // split 0's partial
+  float* pp = p0 + sp * sstride;
 #pragma unroll
-  for (int j = 0; j < DPL; j += 2) __stcg(reinterpret_cast<float2*>(pp + dim0 + j), make_float2(v[j], v[j + 1]));
-  if (lane == 0) __stcg(reinterpret_cast<float2*>(pp + D), make_float2(M, L));
+  for (int j = 0; j < DPL; j += 2) *reinterpret_cast<float2*>(pp + dim0 + j) = make_float2(v[j], v[j + 1]);
+  if (lane == 0) *reinterpret_cast<float2*>(pp + D) = make_float2(M, L);
+  int* counters = a.cnt + (static_cast<int64_t>(qi) * a.Hq + qh) * a.cnt_stride;
+  float Mx, Ls, acc_o[DPL];
+  int ngroups = nsplit, gstride = 1;
+  if (nsplit > kMergeGroup) {
+    const int gr = sp / kMergeGroup, g0 = gr * kMergeGroup, gn = min(kMergeGroup, nsplit - g0);
+    if (!arrive_last(counters + 1 + gr, gn, lane)) return;
+    float* pg = p0 + g0 * sstride;
+    merge_partials<D>(pg, sstride, gn, lane, Mx, Ls, acc_o);
+    __syncwarp();  // every lane has read the group's rows before the first is overwritten
+#pragma unroll
+    for (int j = 0; j < DPL; ++j) __stcg(pg + lane * DPL + j, acc_o[j]);
+    if (lane == 0) __stcg(reinterpret_cast<float2*>(pg + D), make_float2(Mx, Ls));
+    ngroups = (nsplit + kMergeGroup - 1) / kMergeGroup;
+    gstride = kMergeGroup;
+  }
+  if (!arrive_last(counters, ngroups, lane)) return;
+  merge_partials<D>(p0, sstride * gstride, ngroups, lane, Mx, Ls, acc_o);
+  const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
+#pragma unroll
+  for (int j = 0; j < DPL; j += 2)
+    *reinterpret_cast<__nv_bfloat162*>(ka.out + orow + lane * DPL + j) =
+        __floats2bfloat162_rn(acc_o[j] * inv, acc_o[j + 1] * inv);
 }
 
 // ------------------------------------------------- CUDA-core consumer (MHA) --
@@ -809,10 +856,10 @@ __device__ __forceinline__ void store_row(const AttnKernelArgs& ka, const float*
 // head (four lanes for 128) dequantises in registers and keeps its own online softmax.
 
 // The end of a unit for a CUDA-core consumer: merge the lanes' states, then store.
-template <int D>
-__device__ __forceinline__ void finish_unit(const AttnKernelArgs& ka, LaneState& st, int cur_cls, int sp, int qi,
+template <int D, int E>
+__device__ __forceinline__ void finish_unit(const AttnKernelArgs& ka, LaneState<E>& st, int cur_cls, int sp, int qi,
                                             int qh, int nsplit, int base, int lane) {
-  constexpr int LPK = D / 32;  // lanes per key
+  constexpr int LPK = D / E;   // lanes per key
   constexpr int DPL = D / 32;  // dimensions per lane after the merge
   const int part = lane % LPK, kl = lane / LPK;
   // rescale to the common maximum, then reduce-scatter over the key lanes: each
@@ -828,17 +875,17 @@ __device__ __forceinline__ void finish_unit(const AttnKernelArgs& ka, LaneState&
   {
     const float2 s49 = make_float2(pow2f(49) * f, pow2f(49) * f), zf = make_float2(st.zacc * f, st.zacc * f);
 #pragma unroll
-    for (int j = 0; j < 32; j += 2) {
+    for (int j = 0; j < E; j += 2) {
       const float2 r = __ffma2_rn(make_float2(st.acc[j], st.acc[j + 1]), s49, zf);
       st.acc[j] = r.x;
       st.acc[j + 1] = r.y;
     }
   }
 #pragma unroll
-  for (int width = 16, o = 16; o >= LPK; width >>= 1, o >>= 1) {
+  for (int width = E / 2, o = 16; o >= LPK; width >>= 1, o >>= 1) {
     const bool upper = lane & o;
 #pragma unroll
-    for (int i = 0; i < 16; ++i) {
+    for (int i = 0; i < E / 2; ++i) {
       if (i < width) {
         const float keep = upper ? st.acc[width + i] : st.acc[i];
         const float give = upper ? st.acc[i] : st.acc[width + i];
@@ -846,26 +893,26 @@ __device__ __forceinline__ void finish_unit(const AttnKernelArgs& ka, LaneState&
       }
     }
   }
-  // lane (kl, part) now holds dims part*32 + DPL*kl .. + DPL-1 in acc[0 .. DPL-1]
-  store_row<D>(ka, st.acc, part * 32 + DPL * kl, M, L, sp, qi, qh, nsplit, base, lane);
+  // lane (kl, part) now holds dims part*E + DPL*kl .. + DPL-1 in acc[0 .. DPL-1]
+  store_or_merge<D>(ka, st.acc, part * E + DPL * kl, M, L, sp, qi, qh, nsplit, base, lane);
 }
 
-template <int D, int P>
+template <int D, int P, int E>
 __device__ __forceinline__ void run_consumer_cc(const AttnKernelArgs& ka, const CtaRing& cr, int cw, int lane) {
-  constexpr int LPK = D / 32;    // lanes per key
+  constexpr int LPK = D / E;     // lanes per key
   constexpr int KPI = 32 / LPK;  // keys per warp iteration
   const LayerArgs& a = ka.a;
   const int g = a.Hq / a.Hkv;
   const int part = lane % LPK;
-  LaneState st;
-  float qp[32];
+  LaneState<E> st;
+  float qp[E];
   float sumq = 0.f;
   int cur_cls = 3;
   st.m = kNegInf;
   st.l = 0.f;
   st.zacc = 0.f;
 #pragma unroll
-  for (int j = 0; j < 32; ++j) st.acc[j] = 0.f;
+  for (int j = 0; j < E; ++j) st.acc[j] = 0.f;
   // the current unit
   int u_q = 0, u_h = 0, u_kvi = 0, u_lo = 0, u_hi = 0, u_sp = 0, u_ns = 1, u_base = 0;
   bool active = false;
@@ -899,13 +946,13 @@ __device__ __forceinline__ void run_consumer_cc(const AttnKernelArgs& ka, const 
       st.l = 0.f;
       st.zacc = 0.f;
 #pragma unroll
-      for (int j = 0; j < 32; ++j) st.acc[j] = 0.f;
+      for (int j = 0; j < E; ++j) st.acc[j] = 0.f;
       if (active && !(meta & kNoPage)) {
-        const uint32_t qa = smem_u32(cr.ring + ra.y + cw * D * 2 + part * 64);
+        const uint32_t qa = smem_u32(cr.ring + ra.y + cw * D * 2 + part * E * 2);
         const float2 qs2 = make_float2(ka.qscale, ka.qscale);
         float2 sq2 = make_float2(0.f, 0.f);
 #pragma unroll
-        for (int qq = 0; qq < 4; ++qq) {
+        for (int qq = 0; qq < E / 8; ++qq) {
           const uint4 uq = lds128(qa + 16 * qq);
           const uint32_t wv[4] = {uq.x, uq.y, uq.z, uq.w};
 #pragma unroll
@@ -930,17 +977,17 @@ __device__ __forceinline__ void run_consumer_cc(const AttnKernelArgs& ka, const 
         const bool masked = meta & kMask;
         const uint32_t sp = masked ? smem_u32(cr.ring + rc.z) : s0;
         switch (cls) {
-          case 0: consume_page<D, 2, P / KPI>(s0, sp, masked, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
-          case 1: consume_page<D, 4, P / KPI>(s0, sp, masked, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
-          case 2: consume_page<D, 8, P / KPI>(s0, sp, masked, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
-          default: consume_page<D, 16, P / KPI>(s0, sp, masked, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
+          case 0: consume_page<D, 2, P / KPI, E>(s0, sp, masked, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
+          case 1: consume_page<D, 4, P / KPI, E>(s0, sp, masked, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
+          case 2: consume_page<D, 8, P / KPI, E>(s0, sp, masked, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
+          default: consume_page<D, 16, P / KPI, E>(s0, sp, masked, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
         }
       }
     }
     __syncwarp();
     if (lane == 0) mbar_arrive(&cr.empty[slot]);  // the stage's bytes are read
     if ((meta & kLast) && active)
-      finish_unit<D>(ka, st, cur_cls, u_sp, u_q, u_h, u_ns, u_base, lane);
+      finish_unit<D, E>(ka, st, cur_cls, u_sp, u_q, u_h, u_ns, u_base, lane);
   }
 }
 
@@ -1328,7 +1375,7 @@ __device__ __forceinline__ void mma_finish(const AttnKernelArgs& ka, MmaState<D,
 #pragma unroll
     for (int j = 0; j < DPL; ++j) v[j] = row[lane * DPL + j];
     const int qh = kv * g + r;
-    store_row<D>(ka, v, lane * DPL, row[D], row[D + 1], sp, qi, qh, ns, base, lane);
+    store_or_merge<D>(ka, v, lane * DPL, row[D], row[D + 1], sp, qi, qh, ns, base, lane);
   }
   __syncwarp();
 }
@@ -1445,8 +1492,7 @@ __device__ __forceinline__ void run_consumer_mma(const AttnKernelArgs& ka, const
 
 // The prologue every attention kernel shares: barriers, the dependency on the previous
 // kernel, the call's work units.
-__device__ __forceinline__ CtaRing attn_prologue(const AttnKernelArgs& ka, uint8_t* smem, int P, int NQB, int*& pre,
-                                                 int*& perm) {
+__device__ __forceinline__ CtaRing attn_prologue(const AttnKernelArgs& ka, uint8_t* smem, int P, int NQB, int*& pre) {
   const AttnSmem lay(ka.ring_bytes, ka.n, ka.scr_floats);
   CtaRing cr;
   cr.ring = smem + lay.ring;
@@ -1457,7 +1503,6 @@ __device__ __forceinline__ CtaRing attn_prologue(const AttnKernelArgs& ka, uint8
   cr.abort_flag = reinterpret_cast<volatile int*>(smem + lay.flag);
   cr.R = ka.ring_bytes;
   pre = reinterpret_cast<int*>(smem + lay.pre);
-  perm = reinterpret_cast<int*>(smem + lay.perm);
   if (threadIdx.x == 0) {
 #pragma unroll 1
     for (int i = 0; i < kStages; ++i) {
@@ -1469,7 +1514,7 @@ __device__ __forceinline__ CtaRing attn_prologue(const AttnKernelArgs& ka, uint8
   }
   pdl_wait();
   pdl_trigger();
-  plan_units(ka, P, NQB, pre, perm, reinterpret_cast<int*>(smem + lay.info), reinterpret_cast<int*>(smem + lay.red));
+  plan_units(ka, P, NQB, pre, reinterpret_cast<long long*>(smem + lay.red));
   return cr;
 }
 
@@ -1491,14 +1536,15 @@ __device__ __forceinline__ void attn_epilogue(const LayerArgs& a) {
 
 // CUDA-core path: units of kNcw query heads, one per consumer warp.
 template <int D, int P>
-__global__ void __launch_bounds__(32 * (kNcw + 1), kCtasPerSm) attn_kernel(const __grid_constant__ AttnKernelArgs ka) {
+__global__ void __launch_bounds__(32 * (kNcw + 1), cc_ctas_per_sm(D))
+    attn_kernel(const __grid_constant__ AttnKernelArgs ka) {
   extern __shared__ __align__(128) uint8_t smem[];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int NQB = (ka.a.Hq + ka.hpu - 1) / ka.hpu;
-  int *pre, *perm;
-  const CtaRing cr = attn_prologue(ka, smem, P, NQB, pre, perm);
-  if (warp == 0) run_producer<D>(ka, P, NQB, pre, perm, cr, lane);
-  else run_consumer_cc<D, P>(ka, cr, warp - 1, lane);
+  int* pre;
+  const CtaRing cr = attn_prologue(ka, smem, P, NQB, pre);
+  if (warp == 0) run_producer<D>(ka, P, NQB, pre, cr, lane);
+  else run_consumer_cc<D, P, cc_elems(D)>(ka, cr, warp - 1, lane);
   attn_epilogue(ka.a);
 }
 
@@ -1509,10 +1555,10 @@ __global__ void __launch_bounds__(32 * (kNcw + 1), kCtasPerSm) attn_mma_kernel(c
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int NQB = (ka.a.Hq + ka.hpu - 1) / ka.hpu;
   const int P = ka.a.P;
-  int *pre, *perm;
-  const CtaRing cr = attn_prologue(ka, smem, P, NQB, pre, perm);
+  int* pre;
+  const CtaRing cr = attn_prologue(ka, smem, P, NQB, pre);
   if (warp == 0) {
-    run_producer<D>(ka, P, NQB, pre, perm, cr, lane);
+    run_producer<D>(ka, P, NQB, pre, cr, lane);
   } else {
     const AttnSmem lay(ka.ring_bytes, ka.n, ka.scr_floats);
     float* scr = reinterpret_cast<float*>(smem + lay.scr) + (warp - 1) * ka.scr_floats;
@@ -1521,102 +1567,27 @@ __global__ void __launch_bounds__(32 * (kNcw + 1), kCtasPerSm) attn_mma_kernel(c
   attn_epilogue(ka.a);
 }
 
-// ------------------------------------------------------------------ combine --
-// Merges the split partials of every (query, head) of a launch whose query has more
-// than one split: one CTA of kCombineWarps warps per (query, head); warp w folds splits
-// w, w + kCombineWarps, ... over its own maximum, then warp 0 folds the warps and
-// writes the bf16 row.  Chained after the attention kernel (programmatic dependent
-// launch): it reads nothing before that kernel has finished.
-constexpr int kCombineWarps = 4;
-
-struct CombineArgs {
-  const float* part;  // [units][Hq][D + 4] partials of the launch
-  const int2* qtab;   // [n] first partial and splits of each query
-  uint16_t* out;      // [n][Hq][D] bf16 rows of the launch
-  int Hq;
-};
-
-template <int D>
-__global__ void __launch_bounds__(32 * kCombineWarps) attn_combine_kernel(const __grid_constant__ CombineArgs ca) {
-  constexpr int DPL = D / 32;
-  __shared__ float sacc[kCombineWarps][D];
-  __shared__ float sml[kCombineWarps][2];
-  pdl_wait();
-  pdl_trigger();
-  const int qi = blockIdx.x / ca.Hq, qh = blockIdx.x - qi * ca.Hq;
-  const int2 e = ca.qtab[qi];
-  if (e.y <= 1) return;  // written by the attention kernel
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int64_t stride = static_cast<int64_t>(ca.Hq) * (D + 4);
-  const float* p0 = ca.part + (static_cast<int64_t>(e.x) * ca.Hq + qh) * (D + 4) + warp * stride;
-  const int64_t wstride = stride * kCombineWarps;  // between this warp's splits
-  const int cnt = (e.y - warp + kCombineWarps - 1) / kCombineWarps;
-  float Mx = kNegInf;
-  for (int s = lane; s < cnt; s += 32) Mx = fmaxf(Mx, __ldcg(p0 + s * wstride + D));
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) Mx = fmaxf(Mx, __shfl_xor_sync(0xffffffffu, Mx, o));
-  float Ls = 0.f, acc[DPL];
-#pragma unroll
-  for (int j = 0; j < DPL; ++j) acc[j] = 0.f;
-  for (int s0 = 0; s0 < cnt; s0 += 32) {
-    float wl = 0.f;  // lane s: weight of split s0 + s of this warp
-    if (s0 + lane < cnt) {
-      const float2 ml = __ldcg(reinterpret_cast<const float2*>(p0 + (s0 + lane) * wstride + D));
-      wl = (ml.x == kNegInf) ? 0.f : fast_exp2(ml.x - Mx);
-      Ls = fmaf(wl, ml.y, Ls);
-    }
-    const int m = min(32, cnt - s0);
-#pragma unroll 8
-    for (int s = 0; s < m; ++s) {
-      const float wgt = __shfl_sync(0xffffffffu, wl, s);
-      const float* ps = p0 + (s0 + s) * wstride + lane * DPL;
-#pragma unroll
-      for (int j = 0; j < DPL; ++j) acc[j] = fmaf(wgt, __ldcg(ps + j), acc[j]);
-    }
-  }
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) Ls += __shfl_xor_sync(0xffffffffu, Ls, o);
-#pragma unroll
-  for (int j = 0; j < DPL; ++j) sacc[warp][lane * DPL + j] = acc[j];
-  if (lane == 0) {
-    sml[warp][0] = Mx;
-    sml[warp][1] = Ls;
-  }
-  __syncthreads();
-  if (warp != 0) return;
-  float M = kNegInf;
-#pragma unroll
-  for (int w = 0; w < kCombineWarps; ++w) M = fmaxf(M, sml[w][0]);
-  float L = 0.f, o[DPL];
-#pragma unroll
-  for (int j = 0; j < DPL; ++j) o[j] = 0.f;
-#pragma unroll
-  for (int w = 0; w < kCombineWarps; ++w) {
-    const float f = sml[w][0] == kNegInf ? 0.f : fast_exp2(sml[w][0] - M);
-    L = fmaf(f, sml[w][1], L);
-#pragma unroll
-    for (int j = 0; j < DPL; ++j) o[j] = fmaf(f, sacc[w][lane * DPL + j], o[j]);
-  }
-  const float inv = L > 0.f ? 1.f / L : 0.f;
-  uint16_t* orow = ca.out + (static_cast<int64_t>(qi) * ca.Hq + qh) * D + lane * DPL;
-#pragma unroll
-  for (int j = 0; j < DPL; j += 2)
-    *reinterpret_cast<__nv_bfloat162*>(orow + j) = __floats2bfloat162_rn(o[j] * inv, o[j + 1] * inv);
-}
-
-constexpr int kAttnSmemLimit = 72 * 1024;  // dynamic shared memory of one attention CTA
-
 // Done once per cache at creation, so that calls stay legal inside stream capture.
 cudaError_t attn_configure() {
-  const void* kernels[] = {
-      reinterpret_cast<const void*>(attn_kernel<64, 16>),     reinterpret_cast<const void*>(attn_kernel<64, 32>),
-      reinterpret_cast<const void*>(attn_kernel<64, 64>),     reinterpret_cast<const void*>(attn_kernel<128, 16>),
-      reinterpret_cast<const void*>(attn_kernel<128, 32>),    reinterpret_cast<const void*>(attn_kernel<128, 64>),
-      reinterpret_cast<const void*>(attn_mma_kernel<64, 1>),  reinterpret_cast<const void*>(attn_mma_kernel<64, 2>),
-      reinterpret_cast<const void*>(attn_mma_kernel<128, 1>), reinterpret_cast<const void*>(attn_mma_kernel<128, 2>),
-      reinterpret_cast<const void*>(attn_mma_kernel<128, 4>)};
-  for (const void* k : kernels) {
-    const cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, kAttnSmemLimit);
+  struct K {
+    const void* f;
+    int ctas;
+  };
+  const K kernels[] = {
+      {reinterpret_cast<const void*>(attn_kernel<64, 16>), cc_ctas_per_sm(64)},
+      {reinterpret_cast<const void*>(attn_kernel<64, 32>), cc_ctas_per_sm(64)},
+      {reinterpret_cast<const void*>(attn_kernel<64, 64>), cc_ctas_per_sm(64)},
+      {reinterpret_cast<const void*>(attn_kernel<128, 16>), cc_ctas_per_sm(128)},
+      {reinterpret_cast<const void*>(attn_kernel<128, 32>), cc_ctas_per_sm(128)},
+      {reinterpret_cast<const void*>(attn_kernel<128, 64>), cc_ctas_per_sm(128)},
+      {reinterpret_cast<const void*>(attn_mma_kernel<64, 1>), kCtasPerSm},
+      {reinterpret_cast<const void*>(attn_mma_kernel<64, 2>), kCtasPerSm},
+      {reinterpret_cast<const void*>(attn_mma_kernel<128, 1>), kCtasPerSm},
+      {reinterpret_cast<const void*>(attn_mma_kernel<128, 2>), kCtasPerSm},
+      {reinterpret_cast<const void*>(attn_mma_kernel<128, 4>), kCtasPerSm}};
+  for (const K& k : kernels) {
+    const cudaError_t e =
+        cudaFuncSetAttribute(k.f, cudaFuncAttributeMaxDynamicSharedMemorySize, attn_smem_limit(k.ctas));
     if (e != cudaSuccess) return e;
   }
   return cudaSuccess;
@@ -1631,9 +1602,9 @@ static bool use_mma(const Layout& l) {
 
 // Ring bytes an attention call with n queries gets, or -1 when one stage of the
 // widest page (one KV slice, its positions) or of the query rows would not fit.
-static int attn_ring_bytes(const Layout& l, int n, int hpu, int scr_floats) {
+static int attn_ring_bytes(const Layout& l, int n, int hpu, int scr_floats, int limit) {
   const int fixed = AttnSmem(0, n, scr_floats).total;
-  const int ring = (kAttnSmemLimit - fixed) / 128 * 128;
+  const int ring = (limit - fixed) / 128 * 128;
   const int widest = static_cast<int>(l.slice[3]) + 4 * l.P;
   const int qrows = hpu * 2 * l.d;
   if (ring < std::max(widest, qrows)) return -1;
@@ -1646,12 +1617,13 @@ constexpr int kMaxLaunchQueries = 1024;
 
 static cudaError_t launch_one(const Layout& l, const AttnKernelArgs& ka, int num_sms, cudaStream_t s) {
   const bool mma = use_mma(l);
-  const int ring = attn_ring_bytes(l, ka.n, ka.hpu, ka.scr_floats);
+  const int ctas = mma ? kCtasPerSm : cc_ctas_per_sm(l.d);
+  const int ring = attn_ring_bytes(l, ka.n, ka.hpu, ka.scr_floats, attn_smem_limit(ctas));
   if (ring < 0) return cudaErrorInvalidConfiguration;
   AttnKernelArgs k = ka;
   k.ring_bytes = ring;
   const size_t sm = static_cast<size_t>(AttnSmem(ring, k.n, k.scr_floats).total);
-  const dim3 grid(kCtasPerSm * num_sms), block(32 * (kNcw + 1));
+  const dim3 grid(ctas * num_sms), block(32 * (kNcw + 1));
   if (mma) {
     const int ng = l.d / l.G;
     if (l.d == 64) {
@@ -1700,19 +1672,10 @@ static cudaError_t launch_attention(const Layout& l, const LayerArgs& a, int num
     ka.windows = windows ? windows + q0 : nullptr;
     ka.q = static_cast<const uint16_t*>(q_bf16) + q0 * row;
     ka.out = static_cast<uint16_t*>(out_bf16) + q0 * row;
-    ka.a.qtab = a.qtab + q0;
-    cudaError_t e = launch_one(l, ka, num_sms, s);
+    ka.a.cnt = a.cnt + static_cast<int64_t>(q0) * l.Hq * l.cnt_stride;
+    const cudaError_t e = launch_one(l, ka, num_sms, s);
     if (e != cudaSuccess) return e;
-    CombineArgs ca;
-    ca.part = a.part;
-    ca.qtab = ka.a.qtab;
-    ca.out = ka.out;
-    ca.Hq = l.Hq;
-    const dim3 cgrid(ka.n * l.Hq), cblock(32 * kCombineWarps);
-    e = l.d == 64 ? launch_pdl(attn_combine_kernel<64>, cgrid, cblock, 0, s, ca)
-                  : launch_pdl(attn_combine_kernel<128>, cgrid, cblock, 0, s, ca);
-    if (e != cudaSuccess) return e;
-    *launches += 2;
+    ++*launches;
   }
   return cudaSuccess;
 }
@@ -1744,8 +1707,8 @@ extern "C" trr_status trr_decode_attn(trr_cache* cache, int32_t layer, int32_t n
 
 // ------------------------------------------------------ static-scratch variant --
 //
-// trr_decode_attn_static runs the same kernels as trr_decode_attn, but keeps all of its
-// per-call scratch (the query table, fp32 partials and the call's control words) in one
+// trr_decode_attn_static runs the same kernel as trr_decode_attn, but keeps all of its
+// per-call scratch (arrival counters, fp32 partials and the call's control words) in one
 // file-scope device array instead of the cache's scratch region.  Nothing is allocated
 // per call or at set-up.
 namespace trr {
@@ -1772,10 +1735,11 @@ static cudaError_t static_scratch(void** out) {
   return cudaSuccess;
 }
 
-// Clears what a call needs at zero: the control words.
-__global__ void static_scratch_clear_kernel(int32_t* wctrl) {
-  const int i = threadIdx.x;
+// Clears what a call needs at zero: the control words and the arrival counters.
+__global__ void static_scratch_clear_kernel(int32_t* wctrl, int32_t* cnt, int ncnt) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i < kCtrlInts) wctrl[i] = i == kFirstBadQuery ? INT_MAX : 0;
+  for (int j = i; j < ncnt; j += gridDim.x * blockDim.x) cnt[j] = 0;
 }
 
 // Forwards the call's first error to the cache's sticky status word.
@@ -1801,19 +1765,20 @@ extern "C" trr_status trr_decode_attn_static(trr_cache* cache, int32_t layer, in
   // scratch of this call, carved from the static array; reject what does not fit
   auto up = [](int64_t x) { return (x + 255) / 256 * 256; };
   const int64_t b_ctrl = up(4 * kCtrlInts);
-  const int64_t b_qtab = up(8ll * n);
+  const int64_t b_cnt = up(4ll * n * l.units * l.cnt_stride);
   const int64_t b_part = up(4ll * n * l.s_cap * l.units * (l.d + 4));
-  if (b_ctrl + b_qtab + b_part > kStaticScratchBytes) return TRR_ERR_OUT_OF_MEMORY;
+  if (b_ctrl + b_cnt + b_part > kStaticScratchBytes) return TRR_ERR_OUT_OF_MEMORY;
   void* base = nullptr;
   if (static_scratch(&base) != cudaSuccess) return TRR_ERR_CUDA;
   uint8_t* b = static_cast<uint8_t*>(base);
   LayerArgs a = layer_args(l, cache_views(cache), layer);
   int32_t* cache_ctrl = a.ctrl;
   a.ctrl = reinterpret_cast<int32_t*>(b);
-  a.qtab = reinterpret_cast<int2*>(b + b_ctrl);
-  a.part = reinterpret_cast<float*>(b + b_ctrl + b_qtab);
+  a.cnt = reinterpret_cast<int32_t*>(b + b_ctrl);
+  a.part = reinterpret_cast<float*>(b + b_ctrl + b_cnt);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  static_scratch_clear_kernel<<<1, kCtrlInts, 0, s>>>(a.ctrl);
+  const int ncnt = n * l.units * l.cnt_stride;
+  static_scratch_clear_kernel<<<std::max(1, std::min(256, (ncnt + 255) / 256)), 256, 0, s>>>(a.ctrl, a.cnt, ncnt);
   cudaError_t e = cudaGetLastError();
   int launches = 0;
   if (e == cudaSuccess)

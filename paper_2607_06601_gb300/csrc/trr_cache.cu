@@ -37,7 +37,8 @@ LayerArgs layer_args(const Layout& l, const Views& v, int layer) {
   a.plast = v.plast + ls * 4 * l.MP;
   a.lastpg = v.lastpg + ls * 4;
   a.aplan = v.aplan;
-  a.qtab = v.qtab;
+  a.cnt = v.cnt;
+  a.cnt_stride = l.cnt_stride;
   a.part = v.part;
   return a;
 }
@@ -84,6 +85,7 @@ static trr_status make_layout(const trr_cache_config* c, Layout* l) {
   l->pos_split = static_cast<int>(std::max<int64_t>(l->P, l->split_bytes / l->tokb[2]));
   l->s_cap = 1 << 30;
   l->s_cap = std::max(splits_of(l->maxctx, l->pos_split, l->P, l->s_cap), 1);
+  l->cnt_stride = 1 + (l->s_cap + kMergeGroup - 1) / kMergeGroup;
   l->max_items = static_cast<int64_t>(l->max_queries) * l->units * l->s_cap;
 
   const int64_t nls = static_cast<int64_t>(l->L) * l->S;
@@ -102,7 +104,7 @@ static trr_status make_layout(const trr_cache_config* c, Layout* l) {
   l->off_plast = take(16 * nls * l->MP);
   l->off_lastpg = take(16 * nls);
   l->off_aplan = take(static_cast<int64_t>(sizeof(AppendPlan)) * l->max_append);
-  l->off_qtab = take(8 * static_cast<int64_t>(l->max_queries));
+  l->off_cnt = take(4 * static_cast<int64_t>(l->max_queries) * l->units * l->cnt_stride);
   l->off_part = take(4 * l->max_items * (l->Hq / l->units) * (l->d + 4));
   for (int k = 0; k < kClasses; ++k) l->off_pool[k] = take(l->cap[k] * l->page_bytes[k]);
   l->total = off;
@@ -148,6 +150,8 @@ static trr_status clear_metadata(trr_cache* c, cudaStream_t s) {
   ok = ok && cudaMemsetAsync(b + l.off_presence, 0, 4 * nls * l.W32, s) == cudaSuccess;
   ok = ok && cudaMemsetAsync(b + l.off_pt, 0xFF, 3 * (l.off_pfirst - l.off_pt), s) == cudaSuccess;
   ok = ok && cudaMemsetAsync(b + l.off_lastpg, 0xFF, 16 * nls, s) == cudaSuccess;
+  ok = ok && cudaMemsetAsync(b + l.off_cnt, 0, 4 * static_cast<int64_t>(l.max_queries) * l.units * l.cnt_stride, s) ==
+                  cudaSuccess;
   return ok ? TRR_OK : TRR_ERR_CUDA;
 }
 

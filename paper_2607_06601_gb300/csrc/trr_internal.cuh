@@ -31,6 +31,10 @@ enum Ctrl : int {
 // partial page per class), so that a warp holds an item's page ids one per lane.
 constexpr int kItemMaxPages = 28;
 
+// Split partials are merged in groups of this many (then the groups): a query with
+// ns splits per head has 1 + ceil(ns / kMergeGroup) arrival counters per head.
+constexpr int kMergeGroup = 8;
+
 // Byte layout of one cache (see include/trr.h for the documented part).
 struct Layout {
   int L, S, Hq, Hkv, d, G, P, maxctx, MP, W32;
@@ -39,10 +43,11 @@ struct Layout {
   int units;      // attention work units per query split (one per query head)
   int pos_split;  // key positions per split at least (split_bytes of 8-bit tokens)
   int s_cap;      // most splits one query is cut into
+  int cnt_stride; // arrival counters per (query, head): 1 + ceil(s_cap / kMergeGroup)
   int64_t max_items;
   int64_t hdr, tokb[kClasses], slice[kClasses], page_bytes[kClasses];
   int64_t off_ctrl, off_last_pos, off_ntok, off_presence, off_pt, off_pfirst, off_plast, off_lastpg;
-  int64_t off_aplan, off_qtab, off_part, off_pool[kClasses], total;
+  int64_t off_aplan, off_cnt, off_part, off_pool[kClasses], total;
 };
 
 // Splits of a query whose key range spans `range` positions: at least pos_split
@@ -74,7 +79,7 @@ struct Views {  // typed device pointers into the cache memory
   int32_t* plast;
   int32_t* lastpg;
   AppendPlan* aplan;
-  int2* qtab;
+  int32_t* cnt;
   float* part;
   uint8_t* pool[kClasses];
 };
@@ -91,7 +96,7 @@ inline Views make_views(const Layout& l, void* base) {
   v.plast = reinterpret_cast<int32_t*>(b + l.off_plast);
   v.lastpg = reinterpret_cast<int32_t*>(b + l.off_lastpg);
   v.aplan = reinterpret_cast<AppendPlan*>(b + l.off_aplan);
-  v.qtab = reinterpret_cast<int2*>(b + l.off_qtab);
+  v.cnt = reinterpret_cast<int32_t*>(b + l.off_cnt);
   v.part = reinterpret_cast<float*>(b + l.off_part);
   for (int c = 0; c < kClasses; ++c) v.pool[c] = b + l.off_pool[c];
   return v;
@@ -99,7 +104,7 @@ inline Views make_views(const Layout& l, void* base) {
 
 // Everything a kernel needs about one layer of one cache, passed by value.
 struct LayerArgs {
-  int layer, S, Hq, Hkv, d, G, P, maxctx, MP, W32, units, pos_split, s_cap, split_bytes, skip_writes_kv;
+  int layer, S, Hq, Hkv, d, G, P, maxctx, MP, W32, units, pos_split, s_cap, cnt_stride, split_bytes, skip_writes_kv;
   int cap[kClasses];
   int hdr;
   int slice[kClasses];
@@ -113,7 +118,7 @@ struct LayerArgs {
   int32_t* plast;
   int32_t* lastpg;     // this layer: [S][4] id of the page holding token ntok-1 (internal)
   AppendPlan* aplan;
-  int2* qtab;          // [max_queries] (first partial, splits) of each query of the call
+  int32_t* cnt;        // [max_queries][Hq][cnt_stride] split arrivals (zero between calls)
   float* part;         // [max_queries * s_cap * Hq][d + 4] fp32 partials: acc, M, L
   uint8_t* pool[kClasses];
 };
