@@ -124,7 +124,9 @@ TRR_API trr_status trr_create_cache(const trr_cache_config* cfg, trr_cache** out
  *     c_j = clamp(rne((x_j - z) / s), 0, 2^b - 1)   (c_j = 0 when s == 0)
  *   with fl32 = IEEE binary32 round-to-nearest-even and rne taken on the EXACT quotient
  *   (c_j is the nearest level z + c*s, ties to the even c); b = 16 stores the bf16 bits.
- *   seq_ids, positions, k, v, bits, modes: device arrays; 0 <= n <= max_append.
+ *   seq_ids, positions, k, v, bits, modes: device arrays; 0 <= n <= max_append.  They may
+ *   be read while the previous kernel of the stream (a trr_* call) is still running:
+ *   they must not be outputs of that call.
  *   Device-detected errors: seq id out of range or bits/mode not allowed
  *   (INVALID_ARG), a position outside [0, max_context) or not above the sequence's
  *   last one (BAD_POSITION), a pool running out (OUT_OF_PAGES).  Any of these makes
@@ -150,7 +152,9 @@ TRR_API trr_status trr_kv_append(trr_cache* cache, int32_t layer, int32_t n,
  *   Device-detected errors (seq id, mode or window invalid: INVALID_ARG; position
  *   outside [0, max_context): BAD_POSITION) zero that query's row and record the
  *   error of the lowest failing index; other queries are computed.
- *   seq_ids, q_positions, q, modes, windows, out: device; 0 <= n <= max_queries. */
+ *   seq_ids, q_positions, q, modes, windows, out: device; 0 <= n <= max_queries.
+ *   seq_ids, q_positions, modes and windows may be read while the previous kernel of the
+ *   stream (a trr_* call) is still running: they must not be outputs of that call. */
 TRR_API trr_status trr_decode_attn(trr_cache* cache, int32_t layer, int32_t n,
                            const int32_t* seq_ids, const int32_t* q_positions,
                            const void* q_bf16, const uint8_t* modes,

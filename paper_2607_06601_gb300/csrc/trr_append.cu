@@ -319,10 +319,11 @@ __global__ void __launch_bounds__(256) append_fused_kernel(LayerArgs a, int n, c
   __shared__ int s_first_err;
   __shared__ int s_last;
 
-  pdl_wait();
-  pdl_trigger();
   const int e = threadIdx.x, lane = e & 31, warp = e >> 5;
   const bool act = e < n;
+  // The call's own inputs (entries, K/V rows) are read first: no kernel of this library
+  // writes them, so this overlaps the previous kernel of the stream.  Cache metadata and
+  // control words come after the wait.
   // this warp's row (entry, KV head, K|V), loaded while the entries are planned
   const int row = blockIdx.x * (blockDim.x >> 5) + warp;
   const bool has_row = row < n * a.Hkv * 2;
@@ -351,6 +352,8 @@ __global__ void __launch_bounds__(256) append_fused_kernel(LayerArgs a, int n, c
   s_seq[e] = (act && seq >= 0 && seq < a.S) ? seq : -1;
   s_pos[e] = pos;
   s_cls[e] = writes ? c : -1;
+  pdl_wait();
+  pdl_trigger();
   if (e < kClasses) s_next[e] = a.ctrl[kNextPage + e];
   if (e == 0) s_first_err = INT_MAX;
   __syncthreads();

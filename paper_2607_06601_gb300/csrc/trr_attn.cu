@@ -213,6 +213,9 @@ __device__ __forceinline__ uint2 lds64(uint32_t a) {
   asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(a));
   return v;
 }
+__device__ __forceinline__ void sts32(uint32_t a, uint32_t v) {
+  asm volatile("st.shared.u32 [%0], %1;" ::"r"(a), "r"(v) : "memory");
+}
 __device__ __forceinline__ uint32_t lds32(uint32_t a) {
   uint32_t v;
   asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(a));
@@ -1112,7 +1115,8 @@ template <int D, int NG>
 struct MmaState {
   static constexpr int NP = D / 8;   // K pairs per thread and key
   static constexpr int MT = D / 16;  // m-tiles of P.V
-  uint32_t qraw[NP];  // bf16 query of the thread's B column on its D/4 dims
+  uint32_t qaddr;     // shared address of word 0 of the bf16 query of the thread's B column
+                      // on its D/4 dims, kept in the warp's scratch (word i at + 128 i)
   uint32_t kb[NP];    // the q.k B operand in the current class
   float qsum[2];      // qscale * sum of the query over (head, group) of the thread's two columns
   float m[2], l[2], zacc[2];
@@ -1124,16 +1128,19 @@ struct MmaState {
 template <int D, int NG, int B>
 __device__ __forceinline__ void mma_build_kb(MmaState<D, NG>& ms) {
   constexpr int NP = D / 8;
+  uint32_t qraw[NP];
+#pragma unroll
+  for (int i = 0; i < NP; ++i) qraw[i] = lds32(ms.qaddr + 128 * i);
   if (B == 16) {
 #pragma unroll
-    for (int i = 0; i < NP; ++i) ms.kb[i] = ms.qraw[i];
+    for (int i = 0; i < NP; ++i) ms.kb[i] = qraw[i];
   } else {
 #pragma unroll
     for (int i = 0; i < NP; ++i) {
       const int lo = kp_lo<B>(i), hi = kp_hi<B>(i);
       const float f = pow2f(smax_of<B>() - kp_pos<B>(i)) * ms.escale;
-      const float ql = (lo & 1) ? bf_hi(ms.qraw[lo >> 1]) : bf_lo(ms.qraw[lo >> 1]);
-      const float qh = (hi & 1) ? bf_hi(ms.qraw[hi >> 1]) : bf_lo(ms.qraw[hi >> 1]);
+      const float ql = (lo & 1) ? bf_hi(qraw[lo >> 1]) : bf_lo(qraw[lo >> 1]);
+      const float qh = (hi & 1) ? bf_hi(qraw[hi >> 1]) : bf_lo(qraw[hi >> 1]);
       ms.kb[i] = pack_f16x2(ql * f, qh * f);
     }
   }
@@ -1179,18 +1186,25 @@ __device__ __forceinline__ void mma_page(MmaState<D, NG>& ms, uint32_t s0, uint3
   for (int c0 = 0; c0 < fill; c0 += 16) {
     // ------------------------------------------------ scores of keys c0+gid, c0+gid+8
     const int k1 = c0 + gid, k2 = k1 + 8;
-    uint32_t kw1[KW], kw2[KW];
-    lds_words<KW>(kbase + k1 * rowb + tig * (KW * 4), kw1);
-    lds_words<KW>(kbase + k2 * rowb + tig * (KW * 4), kw2);
     float ca[4] = {0.f, 0.f, 0.f, 0.f}, cb[4] = {0.f, 0.f, 0.f, 0.f};
+    // the keys' words in two halves (k-steps 0 .. KS/2-1, then the rest), so that only
+    // half a row per key is live at a time
+    constexpr int KH = KW >= 2 ? 2 : 1, KWH = KW / KH, KSH = KS / KH;
 #pragma unroll
-    for (int s = 0; s < KS; ++s) {
-      if (s & 1)
-        mma_cls<B>(cb, k_pair<B>(kw1, 2 * s), k_pair<B>(kw2, 2 * s), k_pair<B>(kw1, 2 * s + 1),
-                   k_pair<B>(kw2, 2 * s + 1), ms.kb[2 * s], ms.kb[2 * s + 1]);
-      else
-        mma_cls<B>(ca, k_pair<B>(kw1, 2 * s), k_pair<B>(kw2, 2 * s), k_pair<B>(kw1, 2 * s + 1),
-                   k_pair<B>(kw2, 2 * s + 1), ms.kb[2 * s], ms.kb[2 * s + 1]);
+    for (int hf = 0; hf < KH; ++hf) {
+      uint32_t kw1[KWH], kw2[KWH];
+      lds_words<KWH>(kbase + k1 * rowb + tig * (KW * 4) + hf * KWH * 4, kw1);
+      lds_words<KWH>(kbase + k2 * rowb + tig * (KW * 4) + hf * KWH * 4, kw2);
+#pragma unroll
+      for (int s = hf * KSH; s < (hf + 1) * KSH; ++s) {
+        const int i0 = 2 * s - hf * 2 * KSH;  // pair index inside the half
+        if (s & 1)
+          mma_cls<B>(cb, k_pair<B>(kw1, i0), k_pair<B>(kw2, i0), k_pair<B>(kw1, i0 + 1), k_pair<B>(kw2, i0 + 1),
+                     ms.kb[2 * s], ms.kb[2 * s + 1]);
+        else
+          mma_cls<B>(ca, k_pair<B>(kw1, i0), k_pair<B>(kw2, i0), k_pair<B>(kw1, i0 + 1), k_pair<B>(kw2, i0 + 1),
+                     ms.kb[2 * s], ms.kb[2 * s + 1]);
+      }
     }
     bool v1 = k1 < fill, v2 = k2 < fill;
     if (masked) {
@@ -1306,27 +1320,34 @@ __device__ __forceinline__ void mma_page(MmaState<D, NG>& ms, uint32_t s0, uint3
     // V codes of keys (2 tig, 2 tig + 1) and (2 tig + 8, 2 tig + 9) on dims gid * D/8 ..
     const int ka0 = c0 + 2 * tig;
     const uint32_t voff = vbase + (VB >= 4 ? gid * VB : (gid * VB) & ~3);
-    uint32_t wa0[VW], wb0[VW], wa1[VW], wb1[VW];
-    lds_words<VW>(voff + ka0 * rowb, wa0);
-    lds_words<VW>(voff + (ka0 + 1) * rowb, wb0);
-    lds_words<VW>(voff + (ka0 + 8) * rowb, wa1);
-    lds_words<VW>(voff + (ka0 + 9) * rowb, wb1);
-    if (VB < 4) {  // two bytes per key: this thread's half of the word
-      const int sh = ((gid * VB) & 3) * 8;
-      wa0[0] >>= sh; wb0[0] >>= sh; wa1[0] >>= sh; wb1[0] >>= sh;
-    }
     uint32_t m0 = 0xffffffffu, m1 = 0xffffffffu;  // bf16 values of keys out of range read as 0
     if (B == 16) {
       const uint32_t bal1 = __ballot_sync(0xffffffffu, v1), bal2 = __ballot_sync(0xffffffffu, v2);
       m0 = ((bal1 >> (8 * tig)) & 1 ? 0x0000ffffu : 0u) | ((bal1 >> (8 * tig + 4)) & 1 ? 0xffff0000u : 0u);
       m1 = ((bal2 >> (8 * tig)) & 1 ? 0x0000ffffu : 0u) | ((bal2 >> (8 * tig + 4)) & 1 ? 0xffff0000u : 0u);
     }
+    // the words in two halves (m-tiles 0 .. MT/2-1, then the rest)
+    constexpr int VH = VW >= 2 ? 2 : 1, VWH = VW / VH, MTH = MT / VH;
 #pragma unroll
-    for (int t = 0; t < MT; ++t) {
-      const uint32_t a0 = v_pair<B>(wa0, wb0, 2 * t) & m0, a1 = v_pair<B>(wa0, wb0, 2 * t + 1) & m0;
-      const uint32_t a2 = v_pair<B>(wa1, wb1, 2 * t) & m1, a3 = v_pair<B>(wa1, wb1, 2 * t + 1) & m1;
-      mma_cls<B>(ms.acc[t], a0, a1, a2, a3, b0, b1);
-      if (B == 16) mma_bf16(ms.acc[t], a0, a1, a2, a3, bl0, bl1);
+    for (int hf = 0; hf < VH; ++hf) {
+      uint32_t wa0[VWH], wb0[VWH], wa1[VWH], wb1[VWH];
+      const uint32_t vo = voff + hf * VWH * 4;
+      lds_words<VWH>(vo + ka0 * rowb, wa0);
+      lds_words<VWH>(vo + (ka0 + 1) * rowb, wb0);
+      lds_words<VWH>(vo + (ka0 + 8) * rowb, wa1);
+      lds_words<VWH>(vo + (ka0 + 9) * rowb, wb1);
+      if (VB < 4) {  // two bytes per key: this thread's half of the word
+        const int sh = ((gid * VB) & 3) * 8;
+        wa0[0] >>= sh; wb0[0] >>= sh; wa1[0] >>= sh; wb1[0] >>= sh;
+      }
+#pragma unroll
+      for (int t = hf * MTH; t < (hf + 1) * MTH; ++t) {
+        const int j0 = 2 * t - hf * 2 * MTH;  // dim pair inside the half
+        const uint32_t a0 = v_pair<B>(wa0, wb0, j0) & m0, a1 = v_pair<B>(wa0, wb0, j0 + 1) & m0;
+        const uint32_t a2 = v_pair<B>(wa1, wb1, j0) & m1, a3 = v_pair<B>(wa1, wb1, j0 + 1) & m1;
+        mma_cls<B>(ms.acc[t], a0, a1, a2, a3, b0, b1);
+        if (B == 16) mma_bf16(ms.acc[t], a0, a1, a2, a3, bl0, bl1);
+      }
     }
   }
 }
@@ -1400,6 +1421,7 @@ __device__ __forceinline__ void run_consumer_mma(const AttnKernelArgs& ka, const
     col_ok[j] = col_r[j] < g;
   }
   MmaState<D, NG> ms;
+  ms.qaddr = smem_u32(scr) + 4 * lane;
   int cur_cls = 3;
   int u_q = 0, u_kv = 0, u_lo = 0, u_hi = 0, u_sp = 0, u_ns = 1, u_base = 0;
   bool active = false;
@@ -1438,16 +1460,19 @@ __device__ __forceinline__ void run_consumer_mma(const AttnKernelArgs& ka, const
 #pragma unroll
       for (int t = 0; t < MT; ++t) ms.acc[t][0] = ms.acc[t][1] = ms.acc[t][2] = ms.acc[t][3] = 0.f;
       if (active && !(meta & kNoPage)) {
-        // head brow_r's query on the thread's D/4 dims, zero outside its group
+        // head brow_r's query on the thread's D/4 dims, zero outside its group, kept in
+        // the warp's scratch (it is needed again only when the width class changes)
         const uint32_t qa = smem_u32(cr.ring + ra.y + ((cw * g + min(brow_r, g - 1)) * D + tig * (D / 4)) * 2);
-        lds_words<NP>(qa, ms.qraw);
+        uint32_t qraw[NP];
+        lds_words<NP>(qa, qraw);
         float qmax = 0.f, qs = 0.f;
 #pragma unroll
         for (int i = 0; i < NP; ++i) {
-          if (!b_ok) ms.qraw[i] = 0u;
-          const float x0 = bf_lo(ms.qraw[i]), x1 = bf_hi(ms.qraw[i]);
+          if (!b_ok) qraw[i] = 0u;
+          const float x0 = bf_lo(qraw[i]), x1 = bf_hi(qraw[i]);
           qmax = fmaxf(qmax, fmaxf(fabsf(x0), fabsf(x1)));
           qs += x0 + x1;
+          sts32(ms.qaddr + 128 * i, qraw[i]);
         }
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) qmax = fmaxf(qmax, __shfl_xor_sync(0xffffffffu, qmax, o));
@@ -1460,6 +1485,7 @@ __device__ __forceinline__ void run_consumer_mma(const AttnKernelArgs& ka, const
         const int ex = static_cast<int>((__float_as_uint(qmax) >> 23) & 0xff) - 127;
         ms.E = min(100, max(0, ex - 6));
         ms.escale = __int_as_float((127 - ms.E) << 23);
+        __syncwarp();
         mma_build_kb<D, NG, 16>(ms);
       }
     } else if (active) {
@@ -1512,9 +1538,13 @@ __device__ __forceinline__ CtaRing attn_prologue(const AttnKernelArgs& ka, uint8
     *cr.abort_flag = 0;
     fence_barrier_init();
   }
+  // The unit plan reads only the call's own index arrays (sequence ids, positions,
+  // modes, windows), which no kernel of this library writes, so it overlaps the
+  // previous kernel of the stream; everything after the wait may read what that
+  // kernel wrote (cache metadata, pages, control words).
+  plan_units(ka, P, NQB, pre, reinterpret_cast<long long*>(smem + lay.red));
   pdl_wait();
   pdl_trigger();
-  plan_units(ka, P, NQB, pre, reinterpret_cast<long long*>(smem + lay.red));
   return cr;
 }
 
@@ -1661,7 +1691,9 @@ static cudaError_t launch_attention(const Layout& l, const LayerArgs& a, int num
   const bool mma = use_mma(l);
   const int g = l.Hq / l.Hkv;
   ka.hpu = mma ? kNcw * g : kNcw;
-  ka.scr_floats = mma ? g * (l.d + 4) : 0;
+  // tensor-core scratch per consumer warp: the query's bf16 words (4 d floats), later
+  // the unit's rows (g (d + 4) floats)
+  ka.scr_floats = mma ? std::max(4 * l.d, g * (l.d + 4)) : 0;
   const int64_t row = static_cast<int64_t>(l.Hq) * l.d;  // bf16 elements per query
   for (int q0 = 0; q0 < n; q0 += kMaxLaunchQueries) {
     ka.n = std::min(kMaxLaunchQueries, n - q0);
