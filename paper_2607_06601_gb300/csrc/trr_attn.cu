@@ -213,6 +213,11 @@ __device__ __forceinline__ uint2 lds64(uint32_t a) {
   asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(a));
   return v;
 }
+__device__ __forceinline__ int4 lds128i(uint32_t a) {
+  int4 v;
+  asm volatile("ld.shared.v4.s32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a));
+  return v;
+}
 __device__ __forceinline__ void sts32(uint32_t a, uint32_t v) {
   asm volatile("st.shared.u32 [%0], %1;" ::"r"(a), "r"(v) : "memory");
 }
@@ -403,7 +408,7 @@ __host__ __device__ constexpr int attn_smem_limit(int ctas) { return ctas >= 5 ?
 //   a = {meta, ring offset of the stage's bytes, query, lo}
 //   b = {hi (= t), split, splits, unit number of split 0}
 //   c = {first KV slice of the stage (block-relative), KV slices in it, ring offset of
-//        the page's slot positions or -1, 0}
+//        the page's slot positions or -1, bytes of one KV slice}
 // meta = class | fill << 2 | flags | head block << 16.
 enum : int {
   kMask = 1 << 9,     // the page may hold keys outside [lo, hi]: positions follow the slices
@@ -464,7 +469,7 @@ struct AttnSmem {
 
 // Bounded wait that also gives up once *abort is set (by a warp that gave up).
 __device__ __forceinline__ bool mbar_wait_or(uint64_t* bar, uint32_t parity, volatile int* abort) {
-  const uint32_t addr = smem_u32(bar);
+  const uint32_t addr = smem_u32(bar), aaddr = smem_u32(const_cast<int*>(abort));
   for (uint32_t i = 0; i < 50000; ++i) {
     uint32_t done;
     asm volatile(
@@ -473,7 +478,7 @@ __device__ __forceinline__ bool mbar_wait_or(uint64_t* bar, uint32_t parity, vol
         : "r"(addr), "r"(parity), "r"(20000)
         : "memory");
     if (done) return true;
-    if (*abort) return false;
+    if (lds32(aaddr)) return false;
   }
   return false;
 }
@@ -627,7 +632,7 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
   auto release_one = [&]() -> bool {
     const uint32_t slot = released % kStages;
     if (!mbar_wait_or(&cr.empty[slot], (released / kStages) & 1, cr.abort_flag)) return false;
-    rused -= cr.sbytes[slot];
+    rused -= static_cast<int>(lds32(smem_u32(cr.sbytes) + 4 * slot));
     ++released;
     return true;
   };
@@ -733,7 +738,7 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
           const bool last = j == T - 1 && k0 + nk >= nkv;
           const int meta = pm | (last ? kLast : 0) | (qb << 16);
           const uint32_t slot =
-              push(make_int4(meta, off, q, lo), rb, make_int4(k0, nk, posb ? off + nk * slice : -1, 0), taken, need);
+              push(make_int4(meta, off, q, lo), rb, make_int4(k0, nk, posb ? off + nk * slice : -1, slice), taken, need);
           if (lane == 0) {
             bulk_g2s(cr.ring + off, page + a.hdr + static_cast<int64_t>(kv0 + k0) * slice, nk * slice, &cr.full[slot]);
             if (posb) bulk_g2s(cr.ring + off + nk * slice, page, posb, &cr.full[slot]);
@@ -929,11 +934,12 @@ __device__ __forceinline__ void run_consumer_cc(const AttnKernelArgs& ka, const 
       }
       break;
     }
-    const int4 ra = cr.recs[slot * 3 + 0];
+    const uint32_t rec = smem_u32(cr.recs) + slot * 48;
+    const int4 ra = lds128i(rec);
     const int meta = ra.x;
     if (meta & kEnd) break;
     if (meta & kQRows) {
-      const int4 rb = cr.recs[slot * 3 + 1];
+      const int4 rb = lds128i(rec + 16);
       const int qb = meta >> 16;
       u_h = qb * kNcw + cw;
       active = u_h < a.Hq;
@@ -969,14 +975,14 @@ __device__ __forceinline__ void run_consumer_cc(const AttnKernelArgs& ka, const 
         sumq = sq2.x + sq2.y;
       }
     } else if (active) {
-      const int4 rc = cr.recs[slot * 3 + 2];
+      const int4 rc = lds128i(rec + 32);
       if (u_kvi >= rc.x && u_kvi < rc.x + rc.y) {
         const int cls = meta & 3, fill = (meta >> 2) & 127;
         if (cls != cur_cls) {
           rescale_dyn(qp, st.acc, cur_cls, cls);
           cur_cls = cls;
         }
-        const uint32_t s0 = smem_u32(cr.ring + ra.y + (u_kvi - rc.x) * a.slice[cls]);
+        const uint32_t s0 = smem_u32(cr.ring + ra.y + (u_kvi - rc.x) * rc.w);
         const bool masked = meta & kMask;
         const uint32_t sp = masked ? smem_u32(cr.ring + rc.z) : s0;
         switch (cls) {
@@ -1435,11 +1441,12 @@ __device__ __forceinline__ void run_consumer_mma(const AttnKernelArgs& ka, const
       }
       break;
     }
-    const int4 ra = cr.recs[slot * 3 + 0];
+    const uint32_t rec = smem_u32(cr.recs) + slot * 48;
+    const int4 ra = lds128i(rec);
     const int meta = ra.x;
     if (meta & kEnd) break;
     if (meta & kQRows) {
-      const int4 rb = cr.recs[slot * 3 + 1];
+      const int4 rb = lds128i(rec + 16);
       const int qb = meta >> 16;
       u_kv = qb * kNcw + cw;
       active = u_kv < a.Hkv;
@@ -1489,14 +1496,14 @@ __device__ __forceinline__ void run_consumer_mma(const AttnKernelArgs& ka, const
         mma_build_kb<D, NG, 16>(ms);
       }
     } else if (active) {
-      const int4 rc = cr.recs[slot * 3 + 2];
+      const int4 rc = lds128i(rec + 32);
       if (cw >= rc.x && cw < rc.x + rc.y) {
         const int cls = meta & 3, fill = (meta >> 2) & 127;
         if (cls != cur_cls) {
           mma_switch<D, NG>(ms, cur_cls, cls);
           cur_cls = cls;
         }
-        const uint32_t s0 = smem_u32(cr.ring + ra.y + (cw - rc.x) * a.slice[cls]);
+        const uint32_t s0 = smem_u32(cr.ring + ra.y + (cw - rc.x) * rc.w);
         const bool masked = meta & kMask;
         const uint32_t sp = masked ? smem_u32(cr.ring + rc.z) : s0;
         switch (cls) {
