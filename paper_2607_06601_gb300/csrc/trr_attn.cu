@@ -393,6 +393,7 @@ constexpr int kStages = 16;       // stage records a CTA may have in flight
 constexpr int kUnitsPerCta = 3;   // units per CTA of a large call, at most
 constexpr float kMinUnitPositions = 512.f;  // key positions of a large call's unit, at least
 constexpr int kCtasPerSm = 3;     // CTAs per SM
+constexpr int kMmaCtasPerSm = 3;  // CTAs per SM of the tensor-core kernels
 
 // Dims per lane of the CUDA-core consumer (E = 16 would use four lanes per key at d = 64
 // and half the registers, but it issues twice the instructions per key), and its CTAs
@@ -401,7 +402,9 @@ __host__ __device__ constexpr int cc_elems(int) { return 32; }
 __host__ __device__ constexpr int cc_ctas_per_sm(int) { return kCtasPerSm; }
 // dynamic shared memory of one attention CTA with `ctas` CTAs per SM (228 KB per SM,
 // 1 KB of it reserved per CTA)
-__host__ __device__ constexpr int attn_smem_limit(int ctas) { return ctas >= 5 ? 44 * 1024 : 72 * 1024; }
+__host__ __device__ constexpr int attn_smem_limit(int ctas) {
+  return ctas >= 5 ? 44 * 1024 : ctas == 2 ? 110 * 1024 : 72 * 1024;
+}
 
 // Stage record, three int4 words written by the producer before it arrives on the
 // stage's full barrier:
@@ -434,6 +437,7 @@ struct AttnKernelArgs {
   int ring_bytes;    // bytes of the CTA's ring of shared memory
   int hpu;           // query heads per work unit
   int scr_floats;    // per-consumer-warp scratch (floats) of the tensor-core path
+  int defer_merge;   // 1: split partials are merged by the combine kernel (tensor-core path)
 };
 
 // Error of a query's arguments, 0 when it is valid.
@@ -604,6 +608,10 @@ __device__ __forceinline__ void plan_units(const AttnKernelArgs& ka, int P, int 
   }
   if (threadIdx.x == blockDim.x - 1) pre[n] = off;
   __syncthreads();
+  if (ka.defer_merge && blockIdx.x == 0) {  // for the combine kernel
+    int2* qtab = reinterpret_cast<int2*>(a.cnt);
+    for (int q = threadIdx.x; q < n; q += blockDim.x) qtab[q] = make_int2(pre[q], pre[q + 1] - pre[q]);
+  }
 }
 
 // Everything the producer and consumers of one CTA share.
@@ -835,6 +843,7 @@ __device__ __forceinline__ void store_or_merge(const AttnKernelArgs& ka, const f
 #pragma unroll
   for (int j = 0; j < DPL; j += 2) *reinterpret_cast<float2*>(pp + dim0 + j) = make_float2(v[j], v[j + 1]);
   if (lane == 0) *reinterpret_cast<float2*>(pp + D) = make_float2(M, L);
+  if (ka.defer_merge) return;  // the combine kernel merges this query's splits
   int* counters = a.cnt + (static_cast<int64_t>(qi) * a.Hq + qh) * a.cnt_stride;
   float Mx, Ls, acc_o[DPL];
   int ngroups = nsplit, gstride = 1;
@@ -1587,7 +1596,7 @@ __global__ void __launch_bounds__(32 * (kNcw + 1), cc_ctas_per_sm(D))
 
 // Tensor-core path: units of kNcw KV heads with all their query heads.
 template <int D, int NG>
-__global__ void __launch_bounds__(32 * (kNcw + 1), kCtasPerSm) attn_mma_kernel(const __grid_constant__ AttnKernelArgs ka) {
+__global__ void __launch_bounds__(32 * (kNcw + 1), kMmaCtasPerSm) attn_mma_kernel(const __grid_constant__ AttnKernelArgs ka) {
   extern __shared__ __align__(128) uint8_t smem[];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int NQB = (ka.a.Hq + ka.hpu - 1) / ka.hpu;
@@ -1604,6 +1613,90 @@ __global__ void __launch_bounds__(32 * (kNcw + 1), kCtasPerSm) attn_mma_kernel(c
   attn_epilogue(ka.a);
 }
 
+// ------------------------------------------------------------------ combine --
+// Merges the split partials of every (query, head) of a tensor-core launch whose query
+// has more than one split: one CTA of kCombineWarps warps per (query, head); warp w folds splits
+// w, w + kCombineWarps, ... over its own maximum, then warp 0 folds the warps and
+// writes the bf16 row.  Chained after the attention kernel (programmatic dependent
+// launch): it reads nothing before that kernel has finished.
+constexpr int kCombineWarps = 4;
+
+struct CombineArgs {
+  const float* part;  // [units][Hq][D + 4] partials of the launch
+  const int2* qtab;   // [n] first partial and splits of each query (written by CTA 0 of the
+                      // attention kernel, in the arrival-counter region it does not use)
+  uint16_t* out;      // [n][Hq][D] bf16 rows of the launch
+  int Hq;
+};
+
+template <int D>
+__global__ void __launch_bounds__(32 * kCombineWarps) attn_combine_kernel(const __grid_constant__ CombineArgs ca) {
+  constexpr int DPL = D / 32;
+  __shared__ float sacc[kCombineWarps][D];
+  __shared__ float sml[kCombineWarps][2];
+  pdl_wait();
+  pdl_trigger();
+  const int qi = blockIdx.x / ca.Hq, qh = blockIdx.x - qi * ca.Hq;
+  const int2 e = ca.qtab[qi];
+  if (e.y <= 1) return;  // one split: written by the attention kernel
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int64_t stride = static_cast<int64_t>(ca.Hq) * (D + 4);
+  const float* p0 = ca.part + (static_cast<int64_t>(e.x) * ca.Hq + qh) * (D + 4) + warp * stride;
+  const int64_t wstride = stride * kCombineWarps;  // between this warp's splits
+  const int cnt = (e.y - warp + kCombineWarps - 1) / kCombineWarps;
+  float Mx = kNegInf;
+  for (int s = lane; s < cnt; s += 32) Mx = fmaxf(Mx, __ldcg(p0 + s * wstride + D));
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) Mx = fmaxf(Mx, __shfl_xor_sync(0xffffffffu, Mx, o));
+  float Ls = 0.f, acc[DPL];
+#pragma unroll
+  for (int j = 0; j < DPL; ++j) acc[j] = 0.f;
+  for (int s0 = 0; s0 < cnt; s0 += 32) {
+    float wl = 0.f;  // lane s: weight of split s0 + s of this warp
+    if (s0 + lane < cnt) {
+      const float2 ml = __ldcg(reinterpret_cast<const float2*>(p0 + (s0 + lane) * wstride + D));
+      wl = (ml.x == kNegInf) ? 0.f : fast_exp2(ml.x - Mx);
+      Ls = fmaf(wl, ml.y, Ls);
+    }
+    const int m = min(32, cnt - s0);
+#pragma unroll 8
+    for (int s = 0; s < m; ++s) {
+      const float wgt = __shfl_sync(0xffffffffu, wl, s);
+      const float* ps = p0 + (s0 + s) * wstride + lane * DPL;
+#pragma unroll
+      for (int j = 0; j < DPL; ++j) acc[j] = fmaf(wgt, __ldcg(ps + j), acc[j]);
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) Ls += __shfl_xor_sync(0xffffffffu, Ls, o);
+#pragma unroll
+  for (int j = 0; j < DPL; ++j) sacc[warp][lane * DPL + j] = acc[j];
+  if (lane == 0) {
+    sml[warp][0] = Mx;
+    sml[warp][1] = Ls;
+  }
+  __syncthreads();
+  if (warp != 0) return;
+  float M = kNegInf;
+#pragma unroll
+  for (int w = 0; w < kCombineWarps; ++w) M = fmaxf(M, sml[w][0]);
+  float L = 0.f, o[DPL];
+#pragma unroll
+  for (int j = 0; j < DPL; ++j) o[j] = 0.f;
+#pragma unroll
+  for (int w = 0; w < kCombineWarps; ++w) {
+    const float f = sml[w][0] == kNegInf ? 0.f : fast_exp2(sml[w][0] - M);
+    L = fmaf(f, sml[w][1], L);
+#pragma unroll
+    for (int j = 0; j < DPL; ++j) o[j] = fmaf(f, sacc[w][lane * DPL + j], o[j]);
+  }
+  const float inv = L > 0.f ? 1.f / L : 0.f;
+  uint16_t* orow = ca.out + (static_cast<int64_t>(qi) * ca.Hq + qh) * D + lane * DPL;
+#pragma unroll
+  for (int j = 0; j < DPL; j += 2)
+    *reinterpret_cast<__nv_bfloat162*>(orow + j) = __floats2bfloat162_rn(o[j] * inv, o[j + 1] * inv);
+}
+
 // Done once per cache at creation, so that calls stay legal inside stream capture.
 cudaError_t attn_configure() {
   struct K {
@@ -1617,11 +1710,11 @@ cudaError_t attn_configure() {
       {reinterpret_cast<const void*>(attn_kernel<128, 16>), cc_ctas_per_sm(128)},
       {reinterpret_cast<const void*>(attn_kernel<128, 32>), cc_ctas_per_sm(128)},
       {reinterpret_cast<const void*>(attn_kernel<128, 64>), cc_ctas_per_sm(128)},
-      {reinterpret_cast<const void*>(attn_mma_kernel<64, 1>), kCtasPerSm},
-      {reinterpret_cast<const void*>(attn_mma_kernel<64, 2>), kCtasPerSm},
-      {reinterpret_cast<const void*>(attn_mma_kernel<128, 1>), kCtasPerSm},
-      {reinterpret_cast<const void*>(attn_mma_kernel<128, 2>), kCtasPerSm},
-      {reinterpret_cast<const void*>(attn_mma_kernel<128, 4>), kCtasPerSm}};
+      {reinterpret_cast<const void*>(attn_mma_kernel<64, 1>), kMmaCtasPerSm},
+      {reinterpret_cast<const void*>(attn_mma_kernel<64, 2>), kMmaCtasPerSm},
+      {reinterpret_cast<const void*>(attn_mma_kernel<128, 1>), kMmaCtasPerSm},
+      {reinterpret_cast<const void*>(attn_mma_kernel<128, 2>), kMmaCtasPerSm},
+      {reinterpret_cast<const void*>(attn_mma_kernel<128, 4>), kMmaCtasPerSm}};
   for (const K& k : kernels) {
     const cudaError_t e =
         cudaFuncSetAttribute(k.f, cudaFuncAttributeMaxDynamicSharedMemorySize, attn_smem_limit(k.ctas));
@@ -1654,7 +1747,7 @@ constexpr int kMaxLaunchQueries = 1024;
 
 static cudaError_t launch_one(const Layout& l, const AttnKernelArgs& ka, int num_sms, cudaStream_t s) {
   const bool mma = use_mma(l);
-  const int ctas = mma ? kCtasPerSm : cc_ctas_per_sm(l.d);
+  const int ctas = mma ? kMmaCtasPerSm : cc_ctas_per_sm(l.d);
   const int ring = attn_ring_bytes(l, ka.n, ka.hpu, ka.scr_floats, attn_smem_limit(ctas));
   if (ring < 0) return cudaErrorInvalidConfiguration;
   AttnKernelArgs k = ka;
@@ -1698,6 +1791,7 @@ static cudaError_t launch_attention(const Layout& l, const LayerArgs& a, int num
   const bool mma = use_mma(l);
   const int g = l.Hq / l.Hkv;
   ka.hpu = mma ? kNcw * g : kNcw;
+  ka.defer_merge = mma ? 1 : 0;
   // tensor-core scratch per consumer warp: the query's bf16 words (4 d floats), later
   // the unit's rows (g (d + 4) floats)
   ka.scr_floats = mma ? std::max(4 * l.d, g * (l.d + 4)) : 0;
@@ -1712,9 +1806,21 @@ static cudaError_t launch_attention(const Layout& l, const LayerArgs& a, int num
     ka.q = static_cast<const uint16_t*>(q_bf16) + q0 * row;
     ka.out = static_cast<uint16_t*>(out_bf16) + q0 * row;
     ka.a.cnt = a.cnt + static_cast<int64_t>(q0) * l.Hq * l.cnt_stride;
-    const cudaError_t e = launch_one(l, ka, num_sms, s);
+    cudaError_t e = launch_one(l, ka, num_sms, s);
     if (e != cudaSuccess) return e;
     ++*launches;
+    if (mma) {  // the tensor-core path's splits are merged by the combine kernel
+      CombineArgs ca;
+      ca.part = a.part;
+      ca.qtab = reinterpret_cast<const int2*>(ka.a.cnt);
+      ca.out = ka.out;
+      ca.Hq = l.Hq;
+      const dim3 cgrid(ka.n * l.Hq), cblock(32 * kCombineWarps);
+      e = l.d == 64 ? launch_pdl(attn_combine_kernel<64>, cgrid, cblock, 0, s, ca)
+                    : launch_pdl(attn_combine_kernel<128>, cgrid, cblock, 0, s, ca);
+      if (e != cudaSuccess) return e;
+      ++*launches;
+    }
   }
   return cudaSuccess;
 }
