@@ -68,6 +68,10 @@ def lib() -> ctypes.CDLL:
         L.orc_double_to_f16.restype = ctypes.c_uint16
         L.orc_bf16_to_double.argtypes = [ctypes.c_uint16]
         L.orc_bf16_to_double.restype = ctypes.c_double
+        L.orc_argmax.argtypes = [P, I]
+        L.orc_argmax.restype = I
+        L.orc_route_decisions.argtypes = [I, P, P, P, I, I, I, I, I, P, P, P, P, P]
+        L.orc_route_decisions.restype = I
         _lib = L
     return _lib
 
@@ -187,3 +191,32 @@ def double_to_f16(x: float) -> int:
 
 def bf16_to_double(h: int) -> float:
     return lib().orc_bf16_to_double(h)
+
+
+def argmax(z) -> int:
+    """The hard decision of one controller head (Sec. 3.8): first maximum, NaN never."""
+    z = _c(z, np.float32)
+    return int(lib().orc_argmax(_ptr(z), z.shape[0]))
+
+
+def route_decisions(mode_logits, bit_logits, positions, window, num_q_heads, head_dim,
+                    num_kv_heads, skip_writes_kv=0, totals=None):
+    """Hard decisions of n tokens and their cost (Sec. 3.5 / 3.8, Appendix C).
+
+    Returns (modes uint8[n], bits uint8[n], attn_flops int64[n], kv_bits int64[n],
+    totals int64[4]); ``totals`` (if given) is added to, as the C function does."""
+    ml, bl = _c(mode_logits, np.float32), _c(bit_logits, np.float32)
+    pos = _c(positions, np.int32)
+    n = pos.shape[0]
+    assert ml.size == 3 * n and bl.size == 4 * n
+    modes = np.zeros(n, dtype=np.uint8)
+    bits = np.zeros(n, dtype=np.uint8)
+    flops = np.zeros(n, dtype=np.int64)
+    mem = np.zeros(n, dtype=np.int64)
+    tot = np.zeros(4, dtype=np.int64) if totals is None else _c(totals, np.int64).copy()
+    st = lib().orc_route_decisions(n, _ptr(ml), _ptr(bl), _ptr(pos), int(window), int(num_q_heads),
+                                   int(head_dim), int(num_kv_heads), int(skip_writes_kv),
+                                   _ptr(modes), _ptr(bits), _ptr(flops), _ptr(mem), _ptr(tot))
+    if st != 0:
+        raise ValueError(f"orc_route_decisions: {STATUS.get(st, st)}")
+    return modes, bits, flops, mem, tot

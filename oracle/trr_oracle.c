@@ -20,6 +20,8 @@
  *     all positions <= t.  Only stored tokens take part.
  *   - hard decisions at inference, KV stored at the chosen width, paged cache
  *     (Sec. 3.8); grouping tokens by precision (Sec. 7) -> one width class per page.
+ *   - the hard decision itself (arg max of the router's logits, Sec. 3.8) and the
+ *     cost model of Sec. 3.5 / Appendix C evaluated at it (orc_route_decisions).
  *
  * Floating point: fl32(op) is computed as a double operation followed by a cast to
  * float.  For +, -, * and / of binary32 operands this double rounding is innocuous
@@ -556,4 +558,66 @@ int64_t orc_layout(const orc_cache* o, int which) {
   if (which >= 1 && which <= 4) return o->slice[which - 1];
   if (which >= 5 && which <= 8) return o->page_bytes[which - 5];
   return -1;
+}
+
+/* ---------------------------------------------- hard decisions and their cost -- */
+
+/* The hard decision of one controller head (Sec. 3.8: at inference the router takes
+ * the arg max of its logits).  Readings where the paper is silent: the first of equal
+ * maxima wins; a NaN logit is never the maximum; a row of NaN gives option 0.
+ * Returned: the smallest i whose logit is a number no smaller than every other
+ * logit that is a number. */
+int orc_argmax(const float* z, int k) {
+  int i, j;
+  for (i = 0; i < k; i++) {
+    int top = !isnan(z[i]);
+    for (j = 0; j < k && top; j++)
+      if (!isnan(z[j]) && z[j] > z[i]) top = 0;
+    if (top) return i;
+  }
+  return 0;
+}
+
+/* Hard decisions of n tokens at one layer and what they cost.
+ *   mode_logits [n][3]: options skip, local, full (the order of Sec. 3.2(A));
+ *   bit_logits  [n][4]: options b = 2, 4, 8, 16 (Sec. 3.2(C)).
+ * Cost of the one-hot policy (the cost model of Sec. 3.5 evaluated at the hard
+ * decision, as Appendix C's expected_cost does with one-hot a and b):
+ *   attention: for each of the Hq heads, 2 d per key interaction, and a query at
+ *   0-indexed position p interacts with the positions it reads: full -> every j <= p,
+ *   local -> those with j >= p - w + 1 as well (the w-key window), skip -> none.
+ *   Appendix C charges at least one position; a negative p is charged as p = 0.
+ *   memory: 2 d_kv b bits with d_kv = Hkv d (K and V of every KV head); a skip
+ *   token that stores nothing (skip_writes_kv == 0) is charged 0.
+ * totals (added to, not overwritten): [0] sum of attention costs, [1] sum of memory
+ * costs, [2] the dense attention cost (every head full: 2 d Hq (p + 1)), [3] the
+ * dense memory cost (2 d_kv 16), the normalisers C_dense of Appendix C. */
+int orc_route_decisions(int n, const float* mode_logits, const float* bit_logits,
+                        const int32_t* positions, int window, int Hq, int d, int Hkv,
+                        int skip_writes_kv, uint8_t* modes, uint8_t* bits,
+                        int64_t* attn_flops, int64_t* kv_bits, int64_t* totals) {
+  int i;
+  if (n < 0 || window < 1 || Hq < 1 || d < 1 || Hkv < 1) return ORC_INVALID_ARG;
+  for (i = 0; i < n; i++) {
+    int m = orc_argmax(mode_logits + 3 * (int64_t)i, 3);
+    int b = BITS_OF_CLASS[orc_argmax(bit_logits + 4 * (int64_t)i, 4)];
+    int64_t p = positions[i] < 0 ? 0 : positions[i];
+    /* key interactions, counted one position at a time */
+    int64_t keys = 0, dense_keys = 0, j;
+    for (j = 0; j <= p; j++) {
+      dense_keys++;
+      if (m == 2 || (m == 1 && j >= p - window + 1)) keys++;
+    }
+    int64_t flops = (int64_t)Hq * 2 * d * keys;
+    int64_t mem = (m == 0 && !skip_writes_kv) ? 0 : 2 * (int64_t)Hkv * d * b;
+    modes[i] = (uint8_t)m;
+    bits[i] = (uint8_t)b;
+    attn_flops[i] = flops;
+    kv_bits[i] = mem;
+    totals[0] += flops;
+    totals[1] += mem;
+    totals[2] += (int64_t)Hq * 2 * d * dense_keys;
+    totals[3] += 2 * (int64_t)Hkv * d * 16;
+  }
+  return ORC_OK;
 }
