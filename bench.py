@@ -20,6 +20,11 @@ e2e    = the same, through the C ABI with host buffers: pinned H2D of every step
 roofline: the dominant kernel is the trr_decode_attn call (one attention kernel);
          achieved = its algorithmic bytes per call / its average duration from CUDA
          event nodes placed around each call in a second, instrumented replay.
+routed : the same step driven by router logits (Sec. 3.8 hard decisions): per layer
+         trr_route_decisions (cost totals of the executed policy, Sec. 3.5),
+         trr_kv_append_routed and trr_decode_attn_routed, with logits whose arg max is
+         the workload's seeded bits and modes; plus one prefill-sized
+         trr_route_decisions call (2^22 tokens) against the HBM roofline.
 """
 from __future__ import annotations
 
@@ -262,7 +267,9 @@ class Bench:
             s.num_layers, s.batch, s.num_q_heads, s.num_kv_heads, s.head_dim, s.group_size)
         self.window = s.window
         self.e2e_warm, self.e2e_steps = 2, min(args.steps, 20)
-        self.total_steps = args.warmup + 2 * args.steps + self.e2e_warm + self.e2e_steps
+        self.routed_warm, self.routed_steps = 2, min(args.steps, 10)
+        self.total_steps = (args.warmup + 2 * args.steps + self.e2e_warm + self.e2e_steps + self.routed_warm +
+                            self.routed_steps)
         self.grow = 32                                   # tokens a sequence may grow
         self.R = max(1, math.ceil(self.total_steps / self.grow))
         self.P = args.page_size or PAGE
@@ -360,10 +367,16 @@ class Bench:
                 nb, nk, _ = self.acct.query(bits[s], modes[s], int(pos[s]))
                 nbytes += nb
                 keys += nk
+            # router logits whose arg max is the seeded decision (the routed step)
+            ml = torch.rand((self.B, 3), generator=gen, device=self.dev) - 2.0
+            bl = torch.rand((self.B, 4), generator=gen, device=self.dev) - 2.0
+            ml[torch.arange(self.B, device=self.dev), torch.from_numpy(m.astype(np.int64)).to(self.dev)] = 1.0
+            bcls = np.array([BITS.index(int(x)) for x in b], dtype=np.int64)
+            bl[torch.arange(self.B, device=self.dev), torch.from_numpy(bcls).to(self.dev)] = 1.0
             layers.append(dict(
                 seqs=torch.from_numpy(seqs).to(self.dev), pos=torch.from_numpy(pos).to(self.dev),
                 bits=torch.from_numpy(b).to(self.dev), modes=torch.from_numpy(m).to(self.dev),
-                k=k, v=v, q=q,
+                k=k, v=v, q=q, ml=ml.contiguous(), bl=bl.contiguous(),
                 out=torch.empty((self.B, self.Hq, self.d), dtype=torch.bfloat16, device=self.dev)))
         attn_bytes_per_layer = nbytes / self.L
         return dict(layers=layers, bytes=nbytes, keys=keys, attn_bytes_per_layer=attn_bytes_per_layer)
@@ -384,16 +397,114 @@ class Bench:
                 events[1](l)
         return n
 
-    def capture(self, idx, instrument=None):
+    def run_routed_step(self, st, totals, stream=None):
+        """The step driven by router logits: decisions and their cost, then the routed
+        append and attention, which take the same decisions in their own kernels."""
+        c, trr = self.cache, self.trr
+        n = 0
+        for l, x in enumerate(st["layers"]):
+            trr.trr_route_decisions(x["ml"], x["bl"], x["pos"], self.window, self.Hq, self.d, self.Hkv,
+                                    totals=totals, stream=stream)
+            c.append_routed(l, x["seqs"], x["pos"], x["k"], x["v"], x["bl"], x["ml"], stream=stream)
+            n += 1 + c.launches()
+            c.decode_attn_routed(l, x["seqs"], x["pos"], x["q"], x["ml"], window_scalar=self.window,
+                                 out=x["out"], stream=stream)
+            n += c.launches()
+        return n
+
+    def capture(self, idx, instrument=None, totals=None):
         torch = self.torch
         g = torch.cuda.CUDAGraph()
         s = torch.cuda.Stream()
         s.wait_stream(torch.cuda.current_stream())
         with torch.cuda.stream(s):
             with torch.cuda.graph(g, stream=s):
-                launches = self.run_step(self.steps[idx], instrument(idx, s) if instrument else None)
+                if totals is not None:
+                    launches = self.run_routed_step(self.steps[idx], totals)
+                else:
+                    launches = self.run_step(self.steps[idx], instrument(idx, s) if instrument else None)
         torch.cuda.current_stream().wait_stream(s)
         return g, launches
+
+
+def run_routed(bench, dist, r0):
+    """The routed step (decisions from logits) timed over its own steps, and one
+    prefill-sized trr_route_decisions call against the HBM roofline."""
+    torch, trr = bench.torch, bench.trr
+    totals = torch.zeros(4, dtype=torch.int64, device=bench.dev)
+    graphs = [bench.capture(i, totals=totals) for i in range(r0, r0 + bench.routed_warm + bench.routed_steps)]
+    launches = graphs[0][1]
+    for g, _ in graphs[:bench.routed_warm]:
+        g.replay()
+    torch.cuda.synchronize()
+    totals.zero_()
+    if dist:
+        dist.barrier()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for g, _ in graphs[bench.routed_warm:]:
+        g.replay()
+    t1.record()
+    torch.cuda.synchronize()
+    ms = t0.elapsed_time(t1)
+    idx = range(r0 + bench.routed_warm, r0 + bench.routed_warm + bench.routed_steps)
+    nbytes = sum(bench.steps[i]["bytes"] for i in idx)
+    ms, nbytes = across_ranks(dist, "cuda", ms, nbytes)
+    tot = totals.cpu().tolist()
+    del graphs
+
+    # one prefill-sized decision call: 2^22 tokens (210 MB of inputs and outputs)
+    n = 1 << 22
+    gen = torch.Generator(device=bench.dev)
+    gen.manual_seed(_mix(bench.spec.seed, 3))
+    ml = torch.randn((n, 3), generator=gen, device=bench.dev)
+    bl = torch.randn((n, 4), generator=gen, device=bench.dev)
+    pos = torch.randint(0, 8192, (n,), generator=gen, device=bench.dev, dtype=torch.int32)
+    out = dict(modes=torch.empty(n, dtype=torch.uint8, device=bench.dev),
+               bits=torch.empty(n, dtype=torch.uint8, device=bench.dev),
+               attn_flops=torch.empty(n, dtype=torch.int64, device=bench.dev),
+               kv_bits=torch.empty(n, dtype=torch.int64, device=bench.dev))
+    ptot = torch.zeros(4, dtype=torch.int64, device=bench.dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=bench.dev)
+
+    def call():
+        trr.trr_route_decisions(ml, bl, pos, bench.window, bench.Hq, bench.d, bench.Hkv, totals=ptot, **out)
+
+    # one call captured as a graph, so that the timed region holds no host marshalling
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(side):
+        with torch.cuda.graph(graph, stream=side):
+            call()
+    torch.cuda.current_stream().wait_stream(side)
+    for _ in range(3):
+        graph.replay()
+    times = []
+    for _ in range(10):
+        flush.fill_(1)  # evict the inputs from L2 between calls (and keep the GPU busy)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        graph.replay()
+        b.record()
+        torch.cuda.synchronize()
+        times.append(a.elapsed_time(b))
+    del flush, graph
+    us = statistics.median(times) * 1e3
+    per_token = 3 * 4 + 4 * 4 + 4 + 1 + 1 + 8 + 8  # logits, position in; decisions, costs out
+    gbs = n * per_token / (us * 1e-6) / 1e9
+    peak, _ = measured_peaks()
+    return {
+        "value": round(nbytes / (ms * 1e-3) / 1e9, 2), "unit": UNIT,
+        "ms_per_step": round(ms / bench.routed_steps, 5), "steps": bench.routed_steps,
+        "gpu_launches": launches * bench.routed_steps,
+        "budget": {"attn_flops_frac": round(tot[0] / tot[2], 4) if tot[2] else None,
+                   "kv_bits_frac": round(tot[1] / tot[3], 4) if tot[3] else None,
+                   "note": "executed cost / dense cost of the timed steps' tokens (Sec. 3.5, App. C)"},
+        "route_decisions": {"tokens": n, "us_per_call": round(us, 2), "bytes_per_token": per_token,
+                            "achieved_gbs": round(gbs, 1), "peak": peak, "frac": round(gbs / peak, 4),
+                            "l2": "256 MB buffer written between calls"},
+    }
 
 
 def run_gpu(args):
@@ -526,6 +637,7 @@ def run_gpu(args):
     e2e_ms = a0.elapsed_time(a1)
     e2e_bytes = sum(bench.steps[e0 + j]["bytes"] for j in range(bench.e2e_warm, bench.e2e_warm + bench.e2e_steps))
     e2e_ms, e2e_bytes = across_ranks(dist, "cuda", e2e_ms, e2e_bytes)
+    routed = run_routed(bench, dist, e0 + bench.e2e_warm + bench.e2e_steps)
     status = bench.cache.status()
     if status != 0:
         raise RuntimeError(f"device status {status} after the run")
@@ -565,6 +677,7 @@ def run_gpu(args):
                          "kernel": "trr_decode_attn call (attn_kernel, one launch)",
                          "bytes_per_call": round(avg_bytes), "us_per_call": round(avg_ms * 1e3, 3)},
             "clocks": clocks.summary(),
+            "routed": routed,
         }
         if cpu is not None:
             result["cpu_baseline"] = cpu

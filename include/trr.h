@@ -12,7 +12,10 @@
  * and each token's KV is stored at its chosen width in a paged cache (Sec. 3.8).
  * Sec. 7 names the two kernels a production system needs: mode-aware attention over
  * ragged skip/local/full work, and a mixed-precision paged KV cache that groups tokens
- * by precision.  Those are trr_decode_attn and trr_kv_append below.
+ * by precision.  Those are trr_decode_attn and trr_kv_append below.  The hard
+ * decisions themselves (arg max of the router's logits) and their cost under the
+ * model of Sec. 3.5 are trr_route_decisions; trr_kv_append_routed and
+ * trr_decode_attn_routed take the same decisions inside their own kernels.
  *
  * Conventions shared by every entry point
  *   - Pointers marked "device" are CUDA device pointers on the current device; the
@@ -182,6 +185,56 @@ TRR_API trr_status trr_decode_attn(trr_cache* cache, int32_t layer, int32_t n,
 TRR_API trr_status trr_decode_attn_static(trr_cache* cache, int32_t layer, int32_t n,
                                           const int32_t* seq_ids, const int32_t* q_positions,
                                           const void* q_bf16, const uint8_t* modes,
+                                          const int32_t* windows, int32_t window_scalar,
+                                          float softmax_scale, void* out_bf16, void* stream);
+
+/* The router's hard decisions at inference and their cost (Sec. 3.8: the router takes
+ * the arg max of its logits and only the selected computation runs; Sec. 3.5 cost
+ * model, evaluated at the one-hot policy as Appendix C's expected_cost does).
+ *   mode_logits[n][3] (options skip, local, full) and bit_logits[n][4] (options
+ *   b = 2, 4, 8, 16): fp32, device.  Decision = index of the largest logit, the first
+ *   of equal ones; a NaN logit is never chosen; a row of NaN gives option 0.
+ *   Outputs (device, each may be NULL): modes[n], bits[n] (uint8, the values
+ *   trr_kv_append / trr_decode_attn take); attn_flops[n] = Hq * 2 * d * kappa with
+ *   kappa the key positions the query reads at 0-indexed position p = positions[i]:
+ *   full p + 1, local min(p + 1, window), skip 0 (p < 0 is charged as p = 0);
+ *   kv_bits[n] = 2 * Hkv * d * b bits (the cost model's 2 d_kv b), 0 for a skip token
+ *   when skip_writes_kv == 0 (it stores nothing).
+ *   totals[4] (int64, device, ADDED to, so that calls over layers and steps
+ *   accumulate): sum of attn_flops, sum of kv_bits, the dense attention cost
+ *   sum Hq * 2 * d * (p + 1) and the dense memory cost n * 2 * Hkv * d * 16, the
+ *   normalisers of the budget fractions (Appendix C).
+ *   positions, window >= 1 and the head shape are needed only when attn_flops,
+ *   kv_bits or totals is given.  Float arrays 4-byte aligned, int64 arrays 8-byte.
+ *   The logits and positions are read after the previous kernel of the stream has
+ *   finished.  The outputs must not be passed to the very next trr_* call on the
+ *   stream (trr_kv_append and trr_decode_attn read their index arrays while the
+ *   previous kernel still runs): pass the logits to the *_routed calls instead, which
+ *   decide the same way. */
+TRR_API trr_status trr_route_decisions(int32_t n, const float* mode_logits, const float* bit_logits,
+                                       const int32_t* positions, int32_t window, int32_t num_q_heads,
+                                       int32_t head_dim, int32_t num_kv_heads, int32_t skip_writes_kv,
+                                       uint8_t* modes, uint8_t* bits, int64_t* attn_flops,
+                                       int64_t* kv_bits, int64_t* totals, void* stream);
+
+/* trr_kv_append with each entry's mode and bit-width decided in the append's own
+ * planning step from the router's logits, exactly as trr_route_decisions decides:
+ * bit_logits[n][4] (b = 2, 4, 8, 16) and mode_logits[n][3] (skip, local, full), fp32,
+ * device, 4-byte aligned.  Otherwise the same arguments, results and error contract as
+ * trr_kv_append (the logits, like the other inputs, may be read while the previous
+ * kernel of the stream is still running). */
+TRR_API trr_status trr_kv_append_routed(trr_cache* cache, int32_t layer, int32_t n,
+                                        const int32_t* seq_ids, const int32_t* positions,
+                                        const void* k_bf16, const void* v_bf16,
+                                        const float* bit_logits, const float* mode_logits,
+                                        void* stream);
+
+/* trr_decode_attn with each query's mode decided in the attention's planning step from
+ * mode_logits[n][3] (skip, local, full; fp32, device, 4-byte aligned), exactly as
+ * trr_route_decisions decides.  Otherwise the same as trr_decode_attn. */
+TRR_API trr_status trr_decode_attn_routed(trr_cache* cache, int32_t layer, int32_t n,
+                                          const int32_t* seq_ids, const int32_t* q_positions,
+                                          const void* q_bf16, const float* mode_logits,
                                           const int32_t* windows, int32_t window_scalar,
                                           float softmax_scale, void* out_bf16, void* stream);
 

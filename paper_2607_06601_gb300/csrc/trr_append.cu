@@ -19,10 +19,21 @@ __device__ __forceinline__ int class_of_bits(int b) {
   return b == 2 ? 0 : b == 4 ? 1 : b == 8 ? 2 : b == 16 ? 3 : -1;
 }
 
+// An entry's attention mode and bit-width: the caller's, or the hard decisions of its
+// router logits (Sec. 3.8), taken here in the append's own planning step.
+__device__ __forceinline__ int entry_mode(const uint8_t* modes, const float* mode_logits, int e) {
+  return mode_logits ? hard_decision<3>(mode_logits + 3 * e) : modes[e];
+}
+__device__ __forceinline__ int entry_bits(const uint8_t* bits, const float* bit_logits, int e) {
+  return bit_logits ? 2 << hard_decision<4>(bit_logits + 4 * e) : bits[e];
+}
+
 __global__ void __launch_bounds__(1024) append_plan_kernel(LayerArgs a, int n, const int32_t* __restrict__ seq_ids,
                                                            const int32_t* __restrict__ positions,
                                                            const uint8_t* __restrict__ bits,
-                                                           const uint8_t* __restrict__ modes) {
+                                                           const uint8_t* __restrict__ modes,
+                                                           const float* __restrict__ bit_logits,
+                                                           const float* __restrict__ mode_logits) {
   __shared__ int s_seq[1024];
   __shared__ int s_pos[1024];
   __shared__ int s_cls[1024];   // width class when the entry stores KV, else -1
@@ -39,11 +50,11 @@ __global__ void __launch_bounds__(1024) append_plan_kernel(LayerArgs a, int n, c
   if (act) {
     seq = seq_ids[e];
     pos = positions[e];
-    const int m = modes[e];
+    const int m = entry_mode(modes, mode_logits, e);
     if (seq < 0 || seq >= a.S) {
       err = TRR_ERR_INVALID_ARG;
     } else {
-      c = class_of_bits(bits[e]);
+      c = class_of_bits(entry_bits(bits, bit_logits, e));
       if (c < 0 || m > TRR_MODE_FULL) err = TRR_ERR_INVALID_ARG;
       else if (pos < 0 || pos >= a.maxctx) err = TRR_ERR_BAD_POSITION;
     }
@@ -307,6 +318,8 @@ __global__ void __launch_bounds__(256) append_fused_kernel(LayerArgs a, int n, c
                                                            const int32_t* __restrict__ positions,
                                                            const uint8_t* __restrict__ bits,
                                                            const uint8_t* __restrict__ modes,
+                                                           const float* __restrict__ bit_logits,
+                                                           const float* __restrict__ mode_logits,
                                                            const uint16_t* __restrict__ k,
                                                            const uint16_t* __restrict__ v) {
   __shared__ int s_seq[kFusedMax];
@@ -339,11 +352,11 @@ __global__ void __launch_bounds__(256) append_fused_kernel(LayerArgs a, int n, c
   if (act) {
     seq = seq_ids[e];
     pos = positions[e];
-    const int m = modes[e];
+    const int m = entry_mode(modes, mode_logits, e);
     if (seq < 0 || seq >= a.S) {
       err = TRR_ERR_INVALID_ARG;
     } else {
-      c = class_of_bits(bits[e]);
+      c = class_of_bits(entry_bits(bits, bit_logits, e));
       if (c < 0 || m > TRR_MODE_FULL) err = TRR_ERR_INVALID_ARG;
       else if (pos < 0 || pos >= a.maxctx) err = TRR_ERR_BAD_POSITION;
     }
@@ -480,35 +493,56 @@ __global__ void __launch_bounds__(256) append_fused_kernel(LayerArgs a, int n, c
 
 using namespace trr;
 
-extern "C" trr_status trr_kv_append(trr_cache* cache, int32_t layer, int32_t n, const int32_t* seq_ids,
-                                    const int32_t* positions, const void* k_bf16, const void* v_bf16,
-                                    const uint8_t* bits, const uint8_t* modes, void* stream) {
+// One append call: the entries' modes and widths come from `bits` / `modes`, or (with
+// those null) from the router logits.
+static trr_status append_call(trr_cache* cache, int32_t layer, int32_t n, const int32_t* seq_ids,
+                              const int32_t* positions, const void* k_bf16, const void* v_bf16, const uint8_t* bits,
+                              const uint8_t* modes, const float* bit_logits, const float* mode_logits,
+                              void* stream) {
   if (!cache) return TRR_ERR_INVALID_ARG;
   const Layout& l = cache_layout(cache);
   if (layer < 0 || layer >= l.L || n < 0 || n > l.max_append) return TRR_ERR_INVALID_ARG;
   cache_set_launches(cache, 0);
   if (n == 0) return TRR_OK;
-  if (!seq_ids || !positions || !k_bf16 || !v_bf16 || !bits || !modes) return TRR_ERR_INVALID_ARG;
+  if (!seq_ids || !positions || !k_bf16 || !v_bf16 || !(bits || bit_logits) || !(modes || mode_logits))
+    return TRR_ERR_INVALID_ARG;
   if ((reinterpret_cast<uintptr_t>(k_bf16) | reinterpret_cast<uintptr_t>(v_bf16)) & 15)
     return TRR_ERR_INVALID_ARG;  // rows are read 16 bytes at a time
+  if ((reinterpret_cast<uintptr_t>(bit_logits) | reinterpret_cast<uintptr_t>(mode_logits)) & 3)
+    return TRR_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const LayerArgs a = layer_args(l, cache_views(cache), layer);
+  const uint16_t* k = static_cast<const uint16_t*>(k_bf16);
+  const uint16_t* v = static_cast<const uint16_t*>(v_bf16);
   if (n <= kFusedMax) {  // one kernel: 256 threads plan, one warp per (entry, head, K|V) row
     const unsigned blocks = static_cast<unsigned>((static_cast<int64_t>(n) * l.Hkv * 2 + 7) / 8);
     const cudaError_t e =
         l.d == 64 ? launch_pdl(append_fused_kernel<64>, dim3(blocks), dim3(256), 0, s, a, n, seq_ids, positions, bits,
-                               modes, static_cast<const uint16_t*>(k_bf16), static_cast<const uint16_t*>(v_bf16))
+                               modes, bit_logits, mode_logits, k, v)
                   : launch_pdl(append_fused_kernel<128>, dim3(blocks), dim3(256), 0, s, a, n, seq_ids, positions,
-                               bits, modes, static_cast<const uint16_t*>(k_bf16), static_cast<const uint16_t*>(v_bf16));
+                               bits, modes, bit_logits, mode_logits, k, v);
     cache_set_launches(cache, 1);
     return e == cudaSuccess ? TRR_OK : TRR_ERR_CUDA;
   }
   const int threads = (n + 31) / 32 * 32;
-  cudaError_t e = launch_pdl(append_plan_kernel, dim3(1), dim3(threads), 0, s, a, n, seq_ids, positions, bits, modes);
+  cudaError_t e = launch_pdl(append_plan_kernel, dim3(1), dim3(threads), 0, s, a, n, seq_ids, positions, bits, modes,
+                             bit_logits, mode_logits);
   if (e != cudaSuccess) return TRR_ERR_CUDA;
   const int64_t work = static_cast<int64_t>(n) * l.Hkv * 2 * (l.d / l.G);
-  e = launch_pdl(append_write_kernel, dim3(static_cast<unsigned>((work + 255) / 256)), dim3(256), 0, s, a, n,
-                 static_cast<const uint16_t*>(k_bf16), static_cast<const uint16_t*>(v_bf16));
+  e = launch_pdl(append_write_kernel, dim3(static_cast<unsigned>((work + 255) / 256)), dim3(256), 0, s, a, n, k, v);
   cache_set_launches(cache, 2);
   return e == cudaSuccess ? TRR_OK : TRR_ERR_CUDA;
+}
+
+extern "C" trr_status trr_kv_append(trr_cache* cache, int32_t layer, int32_t n, const int32_t* seq_ids,
+                                    const int32_t* positions, const void* k_bf16, const void* v_bf16,
+                                    const uint8_t* bits, const uint8_t* modes, void* stream) {
+  return append_call(cache, layer, n, seq_ids, positions, k_bf16, v_bf16, bits, modes, nullptr, nullptr, stream);
+}
+
+extern "C" trr_status trr_kv_append_routed(trr_cache* cache, int32_t layer, int32_t n, const int32_t* seq_ids,
+                                           const int32_t* positions, const void* k_bf16, const void* v_bf16,
+                                           const float* bit_logits, const float* mode_logits, void* stream) {
+  return append_call(cache, layer, n, seq_ids, positions, k_bf16, v_bf16, nullptr, nullptr, bit_logits, mode_logits,
+                     stream);
 }

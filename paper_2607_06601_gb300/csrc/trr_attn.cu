@@ -427,7 +427,8 @@ struct AttnKernelArgs {
   int n;                       // queries of the call
   const int32_t* seq_ids;
   const int32_t* q_positions;
-  const uint8_t* modes;
+  const uint8_t* modes;        // per-query modes, or null: mode_logits
+  const float* mode_logits;    // [n][3] router logits (skip, local, full), or null
   const int32_t* windows;      // per-query windows, or null: window_scalar
   int window_scalar;
   const uint16_t* q;
@@ -439,6 +440,11 @@ struct AttnKernelArgs {
   int scr_floats;    // per-consumer-warp scratch (floats) of the tensor-core path
   int defer_merge;   // 1: split partials are merged by the combine kernel (tensor-core path)
 };
+
+// Mode of query q: the caller's, or the hard decision of its mode logits.
+__device__ __forceinline__ int query_mode(const AttnKernelArgs& ka, int q) {
+  return ka.mode_logits ? hard_decision<3>(ka.mode_logits + 3 * q) : ka.modes[q];
+}
 
 // Error of a query's arguments, 0 when it is valid.
 __device__ __forceinline__ int query_error(const LayerArgs& a, int seq, int t, int mode, int w) {
@@ -562,7 +568,7 @@ __device__ __forceinline__ void plan_units(const AttnKernelArgs& ka, int P, int 
   const int n = ka.n, lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
   long long rsum = 0;
   for (int q = threadIdx.x; q < n; q += blockDim.x) {
-    const int seq = ka.seq_ids[q], t = ka.q_positions[q], mode = ka.modes[q];
+    const int seq = ka.seq_ids[q], t = ka.q_positions[q], mode = query_mode(ka, q);
     const int w = ka.windows ? ka.windows[q] : ka.window_scalar;
     const int r = query_error(a, seq, t, mode, w) ? 0 : query_range(t, mode, w);
     pre[q] = r;
@@ -691,7 +697,7 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
       else hi_q = mid;
     }
     const int q = lo_q, sp = un - pre[q], ns = pre[q + 1] - pre[q];
-    const int seq = ka.seq_ids[q], t = ka.q_positions[q], mode = ka.modes[q];
+    const int seq = ka.seq_ids[q], t = ka.q_positions[q], mode = query_mode(ka, q);
     const int w = ka.windows ? ka.windows[q] : ka.window_scalar;
     const int err = query_error(a, seq, t, mode, w);
     const int h0 = qb * ka.hpu, nh = min(ka.hpu, a.Hq - h0);
@@ -1780,8 +1786,9 @@ static cudaError_t launch_one(const Layout& l, const AttnKernelArgs& ka, int num
 // counts them.
 static cudaError_t launch_attention(const Layout& l, const LayerArgs& a, int num_sms, int n,
                                     const int32_t* seq_ids, const int32_t* q_positions, const void* q_bf16,
-                                    const uint8_t* modes, const int32_t* windows, int window_scalar,
-                                    float softmax_scale, void* out_bf16, cudaStream_t s, int* launches) {
+                                    const uint8_t* modes, const float* mode_logits, const int32_t* windows,
+                                    int window_scalar, float softmax_scale, void* out_bf16, cudaStream_t s,
+                                    int* launches) {
   *launches = 0;
   AttnKernelArgs ka;
   ka.a = a;
@@ -1801,7 +1808,8 @@ static cudaError_t launch_attention(const Layout& l, const LayerArgs& a, int num
     ka.q0 = q0;
     ka.seq_ids = seq_ids + q0;
     ka.q_positions = q_positions + q0;
-    ka.modes = modes + q0;
+    ka.modes = modes ? modes + q0 : nullptr;
+    ka.mode_logits = mode_logits ? mode_logits + 3 * q0 : nullptr;
     ka.windows = windows ? windows + q0 : nullptr;
     ka.q = static_cast<const uint16_t*>(q_bf16) + q0 * row;
     ka.out = static_cast<uint16_t*>(out_bf16) + q0 * row;
@@ -1844,7 +1852,29 @@ extern "C" trr_status trr_decode_attn(trr_cache* cache, int32_t layer, int32_t n
   const LayerArgs a = layer_args(l, cache_views(cache), layer);
   int launches = 0;
   const cudaError_t e = launch_attention(l, a, cache_num_sms(cache), n, seq_ids, q_positions, q_bf16, modes,
-                                         windows, window_scalar, softmax_scale, out_bf16,
+                                         nullptr, windows, window_scalar, softmax_scale, out_bf16,
+                                         static_cast<cudaStream_t>(stream), &launches);
+  cache_set_launches(cache, launches);
+  return e == cudaSuccess ? TRR_OK : TRR_ERR_CUDA;
+}
+
+extern "C" trr_status trr_decode_attn_routed(trr_cache* cache, int32_t layer, int32_t n, const int32_t* seq_ids,
+                                             const int32_t* q_positions, const void* q_bf16, const float* mode_logits,
+                                             const int32_t* windows, int32_t window_scalar, float softmax_scale,
+                                             void* out_bf16, void* stream) {
+  if (!cache) return TRR_ERR_INVALID_ARG;
+  const Layout& l = cache_layout(cache);
+  if (layer < 0 || layer >= l.L || n < 0 || n > l.max_queries) return TRR_ERR_INVALID_ARG;
+  cache_set_launches(cache, 0);
+  if (n == 0) return TRR_OK;
+  if (!seq_ids || !q_positions || !q_bf16 || !mode_logits || !out_bf16) return TRR_ERR_INVALID_ARG;
+  if (((reinterpret_cast<uintptr_t>(q_bf16) | reinterpret_cast<uintptr_t>(out_bf16)) & 15) ||
+      (reinterpret_cast<uintptr_t>(mode_logits) & 3))
+    return TRR_ERR_INVALID_ARG;
+  const LayerArgs a = layer_args(l, cache_views(cache), layer);
+  int launches = 0;
+  const cudaError_t e = launch_attention(l, a, cache_num_sms(cache), n, seq_ids, q_positions, q_bf16, nullptr,
+                                         mode_logits, windows, window_scalar, softmax_scale, out_bf16,
                                          static_cast<cudaStream_t>(stream), &launches);
   cache_set_launches(cache, launches);
   return e == cudaSuccess ? TRR_OK : TRR_ERR_CUDA;
@@ -1927,7 +1957,7 @@ extern "C" trr_status trr_decode_attn_static(trr_cache* cache, int32_t layer, in
   cudaError_t e = cudaGetLastError();
   int launches = 0;
   if (e == cudaSuccess)
-    e = launch_attention(l, a, cache_num_sms(cache), n, seq_ids, q_positions, q_bf16, modes, windows,
+    e = launch_attention(l, a, cache_num_sms(cache), n, seq_ids, q_positions, q_bf16, modes, nullptr, windows,
                          window_scalar, softmax_scale, out_bf16, s, &launches);
   if (e != cudaSuccess) return TRR_ERR_CUDA;
   static_scratch_status_kernel<<<1, 1, 0, s>>>(a.ctrl, cache_ctrl);

@@ -192,6 +192,24 @@ __device__ __forceinline__ int atom_add_acq_rel(int* p, int v) {
   return old;
 }
 
+// The hard decision of one controller head (Sec. 3.8: at inference the router takes
+// the arg max of its logits): the index of the largest of K logits, the first of equal
+// ones; a NaN is never taken, and a row of NaN gives 0.
+template <int K>
+__device__ __forceinline__ int hard_decision(const float* z) {
+  int best = 0;
+  float top = z[0];
+#pragma unroll
+  for (int i = 1; i < K; ++i) {
+    const float v = z[i];
+    if (v > top || (top != top && v == v)) {
+      top = v;
+      best = i;
+    }
+  }
+  return best;
+}
+
 __device__ __forceinline__ void set_status(int32_t* ctrl, int code) {
   atomicCAS(ctrl + kStatus, 0, code);
 }

@@ -39,7 +39,8 @@ class trr_cache_config(ctypes.Structure):
 
 
 EXPORTS = ("trr_cache_required_bytes", "trr_create_cache", "trr_kv_append", "trr_decode_attn",
-           "trr_decode_attn_static", "trr_destroy", "trr_get_status", "trr_reset", "trr_get_region",
+           "trr_decode_attn_static", "trr_route_decisions", "trr_kv_append_routed",
+           "trr_decode_attn_routed", "trr_destroy", "trr_get_status", "trr_reset", "trr_get_region",
            "trr_last_launch_count")
 
 _lib = None
@@ -66,6 +67,9 @@ def load(build_if_missing: bool = False) -> ctypes.CDLL:
     L.trr_kv_append.argtypes = [P, I32, I32, P, P, P, P, P, P, P]
     L.trr_decode_attn.argtypes = [P, I32, I32, P, P, P, P, P, I32, ctypes.c_float, P, P]
     L.trr_decode_attn_static.argtypes = [P, I32, I32, P, P, P, P, P, I32, ctypes.c_float, P, P]
+    L.trr_route_decisions.argtypes = [I32, P, P, P, I32, I32, I32, I32, I32, P, P, P, P, P, P]
+    L.trr_kv_append_routed.argtypes = [P, I32, I32, P, P, P, P, P, P, P]
+    L.trr_decode_attn_routed.argtypes = [P, I32, I32, P, P, P, P, P, I32, ctypes.c_float, P, P]
     L.trr_destroy.argtypes = [P]
     L.trr_get_status.argtypes = [P, P]
     L.trr_reset.argtypes = [P, P]
@@ -159,6 +163,54 @@ def trr_decode_attn_static(cache, layer, seq_ids, q_positions, q, modes, windows
         _dev(out, torch.bfloat16, "out"), _stream(stream)))
 
 
+def _opt(t, dtype, name):
+    return None if t is None else _dev(t, dtype, name)
+
+
+def trr_route_decisions(mode_logits, bit_logits, positions=None, window=1, num_q_heads=1, head_dim=1,
+                        num_kv_heads=1, skip_writes_kv=0, modes=None, bits=None, attn_flops=None,
+                        kv_bits=None, totals=None, stream=None):
+    """Hard decisions of n tokens (and, with positions, their cost) into the given
+    device tensors; ``totals`` (int64[4]) is added to."""
+    n = mode_logits.shape[0] if mode_logits.dim() else 0
+    if mode_logits.numel() != 3 * n or bit_logits.numel() != 4 * n:
+        raise ValueError("mode_logits must be [n][3] and bit_logits [n][4]")
+    for t, k, name in ((modes, n, "modes"), (bits, n, "bits"), (attn_flops, n, "attn_flops"),
+                       (kv_bits, n, "kv_bits"), (positions, n, "positions"), (totals, 4, "totals")):
+        if t is not None and t.numel() != k:
+            raise ValueError(f"{name} must have {k} elements")
+    _check("trr_route_decisions", load().trr_route_decisions(
+        n, _dev(mode_logits, torch.float32, "mode_logits"), _dev(bit_logits, torch.float32, "bit_logits"),
+        _opt(positions, torch.int32, "positions"), int(window), int(num_q_heads), int(head_dim),
+        int(num_kv_heads), int(skip_writes_kv), _opt(modes, torch.uint8, "modes"),
+        _opt(bits, torch.uint8, "bits"), _opt(attn_flops, torch.int64, "attn_flops"),
+        _opt(kv_bits, torch.int64, "kv_bits"), _opt(totals, torch.int64, "totals"), _stream(stream)))
+
+
+def trr_kv_append_routed(cache, layer, seq_ids, positions, k, v, bit_logits, mode_logits, stream=None):
+    n = seq_ids.numel()
+    if bit_logits.numel() != 4 * n or mode_logits.numel() != 3 * n:
+        raise ValueError("bit_logits must be [n][4] and mode_logits [n][3]")
+    _check("trr_kv_append_routed", load().trr_kv_append_routed(
+        cache, layer, n, _dev(seq_ids, torch.int32, "seq_ids"), _dev(positions, torch.int32, "positions"),
+        _dev(k, torch.bfloat16, "k"), _dev(v, torch.bfloat16, "v"),
+        _dev(bit_logits, torch.float32, "bit_logits"), _dev(mode_logits, torch.float32, "mode_logits"),
+        _stream(stream)))
+
+
+def trr_decode_attn_routed(cache, layer, seq_ids, q_positions, q, mode_logits, windows, window_scalar,
+                           softmax_scale, out, stream=None):
+    n = seq_ids.numel()
+    if mode_logits.numel() != 3 * n:
+        raise ValueError("mode_logits must be [n][3]")
+    win = None if windows is None else _dev(windows, torch.int32, "windows")
+    _check("trr_decode_attn_routed", load().trr_decode_attn_routed(
+        cache, layer, n, _dev(seq_ids, torch.int32, "seq_ids"),
+        _dev(q_positions, torch.int32, "q_positions"), _dev(q, torch.bfloat16, "q"),
+        _dev(mode_logits, torch.float32, "mode_logits"), win, int(window_scalar), float(softmax_scale),
+        _dev(out, torch.bfloat16, "out"), _stream(stream)))
+
+
 def trr_destroy(cache):
     _check("trr_destroy", load().trr_destroy(cache))
 
@@ -207,6 +259,17 @@ class Cache:
             out = torch.empty((seq_ids.numel(), self.Hq, self.d), dtype=torch.bfloat16, device=q.device)
         trr_decode_attn(self.handle, layer, seq_ids, q_positions, q, modes, windows, window_scalar,
                         softmax_scale, out, stream)
+        return out
+
+    def append_routed(self, layer, seq_ids, positions, k, v, bit_logits, mode_logits, stream=None):
+        trr_kv_append_routed(self.handle, layer, seq_ids, positions, k, v, bit_logits, mode_logits, stream)
+
+    def decode_attn_routed(self, layer, seq_ids, q_positions, q, mode_logits, windows=None,
+                           window_scalar=0, softmax_scale=0.0, out=None, stream=None):
+        if out is None:
+            out = torch.empty((seq_ids.numel(), self.Hq, self.d), dtype=torch.bfloat16, device=q.device)
+        trr_decode_attn_routed(self.handle, layer, seq_ids, q_positions, q, mode_logits, windows,
+                               window_scalar, softmax_scale, out, stream)
         return out
 
     def status(self, stream=None) -> int:
