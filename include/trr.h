@@ -174,7 +174,7 @@ TRR_API trr_status trr_decode_attn(trr_cache* cache, int32_t layer, int32_t n,
  *   call, such as an engine running inside a fixed, fully reserved memory budget, and
  *   that need more queries per call than the cache's max_queries scratch was sized
  *   for: n is bounded by the array instead of by max_queries.
- *   The call needs 256 + n * Hq * (4 * (1 + ceil(S_cap / 8)) + S_cap * (4*d + 16))
+ *   The call needs 256 + n * Hq * (4 * (1 + ceil(S_cap / 16)) + S_cap * (4*d + 16))
  *   bytes (plus 256-byte rounding per region), with S_cap the most splits per query of
  *   this cache; a call above 32 MiB returns TRR_ERR_OUT_OF_MEMORY and launches nothing.
  *   The first call on a device looks up the array's device address (once per device,

@@ -33,7 +33,7 @@ constexpr int kItemMaxPages = 28;
 
 // Split partials are merged in groups of this many (then the groups): a query with
 // ns splits per head has 1 + ceil(ns / kMergeGroup) arrival counters per head.
-constexpr int kMergeGroup = 8;
+constexpr int kMergeGroup = 16;
 
 // Byte layout of one cache (see include/trr.h for the documented part).
 struct Layout {
