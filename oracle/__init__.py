@@ -93,10 +93,11 @@ class OracleCache:
 
     def __init__(self, num_layers, max_seqs, num_q_heads, num_kv_heads, head_dim,
                  group_size, page_size, max_context, pages_per_class,
-                 skip_writes_kv=0, no_pool=False):
+                 skip_writes_kv=0, no_pool=False, head_modes=0):
         cfg = np.array([num_layers, max_seqs, num_q_heads, num_kv_heads, head_dim, group_size,
                         page_size, max_context, *pages_per_class, skip_writes_kv,
-                        int(no_pool)], dtype=np.int32)
+                        int(no_pool), int(head_modes)], dtype=np.int32)
+        self.head_modes = int(head_modes)
         self.Hq, self.Hkv, self.d = num_q_heads, num_kv_heads, head_dim
         self.L, self.S, self.P, self.max_context = num_layers, max_seqs, page_size, max_context
         self._h = ctypes.c_void_p()
@@ -118,6 +119,7 @@ class OracleCache:
         bits, modes = _c(bits, np.uint8), _c(modes, np.uint8)
         n = seq_ids.shape[0]
         assert k.size == n * self.Hkv * self.d and v.size == k.size
+        assert modes.size == n * (self.Hq if self.head_modes else 1)
         return lib().orc_append(self._h, layer, n, _ptr(seq_ids), _ptr(positions), _ptr(k),
                                 _ptr(v), _ptr(bits), _ptr(modes))
 
@@ -129,6 +131,7 @@ class OracleCache:
         win = None if windows is None else _c(windows, np.int32)
         n = seq_ids.shape[0]
         assert q.size == n * self.Hq * self.d
+        assert modes.size == n * (self.Hq if self.head_modes else 1)
         out = np.zeros((n, self.Hq, self.d), dtype=np.float64)
         st = lib().orc_decode_attn(self._h, layer, n, _ptr(seq_ids), _ptr(q_positions), _ptr(q),
                                    _ptr(modes), _ptr(win), int(window_scalar), float(scale),
@@ -156,8 +159,13 @@ class OracleCache:
     def page_bytes(self, c):
         return self.layout(5 + c)
 
+    @property
+    def mask_bytes(self):
+        return self.layout(9)
+
     def dequant_token(self, layer, seq, pos, kv_head):
-        """(class index or -1, k float64[d], v float64[d]) of a stored token."""
+        """(class index or -1, k float64[d], v float64[d]) of a stored token; -1 also when
+        (with head_modes) the token does not store KV head kv_head."""
         k = np.zeros(self.d, dtype=np.float64)
         v = np.zeros(self.d, dtype=np.float64)
         c = lib().orc_dequant_token(self._h, layer, seq, pos, kv_head, _ptr(k), _ptr(v))

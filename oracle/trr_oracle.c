@@ -47,7 +47,7 @@
 static const int BITS_OF_CLASS[4] = {2, 4, 8, 16};
 
 typedef struct orc_cache {
-  int L, S, Hq, Hkv, d, G, P, maxctx, skip_writes_kv, no_pool;
+  int L, S, Hq, Hkv, d, G, P, maxctx, skip_writes_kv, no_pool, head_modes;
   int cap[4];
   int MP, W32;
   int32_t* last_pos;   /* [L][S] */
@@ -57,7 +57,7 @@ typedef struct orc_cache {
   int32_t* page_first; /* [L][S][4][MP] */
   int32_t* page_last;  /* [L][S][4][MP] */
   int32_t next_page[4];
-  int64_t hdr, tokb[4], slice[4], page_bytes[4];
+  int64_t hdr, tokb[4], slice[4], maskb, page_bytes[4];
   uint8_t* pool[4];
 } orc_cache;
 
@@ -189,8 +189,42 @@ static uint8_t* page_ptr(const orc_cache* o, int c, int id) {
   return o->pool[c] + (int64_t)id * o->page_bytes[c];
 }
 
-/* cfg: L, S, Hq, Hkv, d, G, P, max_context, cap[4], skip_writes_kv, no_pool.
- * With no_pool = 1 only metadata and nothing of the page bytes is kept. */
+/* Mode of query head h of entry i (modes are [n] or, with head_modes, [n][Hq]). */
+static int mode_of(const orc_cache* o, const uint8_t* modes, int i, int h) {
+  return o->head_modes ? modes[(int64_t)i * o->Hq + h] : modes[i];
+}
+
+/* Whether entry i stores KV for KV head j: always when skip tokens store KV, otherwise
+ * when one of the query heads reading KV head j (h / (Hq / Hkv) = j) is not skip. */
+static int head_stores(const orc_cache* o, const uint8_t* modes, int i, int j) {
+  int g = o->Hq / o->Hkv, h;
+  if (o->skip_writes_kv) return 1;
+  for (h = j * g; h < (j + 1) * g; h++)
+    if (mode_of(o, modes, i, h) != 0) return 1;
+  return 0;
+}
+
+/* Whether entry i takes a slot: some KV head of it is stored. */
+static int entry_stores(const orc_cache* o, const uint8_t* modes, int i) {
+  int j;
+  for (j = 0; j < o->Hkv; j++)
+    if (head_stores(o, modes, i, j)) return 1;
+  return 0;
+}
+
+/* With head_modes, the bit of `slot` in KV head j's 64-bit presence mask, stored
+ * little-endian after the page's KV slices. */
+static int slot_present(const orc_cache* o, const uint8_t* page, int c, int slot, int j) {
+  uint64_t m;
+  if (!o->head_modes) return 1;
+  memcpy(&m, page + o->hdr + o->Hkv * o->slice[c] + 8 * (int64_t)j, 8);
+  return (int)((m >> slot) & 1);
+}
+
+/* cfg: L, S, Hq, Hkv, d, G, P, max_context, cap[4], skip_writes_kv, no_pool, head_modes.
+ * With no_pool = 1 only metadata and nothing of the page bytes is kept.  head_modes = 1:
+ * attention modes are chosen per query head (Sec. 3.2(A): per head by default), modes
+ * arrays are [n][Hq], and every page ends with one 64-bit presence mask per KV head. */
 int orc_create(const int32_t* cfg, orc_cache** out) {
   int c;
   *out = NULL;
@@ -202,21 +236,24 @@ int orc_create(const int32_t* cfg, orc_cache** out) {
   for (c = 0; c < 4; c++) o->cap[c] = cfg[8 + c];
   o->skip_writes_kv = cfg[12];
   o->no_pool = cfg[13];
+  o->head_modes = cfg[14];
   if (o->L < 1 || o->S < 1 || o->Hkv < 1 || o->Hq < o->Hkv || o->Hq % o->Hkv ||
       (o->d != 64 && o->d != 128) || (o->G != 32 && o->G != 64 && o->G != 128) ||
       o->G > o->d || (o->P != 16 && o->P != 32 && o->P != 64) || o->maxctx < 1 ||
-      o->cap[0] < 0 || o->cap[1] < 0 || o->cap[2] < 0 || o->cap[3] < 0) {
+      o->cap[0] < 0 || o->cap[1] < 0 || o->cap[2] < 0 || o->cap[3] < 0 ||
+      (o->head_modes != 0 && o->head_modes != 1)) {
     free(o);
     return ORC_UNSUPPORTED;
   }
   o->MP = (o->maxctx + o->P - 1) / o->P;
   o->W32 = (o->maxctx + 31) / 32;
   o->hdr = roundup(4 * (int64_t)o->P, 128);
+  o->maskb = o->head_modes ? roundup(8 * (int64_t)o->Hkv, 16) : 0;
   for (c = 0; c < 4; c++) {
     int b = BITS_OF_CLASS[c];
     o->tokb[c] = b < 16 ? 2 * (o->d * b / 8) + 2 * (o->d / o->G) * 4 : 4 * o->d;
     o->slice[c] = o->P * o->tokb[c];
-    o->page_bytes[c] = roundup(o->hdr + o->Hkv * o->slice[c], 128);
+    o->page_bytes[c] = roundup(o->hdr + o->Hkv * o->slice[c] + o->maskb, 128);
   }
   int64_t nls = (int64_t)o->L * o->S;
   o->last_pos = (int32_t*)malloc(sizeof(int32_t) * nls);
@@ -258,16 +295,18 @@ void orc_destroy(orc_cache* o) {
 /* Checks of one entry against the running state, in the documented order.
  * tmp_last / tmp_ntok / tmp_next describe the cache as if earlier entries of this
  * call had been applied. */
-static int check_entry(const orc_cache* o, int seq, int pos, int bits, int mode,
-                       const int32_t* tmp_last, const int32_t* tmp_ntok,
+static int check_entry(const orc_cache* o, int seq, int pos, int bits, const uint8_t* modes,
+                       int i, const int32_t* tmp_last, const int32_t* tmp_ntok,
                        const int32_t* tmp_next) {
+  int h;
   if (seq < 0 || seq >= o->S) return ORC_INVALID_ARG;
   int c = class_of_bits(bits);
   if (c < 0) return ORC_INVALID_ARG;
-  if (mode < 0 || mode > 2) return ORC_INVALID_ARG;
+  for (h = 0; h < (o->head_modes ? o->Hq : 1); h++)
+    if (mode_of(o, modes, i, h) > 2) return ORC_INVALID_ARG;
   if (pos < 0 || pos >= o->maxctx) return ORC_BAD_POSITION;
   if (pos <= tmp_last[seq]) return ORC_BAD_POSITION;
-  if (mode == 0 && !o->skip_writes_kv) return ORC_OK;
+  if (!entry_stores(o, modes, i)) return ORC_OK;
   if (tmp_ntok[seq * 4 + c] % o->P == 0 && tmp_next[c] >= o->cap[c]) return ORC_OUT_OF_PAGES;
   return ORC_OK;
 }
@@ -313,11 +352,11 @@ int orc_append(orc_cache* o, int layer, int n, const int32_t* seq_ids,
   memcpy(tmp_ntok, o->ntok + idx_lsc(o, layer, 0, 0), sizeof(int32_t) * o->S * 4);
   memcpy(tmp_next, o->next_page, sizeof(tmp_next));
   for (i = 0; i < n; i++) {
-    int e = check_entry(o, seq_ids[i], positions[i], bits[i], modes[i], tmp_last,
+    int e = check_entry(o, seq_ids[i], positions[i], bits[i], modes, i, tmp_last,
                         tmp_ntok, tmp_next);
     if (e != ORC_OK) { free(tmp_last); free(tmp_ntok); return e; }
     tmp_last[seq_ids[i]] = positions[i];
-    if (modes[i] == 0 && !o->skip_writes_kv) continue;
+    if (!entry_stores(o, modes, i)) continue;
     c = class_of_bits(bits[i]);
     if (tmp_ntok[seq_ids[i] * 4 + c] % o->P == 0) tmp_next[c]++;
     tmp_ntok[seq_ids[i] * 4 + c]++;
@@ -330,7 +369,7 @@ int orc_append(orc_cache* o, int layer, int n, const int32_t* seq_ids,
   for (i = 0; i < n; i++) {
     int s = seq_ids[i], pos = positions[i];
     o->last_pos[idx_ls(o, layer, s)] = pos;
-    if (modes[i] == 0 && !o->skip_writes_kv) continue; /* skip: no KV entry */
+    if (!entry_stores(o, modes, i)) continue; /* skip: no KV entry */
     c = class_of_bits(bits[i]);
     int32_t* nt = &o->ntok[idx_lsc(o, layer, s, c)];
     int kidx = *nt / o->P, slot = *nt % o->P;
@@ -349,6 +388,16 @@ int orc_append(orc_cache* o, int layer, int n, const int32_t* seq_ids,
     for (h = 0; h < o->Hkv; h++)
       write_row(o, page, c, slot, h, k + i * row + (int64_t)h * o->d,
                 v + i * row + (int64_t)h * o->d, &bad);
+    /* head_modes: every KV head's row is written; the heads that store it get their
+     * presence bit (a new page starts with every bit clear) */
+    for (h = 0; h < o->Hkv && o->head_modes; h++) {
+      uint8_t* mw = page + o->hdr + o->Hkv * o->slice[c] + 8 * (int64_t)h;
+      uint64_t m;
+      memcpy(&m, mw, 8);
+      if (slot == 0) m = 0;
+      if (head_stores(o, modes, i, h)) m |= (uint64_t)1 << slot;
+      memcpy(mw, &m, 8);
+    }
   }
   return bad ? ORC_BAD_VALUE : ORC_OK;
 }
@@ -409,6 +458,7 @@ int orc_dequant_token(const orc_cache* o, int layer, int s, int pos, int h, doub
       int fill = tokens_in_page(o, layer, s, c, kidx);
       for (slot = 0; slot < fill; slot++)
         if (slot_position(page, slot) == pos) {
+          if (!slot_present(o, page, c, slot, h)) return -1;
           dequant_slot(o, page, c, slot, h, kout, vout);
           return c;
         }
@@ -449,19 +499,24 @@ int orc_decode_attn(const orc_cache* o, int layer, int n, const int32_t* seq_ids
   }
   for (i = 0; i < n; i++) {
     double* orow = out + (int64_t)i * o->Hq * d;
-    int s = seq_ids[i], t = q_positions[i], mode = modes[i];
+    int s = seq_ids[i], t = q_positions[i];
     int w = windows ? windows[i] : window_scalar;
-    int err = ORC_OK;
-    if (s < 0 || s >= o->S || mode < 0 || mode > 2) err = ORC_INVALID_ARG;
-    else if (t < 0 || t >= o->maxctx) err = ORC_BAD_POSITION;
-    else if (mode == 1 && w < 1) err = ORC_INVALID_ARG;
+    int err = ORC_OK, any_local = 0, any_read = 0;
+    for (h = 0; h < o->Hq; h++) {
+      int m = mode_of(o, modes, i, h);
+      if (m > 2) err = ORC_INVALID_ARG;
+      any_local |= m == 1;
+      any_read |= m != 0;
+    }
+    if (s < 0 || s >= o->S) err = ORC_INVALID_ARG;
+    else if (err == ORC_OK && (t < 0 || t >= o->maxctx)) err = ORC_BAD_POSITION;
+    else if (err == ORC_OK && any_local && w < 1) err = ORC_INVALID_ARG;
     for (j = 0; j < o->Hq * d; j++) orow[j] = 0.0;
     if (err != ORC_OK) {
       if (status == ORC_OK) status = err;
       continue;
     }
-    if (mode == 0) continue; /* Attn^skip = 0 */
-    int lo = mode == 2 ? 0 : (t - w + 1 > 0 ? t - w + 1 : 0);
+    if (!any_read) continue; /* Attn^skip = 0 */
     /* the pages of this (layer, seq), all classes */
     int nref = 0, c, kidx;
     for (c = 0; c < 4; c++) {
@@ -482,7 +537,9 @@ int orc_decode_attn(const orc_cache* o, int layer, int n, const int32_t* seq_ids
       }
     }
     for (h = 0; h < o->Hq; h++) {
-      int kvh = h / group, r, nk = 0, slot;
+      int kvh = h / group, r, nk = 0, slot, mode = mode_of(o, modes, i, h);
+      if (mode == 0) continue; /* Attn^skip = 0 for this head */
+      int lo = mode == 2 ? 0 : (t - w + 1 > 0 ? t - w + 1 : 0);
       for (j = 0; j < d; j++) qd[j] = orc_bf16_to_double(q[((int64_t)i * o->Hq + h) * d + j]);
       /* pass 1: scores of the stored keys lo <= j <= t, and their maximum */
       double mx = -INFINITY;
@@ -493,7 +550,7 @@ int orc_decode_attn(const orc_cache* o, int layer, int n, const int32_t* seq_ids
         for (slot = 0; slot < fill; slot++) {
           int sl = order_seed ? fill - 1 - slot : slot;
           int32_t pos = slot_position(page, sl);
-          if (pos < lo || pos > t) continue;
+          if (pos < lo || pos > t || !slot_present(o, page, cc, sl, kvh)) continue;
           dequant_slot(o, page, cc, sl, kvh, kv, kv + d);
           double dot = 0;
           for (j = 0; j < d; j++) dot += qd[j] * kv[j];
@@ -514,7 +571,7 @@ int orc_decode_attn(const orc_cache* o, int layer, int n, const int32_t* seq_ids
         for (slot = 0; slot < fill; slot++) {
           int sl = order_seed ? fill - 1 - slot : slot;
           int32_t pos = slot_position(page, sl);
-          if (pos < lo || pos > t) continue;
+          if (pos < lo || pos > t || !slot_present(o, page, cc, sl, kvh)) continue;
           dequant_slot(o, page, cc, sl, kvh, kv, kv + d);
           double p = exp(score[nk] - mx);
           denom += p;
@@ -552,11 +609,12 @@ int64_t orc_region(orc_cache* o, int id, void** ptr) {
 }
 
 /* Layout sizes: which = 0 header bytes, 1..4 slice bytes of class 0..3,
- * 5..8 page bytes of class 0..3. */
+ * 5..8 page bytes of class 0..3, 9 bytes of a page's presence masks (head_modes). */
 int64_t orc_layout(const orc_cache* o, int which) {
   if (which == 0) return o->hdr;
   if (which >= 1 && which <= 4) return o->slice[which - 1];
   if (which >= 5 && which <= 8) return o->page_bytes[which - 5];
+  if (which == 9) return o->maskb;
   return -1;
 }
 
