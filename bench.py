@@ -71,7 +71,7 @@ class Accounting:
         m = int(modes_row[t])
         qo = 2 * self.Hq * self.d
         if m == 0:
-            return qo // 2, 0, 0                      # only the zero O row is written
+            return qo, 0, 0                           # only the zero O row is written
         lo = 0 if m == 2 else max(0, t - self.window + 1)
         stored = modes_row[:t + 1] != 0
         b_row = bits_row[:t + 1]
@@ -87,6 +87,44 @@ class Accounting:
             total += n_in * (int(self.tokb[c]) * self.Hkv + 4)
         total += 4 * pages
         return total, keys, pages
+
+    def query_heads(self, bits_row, modes_rows, t):
+        """(bytes, attended keys, pages) of one query with per-head modes (modes_rows
+        [T][Hq]): per KV head, the payload of the keys that store it in the widest range
+        of its reading heads; once per key in the query's widest range its slot position,
+        per page its page-table entry and the presence masks of the KV heads read; Q rows
+        of the heads that read, every O row.  Keys are counted per KV head / Hkv."""
+        mrow = modes_rows[t]
+        g = self.Hq // self.Hkv
+        qo = 2 * self.Hq * self.d
+        if not mrow.any():
+            return qo, 0, 0
+        lo_q = 0 if (mrow == 2).any() else max(0, t - self.window + 1)
+        b_row = bits_row[:t + 1]
+        stored = (modes_rows[:t + 1] != 0).reshape(t + 1, self.Hkv, g).any(2)  # [t+1][Hkv]
+        took = stored.any(1)
+        total = qo + 2 * self.d * int(np.count_nonzero(mrow))
+        keys = pages = nkv = 0
+        for j in range(self.Hkv):
+            mj = mrow[j * g:(j + 1) * g]
+            if not mj.any():
+                continue
+            nkv += 1
+            lo = 0 if (mj == 2).any() else max(0, t - self.window + 1)
+            for c, b in enumerate(BITS):
+                n_in = int(np.count_nonzero(stored[lo:, j] & (b_row[lo:] == b)))
+                keys += n_in
+                total += n_in * int(self.tokb[c])
+        for c, b in enumerate(BITS):
+            sel = took & (b_row == b)
+            before = int(np.count_nonzero(sel[:lo_q]))
+            n_in = int(np.count_nonzero(sel[lo_q:]))
+            if n_in:
+                i0, i1 = before, before + n_in
+                pages += (i1 - 1) // self.P - i0 // self.P + 1
+            total += 4 * n_in
+        total += pages * (4 + 8 * nkv)
+        return total, keys / self.Hkv, pages
 
 
 # ------------------------------------------------------------------ clocks (NVML) --
@@ -268,8 +306,10 @@ class Bench:
         self.L, self.B, self.Hq, self.Hkv, self.d, self.G = (
             s.num_layers, s.batch, s.num_q_heads, s.num_kv_heads, s.head_dim, s.group_size)
         self.window = s.window
+        self.head_modes = int(getattr(args, "head_modes", False))
         self.e2e_warm, self.e2e_steps = 2, 2 * min(args.steps, 10)
-        self.routed_warm, self.routed_steps = 2, min(args.steps, 10)
+        # the routed step decides per token: not run with per-head modes
+        self.routed_warm, self.routed_steps = (0, 0) if self.head_modes else (2, min(args.steps, 10))
         self.total_steps = (args.warmup + 2 * args.steps + self.e2e_warm + self.e2e_steps + self.routed_warm +
                             self.routed_steps)
         self.grow = 32                                   # tokens a sequence may grow
@@ -284,10 +324,12 @@ class Bench:
     def maps(self, layer, r):
         wl = self.wl
         bits = np.empty((self.B, self.maxctx), dtype=np.uint8)
-        modes = np.empty((self.B, self.maxctx), dtype=np.uint8)
+        shape = (self.B, self.maxctx, self.Hq) if self.head_modes else (self.B, self.maxctx)
+        modes = np.empty(shape, dtype=np.uint8)
         spec = self.spec.with_(contexts=("fixed", self.maxctx))
+        draw = wl.head_policy if self.head_modes else wl.policy
         for s in range(self.B):
-            bits[s], modes[s] = wl.policy(spec, layer, r * self.B + s, self.maxctx)
+            bits[s], modes[s] = draw(spec, layer, r * self.B + s, self.maxctx)
         return bits, modes
 
     def setup(self):
@@ -300,12 +342,12 @@ class Bench:
             for r in range(R):
                 bits, modes = self.all_maps[l][r]
                 for s in range(B):
-                    stored = modes[s] != 0
+                    stored = (modes[s] != 0).any(-1) if self.head_modes else modes[s] != 0
                     for c, b in enumerate(BITS):
                         caps[c] += -(-int(np.count_nonzero(stored & (bits[s] == b))) // self.P) + 1
         self.cache = trr.Cache(L, S, self.Hq, self.Hkv, self.d, self.G, self.P, self.maxctx,
                                [int(c) for c in caps], max_append=1024, max_queries=max(B, 64),
-                               split_bytes=self.args.split_bytes)
+                               split_bytes=self.args.split_bytes, head_modes=self.head_modes)
         # prebuild every sequence's context (untimed), K/V drawn on the device
         gen = torch.Generator(device=self.dev)
         self.prebuild_calls = 0
@@ -366,18 +408,20 @@ class Bench:
             k, v = self._kv(self.B, gen, chl)
             q = torch.randn((self.B, self.Hq, self.d), generator=gen, device=self.dev).to(torch.bfloat16)
             for s in range(self.B):
-                nb, nk, _ = self.acct.query(bits[s], modes[s], int(pos[s]))
+                acct = self.acct.query_heads if self.head_modes else self.acct.query
+                nb, nk, _ = acct(bits[s], modes[s], int(pos[s]))
                 nbytes += nb
                 keys += nk
             # router logits whose arg max is the seeded decision (the routed step)
             ml = torch.rand((self.B, 3), generator=gen, device=self.dev) - 2.0
             bl = torch.rand((self.B, 4), generator=gen, device=self.dev) - 2.0
-            ml[torch.arange(self.B, device=self.dev), torch.from_numpy(m.astype(np.int64)).to(self.dev)] = 1.0
+            if not self.head_modes:
+                ml[torch.arange(self.B, device=self.dev), torch.from_numpy(m.astype(np.int64)).to(self.dev)] = 1.0
             bcls = np.array([BITS.index(int(x)) for x in b], dtype=np.int64)
             bl[torch.arange(self.B, device=self.dev), torch.from_numpy(bcls).to(self.dev)] = 1.0
             layers.append(dict(
                 seqs=torch.from_numpy(seqs).to(self.dev), pos=torch.from_numpy(pos).to(self.dev),
-                bits=torch.from_numpy(b).to(self.dev), modes=torch.from_numpy(m).to(self.dev),
+                bits=torch.from_numpy(b).to(self.dev), modes=torch.from_numpy(np.ascontiguousarray(m)).to(self.dev),
                 k=k, v=v, q=q, ml=ml.contiguous(), bl=bl.contiguous(),
                 out=torch.empty((self.B, self.Hq, self.d), dtype=torch.bfloat16, device=self.dev)))
         attn_bytes_per_layer = nbytes / self.L
@@ -664,7 +708,7 @@ def run_gpu(args):
     eager_ms = b0.elapsed_time(b1)
     eager_bytes = sum(bench.steps[e0 + j]["bytes"] for j in range(half, ne))
     eager_ms, eager_bytes = across_ranks(dist, "cuda", eager_ms, eager_bytes)
-    routed = run_routed(bench, dist, e0 + bench.e2e_warm + bench.e2e_steps)
+    routed = None if bench.head_modes else run_routed(bench, dist, e0 + bench.e2e_warm + bench.e2e_steps)
     status = bench.cache.status()
     if status != 0:
         raise RuntimeError(f"device status {status} after the run")
@@ -676,7 +720,7 @@ def run_gpu(args):
     value = job_bytes / (ms * 1e-3) / 1e9
     result = None
     if rank == 0:
-        cpu = cpu_baseline(bench) if (world == 1 and not args.no_cpu_baseline) else None
+        cpu = cpu_baseline(bench) if (world == 1 and not args.no_cpu_baseline and not bench.head_modes) else None
         result = {
             "metric": METRIC, "value": round(value, 2), "unit": UNIT, "n_gpus": world,
             "steps": K, "warmup": W, "ms_per_step": round(ms / K, 5), "higher_is_better": True,
@@ -686,6 +730,8 @@ def run_gpu(args):
                             f"batch {bench.B}/GPU, contexts {describe_ctx(bench)}, window {bench.window}, "
                             f"group {bench.G}, page {bench.P}",
                 "kv_storage": "per-token 2/4/8-bit codes + fp16 scale/zero, or bf16; fp32 accumulation",
+                "modes": "per (token, query head), presence mask per KV head" if bench.head_modes
+                         else "per token",
                 "global_batch": bench.B * world, "replicas": bench.R,
                 "l2": "inputs larger than L2: every step reads its replica's "
                       f"{rank_bytes / K / 1e6:.0f} MB, replicas rotate",
@@ -704,12 +750,14 @@ def run_gpu(args):
                     "eager_how": "the same steps called one by one from Python, no graph (host-launch bound)"},
             "roofline": {"bound": "hbm", "achieved": round(achieved, 2), "peak": peak,
                          "unit": "GB/s", "frac": round(achieved / peak, 4),
-                         "traffic": ncu_traffic(args.workload), "peak_kind": peak_kind,
+                         "traffic": None if bench.head_modes else ncu_traffic(args.workload),
+                         "peak_kind": peak_kind,
                          "kernel": "trr_decode_attn call (attn_kernel, one launch)",
                          "bytes_per_call": round(avg_bytes), "us_per_call": round(avg_ms * 1e3, 3)},
             "clocks": clocks.summary(),
-            "routed": routed,
         }
+        if routed is not None:
+            result["routed"] = routed
         if cpu is not None:
             result["cpu_baseline"] = cpu
     if dist:
@@ -829,6 +877,9 @@ def main():
                     help="tokens per cache page (0: 32)")
     ap.add_argument("--split-bytes", type=int, default=0,
                     help="target KV bytes per split-K work item (0: the library default)")
+    ap.add_argument("--head-modes", action="store_true",
+                    help="a mode per (token, query head), drawn from the workload's mode mix "
+                         "(Sec. 3.2(A)); no routed step and no CPU baseline")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")

@@ -46,7 +46,8 @@
  *     HDR        = roundup(4 * P, 128)           header: int32 positions[P]
  *     TOKB(b)    = 2*(d*b/8) + 2*(d/G)*4   (b < 16)  |  4*d   (b = 16)
  *     SLICE(b)   = P * TOKB(b)                  one KV head of one page
- *     PAGE_BYTES = roundup(HDR + Hkv * SLICE(b), 128)
+ *     MASKB      = roundup(8 * Hkv, 16) with head_modes, else 0
+ *     PAGE_BYTES = roundup(HDR + Hkv * SLICE(b) + MASKB, 128)
  *     head h starts at HDR + h * SLICE(b); inside it, for b < 16:
  *       K codes [P][d*b/8] | V codes [P][d*b/8] | K sz [P][d/G][2] | V sz [P][d/G][2]
  *     where sz = (scale, zero) as IEEE binary16, and for b = 16:
@@ -55,6 +56,9 @@
  *   least significant bits first (2-bit codes 1,2,3,0 -> byte 0x39).
  *   Page allocation: entries are taken in array order; an entry of class c whose
  *   (layer, seq) has ntok % P == 0 opens page next_page[c]++ .
+ *   Per-head modes (head_modes = 1): after the slices, at HDR + Hkv * SLICE(b), one
+ *   little-endian uint64 per KV head: bit `slot` set <=> the token in that slot stores
+ *   that KV head.  A page starts with every bit clear when its slot 0 is written.
  */
 #ifndef TRR_H
 #define TRR_H
@@ -100,6 +104,9 @@ typedef struct trr_cache_config {
   int32_t max_queries;     /* largest n accepted by trr_decode_attn */
   int32_t split_bytes;     /* least KV bytes (of 8-bit tokens) per split-K work item; 0 = 24576 */
   int32_t skip_writes_kv;  /* 0: a skip token stores no KV (default); 1: it stores KV */
+  int32_t head_modes;      /* 0: one mode per token, modes[n] (default); 1: one mode per
+                              query head, modes[n][Hq] (Sec. 3.2(A): per head by default),
+                              with a presence mask per KV head in every page */
   void* pool;              /* device memory of >= trr_cache_required_bytes, or NULL */
   uint64_t pool_bytes;     /* size of `pool` (ignored when pool is NULL) */
 } trr_cache_config;
@@ -122,6 +129,11 @@ TRR_API trr_status trr_create_cache(const trr_cache_config* cfg, trr_cache** out
  *   seq_ids[i] at `layer`, with K/V rows k[i][Hkv][d], v[i][Hkv][d] (bf16, device,
  *   contiguous), bit-width bits[i] in {2,4,8,16} and attention mode modes[i].
  *   A skip token (modes[i] == 0) stores nothing unless skip_writes_kv == 1.
+ *   With head_modes, modes is [n][Hq] (uint8, device): KV head j of entry i is stored
+ *   when a query head reading it (h / (Hq / Hkv) == j) has a mode other than skip, or
+ *   always with skip_writes_kv == 1; an entry none of whose KV heads is stored takes no
+ *   slot.  An entry that takes a slot has every KV head's row written, and its slot's
+ *   bit set in the presence mask of each KV head it stores.
  *   For b < 16 each group of G consecutive elements of a head vector is stored as
  *     z = fp16(min x),  s = fp16(fl32(fl32(max x - min x) / (2^b - 1))),
  *     c_j = clamp(rne((x_j - z) / s), 0, 2^b - 1)   (c_j = 0 when s == 0)
@@ -148,6 +160,9 @@ TRR_API trr_status trr_kv_append(trr_cache* cache, int32_t layer, int32_t n,
  *     local: softmax attention over the stored tokens j with t-w+1 <= j <= t,
  *            w = windows[i] (or window_scalar when windows == NULL), w >= 1
  *     full : softmax attention over the stored tokens j <= t.
+ *   With head_modes, modes is [n][Hq] and each query head h runs its own mode over the
+ *   tokens that store its KV head (presence bit set); the window check applies when any
+ *   head is local, and a mode value outside {0, 1, 2} in any head fails the query.
  *   Query head h reads KV head h / (Hq / Hkv).  Scores are softmax_scale * q.k
  *   (softmax_scale <= 0 means 1/sqrt(d)) with K/V dequantised as z + c*s; fp32
  *   accumulation, bf16 (round-to-nearest-even) output out[i][Hq][d] (device).
@@ -222,7 +237,8 @@ TRR_API trr_status trr_route_decisions(int32_t n, const float* mode_logits, cons
  * bit_logits[n][4] (b = 2, 4, 8, 16) and mode_logits[n][3] (skip, local, full), fp32,
  * device, 4-byte aligned.  Otherwise the same arguments, results and error contract as
  * trr_kv_append (the logits, like the other inputs, may be read while the previous
- * kernel of the stream is still running). */
+ * kernel of the stream is still running).  Decisions are per token: a cache with
+ * head_modes returns TRR_ERR_UNSUPPORTED. */
 TRR_API trr_status trr_kv_append_routed(trr_cache* cache, int32_t layer, int32_t n,
                                         const int32_t* seq_ids, const int32_t* positions,
                                         const void* k_bf16, const void* v_bf16,
@@ -231,7 +247,8 @@ TRR_API trr_status trr_kv_append_routed(trr_cache* cache, int32_t layer, int32_t
 
 /* trr_decode_attn with each query's mode decided in the attention's planning step from
  * mode_logits[n][3] (skip, local, full; fp32, device, 4-byte aligned), exactly as
- * trr_route_decisions decides.  Otherwise the same as trr_decode_attn. */
+ * trr_route_decisions decides.  Otherwise the same as trr_decode_attn.  Decisions are
+ * per token: a cache with head_modes returns TRR_ERR_UNSUPPORTED. */
 TRR_API trr_status trr_decode_attn_routed(trr_cache* cache, int32_t layer, int32_t n,
                                           const int32_t* seq_ids, const int32_t* q_positions,
                                           const void* q_bf16, const float* mode_logits,

@@ -20,9 +20,33 @@ __device__ __forceinline__ int class_of_bits(int b) {
 }
 
 // An entry's attention mode and bit-width: the caller's, or the hard decisions of its
-// router logits (Sec. 3.8), taken here in the append's own planning step.
-__device__ __forceinline__ int entry_mode(const uint8_t* modes, const float* mode_logits, int e) {
-  return mode_logits ? hard_decision<3>(mode_logits + 3 * e) : modes[e];
+// router logits (Sec. 3.8), taken here in the append's own planning step.  With
+// per-head modes (modes[n][Hq]) the largest of the entry's head modes: skip only when
+// every head skips, above full when any head's value is not a mode.
+__device__ __forceinline__ int entry_mode(const LayerArgs& a, const uint8_t* modes, const float* mode_logits, int e) {
+  if (mode_logits) return hard_decision<3>(mode_logits + 3 * e);
+  if (!a.head_modes) return modes[e];
+  int m = 0;
+  const uint8_t* row = modes + static_cast<int64_t>(e) * a.Hq;
+  for (int h = 0; h < a.Hq; ++h) m = max(m, static_cast<int>(row[h]));
+  return m;
+}
+
+// Per-head modes: whether entry e stores KV head j, i.e. whether a query head reading it
+// (h / (Hq / Hkv) == j) does not skip, or skip tokens store KV.
+__device__ __forceinline__ bool head_stores(const LayerArgs& a, const uint8_t* modes, int e, int j) {
+  if (a.skip_writes_kv) return true;
+  const int g = a.Hq / a.Hkv;
+  const uint8_t* row = modes + static_cast<int64_t>(e) * a.Hq + j * g;
+  for (int h = 0; h < g; ++h)
+    if (row[h] != TRR_MODE_SKIP) return true;
+  return false;
+}
+
+// Per-head modes: the page's presence masks, one uint64 per KV head after its slices.
+__device__ __forceinline__ unsigned long long* page_masks(const LayerArgs& a, int c, int pid) {
+  return reinterpret_cast<unsigned long long*>(a.pool[c] + static_cast<int64_t>(pid) * a.page_bytes[c] + a.hdr +
+                                               static_cast<int64_t>(a.Hkv) * a.slice[c]);
 }
 __device__ __forceinline__ int entry_bits(const uint8_t* bits, const float* bit_logits, int e) {
   return bit_logits ? 2 << hard_decision<4>(bit_logits + 4 * e) : bits[e];
@@ -50,7 +74,7 @@ __global__ void __launch_bounds__(1024) append_plan_kernel(LayerArgs a, int n, c
   if (act) {
     seq = seq_ids[e];
     pos = positions[e];
-    const int m = entry_mode(modes, mode_logits, e);
+    const int m = entry_mode(a, modes, mode_logits, e);
     if (seq < 0 || seq >= a.S) {
       err = TRR_ERR_INVALID_ARG;
     } else {
@@ -116,6 +140,10 @@ __global__ void __launch_bounds__(1024) append_plan_kernel(LayerArgs a, int n, c
     a.pt[row] = pid;
     a.pfirst[row] = pos;
     atomicAdd(&s_nopen[c], 1);
+    if (a.head_modes) {  // a new page starts with every presence bit clear
+      unsigned long long* mw = page_masks(a, c, pid);
+      for (int j = 0; j < a.Hkv; ++j) mw[j] = 0ull;
+    }
   }
   __syncthreads();
   if (act) {
@@ -132,6 +160,11 @@ __global__ void __launch_bounds__(1024) append_plan_kernel(LayerArgs a, int n, c
       }
       reinterpret_cast<int32_t*>(a.pool[c] + pid * a.page_bytes[c])[slot] = pos;
       atomicOr(&a.presence[static_cast<int64_t>(seq) * a.W32 + pos / 32], 1u << (pos % 32));
+      if (a.head_modes) {  // the slot's bit for every KV head the entry stores
+        unsigned long long* mw = page_masks(a, c, pid);
+        for (int j = 0; j < a.Hkv; ++j)
+          if (head_stores(a, modes, e, j)) atomicOr(mw + j, 1ull << slot);
+      }
     }
     a.aplan[e] = p;
     if (!later_seq) a.last_pos[seq] = pos;
@@ -352,7 +385,7 @@ __global__ void __launch_bounds__(256) append_fused_kernel(LayerArgs a, int n, c
   if (act) {
     seq = seq_ids[e];
     pos = positions[e];
-    const int m = entry_mode(modes, mode_logits, e);
+    const int m = entry_mode(a, modes, mode_logits, e);
     if (seq < 0 || seq >= a.S) {
       err = TRR_ERR_INVALID_ARG;
     } else {
@@ -481,6 +514,16 @@ __global__ void __launch_bounds__(256) append_fused_kernel(LayerArgs a, int n, c
     }
     if (!later_seq) a.last_pos[seq] = pos;
   }
+  if (a.head_modes) {  // presence masks: openers clear their new pages, then every entry
+                       // sets its slot's bit for the KV heads it stores
+    unsigned long long* mw = (act && writes) ? page_masks(a, c, pid) : nullptr;
+    if (mw && opens)
+      for (int j = 0; j < a.Hkv; ++j) mw[j] = 0ull;
+    __syncthreads();
+    if (mw)
+      for (int j = 0; j < a.Hkv; ++j)
+        if (head_stores(a, modes, e, j)) atomicOr(mw + j, 1ull << (tok % a.P));
+  }
   if (e < kClasses) {
     int opened = 0;
     for (int w = 0; w < 8; ++w) opened += s_wopen[w][e];
@@ -510,6 +553,7 @@ static trr_status append_call(trr_cache* cache, int32_t layer, int32_t n, const 
     return TRR_ERR_INVALID_ARG;  // rows are read 16 bytes at a time
   if ((reinterpret_cast<uintptr_t>(bit_logits) | reinterpret_cast<uintptr_t>(mode_logits)) & 3)
     return TRR_ERR_INVALID_ARG;
+  if (mode_logits && l.head_modes) return TRR_ERR_UNSUPPORTED;  // router decisions are per token
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const LayerArgs a = layer_args(l, cache_views(cache), layer);
   const uint16_t* k = static_cast<const uint16_t*>(k_bf16);

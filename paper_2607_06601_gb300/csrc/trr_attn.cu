@@ -320,10 +320,13 @@ __device__ __forceinline__ void v_acc(uint32_t va, uint32_t vszaddr, float p, La
 // One page of width class B (P = NIT * keys per iteration tokens) at shared address s0;
 // lane -> (key kl, E-dim part), and two keys per lane per iteration (kl and kl + KPI)
 // when NIT is even, so that their dependency chains overlap.  Keys past `fill` are
-// empty slots; with positions at spos (masked pages), keys outside [lo, hi] are masked.
+// empty slots; with positions at spos (masked pages), keys outside [lo, hi] and slots
+// whose bit in pm is clear (per-head modes: the token does not store this KV head) are
+// masked.
 template <int D, int B, int NIT, int E>
-__device__ __forceinline__ void consume_page(uint32_t s0, uint32_t spos, bool masked, int G, int fill, int lo,
-                                             int hi, const float (&qp)[E], float sumq, LaneState<E>& st, int lane) {
+__device__ __forceinline__ void consume_page(uint32_t s0, uint32_t spos, bool masked, uint64_t pm, int G, int fill,
+                                             int lo, int hi, const float (&qp)[E], float sumq, LaneState<E>& st,
+                                             int lane) {
   constexpr int LPK = D / E;
   constexpr int KPI = 32 / LPK;
   constexpr int P = NIT * KPI;
@@ -345,7 +348,7 @@ __device__ __forceinline__ void consume_page(uint32_t s0, uint32_t spos, bool ma
       valid[k] = key < fill;
       if (masked) {
         const int pos = static_cast<int>(lds32(spos + 4 * key));
-        valid[k] = valid[k] && pos >= lo && pos <= hi;
+        valid[k] = valid[k] && pos >= lo && pos <= hi && ((pm >> key) & 1ull);
       }
       dot[k] = k_dot<B, E>(krow + (it + k) * KPI * rowb, ksz + (it + k) * szstep, qp, sumq);
     }
@@ -441,16 +444,37 @@ struct AttnKernelArgs {
   int defer_merge;   // 1: split partials are merged by the combine kernel (tensor-core path)
 };
 
-// Mode of query q: the caller's, or the hard decision of its mode logits.
-__device__ __forceinline__ int query_mode(const AttnKernelArgs& ka, int q) {
-  return ka.mode_logits ? hard_decision<3>(ka.mode_logits + 3 * q) : ka.modes[q];
+// Mode of query q: the caller's, or the hard decision of its mode logits.  With
+// per-head modes (modes[n][Hq]) the largest of its heads' modes, which sets the query's
+// key range (above full when a head's value is not a mode); any_local tells whether a
+// head is local (its window must then be valid).
+__device__ __forceinline__ int query_mode(const AttnKernelArgs& ka, int q, bool& any_local) {
+  if (ka.mode_logits) {
+    const int m = hard_decision<3>(ka.mode_logits + 3 * q);
+    any_local = m == TRR_MODE_LOCAL;
+    return m;
+  }
+  if (!ka.a.head_modes) {
+    const int m = ka.modes[q];
+    any_local = m == TRR_MODE_LOCAL;
+    return m;
+  }
+  const uint8_t* row = ka.modes + static_cast<int64_t>(q) * ka.a.Hq;
+  int m = 0;
+  any_local = false;
+  for (int h = 0; h < ka.a.Hq; ++h) {
+    const int v = row[h];
+    m = max(m, v);
+    any_local |= v == TRR_MODE_LOCAL;
+  }
+  return m;
 }
 
 // Error of a query's arguments, 0 when it is valid.
-__device__ __forceinline__ int query_error(const LayerArgs& a, int seq, int t, int mode, int w) {
+__device__ __forceinline__ int query_error(const LayerArgs& a, int seq, int t, int mode, bool any_local, int w) {
   if (seq < 0 || seq >= a.S || mode > TRR_MODE_FULL) return TRR_ERR_INVALID_ARG;
   if (t < 0 || t >= a.maxctx) return TRR_ERR_BAD_POSITION;
-  if (mode == TRR_MODE_LOCAL && w < 1) return TRR_ERR_INVALID_ARG;
+  if (any_local && w < 1) return TRR_ERR_INVALID_ARG;
   return 0;
 }
 
@@ -568,9 +592,10 @@ __device__ __forceinline__ void plan_units(const AttnKernelArgs& ka, int P, int 
   const int n = ka.n, lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
   long long rsum = 0;
   for (int q = threadIdx.x; q < n; q += blockDim.x) {
-    const int seq = ka.seq_ids[q], t = ka.q_positions[q], mode = query_mode(ka, q);
+    bool any_local;
+    const int seq = ka.seq_ids[q], t = ka.q_positions[q], mode = query_mode(ka, q, any_local);
     const int w = ka.windows ? ka.windows[q] : ka.window_scalar;
-    const int r = query_error(a, seq, t, mode, w) ? 0 : query_range(t, mode, w);
+    const int r = query_error(a, seq, t, mode, any_local, w) ? 0 : query_range(t, mode, w);
     pre[q] = r;
     rsum += r;
   }
@@ -697,18 +722,31 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
       else hi_q = mid;
     }
     const int q = lo_q, sp = un - pre[q], ns = pre[q + 1] - pre[q];
-    const int seq = ka.seq_ids[q], t = ka.q_positions[q], mode = query_mode(ka, q);
+    bool any_local;
+    const int seq = ka.seq_ids[q], t = ka.q_positions[q], mode = query_mode(ka, q, any_local);
     const int w = ka.windows ? ka.windows[q] : ka.window_scalar;
-    const int err = query_error(a, seq, t, mode, w);
+    const int err = query_error(a, seq, t, mode, any_local, w);
     const int h0 = qb * ka.hpu, nh = min(ka.hpu, a.Hq - h0);
-    if (err || mode == TRR_MODE_SKIP) {  // zero rows; the error of the lowest query
-      uint4* o = reinterpret_cast<uint4*>(ka.out + (static_cast<int64_t>(q) * a.Hq + h0) * D);
-      for (int i = lane; i < nh * D / 8; i += 32) o[i] = make_uint4(0, 0, 0, 0);
+    // per-head modes: the block's own widest mode sets its key range, and its heads'
+    // modes (2 bits each) travel in the query-rows record
+    int bmode = mode, hpack = 0;
+    if (a.head_modes && !err) {
+      const int hm = lane < nh ? ka.modes[static_cast<int64_t>(q) * a.Hq + h0 + lane] : 0;
+      bmode = static_cast<int>(__reduce_max_sync(0xffffffffu, static_cast<unsigned>(hm)));
+      hpack = static_cast<int>(__reduce_or_sync(0xffffffffu, static_cast<unsigned>(hm) << (2 * (lane & 15))));
+    }
+    if (err || bmode == TRR_MODE_SKIP) {  // zero rows (once per block); the error of the lowest query
+      if (sp == 0) {
+        uint4* o = reinterpret_cast<uint4*>(ka.out + (static_cast<int64_t>(q) * a.Hq + h0) * D);
+        for (int i = lane; i < nh * D / 8; i += 32) o[i] = make_uint4(0, 0, 0, 0);
+      }
       if (err && qb == 0 && lane == 0) atomicMin(&a.ctrl[kFirstBadQuery], (ka.q0 + q) * 16 + err);
     } else {
-      const int lo = mode == TRR_MODE_FULL ? 0 : max(0, t - w + 1);
+      const int lo = bmode == TRR_MODE_FULL ? 0 : max(0, t - w + 1);
       int wid, wmeta;
       const int T = plan_split(a, P, seq, lo, t, sp, ns, lane, wid, wmeta);
+      // per-head modes: every page brings its slot positions and presence masks
+      if (a.head_modes && lane < T) wmeta |= kMask;
       const int kv0 = h0 / g, nkv = (h0 + nh - 1) / g - kv0 + 1;
       const int4 rb = make_int4(t, sp, ns, pre[q]);
       {  // the unit's query rows
@@ -720,7 +758,8 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
           break;
         }
         const int meta = kQRows | kFirst | (T == 0 ? (kLast | kNoPage) : 0) | (qb << 16);
-        const uint32_t slot = push(make_int4(meta, off, q, lo), rb, make_int4(0, 0, -1, 0), taken, need);
+        const uint32_t slot =
+            push(make_int4(meta, off, q, lo), rb, make_int4(hpack, max(0, t - w + 1), -1, 0), taken, need);
         if (lane == 0)
           bulk_g2s(cr.ring + off, ka.q + (static_cast<int64_t>(q) * a.Hq + h0) * D, need, &cr.full[slot]);
       }
@@ -728,9 +767,11 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
       // is a few shuffles and the copy
       uint64_t pg_src = 0;  // the page
       int pg_geo = 0;       // slice bytes | KV slices per stage << 20
+      // extra bytes of a masked page's stage: positions, and per-head modes' presence masks
+      const int maskx = a.head_modes ? a.maskb + 16 : 0;
       if (lane < T) {
         const int c = wmeta & 3, slice = a.slice[c];
-        const int posb = (wmeta & kMask) ? 4 * P : 0;
+        const int posb = (wmeta & kMask) ? 4 * P + maskx : 0;
         pg_src = reinterpret_cast<uint64_t>(a.pool[c] + static_cast<int64_t>(wid) * a.page_bytes[c]);
         pg_geo = slice | (max(1, (R / 2 - posb) / slice) << 20);
       }
@@ -739,9 +780,12 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
         const int geo = __shfl_sync(0xffffffffu, pg_geo, j);
         const int pm = __shfl_sync(0xffffffffu, wmeta, j);
         const int slice = geo & 0xfffff, maxk = geo >> 20;
-        const int posb = (pm & kMask) ? 4 * P : 0;
         for (int k0 = 0; k0 < nkv; k0 += maxk) {
           const int nk = min(maxk, nkv - k0);
+          // the presence masks of KV heads kv0 + k0 .. + nk - 1, from a 16-byte boundary
+          const int mlo = (8 * (kv0 + k0)) & ~15, mhi = (8 * (kv0 + k0 + nk) + 15) & ~15;
+          const int mb = a.head_modes ? mhi - mlo : 0;
+          const int posb = (pm & kMask) ? 4 * P + mb : 0;
           const int need = nk * slice + posb;
           int taken = 0;
           const int off = reserve(need, taken);
@@ -755,7 +799,10 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
               push(make_int4(meta, off, q, lo), rb, make_int4(k0, nk, posb ? off + nk * slice : -1, slice), taken, need);
           if (lane == 0) {
             bulk_g2s(cr.ring + off, page + a.hdr + static_cast<int64_t>(kv0 + k0) * slice, nk * slice, &cr.full[slot]);
-            if (posb) bulk_g2s(cr.ring + off + nk * slice, page, posb, &cr.full[slot]);
+            if (posb) bulk_g2s(cr.ring + off + nk * slice, page, 4 * P, &cr.full[slot]);
+            if (posb && mb)
+              bulk_g2s(cr.ring + off + nk * slice + 4 * P,
+                       page + a.hdr + static_cast<int64_t>(a.Hkv) * slice + mlo, mb, &cr.full[slot]);
           }
         }
       }
@@ -937,7 +984,7 @@ __device__ __forceinline__ void run_consumer_cc(const AttnKernelArgs& ka, const 
 #pragma unroll
   for (int j = 0; j < E; ++j) st.acc[j] = 0.f;
   // the current unit
-  int u_q = 0, u_h = 0, u_kvi = 0, u_lo = 0, u_hi = 0, u_sp = 0, u_ns = 1, u_base = 0;
+  int u_q = 0, u_h = 0, u_kvi = 0, u_kv0 = 0, u_lo = 0, u_hi = 0, u_sp = 0, u_ns = 1, u_base = 0;
   bool active = false;
   for (uint32_t s = 0;; ++s) {
     const uint32_t slot = s % kStages;
@@ -958,13 +1005,26 @@ __device__ __forceinline__ void run_consumer_cc(const AttnKernelArgs& ka, const 
       const int qb = meta >> 16;
       u_h = qb * kNcw + cw;
       active = u_h < a.Hq;
-      u_kvi = u_h / g - (qb * kNcw) / g;
+      u_kv0 = (qb * kNcw) / g;
+      u_kvi = u_h / g - u_kv0;
       u_q = ra.z;
       u_lo = ra.w;
       u_hi = rb.x;
       u_sp = rb.y;
       u_ns = rb.z;
       u_base = rb.w;
+      if (a.head_modes && active) {  // this head's own mode: {head modes, local lo}
+        const int4 rq = lds128i(rec + 32);
+        const int hm = (rq.x >> (2 * cw)) & 3;
+        if (hm == TRR_MODE_SKIP) {  // a zero row (written once, by split 0), no merge
+          if (u_sp == 0 && lane < D / 8)
+            reinterpret_cast<uint4*>(ka.out + (static_cast<int64_t>(u_q) * a.Hq + u_h) * D)[lane] =
+                make_uint4(0, 0, 0, 0);
+          active = false;
+        } else if (hm == TRR_MODE_LOCAL) {
+          u_lo = rq.y;
+        }
+      }
       cur_cls = 3;  // the neutral scale is class 16's
       st.m = kNegInf;
       st.l = 0.f;
@@ -1000,11 +1060,17 @@ __device__ __forceinline__ void run_consumer_cc(const AttnKernelArgs& ka, const 
         const uint32_t s0 = smem_u32(cr.ring + ra.y + (u_kvi - rc.x) * rc.w);
         const bool masked = meta & kMask;
         const uint32_t sp = masked ? smem_u32(cr.ring + rc.z) : s0;
+        uint64_t pm = ~0ull;  // per-head modes: this KV head's presence mask, after the
+                              // positions; the stage's masks start at a 16-byte boundary
+        if (a.head_modes) {
+          const uint2 m2 = lds64(sp + 4 * P + 8 * ((u_kvi - rc.x) + ((u_kv0 + rc.x) & 1)));
+          pm = (static_cast<uint64_t>(m2.y) << 32) | m2.x;
+        }
         switch (cls) {
-          case 0: consume_page<D, 2, P / KPI, E>(s0, sp, masked, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
-          case 1: consume_page<D, 4, P / KPI, E>(s0, sp, masked, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
-          case 2: consume_page<D, 8, P / KPI, E>(s0, sp, masked, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
-          default: consume_page<D, 16, P / KPI, E>(s0, sp, masked, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
+          case 0: consume_page<D, 2, P / KPI, E>(s0, sp, masked, pm, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
+          case 1: consume_page<D, 4, P / KPI, E>(s0, sp, masked, pm, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
+          case 2: consume_page<D, 8, P / KPI, E>(s0, sp, masked, pm, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
+          default: consume_page<D, 16, P / KPI, E>(s0, sp, masked, pm, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
         }
       }
     }
@@ -1733,7 +1799,7 @@ cudaError_t attn_configure() {
 // one 8-wide mma tile.
 static bool use_mma(const Layout& l) {
   const int g = l.Hq / l.Hkv, ng = l.d / l.G;
-  return g >= 2 && g * ng <= 8;
+  return !l.head_modes && g >= 2 && g * ng <= 8;  // per-head modes: one warp per query head
 }
 
 // Ring bytes an attention call with n queries gets, or -1 when one stage of the
@@ -1741,7 +1807,7 @@ static bool use_mma(const Layout& l) {
 static int attn_ring_bytes(const Layout& l, int n, int hpu, int scr_floats, int limit) {
   const int fixed = AttnSmem(0, n, scr_floats).total;
   const int ring = (limit - fixed) / 128 * 128;
-  const int widest = static_cast<int>(l.slice[3]) + 4 * l.P;
+  const int widest = static_cast<int>(l.slice[3]) + 4 * l.P + (l.head_modes ? static_cast<int>(l.maskb) + 16 : 0);
   const int qrows = hpu * 2 * l.d;
   if (ring < std::max(widest, qrows)) return -1;
   return ring;
@@ -1808,7 +1874,7 @@ static cudaError_t launch_attention(const Layout& l, const LayerArgs& a, int num
     ka.q0 = q0;
     ka.seq_ids = seq_ids + q0;
     ka.q_positions = q_positions + q0;
-    ka.modes = modes ? modes + q0 : nullptr;
+    ka.modes = modes ? modes + static_cast<int64_t>(q0) * (l.head_modes ? l.Hq : 1) : nullptr;
     ka.mode_logits = mode_logits ? mode_logits + 3 * q0 : nullptr;
     ka.windows = windows ? windows + q0 : nullptr;
     ka.q = static_cast<const uint16_t*>(q_bf16) + q0 * row;
@@ -1871,6 +1937,7 @@ extern "C" trr_status trr_decode_attn_routed(trr_cache* cache, int32_t layer, in
   if (((reinterpret_cast<uintptr_t>(q_bf16) | reinterpret_cast<uintptr_t>(out_bf16)) & 15) ||
       (reinterpret_cast<uintptr_t>(mode_logits) & 3))
     return TRR_ERR_INVALID_ARG;
+  if (l.head_modes) return TRR_ERR_UNSUPPORTED;  // router decisions are per token
   const LayerArgs a = layer_args(l, cache_views(cache), layer);
   int launches = 0;
   const cudaError_t e = launch_attention(l, a, cache_num_sms(cache), n, seq_ids, q_positions, q_bf16, nullptr,

@@ -20,6 +20,7 @@ LayerArgs layer_args(const Layout& l, const Views& v, int layer) {
   a.maxctx = l.maxctx; a.MP = l.MP; a.W32 = l.W32; a.units = l.units; a.pos_split = l.pos_split;
   a.s_cap = l.s_cap;
   a.split_bytes = l.split_bytes; a.skip_writes_kv = l.skip_writes_kv;
+  a.head_modes = l.head_modes; a.maskb = static_cast<int>(l.maskb);
   a.hdr = static_cast<int>(l.hdr);
   for (int c = 0; c < kClasses; ++c) {
     a.cap[c] = l.cap[c];
@@ -58,7 +59,8 @@ static trr_status make_layout(const trr_cache_config* c, Layout* l) {
     return TRR_ERR_UNSUPPORTED;
   if (c->page_size != 16 && c->page_size != 32 && c->page_size != 64) return TRR_ERR_UNSUPPORTED;
   if (c->max_append > 1024 || c->max_queries > 4096 || c->skip_writes_kv < 0 ||
-      c->skip_writes_kv > 1 || c->max_context > (1 << 24) || c->max_seqs > (1 << 20))
+      c->skip_writes_kv > 1 || c->head_modes < 0 || c->head_modes > 1 || c->max_context > (1 << 24) ||
+      c->max_seqs > (1 << 20))
     return TRR_ERR_UNSUPPORTED;
   for (int k = 0; k < kClasses; ++k)
     if (c->pages_per_class[k] < 0) return TRR_ERR_INVALID_ARG;
@@ -72,12 +74,15 @@ static trr_status make_layout(const trr_cache_config* c, Layout* l) {
   l->max_queries = c->max_queries;
   l->split_bytes = c->split_bytes ? c->split_bytes : 24576;
   l->skip_writes_kv = c->skip_writes_kv;
+  l->head_modes = c->head_modes;
   l->hdr = roundup(4 * static_cast<int64_t>(l->P), 128);
+  // per-head modes: one 64-bit presence mask per KV head after the slices of a page
+  l->maskb = l->head_modes ? roundup(8 * static_cast<int64_t>(l->Hkv), 16) : 0;
   for (int k = 0; k < kClasses; ++k) {
     const int b = bits_of_class(k);
     l->tokb[k] = b < 16 ? 2 * (l->d * b / 8) + 2 * (l->d / l->G) * 4 : 4 * l->d;
     l->slice[k] = l->P * l->tokb[k];
-    l->page_bytes[k] = roundup(l->hdr + l->Hkv * l->slice[k], 128);
+    l->page_bytes[k] = roundup(l->hdr + l->Hkv * l->slice[k] + l->maskb, 128);
   }
   l->units = l->Hq;
   // splits per query: at least pos_split key positions each (split_bytes of 8-bit

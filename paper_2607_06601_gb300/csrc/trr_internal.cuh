@@ -39,13 +39,13 @@ constexpr int kMergeGroup = 16;
 struct Layout {
   int L, S, Hq, Hkv, d, G, P, maxctx, MP, W32;
   int cap[kClasses];
-  int max_append, max_queries, split_bytes, skip_writes_kv;
+  int max_append, max_queries, split_bytes, skip_writes_kv, head_modes;
   int units;      // attention work units per query split (one per query head)
   int pos_split;  // key positions per split at least (split_bytes of 8-bit tokens)
   int s_cap;      // most splits one query is cut into
   int cnt_stride; // arrival counters per (query, head): 1 + ceil(s_cap / kMergeGroup)
   int64_t max_items;
-  int64_t hdr, tokb[kClasses], slice[kClasses], page_bytes[kClasses];
+  int64_t hdr, tokb[kClasses], slice[kClasses], maskb, page_bytes[kClasses];
   int64_t off_ctrl, off_last_pos, off_ntok, off_presence, off_pt, off_pfirst, off_plast, off_lastpg;
   int64_t off_aplan, off_cnt, off_part, off_pool[kClasses], total;
 };
@@ -105,6 +105,8 @@ inline Views make_views(const Layout& l, void* base) {
 // Everything a kernel needs about one layer of one cache, passed by value.
 struct LayerArgs {
   int layer, S, Hq, Hkv, d, G, P, maxctx, MP, W32, units, pos_split, s_cap, cnt_stride, split_bytes, skip_writes_kv;
+  int head_modes;      // modes are [n][Hq]; pages end with a presence mask per KV head
+  int maskb;           // bytes of a page's presence masks (0 without head_modes)
   int cap[kClasses];
   int hdr;
   int slice[kClasses];

@@ -34,7 +34,8 @@ class trr_cache_config(ctypes.Structure):
                 ("page_size", ctypes.c_int32), ("max_context", ctypes.c_int32),
                 ("pages_per_class", ctypes.c_int32 * 4), ("max_append", ctypes.c_int32),
                 ("max_queries", ctypes.c_int32), ("split_bytes", ctypes.c_int32),
-                ("skip_writes_kv", ctypes.c_int32), ("pool", ctypes.c_void_p),
+                ("skip_writes_kv", ctypes.c_int32), ("head_modes", ctypes.c_int32),
+                ("pool", ctypes.c_void_p),
                 ("pool_bytes", ctypes.c_uint64)]
 
 
@@ -103,7 +104,7 @@ def _dev(t: torch.Tensor, dtype, name):
 
 def make_config(num_layers, max_seqs, num_q_heads, num_kv_heads, head_dim, group_size,
                 page_size, max_context, pages_per_class, max_append=1024, max_queries=1024,
-                split_bytes=0, skip_writes_kv=0) -> trr_cache_config:
+                split_bytes=0, skip_writes_kv=0, head_modes=0) -> trr_cache_config:
     cfg = trr_cache_config()
     cfg.num_layers, cfg.max_seqs = num_layers, max_seqs
     cfg.num_q_heads, cfg.num_kv_heads = num_q_heads, num_kv_heads
@@ -113,6 +114,7 @@ def make_config(num_layers, max_seqs, num_q_heads, num_kv_heads, head_dim, group
         cfg.pages_per_class[i] = int(pages_per_class[i])
     cfg.max_append, cfg.max_queries = max_append, max_queries
     cfg.split_bytes, cfg.skip_writes_kv = split_bytes, skip_writes_kv
+    cfg.head_modes = head_modes
     return cfg
 
 
@@ -239,10 +241,11 @@ class Cache:
 
     def __init__(self, num_layers, max_seqs, num_q_heads, num_kv_heads, head_dim, group_size,
                  page_size, max_context, pages_per_class, max_append=1024, max_queries=1024,
-                 split_bytes=0, skip_writes_kv=0, device=None, zero_pool=False):
+                 split_bytes=0, skip_writes_kv=0, device=None, zero_pool=False, head_modes=0):
         self.cfg = make_config(num_layers, max_seqs, num_q_heads, num_kv_heads, head_dim,
                                group_size, page_size, max_context, pages_per_class, max_append,
-                               max_queries, split_bytes, skip_writes_kv)
+                               max_queries, split_bytes, skip_writes_kv, head_modes)
+        self.head_modes = int(head_modes)
         self.nbytes = trr_cache_required_bytes(self.cfg)
         alloc = torch.zeros if zero_pool else torch.empty
         self.pool = alloc(self.nbytes, dtype=torch.uint8, device=device or torch.cuda.current_device())
@@ -250,11 +253,19 @@ class Cache:
         self.L, self.S, self.Hq, self.Hkv = num_layers, max_seqs, num_q_heads, num_kv_heads
         self.d, self.G, self.P, self.max_context = head_dim, group_size, page_size, max_context
 
+    def _check_modes(self, modes, n):
+        want = n * (self.Hq if self.head_modes else 1)
+        if modes.numel() != want:
+            raise ValueError(f"modes must have {want} elements "
+                             f"({'[n][Hq]' if self.head_modes else '[n]'}), got {modes.numel()}")
+
     def append(self, layer, seq_ids, positions, k, v, bits, modes, stream=None):
+        self._check_modes(modes, seq_ids.numel())
         trr_kv_append(self.handle, layer, seq_ids, positions, k, v, bits, modes, stream)
 
     def decode_attn(self, layer, seq_ids, q_positions, q, modes, windows=None, window_scalar=0,
                     softmax_scale=0.0, out=None, stream=None):
+        self._check_modes(modes, seq_ids.numel())
         if out is None:
             out = torch.empty((seq_ids.numel(), self.Hq, self.d), dtype=torch.bfloat16, device=q.device)
         trr_decode_attn(self.handle, layer, seq_ids, q_positions, q, modes, windows, window_scalar,

@@ -122,6 +122,17 @@ def policy(spec: Spec, layer: int, seq: int, n: int | None = None):
     return bits[:n].copy(), modes[:n].copy()
 
 
+def head_policy(spec: Spec, layer: int, seq: int, n: int | None = None):
+    """Per-token bits and per-(token, query head) modes [n][Hq] of positions 0..n-1 (the
+    paper's default granularity, Sec. 3.2(A)): bits as policy(), every head's mode drawn
+    i.i.d. from the workload's mode mix."""
+    n = spec.max_context if n is None else n
+    bits, _ = policy(spec, layer, seq, n)
+    r = _rng(spec.seed, layer, seq, 3)
+    modes = r.choice(3, size=(spec.max_context, spec.num_q_heads), p=spec.modes_p).astype(np.uint8)
+    return bits, modes[:n].copy()
+
+
 def outlier_channels(spec: Spec, layer: int) -> np.ndarray:
     """Flat (kv head * d + dim) indices of the outlier channels of a layer."""
     if spec.outlier_frac <= 0:

@@ -25,13 +25,15 @@ class Pair:
     """A GPU cache and an oracle cache with one configuration, fed the same calls."""
 
     def __init__(self, L, S, Hq, Hkv, d, G, P, maxctx, caps, skip_writes_kv=0, max_append=1024,
-                 max_queries=1024, split_bytes=0, oracle_pool=True):
+                 max_queries=1024, split_bytes=0, oracle_pool=True, head_modes=0):
         self.gpu = trr.Cache(L, S, Hq, Hkv, d, G, P, maxctx, caps, max_append=max_append,
                              max_queries=max_queries, split_bytes=split_bytes,
-                             skip_writes_kv=skip_writes_kv, zero_pool=True)
+                             skip_writes_kv=skip_writes_kv, zero_pool=True, head_modes=head_modes)
         # zero_pool: unused slots read back as zeros, as the oracle's calloc
         self.orc = oracle.OracleCache(L, S, Hq, Hkv, d, G, P, maxctx, caps,
-                                      skip_writes_kv=skip_writes_kv, no_pool=not oracle_pool)
+                                      skip_writes_kv=skip_writes_kv, no_pool=not oracle_pool,
+                                      head_modes=head_modes)
+        self.head_modes = head_modes
         self.Hq, self.Hkv, self.d, self.P = Hq, Hkv, d, P
 
     def append(self, layer, seqs, pos, k, v, bits, modes, expect=0):
@@ -59,7 +61,8 @@ class Pair:
         assert st_o == expect, f"oracle attention status {st_o}, expected {expect}"
         assert st_g == st_o, f"gpu attention status {st_g} != oracle {st_o}"
         got = out.float().cpu().numpy().astype(np.float64)
-        check_attention(got, ref, modes)
+        # skip rows must be bit-zero: per query, or per (query, head) with head modes
+        check_attention(got, ref, modes.reshape(len(seqs), self.Hq) if self.head_modes else modes)
         return got, ref
 
     def check_regions(self, pools=True):
