@@ -212,19 +212,25 @@ static int entry_stores(const orc_cache* o, const uint8_t* modes, int i) {
   return 0;
 }
 
-/* With head_modes, the bit of `slot` in KV head j's 64-bit presence mask, stored
- * little-endian after the page's KV slices. */
+/* With head_modes, KV head j's 64-bit presence mask (little-endian): the first 8 of the
+ * 16 bytes that end its slice of the page. */
+static uint8_t* mask_ptr(const orc_cache* o, const uint8_t* page, int c, int j) {
+  return (uint8_t*)page + o->hdr + (int64_t)j * o->slice[c] + o->slice[c] - o->maskb;
+}
+
+/* With head_modes, the bit of `slot` in KV head j's presence mask. */
 static int slot_present(const orc_cache* o, const uint8_t* page, int c, int slot, int j) {
   uint64_t m;
   if (!o->head_modes) return 1;
-  memcpy(&m, page + o->hdr + o->Hkv * o->slice[c] + 8 * (int64_t)j, 8);
+  memcpy(&m, mask_ptr(o, page, c, j), 8);
   return (int)((m >> slot) & 1);
 }
 
 /* cfg: L, S, Hq, Hkv, d, G, P, max_context, cap[4], skip_writes_kv, no_pool, head_modes.
  * With no_pool = 1 only metadata and nothing of the page bytes is kept.  head_modes = 1:
  * attention modes are chosen per query head (Sec. 3.2(A): per head by default), modes
- * arrays are [n][Hq], and every page ends with one 64-bit presence mask per KV head. */
+ * arrays are [n][Hq], and every KV head's slice of a page ends with 16 bytes holding its
+ * 64-bit presence mask (then 8 zero bytes). */
 int orc_create(const int32_t* cfg, orc_cache** out) {
   int c;
   *out = NULL;
@@ -248,12 +254,12 @@ int orc_create(const int32_t* cfg, orc_cache** out) {
   o->MP = (o->maxctx + o->P - 1) / o->P;
   o->W32 = (o->maxctx + 31) / 32;
   o->hdr = roundup(4 * (int64_t)o->P, 128);
-  o->maskb = o->head_modes ? roundup(8 * (int64_t)o->Hkv, 16) : 0;
+  o->maskb = o->head_modes ? 16 : 0;
   for (c = 0; c < 4; c++) {
     int b = BITS_OF_CLASS[c];
     o->tokb[c] = b < 16 ? 2 * (o->d * b / 8) + 2 * (o->d / o->G) * 4 : 4 * o->d;
-    o->slice[c] = o->P * o->tokb[c];
-    o->page_bytes[c] = roundup(o->hdr + o->Hkv * o->slice[c] + o->maskb, 128);
+    o->slice[c] = o->P * o->tokb[c] + o->maskb;
+    o->page_bytes[c] = roundup(o->hdr + o->Hkv * o->slice[c], 128);
   }
   int64_t nls = (int64_t)o->L * o->S;
   o->last_pos = (int32_t*)malloc(sizeof(int32_t) * nls);
@@ -391,7 +397,7 @@ int orc_append(orc_cache* o, int layer, int n, const int32_t* seq_ids,
     /* head_modes: every KV head's row is written; the heads that store it get their
      * presence bit (a new page starts with every bit clear) */
     for (h = 0; h < o->Hkv && o->head_modes; h++) {
-      uint8_t* mw = page + o->hdr + o->Hkv * o->slice[c] + 8 * (int64_t)h;
+      uint8_t* mw = mask_ptr(o, page, c, h);
       uint64_t m;
       memcpy(&m, mw, 8);
       if (slot == 0) m = 0;
@@ -609,7 +615,8 @@ int64_t orc_region(orc_cache* o, int id, void** ptr) {
 }
 
 /* Layout sizes: which = 0 header bytes, 1..4 slice bytes of class 0..3,
- * 5..8 page bytes of class 0..3, 9 bytes of a page's presence masks (head_modes). */
+ * 5..8 page bytes of class 0..3, 9 bytes that end each slice for its presence mask
+ * (16 with head_modes, else 0). */
 int64_t orc_layout(const orc_cache* o, int which) {
   if (which == 0) return o->hdr;
   if (which >= 1 && which <= 4) return o->slice[which - 1];

@@ -2,10 +2,11 @@
 default; Appendix C's router emits modes of shape [B, T, H, |A|]).  A cache with
 head_modes takes modes[n][Hq]; KV head j of a token is stored when one of the query
 heads reading it (h / (Hq / Hkv) = j) does not skip (or when skip tokens store KV), and
-pages carry a 64-bit presence mask per KV head.  Pinned against: the per-token cache
-(all heads of a token with one mode give the same results and bytes), an explicit
-per-head mask over dequantised K/V for every per-head policy of tiny contexts, the
-presence bits read straight from the page bytes, and the error contract."""
+every KV head's slice of a page ends with 16 bytes holding its 64-bit presence mask.
+Pinned against: the per-token cache (all heads of a token with one mode give the same
+results and bytes), an explicit per-head mask over dequantised K/V for every per-head
+policy of tiny contexts, the presence bits read straight from the page bytes, and the
+error contract."""
 import itertools
 
 import numpy as np
@@ -48,18 +49,24 @@ def test_equal_head_modes_match_the_per_token_cache(Hq, Hkv):
         assert hed.append(0, np.arange(S), [p] * S, K, V, bits[:, p], np.repeat(m, Hq)) == 0
     for name in ("last_pos", "ntok", "presence", "page_table", "page_first", "page_last", "next_page"):
         assert np.array_equal(tok.region(name), hed.region(name)), name
-    assert tok.mask_bytes == 0 and hed.mask_bytes == -(-8 * Hkv // 16) * 16
+    assert tok.mask_bytes == 0 and hed.mask_bytes == 16
     ntok = hed.region("ntok").view(np.int32).reshape(S, 4)
     for c, b in enumerate((2, 4, 8, 16)):
         pt, ph = tok.region(f"pool{b}"), hed.region(f"pool{b}")
-        body = hed.hdr_bytes + Hkv * hed.slice_bytes(c)
+        sl_t = tok.slice_bytes(c)
+        assert hed.slice_bytes(c) == sl_t + 16
         for pid in range(int(hed.region("next_page").view(np.int32)[c])):
-            a = pt[pid * tok.page_bytes(c):pid * tok.page_bytes(c) + body]
-            bb = ph[pid * hed.page_bytes(c):pid * hed.page_bytes(c) + body]
-            assert np.array_equal(a, bb), (b, pid)
-            masks = ph[pid * hed.page_bytes(c) + body:pid * hed.page_bytes(c) + body + 8 * Hkv].view(np.uint64)
-            fill = bin(int(masks[0])).count("1")
-            assert fill >= 1 and all(int(x) == (1 << fill) - 1 for x in masks)  # every head, every slot
+            a0, b0 = pid * tok.page_bytes(c), pid * hed.page_bytes(c)
+            assert np.array_equal(pt[a0:a0 + tok.hdr_bytes], ph[b0:b0 + hed.hdr_bytes]), (b, pid)
+            masks = []
+            for j in range(Hkv):  # each KV head's slice: the same bytes, then its mask, 8 zeros
+                sa = pt[a0 + tok.hdr_bytes + j * sl_t:][:sl_t]
+                sb = ph[b0 + hed.hdr_bytes + j * (sl_t + 16):][:sl_t + 16]
+                assert np.array_equal(sa, sb[:sl_t]), (b, pid, j)
+                masks.append(int(sb[sl_t:sl_t + 8].view(np.uint64)[0]))
+                assert not sb[sl_t + 8:].any()
+            fill = bin(masks[0]).count("1")
+            assert fill >= 1 and all(x == (1 << fill) - 1 for x in masks)  # every head, every slot
     assert ntok.sum() > 0
     q = bf16_bits(rng.standard_normal((3 * S, Hq, d), dtype=np.float32))
     seqs = np.tile(np.arange(S), 3)
@@ -155,11 +162,12 @@ def test_presence_bits_follow_the_reading_heads():
         assert ntok[c] == pos.size
         pool = o.region(f"pool{b}")
         pt = o.region("page_table").view(np.int32).reshape(4, -1)
-        body = o.hdr_bytes + Hkv * o.slice_bytes(c)
+        slb = o.slice_bytes(c)
         for k in range(-(-pos.size // P)):
             base = int(pt[c, k]) * o.page_bytes(c)
             slots = pool[base:base + 4 * P].view(np.int32)
-            masks = pool[base + body:base + body + 8 * Hkv].view(np.uint64)
+            # KV head j's mask: the first 8 of the 16 bytes that end its slice
+            masks = [pool[base + o.hdr_bytes + (j + 1) * slb - 16:][:8].view(np.uint64)[0] for j in range(Hkv)]
             for sl in range(min(P, pos.size - k * P)):
                 assert slots[sl] == pos[k * P + sl]
                 for j in range(Hkv):
