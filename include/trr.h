@@ -45,9 +45,9 @@
  *   Pools: class c holds pages_per_class[c] pages of PAGE_BYTES(b) bytes each:
  *     HDR        = roundup(4 * P, 128)           header: int32 positions[P]
  *     TOKB(b)    = 2*(d*b/8) + 2*(d/G)*4   (b < 16)  |  4*d   (b = 16)
- *     SLICE(b)   = P * TOKB(b)                  one KV head of one page
- *     MASKB      = roundup(8 * Hkv, 16) with head_modes, else 0
- *     PAGE_BYTES = roundup(HDR + Hkv * SLICE(b) + MASKB, 128)
+ *     SLICE(b)   = P * TOKB(b) + MASKB          one KV head of one page
+ *     MASKB      = 16 with head_modes, else 0
+ *     PAGE_BYTES = roundup(HDR + Hkv * SLICE(b), 128)
  *     head h starts at HDR + h * SLICE(b); inside it, for b < 16:
  *       K codes [P][d*b/8] | V codes [P][d*b/8] | K sz [P][d/G][2] | V sz [P][d/G][2]
  *     where sz = (scale, zero) as IEEE binary16, and for b = 16:
@@ -56,9 +56,9 @@
  *   least significant bits first (2-bit codes 1,2,3,0 -> byte 0x39).
  *   Page allocation: entries are taken in array order; an entry of class c whose
  *   (layer, seq) has ntok % P == 0 opens page next_page[c]++ .
- *   Per-head modes (head_modes = 1): after the slices, at HDR + Hkv * SLICE(b), one
- *   little-endian uint64 per KV head: bit `slot` set <=> the token in that slot stores
- *   that KV head.  A page starts with every bit clear when its slot 0 is written.
+ *   Per-head modes (head_modes = 1): the last 16 bytes of KV head h's slice hold a
+ *   little-endian uint64 (then 8 zero bytes): bit `slot` set <=> the token in that slot
+ *   stores KV head h.  A page starts with every bit clear when its slot 0 is written.
  */
 #ifndef TRR_H
 #define TRR_H

@@ -43,10 +43,11 @@ __device__ __forceinline__ bool head_stores(const LayerArgs& a, const uint8_t* m
   return false;
 }
 
-// Per-head modes: the page's presence masks, one uint64 per KV head after its slices.
-__device__ __forceinline__ unsigned long long* page_masks(const LayerArgs& a, int c, int pid) {
+// Per-head modes: KV head j's presence mask in a page, the first 8 of the 16 bytes that
+// end its slice.
+__device__ __forceinline__ unsigned long long* head_mask(const LayerArgs& a, int c, int pid, int j) {
   return reinterpret_cast<unsigned long long*>(a.pool[c] + static_cast<int64_t>(pid) * a.page_bytes[c] + a.hdr +
-                                               static_cast<int64_t>(a.Hkv) * a.slice[c]);
+                                               static_cast<int64_t>(j + 1) * a.slice[c] - a.maskb);
 }
 __device__ __forceinline__ int entry_bits(const uint8_t* bits, const float* bit_logits, int e) {
   return bit_logits ? 2 << hard_decision<4>(bit_logits + 4 * e) : bits[e];
@@ -140,10 +141,11 @@ __global__ void __launch_bounds__(1024) append_plan_kernel(LayerArgs a, int n, c
     a.pt[row] = pid;
     a.pfirst[row] = pos;
     atomicAdd(&s_nopen[c], 1);
-    if (a.head_modes) {  // a new page starts with every presence bit clear
-      unsigned long long* mw = page_masks(a, c, pid);
-      for (int j = 0; j < a.Hkv; ++j) mw[j] = 0ull;
-    }
+    if (a.head_modes)  // a new page starts with every presence bit (and the padding) clear
+      for (int j = 0; j < a.Hkv; ++j) {
+        head_mask(a, c, pid, j)[0] = 0ull;
+        head_mask(a, c, pid, j)[1] = 0ull;
+      }
   }
   __syncthreads();
   if (act) {
@@ -160,11 +162,9 @@ __global__ void __launch_bounds__(1024) append_plan_kernel(LayerArgs a, int n, c
       }
       reinterpret_cast<int32_t*>(a.pool[c] + pid * a.page_bytes[c])[slot] = pos;
       atomicOr(&a.presence[static_cast<int64_t>(seq) * a.W32 + pos / 32], 1u << (pos % 32));
-      if (a.head_modes) {  // the slot's bit for every KV head the entry stores
-        unsigned long long* mw = page_masks(a, c, pid);
+      if (a.head_modes)  // the slot's bit for every KV head the entry stores
         for (int j = 0; j < a.Hkv; ++j)
-          if (head_stores(a, modes, e, j)) atomicOr(mw + j, 1ull << slot);
-      }
+          if (head_stores(a, modes, e, j)) atomicOr(head_mask(a, c, pid, j), 1ull << slot);
     }
     a.aplan[e] = p;
     if (!later_seq) a.last_pos[seq] = pos;
@@ -516,13 +516,16 @@ __global__ void __launch_bounds__(256) append_fused_kernel(LayerArgs a, int n, c
   }
   if (a.head_modes) {  // presence masks: openers clear their new pages, then every entry
                        // sets its slot's bit for the KV heads it stores
-    unsigned long long* mw = (act && writes) ? page_masks(a, c, pid) : nullptr;
-    if (mw && opens)
-      for (int j = 0; j < a.Hkv; ++j) mw[j] = 0ull;
+    const bool mine = act && writes;
+    if (mine && opens)
+      for (int j = 0; j < a.Hkv; ++j) {
+        head_mask(a, c, pid, j)[0] = 0ull;
+        head_mask(a, c, pid, j)[1] = 0ull;
+      }
     __syncthreads();
-    if (mw)
+    if (mine)
       for (int j = 0; j < a.Hkv; ++j)
-        if (head_stores(a, modes, e, j)) atomicOr(mw + j, 1ull << (tok % a.P));
+        if (head_stores(a, modes, e, j)) atomicOr(head_mask(a, c, pid, j), 1ull << (tok % a.P));
   }
   if (e < kClasses) {
     int opened = 0;

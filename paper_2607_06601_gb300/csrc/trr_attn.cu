@@ -320,10 +320,10 @@ __device__ __forceinline__ void v_acc(uint32_t va, uint32_t vszaddr, float p, La
 // One page of width class B (P = NIT * keys per iteration tokens) at shared address s0;
 // lane -> (key kl, E-dim part), and two keys per lane per iteration (kl and kl + KPI)
 // when NIT is even, so that their dependency chains overlap.  Keys past `fill` are
-// empty slots; with positions at spos (masked pages), keys outside [lo, hi] and slots
-// whose bit in pm is clear (per-head modes: the token does not store this KV head) are
-// masked.
-template <int D, int B, int NIT, int E>
+// empty slots; with positions at spos (masked pages), keys outside [lo, hi] are masked,
+// and with HM (per-head modes) the slots whose bit in pm is clear (the token does not
+// store this KV head).
+template <int D, int B, int NIT, int E, bool HM>
 __device__ __forceinline__ void consume_page(uint32_t s0, uint32_t spos, bool masked, uint64_t pm, int G, int fill,
                                              int lo, int hi, const float (&qp)[E], float sumq, LaneState<E>& st,
                                              int lane) {
@@ -346,9 +346,10 @@ __device__ __forceinline__ void consume_page(uint32_t s0, uint32_t spos, bool ma
     for (int k = 0; k < KP; ++k) {
       const int key = (it + k) * KPI + kl;
       valid[k] = key < fill;
+      if (HM) valid[k] = valid[k] && ((pm >> key) & 1ull);
       if (masked) {
         const int pos = static_cast<int>(lds32(spos + 4 * key));
-        valid[k] = valid[k] && pos >= lo && pos <= hi && ((pm >> key) & 1ull);
+        valid[k] = valid[k] && pos >= lo && pos <= hi;
       }
       dot[k] = k_dot<B, E>(krow + (it + k) * KPI * rowb, ksz + (it + k) * szstep, qp, sumq);
     }
@@ -422,7 +423,8 @@ enum : int {
   kLast = 1 << 11,    // last stage of a unit
   kNoPage = 1 << 12,  // the unit has no page in range
   kEnd = 1 << 13,     // no more units
-  kQRows = 1 << 14    // the stage holds the unit's query rows
+  kQRows = 1 << 14,   // the stage holds the unit's query rows
+  kEarly = 1 << 15    // per-head modes: the page ends before the local window
 };
 
 struct AttnKernelArgs {
@@ -496,7 +498,7 @@ struct AttnSmem {
         empty(full + kStages * 8),
         scr(empty + kStages * 8),
         pre(scr + align16(kNcw * scr_floats * 4)),
-        red(pre + align16(4 * (n + 1))),
+        red(pre + align16(4 * (n + 2))),
         flag(red + 16 * 8),
         total(flag + 16) {}
 };
@@ -522,12 +524,14 @@ __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
 }
 
 // Pages of split sp (of ns) of a query of sequence seq over key positions [lo, t]:
-// returns their number T (<= kItemMaxPages + 4); lane j < T gets page j's id in wid and
-// class | fill << 2 | kMask in wmeta.  Pages are listed class by class, each class's in
+// returns their number T (<= kItemMaxPages + 4); lane j < T gets page j's id in wid,
+// class | fill << 2 | kMask in wmeta and, when wfirst / wlast are given, the page's first
+// and last positions.  Pages are listed class by class, each class's in
 // position order; split sp of ns takes np / ns of a class's np pages in range, one more
 // when sp < np % ns.
 __device__ __forceinline__ int plan_split(const LayerArgs& a, int P, int seq, int lo, int t, int sp, int ns,
-                                          int lane, int& wid, int& wmeta) {
+                                          int lane, int& wid, int& wmeta, int* wfirst = nullptr,
+                                          int* wlast = nullptr) {
   int nt[kClasses];
 #pragma unroll
   for (int c = 0; c < kClasses; ++c) nt[c] = a.ntok[seq * 4 + c];
@@ -577,6 +581,10 @@ __device__ __forceinline__ int plan_split(const LayerArgs& a, int P, int seq, in
   if (lane < T) {
     const int f = pick(first);
     wid = from_tail >= 0 ? from_tail : a.pt[static_cast<int64_t>(seq * 4 + c) * a.MP + kid];
+    if (wfirst) {  // the page's first and last positions
+      *wfirst = a.pfirst[static_cast<int64_t>(seq * 4 + c) * a.MP + kid];
+      *wlast = a.plast[static_cast<int64_t>(seq * 4 + c) * a.MP + kid];
+    }
     const int fill = min(P, pick(nt) - kid * P);
     // slot positions are needed on a page that may hold keys outside [lo, t]
     const bool mask = (lo > 0 && kid == f) || (upper_mask && kid == f + pick(npr) - 1);
@@ -586,7 +594,8 @@ __device__ __forceinline__ int plan_split(const LayerArgs& a, int P, int seq, in
 }
 
 // The work units of a call, computed the same way by every CTA: query q gets ns_q
-// splits from its key range; pre[q] numbers its first split, pre[n] counts them all.
+// splits from its key range (per-head modes: its widest head's); pre[q] numbers its
+// first split, pre[n] counts them all, pre[n + 1] is the call's key positions per split.
 __device__ __forceinline__ void plan_units(const AttnKernelArgs& ka, int P, int NQB, int* pre, long long* red) {
   const LayerArgs& a = ka.a;
   const int n = ka.n, lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
@@ -620,7 +629,11 @@ __device__ __forceinline__ void plan_units(const AttnKernelArgs& ka, int P, int 
   const int chunk = (n + blockDim.x - 1) / blockDim.x;
   const int q0 = min(n, static_cast<int>(threadIdx.x) * chunk), q1 = min(n, q0 + chunk);
   int mine = 0;
-  for (int q = q0; q < q1; ++q) mine += splits_of(pre[q], pos_split, P, a.s_cap);
+  for (int q = q0; q < q1; ++q) {  // pre[q] becomes the query's split count
+    const int ns = splits_of(pre[q], pos_split, P, a.s_cap);
+    pre[q] = ns;
+    mine += ns;
+  }
   int incl = mine;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
@@ -633,11 +646,14 @@ __device__ __forceinline__ void plan_units(const AttnKernelArgs& ka, int P, int 
   int off = incl - mine;
   for (int k = 0; k < warp; ++k) off += static_cast<int>(red[8 + k]);
   for (int q = q0; q < q1; ++q) {
-    const int ns = splits_of(pre[q], pos_split, P, a.s_cap);
+    const int ns = pre[q];
     pre[q] = off;
     off += ns;
   }
-  if (threadIdx.x == blockDim.x - 1) pre[n] = off;
+  if (threadIdx.x == blockDim.x - 1) {
+    pre[n] = off;
+    pre[n + 1] = pos_split;  // for per-block split counts (per-head modes)
+  }
   __syncthreads();
   if (ka.defer_merge && blockIdx.x == 0) {  // for the combine kernel
     int2* qtab = reinterpret_cast<int2*>(a.cnt);
@@ -721,7 +737,8 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
       if (pre[mid] <= un) lo_q = mid;
       else hi_q = mid;
     }
-    const int q = lo_q, sp = un - pre[q], ns = pre[q + 1] - pre[q];
+    const int q = lo_q, sp = un - pre[q];
+    int ns = pre[q + 1] - pre[q];
     bool any_local;
     const int seq = ka.seq_ids[q], t = ka.q_positions[q], mode = query_mode(ka, q, any_local);
     const int w = ka.windows ? ka.windows[q] : ka.window_scalar;
@@ -730,10 +747,29 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
     // per-head modes: the block's own widest mode sets its key range, and its heads'
     // modes (2 bits each) travel in the query-rows record
     int bmode = mode, hpack = 0;
+    const int kv0 = h0 / g, nkv = (h0 + nh - 1) / g - kv0 + 1;
+    // the block's KV heads (bit k: kv0 + k) that a page must bring: every one, or with
+    // per-head modes those read by a full head of the block (pages before the local
+    // window) and those read by any head of the block (the other pages)
+    unsigned need_full = (1u << nkv) - 1u, need_any = need_full;
     if (a.head_modes && !err) {
       const int hm = lane < nh ? ka.modes[static_cast<int64_t>(q) * a.Hq + h0 + lane] : 0;
       bmode = static_cast<int>(__reduce_max_sync(0xffffffffu, static_cast<unsigned>(hm)));
       hpack = static_cast<int>(__reduce_or_sync(0xffffffffu, static_cast<unsigned>(hm) << (2 * (lane & 15))));
+      const unsigned kbit = 1u << (((h0 + (lane & 15)) / g - kv0) & 31);
+      need_full = __reduce_or_sync(0xffffffffu, (lane < nh && hm == TRR_MODE_FULL) ? kbit : 0u);
+      need_any = __reduce_or_sync(0xffffffffu, (lane < nh && hm != TRR_MODE_SKIP) ? kbit : 0u);
+    }
+    if (a.head_modes && !err && bmode == TRR_MODE_LOCAL) {
+      // per-head modes, a block of local and skip heads in a query whose widest head is
+      // full: the block's own split count, from its window; its splits past that have
+      // nothing to do, and its heads merge that many partials
+      ns = min(ns, splits_of(query_range(t, TRR_MODE_LOCAL, w), pre[n + 1], P, a.s_cap));
+      if (sp >= ns) {
+        __syncwarp();
+        u = __shfl_sync(0xffffffffu, u_next, 0);
+        continue;
+      }
     }
     if (err || bmode == TRR_MODE_SKIP) {  // zero rows (once per block); the error of the lowest query
       if (sp == 0) {
@@ -743,11 +779,16 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
       if (err && qb == 0 && lane == 0) atomicMin(&a.ctrl[kFirstBadQuery], (ka.q0 + q) * 16 + err);
     } else {
       const int lo = bmode == TRR_MODE_FULL ? 0 : max(0, t - w + 1);
-      int wid, wmeta;
-      const int T = plan_split(a, P, seq, lo, t, sp, ns, lane, wid, wmeta);
-      // per-head modes: every page brings its slot positions and presence masks
-      if (a.head_modes && lane < T) wmeta |= kMask;
-      const int kv0 = h0 / g, nkv = (h0 + nh - 1) / g - kv0 + 1;
+      int wid, wmeta, wfirst = 0, wlast = INT_MAX;
+      const int T = plan_split(a, P, seq, lo, t, sp, ns, lane, wid, wmeta, a.head_modes ? &wfirst : nullptr,
+                               a.head_modes ? &wlast : nullptr);
+      const int lo_local = max(0, t - w + 1);
+      // per-head modes: a page before the local window is read by the block's full heads
+      // only; a page across the window's start brings its slot positions
+      if (a.head_modes && lane < T) {
+        if (wlast < lo_local) wmeta |= kEarly;
+        else if (wfirst < lo_local) wmeta |= kMask;
+      }
       const int4 rb = make_int4(t, sp, ns, pre[q]);
       {  // the unit's query rows
         const int need = nh * D * 2;
@@ -767,11 +808,10 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
       // is a few shuffles and the copy
       uint64_t pg_src = 0;  // the page
       int pg_geo = 0;       // slice bytes | KV slices per stage << 20
-      // extra bytes of a masked page's stage: positions, and per-head modes' presence masks
-      const int maskx = a.head_modes ? a.maskb + 16 : 0;
+      const unsigned pg_need = wlast < lo_local ? need_full : need_any;  // the KV heads it brings
       if (lane < T) {
         const int c = wmeta & 3, slice = a.slice[c];
-        const int posb = (wmeta & kMask) ? 4 * P + maskx : 0;
+        const int posb = (wmeta & kMask) ? 4 * P : 0;
         pg_src = reinterpret_cast<uint64_t>(a.pool[c] + static_cast<int64_t>(wid) * a.page_bytes[c]);
         pg_geo = slice | (max(1, (R / 2 - posb) / slice) << 20);
       }
@@ -779,13 +819,13 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
         const uint8_t* page = reinterpret_cast<const uint8_t*>(__shfl_sync(0xffffffffu, pg_src, j));
         const int geo = __shfl_sync(0xffffffffu, pg_geo, j);
         const int pm = __shfl_sync(0xffffffffu, wmeta, j);
+        const unsigned needed = __shfl_sync(0xffffffffu, pg_need, j);
         const int slice = geo & 0xfffff, maxk = geo >> 20;
-        for (int k0 = 0; k0 < nkv; k0 += maxk) {
-          const int nk = min(maxk, nkv - k0);
-          // the presence masks of KV heads kv0 + k0 .. + nk - 1, from a 16-byte boundary
-          const int mlo = (8 * (kv0 + k0)) & ~15, mhi = (8 * (kv0 + k0 + nk) + 15) & ~15;
-          const int mb = a.head_modes ? mhi - mlo : 0;
-          const int posb = (pm & kMask) ? 4 * P + mb : 0;
+        // one stage per run of consecutive needed KV heads, at most maxk slices each
+        for (int k0 = __ffs(needed) - 1; k0 >= 0 && k0 < nkv;) {
+          int nk = 1;
+          while (nk < maxk && k0 + nk < nkv && ((needed >> (k0 + nk)) & 1u)) ++nk;
+          const int posb = (pm & kMask) ? 4 * P : 0;
           const int need = nk * slice + posb;
           int taken = 0;
           const int off = reserve(need, taken);
@@ -793,17 +833,16 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
             ok = false;
             break;
           }
-          const bool last = j == T - 1 && k0 + nk >= nkv;
+          const unsigned later = needed >> (k0 + nk);  // needed KV heads after this stage
+          const bool last = j == T - 1 && later == 0;
           const int meta = pm | (last ? kLast : 0) | (qb << 16);
           const uint32_t slot =
               push(make_int4(meta, off, q, lo), rb, make_int4(k0, nk, posb ? off + nk * slice : -1, slice), taken, need);
           if (lane == 0) {
             bulk_g2s(cr.ring + off, page + a.hdr + static_cast<int64_t>(kv0 + k0) * slice, nk * slice, &cr.full[slot]);
-            if (posb) bulk_g2s(cr.ring + off + nk * slice, page, 4 * P, &cr.full[slot]);
-            if (posb && mb)
-              bulk_g2s(cr.ring + off + nk * slice + 4 * P,
-                       page + a.hdr + static_cast<int64_t>(a.Hkv) * slice + mlo, mb, &cr.full[slot]);
+            if (posb) bulk_g2s(cr.ring + off + nk * slice, page, posb, &cr.full[slot]);
           }
+          k0 = later ? k0 + nk + __ffs(later) - 1 : nkv;
         }
       }
       if (!ok) break;
@@ -967,7 +1006,7 @@ __device__ __forceinline__ void finish_unit(const AttnKernelArgs& ka, LaneState<
   store_or_merge<D>(ka, st.acc, part * E + DPL * kl, M, L, sp, qi, qh, nsplit, base, lane);
 }
 
-template <int D, int P, int E>
+template <int D, int P, int E, bool HM>
 __device__ __forceinline__ void run_consumer_cc(const AttnKernelArgs& ka, const CtaRing& cr, int cw, int lane) {
   constexpr int LPK = D / E;     // lanes per key
   constexpr int KPI = 32 / LPK;  // keys per warp iteration
@@ -984,7 +1023,8 @@ __device__ __forceinline__ void run_consumer_cc(const AttnKernelArgs& ka, const 
 #pragma unroll
   for (int j = 0; j < E; ++j) st.acc[j] = 0.f;
   // the current unit
-  int u_q = 0, u_h = 0, u_kvi = 0, u_kv0 = 0, u_lo = 0, u_hi = 0, u_sp = 0, u_ns = 1, u_base = 0;
+  int u_q = 0, u_h = 0, u_kvi = 0, u_lo = 0, u_hi = 0, u_sp = 0, u_ns = 1, u_base = 0;
+  bool u_local = false;  // per-head modes: this warp's head is local (it skips early pages)
   bool active = false;
   for (uint32_t s = 0;; ++s) {
     const uint32_t slot = s % kStages;
@@ -1005,15 +1045,15 @@ __device__ __forceinline__ void run_consumer_cc(const AttnKernelArgs& ka, const 
       const int qb = meta >> 16;
       u_h = qb * kNcw + cw;
       active = u_h < a.Hq;
-      u_kv0 = (qb * kNcw) / g;
-      u_kvi = u_h / g - u_kv0;
+      u_kvi = u_h / g - (qb * kNcw) / g;
       u_q = ra.z;
       u_lo = ra.w;
       u_hi = rb.x;
       u_sp = rb.y;
       u_ns = rb.z;
       u_base = rb.w;
-      if (a.head_modes && active) {  // this head's own mode: {head modes, local lo}
+      u_local = false;
+      if (HM && active) {  // this head's own mode: {head modes, local lo}
         const int4 rq = lds128i(rec + 32);
         const int hm = (rq.x >> (2 * cw)) & 3;
         if (hm == TRR_MODE_SKIP) {  // a zero row (written once, by split 0), no merge
@@ -1023,6 +1063,7 @@ __device__ __forceinline__ void run_consumer_cc(const AttnKernelArgs& ka, const 
           active = false;
         } else if (hm == TRR_MODE_LOCAL) {
           u_lo = rq.y;
+          u_local = true;
         }
       }
       cur_cls = 3;  // the neutral scale is class 16's
@@ -1051,7 +1092,7 @@ __device__ __forceinline__ void run_consumer_cc(const AttnKernelArgs& ka, const 
       }
     } else if (active) {
       const int4 rc = lds128i(rec + 32);
-      if (u_kvi >= rc.x && u_kvi < rc.x + rc.y) {
+      if (u_kvi >= rc.x && u_kvi < rc.x + rc.y && !(HM && u_local && (meta & kEarly))) {
         const int cls = meta & 3, fill = (meta >> 2) & 127;
         if (cls != cur_cls) {
           rescale_dyn(qp, st.acc, cur_cls, cls);
@@ -1060,17 +1101,17 @@ __device__ __forceinline__ void run_consumer_cc(const AttnKernelArgs& ka, const 
         const uint32_t s0 = smem_u32(cr.ring + ra.y + (u_kvi - rc.x) * rc.w);
         const bool masked = meta & kMask;
         const uint32_t sp = masked ? smem_u32(cr.ring + rc.z) : s0;
-        uint64_t pm = ~0ull;  // per-head modes: this KV head's presence mask, after the
-                              // positions; the stage's masks start at a 16-byte boundary
-        if (a.head_modes) {
-          const uint2 m2 = lds64(sp + 4 * P + 8 * ((u_kvi - rc.x) + ((u_kv0 + rc.x) & 1)));
+        uint64_t pm = ~0ull;  // per-head modes: this KV head's presence mask, which ends
+                              // its slice
+        if (HM) {
+          const uint2 m2 = lds64(s0 + rc.w - a.maskb);
           pm = (static_cast<uint64_t>(m2.y) << 32) | m2.x;
         }
         switch (cls) {
-          case 0: consume_page<D, 2, P / KPI, E>(s0, sp, masked, pm, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
-          case 1: consume_page<D, 4, P / KPI, E>(s0, sp, masked, pm, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
-          case 2: consume_page<D, 8, P / KPI, E>(s0, sp, masked, pm, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
-          default: consume_page<D, 16, P / KPI, E>(s0, sp, masked, pm, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
+          case 0: consume_page<D, 2, P / KPI, E, HM>(s0, sp, masked, pm, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
+          case 1: consume_page<D, 4, P / KPI, E, HM>(s0, sp, masked, pm, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
+          case 2: consume_page<D, 8, P / KPI, E, HM>(s0, sp, masked, pm, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
+          default: consume_page<D, 16, P / KPI, E, HM>(s0, sp, masked, pm, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
         }
       }
     }
@@ -1652,8 +1693,9 @@ __device__ __forceinline__ void attn_epilogue(const LayerArgs& a) {
   }
 }
 
-// CUDA-core path: units of kNcw query heads, one per consumer warp.
-template <int D, int P>
+// CUDA-core path: units of kNcw query heads, one per consumer warp; HM: per-head modes
+// (presence masks read with every page).
+template <int D, int P, bool HM>
 __global__ void __launch_bounds__(32 * (kNcw + 1), cc_ctas_per_sm(D))
     attn_kernel(const __grid_constant__ AttnKernelArgs ka) {
   extern __shared__ __align__(128) uint8_t smem[];
@@ -1662,7 +1704,7 @@ __global__ void __launch_bounds__(32 * (kNcw + 1), cc_ctas_per_sm(D))
   int* pre;
   const CtaRing cr = attn_prologue(ka, smem, P, NQB, pre);
   if (warp == 0) run_producer<D>(ka, P, NQB, pre, cr, lane);
-  else run_consumer_cc<D, P, cc_elems(D)>(ka, cr, warp - 1, lane);
+  else run_consumer_cc<D, P, cc_elems(D), HM>(ka, cr, warp - 1, lane);
   attn_epilogue(ka.a);
 }
 
@@ -1776,12 +1818,18 @@ cudaError_t attn_configure() {
     int ctas;
   };
   const K kernels[] = {
-      {reinterpret_cast<const void*>(attn_kernel<64, 16>), cc_ctas_per_sm(64)},
-      {reinterpret_cast<const void*>(attn_kernel<64, 32>), cc_ctas_per_sm(64)},
-      {reinterpret_cast<const void*>(attn_kernel<64, 64>), cc_ctas_per_sm(64)},
-      {reinterpret_cast<const void*>(attn_kernel<128, 16>), cc_ctas_per_sm(128)},
-      {reinterpret_cast<const void*>(attn_kernel<128, 32>), cc_ctas_per_sm(128)},
-      {reinterpret_cast<const void*>(attn_kernel<128, 64>), cc_ctas_per_sm(128)},
+      {reinterpret_cast<const void*>(attn_kernel<64, 16, false>), cc_ctas_per_sm(64)},
+      {reinterpret_cast<const void*>(attn_kernel<64, 32, false>), cc_ctas_per_sm(64)},
+      {reinterpret_cast<const void*>(attn_kernel<64, 64, false>), cc_ctas_per_sm(64)},
+      {reinterpret_cast<const void*>(attn_kernel<128, 16, false>), cc_ctas_per_sm(128)},
+      {reinterpret_cast<const void*>(attn_kernel<128, 32, false>), cc_ctas_per_sm(128)},
+      {reinterpret_cast<const void*>(attn_kernel<128, 64, false>), cc_ctas_per_sm(128)},
+      {reinterpret_cast<const void*>(attn_kernel<64, 16, true>), cc_ctas_per_sm(64)},
+      {reinterpret_cast<const void*>(attn_kernel<64, 32, true>), cc_ctas_per_sm(64)},
+      {reinterpret_cast<const void*>(attn_kernel<64, 64, true>), cc_ctas_per_sm(64)},
+      {reinterpret_cast<const void*>(attn_kernel<128, 16, true>), cc_ctas_per_sm(128)},
+      {reinterpret_cast<const void*>(attn_kernel<128, 32, true>), cc_ctas_per_sm(128)},
+      {reinterpret_cast<const void*>(attn_kernel<128, 64, true>), cc_ctas_per_sm(128)},
       {reinterpret_cast<const void*>(attn_mma_kernel<64, 1>), kMmaCtasPerSm},
       {reinterpret_cast<const void*>(attn_mma_kernel<64, 2>), kMmaCtasPerSm},
       {reinterpret_cast<const void*>(attn_mma_kernel<128, 1>), kMmaCtasPerSm},
@@ -1807,7 +1855,7 @@ static bool use_mma(const Layout& l) {
 static int attn_ring_bytes(const Layout& l, int n, int hpu, int scr_floats, int limit) {
   const int fixed = AttnSmem(0, n, scr_floats).total;
   const int ring = (limit - fixed) / 128 * 128;
-  const int widest = static_cast<int>(l.slice[3]) + 4 * l.P + (l.head_modes ? static_cast<int>(l.maskb) + 16 : 0);
+  const int widest = static_cast<int>(l.slice[3]) + 4 * l.P;
   const int qrows = hpu * 2 * l.d;
   if (ring < std::max(widest, qrows)) return -1;
   return ring;
@@ -1838,14 +1886,24 @@ static cudaError_t launch_one(const Layout& l, const AttnKernelArgs& ka, int num
   }
   // one kernel per head size and page size: the page loop unrolls, and a kernel's code
   // holds only the four width classes it can meet
-  if (l.d == 64) {
-    if (l.P == 16) return launch_pdl(attn_kernel<64, 16>, grid, block, sm, s, k);
-    if (l.P == 32) return launch_pdl(attn_kernel<64, 32>, grid, block, sm, s, k);
-    return launch_pdl(attn_kernel<64, 64>, grid, block, sm, s, k);
+  if (l.head_modes) {
+    if (l.d == 64) {
+      if (l.P == 16) return launch_pdl(attn_kernel<64, 16, true>, grid, block, sm, s, k);
+      if (l.P == 32) return launch_pdl(attn_kernel<64, 32, true>, grid, block, sm, s, k);
+      return launch_pdl(attn_kernel<64, 64, true>, grid, block, sm, s, k);
+    }
+    if (l.P == 16) return launch_pdl(attn_kernel<128, 16, true>, grid, block, sm, s, k);
+    if (l.P == 32) return launch_pdl(attn_kernel<128, 32, true>, grid, block, sm, s, k);
+    return launch_pdl(attn_kernel<128, 64, true>, grid, block, sm, s, k);
   }
-  if (l.P == 16) return launch_pdl(attn_kernel<128, 16>, grid, block, sm, s, k);
-  if (l.P == 32) return launch_pdl(attn_kernel<128, 32>, grid, block, sm, s, k);
-  return launch_pdl(attn_kernel<128, 64>, grid, block, sm, s, k);
+  if (l.d == 64) {
+    if (l.P == 16) return launch_pdl(attn_kernel<64, 16, false>, grid, block, sm, s, k);
+    if (l.P == 32) return launch_pdl(attn_kernel<64, 32, false>, grid, block, sm, s, k);
+    return launch_pdl(attn_kernel<64, 64, false>, grid, block, sm, s, k);
+  }
+  if (l.P == 16) return launch_pdl(attn_kernel<128, 16, false>, grid, block, sm, s, k);
+  if (l.P == 32) return launch_pdl(attn_kernel<128, 32, false>, grid, block, sm, s, k);
+  return launch_pdl(attn_kernel<128, 64, false>, grid, block, sm, s, k);
 }
 
 // The launches of an attention call with the given scratch views in `a`; *launches

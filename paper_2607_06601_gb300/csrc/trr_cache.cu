@@ -76,13 +76,14 @@ static trr_status make_layout(const trr_cache_config* c, Layout* l) {
   l->skip_writes_kv = c->skip_writes_kv;
   l->head_modes = c->head_modes;
   l->hdr = roundup(4 * static_cast<int64_t>(l->P), 128);
-  // per-head modes: one 64-bit presence mask per KV head after the slices of a page
-  l->maskb = l->head_modes ? roundup(8 * static_cast<int64_t>(l->Hkv), 16) : 0;
+  // per-head modes: each KV head's slice of a page ends with 16 bytes holding its 64-bit
+  // presence mask, so that the copy of a slice brings its mask
+  l->maskb = l->head_modes ? 16 : 0;
   for (int k = 0; k < kClasses; ++k) {
     const int b = bits_of_class(k);
     l->tokb[k] = b < 16 ? 2 * (l->d * b / 8) + 2 * (l->d / l->G) * 4 : 4 * l->d;
-    l->slice[k] = l->P * l->tokb[k];
-    l->page_bytes[k] = roundup(l->hdr + l->Hkv * l->slice[k] + l->maskb, 128);
+    l->slice[k] = l->P * l->tokb[k] + l->maskb;
+    l->page_bytes[k] = roundup(l->hdr + l->Hkv * l->slice[k], 128);
   }
   l->units = l->Hq;
   // splits per query: at least pos_split key positions each (split_bytes of 8-bit

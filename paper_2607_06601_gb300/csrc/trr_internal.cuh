@@ -105,8 +105,8 @@ inline Views make_views(const Layout& l, void* base) {
 // Everything a kernel needs about one layer of one cache, passed by value.
 struct LayerArgs {
   int layer, S, Hq, Hkv, d, G, P, maxctx, MP, W32, units, pos_split, s_cap, cnt_stride, split_bytes, skip_writes_kv;
-  int head_modes;      // modes are [n][Hq]; pages end with a presence mask per KV head
-  int maskb;           // bytes of a page's presence masks (0 without head_modes)
+  int head_modes;      // modes are [n][Hq]; each KV head's slice ends with its presence mask
+  int maskb;           // bytes that end a slice for its presence mask (16, or 0 without head_modes)
   int cap[kClasses];
   int hdr;
   int slice[kClasses];
