@@ -11,7 +11,7 @@ import torch
 
 from paper_2607_06601_gb300 import trr
 from paper_2607_06601_gb300 import workloads as wl
-from tests._parity import Pair, dev
+from tests._parity import Pair, check_attention, dev
 
 pytestmark = pytest.mark.gpu
 
@@ -206,3 +206,23 @@ def test_160m_shape_per_head():
     pair.check_regions()
     q = np.stack([wl.q(spec, 0, s, last, ctx)[0] for s in range(B)])
     pair.attend(0, range(B), [last] * B, q, hm, window_scalar=spec.window)
+
+
+def test_static_scratch_entry_with_head_modes():
+    """trr_decode_attn_static on a per-head cache: the oracle's rows within tolerance and
+    the same bits as trr_decode_attn, on two calls in a row."""
+    rng = np.random.default_rng(61)
+    ctxs = [300, 120]
+    pair = _setup(rng, 64, 32, 16, 8, 4, ctxs, 1024)
+    seqs, ts, hm, ws = _queries(rng, ctxs, 8)
+    q = wl.bf16_bits(rng.standard_normal((len(seqs), 8, 64), dtype=np.float32))
+    got, ref = pair.attend(0, seqs, ts, q, hm, windows=ws)
+    args = (dev(np.asarray(seqs, np.int32), torch.int32), dev(np.asarray(ts, np.int32), torch.int32),
+            dev(q, torch.bfloat16), dev(hm, torch.uint8), dev(np.asarray(ws, np.int32), torch.int32))
+    for _ in range(2):
+        out = torch.full((len(seqs), 8, 64), float("nan"), dtype=torch.bfloat16, device="cuda")
+        trr.trr_decode_attn_static(pair.gpu.handle, 0, *args, 0, 0.0, out)
+        st = out.float().cpu().numpy().astype(np.float64)
+        check_attention(st, ref, hm)
+        assert np.array_equal(st, got)
+    assert pair.gpu.status() == 0
