@@ -61,9 +61,10 @@ def token_bytes(d, G):
 class Accounting:
     """Algorithmic bytes / attended keys of decode queries, from the seeded maps."""
 
-    def __init__(self, spec, d, G, Hq, Hkv, window, P=PAGE):
+    def __init__(self, spec, d, G, Hq, Hkv, window, P=PAGE, skip_writes_kv=0):
         self.tokb = np.array(token_bytes(d, G), dtype=np.int64)
         self.Hq, self.Hkv, self.d, self.window, self.P = Hq, Hkv, d, window, P
+        self.swk = int(skip_writes_kv)  # 1: skip tokens store KV too
 
     def query(self, bits_row, modes_row, t):
         """(bytes, attended keys, pages) of one query at position t of one sequence
@@ -73,7 +74,7 @@ class Accounting:
         if m == 0:
             return qo, 0, 0                           # only the zero O row is written
         lo = 0 if m == 2 else max(0, t - self.window + 1)
-        stored = modes_row[:t + 1] != 0
+        stored = (modes_row[:t + 1] != 0) | bool(self.swk)
         b_row = bits_row[:t + 1]
         total, keys, pages = 2 * qo, 0, 0
         for c, b in enumerate(BITS):
@@ -101,7 +102,7 @@ class Accounting:
             return qo, 0, 0
         lo_q = 0 if (mrow == 2).any() else max(0, t - self.window + 1)
         b_row = bits_row[:t + 1]
-        stored = (modes_rows[:t + 1] != 0).reshape(t + 1, self.Hkv, g).any(2)  # [t+1][Hkv]
+        stored = (modes_rows[:t + 1] != 0).reshape(t + 1, self.Hkv, g).any(2) | bool(self.swk)  # [t+1][Hkv]
         took = stored.any(1)
         total = qo + 2 * self.d * int(np.count_nonzero(mrow))
         keys = pages = nkv = 0
@@ -307,6 +308,7 @@ class Bench:
             s.num_layers, s.batch, s.num_q_heads, s.num_kv_heads, s.head_dim, s.group_size)
         self.window = s.window
         self.head_modes = int(getattr(args, "head_modes", False))
+        self.swk = int(getattr(args, "skip_writes_kv", False))
         self.e2e_warm, self.e2e_steps = 2, 2 * min(args.steps, 10)
         # the routed step decides per token: not run with per-head modes
         self.routed_warm, self.routed_steps = (0, 0) if self.head_modes else (2, min(args.steps, 10))
@@ -315,7 +317,7 @@ class Bench:
         self.grow = 32                                   # tokens a sequence may grow
         self.R = max(1, math.ceil(self.total_steps / self.grow))
         self.P = args.page_size or PAGE
-        self.acct = Accounting(s, self.d, self.G, self.Hq, self.Hkv, self.window, self.P)
+        self.acct = Accounting(s, self.d, self.G, self.Hq, self.Hkv, self.window, self.P, self.swk)
         self.ctx = wl.contexts(s)                       # prebuilt context per sequence
         self.maxctx = int(self.ctx.max()) + math.ceil(self.total_steps / self.R) + 1
         self.dev = torch.device("cuda", torch.cuda.current_device())
@@ -343,11 +345,13 @@ class Bench:
                 bits, modes = self.all_maps[l][r]
                 for s in range(B):
                     stored = (modes[s] != 0).any(-1) if self.head_modes else modes[s] != 0
+                    stored = stored | bool(self.swk)
                     for c, b in enumerate(BITS):
                         caps[c] += -(-int(np.count_nonzero(stored & (bits[s] == b))) // self.P) + 1
         self.cache = trr.Cache(L, S, self.Hq, self.Hkv, self.d, self.G, self.P, self.maxctx,
                                [int(c) for c in caps], max_append=1024, max_queries=max(B, 64),
-                               split_bytes=self.args.split_bytes, head_modes=self.head_modes)
+                               split_bytes=self.args.split_bytes, head_modes=self.head_modes,
+                               skip_writes_kv=self.swk)
         # prebuild every sequence's context (untimed), K/V drawn on the device
         gen = torch.Generator(device=self.dev)
         self.prebuild_calls = 0
@@ -450,7 +454,7 @@ class Bench:
         n = 0
         for l, x in enumerate(st["layers"]):
             trr.trr_route_decisions(x["ml"], x["bl"], x["pos"], self.window, self.Hq, self.d, self.Hkv,
-                                    totals=totals, stream=stream)
+                                    skip_writes_kv=self.swk, totals=totals, stream=stream)
             c.append_routed(l, x["seqs"], x["pos"], x["k"], x["v"], x["bl"], x["ml"], stream=stream)
             n += 1 + c.launches()
             c.decode_attn_routed(l, x["seqs"], x["pos"], x["q"], x["ml"], window_scalar=self.window,
@@ -720,7 +724,8 @@ def run_gpu(args):
     value = job_bytes / (ms * 1e-3) / 1e9
     result = None
     if rank == 0:
-        cpu = cpu_baseline(bench) if (world == 1 and not args.no_cpu_baseline and not bench.head_modes) else None
+        cpu = (cpu_baseline(bench) if (world == 1 and not args.no_cpu_baseline and not bench.head_modes
+                                       and not bench.swk) else None)
         result = {
             "metric": METRIC, "value": round(value, 2), "unit": UNIT, "n_gpus": world,
             "steps": K, "warmup": W, "ms_per_step": round(ms / K, 5), "higher_is_better": True,
@@ -732,6 +737,7 @@ def run_gpu(args):
                 "kv_storage": "per-token 2/4/8-bit codes + fp16 scale/zero, or bf16; fp32 accumulation",
                 "modes": "per (token, query head), presence mask per KV head" if bench.head_modes
                          else "per token",
+                "skip_tokens_store_kv": bool(bench.swk),
                 "global_batch": bench.B * world, "replicas": bench.R,
                 "l2": "inputs larger than L2: every step reads its replica's "
                       f"{rank_bytes / K / 1e6:.0f} MB, replicas rotate",
@@ -750,7 +756,7 @@ def run_gpu(args):
                     "eager_how": "the same steps called one by one from Python, no graph (host-launch bound)"},
             "roofline": {"bound": "hbm", "achieved": round(achieved, 2), "peak": peak,
                          "unit": "GB/s", "frac": round(achieved / peak, 4),
-                         "traffic": None if bench.head_modes else ncu_traffic(args.workload),
+                         "traffic": None if (bench.head_modes or bench.swk) else ncu_traffic(args.workload),
                          "peak_kind": peak_kind,
                          "kernel": "trr_decode_attn call (attn_kernel, one launch)",
                          "bytes_per_call": round(avg_bytes), "us_per_call": round(avg_ms * 1e3, 3)},
@@ -877,6 +883,9 @@ def main():
                     help="tokens per cache page (0: 32)")
     ap.add_argument("--split-bytes", type=int, default=0,
                     help="target KV bytes per split-K work item (0: the library default)")
+    ap.add_argument("--skip-writes-kv", action="store_true",
+                    help="skip tokens store their KV too (the paper's Principle 1 reading; default: "
+                         "they store nothing); no CPU baseline")
     ap.add_argument("--head-modes", action="store_true",
                     help="a mode per (token, query head), drawn from the workload's mode mix "
                          "(Sec. 3.2(A)); no routed step and no CPU baseline")
