@@ -314,12 +314,15 @@ class Bench:
         self.routed_warm, self.routed_steps = (0, 0) if self.head_modes else (2, min(args.steps, 10))
         self.total_steps = (args.warmup + 2 * args.steps + self.e2e_warm + self.e2e_steps + self.routed_warm +
                             self.routed_steps)
+        self.C = max(1, int(getattr(args, "chunk", 1)))  # new tokens (and queries) per sequence per step
+        if self.B * self.C > 1024:
+            raise SystemExit("batch x chunk must be at most 1024 (one append call per layer)")
         self.grow = 32                                   # tokens a sequence may grow
-        self.R = max(1, math.ceil(self.total_steps / self.grow))
+        self.R = max(1, math.ceil(self.total_steps * self.C / self.grow))
         self.P = args.page_size or PAGE
         self.acct = Accounting(s, self.d, self.G, self.Hq, self.Hkv, self.window, self.P, self.swk)
         self.ctx = wl.contexts(s)                       # prebuilt context per sequence
-        self.maxctx = int(self.ctx.max()) + math.ceil(self.total_steps / self.R) + 1
+        self.maxctx = int(self.ctx.max()) + math.ceil(self.total_steps / self.R) * self.C + 1
         self.dev = torch.device("cuda", torch.cuda.current_device())
 
     # ---- maps
@@ -349,7 +352,7 @@ class Bench:
                     for c, b in enumerate(BITS):
                         caps[c] += -(-int(np.count_nonzero(stored & (bits[s] == b))) // self.P) + 1
         self.cache = trr.Cache(L, S, self.Hq, self.Hkv, self.d, self.G, self.P, self.maxctx,
-                               [int(c) for c in caps], max_append=1024, max_queries=max(B, 64),
+                               [int(c) for c in caps], max_append=1024, max_queries=max(B * self.C, 64),
                                split_bytes=self.args.split_bytes, head_modes=self.head_modes,
                                skip_writes_kv=self.swk)
         # prebuild every sequence's context (untimed), K/V drawn on the device
@@ -401,33 +404,35 @@ class Bench:
         gen = torch.Generator(device=self.dev)
         layers = []
         nbytes = keys = 0
+        n = self.B * self.C  # entries (and queries) per layer: C consecutive tokens per sequence
+        srow = np.repeat(np.arange(self.B), self.C)
         for l in range(self.L):
             bits, modes = self.all_maps[l][r]
-            pos = (self.ctx + grow).astype(np.int32)
-            seqs = (r * self.B + np.arange(self.B)).astype(np.int32)
-            b = bits[np.arange(self.B), pos]
-            m = modes[np.arange(self.B), pos]
+            pos = (self.ctx[srow] + grow * self.C + np.tile(np.arange(self.C), self.B)).astype(np.int32)
+            seqs = (r * self.B + srow).astype(np.int32)
+            b = bits[srow, pos]
+            m = modes[srow, pos]
             gen.manual_seed(_mix(self.spec.seed, 2, i, l))
             chl = torch.tensor(self.wl.outlier_channels(self.spec, l), dtype=torch.long, device=self.dev)
-            k, v = self._kv(self.B, gen, chl)
-            q = torch.randn((self.B, self.Hq, self.d), generator=gen, device=self.dev).to(torch.bfloat16)
-            for s in range(self.B):
-                acct = self.acct.query_heads if self.head_modes else self.acct.query
-                nb, nk, _ = acct(bits[s], modes[s], int(pos[s]))
+            k, v = self._kv(n, gen, chl)
+            q = torch.randn((n, self.Hq, self.d), generator=gen, device=self.dev).to(torch.bfloat16)
+            acct = self.acct.query_heads if self.head_modes else self.acct.query
+            for e in range(n):  # every query sees the chunk's tokens up to its own position
+                nb, nk, _ = acct(bits[srow[e]], modes[srow[e]], int(pos[e]))
                 nbytes += nb
                 keys += nk
             # router logits whose arg max is the seeded decision (the routed step)
-            ml = torch.rand((self.B, 3), generator=gen, device=self.dev) - 2.0
-            bl = torch.rand((self.B, 4), generator=gen, device=self.dev) - 2.0
+            ml = torch.rand((n, 3), generator=gen, device=self.dev) - 2.0
+            bl = torch.rand((n, 4), generator=gen, device=self.dev) - 2.0
             if not self.head_modes:
-                ml[torch.arange(self.B, device=self.dev), torch.from_numpy(m.astype(np.int64)).to(self.dev)] = 1.0
+                ml[torch.arange(n, device=self.dev), torch.from_numpy(m.astype(np.int64)).to(self.dev)] = 1.0
             bcls = np.array([BITS.index(int(x)) for x in b], dtype=np.int64)
-            bl[torch.arange(self.B, device=self.dev), torch.from_numpy(bcls).to(self.dev)] = 1.0
+            bl[torch.arange(n, device=self.dev), torch.from_numpy(bcls).to(self.dev)] = 1.0
             layers.append(dict(
                 seqs=torch.from_numpy(seqs).to(self.dev), pos=torch.from_numpy(pos).to(self.dev),
                 bits=torch.from_numpy(b).to(self.dev), modes=torch.from_numpy(np.ascontiguousarray(m)).to(self.dev),
                 k=k, v=v, q=q, ml=ml.contiguous(), bl=bl.contiguous(),
-                out=torch.empty((self.B, self.Hq, self.d), dtype=torch.bfloat16, device=self.dev)))
+                out=torch.empty((n, self.Hq, self.d), dtype=torch.bfloat16, device=self.dev)))
         attn_bytes_per_layer = nbytes / self.L
         return dict(layers=layers, bytes=nbytes, keys=keys, attn_bytes_per_layer=attn_bytes_per_layer)
 
@@ -725,7 +730,7 @@ def run_gpu(args):
     result = None
     if rank == 0:
         cpu = (cpu_baseline(bench) if (world == 1 and not args.no_cpu_baseline and not bench.head_modes
-                                       and not bench.swk) else None)
+                                       and not bench.swk and bench.C == 1) else None)
         result = {
             "metric": METRIC, "value": round(value, 2), "unit": UNIT, "n_gpus": world,
             "steps": K, "warmup": W, "ms_per_step": round(ms / K, 5), "higher_is_better": True,
@@ -738,6 +743,7 @@ def run_gpu(args):
                 "modes": "per (token, query head), presence mask per KV head" if bench.head_modes
                          else "per token",
                 "skip_tokens_store_kv": bool(bench.swk),
+                "queries_per_seq": bench.C,
                 "global_batch": bench.B * world, "replicas": bench.R,
                 "l2": "inputs larger than L2: every step reads its replica's "
                       f"{rank_bytes / K / 1e6:.0f} MB, replicas rotate",
@@ -756,7 +762,8 @@ def run_gpu(args):
                     "eager_how": "the same steps called one by one from Python, no graph (host-launch bound)"},
             "roofline": {"bound": "hbm", "achieved": round(achieved, 2), "peak": peak,
                          "unit": "GB/s", "frac": round(achieved / peak, 4),
-                         "traffic": None if (bench.head_modes or bench.swk) else ncu_traffic(args.workload),
+                         "traffic": None if (bench.head_modes or bench.swk or bench.C > 1)
+                         else ncu_traffic(args.workload),
                          "peak_kind": peak_kind,
                          "kernel": "trr_decode_attn call (attn_kernel, one launch)",
                          "bytes_per_call": round(avg_bytes), "us_per_call": round(avg_ms * 1e3, 3)},
@@ -775,7 +782,7 @@ def run_gpu(args):
 def describe_ctx(bench):
     c = bench.ctx
     lo, hi = int(c.min()), int(c.max())
-    grow = math.ceil(bench.total_steps / bench.R)
+    grow = math.ceil(bench.total_steps / bench.R) * bench.C
     base = f"{lo}" if lo == hi else f"{lo}-{hi}"
     return f"{base} (+ up to {grow} decoded)"
 
@@ -883,6 +890,9 @@ def main():
                     help="tokens per cache page (0: 32)")
     ap.add_argument("--split-bytes", type=int, default=0,
                     help="target KV bytes per split-K work item (0: the library default)")
+    ap.add_argument("--chunk", type=int, default=1,
+                    help="new tokens and queries per sequence per step (chunked decode / speculative "
+                         "verification: each query attends up to its own position); no CPU baseline")
     ap.add_argument("--skip-writes-kv", action="store_true",
                     help="skip tokens store their KV too (the paper's Principle 1 reading; default: "
                          "they store nothing); no CPU baseline")

@@ -287,3 +287,34 @@ def test_all2_full():
     pair.check_regions()
     q = wl.bf16_bits(rng.standard_normal((4, 8, 64), dtype=np.float32))
     pair.attend(0, range(4), [299, 200, 100, 0], q, [FULL] * 4)
+
+
+def test_chunked_decode_several_queries_per_sequence():
+    """Several queries of one sequence in one call (chunked decode, speculative
+    verification): each sequence appends a chunk of C tokens in one call, then its C
+    queries attend in one call, each up to its own position (causal inside the chunk),
+    with mixed modes and windows; chunks repeat so later ones see earlier ones."""
+    rng = np.random.default_rng(88)
+    S, Hq, Hkv, d, P, C = 4, 8, 8, 64, 32, 8
+    ctxs = [300, 64, 129, 1]
+    maxctx = max(ctxs) + 3 * C
+    pair = Pair(1, S, Hq, Hkv, d, 32, P, maxctx, [S * (maxctx // P + 2)] * 4)
+
+    def chunk(pos_of):  # one append call of every sequence's positions, then their queries
+        seqs = np.concatenate([[s] * len(pos_of[s]) for s in range(S)]).astype(np.int32)
+        pos = np.concatenate([pos_of[s] for s in range(S)]).astype(np.int32)
+        n = len(seqs)
+        modes = rng.choice(3, size=n, p=[0.2, 0.4, 0.4])
+        pair.append(0, seqs, pos, wl.bf16_bits(rng.standard_normal((n, Hkv, d), dtype=np.float32)),
+                    wl.bf16_bits(rng.standard_normal((n, Hkv, d), dtype=np.float32)),
+                    rng.choice([2, 4, 8, 16], size=n), modes)
+        return seqs, pos, modes
+
+    chunk([np.arange(c) for c in ctxs])  # the prefilled contexts
+    nxt = list(ctxs)
+    for _ in range(3):
+        seqs, pos, modes = chunk([np.arange(nxt[s], nxt[s] + C) for s in range(S)])
+        q = wl.bf16_bits(rng.standard_normal((len(seqs), Hq, d), dtype=np.float32))
+        pair.attend(0, seqs, pos, q, modes, windows=rng.choice([1, 3, 8, 40, 500], size=len(seqs)))
+        nxt = [x + C for x in nxt]
+    pair.check_regions()
