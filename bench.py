@@ -237,12 +237,17 @@ def measured_peaks():
 
 
 def kernel_source_digest():
-    """sha256 (16 hex digits) of the sources that decide what the attention kernel does:
-    the kernel, the cache layout and the shared header."""
+    """sha256 (16 hex digits) of the code that decides what the attention kernel does:
+    the kernel, the cache layout and the shared header, with comments and blank space
+    removed (a change of wording does not change the kernel)."""
     import hashlib
+    import re
     h = hashlib.sha256()
     for f in ("trr_attn.cu", "trr_cache.cu", "trr_internal.cuh"):
-        h.update(open(os.path.join(ROOT, "paper_2607_06601_gb300", "csrc", f), "rb").read())
+        src = open(os.path.join(ROOT, "paper_2607_06601_gb300", "csrc", f)).read()
+        src = re.sub(r"/\*.*?\*/", " ", src, flags=re.S)
+        src = re.sub(r"//[^\n]*", " ", src)
+        h.update(" ".join(src.split()).encode())
     return h.hexdigest()[:16]
 
 

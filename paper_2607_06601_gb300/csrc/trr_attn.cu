@@ -27,6 +27,12 @@
 //      the groups), each by the last arrival, which resets its counter.
 //   5. The last CTA to finish records the error of the lowest failing query.
 //
+// Per-head modes (a cache with head_modes): the query's widest head mode sizes its
+// splits; a unit reads the pages of its head block's widest mode (a block of local and
+// skip heads only its window's splits); every slice of a page ends with its KV head's
+// presence mask, which the consumer applies per key; pages before the window come only
+// for the KV heads a full head of the block reads; a skip head writes its zero row.
+//
 // CUDA-core dequantisation: k = z + c*s, so q.k = s * sum(q_i c_i) + z * sum(q_i).  A
 // code is masked in place (no shift) and its bits read as a binary32 subnormal,
 // c * 2^(e-149) where e is its bit offset; the query is pre-scaled per width class by
@@ -415,7 +421,9 @@ __host__ __device__ constexpr int attn_smem_limit(int ctas) {
 //   a = {meta, ring offset of the stage's bytes, query, lo}
 //   b = {hi (= t), split, splits, unit number of split 0}
 //   c = {first KV slice of the stage (block-relative), KV slices in it, ring offset of
-//        the page's slot positions or -1, bytes of one KV slice}
+//        the page's slot positions or -1, bytes of one KV slice}; in a query-rows
+//        stage {the block's head modes, 2 bits per head (per-head modes), the local
+//        window's first position, -1, 0}
 // meta = class | fill << 2 | flags | head block << 16.
 enum : int {
   kMask = 1 << 9,     // the page may hold keys outside [lo, hi]: positions follow the slices
