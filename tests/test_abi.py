@@ -60,3 +60,23 @@ def test_host_validation_without_gpu(lib):
     assert lib.trr_kv_append(None, 0, 0, None, None, None, None, None, None, None) == 1
     assert lib.trr_decode_attn(None, 0, 0, None, None, None, None, None, 0, 0.0, None, None) == 1
     assert lib.trr_last_launch_count(None) == 0
+
+
+def test_per_head_layout_matches_the_oracle(lib):
+    """With head_modes the library's pages grow by the presence masks exactly as the
+    oracle lays them out (16 bytes per KV head slice, pages rounded to 128): the required
+    bytes differ from the per-token cache's by the pools' difference alone."""
+    import oracle
+    base = dict(num_layers=2, max_seqs=8, num_q_heads=12, num_kv_heads=4, head_dim=64,
+                group_size=32, page_size=32, max_context=1024, pages_per_class=[10, 20, 30, 40])
+    tok = trr.trr_cache_required_bytes(trr.make_config(**base))
+    hed = trr.trr_cache_required_bytes(trr.make_config(**base, head_modes=1))
+    o0 = oracle.OracleCache(1, 1, 12, 4, 64, 32, 32, 64, [1] * 4, no_pool=True)
+    o1 = oracle.OracleCache(1, 1, 12, 4, 64, 32, 32, 64, [1] * 4, no_pool=True, head_modes=1)
+    grow = sum(cap * (o1.page_bytes(c) - o0.page_bytes(c)) for c, cap in enumerate(base["pages_per_class"]))
+    assert grow > 0 and o1.slice_bytes(0) == o0.slice_bytes(0) + 16
+    # the pools are 256-byte aligned regions: the difference is the pools' own up to that
+    assert abs((hed - tok) - grow) < 4 * 256
+    cfg = trr.make_config(**base, head_modes=2)
+    out = ctypes.c_uint64()
+    assert lib.trr_cache_required_bytes(ctypes.byref(cfg), ctypes.byref(out)) == 6  # not a mode setting
