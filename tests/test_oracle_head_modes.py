@@ -139,6 +139,16 @@ def test_brute_force_per_head_policies_mha_and_sampled_three_tokens():
     assert _brute(3, 2, 1, pick[:100], swk=1) == 100
 
 
+def test_brute_force_per_head_policies_two_query_groups():
+    """Four query heads over two KV heads (groups of 2): sampled per-head policies of
+    2-3 token contexts, so that a head's KV head (h // 2) differs from h and from h % 2."""
+    rng = np.random.default_rng(11)
+    pol = list(itertools.product([2, 4, 8, 16], itertools.product([SKIP, LOCAL, FULL], repeat=4)))
+    for T, n in ((2, 300), (3, 150)):
+        cases = [tuple(pol[i] for i in rng.choice(len(pol), size=T)) for _ in range(n)]
+        assert _brute(T, 4, 2, cases) == n
+
+
 def test_presence_bits_follow_the_reading_heads():
     """The page's mask bits, read from its bytes: set for the KV heads that a
     non-skip query head reads, for every stored token, and for nothing else."""
@@ -186,6 +196,8 @@ def test_per_head_error_contract():
     q = bf16_bits(np.ones((2, Hq, d), dtype=np.float32))
     st, out = o.decode_attn(0, [0, 0], [0, 0], q, [FULL] * 4 + [LOCAL, SKIP, FULL, SKIP], window_scalar=0)
     assert st == 1 and not out[1].any() and out[0].any()   # local head with w < 1: that query fails
+    st, out = o.decode_attn(0, [0, 0], [0, 0], q, [FULL] * 4 + [FULL, SKIP, LOCAL, SKIP], window_scalar=0)
+    assert st == 1 and not out[1].any() and out[0].any()   # the local head need not be the first
     st, out = o.decode_attn(0, [0], [0], q[:1], [SKIP, FULL, SKIP, SKIP], window_scalar=0)
     # head 1 reads KV head 0, which token 0 stores (head 0 full): a row; skip heads: zeros
     assert st == 0 and out[0, 1].any() and not out[0, [0, 2, 3]].any()
