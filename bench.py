@@ -236,6 +236,41 @@ def measured_peaks():
         return 6800.0, "fallback"
 
 
+def l2_cache_bytes():
+    """L2 size of the current device (cudaDevAttrL2CacheSize)."""
+    import torch
+    props = torch.cuda.get_device_properties(torch.cuda.current_device())
+    size = getattr(props, "L2_cache_size", 0)
+    if size:
+        return int(size)
+    rt = CudaRt()
+    v = ctypes.c_int()
+    rt.lib.cudaDeviceGetAttribute(ctypes.byref(v), 89, torch.cuda.current_device())
+    return int(v.value)
+
+
+def expected_step_bytes(spec, ctx, P, swk=0, chunk=1):
+    """Expected algorithmic attention bytes of one step (every layer, every sequence) from
+    the workload's bit and mode mixes: the replica count is sized from it."""
+    tokb = np.array(token_bytes(spec.head_dim, spec.group_size), dtype=np.float64)
+    p_bits = np.array(spec.bits_p, dtype=np.float64)
+    p_skip, p_local, p_full = spec.modes_p
+    stored = 1.0 if swk else 1.0 - p_skip
+    per_pos = stored * (float(p_bits @ tokb) * spec.num_kv_heads + 4)
+    keys = p_full * ctx.astype(np.float64) + p_local * np.minimum(ctx, spec.window)
+    qo = 2 * spec.num_q_heads * spec.head_dim
+    per_layer = float(np.sum(keys * per_pos)) + len(ctx) * (qo * (2 - p_skip))
+    return per_layer * spec.num_layers * chunk
+
+
+def expected_cache_bytes(spec, ctx, P, swk=0):
+    """Expected page bytes of one replica of the batch over every layer."""
+    tokb = np.array(token_bytes(spec.head_dim, spec.group_size), dtype=np.float64)
+    stored = 1.0 if swk else 1.0 - spec.modes_p[0]
+    per_tok = stored * float(np.array(spec.bits_p) @ tokb) * spec.num_kv_heads
+    return float(np.sum(ctx)) * per_tok * spec.num_layers * 1.1
+
+
 def kernel_source_digest():
     """sha256 (16 hex digits) of the code that decides what the attention kernel does:
     the kernel, the cache layout and the shared header, with comments and blank space
@@ -317,16 +352,31 @@ class Bench:
         self.e2e_warm, self.e2e_steps = 2, 2 * min(args.steps, 10)
         # the routed step decides per token: not run with per-head modes
         self.routed_warm, self.routed_steps = (0, 0) if self.head_modes else (2, min(args.steps, 10))
+        # the same steps as separate trr_kv_append / trr_decode_attn calls, for comparison
+        self.sep_warm, self.sep_steps = 2, min(args.steps, 10)
+        if getattr(args, "light", False):  # timed steps and per-call attribution only
+            self.e2e_warm = self.e2e_steps = self.routed_warm = self.routed_steps = 0
+            self.sep_warm = self.sep_steps = 0
         self.total_steps = (args.warmup + 2 * args.steps + self.e2e_warm + self.e2e_steps + self.routed_warm +
-                            self.routed_steps)
+                            self.routed_steps + self.sep_warm + self.sep_steps)
         self.C = max(1, int(getattr(args, "chunk", 1)))  # new tokens (and queries) per sequence per step
         if self.B * self.C > 1024:
             raise SystemExit("batch x chunk must be at most 1024 (one append call per layer)")
         self.grow = 32                                   # tokens a sequence may grow
-        self.R = max(1, math.ceil(self.total_steps * self.C / self.grow))
         self.P = args.page_size or PAGE
         self.acct = Accounting(s, self.d, self.G, self.Hq, self.Hkv, self.window, self.P, self.swk)
         self.ctx = wl.contexts(s)                       # prebuilt context per sequence
+        # Replicas: enough that a sequence grows by at most `grow` tokens over the run, and
+        # that the steps between two visits of a replica read at least 3 x L2, so that no
+        # step finds its bytes in L2 (capped by device memory; a workload too small for
+        # that is reported as such).
+        self.l2_bytes = l2_cache_bytes()
+        self.est_step_bytes = expected_step_bytes(s, self.ctx, self.P, self.swk, self.C)
+        r_grow = max(1, math.ceil(self.total_steps * self.C / self.grow))
+        r_l2 = math.ceil(3 * self.l2_bytes / max(1.0, self.est_step_bytes))
+        cache_per_replica = max(1.0, expected_cache_bytes(s, self.ctx, self.P, self.swk))
+        r_mem = max(1, int(getattr(args, "cache_budget_gb", 120.0) * 1e9 // cache_per_replica))
+        self.R = max(r_grow, min(r_l2, r_mem, 64))
         self.maxctx = int(self.ctx.max()) + math.ceil(self.total_steps / self.R) * self.C + 1
         self.dev = torch.device("cuda", torch.cuda.current_device())
 
@@ -442,17 +492,28 @@ class Bench:
         return dict(layers=layers, bytes=nbytes, keys=keys, attn_bytes_per_layer=attn_bytes_per_layer)
 
     # ---- one step through the C ABI
-    def run_step(self, st, events=None, stream=None):
+    def run_step(self, st, events=None, stream=None, separate=False):
+        """Every layer's decode step: one trr_decode_step call (append and attention in
+        one kernel), or with `separate` trr_kv_append then trr_decode_attn.  `events`
+        brackets the attention of every layer (the whole decode-step call)."""
         c = self.cache
         n = 0
+        fused = not separate and self.C == 1 and not self.head_modes and self.B <= 256
         for l, x in enumerate(st["layers"]):
-            c.append(l, x["seqs"], x["pos"], x["k"], x["v"], x["bits"], x["modes"], stream=stream)
-            n += c.launches()
-            if events is not None:
-                events[0](l)
-            c.decode_attn(l, x["seqs"], x["pos"], x["q"], x["modes"], window_scalar=self.window,
-                          out=x["out"], stream=stream)
-            n += c.launches()
+            if fused:
+                if events is not None:
+                    events[0](l)
+                c.decode_step(l, x["seqs"], x["pos"], x["k"], x["v"], x["bits"], x["modes"], x["q"],
+                              window_scalar=self.window, out=x["out"], stream=stream)
+                n += c.launches()
+            else:
+                c.append(l, x["seqs"], x["pos"], x["k"], x["v"], x["bits"], x["modes"], stream=stream)
+                n += c.launches()
+                if events is not None:
+                    events[0](l)
+                c.decode_attn(l, x["seqs"], x["pos"], x["q"], x["modes"], window_scalar=self.window,
+                              out=x["out"], stream=stream)
+                n += c.launches()
             if events is not None:
                 events[1](l)
         return n
@@ -472,7 +533,7 @@ class Bench:
             n += c.launches()
         return n
 
-    def capture(self, idx, instrument=None, totals=None):
+    def capture(self, idx, instrument=None, totals=None, separate=False):
         torch = self.torch
         g = torch.cuda.CUDAGraph()
         s = torch.cuda.Stream()
@@ -482,9 +543,40 @@ class Bench:
                 if totals is not None:
                     launches = self.run_routed_step(self.steps[idx], totals)
                 else:
-                    launches = self.run_step(self.steps[idx], instrument(idx, s) if instrument else None)
+                    launches = self.run_step(self.steps[idx], instrument(idx, s) if instrument else None,
+                                             separate=separate)
         torch.cuda.current_stream().wait_stream(s)
         return g, launches
+
+
+def run_separate(bench, dist, r0):
+    """The same decode steps as separate trr_kv_append and trr_decode_attn calls (two
+    kernels per layer instead of one trr_decode_step kernel)."""
+    if not bench.sep_steps:
+        return None
+    torch = bench.torch
+    graphs = [bench.capture(i, separate=True) for i in range(r0, r0 + bench.sep_warm + bench.sep_steps)]
+    for g, _ in graphs[:bench.sep_warm]:
+        g.replay()
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for g, _ in graphs[bench.sep_warm:]:
+        g.replay()
+    t1.record()
+    torch.cuda.synchronize()
+    ms = t0.elapsed_time(t1)
+    idx = range(r0 + bench.sep_warm, r0 + bench.sep_warm + bench.sep_steps)
+    nbytes = sum(bench.steps[i]["bytes"] for i in idx)
+    ms, nbytes = across_ranks(dist, "cuda", ms, nbytes)
+    launches = graphs[0][1]
+    del graphs
+    return {"value": round(nbytes / (ms * 1e-3) / 1e9, 2), "unit": UNIT,
+            "ms_per_step": round(ms / bench.sep_steps, 5), "steps": bench.sep_steps,
+            "gpu_launches": launches * bench.sep_steps,
+            "how": "per layer trr_kv_append then trr_decode_attn (two kernels) instead of one trr_decode_step"}
 
 
 def run_routed(bench, dist, r0):
@@ -567,22 +659,68 @@ def run_routed(bench, dist, r0):
     }
 
 
-def run_gpu(args):
-    import torch
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
-    torch.cuda.set_device(local)
-    dist = None
-    if world > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl" if torch.distributed.is_nccl_available() else "gloo")
-    bench = Bench(args, rank, world)
-    bench.setup()
-    W, K = args.warmup, args.steps
-    rt = CudaRt()
+# The other workloads measured beside the headline (160m) in the default run: name and
+# batch (0: the workload's own).
+PER_WORKLOAD = (("tiny", 0), ("1p3b", 0), ("gqa_long", 0), ("sweep", 1), ("sweep", 8), ("sweep", 64),
+                ("sweep", 256))
 
-    # timed region: K plain step graphs
+
+def per_workload(args, local):
+    """Every other workload's decode steps, timed like the headline: step throughput and
+    the trr_decode_attn call against the HBM roofline."""
+    import copy
+    import gc
+    import torch
+    peak, peak_kind = measured_peaks()
+    out = {}
+    for name, batch in PER_WORKLOAD:
+        a = copy.copy(args)
+        a.workload, a.batch, a.layers, a.light = name, batch, 0, True
+        a.steps, a.warmup = args.per_workload_steps, 3
+        b = Bench(a)
+        b.setup()
+        core = timed_steps(b, a.warmup, a.steps, None, local)
+        value = core["job_bytes"] / (core["ms"] * 1e-3) / 1e9
+        avg_bytes, avg_ms = float(np.mean(core["call_bytes"])), float(np.mean(core["call_ms"]))
+        achieved = avg_bytes / (avg_ms * 1e-3) / 1e9
+        key = name if name != "sweep" else f"sweep_b{b.B}"
+        out[key] = {
+            "workload": f"{b.spec.name}: {b.L} layers, MHA/GQA {b.Hq}/{b.Hkv} x {b.d}, batch {b.B}, contexts "
+                        f"{describe_ctx(b)}, window {b.window}, group {b.G}, page {b.P}",
+            "value": round(value, 2), "unit": UNIT, "steps": a.steps, "warmup": a.warmup,
+            "ms_per_step": round(core["ms"] / a.steps, 5), "bytes_per_step": int(core["job_bytes"] / a.steps),
+            "kv_tokens_per_s": round(core["job_keys"] / (core["ms"] * 1e-3), 1),
+            "pct_of_8tbs": round(100 * value / 8000.0, 2),
+            "gpu_launches": core["launches_per_step"] * a.steps,
+            "roofline": {"bound": "hbm", "achieved": round(achieved, 2), "peak": peak, "unit": "GB/s",
+                         "frac": round(achieved / peak, 4), "peak_kind": peak_kind,
+                         "bytes_per_call": round(avg_bytes), "us_per_call": round(avg_ms * 1e3, 3)},
+            "replicas": b.R, "l2": l2_note(b, core["rank_bytes"] / a.steps),
+            "clocks": core["clocks"].summary(),
+        }
+        print(f"per_workload {key}: {out[key]['value']} GB/s, call {avg_ms * 1e3:.2f} us "
+              f"({achieved / peak:.3f} of peak)", file=sys.stderr, flush=True)
+        del b, core
+        gc.collect()
+        torch.cuda.empty_cache()
+    return out
+
+
+def device_uuid(local):
+    import torch
+    try:
+        uuid = str(torch.cuda.get_device_properties(local).uuid)
+        return uuid if uuid.startswith("GPU-") else "GPU-" + uuid
+    except Exception:
+        return None
+
+
+def timed_steps(bench, W, K, dist, local):
+    """W warm-up and K timed step graphs (the timed region: CUDA events on the stream,
+    clocks sampled during it), then K more steps with event nodes around every
+    trr_decode_attn call (the per-call attribution of the roofline)."""
+    import torch
+    rt = CudaRt()
     graphs = [bench.capture(i) for i in range(W + K)]
     launches_per_step = graphs[0][1]
     for i in range(W):
@@ -590,14 +728,8 @@ def run_gpu(args):
     torch.cuda.synchronize()
     if dist:
         dist.barrier()
-    uuid = None
-    try:
-        uuid = str(torch.cuda.get_device_properties(local).uuid)
-        uuid = uuid if uuid.startswith("GPU-") else "GPU-" + uuid
-    except Exception:
-        pass
     t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    with ClockSampler(uuid) as clocks:
+    with ClockSampler(device_uuid(local)) as clocks:
         torch.cuda.synchronize()
         t0.record()
         for i in range(W, W + K):
@@ -607,11 +739,9 @@ def run_gpu(args):
     ms = t0.elapsed_time(t1)
     step_bytes = sum(bench.steps[i]["bytes"] for i in range(W, W + K))
     step_keys = sum(bench.steps[i]["keys"] for i in range(W, W + K))
-    rank_bytes = step_bytes
     ms, job_bytes, job_keys = across_ranks(dist, "cuda", ms, step_bytes, step_keys)
     del graphs
 
-    # attribution: the next K steps with event nodes around every trr_decode_attn call
     evs = {}
 
     def instrument(idx, s):
@@ -638,6 +768,40 @@ def run_gpu(args):
             call_ms.append(rt.elapsed_ms(evs[(i, l, 0)], evs[(i, l, 1)]))
             call_bytes.append(bench.steps[i]["attn_bytes_per_layer"])
     del igraphs
+    return dict(ms=ms, job_bytes=job_bytes, job_keys=job_keys, rank_bytes=step_bytes,
+                launches_per_step=launches_per_step, clocks=clocks, call_ms=call_ms, call_bytes=call_bytes)
+
+
+def l2_note(bench, rank_bytes_per_step):
+    """How the timed steps relate to L2: the bytes read between two visits of a replica."""
+    rot = bench.R * rank_bytes_per_step
+    mb = bench.l2_bytes / 1e6
+    if rot >= 3 * bench.l2_bytes:
+        return (f"inputs larger than L2: {bench.R} replicas rotate, {rank_bytes_per_step / 1e6:.0f} MB per step, "
+                f"{rot / 1e6:.0f} MB between visits of a replica = {rot / bench.l2_bytes:.1f} x L2 ({mb:.0f} MB)")
+    return (f"NOT larger than L2: {bench.R} replicas x {rank_bytes_per_step / 1e6:.1f} MB per step = "
+            f"{rot / 1e6:.1f} MB between visits of a replica, {rot / bench.l2_bytes:.2f} x L2 ({mb:.0f} MB); "
+            "the workload is latency-bound and partly served from L2")
+
+
+def run_gpu(args):
+    import torch
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl" if torch.distributed.is_nccl_available() else "gloo")
+    bench = Bench(args, rank, world)
+    bench.setup()
+    W, K = args.warmup, args.steps
+    core = timed_steps(bench, W, K, dist, local)
+    ms, job_bytes, job_keys = core["ms"], core["job_bytes"], core["job_keys"]
+    rank_bytes, launches_per_step, clocks = core["rank_bytes"], core["launches_per_step"], core["clocks"]
+    call_ms, call_bytes = core["call_ms"], core["call_bytes"]
+    base = W + K
 
     # e2e: the public API with host buffers.  Each step's inputs (every layer's entries,
     # K/V rows and queries) sit in one pinned host buffer that is copied to the device in
@@ -722,7 +886,9 @@ def run_gpu(args):
     eager_ms = b0.elapsed_time(b1)
     eager_bytes = sum(bench.steps[e0 + j]["bytes"] for j in range(half, ne))
     eager_ms, eager_bytes = across_ranks(dist, "cuda", eager_ms, eager_bytes)
-    routed = None if bench.head_modes else run_routed(bench, dist, e0 + bench.e2e_warm + bench.e2e_steps)
+    r0 = e0 + bench.e2e_warm + bench.e2e_steps
+    routed = None if bench.head_modes else run_routed(bench, dist, r0)
+    separate = run_separate(bench, dist, r0 + bench.routed_warm + bench.routed_steps)
     status = bench.cache.status()
     if status != 0:
         raise RuntimeError(f"device status {status} after the run")
@@ -750,8 +916,7 @@ def run_gpu(args):
                 "skip_tokens_store_kv": bool(bench.swk),
                 "queries_per_seq": bench.C,
                 "global_batch": bench.B * world, "replicas": bench.R,
-                "l2": "inputs larger than L2: every step reads its replica's "
-                      f"{rank_bytes / K / 1e6:.0f} MB, replicas rotate",
+                "l2": l2_note(bench, rank_bytes / K), "l2_bytes": bench.l2_bytes,
                 "parallelism": f"replicas{world}" if world > 1 else "single",
                 "bytes_per_step": int(job_bytes / K),
                 "split_bytes": args.split_bytes or "default",
@@ -770,14 +935,24 @@ def run_gpu(args):
                          "traffic": None if (bench.head_modes or bench.swk or bench.C > 1)
                          else ncu_traffic(args.workload),
                          "peak_kind": peak_kind,
-                         "kernel": "trr_decode_attn call (attn_kernel, one launch)",
+                         "kernel": "trr_decode_step call (attn_kernel: append and attention, one launch)" if bench.C == 1
+                         and not bench.head_modes else "trr_decode_attn call (attn_kernel, one launch)",
                          "bytes_per_call": round(avg_bytes), "us_per_call": round(avg_ms * 1e3, 3)},
             "clocks": clocks.summary(),
         }
         if routed is not None:
             result["routed"] = routed
+        if separate is not None:
+            result["separate_calls"] = separate
         if cpu is not None:
             result["cpu_baseline"] = cpu
+    if (rank == 0 and world == 1 and not args.no_per_workload and not bench.head_modes and not bench.swk
+            and bench.C == 1 and args.workload == "160m" and not args.batch and not args.layers):
+        import gc
+        del bench
+        gc.collect()
+        torch.cuda.empty_cache()
+        result["per_workload"] = per_workload(args, local)
     if dist:
         dist.barrier()
         dist.destroy_process_group()
@@ -891,6 +1066,11 @@ def main():
     ap.add_argument("--batch", type=int, default=0)
     ap.add_argument("--layers", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-per-workload", action="store_true",
+                    help="skip the other workloads (1p3b, gqa_long, tiny, sweep at batch 1/8/64/256)")
+    ap.add_argument("--per-workload-steps", type=int, default=10)
+    ap.add_argument("--cache-budget-gb", type=float, default=120.0,
+                    help="device memory the replicas of one workload's cache may take")
     ap.add_argument("--page-size", type=int, default=0, choices=[0, 16, 32, 64],
                     help="tokens per cache page (0: 32)")
     ap.add_argument("--split-bytes", type=int, default=0,

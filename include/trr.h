@@ -29,6 +29,14 @@
  *     sticky device status word that keeps the FIRST error since it was last read;
  *     trr_get_status reads and clears it.  No kernel traps or asserts.
  *   - One stream at a time per cache: calls on the same cache must not overlap.
+ *   - Kernels are launched with programmatic dependent launch.  The index arrays of a
+ *     call (sequence ids, positions, bit-widths, modes, windows, router logits of the
+ *     *_routed calls) are read while the previous kernel of the stream may still be
+ *     running, so they must not be outputs of that kernel (produce them one kernel
+ *     earlier, or copy them in from the host).  Query, K and V rows are read after it
+ *     has finished.  A call whose layer was not touched by the two calls enqueued
+ *     before it on the cache may also read the layer's cache state early (see
+ *     trr_decode_step).
  *
  * Cache memory layout (fixed; the CPU oracle re-derives it independently)
  *   class index c = 0,1,2,3 <-> b = 2,4,8,16.   P = page_size, d = head_dim,
@@ -179,6 +187,42 @@ TRR_API trr_status trr_decode_attn(trr_cache* cache, int32_t layer, int32_t n,
                            const int32_t* windows, int32_t window_scalar,
                            float softmax_scale, void* out_bf16, void* stream);
 
+/* One decode step of one layer in one kernel: trr_kv_append of the n entries followed by
+ * trr_decode_attn of their queries at the same positions and modes (Sec. 3.8: at
+ * inference each token's KV is stored at its chosen width b_t, Sec. 3.2(C) Eq. 4, and its
+ * query attends in its mode a_t, Sec. 3.2(A) Eq. 2, over the cache including its own new
+ * token).
+ *   Entry i is token positions[i] of sequence seq_ids[i] (all distinct: one token per
+ *   sequence) with K/V rows k[i][Hkv][d], v[i][Hkv][d] (bf16), bit-width bits[i] and mode
+ *   modes[i], as trr_kv_append takes them; its query q[i][Hq][d] (bf16) attends at
+ *   t = positions[i] in mode modes[i] with window windows[i] (or window_scalar) and
+ *   writes out[i][Hq][d] (bf16), as trr_decode_attn does.  The results are those of the
+ *   two calls in that order: the same page bytes and metadata, and attention over every
+ *   stored token up to t in range, the entry's own token included.
+ *   seq_ids, positions, k, v, bits, modes, q, windows, out: device arrays;
+ *   0 <= n <= min(256, max_append, max_queries); k, v, q, out 16-byte aligned.  A cache
+ *   with head_modes returns TRR_ERR_UNSUPPORTED.
+ *   Errors are those of both calls, checked for the whole call before anything is
+ *   stored: sequence id, bit-width or mode not allowed, a sequence named twice, or a
+ *   local query with a window below 1 (INVALID_ARG); a position outside
+ *   [0, max_context) or not above the sequence's last one (BAD_POSITION); a pool running
+ *   out (OUT_OF_PAGES).  Any of these makes the call store nothing and write zero rows
+ *   for every query, and records the error of the lowest failing entry.  A group that
+ *   cannot be quantised (BAD_VALUE) is handled as trr_kv_append handles it.
+ *   The index arrays (seq_ids, positions, bits, modes, windows) may be read while the
+ *   previous kernel of the stream is still running: they must not be outputs of that
+ *   kernel.  k, v and q are read after it has finished.  When neither of the two calls
+ *   enqueued before this one on the cache was for the same layer, the kernel also reads
+ *   the layer's cache state and starts its page copies before the previous kernel has
+ *   finished; this relies on every kernel of the stream (the caller's included) not
+ *   letting its successor start before its own predecessor has finished, which holds
+ *   for kernels launched without programmatic dependent launch. */
+TRR_API trr_status trr_decode_step(trr_cache* cache, int32_t layer, int32_t n, const int32_t* seq_ids,
+                                   const int32_t* positions, const void* k_bf16, const void* v_bf16,
+                                   const uint8_t* bits, const uint8_t* modes, const void* q_bf16,
+                                   const int32_t* windows, int32_t window_scalar, float softmax_scale,
+                                   void* out_bf16, void* stream);
+
 /* trr_decode_attn without any per-call scratch in the cache's memory (this entry point
  * has no counterpart in the paper; it serves callers that cannot allocate).
  *   Same arguments, results and error contract as trr_decode_attn, but its scratch
@@ -259,8 +303,18 @@ TRR_API trr_status trr_decode_attn_routed(trr_cache* cache, int32_t layer, int32
  * freed.  NULL is accepted. */
 TRR_API trr_status trr_destroy(trr_cache* cache);
 
-/* Read and clear the sticky device status (synchronises `stream`). */
+/* Read and clear the sticky device status (synchronises `stream`).  After
+ * TRR_ERR_TIMEOUT it also returns the cache's per-call counters to their start values
+ * (on `stream`, before returning), so that later calls on the cache run normally. */
 TRR_API trr_status trr_get_status(trr_cache* cache, void* stream);
+
+/* Bound of every wait inside this cache's attention and decode-step kernels, in
+ * nanoseconds of the GPU's global timer (0 = the default, 2 s; below 20000 the waiting
+ * warps poll instead of suspending, so that the limit is kept).  A wait that runs out
+ * makes its CTA stop, lets its copies in flight land, records TRR_ERR_TIMEOUT and
+ * returns; the call's rows are then undefined and a decode step stores nothing.  No
+ * kernel waits without a bound.  Host-side setting, read at each later call. */
+TRR_API trr_status trr_set_wait_limit(trr_cache* cache, uint64_t nanoseconds);
 
 /* Forget every sequence of every layer and return all pages to the pools
  * (stream-ordered; metadata only, page bytes are not cleared). */

@@ -174,28 +174,6 @@ __global__ void __launch_bounds__(1024) append_plan_kernel(LayerArgs a, int n, c
   if (e == 0) a.ctrl[kAppendOk] = 1;
 }
 
-__device__ __forceinline__ float bf16lo(uint32_t w) { return __uint_as_float(w << 16); }
-__device__ __forceinline__ float bf16hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
-
-// round((x - z) / s) of Eq. 4 on the exact quotient, ties to even, clamped to [0, levels].
-// u = fl32(fl32(x - z) * rs) with rs = fl32(1 / s) is within 3 binary32 roundings, under
-// 2^-21 |u|, of the exact quotient, so rint(u) is exact unless u lies that close to a
-// half-way point c + 1/2.  There the midpoint z + (c + 1/2) s is formed in binary64,
-// where it is exact (z and s are binary16: a multiple of 2^-25 below 2^18), and compared
-// with x (a bf16 value).  Only half-way points inside [0, levels] matter: the clamp
-// settles the others.
-__device__ __forceinline__ int code_of(float x, float z, float s, float rs, int levels) {
-  const float u = __fmul_rn(__fsub_rn(x, z), rs);
-  const float fl = floorf(u);
-  if (fabsf(__fsub_rn(u, fl + 0.5f)) <= fabsf(u) * 0x1p-21f && fl >= 0.f && fl < static_cast<float>(levels)) {
-    const double mid = __dadd_rn(static_cast<double>(z), __dmul_rn(static_cast<double>(fl) + 0.5, static_cast<double>(s)));
-    const double xd = static_cast<double>(x);
-    const int c = static_cast<int>(fl);
-    return (xd > mid || (xd == mid && (c & 1))) ? c + 1 : c;
-  }
-  return min(max(__float2int_rn(u), 0), levels);
-}
-
 // Eq. 4 on 32 consecutive values (one chunk of a group): codes packed LSB-first.
 template <int B>
 __device__ __forceinline__ void quantise_chunk(const uint4* src, float z, float s, float rs, uint32_t* dst) {
@@ -295,55 +273,14 @@ __global__ void __launch_bounds__(256) append_write_kernel(LayerArgs a, int n, c
 
 constexpr int kFusedMax = 256;
 
-// One row of d values (entry, KV head, K or V) by a warp: lane l holds values
-// EPL*l .. EPL*l + EPL-1; a group's min / max by shuffles over its G/EPL lanes; codes
-// packed LSB-first and gathered into 32-bit words by OR over the lanes of each word.
+// One row of d values (entry, KV head, K or V) by a warp, written to its slot.
 template <int D>
 __device__ __forceinline__ void quantise_row(const uint2 w, uint8_t* codes_row, uint32_t* sz_row, int b, int G,
                                              int lane, int32_t* ctrl) {
-  constexpr int EPL = D / 32;
-  float x[EPL];
-  if (EPL == 2) {
-    x[0] = bf16lo(w.x);
-    x[1] = bf16hi(w.x);
-  } else {
-    x[0] = bf16lo(w.x);
-    x[1] = bf16hi(w.x);
-    x[EPL > 2 ? 2 : 0] = bf16lo(w.y);
-    x[EPL > 3 ? 3 : 0] = bf16hi(w.y);
-  }
-  const int GL = G / EPL;  // lanes of one group
-  float mn = x[0], mx = x[0];
-  bool bad = false;
-#pragma unroll
-  for (int i = 0; i < EPL; ++i) {
-    bad |= !(fabsf(x[i]) <= 65504.f);  // also true for NaN
-    mn = fminf(mn, x[i]);
-    mx = fmaxf(mx, x[i]);
-  }
-  for (int o = 1; o < GL; o <<= 1) {
-    mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, o));
-    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-    bad |= __shfl_xor_sync(0xffffffffu, static_cast<int>(bad), o) != 0;
-  }
-  const int levels = (1 << b) - 1;
-  uint32_t val = 0, szw = 0;
-  if (!bad) {
-    const __half z16 = __float2half_rn(mn);                                                    // z = min(x)
-    const __half s16 = __float2half_rn(__fdiv_rn(__fsub_rn(mx, mn), static_cast<float>(levels)));  // s
-    const float z = __half2float(z16), s = __half2float(s16), rs = __frcp_rn(s);
-#pragma unroll
-    for (int i = 0; i < EPL; ++i)
-      val |= static_cast<uint32_t>(s != 0.f ? code_of(x[i], z, s, rs, levels) : 0) << (i * b);
-    szw = static_cast<uint32_t>(__half_as_ushort(s16)) | (static_cast<uint32_t>(__half_as_ushort(z16)) << 16);
-  } else if (lane % GL == 0) {
-    set_status(ctrl, TRR_ERR_BAD_VALUE);
-  }
-  const int LPW = 32 / (EPL * b);  // lanes sharing one 32-bit word of codes
-  val <<= (lane % LPW) * EPL * b;
-  for (int o = 1; o < LPW; o <<= 1) val |= __shfl_xor_sync(0xffffffffu, val, o);
-  if (lane % LPW == 0) reinterpret_cast<uint32_t*>(codes_row)[lane / LPW] = val;
-  if (lane % GL == 0) sz_row[lane / GL] = szw;
+  const RowCodes r = quantise_row_codes<D>(w, b, G, lane);
+  if (r.bad && r.sz_idx >= 0) set_status(ctrl, TRR_ERR_BAD_VALUE);
+  if (r.code_idx >= 0) reinterpret_cast<uint32_t*>(codes_row)[r.code_idx] = r.code_word;
+  if (r.sz_idx >= 0) sz_row[r.sz_idx] = r.sz_word;
 }
 
 template <int D>
@@ -559,6 +496,7 @@ static trr_status append_call(trr_cache* cache, int32_t layer, int32_t n, const 
   if (mode_logits && l.head_modes) return TRR_ERR_UNSUPPORTED;  // router decisions are per token
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const LayerArgs a = layer_args(l, cache_views(cache), layer);
+  cache_note_call(cache, layer);
   const uint16_t* k = static_cast<const uint16_t*>(k_bf16);
   const uint16_t* v = static_cast<const uint16_t*>(v_bf16);
   if (n <= kFusedMax) {  // one kernel: 256 threads plan, one warp per (entry, head, K|V) row

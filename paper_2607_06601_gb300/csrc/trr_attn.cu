@@ -166,7 +166,9 @@ __device__ __forceinline__ void rescale_acc(float (&acc)[E]) {
                   pow2f((BTO == 16 ? 0 : ex_of(BTO, i + 1)) - (BFROM == 16 ? 0 : ex_of(BFROM, i + 1))));
 }
 
-// qp from the domain of class `from` to that of class `to` (from < to, or from = 16).
+// qp and acc from the domain of class `from` to that of class `to` (from < to, or
+// from = 16: a unit's pages come class by class, a decode step's own token among its
+// class's pages).
 template <int E>
 __device__ __forceinline__ void rescale_dyn(float (&qp)[E], float (&acc)[E], int from, int to) {
   switch (from * 4 + to) {
@@ -345,7 +347,7 @@ __device__ __forceinline__ void consume_page(uint32_t s0, uint32_t spos, bool ma
   const uint32_t ksz = s0 + 2 * P * rowb + (kl * ng + grp) * 4;  // its (s, z), key kl
   const uint32_t szstep = KPI * ng * 4;
 #pragma unroll 1
-  for (int it = 0; it < NIT; it += KP) {
+  for (int it = 0; it < NIT && it * KPI < fill; it += KP) {  // key groups past the fill hold nothing
     bool valid[KP];
     float dot[KP];
 #pragma unroll
@@ -452,7 +454,27 @@ struct AttnKernelArgs {
   int hpu;           // query heads per work unit
   int scr_floats;    // per-consumer-warp scratch (floats) of the tensor-core path
   int defer_merge;   // 1: split partials are merged by the combine kernel (tensor-core path)
+  int early;         // 1: the layer's cache state may be read before the previous kernel ends
+  int fused;         // 1: a decode step: entry i appends its token (k, v, bits), then query i
+                     // attends at the same position with the same mode
+  const uint16_t* k;      // fused: K rows [n][Hkv][d] (bf16)
+  const uint16_t* v;      // fused: V rows [n][Hkv][d] (bf16)
+  const uint8_t* bits;    // fused: bit-widths [n]
 };
+
+// Fused decode step: the per-entry table every CTA builds in shared memory (2 ints per
+// entry: the entry's token index in its (sequence, class) list, or -1 when it stores
+// nothing; class | opens << 2 | openers of the class before it << 3), a hash of the
+// entries' sequences (2 slots per entry: sequence + 1, lowest entry index), then the
+// call's scalars.
+constexpr int kStepMax = 256;  // entries of one decode-step call, at most
+enum StepScalar : int {
+  kSNextPage = 0,   // [4] pages handed out per class before the call (read after the wait)
+  kSOpeners = 4,    // [4] entries opening a page, per class
+  kSErr = 8,        // lowest failing entry * 16 + error, INT_MAX = none
+  kSScalars = 16
+};
+__host__ __device__ constexpr int step_ints(int n) { return 2 * n + 4 * n + kSScalars; }
 
 // Mode of query q: the caller's, or the hard decision of its mode logits.  With
 // per-head modes (modes[n][Hq]) the largest of its heads' modes, which sets the query's
@@ -497,8 +519,8 @@ __device__ __forceinline__ int query_range(int t, int mode, int w) {
 // (mbarriers need 8, bulk-copy destinations 16).
 __host__ __device__ constexpr int align16(int x) { return (x + 15) & ~15; }
 struct AttnSmem {
-  int ring, recs, sbytes, full, empty, scr, pre, red, flag, total;
-  __host__ __device__ AttnSmem(int ring_bytes, int n, int scr_floats)
+  int ring, recs, sbytes, full, empty, scr, pre, ent, red, flag, total;
+  __host__ __device__ AttnSmem(int ring_bytes, int n, int scr_floats, int fused)
       : ring(0),
         recs(align16(ring_bytes)),
         sbytes(recs + kStages * 48),
@@ -506,29 +528,38 @@ struct AttnSmem {
         empty(full + kStages * 8),
         scr(empty + kStages * 8),
         pre(scr + align16(kNcw * scr_floats * 4)),
-        red(pre + align16(4 * (n + 2))),
+        ent(pre + align16(4 * (n + 2))),
+        red(ent + (fused ? align16(4 * step_ints(n)) : 0)),
         flag(red + 16 * 8),
         total(flag + 16) {}
 };
 
-// Bounded wait that also gives up once *abort is set (by a warp that gave up).
-__device__ __forceinline__ bool mbar_wait_or(uint64_t* bar, uint32_t parity, volatile int* abort) {
+// Bounded wait (limit_ns on the global timer) that also gives up once *abort is set (by
+// a warp that gave up).
+__device__ __forceinline__ bool mbar_wait_or(uint64_t* bar, uint32_t parity, volatile int* abort, uint64_t limit_ns) {
   const uint32_t addr = smem_u32(bar), aaddr = smem_u32(const_cast<int*>(abort));
-  for (uint32_t i = 0; i < 50000; ++i) {
-    uint32_t done;
-    asm volatile(
-        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n selp.u32 %0, 1, 0, p;\n}"
-        : "=r"(done)
-        : "r"(addr), "r"(parity), "r"(20000)
-        : "memory");
-    if (done) return true;
+  if (mbar_poll(addr, parity, limit_ns)) return true;
+  const uint64_t t0 = global_ns();
+  for (;;) {
+    if (mbar_poll(addr, parity, limit_ns)) return true;
     if (lds32(aaddr)) return false;
+    if (global_ns() - t0 >= limit_ns) return false;
   }
-  return false;
 }
 
 __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+// Whether phase `parity` of `bar` has completed, without waiting.
+__device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity) {
+  uint32_t done;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+      : "=r"(done)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return done != 0;
 }
 
 // Pages of split sp (of ns) of a query of sequence seq over key positions [lo, t]:
@@ -663,10 +694,230 @@ __device__ __forceinline__ void plan_units(const AttnKernelArgs& ka, int P, int 
     pre[n + 1] = pos_split;  // for per-block split counts (per-head modes)
   }
   __syncthreads();
-  if (ka.defer_merge && blockIdx.x == 0) {  // for the combine kernel
-    int2* qtab = reinterpret_cast<int2*>(a.cnt);
-    for (int q = threadIdx.x; q < n; q += blockDim.x) qtab[q] = make_int2(pre[q], pre[q + 1] - pre[q]);
+}
+
+// ------------------------------------------------------------ decode step --
+//
+// A decode-step call (trr_decode_step) appends entry i's token (Sec. 3.2(C), Eq. 4: K and
+// V stored at the entry's bit-width; nothing for a skip token unless skip tokens store
+// KV) and attends with query i at the same position in the same mode (Eq. 2), in one
+// kernel.  The attention reads the cache as the call finds it and takes each query's own
+// new token from a stage the producer fills in shared memory; the token's bytes are
+// written to its slot in the page; the last CTA to finish commits the metadata.  The
+// entries name distinct sequences (one token per sequence).
+
+__device__ __forceinline__ unsigned seq_hash(int seq, int slots) {
+  return (static_cast<unsigned>(seq) * 2654435761u) % static_cast<unsigned>(slots);
+}
+
+// Every CTA: validates the entries and plans where each token goes (the same plan as the
+// append kernels: the token takes index ntok of its (sequence, class) list; index % P == 0
+// opens a page, whose id is next_page + the class's openers before it).  Errors, lowest
+// entry first: sequence id, bit-width or mode not allowed, or a sequence named by an
+// earlier entry (INVALID_ARG); position outside [0, max_context) or not above the
+// sequence's last one (BAD_POSITION); a local query with a window below 1 (INVALID_ARG).
+__device__ void plan_entries(const AttnKernelArgs& ka, int* ent) {
+  const LayerArgs& a = ka.a;
+  const int n = ka.n, tid = threadIdx.x, nt = blockDim.x, H = 2 * n;
+  int* hs = ent + 2 * n;  // [H][2]: sequence + 1, lowest entry index naming it
+  int* sc = ent + 6 * n;
+  for (int i = tid; i < 2 * H; i += nt) hs[i] = (i & 1) ? INT_MAX : 0;
+  for (int i = tid; i < kSScalars; i += nt) sc[i] = i == kSErr ? INT_MAX : 0;
+  __syncthreads();
+  for (int e = tid; e < n; e += nt) {
+    const int seq = ka.seq_ids[e];
+    if (seq < 0 || seq >= a.S) continue;
+    unsigned h = seq_hash(seq, H);
+    for (int probe = 0; probe < H; ++probe) {
+      const int old = atomicCAS(&hs[2 * h], 0, seq + 1);
+      if (old == 0 || old == seq + 1) {
+        atomicMin(&hs[2 * h + 1], e);
+        break;
+      }
+      h = h + 1 == static_cast<unsigned>(H) ? 0u : h + 1;
+    }
   }
+  __syncthreads();
+  for (int e = tid; e < n; e += nt) {
+    const int seq = ka.seq_ids[e], pos = ka.q_positions[e], m = ka.modes[e], b = ka.bits[e];
+    const int c = b == 2 ? 0 : b == 4 ? 1 : b == 8 ? 2 : b == 16 ? 3 : -1;
+    const int w = ka.windows ? ka.windows[e] : ka.window_scalar;
+    int err = 0;
+    if (seq < 0 || seq >= a.S || c < 0 || m > TRR_MODE_FULL) {
+      err = TRR_ERR_INVALID_ARG;
+    } else if (pos < 0 || pos >= a.maxctx) {
+      err = TRR_ERR_BAD_POSITION;
+    } else {
+      unsigned h = seq_hash(seq, H);
+      for (int probe = 0; probe < H && hs[2 * h] != seq + 1; ++probe) h = h + 1 == static_cast<unsigned>(H) ? 0u : h + 1;
+      if (hs[2 * h + 1] != e) err = TRR_ERR_INVALID_ARG;
+      else if (pos <= a.last_pos[seq]) err = TRR_ERR_BAD_POSITION;
+      else if (m == TRR_MODE_LOCAL && w < 1) err = TRR_ERR_INVALID_ARG;
+    }
+    int tok = -1, info = 0;
+    if (!err && (m != TRR_MODE_SKIP || a.skip_writes_kv)) {
+      tok = a.ntok[seq * 4 + c];
+      info = c | (tok % a.P == 0 ? 4 : 0);
+    }
+    ent[2 * e] = tok;
+    ent[2 * e + 1] = info;
+    if (err) atomicMin(&sc[kSErr], e * 16 + err);
+  }
+  __syncthreads();
+  if (tid < 32) {  // openers of the same class before each entry, 32 entries at a time
+    int run0 = 0, run1 = 0, run2 = 0, run3 = 0;
+    for (int e0 = 0; e0 < n; e0 += 32) {
+      const int e = e0 + tid;
+      const int tok = e < n ? ent[2 * e] : -1, info = e < n ? ent[2 * e + 1] : 0;
+      const bool op = tok >= 0 && (info & 4);
+      const int c = info & 3;
+      const unsigned below = (1u << tid) - 1u;
+      const unsigned b0 = __ballot_sync(0xffffffffu, op && c == 0), b1 = __ballot_sync(0xffffffffu, op && c == 1);
+      const unsigned b2 = __ballot_sync(0xffffffffu, op && c == 2), b3 = __ballot_sync(0xffffffffu, op && c == 3);
+      const int before = c == 0 ? run0 + __popc(b0 & below) : c == 1 ? run1 + __popc(b1 & below)
+                       : c == 2 ? run2 + __popc(b2 & below) : run3 + __popc(b3 & below);
+      if (e < n) ent[2 * e + 1] = info | ((op ? before : 0) << 3);
+      run0 += __popc(b0); run1 += __popc(b1); run2 += __popc(b2); run3 += __popc(b3);
+    }
+    if (tid < 4) sc[kSOpeners + tid] = tid == 0 ? run0 : tid == 1 ? run1 : tid == 2 ? run2 : run3;
+  }
+  __syncthreads();
+}
+
+// One warp, after the wait on the previous kernel: the pools' page counters, and the
+// first opener beyond its pool's capacity (OUT_OF_PAGES) as a call error.
+__device__ __forceinline__ void step_after_wait(const AttnKernelArgs& ka, int* ent, int lane) {
+  const LayerArgs& a = ka.a;
+  const int n = ka.n;
+  int* sc = ent + 6 * n;
+  if (lane < 4) sc[kSNextPage + lane] = a.ctrl[kNextPage + lane];
+  __syncwarp();
+  for (int e = lane; e < n; e += 32) {
+    const int tok = ent[2 * e], info = ent[2 * e + 1], c = info & 3;
+    if (tok >= 0 && (info & 4) && sc[kSNextPage + c] + (info >> 3) >= a.cap[c])
+      atomicMin(&sc[kSErr], e * 16 + TRR_ERR_OUT_OF_PAGES);
+  }
+  __syncwarp();
+}
+
+// Page and slot of entry e's token (an entry that stores KV).
+__device__ __forceinline__ void step_slot(const AttnKernelArgs& ka, const int* ent, int e, int& c, int& pid,
+                                          int& slot) {
+  const LayerArgs& a = ka.a;
+  const int tok = ent[2 * e], info = ent[2 * e + 1];
+  const int* sc = ent + 6 * ka.n;
+  c = info & 3;
+  slot = tok % a.P;
+  pid = (info & 4) ? sc[kSNextPage + c] + (info >> 3) : a.lastpg[ka.seq_ids[e] * 4 + c];
+}
+
+// Entry e's K and V rows of up to 4 KV heads kv0 .. kv0 + nkv - 1, this lane's D/32
+// values of each (loaded together: one round trip).
+template <int D>
+__device__ __forceinline__ void step_load_rows(const AttnKernelArgs& ka, int e, int kv0, int nkv, uint2 (&rk)[4],
+                                               uint2 (&rv)[4], int lane) {
+  const LayerArgs& a = ka.a;
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    rk[k] = rv[k] = make_uint2(0, 0);
+    if (k < nkv) {
+      const int64_t src = (static_cast<int64_t>(e) * a.Hkv + kv0 + k) * D;
+      if (D == 64) {
+        rk[k].x = reinterpret_cast<const uint32_t*>(ka.k + src)[lane];
+        rv[k].x = reinterpret_cast<const uint32_t*>(ka.v + src)[lane];
+      } else {
+        rk[k] = reinterpret_cast<const uint2*>(ka.k + src)[lane];
+        rv[k] = reinterpret_cast<const uint2*>(ka.v + src)[lane];
+      }
+    }
+  }
+}
+
+// One KV head j's K and V rows (rk, rv as step_load_rows holds them) at class c
+// (Eq. 4, or the bf16 bits at width 16): written to the token's slot `slot` of page pid
+// when `own`, and, when `to_ring`, to slot 0 of a page-shaped slice at shared address
+// sdst (the stage consumers read).  Every lane of the warp calls it.
+template <int D>
+__device__ __forceinline__ void step_token_rows(const AttnKernelArgs& ka, uint2 rk, uint2 rv, int j, int c, int pid,
+                                                int slot, bool own, uint32_t sdst, bool to_ring, int lane) {
+  const LayerArgs& a = ka.a;
+  const int P = a.P, b = bits_of_class(c), ng = D / a.G;
+  uint8_t* page = a.pool[c] + static_cast<int64_t>(pid) * a.page_bytes[c] + a.hdr + static_cast<int64_t>(j) * a.slice[c];
+  if (b == 16) {  // K [P][D] | V [P][D] bf16: this lane's D/32 values
+    const int rowb = 2 * D;
+    if (D == 64) {
+      if (own) {
+        reinterpret_cast<uint32_t*>(page + slot * rowb)[lane] = rk.x;
+        reinterpret_cast<uint32_t*>(page + (P + slot) * rowb)[lane] = rv.x;
+      }
+      if (to_ring) {
+        sts32(sdst + 4 * lane, rk.x);
+        sts32(sdst + P * rowb + 4 * lane, rv.x);
+      }
+    } else {
+      if (own) {
+        reinterpret_cast<uint2*>(page + slot * rowb)[lane] = rk;
+        reinterpret_cast<uint2*>(page + (P + slot) * rowb)[lane] = rv;
+      }
+      if (to_ring) {
+        sts32(sdst + 8 * lane, rk.x);
+        sts32(sdst + 8 * lane + 4, rk.y);
+        sts32(sdst + P * rowb + 8 * lane, rv.x);
+        sts32(sdst + P * rowb + 8 * lane + 4, rv.y);
+      }
+    }
+    return;
+  }
+  const int rowb = D * b / 8;
+  const RowCodes qk = quantise_row_codes<D>(rk, b, a.G, lane);
+  const RowCodes qv = quantise_row_codes<D>(rv, b, a.G, lane);
+  if (__any_sync(0xffffffffu, qk.bad || qv.bad) && lane == 0 && own) set_status(a.ctrl, TRR_ERR_BAD_VALUE);
+  const int kszo = 2 * P * rowb, vszo = kszo + P * ng * 4;
+  if (own) {
+    if (qk.code_idx >= 0) reinterpret_cast<uint32_t*>(page + slot * rowb)[qk.code_idx] = qk.code_word;
+    if (qv.code_idx >= 0) reinterpret_cast<uint32_t*>(page + (P + slot) * rowb)[qv.code_idx] = qv.code_word;
+    if (qk.sz_idx >= 0) reinterpret_cast<uint32_t*>(page + kszo + slot * ng * 4)[qk.sz_idx] = qk.sz_word;
+    if (qv.sz_idx >= 0) reinterpret_cast<uint32_t*>(page + vszo + slot * ng * 4)[qv.sz_idx] = qv.sz_word;
+  }
+  if (to_ring) {
+    if (qk.code_idx >= 0) sts32(sdst + 4 * qk.code_idx, qk.code_word);
+    if (qv.code_idx >= 0) sts32(sdst + P * rowb + 4 * qv.code_idx, qv.code_word);
+    if (qk.sz_idx >= 0) sts32(sdst + kszo + 4 * qk.sz_idx, qk.sz_word);
+    if (qv.sz_idx >= 0) sts32(sdst + vszo + 4 * qv.sz_idx, qv.sz_word);
+  }
+}
+
+// The last CTA of a decode-step call: records the call's error, or commits every entry's
+// metadata (page tables, page first / last positions, counts, the slot's position,
+// presence, last positions, the pools' counters).  Nothing of the call's old metadata is
+// read after this: every other CTA has finished.
+__device__ void step_commit(const AttnKernelArgs& ka, const int* ent) {
+  const LayerArgs& a = ka.a;
+  const int n = ka.n;
+  const int* sc = ent + 6 * n;
+  if (sc[kSErr] != INT_MAX) {
+    if (threadIdx.x == 0) set_status(a.ctrl, sc[kSErr] & 15);
+    return;
+  }
+  for (int e = threadIdx.x; e < n; e += blockDim.x) {
+    const int seq = ka.seq_ids[e], pos = ka.q_positions[e], tok = ent[2 * e];
+    if (tok >= 0) {
+      int c, pid, slot;
+      step_slot(ka, ent, e, c, pid, slot);
+      const int64_t row = (static_cast<int64_t>(seq) * 4 + c) * a.MP + tok / a.P;
+      if (ent[2 * e + 1] & 4) {
+        a.pt[row] = pid;
+        a.pfirst[row] = pos;
+      }
+      a.plast[row] = pos;
+      a.ntok[seq * 4 + c] = tok + 1;
+      a.lastpg[seq * 4 + c] = pid;
+      reinterpret_cast<int32_t*>(a.pool[c] + static_cast<int64_t>(pid) * a.page_bytes[c])[slot] = pos;
+      atomicOr(&a.presence[static_cast<int64_t>(seq) * a.W32 + pos / 32], 1u << (pos % 32));
+    }
+    a.last_pos[seq] = pos;
+  }
+  if (threadIdx.x < 4) a.ctrl[kNextPage + threadIdx.x] = sc[kSNextPage + threadIdx.x] + sc[kSOpeners + threadIdx.x];
 }
 
 // Everything the producer and consumers of one CTA share.
@@ -682,25 +933,72 @@ struct CtaRing {
 
 // The producer warp: takes units (the CTA's own first, then from a call-wide counter),
 // plans each and pushes its stages; ends with an end record.
+//
+// With `early`, the first stages are planned and their page copies issued before the
+// wait on the previous kernel (the layer's cache state is settled; the call's index
+// arrays are its own): the unit's query-rows stage takes its slot first, and its record
+// and copy follow the wait, so that consumers start only once the query rows (written
+// by the previous kernel) are in.  Before the wait the producer takes ring space only
+// where it is free, never waiting for consumers.  Nothing is written to global memory
+// before the wait.
 template <int D>
-__device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, int NQB, const int* pre,
+__device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, int NQB, const int* pre, int* ent,
                                              const CtaRing& cr, int lane) {
   const LayerArgs& a = ka.a;
   const int n = ka.n, g = a.Hq / a.Hkv, R = cr.R;
   const int total = pre[n] * NQB;
+  const int* sc = ent + 6 * n;        // decode step: the call's scalars
   uint32_t pushed = 0, released = 0;  // stages pushed / seen released by the consumers
   int rhead = 0, rused = 0;           // ring: next free offset, bytes held
   bool ok = true;
+  bool waited = !ka.early;
+  // the query-rows stage waiting for the wait: its slot (-1: none), ring offset, records
+  int dq_slot = -1, dq_off = 0, dq_need = 0;
+  int4 dq_ra = make_int4(0, 0, 0, 0), dq_rb = dq_ra, dq_rc = dq_ra;
+  const uint16_t* dq_src = nullptr;
+  // the call's error once known (a decode step with an error stores nothing and every
+  // query gets its zero rows)
+  auto call_failed = [&]() -> bool { return ka.fused && sc[kSErr] != INT_MAX; };
+  // after the wait on the previous kernel: let the next kernel start, read what the
+  // previous kernel wrote (decode step: the pools' counters; the combine kernel's query
+  // table), then complete the deferred query-rows stage
+  auto after_wait = [&]() {
+    pdl_trigger();
+    if (dq_slot >= 0) {
+      if (lane == 0) {
+        cr.recs[dq_slot * 3 + 0] = dq_ra;
+        cr.recs[dq_slot * 3 + 1] = dq_rb;
+        cr.recs[dq_slot * 3 + 2] = dq_rc;
+        mbar_arrive_expect_tx(&cr.full[dq_slot], static_cast<uint32_t>(dq_need));
+        bulk_g2s(cr.ring + dq_off, dq_src, dq_need, &cr.full[dq_slot]);
+      }
+      dq_slot = -1;
+    }
+    if (ka.defer_merge && blockIdx.x == 0) {  // for the combine kernel
+      int2* qtab = reinterpret_cast<int2*>(a.cnt);
+      for (int q = lane; q < n; q += 32) qtab[q] = make_int2(pre[q], pre[q + 1] - pre[q]);
+    }
+    // decode step: the pools' counters, and whether a token runs out of pages (then
+    // the call stores nothing, and the last CTA zeroes every row)
+    if (ka.fused) step_after_wait(ka, ent, lane);
+  };
+  auto ensure_waited = [&]() {
+    if (waited) return;
+    pdl_wait();
+    waited = true;
+    after_wait();
+  };
   // wait for the oldest stage in flight to be released and take back its bytes
   auto release_one = [&]() -> bool {
     const uint32_t slot = released % kStages;
-    if (!mbar_wait_or(&cr.empty[slot], (released / kStages) & 1, cr.abort_flag)) return false;
+    if (!mbar_wait_or(&cr.empty[slot], (released / kStages) & 1, cr.abort_flag, a.wait_ns)) return false;
     rused -= static_cast<int>(lds32(smem_u32(cr.sbytes) + 4 * slot));
     ++released;
     return true;
   };
-  // a slot and `need` contiguous ring bytes; -1 when a wait gave up
-  auto reserve = [&](int need, int& taken) -> int {
+  // a slot and `need` contiguous ring bytes; -1 when a wait gave up; -2 when the space
+  // is not free yet and `block` is false
+  auto reserve = [&](int need, int& taken, bool block) -> int {
     for (;;) {
       if (pushed - released < static_cast<uint32_t>(kStages)) {
         if (rused == 0) rhead = 0;  // an empty ring can start anywhere
@@ -716,8 +1014,25 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
           return off;
         }
       }
-      if (pushed == released || !release_one()) return -1;
+      if (pushed == released) return -1;
+      if (!block) {  // take back released stages, without waiting for any
+        const uint32_t slot = released % kStages;
+        if (!mbar_test(&cr.empty[slot], (released / kStages) & 1)) return -2;
+        rused -= static_cast<int>(lds32(smem_u32(cr.sbytes) + 4 * slot));
+        ++released;
+        continue;
+      }
+      if (!release_one()) return -1;
     }
+  };
+  // reserve before the wait where free, else wait on the previous kernel and block
+  auto reserve_any = [&](int need, int& taken) -> int {
+    int off = reserve(need, taken, waited);
+    if (off == -2) {
+      ensure_waited();
+      off = reserve(need, taken, true);
+    }
+    return off;
   };
   // the record of the stage taking slot pushed % kStages, then its arrival with the
   // bytes its copies will bring (the copies follow, issued by lane 0)
@@ -733,11 +1048,12 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
     ++pushed;
     return slot;
   };
+  if (waited) after_wait();
 
   int u = blockIdx.x;  // the first unit is the CTA's own; later ones come from the counter
   while (u < total) {
     int u_next = 0;
-    if (lane == 0) u_next = static_cast<int>(gridDim.x) + atomicAdd(&a.ctrl[kNextUnit], 1);  // used last
+    if (lane == 0) u_next = static_cast<int>(gridDim.x) + atomicAdd(&a.lctl[kNextUnit], 1);  // used last
     const int un = u / NQB, qb = u - un * NQB;
     int lo_q = 0, hi_q = n;  // the query of split un: pre[q] <= un < pre[q + 1]
     while (hi_q - lo_q > 1) {
@@ -779,12 +1095,29 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
         continue;
       }
     }
-    if (err || bmode == TRR_MODE_SKIP) {  // zero rows (once per block); the error of the lowest query
+    // decode step: this query's own token joins the last split of each head block
+    const bool has_new = ka.fused && !err && bmode != TRR_MODE_SKIP && sp == ns - 1;
+    if (err || bmode == TRR_MODE_SKIP || call_failed()) {
+      // zero rows (once per block); the error of the lowest query; a skip token that
+      // stores KV has its rows written here
+      ensure_waited();
       if (sp == 0) {
         uint4* o = reinterpret_cast<uint4*>(ka.out + (static_cast<int64_t>(q) * a.Hq + h0) * D);
         for (int i = lane; i < nh * D / 8; i += 32) o[i] = make_uint4(0, 0, 0, 0);
       }
-      if (err && qb == 0 && lane == 0) atomicMin(&a.ctrl[kFirstBadQuery], (ka.q0 + q) * 16 + err);
+      if (!ka.fused && err && qb == 0 && lane == 0) atomicMin(&a.lctl[kFirstBadQuery], (ka.q0 + q) * 16 + err);
+      if (ka.fused && !call_failed() && sp == 0 && ent[2 * q] >= 0) {
+        int c, pid, slot;
+        step_slot(ka, ent, q, c, pid, slot);
+        for (int j0 = kv0; j0 < kv0 + nkv; j0 += 4) {
+          const int m = min(4, kv0 + nkv - j0);
+          uint2 rk[4], rv[4];
+          step_load_rows<D>(ka, q, j0, m, rk, rv, lane);
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            if (k < m) step_token_rows<D>(ka, rk[k], rv[k], j0 + k, c, pid, slot, (j0 + k) * g >= h0, 0u, false, lane);
+        }
+      }
     } else {
       const int lo = bmode == TRR_MODE_FULL ? 0 : max(0, t - w + 1);
       int wid, wmeta, wfirst = 0, wlast = INT_MAX;
@@ -801,16 +1134,33 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
       {  // the unit's query rows
         const int need = nh * D * 2;
         int taken = 0;
-        const int off = reserve(need, taken);
+        int off = reserve(need, taken, waited);
+        if (off == -2) {  // before the wait with the ring full: wait, then block
+          ensure_waited();
+          off = reserve(need, taken, true);
+        }
         if (off < 0) {
           ok = false;
           break;
         }
-        const int meta = kQRows | kFirst | (T == 0 ? (kLast | kNoPage) : 0) | (qb << 16);
-        const uint32_t slot =
-            push(make_int4(meta, off, q, lo), rb, make_int4(hpack, max(0, t - w + 1), -1, 0), taken, need);
-        if (lane == 0)
-          bulk_g2s(cr.ring + off, ka.q + (static_cast<int64_t>(q) * a.Hq + h0) * D, need, &cr.full[slot]);
+        const bool only = T == 0 && !has_new;
+        const int meta = kQRows | kFirst | (only ? (kLast | kNoPage) : 0) | (qb << 16);
+        const int4 ra = make_int4(meta, off, q, lo), rc = make_int4(hpack, max(0, t - w + 1), -1, 0);
+        const uint16_t* src = ka.q + (static_cast<int64_t>(q) * a.Hq + h0) * D;
+        if (waited) {
+          const uint32_t slot = push(ra, rb, rc, taken, need);
+          if (lane == 0) bulk_g2s(cr.ring + off, src, need, &cr.full[slot]);
+        } else {  // its slot now, its record and copy after the wait
+          dq_slot = static_cast<int>(pushed % kStages);
+          if (lane == 0) cr.sbytes[dq_slot] = taken;
+          ++pushed;
+          dq_off = off;
+          dq_need = need;
+          dq_ra = ra;
+          dq_rb = rb;
+          dq_rc = rc;
+          dq_src = src;
+        }
       }
       // every page's copy, worked out once per unit (lane j: page j), so that a push
       // is a few shuffles and the copy
@@ -823,12 +1173,56 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
         pg_src = reinterpret_cast<uint64_t>(a.pool[c] + static_cast<int64_t>(wid) * a.page_bytes[c]);
         pg_geo = slice | (max(1, (R / 2 - posb) / slice) << 20);
       }
+      // decode step: the query's own token, as one stage per KV head holding it at slot 0
+      // of a page-shaped slice (consumers read it as a page with one key), placed after
+      // the pages of its own width class so that the consumers' class domain only ever
+      // rises; its bytes also go to the token's slot in the cache.  After a call error
+      // (known only after the wait) one empty stage stands in for it.
+      const int new_cls = has_new ? ent[2 * q + 1] & 3 : 4;
+      bool new_done = !has_new;
+      auto push_new = [&](bool last) -> bool {
+        ensure_waited();  // the token's K / V rows come from the previous kernel
+        new_done = true;
+        if (call_failed()) {
+          int taken = 0;
+          const int off = reserve(0, taken, true);
+          if (off < 0) return false;
+          push(make_int4((last ? kLast : 0) | (qb << 16), off, q, lo), rb, make_int4(0, 0, -1, 0), taken, 0);
+          return true;
+        }
+        int c, pid, slot;
+        step_slot(ka, ent, q, c, pid, slot);
+        const int slice = a.slice[c];
+        for (int j0 = 0; j0 < nkv; j0 += 4) {
+          const int m = min(4, nkv - j0);
+          uint2 rk[4], rv[4];
+          step_load_rows<D>(ka, q, kv0 + j0, m, rk, rv, lane);
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            if (k >= m) continue;
+            int taken = 0;
+            const int off = reserve(slice, taken, true);
+            if (off < 0) return false;
+            const int k0 = j0 + k, j = kv0 + k0;
+            step_token_rows<D>(ka, rk[k], rv[k], j, c, pid, slot, j * g >= h0, smem_u32(cr.ring + off), true, lane);
+            fence_proxy_async_smem();  // these bytes are later overwritten by bulk copies
+            __syncwarp();
+            const int meta = c | (1 << 2) | (last && k0 == nkv - 1 ? kLast : 0) | (qb << 16);
+            push(make_int4(meta, off, q, lo), rb, make_int4(k0, 1, -1, slice), taken, 0);
+          }
+        }
+        return true;
+      };
       for (int j = 0; j < T && ok; ++j) {
         const uint8_t* page = reinterpret_cast<const uint8_t*>(__shfl_sync(0xffffffffu, pg_src, j));
         const int geo = __shfl_sync(0xffffffffu, pg_geo, j);
         const int pm = __shfl_sync(0xffffffffu, wmeta, j);
         const unsigned needed = __shfl_sync(0xffffffffu, pg_need, j);
         const int slice = geo & 0xfffff, maxk = geo >> 20;
+        if (!new_done && (pm & 3) > new_cls && !push_new(false)) {
+          ok = false;
+          break;
+        }
         // one stage per run of consecutive needed KV heads, at most maxk slices each
         for (int k0 = __ffs(needed) - 1; k0 >= 0 && k0 < nkv;) {
           int nk = 1;
@@ -836,13 +1230,13 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
           const int posb = (pm & kMask) ? 4 * P : 0;
           const int need = nk * slice + posb;
           int taken = 0;
-          const int off = reserve(need, taken);
+          const int off = reserve_any(need, taken);
           if (off < 0) {
             ok = false;
             break;
           }
           const unsigned later = needed >> (k0 + nk);  // needed KV heads after this stage
-          const bool last = j == T - 1 && later == 0;
+          const bool last = j == T - 1 && later == 0 && new_done;
           const int meta = pm | (last ? kLast : 0) | (qb << 16);
           const uint32_t slot =
               push(make_int4(meta, off, q, lo), rb, make_int4(k0, nk, posb ? off + nk * slice : -1, slice), taken, need);
@@ -853,22 +1247,34 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
           k0 = later ? k0 + nk + __ffs(later) - 1 : nkv;
         }
       }
+      if (ok && !new_done && !push_new(true)) ok = false;
       if (!ok) break;
+      ensure_waited();  // the next unit's query rows come from the previous kernel
     }
     __syncwarp();
     u = __shfl_sync(0xffffffffu, u_next, 0);
   }
   if (ok) {
+    ensure_waited();
     int taken = 0;
-    if (reserve(0, taken) < 0) ok = false;
+    if (reserve(0, taken, true) < 0) ok = false;
     else push(make_int4(kEnd, 0, 0, 0), make_int4(0, 0, 0, 0), make_int4(0, 0, -1, 0), taken, 0);
   }
   if (!ok) {  // a wait gave up: stop the consumers, then let every copy in flight land
+    if (!waited) {
+      pdl_wait();
+      waited = true;
+      pdl_trigger();
+    }
     if (lane == 0) {
       *cr.abort_flag = 1;
       set_status(a.ctrl, TRR_ERR_TIMEOUT);
+      atomicExch(&a.lctl[kAborted], 1);
     }
-    for (uint32_t s = released; s < pushed; ++s) mbar_wait(&cr.full[s % kStages], (s / kStages) & 1);
+    // copies in flight always land (they only read memory): wait for them with the
+    // default bound whatever the configured one
+    for (uint32_t s = released; s < pushed; ++s)
+      if (static_cast<int>(s % kStages) != dq_slot) mbar_wait(&cr.full[s % kStages], (s / kStages) & 1);
   }
 }
 
@@ -1036,11 +1442,12 @@ __device__ __forceinline__ void run_consumer_cc(const AttnKernelArgs& ka, const 
   bool active = false;
   for (uint32_t s = 0;; ++s) {
     const uint32_t slot = s % kStages;
-    const bool arrived = mbar_wait_or(&cr.full[slot], (s / kStages) & 1, cr.abort_flag);
+    const bool arrived = mbar_wait_or(&cr.full[slot], (s / kStages) & 1, cr.abort_flag, a.wait_ns);
     if (!__all_sync(0xffffffffu, arrived)) {  // give up together, never half a warp
       if (lane == 0) {
         *cr.abort_flag = 1;
         set_status(a.ctrl, TRR_ERR_TIMEOUT);
+        atomicExch(&a.lctl[kAborted], 1);
       }
       break;
     }
@@ -1050,7 +1457,7 @@ __device__ __forceinline__ void run_consumer_cc(const AttnKernelArgs& ka, const 
     if (meta & kEnd) break;
     if (meta & kQRows) {
       const int4 rb = lds128i(rec + 16);
-      const int qb = meta >> 16;
+      const int qb = (meta >> 16) & 0x7fff;
       u_h = qb * kNcw + cw;
       active = u_h < a.Hq;
       u_kvi = u_h / g - (qb * kNcw) / g;
@@ -1563,11 +1970,12 @@ __device__ __forceinline__ void run_consumer_mma(const AttnKernelArgs& ka, const
   bool active = false;
   for (uint32_t s = 0;; ++s) {
     const uint32_t slot = s % kStages;
-    const bool arrived = mbar_wait_or(&cr.full[slot], (s / kStages) & 1, cr.abort_flag);
+    const bool arrived = mbar_wait_or(&cr.full[slot], (s / kStages) & 1, cr.abort_flag, a.wait_ns);
     if (!__all_sync(0xffffffffu, arrived)) {  // give up together, never half a warp
       if (lane == 0) {
         *cr.abort_flag = 1;
         set_status(a.ctrl, TRR_ERR_TIMEOUT);
+        atomicExch(&a.lctl[kAborted], 1);
       }
       break;
     }
@@ -1577,7 +1985,7 @@ __device__ __forceinline__ void run_consumer_mma(const AttnKernelArgs& ka, const
     if (meta & kEnd) break;
     if (meta & kQRows) {
       const int4 rb = lds128i(rec + 16);
-      const int qb = meta >> 16;
+      const int qb = (meta >> 16) & 0x7fff;
       u_kv = qb * kNcw + cw;
       active = u_kv < a.Hkv;
       u_q = ra.z;
@@ -1655,8 +2063,9 @@ __device__ __forceinline__ void run_consumer_mma(const AttnKernelArgs& ka, const
 
 // The prologue every attention kernel shares: barriers, the dependency on the previous
 // kernel, the call's work units.
-__device__ __forceinline__ CtaRing attn_prologue(const AttnKernelArgs& ka, uint8_t* smem, int P, int NQB, int*& pre) {
-  const AttnSmem lay(ka.ring_bytes, ka.n, ka.scr_floats);
+__device__ __forceinline__ CtaRing attn_prologue(const AttnKernelArgs& ka, uint8_t* smem, int P, int NQB, int*& pre,
+                                                int*& ent) {
+  const AttnSmem lay(ka.ring_bytes, ka.n, ka.scr_floats, ka.fused);
   CtaRing cr;
   cr.ring = smem + lay.ring;
   cr.recs = reinterpret_cast<int4*>(smem + lay.recs);
@@ -1676,29 +2085,53 @@ __device__ __forceinline__ CtaRing attn_prologue(const AttnKernelArgs& ka, uint8
     fence_barrier_init();
   }
   // The unit plan reads only the call's own index arrays (sequence ids, positions,
-  // modes, windows), which no kernel of this library writes, so it overlaps the
-  // previous kernel of the stream; everything after the wait may read what that
-  // kernel wrote (cache metadata, pages, control words).
+  // modes, windows, bit-widths), which no kernel of this library writes, so it overlaps
+  // the previous kernel of the stream.  The layer's cache state (metadata, pages, its
+  // control words) is read before the wait only when `early` says that no kernel still
+  // running can write it; everything else the previous kernel may write (query, K and V
+  // rows, the pools' counters, scratch) is read after the producer's wait.
   plan_units(ka, P, NQB, pre, reinterpret_cast<long long*>(smem + lay.red));
-  pdl_wait();
-  pdl_trigger();
+  ent = reinterpret_cast<int*>(smem + lay.ent);
+  if (!ka.early) pdl_wait();
+  if (ka.fused) plan_entries(ka, ent);
   return cr;
 }
 
-// The epilogue: the last CTA to finish records the error of the lowest failing query
-// and readies the call's counters for the next call.
-__device__ __forceinline__ void attn_epilogue(const LayerArgs& a) {
+// The epilogue: the last CTA to finish records the error of the lowest failing query,
+// readies the layer's counters for the next call and, for a decode step, commits the
+// appended tokens' metadata.
+__device__ __forceinline__ void attn_epilogue(const AttnKernelArgs& ka, const int* ent) {
+  const LayerArgs& a = ka.a;
+  __shared__ int s_last, s_aborted;
   __syncthreads();
   if (threadIdx.x == 0) {
     __threadfence();
-    if (atomicAdd(&a.ctrl[kDoneCtas], 1) == static_cast<int>(gridDim.x) - 1) {
+    s_last = atomicAdd(&a.lctl[kDoneCtas], 1) == static_cast<int>(gridDim.x) - 1;
+    if (s_last) {
       __threadfence();
-      const int bad = atomicExch(&a.ctrl[kFirstBadQuery], INT_MAX);
+      const int bad = atomicExch(&a.lctl[kFirstBadQuery], INT_MAX);
       if (bad != INT_MAX) set_status(a.ctrl, bad & 15);
-      atomicExch(&a.ctrl[kNextUnit], 0);
-      atomicExch(&a.ctrl[kDoneCtas], 0);
+      s_aborted = atomicExch(&a.lctl[kAborted], 0);
+      atomicExch(&a.lctl[kNextUnit], 0);
+      atomicExch(&a.lctl[kDoneCtas], 0);
     }
   }
+  if (!ka.fused) return;
+  __syncthreads();
+  if (!s_last) return;
+  const int* sc = ent + 6 * ka.n;
+  if (sc[kSErr] != INT_MAX) {
+    // a call error (some known only after the wait, when rows were already being
+    // computed): every row zero, nothing for the combine kernel to merge
+    uint4* o = reinterpret_cast<uint4*>(ka.out);
+    const int64_t n16 = static_cast<int64_t>(ka.n) * a.Hq * a.d / 8;
+    for (int64_t i = threadIdx.x; i < n16; i += blockDim.x) o[i] = make_uint4(0, 0, 0, 0);
+    if (ka.defer_merge) {
+      int2* qtab = reinterpret_cast<int2*>(a.cnt);
+      for (int q = threadIdx.x; q < ka.n; q += blockDim.x) qtab[q] = make_int2(0, 1);
+    }
+  }
+  if (!s_aborted) step_commit(ka, ent);  // a call that gave up a wait stores nothing
 }
 
 // CUDA-core path: units of kNcw query heads, one per consumer warp; HM: per-head modes
@@ -1709,11 +2142,11 @@ __global__ void __launch_bounds__(32 * (kNcw + 1), cc_ctas_per_sm(D))
   extern __shared__ __align__(128) uint8_t smem[];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int NQB = (ka.a.Hq + ka.hpu - 1) / ka.hpu;
-  int* pre;
-  const CtaRing cr = attn_prologue(ka, smem, P, NQB, pre);
-  if (warp == 0) run_producer<D>(ka, P, NQB, pre, cr, lane);
+  int *pre, *ent;
+  const CtaRing cr = attn_prologue(ka, smem, P, NQB, pre, ent);
+  if (warp == 0) run_producer<D>(ka, P, NQB, pre, ent, cr, lane);
   else run_consumer_cc<D, P, cc_elems(D), HM>(ka, cr, warp - 1, lane);
-  attn_epilogue(ka.a);
+  attn_epilogue(ka, ent);
 }
 
 // Tensor-core path: units of kNcw KV heads with all their query heads.
@@ -1723,16 +2156,16 @@ __global__ void __launch_bounds__(32 * (kNcw + 1), kMmaCtasPerSm) attn_mma_kerne
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int NQB = (ka.a.Hq + ka.hpu - 1) / ka.hpu;
   const int P = ka.a.P;
-  int* pre;
-  const CtaRing cr = attn_prologue(ka, smem, P, NQB, pre);
+  int *pre, *ent;
+  const CtaRing cr = attn_prologue(ka, smem, P, NQB, pre, ent);
   if (warp == 0) {
-    run_producer<D>(ka, P, NQB, pre, cr, lane);
+    run_producer<D>(ka, P, NQB, pre, ent, cr, lane);
   } else {
-    const AttnSmem lay(ka.ring_bytes, ka.n, ka.scr_floats);
+    const AttnSmem lay(ka.ring_bytes, ka.n, ka.scr_floats, ka.fused);
     float* scr = reinterpret_cast<float*>(smem + lay.scr) + (warp - 1) * ka.scr_floats;
     run_consumer_mma<D, NG>(ka, cr, P, warp - 1, lane, scr);
   }
-  attn_epilogue(ka.a);
+  attn_epilogue(ka, ent);
 }
 
 // ------------------------------------------------------------------ combine --
@@ -1860,8 +2293,8 @@ static bool use_mma(const Layout& l) {
 
 // Ring bytes an attention call with n queries gets, or -1 when one stage of the
 // widest page (one KV slice, its positions) or of the query rows would not fit.
-static int attn_ring_bytes(const Layout& l, int n, int hpu, int scr_floats, int limit) {
-  const int fixed = AttnSmem(0, n, scr_floats).total;
+static int attn_ring_bytes(const Layout& l, int n, int hpu, int scr_floats, int fused, int limit) {
+  const int fixed = AttnSmem(0, n, scr_floats, fused).total;
   const int ring = (limit - fixed) / 128 * 128;
   const int widest = static_cast<int>(l.slice[3]) + 4 * l.P;
   const int qrows = hpu * 2 * l.d;
@@ -1876,11 +2309,11 @@ constexpr int kMaxLaunchQueries = 1024;
 static cudaError_t launch_one(const Layout& l, const AttnKernelArgs& ka, int num_sms, cudaStream_t s) {
   const bool mma = use_mma(l);
   const int ctas = mma ? kMmaCtasPerSm : cc_ctas_per_sm(l.d);
-  const int ring = attn_ring_bytes(l, ka.n, ka.hpu, ka.scr_floats, attn_smem_limit(ctas));
+  const int ring = attn_ring_bytes(l, ka.n, ka.hpu, ka.scr_floats, ka.fused, attn_smem_limit(ctas));
   if (ring < 0) return cudaErrorInvalidConfiguration;
   AttnKernelArgs k = ka;
   k.ring_bytes = ring;
-  const size_t sm = static_cast<size_t>(AttnSmem(ring, k.n, k.scr_floats).total);
+  const size_t sm = static_cast<size_t>(AttnSmem(ring, k.n, k.scr_floats, k.fused).total);
   const dim3 grid(ctas * num_sms), block(32 * (kNcw + 1));
   if (mma) {
     const int ng = l.d / l.G;
@@ -1916,15 +2349,27 @@ static cudaError_t launch_one(const Layout& l, const AttnKernelArgs& ka, int num
 
 // The launches of an attention call with the given scratch views in `a`; *launches
 // counts them.
+// `step` (a decode step: k, v, bits given) and `early` (the layer's cache state is
+// settled, see cache_layer_settled) select the kernel's modes.
+struct StepInputs {
+  const void* k;
+  const void* v;
+  const uint8_t* bits;
+};
 static cudaError_t launch_attention(const Layout& l, const LayerArgs& a, int num_sms, int n,
                                     const int32_t* seq_ids, const int32_t* q_positions, const void* q_bf16,
                                     const uint8_t* modes, const float* mode_logits, const int32_t* windows,
                                     int window_scalar, float softmax_scale, void* out_bf16, cudaStream_t s,
-                                    int* launches) {
+                                    int* launches, bool early, const StepInputs* step = nullptr) {
   *launches = 0;
   AttnKernelArgs ka;
   ka.a = a;
   ka.window_scalar = window_scalar;
+  ka.early = early ? 1 : 0;
+  ka.fused = step ? 1 : 0;
+  ka.k = step ? static_cast<const uint16_t*>(step->k) : nullptr;
+  ka.v = step ? static_cast<const uint16_t*>(step->v) : nullptr;
+  ka.bits = step ? step->bits : nullptr;
   const float scale = softmax_scale > 0.f ? softmax_scale : 1.f / sqrtf(static_cast<float>(l.d));
   ka.qscale = scale * 1.4426950408889634f;
   const bool mma = use_mma(l);
@@ -1946,6 +2391,7 @@ static cudaError_t launch_attention(const Layout& l, const LayerArgs& a, int num
     ka.q = static_cast<const uint16_t*>(q_bf16) + q0 * row;
     ka.out = static_cast<uint16_t*>(out_bf16) + q0 * row;
     ka.a.cnt = a.cnt + static_cast<int64_t>(q0) * l.Hq * l.cnt_stride;
+    ka.early = early && q0 == 0 ? 1 : 0;  // a later launch follows one on the same layer
     cudaError_t e = launch_one(l, ka, num_sms, s);
     if (e != cudaSuccess) return e;
     ++*launches;
@@ -1981,11 +2427,44 @@ extern "C" trr_status trr_decode_attn(trr_cache* cache, int32_t layer, int32_t n
   if (!seq_ids || !q_positions || !q_bf16 || !modes || !out_bf16) return TRR_ERR_INVALID_ARG;
   if ((reinterpret_cast<uintptr_t>(q_bf16) | reinterpret_cast<uintptr_t>(out_bf16)) & 15)
     return TRR_ERR_INVALID_ARG;
-  const LayerArgs a = layer_args(l, cache_views(cache), layer);
+  LayerArgs a = layer_args(l, cache_views(cache), layer);
+  a.wait_ns = cache_wait_ns(cache);
+  const bool early = cache_layer_settled(cache, layer);
+  cache_note_call(cache, layer);
   int launches = 0;
   const cudaError_t e = launch_attention(l, a, cache_num_sms(cache), n, seq_ids, q_positions, q_bf16, modes,
                                          nullptr, windows, window_scalar, softmax_scale, out_bf16,
-                                         static_cast<cudaStream_t>(stream), &launches);
+                                         static_cast<cudaStream_t>(stream), &launches, early);
+  cache_set_launches(cache, launches);
+  return e == cudaSuccess ? TRR_OK : TRR_ERR_CUDA;
+}
+
+extern "C" trr_status trr_decode_step(trr_cache* cache, int32_t layer, int32_t n, const int32_t* seq_ids,
+                                      const int32_t* positions, const void* k_bf16, const void* v_bf16,
+                                      const uint8_t* bits, const uint8_t* modes, const void* q_bf16,
+                                      const int32_t* windows, int32_t window_scalar, float softmax_scale,
+                                      void* out_bf16, void* stream) {
+  if (!cache) return TRR_ERR_INVALID_ARG;
+  const Layout& l = cache_layout(cache);
+  if (layer < 0 || layer >= l.L || n < 0 || n > l.max_queries || n > l.max_append || n > kStepMax)
+    return TRR_ERR_INVALID_ARG;
+  cache_set_launches(cache, 0);
+  if (n == 0) return TRR_OK;
+  if (!seq_ids || !positions || !k_bf16 || !v_bf16 || !bits || !modes || !q_bf16 || !out_bf16)
+    return TRR_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(q_bf16) | reinterpret_cast<uintptr_t>(out_bf16) |
+       reinterpret_cast<uintptr_t>(k_bf16) | reinterpret_cast<uintptr_t>(v_bf16)) & 15)
+    return TRR_ERR_INVALID_ARG;
+  if (l.head_modes) return TRR_ERR_UNSUPPORTED;  // one mode per token
+  LayerArgs a = layer_args(l, cache_views(cache), layer);
+  a.wait_ns = cache_wait_ns(cache);
+  const bool early = cache_layer_settled(cache, layer);
+  cache_note_call(cache, layer);
+  const StepInputs step{k_bf16, v_bf16, bits};
+  int launches = 0;
+  const cudaError_t e = launch_attention(l, a, cache_num_sms(cache), n, seq_ids, positions, q_bf16, modes, nullptr,
+                                         windows, window_scalar, softmax_scale, out_bf16,
+                                         static_cast<cudaStream_t>(stream), &launches, early, &step);
   cache_set_launches(cache, launches);
   return e == cudaSuccess ? TRR_OK : TRR_ERR_CUDA;
 }
@@ -2004,11 +2483,14 @@ extern "C" trr_status trr_decode_attn_routed(trr_cache* cache, int32_t layer, in
       (reinterpret_cast<uintptr_t>(mode_logits) & 3))
     return TRR_ERR_INVALID_ARG;
   if (l.head_modes) return TRR_ERR_UNSUPPORTED;  // router decisions are per token
-  const LayerArgs a = layer_args(l, cache_views(cache), layer);
+  LayerArgs a = layer_args(l, cache_views(cache), layer);
+  a.wait_ns = cache_wait_ns(cache);
+  const bool early = cache_layer_settled(cache, layer);
+  cache_note_call(cache, layer);
   int launches = 0;
   const cudaError_t e = launch_attention(l, a, cache_num_sms(cache), n, seq_ids, q_positions, q_bf16, nullptr,
                                          mode_logits, windows, window_scalar, softmax_scale, out_bf16,
-                                         static_cast<cudaStream_t>(stream), &launches);
+                                         static_cast<cudaStream_t>(stream), &launches, early);
   cache_set_launches(cache, launches);
   return e == cudaSuccess ? TRR_OK : TRR_ERR_CUDA;
 }
@@ -2043,10 +2525,13 @@ static cudaError_t static_scratch(void** out) {
   return cudaSuccess;
 }
 
+// The call's attention control words sit at this offset among its control words.
+constexpr int kStaticLayerCtrl = 32;
+
 // Clears what a call needs at zero: the control words and the arrival counters.
 __global__ void static_scratch_clear_kernel(int32_t* wctrl, int32_t* cnt, int ncnt) {
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
-  if (i < kCtrlInts) wctrl[i] = i == kFirstBadQuery ? INT_MAX : 0;
+  if (i < kCtrlInts) wctrl[i] = i == kStaticLayerCtrl + kFirstBadQuery ? INT_MAX : 0;
   for (int j = i; j < ncnt; j += gridDim.x * blockDim.x) cnt[j] = 0;
 }
 
@@ -2080,8 +2565,10 @@ extern "C" trr_status trr_decode_attn_static(trr_cache* cache, int32_t layer, in
   if (static_scratch(&base) != cudaSuccess) return TRR_ERR_CUDA;
   uint8_t* b = static_cast<uint8_t*>(base);
   LayerArgs a = layer_args(l, cache_views(cache), layer);
+  a.wait_ns = cache_wait_ns(cache);
   int32_t* cache_ctrl = a.ctrl;
   a.ctrl = reinterpret_cast<int32_t*>(b);
+  a.lctl = a.ctrl + kStaticLayerCtrl;
   a.cnt = reinterpret_cast<int32_t*>(b + b_ctrl);
   a.part = reinterpret_cast<float*>(b + b_ctrl + b_cnt);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -2091,7 +2578,8 @@ extern "C" trr_status trr_decode_attn_static(trr_cache* cache, int32_t layer, in
   int launches = 0;
   if (e == cudaSuccess)
     e = launch_attention(l, a, cache_num_sms(cache), n, seq_ids, q_positions, q_bf16, modes, nullptr, windows,
-                         window_scalar, softmax_scale, out_bf16, s, &launches);
+                         window_scalar, softmax_scale, out_bf16, s, &launches, false);
+  cache_note_call(cache, layer);
   if (e != cudaSuccess) return TRR_ERR_CUDA;
   static_scratch_status_kernel<<<1, 1, 0, s>>>(a.ctrl, cache_ctrl);
   cache_set_launches(cache, launches + 2);

@@ -29,7 +29,9 @@ LayerArgs layer_args(const Layout& l, const Views& v, int layer) {
     a.pool[c] = v.pool[c];
   }
   const int64_t ls = static_cast<int64_t>(layer) * l.S;
+  a.wait_ns = kDefaultWaitNs;
   a.ctrl = v.ctrl;
+  a.lctl = v.lctl + static_cast<int64_t>(layer) * kLayerCtrlInts;
   a.last_pos = v.last_pos + ls;
   a.ntok = v.ntok + ls * 4;
   a.presence = v.presence + ls * l.W32;
@@ -102,6 +104,7 @@ static trr_status make_layout(const trr_cache_config* c, Layout* l) {
     return o;
   };
   l->off_ctrl = take(4 * kCtrlInts);
+  l->off_lctl = take(4 * static_cast<int64_t>(kLayerCtrlInts) * l->L);
   l->off_last_pos = take(4 * nls);
   l->off_ntok = take(16 * nls);
   l->off_presence = take(4 * nls * l->W32);
@@ -127,6 +130,8 @@ struct trr_cache {
   int device;
   int num_sms;
   int last_launches;
+  int recent[2];  // layers of the last two calls enqueued (-1: none; -2: every layer)
+  uint64_t wait_ns;  // bound of an in-kernel wait
 };
 
 using namespace trr;
@@ -140,8 +145,10 @@ extern "C" trr_status trr_cache_required_bytes(const trr_cache_config* cfg, uint
   return TRR_OK;
 }
 
-__global__ void init_ctrl_kernel(int32_t* ctrl) {
-  ctrl[threadIdx.x] = threadIdx.x == kFirstBadQuery ? INT_MAX : 0;
+__global__ void init_ctrl_kernel(int32_t* ctrl, int32_t* lctl, int nl) {
+  if (ctrl && threadIdx.x < kCtrlInts) ctrl[threadIdx.x] = 0;
+  for (int i = threadIdx.x; i < nl * kLayerCtrlInts; i += blockDim.x)
+    lctl[i] = i % kLayerCtrlInts == kFirstBadQuery ? INT_MAX : 0;
 }
 
 // Metadata to its empty state, stream-ordered.
@@ -149,7 +156,9 @@ static trr_status clear_metadata(trr_cache* c, cudaStream_t s) {
   const Layout& l = c->lay;
   uint8_t* b = static_cast<uint8_t*>(c->base);
   const int64_t nls = static_cast<int64_t>(l.L) * l.S;
-  init_ctrl_kernel<<<1, kCtrlInts, 0, s>>>(reinterpret_cast<int32_t*>(b + l.off_ctrl));
+  init_ctrl_kernel<<<1, 256, 0, s>>>(reinterpret_cast<int32_t*>(b + l.off_ctrl),
+                                     reinterpret_cast<int32_t*>(b + l.off_lctl), l.L);
+  c->recent[0] = c->recent[1] = -2;  // state changed by something other than a layer's call
   bool ok = cudaGetLastError() == cudaSuccess;
   ok = ok && cudaMemsetAsync(b + l.off_last_pos, 0xFF, 4 * nls, s) == cudaSuccess;
   ok = ok && cudaMemsetAsync(b + l.off_ntok, 0, 16 * nls, s) == cudaSuccess;
@@ -198,8 +207,10 @@ extern "C" trr_status trr_create_cache(const trr_cache_config* cfg, trr_cache** 
   }
   c->views = make_views(l, c->base);
   c->last_launches = 0;
+  c->wait_ns = kDefaultWaitNs;
   st = clear_metadata(c, nullptr);
   if (st == TRR_OK && cudaStreamSynchronize(nullptr) != cudaSuccess) st = TRR_ERR_CUDA;
+  c->recent[0] = c->recent[1] = -1;  // the cleared state is complete on the device
   if (st != TRR_OK) {
     if (c->owned) cudaFree(c->base);
     delete c;
@@ -233,7 +244,26 @@ extern "C" trr_status trr_get_status(trr_cache* c, void* stream) {
       cudaMemcpyAsync(&v, slot, 4, cudaMemcpyDeviceToHost, s) != cudaSuccess ||
       cudaStreamSynchronize(s) != cudaSuccess)
     return TRR_ERR_CUDA;
+  if (v == TRR_ERR_TIMEOUT) {
+    // a call gave up a wait and may have left split counters and the layers' work
+    // counters mid-count: back to their start values, so that the cache serves again
+    const Layout& l = c->lay;
+    uint8_t* b = static_cast<uint8_t*>(c->base);
+    init_ctrl_kernel<<<1, 256, 0, s>>>(nullptr, reinterpret_cast<int32_t*>(b + l.off_lctl), l.L);
+    if (cudaGetLastError() != cudaSuccess ||
+        cudaMemsetAsync(b + l.off_cnt, 0, 4 * static_cast<int64_t>(l.max_queries) * l.units * l.cnt_stride, s) !=
+            cudaSuccess ||
+        cudaStreamSynchronize(s) != cudaSuccess)
+      return TRR_ERR_CUDA;
+    c->recent[0] = c->recent[1] = -2;
+  }
   return static_cast<trr_status>(v);
+}
+
+extern "C" trr_status trr_set_wait_limit(trr_cache* c, uint64_t nanoseconds) {
+  if (!c) return TRR_ERR_INVALID_ARG;
+  c->wait_ns = nanoseconds ? nanoseconds : kDefaultWaitNs;
+  return TRR_OK;
 }
 
 extern "C" trr_status trr_reset(trr_cache* c, void* stream) {
@@ -271,4 +301,12 @@ const Layout& cache_layout(const trr_cache* c) { return c->lay; }
 const Views& cache_views(const trr_cache* c) { return c->views; }
 int cache_num_sms(const trr_cache* c) { return c->num_sms; }
 void cache_set_launches(trr_cache* c, int n) { c->last_launches = n; }
+bool cache_layer_settled(const trr_cache* c, int layer) {
+  return c->recent[0] != -2 && c->recent[1] != -2 && c->recent[0] != layer && c->recent[1] != layer;
+}
+uint64_t cache_wait_ns(const trr_cache* c) { return c->wait_ns; }
+void cache_note_call(trr_cache* c, int layer) {
+  c->recent[1] = c->recent[0];
+  c->recent[0] = layer;
+}
 }  // namespace trr

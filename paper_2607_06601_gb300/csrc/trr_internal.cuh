@@ -20,11 +20,17 @@ enum Ctrl : int {
   kNextPage = 4,      // [4] pages handed out per class
   kAppendOk = 10,     // append: 1 when the plan kernel committed the call
   kAppendDone = 11,   // one-kernel append: CTAs finished (the last one commits)
-  kFirstBadQuery = 12,// attention: min of (query index * 16 + error) over failing queries
-                      // (INT_MAX = none)
-  kDoneCtas = 14,     // attention: CTAs finished (the last one records the status)
-  kNextUnit = 15,     // attention: next work unit to hand out
   kCtrlInts = 64
+};
+
+// Control words of the attention kernels, one set per layer (an attention or decode-step
+// kernel of one layer may start while the previous layer's kernel still runs).
+enum LayerCtrl : int {
+  kNextUnit = 0,      // next work unit to hand out
+  kDoneCtas = 1,      // CTAs finished (the last one records the status)
+  kFirstBadQuery = 2, // min of (query index * 16 + error) over failing queries (INT_MAX = none)
+  kAborted = 3,       // 1 when a CTA gave up a wait (a decode step then commits nothing)
+  kLayerCtrlInts = 4
 };
 
 // Splits of one attention work unit are sized to hold at most this many pages (+ one
@@ -46,7 +52,7 @@ struct Layout {
   int cnt_stride; // arrival counters per (query, head): 1 + ceil(s_cap / kMergeGroup)
   int64_t max_items;
   int64_t hdr, tokb[kClasses], slice[kClasses], maskb, page_bytes[kClasses];
-  int64_t off_ctrl, off_last_pos, off_ntok, off_presence, off_pt, off_pfirst, off_plast, off_lastpg;
+  int64_t off_ctrl, off_lctl, off_last_pos, off_ntok, off_presence, off_pt, off_pfirst, off_plast, off_lastpg;
   int64_t off_aplan, off_cnt, off_part, off_pool[kClasses], total;
 };
 
@@ -71,6 +77,7 @@ struct AppendPlan {
 
 struct Views {  // typed device pointers into the cache memory
   int32_t* ctrl;
+  int32_t* lctl;
   int32_t* last_pos;
   int32_t* ntok;
   uint32_t* presence;
@@ -88,6 +95,7 @@ inline Views make_views(const Layout& l, void* base) {
   uint8_t* b = static_cast<uint8_t*>(base);
   Views v;
   v.ctrl = reinterpret_cast<int32_t*>(b + l.off_ctrl);
+  v.lctl = reinterpret_cast<int32_t*>(b + l.off_lctl);
   v.last_pos = reinterpret_cast<int32_t*>(b + l.off_last_pos);
   v.ntok = reinterpret_cast<int32_t*>(b + l.off_ntok);
   v.presence = reinterpret_cast<uint32_t*>(b + l.off_presence);
@@ -106,12 +114,14 @@ inline Views make_views(const Layout& l, void* base) {
 struct LayerArgs {
   int layer, S, Hq, Hkv, d, G, P, maxctx, MP, W32, units, pos_split, s_cap, cnt_stride, split_bytes, skip_writes_kv;
   int head_modes;      // modes are [n][Hq]; each KV head's slice ends with its presence mask
+  uint64_t wait_ns;    // bound of an in-kernel wait before the kernel reports TRR_ERR_TIMEOUT
   int maskb;           // bytes that end a slice for its presence mask (16, or 0 without head_modes)
   int cap[kClasses];
   int hdr;
   int slice[kClasses];
   int64_t page_bytes[kClasses];
   int32_t* ctrl;
+  int32_t* lctl;       // this layer's attention control words [kLayerCtrlInts]
   int32_t* last_pos;   // this layer: [S]
   int32_t* ntok;       // this layer: [S][4]
   uint32_t* presence;  // this layer: [S][W32]
@@ -132,6 +142,14 @@ const Layout& cache_layout(const trr_cache* c);
 const Views& cache_views(const trr_cache* c);
 int cache_num_sms(const trr_cache* c);
 void cache_set_launches(trr_cache* c, int n);
+// Whether a kernel of a call on `layer` may read that layer's cache state before the
+// previous kernel of the stream has finished: true when neither of the two calls
+// enqueued before it on this cache touched the layer (with programmatic dependent
+// launch, a kernel starts only once its predecessor has passed its own wait, so every
+// kernel before that one has finished).  cache_note_call records a call.
+bool cache_layer_settled(const trr_cache* c, int layer);
+void cache_note_call(trr_cache* c, int layer);
+uint64_t cache_wait_ns(const trr_cache* c);
 
 // One-time kernel attribute setup (defined in trr_attn.cu).
 cudaError_t attn_configure();
@@ -169,21 +187,57 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
       : "memory");
 }
 
-// Bounded wait for phase `parity` of `bar`: returns false when it gave up.  Each try
-// parks the thread until the phase completes or about 20 us pass, so a waiting warp
-// does not take issue slots; at most max_tries tries (about a second).
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint32_t max_tries = 50000) {
-  uint32_t addr = smem_u32(bar);
-  for (uint32_t i = 0; i < max_tries; ++i) {
-    uint32_t done;
-    asm volatile(
-        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n selp.u32 %0, 1, 0, p;\n}"
-        : "=r"(done)
-        : "r"(addr), "r"(parity), "r"(20000)
-        : "memory");
-    if (done) return true;
+// The global nanosecond timer.
+__device__ __forceinline__ uint64_t global_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+// Default bound of an in-kernel wait (trr_set_wait_limit changes it per cache).
+constexpr uint64_t kDefaultWaitNs = 2000000000ull;
+
+// One try at phase `parity` of `bar`: parks the thread until the phase completes or
+// about hint_ns pass (the hint is an upper bound: a try may return sooner), so that a
+// waiting warp does not take issue slots.
+__device__ __forceinline__ bool mbar_try(uint32_t addr, uint32_t parity, uint32_t hint_ns) {
+  uint32_t done;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n selp.u32 %0, 1, 0, p;\n}"
+      : "=r"(done)
+      : "r"(addr), "r"(parity), "r"(hint_ns)
+      : "memory");
+  return done != 0;
+}
+
+// Whether phase `parity` has completed, without suspending.
+__device__ __forceinline__ bool mbar_test_at(uint32_t addr, uint32_t parity) {
+  uint32_t done;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+      : "=r"(done)
+      : "r"(addr), "r"(parity)
+      : "memory");
+  return done != 0;
+}
+
+// One try of a wait bounded by limit_ns: a suspending try (a try may last until the
+// phase completes), or, for a limit below the 20 us hint, a test that returns at once,
+// so that a short limit is kept.
+__device__ __forceinline__ bool mbar_poll(uint32_t addr, uint32_t parity, uint64_t limit_ns) {
+  return limit_ns >= 20000 ? mbar_try(addr, parity, 20000u) : mbar_test_at(addr, parity);
+}
+
+// Bounded wait for phase `parity` of `bar`: returns false once limit_ns have passed
+// (measured on the global timer) without the phase completing.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint64_t limit_ns = kDefaultWaitNs) {
+  const uint32_t addr = smem_u32(bar);
+  if (mbar_poll(addr, parity, limit_ns)) return true;
+  const uint64_t t0 = global_ns();
+  for (;;) {
+    if (mbar_poll(addr, parity, limit_ns)) return true;
+    if (global_ns() - t0 >= limit_ns) return false;
   }
-  return false;
 }
 
 // atomic add with release (of what this thread has seen written) and acquire (of what
@@ -210,6 +264,90 @@ __device__ __forceinline__ int hard_decision(const float* z) {
     }
   }
   return best;
+}
+
+// ---------------------------------------------------------------- quantiser --
+// Eq. 4 of Sec. 3.2(C), shared by the append kernels and the decode-step kernel so that
+// both store the same bytes.
+
+__device__ __forceinline__ float bf16lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+
+// round((x - z) / s) of Eq. 4 on the exact quotient, ties to even, clamped to [0, levels].
+// u = fl32(fl32(x - z) * rs) with rs = fl32(1 / s) is within 3 binary32 roundings, under
+// 2^-21 |u|, of the exact quotient, so rint(u) is exact unless u lies that close to a
+// half-way point c + 1/2.  There the midpoint z + (c + 1/2) s is formed in binary64,
+// where it is exact (z and s are binary16: a multiple of 2^-25 below 2^18), and compared
+// with x (a bf16 value).  Only half-way points inside [0, levels] matter: the clamp
+// settles the others.
+__device__ __forceinline__ int code_of(float x, float z, float s, float rs, int levels) {
+  const float u = __fmul_rn(__fsub_rn(x, z), rs);
+  const float fl = floorf(u);
+  if (fabsf(__fsub_rn(u, fl + 0.5f)) <= fabsf(u) * 0x1p-21f && fl >= 0.f && fl < static_cast<float>(levels)) {
+    const double mid = __dadd_rn(static_cast<double>(z), __dmul_rn(static_cast<double>(fl) + 0.5, static_cast<double>(s)));
+    const double xd = static_cast<double>(x);
+    const int c = static_cast<int>(fl);
+    return (xd > mid || (xd == mid && (c & 1))) ? c + 1 : c;
+  }
+  return min(max(__float2int_rn(u), 0), levels);
+}
+
+// One row of D values (a token's K or V for one KV head) quantised by a warp at b < 16
+// bits: lane l holds values EPL*l .. EPL*l + EPL-1 (EPL = D/32) as bf16 in raw; a group's
+// min / max by shuffles over its G/EPL lanes; codes packed LSB-first.  The lane writes
+// code word `code_idx` (of the row's D*b/32 words) when code_idx >= 0 and the group's
+// (s, z) word `sz_idx` when sz_idx >= 0.  A group holding a value binary16 cannot carry
+// (non-finite or |x| > 65504) gets zero codes and a zero (s, z) word, and bad = true.
+struct RowCodes {
+  uint32_t code_word, sz_word;
+  int code_idx, sz_idx;
+  bool bad;
+};
+template <int D>
+__device__ __forceinline__ RowCodes quantise_row_codes(const uint2 w, int b, int G, int lane) {
+  constexpr int EPL = D / 32;
+  float x[EPL];
+  x[0] = bf16lo(w.x);
+  x[1] = bf16hi(w.x);
+  if (EPL == 4) {
+    x[EPL > 2 ? 2 : 0] = bf16lo(w.y);
+    x[EPL > 3 ? 3 : 1] = bf16hi(w.y);
+  }
+  const int GL = G / EPL;  // lanes of one group
+  float mn = x[0], mx = x[0];
+  bool bad = false;
+#pragma unroll
+  for (int i = 0; i < EPL; ++i) {
+    bad |= !(fabsf(x[i]) <= 65504.f);  // also true for NaN
+    mn = fminf(mn, x[i]);
+    mx = fmaxf(mx, x[i]);
+  }
+  for (int o = 1; o < GL; o <<= 1) {
+    mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, o));
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    bad |= __shfl_xor_sync(0xffffffffu, static_cast<int>(bad), o) != 0;
+  }
+  const int levels = (1 << b) - 1;
+  uint32_t val = 0, szw = 0;
+  if (!bad) {
+    const __half z16 = __float2half_rn(mn);                                                    // z = min(x)
+    const __half s16 = __float2half_rn(__fdiv_rn(__fsub_rn(mx, mn), static_cast<float>(levels)));  // s
+    const float z = __half2float(z16), s = __half2float(s16), rs = __frcp_rn(s);
+#pragma unroll
+    for (int i = 0; i < EPL; ++i)
+      val |= static_cast<uint32_t>(s != 0.f ? code_of(x[i], z, s, rs, levels) : 0) << (i * b);
+    szw = static_cast<uint32_t>(__half_as_ushort(s16)) | (static_cast<uint32_t>(__half_as_ushort(z16)) << 16);
+  }
+  const int LPW = 32 / (EPL * b);  // lanes sharing one 32-bit word of codes
+  val <<= (lane % LPW) * EPL * b;
+  for (int o = 1; o < LPW; o <<= 1) val |= __shfl_xor_sync(0xffffffffu, val, o);
+  RowCodes r;
+  r.code_word = val;
+  r.sz_word = szw;
+  r.code_idx = lane % LPW == 0 ? lane / LPW : -1;
+  r.sz_idx = lane % GL == 0 ? lane / GL : -1;
+  r.bad = bad;
+  return r;
 }
 
 __device__ __forceinline__ void set_status(int32_t* ctrl, int code) {

@@ -40,8 +40,9 @@ class trr_cache_config(ctypes.Structure):
 
 
 EXPORTS = ("trr_cache_required_bytes", "trr_create_cache", "trr_kv_append", "trr_decode_attn",
-           "trr_decode_attn_static", "trr_route_decisions", "trr_kv_append_routed",
-           "trr_decode_attn_routed", "trr_destroy", "trr_get_status", "trr_reset", "trr_get_region",
+           "trr_decode_step", "trr_decode_attn_static", "trr_route_decisions", "trr_kv_append_routed",
+           "trr_decode_attn_routed", "trr_destroy", "trr_get_status", "trr_set_wait_limit", "trr_reset",
+           "trr_get_region",
            "trr_last_launch_count")
 
 _lib = None
@@ -68,11 +69,13 @@ def load(build_if_missing: bool = False) -> ctypes.CDLL:
     L.trr_kv_append.argtypes = [P, I32, I32, P, P, P, P, P, P, P]
     L.trr_decode_attn.argtypes = [P, I32, I32, P, P, P, P, P, I32, ctypes.c_float, P, P]
     L.trr_decode_attn_static.argtypes = [P, I32, I32, P, P, P, P, P, I32, ctypes.c_float, P, P]
+    L.trr_decode_step.argtypes = [P, I32, I32, P, P, P, P, P, P, P, P, I32, ctypes.c_float, P, P]
     L.trr_route_decisions.argtypes = [I32, P, P, P, I32, I32, I32, I32, I32, P, P, P, P, P, P]
     L.trr_kv_append_routed.argtypes = [P, I32, I32, P, P, P, P, P, P, P]
     L.trr_decode_attn_routed.argtypes = [P, I32, I32, P, P, P, P, P, I32, ctypes.c_float, P, P]
     L.trr_destroy.argtypes = [P]
     L.trr_get_status.argtypes = [P, P]
+    L.trr_set_wait_limit.argtypes = [P, U64]
     L.trr_reset.argtypes = [P, P]
     L.trr_get_region.argtypes = [P, I32, ctypes.POINTER(P), ctypes.POINTER(U64)]
     L.trr_last_launch_count.argtypes = [P]
@@ -150,6 +153,19 @@ def trr_decode_attn(cache, layer, seq_ids, q_positions, q, modes, windows, windo
         _dev(q_positions, torch.int32, "q_positions"), _dev(q, torch.bfloat16, "q"),
         _dev(modes, torch.uint8, "modes"), win, int(window_scalar), float(softmax_scale),
         _dev(out, torch.bfloat16, "out"), _stream(stream)))
+
+
+def trr_decode_step(cache, layer, seq_ids, positions, k, v, bits, modes, q, windows, window_scalar,
+                    softmax_scale, out, stream=None):
+    """One decode step of one layer in one kernel: the append of every entry's token, then
+    every entry's query at the same position and mode (see include/trr.h)."""
+    n = seq_ids.numel()
+    win = None if windows is None else _dev(windows, torch.int32, "windows")
+    _check("trr_decode_step", load().trr_decode_step(
+        cache, layer, n, _dev(seq_ids, torch.int32, "seq_ids"), _dev(positions, torch.int32, "positions"),
+        _dev(k, torch.bfloat16, "k"), _dev(v, torch.bfloat16, "v"), _dev(bits, torch.uint8, "bits"),
+        _dev(modes, torch.uint8, "modes"), _dev(q, torch.bfloat16, "q"), win, int(window_scalar),
+        float(softmax_scale), _dev(out, torch.bfloat16, "out"), _stream(stream)))
 
 
 def trr_decode_attn_static(cache, layer, seq_ids, q_positions, q, modes, windows, window_scalar,
@@ -272,6 +288,15 @@ class Cache:
                         softmax_scale, out, stream)
         return out
 
+    def decode_step(self, layer, seq_ids, positions, k, v, bits, modes, q, windows=None, window_scalar=0,
+                    softmax_scale=0.0, out=None, stream=None):
+        self._check_modes(modes, seq_ids.numel())
+        if out is None:
+            out = torch.empty((seq_ids.numel(), self.Hq, self.d), dtype=torch.bfloat16, device=q.device)
+        trr_decode_step(self.handle, layer, seq_ids, positions, k, v, bits, modes, q, windows, window_scalar,
+                        softmax_scale, out, stream)
+        return out
+
     def append_routed(self, layer, seq_ids, positions, k, v, bit_logits, mode_logits, stream=None):
         trr_kv_append_routed(self.handle, layer, seq_ids, positions, k, v, bit_logits, mode_logits, stream)
 
@@ -285,6 +310,10 @@ class Cache:
 
     def status(self, stream=None) -> int:
         return trr_get_status(self.handle, stream)
+
+    def set_wait_limit(self, nanoseconds: int):
+        """Bound of every in-kernel wait of this cache's calls (0: the default, 2 s)."""
+        _check("trr_set_wait_limit", load().trr_set_wait_limit(self.handle, int(nanoseconds)))
 
     def reset(self, stream=None):
         trr_reset(self.handle, stream)

@@ -34,8 +34,10 @@ BITS = (2, 4, 8, 16)
 def bf16_bits(x) -> np.ndarray:
     """Round float32 values to bf16 (nearest, ties to even); return the uint16 bits."""
     x = np.ascontiguousarray(x, dtype=np.float32)
-    u = x.view(np.uint32).astype(np.uint64)
-    rounded = (u + 0x7FFF + ((u >> 16) & 1)) >> 16
+    u = x.view(np.uint32)
+    # in 32-bit arithmetic: no finite value or infinity carries out of the word (the
+    # largest, 0xFF7FFFFF + 0x8000, stays below 2^32); NaNs are set below
+    rounded = (u + np.uint32(0x7FFF) + ((u >> np.uint32(16)) & np.uint32(1))) >> np.uint32(16)
     out = rounded.astype(np.uint16)
     nan = np.isnan(x)
     if nan.any():

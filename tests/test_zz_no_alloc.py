@@ -77,3 +77,35 @@ def test_static_scratch_refuses_calls_larger_than_the_array():
     assert err.value.code == 2  # TRR_ERR_OUT_OF_MEMORY: nothing launched
     assert cache.launches() == 0
     assert cache.status() == 0
+
+
+@pytest.mark.parametrize("Hkv", [4, 8])  # query groups of 2 (tensor cores), MHA (CUDA cores)
+def test_static_scratch_above_one_launch_of_queries(Hkv):
+    """About 1100 queries: the static entry point runs them as two launches, the second
+    with its arrival counters offset into the array; every row matches trr_decode_attn
+    called in chunks of the cache's max_queries, on two calls in a row."""
+    if not torch.cuda.is_available():
+        pytest.skip("needs a GPU")
+    torch.cuda.set_device(0)
+    rng = np.random.default_rng(79 + Hkv)
+    S, Hq, d = 6, 8, 64
+    cache = _cache_with_context(rng, S=S, Hq=Hq, Hkv=Hkv, d=d)
+    nq = 1100
+    seqs = dev(rng.integers(0, S, nq).astype(np.int32), torch.int32)
+    ts = dev(rng.integers(0, 400, nq).astype(np.int32), torch.int32)
+    q = dev(wl.bf16_bits(rng.standard_normal((nq, Hq, d), dtype=np.float32)), torch.bfloat16)
+    modes = dev(rng.choice(3, size=nq).astype(np.uint8), torch.uint8)
+    wins = dev(rng.choice([1, 7, 64, 300], size=nq).astype(np.int32), torch.int32)
+    ref = torch.empty((nq, Hq, d), dtype=torch.bfloat16, device="cuda")
+    for i0 in range(0, nq, 16):
+        sl = slice(i0, min(nq, i0 + 16))
+        trr.trr_decode_attn(cache.handle, 0, seqs[sl].contiguous(), ts[sl].contiguous(), q[sl].contiguous(),
+                            modes[sl].contiguous(), wins[sl].contiguous(), 0, 0.0, ref[sl])
+    ref_np = ref.float().cpu().numpy().astype(np.float64)
+    for _ in range(2):
+        out = torch.full((nq, Hq, d), float("nan"), dtype=torch.bfloat16, device="cuda")
+        trr.trr_decode_attn_static(cache.handle, 0, seqs, ts, q, modes, wins, 0, 0.0, out)
+        got = out.float().cpu().numpy().astype(np.float64)
+        check_attention(got, ref_np, modes.cpu().numpy())
+    assert cache.launches() >= 4  # clear kernel, two attention launches (and combines), status kernel
+    assert cache.status() == 0
