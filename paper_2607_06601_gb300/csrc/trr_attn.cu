@@ -147,52 +147,51 @@ __device__ __forceinline__ void fmul2_inplace(float& x0, float& x1, float f0, fl
   x1 = r.y;
 }
 
-template <int BFROM, int BTO, int E>
-__device__ __forceinline__ void rescale_q(float (&qp)[E]) {
-#pragma unroll
-  for (int i = 0; i < E; i += 2)
-    fmul2_inplace(qp[i], qp[i + 1], pow2f(qe_of(BTO, i) - qe_of(BFROM, i)),
-                  pow2f(qe_of(BTO, i + 1) - qe_of(BFROM, i + 1)));
+// The factors that move a lane's query and V accumulators between the domains of two
+// width classes, element by element (E = 32 elements per lane): row from * 4 + to.  One
+// table read by every class change keeps a single copy of the code in the consumer's
+// loop (a switch over templated copies made the loop several kilobytes larger).
+struct RescaleTable {
+  float q[16][32];    // query: 2^(qe(to, i) - qe(from, i))
+  float acc[16][32];  // V accumulators: 2^(ex(to, i) - ex(from, i)), ex = 0 at width 16
+};
+__host__ __device__ constexpr float pow2c(int e) {
+  float r = 1.f;
+  for (; e > 0; --e) r *= 2.f;
+  for (; e < 0; ++e) r *= 0.5f;
+  return r;
 }
-
-// V is accumulated as acc_i * 2^(ex_i(B) - 49) while class B's pages are consumed
-// (B = 16: ex = 0), so that every element of a key takes the same weight p*s*2^100.
-template <int BFROM, int BTO, int E>
-__device__ __forceinline__ void rescale_acc(float (&acc)[E]) {
-#pragma unroll
-  for (int i = 0; i < E; i += 2)
-    fmul2_inplace(acc[i], acc[i + 1],
-                  pow2f((BTO == 16 ? 0 : ex_of(BTO, i)) - (BFROM == 16 ? 0 : ex_of(BFROM, i))),
-                  pow2f((BTO == 16 ? 0 : ex_of(BTO, i + 1)) - (BFROM == 16 ? 0 : ex_of(BFROM, i + 1))));
+__host__ __device__ constexpr RescaleTable make_rescale_table() {
+  RescaleTable t{};
+  for (int from = 0; from < 4; ++from)
+    for (int to = 0; to < 4; ++to)
+      for (int i = 0; i < 32; ++i) {
+        const int bf = bits_of_class(from), bt = bits_of_class(to);
+        t.q[from * 4 + to][i] = pow2c(qe_of(bt, i) - qe_of(bf, i));
+        t.acc[from * 4 + to][i] = pow2c((bt == 16 ? 0 : ex_of(bt, i)) - (bf == 16 ? 0 : ex_of(bf, i)));
+      }
+  return t;
 }
+__constant__ RescaleTable kRescale = make_rescale_table();
 
-// qp and acc from the domain of class `from` to that of class `to` (from < to, or
-// from = 16: a unit's pages come class by class, a decode step's own token among its
-// class's pages).
+// qp and acc from the domain of class `from` to that of class `to`.
 template <int E>
 __device__ __forceinline__ void rescale_dyn(float (&qp)[E], float (&acc)[E], int from, int to) {
-  switch (from * 4 + to) {
-    case 1: rescale_q<2, 4>(qp); rescale_acc<2, 4>(acc); break;
-    case 2: rescale_q<2, 8>(qp); rescale_acc<2, 8>(acc); break;
-    case 3: rescale_q<2, 16>(qp); rescale_acc<2, 16>(acc); break;
-    case 6: rescale_q<4, 8>(qp); rescale_acc<4, 8>(acc); break;
-    case 7: rescale_q<4, 16>(qp); rescale_acc<4, 16>(acc); break;
-    case 11: rescale_q<8, 16>(qp); rescale_acc<8, 16>(acc); break;
-    case 12: rescale_q<16, 2>(qp); rescale_acc<16, 2>(acc); break;
-    case 13: rescale_q<16, 4>(qp); rescale_acc<16, 4>(acc); break;
-    case 14: rescale_q<16, 8>(qp); rescale_acc<16, 8>(acc); break;
-    default: break;
+  static_assert(E == 32, "one factor per element of a lane's 32");
+  const float* qf = kRescale.q[from * 4 + to];
+  const float* af = kRescale.acc[from * 4 + to];
+#pragma unroll
+  for (int i = 0; i < E; i += 2) {
+    fmul2_inplace(qp[i], qp[i + 1], qf[i], qf[i + 1]);
+    fmul2_inplace(acc[i], acc[i + 1], af[i], af[i + 1]);
   }
 }
 // acc from class `from`'s domain back to class 16's (the common one of the merge)
 template <int E>
 __device__ __forceinline__ void acc_to_neutral(float (&acc)[E], int from) {
-  switch (from) {
-    case 0: rescale_acc<2, 16>(acc); break;
-    case 1: rescale_acc<4, 16>(acc); break;
-    case 2: rescale_acc<8, 16>(acc); break;
-    default: break;
-  }
+  const float* af = kRescale.acc[from * 4 + 3];
+#pragma unroll
+  for (int i = 0; i < E; i += 2) fmul2_inplace(acc[i], acc[i + 1], af[i], af[i + 1]);
 }
 
 // 2^x with the hardware approximation (relative error about 2^-22; results below the
@@ -338,11 +337,13 @@ __device__ __forceinline__ void consume_page(uint32_t s0, uint32_t spos, bool ma
   constexpr int LPK = D / E;
   constexpr int KPI = 32 / LPK;
   constexpr int P = NIT * KPI;
-  constexpr int KP = NIT % 2 == 0 ? 2 : 1;  // keys per lane per iteration
+  constexpr int KP = 1;  // keys per lane per iteration (one: half the code of two, which the
+                         // instruction cache favours over the second key's overlap)
   constexpr int rowb = B == 16 ? 2 * D : D * B / 8;  // bytes of one key's row of K (or V)
   const int part = lane % LPK, kl = lane / LPK;
-  const int ng = D / G;
-  const int grp = part * E / G;
+  const int lg = __ffs(G) - 1;  // G is a power of two: shifts, not divisions
+  const int ng = D >> lg;
+  const int grp = (part * E) >> lg;
   const uint32_t krow = s0 + kl * rowb + part * (E * B / 8);   // this lane's K bytes, key kl
   const uint32_t ksz = s0 + 2 * P * rowb + (kl * ng + grp) * 4;  // its (s, z), key kl
   const uint32_t szstep = KPI * ng * 4;
@@ -422,8 +423,10 @@ __host__ __device__ constexpr int attn_smem_limit(int ctas) {
 // stage's full barrier:
 //   a = {meta, ring offset of the stage's bytes, query, lo}
 //   b = {hi (= t), split, splits, unit number of split 0}
-//   c = {first KV slice of the stage (block-relative), KV slices in it, ring offset of
-//        the page's slot positions or -1, bytes of one KV slice}; in a query-rows
+//   c = {first KV slice of the stage (block-relative), KV slices per page | pages of the
+//        stage << 8, ring offset of the page's slot positions or -1, bytes of one KV
+//        slice}; a stage of several pages holds full pages of one class, each page's
+//        slices after the previous page's (the last page's fill is in meta); in a query-rows
 //        stage {the block's head modes, 2 bits per head (per-head modes), the local
 //        window's first position, -1, 0}
 // meta = class | fill << 2 | flags | head block << 16.
@@ -530,7 +533,7 @@ struct AttnSmem {
         pre(scr + align16(kNcw * scr_floats * 4)),
         ent(pre + align16(4 * (n + 2))),
         red(ent + (fused ? align16(4 * step_ints(n)) : 0)),
-        flag(red + 16 * 8),
+        flag(red + 16 * 8),  // the abort flag; at flag + 8 the entry table's readiness mbarrier
         total(flag + 16) {}
 };
 
@@ -716,14 +719,19 @@ __device__ __forceinline__ unsigned seq_hash(int seq, int slots) {
 // entry first: sequence id, bit-width or mode not allowed, or a sequence named by an
 // earlier entry (INVALID_ARG); position outside [0, max_context) or not above the
 // sequence's last one (BAD_POSITION); a local query with a window below 1 (INVALID_ARG).
+// Run by the kNcw consumer warps (threads 32 .. 32 * (kNcw + 1) - 1) while the producer
+// plans its first unit; they synchronise among themselves on named barrier 1.
+__device__ __forceinline__ void consumers_sync() {
+  asm volatile("bar.sync 1, %0;" ::"r"(32 * kNcw) : "memory");
+}
 __device__ void plan_entries(const AttnKernelArgs& ka, int* ent) {
   const LayerArgs& a = ka.a;
-  const int n = ka.n, tid = threadIdx.x, nt = blockDim.x, H = 2 * n;
+  const int n = ka.n, tid = threadIdx.x - 32, nt = 32 * kNcw, H = 2 * n;
   int* hs = ent + 2 * n;  // [H][2]: sequence + 1, lowest entry index naming it
   int* sc = ent + 6 * n;
   for (int i = tid; i < 2 * H; i += nt) hs[i] = (i & 1) ? INT_MAX : 0;
   for (int i = tid; i < kSScalars; i += nt) sc[i] = i == kSErr ? INT_MAX : 0;
-  __syncthreads();
+  consumers_sync();
   for (int e = tid; e < n; e += nt) {
     const int seq = ka.seq_ids[e];
     if (seq < 0 || seq >= a.S) continue;
@@ -737,7 +745,7 @@ __device__ void plan_entries(const AttnKernelArgs& ka, int* ent) {
       h = h + 1 == static_cast<unsigned>(H) ? 0u : h + 1;
     }
   }
-  __syncthreads();
+  consumers_sync();
   for (int e = tid; e < n; e += nt) {
     const int seq = ka.seq_ids[e], pos = ka.q_positions[e], m = ka.modes[e], b = ka.bits[e];
     const int c = b == 2 ? 0 : b == 4 ? 1 : b == 8 ? 2 : b == 16 ? 3 : -1;
@@ -763,7 +771,7 @@ __device__ void plan_entries(const AttnKernelArgs& ka, int* ent) {
     ent[2 * e + 1] = info;
     if (err) atomicMin(&sc[kSErr], e * 16 + err);
   }
-  __syncthreads();
+  consumers_sync();
   if (tid < 32) {  // openers of the same class before each entry, 32 entries at a time
     int run0 = 0, run1 = 0, run2 = 0, run3 = 0;
     for (int e0 = 0; e0 < n; e0 += 32) {
@@ -781,7 +789,7 @@ __device__ void plan_entries(const AttnKernelArgs& ka, int* ent) {
     }
     if (tid < 4) sc[kSOpeners + tid] = tid == 0 ? run0 : tid == 1 ? run1 : tid == 2 ? run2 : run3;
   }
-  __syncthreads();
+  consumers_sync();
 }
 
 // One warp, after the wait on the previous kernel: the pools' page counters, and the
@@ -928,6 +936,7 @@ struct CtaRing {
   uint64_t* full;
   uint64_t* empty;
   volatile int* abort_flag;
+  uint64_t* ent_ready;  // decode step: completes when the consumers have built the entry table
   int R;
 };
 
@@ -956,9 +965,29 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
   int dq_slot = -1, dq_off = 0, dq_need = 0;
   int4 dq_ra = make_int4(0, 0, 0, 0), dq_rb = dq_ra, dq_rc = dq_ra;
   const uint16_t* dq_src = nullptr;
+  // decode step: the entry table the consumers build, waited for where it is first
+  // needed (the producer plans its first unit meanwhile); then, after the wait on the
+  // previous kernel, the pools' counters and whether a token runs out of pages (the call
+  // then stores nothing, and the last CTA zeroes every row)
+  bool have_ent = !ka.fused, have_pages = !ka.fused;
+  auto ent_sync = [&]() {
+    if (have_ent) return;
+    have_ent = true;
+    if (!mbar_wait(cr.ent_ready, 0, a.wait_ns)) {
+      if (lane == 0) {
+        *cr.abort_flag = 1;
+        set_status(a.ctrl, TRR_ERR_TIMEOUT);
+        atomicExch(&a.lctl[kAborted], 1);
+      }
+    }
+  };
   // the call's error once known (a decode step with an error stores nothing and every
   // query gets its zero rows)
-  auto call_failed = [&]() -> bool { return ka.fused && sc[kSErr] != INT_MAX; };
+  auto call_failed = [&]() -> bool {
+    if (!ka.fused) return false;
+    ent_sync();
+    return sc[kSErr] != INT_MAX;
+  };
   // after the wait on the previous kernel: let the next kernel start, read what the
   // previous kernel wrote (decode step: the pools' counters; the combine kernel's query
   // table), then complete the deferred query-rows stage
@@ -978,15 +1007,19 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
       int2* qtab = reinterpret_cast<int2*>(a.cnt);
       for (int q = lane; q < n; q += 32) qtab[q] = make_int2(pre[q], pre[q + 1] - pre[q]);
     }
-    // decode step: the pools' counters, and whether a token runs out of pages (then
-    // the call stores nothing, and the last CTA zeroes every row)
-    if (ka.fused) step_after_wait(ka, ent, lane);
   };
   auto ensure_waited = [&]() {
     if (waited) return;
     pdl_wait();
     waited = true;
     after_wait();
+  };
+  auto pages_ready = [&]() {  // decode step: next_page and the out-of-pages check
+    if (have_pages) return;
+    have_pages = true;
+    ensure_waited();
+    ent_sync();
+    step_after_wait(ka, ent, lane);
   };
   // wait for the oldest stage in flight to be released and take back its bytes
   auto release_one = [&]() -> bool {
@@ -1097,6 +1130,12 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
     }
     // decode step: this query's own token joins the last split of each head block
     const bool has_new = ka.fused && !err && bmode != TRR_MODE_SKIP && sp == ns - 1;
+    // the unit's pages, planned before the check that waits for the entry table
+    const int lo = bmode == TRR_MODE_FULL ? 0 : max(0, t - w + 1);
+    int wid = -1, wmeta = 0, wfirst = 0, wlast = INT_MAX, T = 0;
+    if (!err && bmode != TRR_MODE_SKIP)
+      T = plan_split(a, P, seq, lo, t, sp, ns, lane, wid, wmeta, a.head_modes ? &wfirst : nullptr,
+                     a.head_modes ? &wlast : nullptr);
     if (err || bmode == TRR_MODE_SKIP || call_failed()) {
       // zero rows (once per block); the error of the lowest query; a skip token that
       // stores KV has its rows written here
@@ -1107,6 +1146,7 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
       }
       if (!ka.fused && err && qb == 0 && lane == 0) atomicMin(&a.lctl[kFirstBadQuery], (ka.q0 + q) * 16 + err);
       if (ka.fused && !call_failed() && sp == 0 && ent[2 * q] >= 0) {
+        pages_ready();
         int c, pid, slot;
         step_slot(ka, ent, q, c, pid, slot);
         for (int j0 = kv0; j0 < kv0 + nkv; j0 += 4) {
@@ -1119,10 +1159,6 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
         }
       }
     } else {
-      const int lo = bmode == TRR_MODE_FULL ? 0 : max(0, t - w + 1);
-      int wid, wmeta, wfirst = 0, wlast = INT_MAX;
-      const int T = plan_split(a, P, seq, lo, t, sp, ns, lane, wid, wmeta, a.head_modes ? &wfirst : nullptr,
-                               a.head_modes ? &wlast : nullptr);
       const int lo_local = max(0, t - w + 1);
       // per-head modes: a page before the local window is read by the block's full heads
       // only; a page across the window's start brings its slot positions
@@ -1182,17 +1218,44 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
       bool new_done = !has_new;
       auto push_new = [&](bool last) -> bool {
         ensure_waited();  // the token's K / V rows come from the previous kernel
+        pages_ready();
         new_done = true;
         if (call_failed()) {
           int taken = 0;
           const int off = reserve(0, taken, true);
           if (off < 0) return false;
-          push(make_int4((last ? kLast : 0) | (qb << 16), off, q, lo), rb, make_int4(0, 0, -1, 0), taken, 0);
+          push(make_int4((last ? kLast : 0) | (qb << 16), off, q, lo), rb, make_int4(0, 1 << 8, -1, 0), taken, 0);
           return true;
         }
         int c, pid, slot;
         step_slot(ka, ent, q, c, pid, slot);
         const int slice = a.slice[c];
+        // every KV head's slot 0 in one stage when the class's regions allow it: head j's
+        // K codes, V codes, K (s, z) and V (s, z) each at j rows (j * rowb bytes) past the
+        // region's start, so that a consumer reads its head as a page-shaped slice at
+        // j * rowb; the reservation covers what the consumers read of the slots past the
+        // fill
+        const int b = bits_of_class(c), rowb = b == 16 ? 2 * D : D * b / 8, ng = D / a.G;
+        if (nkv <= 4 && (b == 16 || (nkv - 1) * rowb + ng * 4 <= P * ng * 4)) {
+          const int span = b == 16 ? (nkv - 1 + P + 16) * rowb : (nkv - 1) * rowb + 2 * P * rowb + (P + 16) * ng * 4;
+          int taken = 0;
+          const int off = reserve(align16(span), taken, true);
+          if (off < 0) return false;
+          uint2 rk[4], rv[4];
+          step_load_rows<D>(ka, q, kv0, nkv, rk, rv, lane);
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            if (k >= nkv) continue;
+            const int j = kv0 + k;
+            step_token_rows<D>(ka, rk[k], rv[k], j, c, pid, slot, j * g >= h0, smem_u32(cr.ring + off + k * rowb), true,
+                               lane);
+          }
+          fence_proxy_async_smem();  // these bytes are later overwritten by bulk copies
+          __syncwarp();
+          const int meta = c | (1 << 2) | (last ? kLast : 0) | (qb << 16);
+          push(make_int4(meta, off, q, lo), rb, make_int4(0, nkv | (1 << 8), -1, rowb), taken, 0);
+          return true;
+        }
         for (int j0 = 0; j0 < nkv; j0 += 4) {
           const int m = min(4, nkv - j0);
           uint2 rk[4], rv[4];
@@ -1208,7 +1271,7 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
             fence_proxy_async_smem();  // these bytes are later overwritten by bulk copies
             __syncwarp();
             const int meta = c | (1 << 2) | (last && k0 == nkv - 1 ? kLast : 0) | (qb << 16);
-            push(make_int4(meta, off, q, lo), rb, make_int4(k0, 1, -1, slice), taken, 0);
+            push(make_int4(meta, off, q, lo), rb, make_int4(k0, 1 | (1 << 8), -1, slice), taken, 0);
           }
         }
         return true;
@@ -1216,12 +1279,42 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
       for (int j = 0; j < T && ok; ++j) {
         const uint8_t* page = reinterpret_cast<const uint8_t*>(__shfl_sync(0xffffffffu, pg_src, j));
         const int geo = __shfl_sync(0xffffffffu, pg_geo, j);
-        const int pm = __shfl_sync(0xffffffffu, wmeta, j);
+        int pm = __shfl_sync(0xffffffffu, wmeta, j);
         const unsigned needed = __shfl_sync(0xffffffffu, pg_need, j);
         const int slice = geo & 0xfffff, maxk = geo >> 20;
         if (!new_done && (pm & 3) > new_cls && !push_new(false)) {
           ok = false;
           break;
+        }
+        const unsigned all = (1u << nkv) - 1u;
+        if (!a.head_modes && !(pm & kMask) && needed == all && nkv <= maxk) {
+          // a run of full pages of this class, every KV head of the block: one stage
+          // holding up to R/2 bytes of them (a page's slices after the other), one copy
+          // per page; only the run's last page may hold fewer than P tokens
+          const int pb = nkv * slice;
+          int run = 1;
+          while (j + run < T && (run + 1) * pb <= R / 2) {
+            const int pm2 = __shfl_sync(0xffffffffu, wmeta, j + run);
+            if ((pm2 & (3 | kMask)) != (pm & 3) || ((pm >> 2) & 127) != P) break;
+            pm = pm2;
+            ++run;
+          }
+          int taken = 0;
+          const int off = reserve_any(run * pb, taken);
+          if (off < 0) {
+            ok = false;
+            break;
+          }
+          const bool last = j + run == T && new_done;
+          const int meta = pm | (last ? kLast : 0) | (qb << 16);
+          const uint32_t slot =
+              push(make_int4(meta, off, q, lo), rb, make_int4(0, nkv | (run << 8), -1, slice), taken, run * pb);
+          for (int r = 0; r < run; ++r) {
+            const uint8_t* pg = reinterpret_cast<const uint8_t*>(__shfl_sync(0xffffffffu, pg_src, j + r));
+            if (lane == 0) bulk_g2s(cr.ring + off + r * pb, pg + a.hdr + static_cast<int64_t>(kv0) * slice, pb, &cr.full[slot]);
+          }
+          j += run - 1;
+          continue;
         }
         // one stage per run of consecutive needed KV heads, at most maxk slices each
         for (int k0 = __ffs(needed) - 1; k0 >= 0 && k0 < nkv;) {
@@ -1238,8 +1331,8 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
           const unsigned later = needed >> (k0 + nk);  // needed KV heads after this stage
           const bool last = j == T - 1 && later == 0 && new_done;
           const int meta = pm | (last ? kLast : 0) | (qb << 16);
-          const uint32_t slot =
-              push(make_int4(meta, off, q, lo), rb, make_int4(k0, nk, posb ? off + nk * slice : -1, slice), taken, need);
+          const uint32_t slot = push(make_int4(meta, off, q, lo), rb,
+                                     make_int4(k0, nk | (1 << 8), posb ? off + nk * slice : -1, slice), taken, need);
           if (lane == 0) {
             bulk_g2s(cr.ring + off, page + a.hdr + static_cast<int64_t>(kv0 + k0) * slice, nk * slice, &cr.full[slot]);
             if (posb) bulk_g2s(cr.ring + off + nk * slice, page, posb, &cr.full[slot]);
@@ -1256,6 +1349,7 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
   }
   if (ok) {
     ensure_waited();
+    pages_ready();  // the last CTA commits from them
     int taken = 0;
     if (reserve(0, taken, true) < 0) ok = false;
     else push(make_int4(kEnd, 0, 0, 0), make_int4(0, 0, 0, 0), make_int4(0, 0, -1, 0), taken, 0);
@@ -1507,26 +1601,30 @@ __device__ __forceinline__ void run_consumer_cc(const AttnKernelArgs& ka, const 
       }
     } else if (active) {
       const int4 rc = lds128i(rec + 32);
-      if (u_kvi >= rc.x && u_kvi < rc.x + rc.y && !(HM && u_local && (meta & kEarly))) {
-        const int cls = meta & 3, fill = (meta >> 2) & 127;
+      const int nks = rc.y & 255, npg = rc.y >> 8;  // KV slices per page, pages of the stage
+      if (u_kvi >= rc.x && u_kvi < rc.x + nks && !(HM && u_local && (meta & kEarly))) {
+        const int cls = meta & 3, fill = (meta >> 2) & 127;  // the last page's fill; the others are full
         if (cls != cur_cls) {
           rescale_dyn(qp, st.acc, cur_cls, cls);
           cur_cls = cls;
         }
-        const uint32_t s0 = smem_u32(cr.ring + ra.y + (u_kvi - rc.x) * rc.w);
         const bool masked = meta & kMask;
-        const uint32_t sp = masked ? smem_u32(cr.ring + rc.z) : s0;
-        uint64_t pm = ~0ull;  // per-head modes: this KV head's presence mask, which ends
-                              // its slice
-        if (HM) {
-          const uint2 m2 = lds64(s0 + rc.w - a.maskb);
-          pm = (static_cast<uint64_t>(m2.y) << 32) | m2.x;
-        }
-        switch (cls) {
-          case 0: consume_page<D, 2, P / KPI, E, HM>(s0, sp, masked, pm, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
-          case 1: consume_page<D, 4, P / KPI, E, HM>(s0, sp, masked, pm, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
-          case 2: consume_page<D, 8, P / KPI, E, HM>(s0, sp, masked, pm, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
-          default: consume_page<D, 16, P / KPI, E, HM>(s0, sp, masked, pm, a.G, fill, u_lo, u_hi, qp, sumq, st, lane); break;
+        for (int pg = 0; pg < npg; ++pg) {
+          const uint32_t s0 = smem_u32(cr.ring + ra.y + (pg * nks + u_kvi - rc.x) * rc.w);
+          const int f = pg == npg - 1 ? fill : P;
+          const uint32_t sp = masked ? smem_u32(cr.ring + rc.z) : s0;
+          uint64_t pm = ~0ull;  // per-head modes: this KV head's presence mask, which ends
+                                // its slice
+          if (HM) {
+            const uint2 m2 = lds64(s0 + rc.w - a.maskb);
+            pm = (static_cast<uint64_t>(m2.y) << 32) | m2.x;
+          }
+          switch (cls) {
+            case 0: consume_page<D, 2, P / KPI, E, HM>(s0, sp, masked, pm, a.G, f, u_lo, u_hi, qp, sumq, st, lane); break;
+            case 1: consume_page<D, 4, P / KPI, E, HM>(s0, sp, masked, pm, a.G, f, u_lo, u_hi, qp, sumq, st, lane); break;
+            case 2: consume_page<D, 8, P / KPI, E, HM>(s0, sp, masked, pm, a.G, f, u_lo, u_hi, qp, sumq, st, lane); break;
+            default: consume_page<D, 16, P / KPI, E, HM>(s0, sp, masked, pm, a.G, f, u_lo, u_hi, qp, sumq, st, lane); break;
+          }
         }
       }
     }
@@ -2035,20 +2133,24 @@ __device__ __forceinline__ void run_consumer_mma(const AttnKernelArgs& ka, const
       }
     } else if (active) {
       const int4 rc = lds128i(rec + 32);
-      if (cw >= rc.x && cw < rc.x + rc.y) {
-        const int cls = meta & 3, fill = (meta >> 2) & 127;
+      const int nks = rc.y & 255, npg = rc.y >> 8;  // KV slices per page, pages of the stage
+      if (cw >= rc.x && cw < rc.x + nks) {
+        const int cls = meta & 3, fill = (meta >> 2) & 127;  // the last page's fill; the others are full
         if (cls != cur_cls) {
           mma_switch<D, NG>(ms, cur_cls, cls);
           cur_cls = cls;
         }
-        const uint32_t s0 = smem_u32(cr.ring + ra.y + (cw - rc.x) * rc.w);
         const bool masked = meta & kMask;
-        const uint32_t sp = masked ? smem_u32(cr.ring + rc.z) : s0;
-        switch (cls) {
-          case 0: mma_page<D, NG, 2>(ms, s0, sp, masked, P, fill, u_lo, u_hi, ka.qscale, col_ok, col_gi, lane); break;
-          case 1: mma_page<D, NG, 4>(ms, s0, sp, masked, P, fill, u_lo, u_hi, ka.qscale, col_ok, col_gi, lane); break;
-          case 2: mma_page<D, NG, 8>(ms, s0, sp, masked, P, fill, u_lo, u_hi, ka.qscale, col_ok, col_gi, lane); break;
-          default: mma_page<D, NG, 16>(ms, s0, sp, masked, P, fill, u_lo, u_hi, ka.qscale, col_ok, col_gi, lane); break;
+        for (int pg = 0; pg < npg; ++pg) {
+          const uint32_t s0 = smem_u32(cr.ring + ra.y + (pg * nks + cw - rc.x) * rc.w);
+          const int f = pg == npg - 1 ? fill : P;
+          const uint32_t sp = masked ? smem_u32(cr.ring + rc.z) : s0;
+          switch (cls) {
+            case 0: mma_page<D, NG, 2>(ms, s0, sp, masked, P, f, u_lo, u_hi, ka.qscale, col_ok, col_gi, lane); break;
+            case 1: mma_page<D, NG, 4>(ms, s0, sp, masked, P, f, u_lo, u_hi, ka.qscale, col_ok, col_gi, lane); break;
+            case 2: mma_page<D, NG, 8>(ms, s0, sp, masked, P, f, u_lo, u_hi, ka.qscale, col_ok, col_gi, lane); break;
+            default: mma_page<D, NG, 16>(ms, s0, sp, masked, P, f, u_lo, u_hi, ka.qscale, col_ok, col_gi, lane); break;
+          }
         }
       }
     }
@@ -2073,6 +2175,7 @@ __device__ __forceinline__ CtaRing attn_prologue(const AttnKernelArgs& ka, uint8
   cr.full = reinterpret_cast<uint64_t*>(smem + lay.full);
   cr.empty = reinterpret_cast<uint64_t*>(smem + lay.empty);
   cr.abort_flag = reinterpret_cast<volatile int*>(smem + lay.flag);
+  cr.ent_ready = reinterpret_cast<uint64_t*>(smem + lay.flag + 8);
   cr.R = ka.ring_bytes;
   pre = reinterpret_cast<int*>(smem + lay.pre);
   if (threadIdx.x == 0) {
@@ -2081,6 +2184,7 @@ __device__ __forceinline__ CtaRing attn_prologue(const AttnKernelArgs& ka, uint8
       mbar_init(&cr.full[i], 1);
       mbar_init(&cr.empty[i], kNcw);
     }
+    mbar_init(cr.ent_ready, kNcw);
     *cr.abort_flag = 0;
     fence_barrier_init();
   }
@@ -2093,7 +2197,11 @@ __device__ __forceinline__ CtaRing attn_prologue(const AttnKernelArgs& ka, uint8
   plan_units(ka, P, NQB, pre, reinterpret_cast<long long*>(smem + lay.red));
   ent = reinterpret_cast<int*>(smem + lay.ent);
   if (!ka.early) pdl_wait();
-  if (ka.fused) plan_entries(ka, ent);
+  if (ka.fused && threadIdx.x >= 32) {  // the consumers build the entry table
+    plan_entries(ka, ent);
+    __syncwarp();
+    if ((threadIdx.x & 31) == 0) mbar_arrive(cr.ent_ready);
+  }
   return cr;
 }
 
