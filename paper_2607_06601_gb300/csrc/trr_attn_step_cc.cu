@@ -1,0 +1,39 @@
+// trr_attn_step_cc.cu - the CUDA-core kernels of trr_decode_step (the append of every
+// entry's token and the attention of its query in one kernel): one instance per head
+// size and page size.
+#include "trr_attn.cuh"
+
+namespace trr {
+
+cudaError_t launch_attn_step_cc(const Layout& l, dim3 grid, dim3 block, size_t smem, cudaStream_t s, const AttnKernelArgs& k) {
+  if (l.d == 64) {
+    if (l.P == 16) return launch_pdl(attn_kernel<64, 16, false, true>, grid, block, smem, s, k);
+    if (l.P == 32) return launch_pdl(attn_kernel<64, 32, false, true>, grid, block, smem, s, k);
+    return launch_pdl(attn_kernel<64, 64, false, true>, grid, block, smem, s, k);
+  }
+  if (l.P == 16) return launch_pdl(attn_kernel<128, 16, false, true>, grid, block, smem, s, k);
+  if (l.P == 32) return launch_pdl(attn_kernel<128, 32, false, true>, grid, block, smem, s, k);
+  return launch_pdl(attn_kernel<128, 64, false, true>, grid, block, smem, s, k);
+}
+
+cudaError_t configure_attn_step_cc() {
+  const void* k64[] = {reinterpret_cast<const void*>(attn_kernel<64, 16, false, true>),
+                       reinterpret_cast<const void*>(attn_kernel<64, 32, false, true>),
+                       reinterpret_cast<const void*>(attn_kernel<64, 64, false, true>)};
+  const void* k128[] = {reinterpret_cast<const void*>(attn_kernel<128, 16, false, true>),
+                        reinterpret_cast<const void*>(attn_kernel<128, 32, false, true>),
+                        reinterpret_cast<const void*>(attn_kernel<128, 64, false, true>)};
+  for (const void* f : k64) {
+    const cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               attn_smem_limit(cc_ctas_per_sm(64)));
+    if (e != cudaSuccess) return e;
+  }
+  for (const void* f : k128) {
+    const cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               attn_smem_limit(cc_ctas_per_sm(128)));
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+}  // namespace trr
