@@ -431,6 +431,8 @@ __host__ __device__ constexpr int attn_smem_limit(int ctas) {
 //        stage {the block's head modes, 2 bits per head (per-head modes), the local
 //        window's first position, -1, 0}
 // meta = class | fill << 2 | flags | head block << 16.
+// A decode step's new-token stage has c.z = kNewRows: it arrives with no bytes, and each
+// consumer warp first writes its KV head's slot 0 into it (and into the cache's page).
 enum : int {
   kMask = 1 << 9,     // the page may hold keys outside [lo, hi]: positions follow the slices
   kFirst = 1 << 10,   // first stage of a unit (its query rows)
@@ -440,6 +442,8 @@ enum : int {
   kQRows = 1 << 14,   // the stage holds the unit's query rows
   kEarly = 1 << 15    // per-head modes: the page ends before the local window
 };
+
+constexpr int kNewRows = -2;
 
 struct AttnKernelArgs {
   LayerArgs a;
@@ -896,6 +900,22 @@ __device__ __forceinline__ void step_token_rows(const AttnKernelArgs& ka, uint2 
   }
 }
 
+// A consumer warp at a new-token stage: entry q's K and V rows of KV head j, quantised
+// into the stage at shared address sdst (slot 0 of a page-shaped slice) and, when `own`,
+// into the token's slot in the cache.  Writes of generic proxy to ring bytes that bulk
+// copies later overwrite: fenced for the async proxy.
+template <int D>
+__device__ __forceinline__ void step_new_rows(const AttnKernelArgs& ka, const int* ent, int q, int j, bool own,
+                                              uint32_t sdst, int lane) {
+  int c, pid, slot;
+  step_slot(ka, ent, q, c, pid, slot);
+  uint2 rk[4], rv[4];
+  step_load_rows<D>(ka, q, j, 1, rk, rv, lane);
+  step_token_rows<D>(ka, rk[0], rv[0], j, c, pid, slot, own, sdst, true, lane);
+  fence_proxy_async_smem();
+  __syncwarp();
+}
+
 // The last CTA of a decode-step call: records the call's error, or commits every entry's
 // metadata (page tables, page first / last positions, counts, the slot's position,
 // presence, last positions, the pools' counters).  Nothing of the call's old metadata is
@@ -1210,11 +1230,13 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
         pg_src = reinterpret_cast<uint64_t>(a.pool[c] + static_cast<int64_t>(wid) * a.page_bytes[c]);
         pg_geo = slice | (max(1, (R / 2 - posb) / slice) << 20);
       }
-      // decode step: the query's own token, as one stage per KV head holding it at slot 0
-      // of a page-shaped slice (consumers read it as a page with one key), placed after
-      // the pages of its own width class so that the consumers' class domain only ever
-      // rises; its bytes also go to the token's slot in the cache.  After a call error
-      // (known only after the wait) one empty stage stands in for it.
+      // decode step: the query's own token, as a stage holding it at slot 0 of a
+      // page-shaped slice per KV head (consumers read it as a page with one key), placed
+      // after the pages of its own width class so that the consumers' class domain only
+      // ever rises.  The stage comes with no bytes: each consumer warp quantises its KV
+      // head's rows into it and into the token's slot in the cache, so that the producer
+      // goes on issuing copies.  After a call error (known only after the wait) one empty
+      // stage stands in for it.
       const int new_cls = has_new ? ent[2 * q + 1] & 3 : 4;
       bool new_done = !has_new;
       auto push_new = [&](bool last) -> bool {
@@ -1228,8 +1250,7 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
           push(make_int4((last ? kLast : 0) | (qb << 16), off, q, lo), rb, make_int4(0, 1 << 8, -1, 0), taken, 0);
           return true;
         }
-        int c, pid, slot;
-        step_slot(ka, ent, q, c, pid, slot);
+        const int c = ent[2 * q + 1] & 3;
         const int slice = a.slice[c];
         // every KV head's slot 0 in one stage when the class's regions allow it: head j's
         // K codes, V codes, K (s, z) and V (s, z) each at j rows (j * rowb bytes) past the
@@ -1242,38 +1263,16 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
           int taken = 0;
           const int off = reserve(align16(span), taken, true);
           if (off < 0) return false;
-          uint2 rk[4], rv[4];
-          step_load_rows<D>(ka, q, kv0, nkv, rk, rv, lane);
-#pragma unroll
-          for (int k = 0; k < 4; ++k) {
-            if (k >= nkv) continue;
-            const int j = kv0 + k;
-            step_token_rows<D>(ka, rk[k], rv[k], j, c, pid, slot, j * g >= h0, smem_u32(cr.ring + off + k * rowb), true,
-                               lane);
-          }
-          fence_proxy_async_smem();  // these bytes are later overwritten by bulk copies
-          __syncwarp();
           const int meta = c | (1 << 2) | (last ? kLast : 0) | (qb << 16);
-          push(make_int4(meta, off, q, lo), rb, make_int4(0, nkv | (1 << 8), -1, rowb), taken, 0);
+          push(make_int4(meta, off, q, lo), rb, make_int4(0, nkv | (1 << 8), kNewRows, rowb), taken, 0);
           return true;
         }
-        for (int j0 = 0; j0 < nkv; j0 += 4) {
-          const int m = min(4, nkv - j0);
-          uint2 rk[4], rv[4];
-          step_load_rows<D>(ka, q, kv0 + j0, m, rk, rv, lane);
-#pragma unroll
-          for (int k = 0; k < 4; ++k) {
-            if (k >= m) continue;
-            int taken = 0;
-            const int off = reserve(slice, taken, true);
-            if (off < 0) return false;
-            const int k0 = j0 + k, j = kv0 + k0;
-            step_token_rows<D>(ka, rk[k], rv[k], j, c, pid, slot, j * g >= h0, smem_u32(cr.ring + off), true, lane);
-            fence_proxy_async_smem();  // these bytes are later overwritten by bulk copies
-            __syncwarp();
-            const int meta = c | (1 << 2) | (last && k0 == nkv - 1 ? kLast : 0) | (qb << 16);
-            push(make_int4(meta, off, q, lo), rb, make_int4(k0, 1 | (1 << 8), -1, slice), taken, 0);
-          }
+        for (int k0 = 0; k0 < nkv; ++k0) {  // otherwise one stage per KV head
+          int taken = 0;
+          const int off = reserve(slice, taken, true);
+          if (off < 0) return false;
+          const int meta = c | (1 << 2) | (last && k0 == nkv - 1 ? kLast : 0) | (qb << 16);
+          push(make_int4(meta, off, q, lo), rb, make_int4(k0, 1 | (1 << 8), kNewRows, slice), taken, 0);
         }
         return true;
       };
@@ -1515,8 +1514,9 @@ __device__ __forceinline__ void finish_unit(const AttnKernelArgs& ka, LaneState<
   store_or_merge<D>(ka, st.acc, part * E + DPL * kl, M, L, sp, qi, qh, nsplit, base, lane);
 }
 
-template <int D, int P, int E, bool HM>
-__device__ __forceinline__ void run_consumer_cc(const AttnKernelArgs& ka, const CtaRing& cr, int cw, int lane) {
+template <int D, int P, int E, bool HM, bool STEP>
+__device__ __forceinline__ void run_consumer_cc(const AttnKernelArgs& ka, const CtaRing& cr, const int* ent, int cw,
+                                                int lane) {
   constexpr int LPK = D / E;     // lanes per key
   constexpr int KPI = 32 / LPK;  // keys per warp iteration
   const LayerArgs& a = ka.a;
@@ -1605,6 +1605,12 @@ __device__ __forceinline__ void run_consumer_cc(const AttnKernelArgs& ka, const 
       const int nks = rc.y & 255, npg = rc.y >> 8;  // KV slices per page, pages of the stage
       if (u_kvi >= rc.x && u_kvi < rc.x + nks && !(HM && u_local && (meta & kEarly))) {
         const int cls = meta & 3, fill = (meta >> 2) & 127;  // the last page's fill; the others are full
+        if (STEP && rc.z == kNewRows) {  // the query's own token: this warp's KV head (warps that
+                                         // share a KV head write the same bytes); the keys past
+                                         // the fill that consume_page reads are never used
+          const int j = u_h / g;
+          step_new_rows<D>(ka, ent, u_q, j, j * g >= u_h - cw, smem_u32(cr.ring + ra.y + (u_kvi - rc.x) * rc.w), lane);
+        }
         if (cls != cur_cls) {
           rescale_dyn(qp, st.acc, cur_cls, cls);
           cur_cls = cls;
@@ -2043,9 +2049,9 @@ __device__ __forceinline__ void mma_finish(const AttnKernelArgs& ka, MmaState<D,
   __syncwarp();
 }
 
-template <int D, int NG>
-__device__ __forceinline__ void run_consumer_mma(const AttnKernelArgs& ka, const CtaRing& cr, int P, int cw, int lane,
-                                                 float* scr) {
+template <int D, int NG, bool STEP>
+__device__ __forceinline__ void run_consumer_mma(const AttnKernelArgs& ka, const CtaRing& cr, const int* ent, int P, int cw,
+                                                 int lane, float* scr) {
   constexpr int NP = D / 8, MT = D / 16, G = D / NG;
   const LayerArgs& a = ka.a;
   const int g = a.Hq / a.Hkv;
@@ -2137,6 +2143,8 @@ __device__ __forceinline__ void run_consumer_mma(const AttnKernelArgs& ka, const
       const int nks = rc.y & 255, npg = rc.y >> 8;  // KV slices per page, pages of the stage
       if (cw >= rc.x && cw < rc.x + nks) {
         const int cls = meta & 3, fill = (meta >> 2) & 127;  // the last page's fill; the others are full
+        if (STEP && rc.z == kNewRows)  // the query's own token, this warp's KV head
+          step_new_rows<D>(ka, ent, u_q, u_kv, true, smem_u32(cr.ring + ra.y + (cw - rc.x) * rc.w), lane);
         if (cls != cur_cls) {
           mma_switch<D, NG>(ms, cur_cls, cls);
           cur_cls = cls;
@@ -2256,7 +2264,7 @@ __global__ void __launch_bounds__(32 * (kNcw + 1), cc_ctas_per_sm(D))
   int *pre, *ent;
   const CtaRing cr = attn_prologue<STEP>(ka, smem, P, NQB, pre, ent);
   if (warp == 0) run_producer<D, STEP>(ka, P, NQB, pre, ent, cr, lane);
-  else run_consumer_cc<D, P, cc_elems(D), HM>(ka, cr, warp - 1, lane);
+  else run_consumer_cc<D, P, cc_elems(D), HM, STEP>(ka, cr, ent, warp - 1, lane);
   attn_epilogue<STEP>(ka, ent);
 }
 
@@ -2274,7 +2282,7 @@ __global__ void __launch_bounds__(32 * (kNcw + 1), kMmaCtasPerSm) attn_mma_kerne
   } else {
     const AttnSmem lay(ka.ring_bytes, ka.n, ka.scr_floats, STEP);
     float* scr = reinterpret_cast<float*>(smem + lay.scr) + (warp - 1) * ka.scr_floats;
-    run_consumer_mma<D, NG>(ka, cr, P, warp - 1, lane, scr);
+    run_consumer_mma<D, NG, STEP>(ka, cr, ent, P, warp - 1, lane, scr);
   }
   attn_epilogue<STEP>(ka, ent);
 }
