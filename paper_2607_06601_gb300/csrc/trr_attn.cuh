@@ -1151,13 +1151,15 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
     }
     // decode step: this query's own token joins the last split of each head block
     const bool has_new = STEP && !err && bmode != TRR_MODE_SKIP && sp == ns - 1;
-    // the unit's pages, planned before the check that waits for the entry table
+    // the unit's pages.  A decode step does not wait for its entry table here: a call
+    // error makes the last CTA zero every row, so units run as if there were none and
+    // only the new-token stage needs the table
     const int lo = bmode == TRR_MODE_FULL ? 0 : max(0, t - w + 1);
     int wid = -1, wmeta = 0, wfirst = 0, wlast = INT_MAX, T = 0;
     if (!err && bmode != TRR_MODE_SKIP)
       T = plan_split(a, P, seq, lo, t, sp, ns, lane, wid, wmeta, a.head_modes ? &wfirst : nullptr,
                      a.head_modes ? &wlast : nullptr);
-    if (err || bmode == TRR_MODE_SKIP || call_failed()) {
+    if (err || bmode == TRR_MODE_SKIP) {
       // zero rows (once per block); the error of the lowest query; a skip token that
       // stores KV has its rows written here
       ensure_waited();
