@@ -686,6 +686,8 @@ def per_workload(args, local):
         avg_bytes, avg_ms = float(np.mean(core["call_bytes"])), float(np.mean(core["call_ms"]))
         in_stream = core["launches_per_step"] == b.L  # as for the headline
         launch_ms = (core["ms"] / a.steps) / b.L if in_stream else avg_ms
+        if in_stream:
+            avg_bytes = core["rank_bytes"] / a.steps / b.L
         achieved = avg_bytes / (launch_ms * 1e-3) / 1e9
         key = name if name != "sweep" else f"sweep_b{b.B}"
         out[key] = {
@@ -909,6 +911,8 @@ def run_gpu(args):
     # the previous one's end as in serving.  Otherwise the bracketed calls.
     in_stream = launches_per_step == bench.L
     launch_ms = (ms / K) / bench.L if in_stream else avg_ms
+    if in_stream:  # the timed steps' own bytes (modes differ from step to step)
+        avg_bytes = rank_bytes / K / bench.L
     achieved = avg_bytes / (launch_ms * 1e-3) / 1e9
     value = job_bytes / (ms * 1e-3) / 1e9
     result = None

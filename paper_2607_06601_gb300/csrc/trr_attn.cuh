@@ -148,53 +148,6 @@ __device__ __forceinline__ void fmul2_inplace(float& x0, float& x1, float f0, fl
   x1 = r.y;
 }
 
-// The factors that move a lane's query and V accumulators between the domains of two
-// width classes, element by element (E = 32 elements per lane): row from * 4 + to.  One
-// table read by every class change keeps a single copy of the code in the consumer's
-// loop (a switch over templated copies made the loop several kilobytes larger).
-struct RescaleTable {
-  float q[16][32];    // query: 2^(qe(to, i) - qe(from, i))
-  float acc[16][32];  // V accumulators: 2^(ex(to, i) - ex(from, i)), ex = 0 at width 16
-};
-__host__ __device__ constexpr float pow2c(int e) {
-  float r = 1.f;
-  for (; e > 0; --e) r *= 2.f;
-  for (; e < 0; ++e) r *= 0.5f;
-  return r;
-}
-__host__ __device__ constexpr RescaleTable make_rescale_table() {
-  RescaleTable t{};
-  for (int from = 0; from < 4; ++from)
-    for (int to = 0; to < 4; ++to)
-      for (int i = 0; i < 32; ++i) {
-        const int bf = bits_of_class(from), bt = bits_of_class(to);
-        t.q[from * 4 + to][i] = pow2c(qe_of(bt, i) - qe_of(bf, i));
-        t.acc[from * 4 + to][i] = pow2c((bt == 16 ? 0 : ex_of(bt, i)) - (bf == 16 ? 0 : ex_of(bf, i)));
-      }
-  return t;
-}
-static __constant__ RescaleTable kRescale = make_rescale_table();
-
-// qp and acc from the domain of class `from` to that of class `to`.
-template <int E>
-__device__ __forceinline__ void rescale_dyn(float (&qp)[E], float (&acc)[E], int from, int to) {
-  static_assert(E == 32, "one factor per element of a lane's 32");
-  const float* qf = kRescale.q[from * 4 + to];
-  const float* af = kRescale.acc[from * 4 + to];
-#pragma unroll
-  for (int i = 0; i < E; i += 2) {
-    fmul2_inplace(qp[i], qp[i + 1], qf[i], qf[i + 1]);
-    fmul2_inplace(acc[i], acc[i + 1], af[i], af[i + 1]);
-  }
-}
-// acc from class `from`'s domain back to class 16's (the common one of the merge)
-template <int E>
-__device__ __forceinline__ void acc_to_neutral(float (&acc)[E], int from) {
-  const float* af = kRescale.acc[from * 4 + 3];
-#pragma unroll
-  for (int i = 0; i < E; i += 2) fmul2_inplace(acc[i], acc[i + 1], af[i], af[i + 1]);
-}
-
 // 2^x with the hardware approximation (relative error about 2^-22; results below the
 // binary32 normal range flush to zero, far below a softmax sum's resolution).
 __device__ __forceinline__ float fast_exp2(float x) {
@@ -234,6 +187,55 @@ __device__ __forceinline__ uint32_t lds32(uint32_t a) {
   asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(a));
   return v;
 }
+
+// The factors that move a lane's query and V accumulators between the domains of two
+// width classes, element by element (E = 32 elements per lane): row from * 4 + to.  One
+// table read by every class change keeps a single copy of the code in the consumer's
+// loop (a switch over templated copies made the loop several kilobytes larger).  Each
+// CTA of the CUDA-core kernels writes the table into its shared memory before the wait
+// on the previous kernel, and a class change reads its row with warp-wide broadcast
+// loads (from constant memory, whose cache misses, a switch took about 470 cycles).
+struct RescaleTable {
+  float q[16][32];    // query: 2^(qe(to, i) - qe(from, i))
+  float acc[16][32];  // V accumulators: 2^(ex(to, i) - ex(from, i)), ex = 0 at width 16
+};
+constexpr int kRescaleFloats = static_cast<int>(sizeof(RescaleTable) / 4);
+
+// Entry k of the table (k < kRescaleFloats), as the struct lays it out.
+__device__ __forceinline__ float rescale_entry(int k) {
+  const bool is_acc = k >= 16 * 32;
+  const int row = (k >> 5) & 15, i = k & 31, bf = bits_of_class(row >> 2), bt = bits_of_class(row & 3);
+  const int e = is_acc ? (bt == 16 ? 0 : ex_of(bt, i)) - (bf == 16 ? 0 : ex_of(bf, i)) : qe_of(bt, i) - qe_of(bf, i);
+  return pow2f(e);
+}
+
+// qp and acc from the domain of class `from` to that of class `to`; tbl: the table's
+// shared-memory address.
+template <int E>
+__device__ __forceinline__ void rescale_dyn(float (&qp)[E], float (&acc)[E], int from, int to, uint32_t tbl) {
+  static_assert(E == 32, "one factor per element of a lane's 32");
+  const uint32_t qf = tbl + (from * 4 + to) * 128, af = qf + 16 * 32 * 4;
+#pragma unroll
+  for (int i = 0; i < E; i += 4) {
+    const uint4 fq = lds128(qf + 4 * i), fa = lds128(af + 4 * i);
+    fmul2_inplace(qp[i], qp[i + 1], __uint_as_float(fq.x), __uint_as_float(fq.y));
+    fmul2_inplace(qp[i + 2], qp[i + 3], __uint_as_float(fq.z), __uint_as_float(fq.w));
+    fmul2_inplace(acc[i], acc[i + 1], __uint_as_float(fa.x), __uint_as_float(fa.y));
+    fmul2_inplace(acc[i + 2], acc[i + 3], __uint_as_float(fa.z), __uint_as_float(fa.w));
+  }
+}
+// acc from class `from`'s domain back to class 16's (the common one of the merge)
+template <int E>
+__device__ __forceinline__ void acc_to_neutral(float (&acc)[E], int from, uint32_t tbl) {
+  const uint32_t af = tbl + 16 * 32 * 4 + (from * 4 + 3) * 128;
+#pragma unroll
+  for (int i = 0; i < E; i += 4) {
+    const uint4 fa = lds128(af + 4 * i);
+    fmul2_inplace(acc[i], acc[i + 1], __uint_as_float(fa.x), __uint_as_float(fa.y));
+    fmul2_inplace(acc[i + 2], acc[i + 3], __uint_as_float(fa.z), __uint_as_float(fa.w));
+  }
+}
+
 
 // The NW words of a lane's codes at shared address a (4 NW-byte aligned), in as few
 // loads as possible (one 4-, 8- or 16-byte load per row part keeps the warp's request
@@ -527,7 +529,7 @@ __device__ __forceinline__ int query_range(int t, int mode, int w) {
 // (mbarriers need 8, bulk-copy destinations 16).
 __host__ __device__ constexpr int align16(int x) { return (x + 15) & ~15; }
 struct AttnSmem {
-  int ring, recs, sbytes, full, empty, scr, pre, ent, red, flag, total;
+  int ring, recs, sbytes, full, empty, scr, pre, ent, red, resc, flag, total;
   __host__ __device__ AttnSmem(int ring_bytes, int n, int scr_floats, int fused)
       : ring(0),
         recs(align16(ring_bytes)),
@@ -538,7 +540,9 @@ struct AttnSmem {
         pre(scr + align16(kNcw * scr_floats * 4)),
         ent(pre + align16(4 * (n + 2))),
         red(ent + (fused ? align16(4 * step_ints(n)) : 0)),
-        flag(red + 16 * 8),  // the abort flag; at flag + 8 the entry table's readiness mbarrier
+        resc(red + 16 * 8),  // the class-change factors (CUDA-core consumers, which have no scratch)
+        flag(resc + (scr_floats == 0 ? 4 * kRescaleFloats : 0)),  // the abort flag; at flag + 8
+                                                                    // the entry table's readiness mbarrier
         total(flag + 16) {}
 };
 
@@ -958,6 +962,7 @@ struct CtaRing {
   uint64_t* empty;
   volatile int* abort_flag;
   uint64_t* ent_ready;  // decode step: completes when the consumers have built the entry table
+  uint32_t resc;        // shared address of the class-change factors (CUDA-core kernels)
   int R;
 };
 
@@ -1477,13 +1482,13 @@ __device__ __forceinline__ void store_or_merge(const AttnKernelArgs& ka, const f
 // The end of a unit for a CUDA-core consumer: merge the lanes' states, then store.
 template <int D, int E>
 __device__ __forceinline__ void finish_unit(const AttnKernelArgs& ka, LaneState<E>& st, int cur_cls, int sp, int qi,
-                                            int qh, int nsplit, int base, int lane) {
+                                            int qh, int nsplit, int base, uint32_t tbl, int lane) {
   constexpr int LPK = D / E;   // lanes per key
   constexpr int DPL = D / 32;  // dimensions per lane after the merge
   const int part = lane % LPK, kl = lane / LPK;
   // rescale to the common maximum, then reduce-scatter over the key lanes: each
   // halving step keeps half of the 32 dims and sends the other half to the partner
-  acc_to_neutral(st.acc, cur_cls);
+  acc_to_neutral(st.acc, cur_cls, tbl);
   float M = st.m;
 #pragma unroll
   for (int o = LPK; o < 32; o <<= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
@@ -1614,7 +1619,7 @@ __device__ __forceinline__ void run_consumer_cc(const AttnKernelArgs& ka, const 
           step_new_rows<D>(ka, ent, u_q, j, j * g >= u_h - cw, smem_u32(cr.ring + ra.y + (u_kvi - rc.x) * rc.w), lane);
         }
         if (cls != cur_cls) {
-          rescale_dyn(qp, st.acc, cur_cls, cls);
+          rescale_dyn(qp, st.acc, cur_cls, cls, cr.resc);
           cur_cls = cls;
         }
         const bool masked = meta & kMask;
@@ -1640,7 +1645,7 @@ __device__ __forceinline__ void run_consumer_cc(const AttnKernelArgs& ka, const 
     __syncwarp();
     if (lane == 0) mbar_arrive(&cr.empty[slot]);  // the stage's bytes are read
     if ((meta & kLast) && active)
-      finish_unit<D, E>(ka, st, cur_cls, u_sp, u_q, u_h, u_ns, u_base, lane);
+      finish_unit<D, E>(ka, st, cur_cls, u_sp, u_q, u_h, u_ns, u_base, cr.resc, lane);
   }
 }
 
@@ -2188,8 +2193,14 @@ __device__ __forceinline__ CtaRing attn_prologue(const AttnKernelArgs& ka, uint8
   cr.empty = reinterpret_cast<uint64_t*>(smem + lay.empty);
   cr.abort_flag = reinterpret_cast<volatile int*>(smem + lay.flag);
   cr.ent_ready = reinterpret_cast<uint64_t*>(smem + lay.flag + 8);
+  cr.resc = smem_u32(smem + lay.resc);
   cr.R = ka.ring_bytes;
   pre = reinterpret_cast<int*>(smem + lay.pre);
+  if (ka.scr_floats == 0) {  // the CUDA-core consumers' class-change factors (the unit plan's
+                             // barriers order these writes before any read)
+    float* t = reinterpret_cast<float*>(smem + lay.resc);
+    for (int k = threadIdx.x; k < kRescaleFloats; k += blockDim.x) t[k] = rescale_entry(k);
+  }
   if (threadIdx.x == 0) {
 #pragma unroll 1
     for (int i = 0; i < kStages; ++i) {
