@@ -10,7 +10,8 @@
 //      heads.  The same deterministic computation in every CTA takes the place of a
 //      planning kernel.  Splits are sized for about one unit per CTA on a small call
 //      and up to three on a large one.
-//   2. The producer warp takes units (its CTA's own first, then from a call-wide
+//   2. The producer warp takes units (on a small call from a call-wide counter as its
+//      CTA starts and finishes them; on a large one its CTA's own first, then from the
 //      counter) and plans each once: the sequence's per-class token counts, a 32-way
 //      search of the pages' first / last positions at window edges, the split's share
 //      of every class's pages in range.  It pushes the unit through the ring as stages
@@ -966,8 +967,8 @@ struct CtaRing {
   int R;
 };
 
-// The producer warp: takes units (the CTA's own first, then from a call-wide counter),
-// plans each and pushes its stages; ends with an end record.
+// The producer warp: takes units, plans each and pushes its stages; ends with an end
+// record.
 //
 // With `early`, the first stages are planned and their page copies issued before the
 // wait on the previous kernel (the layer's cache state is settled; the call's index
@@ -1109,10 +1110,21 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
   };
   if (waited) after_wait();
 
-  int u = blockIdx.x;  // the first unit is the CTA's own; later ones come from the counter
+  // A call with no more units than CTAs hands them out on demand from the call-wide
+  // counter: a CTA takes its first unit as it starts and another only once its consumers
+  // are done with the current one.  The CTAs that start last (on SM slots the previous
+  // kernel frees as it ends) then get the last units, or none.  A larger call gives each
+  // CTA its own first unit and lets the producer take the next from the counter while
+  // the consumers work on the current one.
+  const bool on_demand = total <= static_cast<int>(gridDim.x);
+  int u = static_cast<int>(blockIdx.x);
+  if (on_demand) {
+    if (lane == 0) u = atomicAdd(&a.lctl[kNextUnit], 1);
+    u = __shfl_sync(0xffffffffu, u, 0);
+  }
   while (u < total) {
     int u_next = 0;
-    if (lane == 0) u_next = static_cast<int>(gridDim.x) + atomicAdd(&a.lctl[kNextUnit], 1);  // used last
+    if (!on_demand && lane == 0) u_next = static_cast<int>(gridDim.x) + atomicAdd(&a.lctl[kNextUnit], 1);  // used last
     const int un = u / NQB, qb = u - un * NQB;
     int lo_q = 0, hi_q = n;  // the query of split un: pre[q] <= un < pre[q + 1]
     while (hi_q - lo_q > 1) {
@@ -1150,6 +1162,7 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
       ns = min(ns, splits_of(query_range(t, TRR_MODE_LOCAL, w), pre[n + 1], P, a.s_cap));
       if (sp >= ns) {
         __syncwarp();
+        if (on_demand && lane == 0) u_next = atomicAdd(&a.lctl[kNextUnit], 1);
         u = __shfl_sync(0xffffffffu, u_next, 0);
         continue;
       }
@@ -1352,6 +1365,11 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
       ensure_waited();  // the next unit's query rows come from the previous kernel
     }
     __syncwarp();
+    if (on_demand) {  // the consumers first finish this unit
+      while (ok && released < pushed) ok = release_one();
+      if (!ok) break;
+      if (lane == 0) u_next = atomicAdd(&a.lctl[kNextUnit], 1);
+    }
     u = __shfl_sync(0xffffffffu, u_next, 0);
   }
   if (ok) {
@@ -1384,30 +1402,45 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
 template <int D>
 __device__ __forceinline__ void merge_partials(const float* p0, int64_t stride, int count, int lane, float& Mx,
                                                float& Ls, float (&acc_o)[D / 32]) {
-  constexpr int DPL = D / 32;
+  // Chunks of CH partials: each chunk's (max, sum) words and rows are loaded together
+  // (one round trip to L2 for up to CH splits), then folded into the running result;
+  // CH keeps the rows within the registers the consumers have free at this point.
+  constexpr int DPL = D / 32, CH = D == 64 ? 8 : 4;
   Mx = kNegInf;
-  for (int s = lane; s < count; s += 32) Mx = fmaxf(Mx, __ldcg(p0 + s * stride + D));
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) Mx = fmaxf(Mx, __shfl_xor_sync(0xffffffffu, Mx, o));
-  Ls = 0.f;
+  float lsum = 0.f;  // lane s: the weighted sums of the partials it reads the words of
 #pragma unroll
   for (int j = 0; j < DPL; ++j) acc_o[j] = 0.f;
-  for (int s0 = 0; s0 < count; s0 += 32) {
-    float wl = 0.f;  // lane s: weight of row s0 + s
-    if (s0 + lane < count) {
-      const float2 ml = __ldcg(reinterpret_cast<const float2*>(p0 + (s0 + lane) * stride + D));
-      wl = (ml.x == kNegInf) ? 0.f : fast_exp2(ml.x - Mx);
-      Ls = fmaf(wl, ml.y, Ls);
-    }
-    const int cnt = min(32, count - s0);
-#pragma unroll 8
-    for (int s = 0; s < cnt; ++s) {
-      const float wgt = __shfl_sync(0xffffffffu, wl, s);
-      const float* ps = p0 + (s0 + s) * stride + lane * DPL;
+  for (int s0 = 0; s0 < count; s0 += CH) {
+    const int cnt = min(CH, count - s0);
+    float2 ml = make_float2(kNegInf, 0.f);
+    if (lane < cnt) ml = __ldcg(reinterpret_cast<const float2*>(p0 + (s0 + lane) * stride + D));
+    float rows[CH][DPL];
 #pragma unroll
-      for (int j = 0; j < DPL; ++j) acc_o[j] = fmaf(wgt, __ldcg(ps + j), acc_o[j]);
+    for (int s = 0; s < CH; ++s) {
+#pragma unroll
+      for (int j = 0; j < DPL; ++j) rows[s][j] = s < cnt ? __ldcg(p0 + (s0 + s) * stride + lane * DPL + j) : 0.f;
+    }
+    float cm = ml.x;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) cm = fmaxf(cm, __shfl_xor_sync(0xffffffffu, cm, o));
+    const float nm = fmaxf(Mx, cm);
+    if (nm != kNegInf) {
+      const float f = Mx == kNegInf ? 0.f : fast_exp2(Mx - nm);  // the earlier chunks' scale
+#pragma unroll
+      for (int j = 0; j < DPL; ++j) acc_o[j] *= f;
+      lsum *= f;
+      const float wl = ml.x == kNegInf ? 0.f : fast_exp2(ml.x - nm);  // lane s: weight of row s0 + s
+      lsum = fmaf(wl, ml.y, lsum);
+#pragma unroll
+      for (int s = 0; s < CH; ++s) {
+        const float wgt = __shfl_sync(0xffffffffu, wl, s);
+#pragma unroll
+        for (int j = 0; j < DPL; ++j) acc_o[j] = fmaf(wgt, rows[s][j], acc_o[j]);
+      }
+      Mx = nm;
     }
   }
+  Ls = lsum;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) Ls += __shfl_xor_sync(0xffffffffu, Ls, o);
 }
