@@ -620,10 +620,14 @@ __device__ __forceinline__ int plan_split(const LayerArgs& a, int P, int seq, in
   T = min(T, kItemMaxPages + kClasses);  // the split bound keeps T within this
   wid = -1;
   wmeta = 0;
-  const int t1 = tc[0], t2 = t1 + tc[1], t3 = t2 + tc[2];
-  const int c = (lane >= t1) + (lane >= t2) + (lane >= t3);
+  // lanes take the pages class by class from the widest (bf16) down: the largest copies
+  // are issued first, while the ring is empty (before the wait on the previous kernel),
+  // and the small ones stream in behind them as the consumers free the ring
+  const int t1 = tc[3], t2 = t1 + tc[2], t3 = t2 + tc[1];
+  const int r = (lane >= t1) + (lane >= t2) + (lane >= t3);  // rank in that order
+  const int c = 3 - r;
   auto pick = [c](const int (&v)[kClasses]) { return c == 0 ? v[0] : c == 1 ? v[1] : c == 2 ? v[2] : v[3]; };
-  const int kid = pick(beg) + lane - (c == 0 ? 0 : c == 1 ? t1 : c == 2 ? t2 : t3);
+  const int kid = pick(beg) + lane - (r == 0 ? 0 : r == 1 ? t1 : r == 2 ? t2 : t3);
   int from_tail = -1;
 #pragma unroll
   for (int cc = 0; cc < kClasses; ++cc) {
@@ -902,6 +906,20 @@ __device__ __forceinline__ void step_token_rows(const AttnKernelArgs& ka, uint2 
     if (qv.code_idx >= 0) sts32(sdst + P * rowb + 4 * qv.code_idx, qv.code_word);
     if (qk.sz_idx >= 0) sts32(sdst + kszo + 4 * qk.sz_idx, qk.sz_word);
     if (qv.sz_idx >= 0) sts32(sdst + vszo + 4 * qv.sz_idx, qv.sz_word);
+  }
+}
+
+// A consumer warp at the query rows of a unit that holds its query's new token (the
+// query's last split): the token's K and V rows of KV head j into L1, one 128-byte line
+// per lane, so that the new-token stage later finds them there.  The query-rows stage
+// follows the producer's wait on the previous kernel (which wrote the rows).
+template <int D>
+__device__ __forceinline__ void step_prefetch_rows(const AttnKernelArgs& ka, int q, int j, int lane) {
+  constexpr int kLines = D * 2 / 128;  // 128-byte lines of one row
+  if (lane < 2 * kLines) {
+    const uint16_t* src =
+        ((lane & 1) ? ka.v : ka.k) + (static_cast<int64_t>(q) * ka.a.Hkv + j) * D + (lane >> 1) * 64;
+    asm volatile("prefetch.global.L1 [%0];" ::"l"(src));
   }
 }
 
@@ -1251,13 +1269,12 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
         pg_geo = slice | (max(1, (R / 2 - posb) / slice) << 20);
       }
       // decode step: the query's own token, as a stage holding it at slot 0 of a
-      // page-shaped slice per KV head (consumers read it as a page with one key), placed
-      // after the pages of its own width class so that the consumers' class domain only
-      // ever rises.  The stage comes with no bytes: each consumer warp quantises its KV
-      // head's rows into it and into the token's slot in the cache, so that the producer
-      // goes on issuing copies.  After a call error (known only after the wait) one empty
-      // stage stands in for it.
-      const int new_cls = has_new ? ent[2 * q + 1] & 3 : 4;
+      // page-shaped slice per KV head (consumers read it as a page with one key), after
+      // the unit's pages (the wait on the previous kernel that it needs then holds back
+      // no page copy).  The stage comes with no bytes: each consumer warp quantises its
+      // KV head's rows into it and into the token's slot in the cache, so that the
+      // producer goes on issuing copies.  After a call error (known only after the wait)
+      // one empty stage stands in for it.
       bool new_done = !has_new;
       auto push_new = [&](bool last) -> bool {
         ensure_waited();  // the token's K / V rows come from the previous kernel
@@ -1302,10 +1319,6 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
         int pm = __shfl_sync(0xffffffffu, wmeta, j);
         const unsigned needed = __shfl_sync(0xffffffffu, pg_need, j);
         const int slice = geo & 0xfffff, maxk = geo >> 20;
-        if (!new_done && (pm & 3) > new_cls && !push_new(false)) {
-          ok = false;
-          break;
-        }
         const unsigned all = (1u << nkv) - 1u;
         if (!a.head_modes && !(pm & kMask) && needed == all && nkv <= maxk) {
           // a run of full pages of this class, every KV head of the block: one stage
@@ -1603,6 +1616,7 @@ __device__ __forceinline__ void run_consumer_cc(const AttnKernelArgs& ka, const 
       u_ns = rb.z;
       u_base = rb.w;
       u_local = false;
+      if (STEP && active && u_sp == u_ns - 1) step_prefetch_rows<D>(ka, u_q, u_h / g, lane);
       if (HM && active) {  // this head's own mode: {head modes, local lo}
         const int4 rq = lds128i(rec + 32);
         const int hm = (rq.x >> (2 * cw)) & 3;
@@ -2139,6 +2153,7 @@ __device__ __forceinline__ void run_consumer_mma(const AttnKernelArgs& ka, const
       u_sp = rb.y;
       u_ns = rb.z;
       u_base = rb.w;
+      if (STEP && active && u_sp == u_ns - 1) step_prefetch_rows<D>(ka, u_q, u_kv, lane);
       cur_cls = 3;
 #pragma unroll
       for (int j = 0; j < 2; ++j) {
