@@ -476,8 +476,9 @@ struct AttnKernelArgs {
 // Fused decode step: the per-entry table every CTA builds in shared memory (2 ints per
 // entry: the entry's token index in its (sequence, class) list, or -1 when it stores
 // nothing; class | opens << 2 | openers of the class before it << 3), a hash of the
-// entries' sequences (2 slots per entry: sequence + 1, lowest entry index), then the
-// call's scalars.
+// entries' sequences (2 slots per entry: sequence + 1, lowest entry index; once the
+// entries are checked, its first n ints hold the page of each token that goes into its
+// class's last page), then the call's scalars.
 constexpr int kStepMax = 256;  // entries of one decode-step call, at most
 enum StepScalar : int {
   kSNextPage = 0,   // [4] pages handed out per class before the call (read after the wait)
@@ -760,7 +761,11 @@ static __device__ void plan_entries(const AttnKernelArgs& ka, int* ent) {
     }
   }
   consumers_sync();
-  for (int e = tid; e < n; e += nt) {
+  int lp[(kStepMax + 32 * kNcw - 1) / (32 * kNcw)];  // page of each of this thread's tokens
+                                                        // that goes into its class's last page
+#pragma unroll
+  for (int k = 0; k < (kStepMax + 32 * kNcw - 1) / (32 * kNcw); ++k) lp[k] = -1;
+  for (int e = tid, k = 0; e < n; e += nt, ++k) {
     const int seq = ka.seq_ids[e], pos = ka.q_positions[e], m = ka.modes[e], b = ka.bits[e];
     const int c = b == 2 ? 0 : b == 4 ? 1 : b == 8 ? 2 : b == 16 ? 3 : -1;
     const int w = ka.windows ? ka.windows[e] : ka.window_scalar;
@@ -780,12 +785,22 @@ static __device__ void plan_entries(const AttnKernelArgs& ka, int* ent) {
     if (!err && (m != TRR_MODE_SKIP || a.skip_writes_kv)) {
       tok = a.ntok[seq * 4 + c];
       info = c | (tok % a.P == 0 ? 4 : 0);
+      if (tok % a.P != 0) {
+#pragma unroll
+        for (int kk = 0; kk < (kStepMax + 32 * kNcw - 1) / (32 * kNcw); ++kk)
+          if (kk == k) lp[kk] = a.lastpg[seq * 4 + c];
+      }
     }
     ent[2 * e] = tok;
     ent[2 * e + 1] = info;
     if (err) atomicMin(&sc[kSErr], e * 16 + err);
   }
-  consumers_sync();
+  consumers_sync();  // the hash is read no more: its first n ints take the last pages
+  for (int e = tid, k = 0; e < n; e += nt, ++k) {
+#pragma unroll
+    for (int kk = 0; kk < (kStepMax + 32 * kNcw - 1) / (32 * kNcw); ++kk)
+      if (kk == k) hs[e] = lp[kk];
+  }
   if (tid < 32) {  // openers of the same class before each entry, 32 entries at a time
     int run0 = 0, run1 = 0, run2 = 0, run3 = 0;
     for (int e0 = 0; e0 < n; e0 += 32) {
@@ -830,7 +845,7 @@ __device__ __forceinline__ void step_slot(const AttnKernelArgs& ka, const int* e
   const int* sc = ent + 6 * ka.n;
   c = info & 3;
   slot = tok % a.P;
-  pid = (info & 4) ? sc[kSNextPage + c] + (info >> 3) : a.lastpg[ka.seq_ids[e] * 4 + c];
+  pid = (info & 4) ? sc[kSNextPage + c] + (info >> 3) : ent[2 * ka.n + e];  // the class's last page
 }
 
 // Entry e's K and V rows of up to 4 KV heads kv0 .. kv0 + nkv - 1, this lane's D/32
