@@ -878,7 +878,7 @@ template <int D>
 __device__ __forceinline__ void step_token_rows(const AttnKernelArgs& ka, uint2 rk, uint2 rv, int j, int c, int pid,
                                                 int slot, bool own, uint32_t sdst, bool to_ring, int lane) {
   const LayerArgs& a = ka.a;
-  const int P = a.P, b = bits_of_class(c), ng = D / a.G;
+  const int P = a.P, b = bits_of_class(c), ng = D >> (__ffs(a.G) - 1);  // G: a power of two
   uint8_t* page = a.pool[c] + static_cast<int64_t>(pid) * a.page_bytes[c] + a.hdr + static_cast<int64_t>(j) * a.slice[c];
   if (b == 16) {  // K [P][D] | V [P][D] bf16: this lane's D/32 values
     const int rowb = 2 * D;
@@ -906,22 +906,24 @@ __device__ __forceinline__ void step_token_rows(const AttnKernelArgs& ka, uint2 
     return;
   }
   const int rowb = D * b / 8;
-  const RowCodes qk = quantise_row_codes<D>(rk, b, a.G, lane);
-  const RowCodes qv = quantise_row_codes<D>(rv, b, a.G, lane);
-  if (__any_sync(0xffffffffu, qk.bad || qv.bad) && lane == 0 && own) set_status(a.ctrl, TRR_ERR_BAD_VALUE);
-  const int kszo = 2 * P * rowb, vszo = kszo + P * ng * 4;
-  if (own) {
-    if (qk.code_idx >= 0) reinterpret_cast<uint32_t*>(page + slot * rowb)[qk.code_idx] = qk.code_word;
-    if (qv.code_idx >= 0) reinterpret_cast<uint32_t*>(page + (P + slot) * rowb)[qv.code_idx] = qv.code_word;
-    if (qk.sz_idx >= 0) reinterpret_cast<uint32_t*>(page + kszo + slot * ng * 4)[qk.sz_idx] = qk.sz_word;
-    if (qv.sz_idx >= 0) reinterpret_cast<uint32_t*>(page + vszo + slot * ng * 4)[qv.sz_idx] = qv.sz_word;
+  // K, then V, through one copy of the quantiser (this code runs once per unit, so its
+  // size, not its speed, decides: every instruction of it is a cold fetch)
+  bool bad = false;
+#pragma unroll 1
+  for (int kv = 0; kv < 2; ++kv) {
+    const RowCodes r = quantise_row_codes<D>(kv ? rv : rk, b, a.G, lane);
+    bad |= r.bad;
+    const int coff = (kv * P + slot) * rowb, soff = 2 * P * rowb + kv * P * ng * 4;
+    if (own) {
+      if (r.code_idx >= 0) reinterpret_cast<uint32_t*>(page + coff)[r.code_idx] = r.code_word;
+      if (r.sz_idx >= 0) reinterpret_cast<uint32_t*>(page + soff + slot * ng * 4)[r.sz_idx] = r.sz_word;
+    }
+    if (to_ring) {
+      if (r.code_idx >= 0) sts32(sdst + kv * P * rowb + 4 * r.code_idx, r.code_word);
+      if (r.sz_idx >= 0) sts32(sdst + soff + 4 * r.sz_idx, r.sz_word);
+    }
   }
-  if (to_ring) {
-    if (qk.code_idx >= 0) sts32(sdst + 4 * qk.code_idx, qk.code_word);
-    if (qv.code_idx >= 0) sts32(sdst + P * rowb + 4 * qv.code_idx, qv.code_word);
-    if (qk.sz_idx >= 0) sts32(sdst + kszo + 4 * qk.sz_idx, qk.sz_word);
-    if (qv.sz_idx >= 0) sts32(sdst + vszo + 4 * qv.sz_idx, qv.sz_word);
-  }
+  if (__any_sync(0xffffffffu, bad) && lane == 0 && own) set_status(a.ctrl, TRR_ERR_BAD_VALUE);
 }
 
 // A consumer warp at the query rows of a unit that holds its query's new token (the
@@ -1309,7 +1311,7 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
         // region's start, so that a consumer reads its head as a page-shaped slice at
         // j * rowb; the reservation covers what the consumers read of the slots past the
         // fill
-        const int b = bits_of_class(c), rowb = b == 16 ? 2 * D : D * b / 8, ng = D / a.G;
+        const int b = bits_of_class(c), rowb = b == 16 ? 2 * D : D * b / 8, ng = D >> (__ffs(a.G) - 1);
         if (nkv <= 4 && (b == 16 || (nkv - 1) * rowb + ng * 4 <= P * ng * 4)) {
           const int span = b == 16 ? (nkv - 1 + P + 16) * rowb : (nkv - 1) * rowb + 2 * P * rowb + (P + 16) * ng * 4;
           int taken = 0;

@@ -313,7 +313,8 @@ __device__ __forceinline__ RowCodes quantise_row_codes(const uint2 w, int b, int
     x[EPL > 2 ? 2 : 0] = bf16lo(w.y);
     x[EPL > 3 ? 3 : 1] = bf16hi(w.y);
   }
-  const int GL = G / EPL;  // lanes of one group
+  const int lgl = __ffs(G) - 1 - (EPL == 4 ? 2 : 1), GL = 1 << lgl;  // lanes of one group (powers of two:
+                                                                      // shifts and masks, no division)
   float mn = x[0], mx = x[0];
   bool bad = false;
 #pragma unroll
@@ -338,14 +339,14 @@ __device__ __forceinline__ RowCodes quantise_row_codes(const uint2 w, int b, int
       val |= static_cast<uint32_t>(s != 0.f ? code_of(x[i], z, s, rs, levels) : 0) << (i * b);
     szw = static_cast<uint32_t>(__half_as_ushort(s16)) | (static_cast<uint32_t>(__half_as_ushort(z16)) << 16);
   }
-  const int LPW = 32 / (EPL * b);  // lanes sharing one 32-bit word of codes
-  val <<= (lane % LPW) * EPL * b;
+  const int lpw = 5 - (__ffs(EPL * b) - 1), LPW = 1 << lpw;  // lanes sharing one 32-bit word of codes
+  val <<= (lane & (LPW - 1)) * EPL * b;
   for (int o = 1; o < LPW; o <<= 1) val |= __shfl_xor_sync(0xffffffffu, val, o);
   RowCodes r;
   r.code_word = val;
   r.sz_word = szw;
-  r.code_idx = lane % LPW == 0 ? lane / LPW : -1;
-  r.sz_idx = lane % GL == 0 ? lane / GL : -1;
+  r.code_idx = (lane & (LPW - 1)) == 0 ? lane >> lpw : -1;
+  r.sz_idx = (lane & (GL - 1)) == 0 ? lane >> lgl : -1;
   r.bad = bad;
   return r;
 }
