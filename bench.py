@@ -944,7 +944,7 @@ def run_gpu(args):
             "e2e": {"value": round(e2e_bytes / (e2e_ms * 1e-3) / 1e9, 2), "unit": UNIT,
                     "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
                     "how": "per step one CUDA graph of: pinned H2D copy of the step's inputs, the step's "
-                           "trr_kv_append / trr_decode_attn calls, D2H copy of every output row",
+                           "API calls (trr_decode_step per layer), D2H copy of every output row",
                     "eager_value": round(eager_bytes / (eager_ms * 1e-3) / 1e9, 2),
                     "eager_how": "the same steps called one by one from Python, no graph (host-launch bound)"},
             "roofline": {"bound": "hbm", "achieved": round(achieved, 2), "peak": peak,
