@@ -34,9 +34,9 @@
  *     *_routed calls) are read while the previous kernel of the stream may still be
  *     running, so they must not be outputs of that kernel (produce them one kernel
  *     earlier, or copy them in from the host).  Query, K and V rows are read after it
- *     has finished.  A call whose layer was not touched by the two calls enqueued
- *     before it on the cache may also read the layer's cache state early (see
- *     trr_decode_step).
+ *     has finished.  A decode step (trr_decode_step) whose layer was not touched by the
+ *     two calls enqueued before it on the cache also reads the layer's cache state early
+ *     (see there); the other calls read the cache only after the previous kernel.
  *
  * Cache memory layout (fixed; the CPU oracle re-derives it independently)
  *   class index c = 0,1,2,3 <-> b = 2,4,8,16.   P = page_size, d = head_dim,
