@@ -87,3 +87,21 @@ def test_per_token_accounting_is_per_head_with_equal_heads(swk):
         y = a.query_heads(bits, hm, int(t))
         assert x[1] == y[1] and x[2] == y[2]
         assert y[0] - x[0] == (8 * Hkv * y[2] if modes[t] else 0)
+
+
+def test_threaded_oracle_baseline_runs_the_same_queries():
+    """The CPU baseline's oracle sample: with a budget that lets every query of the
+    sample run, one thread and four threads process the same queries (same algorithmic
+    bytes, keys and count), each query's bytes being the accounting's."""
+    spec = wl.SPECS["tiny"]
+    sample = bench.OracleSample(spec, 4, spec.window)
+    assert sample.n_queries == int(wl.contexts(spec).min()) * sample.n_seqs
+    one = sample.run(60.0, threads=1)
+    four = sample.run(60.0, threads=4)
+    assert one[2] == four[2] == sample.n_queries
+    assert one[:3] == four[:3]
+    total = 0
+    for j in range(sample.n_queries):
+        nb, _ = sample.query(j)
+        total += nb
+    assert total == one[0]
