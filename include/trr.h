@@ -62,6 +62,13 @@
  *       K [P][d] bf16 | V [P][d] bf16.
  *   Code packing: element j of a head vector sits at byte floor(j*b/8), bit (j*b) % 8,
  *   least significant bits first (2-bit codes 1,2,3,0 -> byte 0x39).
+ *   Chunk order of 8- and 16-bit rows: in every cache except those of query groups
+ *   g = Hq/Hkv >= 2 with g * (d/G) <= 8 and head_modes = 0, the K and V code regions of
+ *   b = 8 and b = 16 slices store byte x of the slice (x counted from the slice's start,
+ *   x < 2*P*d*b/8) at x' = 128*n + 16*(k XOR (n % 8)) + x % 16, where n = x / 128 and
+ *   k = (x / 16) % 8: each 128-byte line keeps its 16-byte chunks in a permuted order
+ *   (the order the attention's lanes read them without shared-memory bank conflicts).
+ *   Everything else (b = 2 and 4, scales, positions, masks) is stored as above.
  *   Page allocation: entries are taken in array order; an entry of class c whose
  *   (layer, seq) has ntok % P == 0 opens page next_page[c]++ .
  *   Per-head modes (head_modes = 1): the last 16 bytes of KV head h's slice hold a

@@ -48,6 +48,8 @@ static const int BITS_OF_CLASS[4] = {2, 4, 8, 16};
 
 typedef struct orc_cache {
   int L, S, Hq, Hkv, d, G, P, maxctx, skip_writes_kv, no_pool, head_modes;
+  int chunk_order;     /* 1: 8- and 16-bit code rows keep each 128-byte line's 16-byte
+                          chunks in the documented permuted order (see stored_at) */
   int cap[4];
   int MP, W32;
   int32_t* last_pos;   /* [L][S] */
@@ -255,6 +257,13 @@ int orc_create(const int32_t* cfg, orc_cache** out) {
   o->W32 = (o->maxctx + 31) / 32;
   o->hdr = roundup(4 * (int64_t)o->P, 128);
   o->maskb = o->head_modes ? 16 : 0;
+  {
+    /* The documented rule: the permuted chunk order applies to every cache except those
+     * read by the tensor-core path, i.e. query groups of g >= 2 whose g * (d / G)
+     * (head, group) columns fit 8, without per-head modes. */
+    int g = o->Hq / o->Hkv, cols = g * (o->d / o->G);
+    o->chunk_order = (!o->head_modes && g >= 2 && cols <= 8) ? 0 : 1;
+  }
   for (c = 0; c < 4; c++) {
     int b = BITS_OF_CLASS[c];
     o->tokb[c] = b < 16 ? 2 * (o->d * b / 8) + 2 * (o->d / o->G) * 4 : 4 * o->d;
@@ -317,29 +326,46 @@ static int check_entry(const orc_cache* o, int seq, int pos, int bits, const uin
   return ORC_OK;
 }
 
+/* The stored position of byte x of a KV slice (x counted from the slice's start) in an
+ * 8- or 16-bit code region of a cache with the permuted chunk order: line n = x / 128
+ * keeps its 16-byte chunk k = (x / 16) % 8 at chunk k XOR (n % 8) of the same line. */
+static int64_t stored_at(const orc_cache* o, int b, int64_t x) {
+  if (!o->chunk_order || b < 8) return x;
+  int64_t n = x / 128, k = (x / 16) % 8;
+  return n * 128 + (k ^ (n % 8)) * 16 + x % 16;
+}
+
 static void write_row(orc_cache* o, uint8_t* page, int c, int slot, int h,
                       const uint16_t* krow, const uint16_t* vrow, int* bad) {
   int b = BITS_OF_CLASS[c], d = o->d, G = o->G, P = o->P;
   uint8_t* sl = page + o->hdr + (int64_t)h * o->slice[c];
+  int64_t j;
+  uint8_t row[256]; /* one K or V code row in its logical byte order (d * b / 8 <= 256);
+                       rows start on 16 bytes and are moved a 16-byte chunk at a time */
   if (b == 16) {
-    memcpy(sl + (int64_t)slot * d * 2, krow, (size_t)d * 2);
-    memcpy(sl + (int64_t)P * d * 2 + (int64_t)slot * d * 2, vrow, (size_t)d * 2);
+    for (int which = 0; which < 2; which++) {
+      int64_t at = (int64_t)which * P * d * 2 + (int64_t)slot * d * 2;
+      memcpy(row, which ? vrow : krow, (size_t)d * 2);
+      for (j = 0; j < d * 2; j += 16) memcpy(sl + stored_at(o, b, at + j), row + j, 16);
+    }
     return;
   }
   int rowb = d * b / 8, ng = d / G, which, g;
   uint8_t codes[128];
   for (which = 0; which < 2; which++) { /* 0 = K, 1 = V */
     const uint16_t* x = which ? vrow : krow;
-    uint8_t* crow = sl + (int64_t)which * P * rowb + (int64_t)slot * rowb;
+    int64_t at = (int64_t)which * P * rowb + (int64_t)slot * rowb;
     uint8_t* szrow = sl + 2 * (int64_t)P * rowb + (int64_t)which * P * ng * 4 +
                      (int64_t)slot * ng * 4;
+    memset(row, 0, sizeof(row));
     for (g = 0; g < ng; g++) {
       uint16_t s16, z16;
       *bad |= orc_quantize_group(x + g * G, G, b, &s16, &z16, codes);
-      orc_pack_codes(codes, G, b, crow + g * G * b / 8);
+      orc_pack_codes(codes, G, b, row + g * G * b / 8);
       memcpy(szrow + g * 4, &s16, 2); /* little-endian host, as on the GPU */
       memcpy(szrow + g * 4 + 2, &z16, 2);
     }
+    for (j = 0; j < rowb; j += 16) memcpy(sl + stored_at(o, b, at + j), row + j, 16);
   }
 }
 
@@ -415,10 +441,12 @@ static void dequant_slot(const orc_cache* o, const uint8_t* page, int c, int slo
                          double* kout, double* vout) {
   int b = BITS_OF_CLASS[c], d = o->d, G = o->G, P = o->P, j, which;
   const uint8_t* sl = page + o->hdr + (int64_t)h * o->slice[c];
+  uint8_t r[256]; /* the row in its logical byte order */
   for (which = 0; which < 2; which++) {
     double* outv = which ? vout : kout;
     if (b == 16) {
-      const uint8_t* r = sl + (int64_t)which * P * d * 2 + (int64_t)slot * d * 2;
+      int64_t at = (int64_t)which * P * d * 2 + (int64_t)slot * d * 2, x;
+      for (x = 0; x < d * 2; x += 16) memcpy(r + x, sl + stored_at(o, b, at + x), 16);
       for (j = 0; j < d; j++) {
         uint16_t h16;
         memcpy(&h16, r + 2 * j, 2);
@@ -427,7 +455,9 @@ static void dequant_slot(const orc_cache* o, const uint8_t* page, int c, int slo
       continue;
     }
     int rowb = d * b / 8, ng = d / G;
-    const uint8_t* crow = sl + (int64_t)which * P * rowb + (int64_t)slot * rowb;
+    int64_t at = (int64_t)which * P * rowb + (int64_t)slot * rowb, x;
+    for (x = 0; x < rowb; x += 16) memcpy(r + x, sl + stored_at(o, b, at + x), 16);
+    const uint8_t* crow = r;
     const uint8_t* szrow = sl + 2 * (int64_t)P * rowb + (int64_t)which * P * ng * 4 +
                            (int64_t)slot * ng * 4;
     for (j = 0; j < d; j++) {

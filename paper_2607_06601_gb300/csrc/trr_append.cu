@@ -176,7 +176,8 @@ __global__ void __launch_bounds__(1024) append_plan_kernel(LayerArgs a, int n, c
 
 // Eq. 4 on 32 consecutive values (one chunk of a group): codes packed LSB-first.
 template <int B>
-__device__ __forceinline__ void quantise_chunk(const uint4* src, float z, float s, float rs, uint32_t* dst) {
+__device__ __forceinline__ void quantise_chunk(const uint4* src, float z, float s, float rs, uint8_t* sl, int64_t off,
+                                               bool sw) {
   constexpr int levels = (1 << B) - 1;
   constexpr int per_word = 32 / B;
   uint32_t words[B];
@@ -195,7 +196,10 @@ __device__ __forceinline__ void quantise_chunk(const uint4* src, float z, float 
     }
   }
 #pragma unroll
-  for (int w = 0; w < B; ++w) dst[w] = words[w];
+  for (int w = 0; w < B; ++w) {  // word w at byte off + 4 w of the slice (swizzled: sw)
+    const int64_t o = off + 4 * w;
+    *reinterpret_cast<uint32_t*>(sl + (sw ? swz_off(o) : o)) = words[w];
+  }
 }
 
 __global__ void __launch_bounds__(256) append_write_kernel(LayerArgs a, int n, const uint16_t* __restrict__ k,
@@ -218,10 +222,12 @@ __global__ void __launch_bounds__(256) append_write_kernel(LayerArgs a, int n, c
   const uint16_t* src = (which ? v : k) + (static_cast<int64_t>(e) * a.Hkv + h) * a.d + g * a.G;
   uint8_t* sl = a.pool[p.cls] + p.page * a.page_bytes[p.cls] + a.hdr + static_cast<int64_t>(h) * a.slice[p.cls];
   const uint4* s4 = reinterpret_cast<const uint4*>(src);
-  if (b == 16) {  // native precision: copy the bf16 bits
-    uint4* dst = reinterpret_cast<uint4*>(sl + static_cast<int64_t>(which) * a.P * a.d * 2 +
-                                          static_cast<int64_t>(p.slot) * a.d * 2 + g * a.G * 2);
-    for (int i = 0; i < a.G / 8; ++i) dst[i] = s4[i];
+  if (b == 16) {  // native precision: copy the bf16 bits, 16 bytes (one chunk) at a time
+    const int64_t off = static_cast<int64_t>(which) * a.P * a.d * 2 + static_cast<int64_t>(p.slot) * a.d * 2 + g * a.G * 2;
+    for (int i = 0; i < a.G / 8; ++i) {
+      const int64_t o = off + 16 * i;
+      *reinterpret_cast<uint4*>(sl + (a.swz ? swz_off(o) : o)) = s4[i];
+    }
     return;
   }
   // min / max of the group; values binary16 cannot carry make the group all zeros
@@ -239,13 +245,16 @@ __global__ void __launch_bounds__(256) append_write_kernel(LayerArgs a, int n, c
     }
   }
   const int rowb = a.d * b / 8;
-  uint32_t* codes = reinterpret_cast<uint32_t*>(sl + static_cast<int64_t>(which) * a.P * rowb +
-                                                static_cast<int64_t>(p.slot) * rowb + g * a.G * b / 8);
+  const bool sw = a.swz && b == 8;  // 8-bit rows of a swizzled cache
+  const int64_t coff = static_cast<int64_t>(which) * a.P * rowb + static_cast<int64_t>(p.slot) * rowb + g * a.G * b / 8;
   uint32_t* sz = reinterpret_cast<uint32_t*>(sl + 2 * static_cast<int64_t>(a.P) * rowb +
                                              static_cast<int64_t>(which) * a.P * ng * 4 +
                                              static_cast<int64_t>(p.slot) * ng * 4 + g * 4);
   if (bad) {
-    for (int i = 0; i < a.G * b / 32; ++i) codes[i] = 0;
+    for (int i = 0; i < a.G * b / 32; ++i) {
+      const int64_t o = coff + 4 * i;
+      *reinterpret_cast<uint32_t*>(sl + (sw ? swz_off(o) : o)) = 0;
+    }
     *sz = 0;
     set_status(a.ctrl, TRR_ERR_BAD_VALUE);
     return;
@@ -255,10 +264,10 @@ __global__ void __launch_bounds__(256) append_write_kernel(LayerArgs a, int n, c
   const __half s16 = __float2half_rn(__fdiv_rn(__fsub_rn(mx, mn), levels));  // s
   const float z = __half2float(z16), s = __half2float(s16), rs = __frcp_rn(s);
   for (int q = 0; q < a.G / 32; ++q) {
-    uint32_t* dst = codes + q * b;  // 32 codes of b bits = b words
-    if (b == 2) quantise_chunk<2>(s4 + 4 * q, z, s, rs, dst);
-    else if (b == 4) quantise_chunk<4>(s4 + 4 * q, z, s, rs, dst);
-    else quantise_chunk<8>(s4 + 4 * q, z, s, rs, dst);
+    const int64_t off = coff + 4 * q * b;  // 32 codes of b bits = b words
+    if (b == 2) quantise_chunk<2>(s4 + 4 * q, z, s, rs, sl, off, false);
+    else if (b == 4) quantise_chunk<4>(s4 + 4 * q, z, s, rs, sl, off, false);
+    else quantise_chunk<8>(s4 + 4 * q, z, s, rs, sl, off, sw);
   }
   *sz = static_cast<uint32_t>(__half_as_ushort(s16)) | (static_cast<uint32_t>(__half_as_ushort(z16)) << 16);
 }
@@ -274,12 +283,16 @@ __global__ void __launch_bounds__(256) append_write_kernel(LayerArgs a, int n, c
 constexpr int kFusedMax = 256;
 
 // One row of d values (entry, KV head, K or V) by a warp, written to its slot.
+// The codes go to byte row_off of the slice sl (swizzled when sw).
 template <int D>
-__device__ __forceinline__ void quantise_row(const uint2 w, uint8_t* codes_row, uint32_t* sz_row, int b, int G,
-                                             int lane, int32_t* ctrl) {
+__device__ __forceinline__ void quantise_row(const uint2 w, uint8_t* sl, int64_t row_off, bool sw, uint32_t* sz_row,
+                                             int b, int G, int lane, int32_t* ctrl) {
   const RowCodes r = quantise_row_codes<D>(w, b, G, lane);
   if (r.bad && r.sz_idx >= 0) set_status(ctrl, TRR_ERR_BAD_VALUE);
-  if (r.code_idx >= 0) reinterpret_cast<uint32_t*>(codes_row)[r.code_idx] = r.code_word;
+  if (r.code_idx >= 0) {
+    const int64_t o = row_off + 4 * r.code_idx;
+    *reinterpret_cast<uint32_t*>(sl + (sw ? swz_off(o) : o)) = r.code_word;
+  }
   if (r.sz_idx >= 0) sz_row[r.sz_idx] = r.sz_word;
 }
 
@@ -414,16 +427,17 @@ __global__ void __launch_bounds__(256) append_fused_kernel(LayerArgs a, int n, c
       const int b = bits_of_class(rc), slot = s_k[re] % a.P;
       uint8_t* sl = a.pool[rc] + static_cast<int64_t>(s_pid[re]) * a.page_bytes[rc] + a.hdr +
                     static_cast<int64_t>(rh) * a.slice[rc];
-      if (b == 16) {
-        uint32_t* dst = reinterpret_cast<uint32_t*>(sl + (static_cast<int64_t>(which) * a.P + slot) * D * 2);
-        if (D == 64) dst[lane] = raw.x;
-        else reinterpret_cast<uint2*>(dst)[lane] = raw;
+      if (b == 16) {  // this lane's D/32 values (4 or 8 bytes: inside one 16-byte chunk)
+        const int64_t o = (static_cast<int64_t>(which) * a.P + slot) * D * 2 + lane * (D / 16);
+        uint8_t* dst = sl + (a.swz ? swz_off(o) : o);
+        if (D == 64) *reinterpret_cast<uint32_t*>(dst) = raw.x;
+        else *reinterpret_cast<uint2*>(dst) = raw;
       } else {
         const int rowb = D * b / 8, ng = D / a.G;
-        uint8_t* codes_row = sl + (static_cast<int64_t>(which) * a.P + slot) * rowb;
         uint32_t* sz_row = reinterpret_cast<uint32_t*>(sl + 2 * static_cast<int64_t>(a.P) * rowb +
                                                       (static_cast<int64_t>(which) * a.P + slot) * ng * 4);
-        quantise_row<D>(raw, codes_row, sz_row, b, a.G, lane, a.ctrl);
+        quantise_row<D>(raw, sl, (static_cast<int64_t>(which) * a.P + slot) * rowb, a.swz && b == 8, sz_row, b, a.G,
+                        lane, a.ctrl);
       }
     }
   }

@@ -22,9 +22,8 @@ cudaError_t attn_configure() {
 
 // The tensor-core path serves query groups (g >= 2) whose (head, group) columns fit
 // one 8-wide mma tile.
-static bool use_mma(const Layout& l) {
-  const int g = l.Hq / l.Hkv, ng = l.d / l.G;
-  return !l.head_modes && g >= 2 && g * ng <= 8;  // per-head modes: one warp per query head
+static bool use_mma(const Layout& l) {  // per-head modes: one warp per query head
+  return uses_mma(l.Hq, l.Hkv, l.d, l.G, l.head_modes);
 }
 
 // Ring bytes an attention call with n queries gets, or -1 when one stage of the

@@ -260,15 +260,22 @@ __device__ __forceinline__ void lds_codes(uint32_t a, uint32_t* w) {
 // One page of width class B (P = NIT * keys per iteration tokens) at shared address s0;
 // lane -> (key kl, 32-dim part).  Keys past `fill` are empty slots; with positions at
 // spos (masked pages), keys outside [lo, hi] are masked too.
+// A lane's q-th 16-byte chunk of a key's 8- or 16-bit row in a swizzled slice: the row
+// part it reads starts at chunk c0 of its 128-byte line, whose chunks are stored in the
+// order chunk ^ xm (xm: the line's index mod 8; see swz_off).
+__device__ __forceinline__ uint32_t swz_chunk(uint32_t a, int c0, int xm, int q) {
+  return a + static_cast<uint32_t>((((c0 + q) ^ xm) - c0) * 16);
+}
+
 // q.k of one key at shared address ka (this lane's E dims) in class B, with its (s, z)
 // word at kszaddr for B < 16: s * sum(q_i c_i) + z * sum(q_i) in the domain of qp.
 template <int B, int E>
-__device__ __forceinline__ float k_dot(uint32_t ka, uint32_t kszaddr, const float (&qp)[E], float sumq) {
+__device__ __forceinline__ float k_dot(uint32_t ka, uint32_t kszaddr, const float (&qp)[E], float sumq, int c0, int xm) {
   float2 d2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
   if (B == 16) {
 #pragma unroll
     for (int q = 0; q < E / 8; ++q) {
-      const uint4 u = lds128(ka + 16 * q);
+      const uint4 u = lds128(swz_chunk(ka, c0, xm, q));
       d2[0] = ffma2(make_float2(qp[8 * q + 0], qp[8 * q + 1]), make_float2(bf_lo(u.x), bf_hi(u.x)), d2[0]);
       d2[1] = ffma2(make_float2(qp[8 * q + 2], qp[8 * q + 3]), make_float2(bf_lo(u.y), bf_hi(u.y)), d2[1]);
       d2[0] = ffma2(make_float2(qp[8 * q + 4], qp[8 * q + 5]), make_float2(bf_lo(u.z), bf_hi(u.z)), d2[0]);
@@ -278,7 +285,15 @@ __device__ __forceinline__ float k_dot(uint32_t ka, uint32_t kszaddr, const floa
   }
   constexpr int NW = E * B / 32;
   uint32_t w[NW], h[NW];
-  lds_codes<NW>(ka, w);
+  if (B == 8) {  // two chunks of the swizzled row
+#pragma unroll
+    for (int q = 0; q < NW / 4; ++q) {
+      const uint4 u = lds128(swz_chunk(ka, c0, xm, q));
+      w[4 * q] = u.x; w[4 * q + 1] = u.y; w[4 * q + 2] = u.z; w[4 * q + 3] = u.w;
+    }
+  } else {
+    lds_codes<NW>(ka, w);
+  }
   if (B != 8) high_parts<B, NW>(w, h);
   const uint32_t szw = lds32(kszaddr);
 #pragma unroll
@@ -292,13 +307,13 @@ __device__ __forceinline__ float k_dot(uint32_t ka, uint32_t kszaddr, const floa
 // acc += p * v for one key's V at shared address va (this lane's E dims) in class B,
 // with its (s, z) word at vszaddr for B < 16.
 template <int B, int E>
-__device__ __forceinline__ void v_acc(uint32_t va, uint32_t vszaddr, float p, LaneState<E>& st) {
+__device__ __forceinline__ void v_acc(uint32_t va, uint32_t vszaddr, float p, LaneState<E>& st, int c0, int xm) {
   if (B == 16) {
     const float wv = p * pow2f(-49);
     const float2 w2 = make_float2(wv, wv);
 #pragma unroll
     for (int q = 0; q < E / 8; ++q) {
-      const uint4 u = lds128(va + 16 * q);
+      const uint4 u = lds128(swz_chunk(va, c0, xm, q));
       const uint32_t uw[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
       for (int h = 0; h < 4; ++h) {
@@ -312,7 +327,15 @@ __device__ __forceinline__ void v_acc(uint32_t va, uint32_t vszaddr, float p, La
   }
   constexpr int NW = E * B / 32;
   uint32_t w[NW], h[NW];
-  lds_codes<NW>(va, w);
+  if (B == 8) {  // two chunks of the swizzled row
+#pragma unroll
+    for (int q = 0; q < NW / 4; ++q) {
+      const uint4 u = lds128(swz_chunk(va, c0, xm, q));
+      w[4 * q] = u.x; w[4 * q + 1] = u.y; w[4 * q + 2] = u.z; w[4 * q + 3] = u.w;
+    }
+  } else {
+    lds_codes<NW>(va, w);
+  }
   if (B != 8) high_parts<B, NW>(w, h);
   const uint32_t szw = lds32(vszaddr);
   const float2 sz = __half22float2(*reinterpret_cast<const __half2*>(&szw));  // (s, z)
@@ -349,6 +372,11 @@ __device__ __forceinline__ void consume_page(uint32_t s0, uint32_t spos, bool ma
   const int ng = D >> lg;
   const int grp = (part * E) >> lg;
   const uint32_t krow = s0 + kl * rowb + part * (E * B / 8);   // this lane's K bytes, key kl
+  // 8- and 16-bit rows are swizzled (every cache of this consumer): the lane's first chunk
+  // in its line and the line's index mod 8 (the same for every key it reads, as a key
+  // group spans a multiple of 8 lines, and for the V rows, which start on such a line)
+  const int o0 = kl * rowb + part * (E * B / 8);
+  const int c0 = (o0 >> 4) & 7, xm = B >= 8 ? (o0 >> 7) & 7 : 0;
   const uint32_t ksz = s0 + 2 * P * rowb + (kl * ng + grp) * 4;  // its (s, z), key kl
   const uint32_t szstep = KPI * ng * 4;
 #pragma unroll 1
@@ -364,7 +392,7 @@ __device__ __forceinline__ void consume_page(uint32_t s0, uint32_t spos, bool ma
         const int pos = static_cast<int>(lds32(spos + 4 * key));
         valid[k] = valid[k] && pos >= lo && pos <= hi;
       }
-      dot[k] = k_dot<B, E>(krow + (it + k) * KPI * rowb, ksz + (it + k) * szstep, qp, sumq);
+      dot[k] = k_dot<B, E>(krow + (it + k) * KPI * rowb, ksz + (it + k) * szstep, qp, sumq, c0, xm);
     }
 #pragma unroll
     for (int k = 0; k < KP; ++k) {
@@ -390,7 +418,7 @@ __device__ __forceinline__ void consume_page(uint32_t s0, uint32_t spos, bool ma
         const float p = fast_exp2(dot[k] - st.m);
         st.l += p;
         const uint32_t va = krow + (it + k) * KPI * rowb + P * rowb;
-        v_acc<B, E>(va, ksz + (it + k) * szstep + P * ng * 4, p, st);
+        v_acc<B, E>(va, ksz + (it + k) * szstep + P * ng * 4, p, st, c0, xm);
       }
     }
   }
@@ -880,27 +908,33 @@ __device__ __forceinline__ void step_token_rows(const AttnKernelArgs& ka, uint2 
   const LayerArgs& a = ka.a;
   const int P = a.P, b = bits_of_class(c), ng = D >> (__ffs(a.G) - 1);  // G: a power of two
   uint8_t* page = a.pool[c] + static_cast<int64_t>(pid) * a.page_bytes[c] + a.hdr + static_cast<int64_t>(j) * a.slice[c];
+  // 8- and 16-bit code rows are swizzled in a cache of the CUDA-core consumer (swz_off,
+  // relative to the slice: the page's slice, and the page-shaped slice at sdst that the
+  // consumers read from the ring); a lane's 4 or 8 bytes stay inside one 16-byte chunk
+  const bool sw = a.swz && b >= 8;
+  auto pg = [&](int64_t o) -> uint8_t* { return page + (sw ? swz_off(o) : o); };
+  auto rg = [&](int o) -> uint32_t { return sdst + static_cast<uint32_t>(sw ? swz_off(o) : o); };
   if (b == 16) {  // K [P][D] | V [P][D] bf16: this lane's D/32 values
     const int rowb = 2 * D;
     if (D == 64) {
       if (own) {
-        reinterpret_cast<uint32_t*>(page + slot * rowb)[lane] = rk.x;
-        reinterpret_cast<uint32_t*>(page + (P + slot) * rowb)[lane] = rv.x;
+        *reinterpret_cast<uint32_t*>(pg(slot * rowb + 4 * lane)) = rk.x;
+        *reinterpret_cast<uint32_t*>(pg((P + slot) * rowb + 4 * lane)) = rv.x;
       }
       if (to_ring) {
-        sts32(sdst + 4 * lane, rk.x);
-        sts32(sdst + P * rowb + 4 * lane, rv.x);
+        sts32(rg(4 * lane), rk.x);
+        sts32(rg(P * rowb + 4 * lane), rv.x);
       }
     } else {
       if (own) {
-        reinterpret_cast<uint2*>(page + slot * rowb)[lane] = rk;
-        reinterpret_cast<uint2*>(page + (P + slot) * rowb)[lane] = rv;
+        *reinterpret_cast<uint2*>(pg(slot * rowb + 8 * lane)) = rk;
+        *reinterpret_cast<uint2*>(pg((P + slot) * rowb + 8 * lane)) = rv;
       }
       if (to_ring) {
-        sts32(sdst + 8 * lane, rk.x);
-        sts32(sdst + 8 * lane + 4, rk.y);
-        sts32(sdst + P * rowb + 8 * lane, rv.x);
-        sts32(sdst + P * rowb + 8 * lane + 4, rv.y);
+        sts32(rg(8 * lane), rk.x);
+        sts32(rg(8 * lane) + 4, rk.y);
+        sts32(rg(P * rowb + 8 * lane), rv.x);
+        sts32(rg(P * rowb + 8 * lane) + 4, rv.y);
       }
     }
     return;
@@ -915,11 +949,11 @@ __device__ __forceinline__ void step_token_rows(const AttnKernelArgs& ka, uint2 
     bad |= r.bad;
     const int coff = (kv * P + slot) * rowb, soff = 2 * P * rowb + kv * P * ng * 4;
     if (own) {
-      if (r.code_idx >= 0) reinterpret_cast<uint32_t*>(page + coff)[r.code_idx] = r.code_word;
+      if (r.code_idx >= 0) *reinterpret_cast<uint32_t*>(pg(coff + 4 * r.code_idx)) = r.code_word;
       if (r.sz_idx >= 0) reinterpret_cast<uint32_t*>(page + soff + slot * ng * 4)[r.sz_idx] = r.sz_word;
     }
     if (to_ring) {
-      if (r.code_idx >= 0) sts32(sdst + kv * P * rowb + 4 * r.code_idx, r.code_word);
+      if (r.code_idx >= 0) sts32(rg(kv * P * rowb + 4 * r.code_idx), r.code_word);
       if (r.sz_idx >= 0) sts32(sdst + soff + 4 * r.sz_idx, r.sz_word);
     }
   }

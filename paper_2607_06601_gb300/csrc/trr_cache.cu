@@ -20,7 +20,7 @@ LayerArgs layer_args(const Layout& l, const Views& v, int layer) {
   a.maxctx = l.maxctx; a.MP = l.MP; a.W32 = l.W32; a.units = l.units; a.pos_split = l.pos_split;
   a.s_cap = l.s_cap;
   a.split_bytes = l.split_bytes; a.skip_writes_kv = l.skip_writes_kv;
-  a.head_modes = l.head_modes; a.maskb = static_cast<int>(l.maskb);
+  a.head_modes = l.head_modes; a.maskb = static_cast<int>(l.maskb); a.swz = l.swz;
   a.hdr = static_cast<int>(l.hdr);
   for (int c = 0; c < kClasses; ++c) {
     a.cap[c] = l.cap[c];
@@ -77,6 +77,7 @@ static trr_status make_layout(const trr_cache_config* c, Layout* l) {
   l->split_bytes = c->split_bytes ? c->split_bytes : 24576;
   l->skip_writes_kv = c->skip_writes_kv;
   l->head_modes = c->head_modes;
+  l->swz = uses_mma(l->Hq, l->Hkv, l->d, l->G, l->head_modes) ? 0 : 1;
   l->hdr = roundup(4 * static_cast<int64_t>(l->P), 128);
   // per-head modes: each KV head's slice of a page ends with 16 bytes holding its 64-bit
   // presence mask, so that the copy of a slice brings its mask

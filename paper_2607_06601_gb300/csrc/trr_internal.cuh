@@ -46,6 +46,7 @@ struct Layout {
   int L, S, Hq, Hkv, d, G, P, maxctx, MP, W32;
   int cap[kClasses];
   int max_append, max_queries, split_bytes, skip_writes_kv, head_modes;
+  int swz;        // 8- and 16-bit code rows stored swizzled (caches of the CUDA-core consumer)
   int units;      // attention work units per query split (one per query head)
   int pos_split;  // key positions per split at least (split_bytes of 8-bit tokens)
   int s_cap;      // most splits one query is cut into
@@ -65,6 +66,23 @@ __host__ __device__ inline int splits_of(int range, int pos_split, int P, int s_
   const int by_pages = ((range + P - 1) / P + 2 * kClasses + kItemMaxPages - 1) / kItemMaxPages;
   const int ns = by_len > by_pages ? by_len : by_pages;
   return ns < s_cap ? ns : s_cap;
+}
+
+// The tensor-core consumer serves query groups (g >= 2) whose (head, group) columns fit
+// one 8-wide mma tile, without per-head modes; every other cache is read by the
+// CUDA-core consumer, whose lanes read 8- and 16-bit code rows in a pattern that the
+// swizzle below makes free of shared-memory bank conflicts.
+__host__ __device__ inline bool uses_mma(int Hq, int Hkv, int d, int G, int head_modes) {
+  const int g = Hq / Hkv, ng = d / G;
+  return !head_modes && g >= 2 && g * ng <= 8;
+}
+
+// Where byte o of a KV slice's K or V code region (o counted from the slice's start)
+// is stored in a swizzled cache, for 8- and 16-bit pages: each 128-byte line keeps its
+// 16-byte chunks in the order chunk ^ (line % 8).  Both regions start on a line of the
+// slice.  2- and 4-bit rows, scales, positions and masks are stored plainly.
+__host__ __device__ inline int64_t swz_off(int64_t o) {
+  return (o & ~static_cast<int64_t>(127)) | ((((o >> 4) ^ (o >> 7)) & 7) << 4) | (o & 15);
 }
 
 // Per-entry plan written by the append plan kernel.
@@ -114,6 +132,7 @@ inline Views make_views(const Layout& l, void* base) {
 struct LayerArgs {
   int layer, S, Hq, Hkv, d, G, P, maxctx, MP, W32, units, pos_split, s_cap, cnt_stride, split_bytes, skip_writes_kv;
   int head_modes;      // modes are [n][Hq]; each KV head's slice ends with its presence mask
+  int swz;             // 8- and 16-bit code rows stored swizzled (see swz_off)
   uint64_t wait_ns;    // bound of an in-kernel wait before the kernel reports TRR_ERR_TIMEOUT
   int maskb;           // bytes that end a slice for its presence mask (16, or 0 without head_modes)
   int cap[kClasses];

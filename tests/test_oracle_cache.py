@@ -3,6 +3,7 @@ Sec. 7: tokens grouped by precision): allocation invariants, bulk == incremental
 append, the error contract, the byte layout checked by hand, and the stored values
 against the quantiser pinned in test_oracle_quantizer.py."""
 import numpy as np
+import pytest
 
 import oracle
 from paper_2607_06601_gb300.workloads import bf16_bits, bf16_to_f32
@@ -114,6 +115,37 @@ def test_byte_layout_by_hand():
                                int(np.float16(-15).view(np.uint16))]
     assert list(vc[1, :16]) == [int(15 - ramp[2 * j]) | (int(15 - ramp[2 * j + 1]) << 4)
                                 for j in range(16)]
+
+
+@pytest.mark.parametrize("Hq,Hkv,permuted", [(2, 2, True), (4, 2, False), (16, 2, True)])
+def test_chunk_order_of_wide_rows_by_hand(Hq, Hkv, permuted):
+    """One 8-bit and one 16-bit token at slot 3, d = 64, G = 32, P = 16: where every
+    16-byte chunk of their K rows is stored.  In a cache read by the CUDA-core path (MHA;
+    query groups too wide for one 8-column mma tile) line n of a slice keeps logical chunk
+    k at chunk k ^ (n % 8); in a tensor-core cache (g = 2: 4 columns) rows are plain."""
+    d, G, P, slot = 64, 32, 16, 3
+    o = oracle.OracleCache(1, 2, Hq, Hkv, d, G, P, 32, [2] * 4)
+    rng = np.random.default_rng(3)
+    K = bf16_bits(rng.standard_normal((2, Hkv, d), dtype=np.float32))
+    V = bf16_bits(rng.standard_normal((2, Hkv, d), dtype=np.float32))
+    for p in range(slot + 1):  # the fourth token of each sequence lands in slot 3
+        assert o.append(0, [0, 1], [p, p], K, V, [16, 8], [FULL, FULL]) == 0
+    for b, c, seq in ((16, 3, 0), (8, 2, 1)):
+        rowb = d * b // 8
+        page = o.region(f"pool{b}")[:o.page_bytes(c)]
+        sl = page[o.hdr_bytes:o.hdr_bytes + o.slice_bytes(c)]     # KV head 0
+        if b == 16:
+            logical = K[seq, 0].view(np.uint8)
+        else:  # 8-bit codes: one byte each, in element order
+            _, _, c0, _ = oracle.quantize_group(K[seq, 0][:32], 8)
+            _, _, c1, _ = oracle.quantize_group(K[seq, 0][32:], 8)
+            logical = np.concatenate([c0, c1]).astype(np.uint8)
+        assert logical.size == rowb
+        for k in range(rowb // 16):
+            x = slot * rowb + 16 * k                       # logical offset in the slice
+            n, ch = x // 128, (x // 16) % 8
+            at = n * 128 + ((ch ^ (n % 8)) if permuted else ch) * 16
+            assert np.array_equal(sl[at:at + 16], logical[16 * k:16 * k + 16]), (b, k)
 
 
 def test_stored_values_are_the_quantiser_output():

@@ -33,6 +33,27 @@ def _heads_store(hmodes, Hq, Hkv, swk=0):
     return np.stack([(hm[:, j * g:(j + 1) * g] != SKIP).any(1) | bool(swk) for j in range(Hkv)], 1)
 
 
+def _permuted(Hq, Hkv, d, G, head_modes):
+    """The documented rule: 8- and 16-bit code rows keep a permuted chunk order in every
+    cache except those of query groups g >= 2 whose g * (d / G) columns fit 8, without
+    per-head modes (the tensor-core path's)."""
+    g = Hq // Hkv
+    return not (not head_modes and g >= 2 and g * (d // G) <= 8)
+
+
+def _logical(sl, b, code_bytes):
+    """A slice's bytes with its K and V code regions (the first code_bytes) back in
+    logical order: line n keeps logical chunk k at chunk k ^ (n % 8)."""
+    out = sl.copy()
+    if b < 8:
+        return out
+    for n in range(code_bytes // 128):
+        for k in range(8):
+            src = n * 128 + (k ^ (n % 8)) * 16
+            out[n * 128 + k * 16:n * 128 + k * 16 + 16] = sl[src:src + 16]
+    return out
+
+
 @pytest.mark.parametrize("Hq,Hkv", [(4, 2), (4, 4), (8, 1)])
 def test_equal_head_modes_match_the_per_token_cache(Hq, Hkv):
     rng = np.random.default_rng(Hq * 10 + Hkv)
@@ -59,10 +80,13 @@ def test_equal_head_modes_match_the_per_token_cache(Hq, Hkv):
             a0, b0 = pid * tok.page_bytes(c), pid * hed.page_bytes(c)
             assert np.array_equal(pt[a0:a0 + tok.hdr_bytes], ph[b0:b0 + hed.hdr_bytes]), (b, pid)
             masks = []
+            code_bytes = 2 * P * (d * b // 8 if b < 16 else 2 * d)
             for j in range(Hkv):  # each KV head's slice: the same bytes, then its mask, 8 zeros
                 sa = pt[a0 + tok.hdr_bytes + j * sl_t:][:sl_t]
                 sb = ph[b0 + hed.hdr_bytes + j * (sl_t + 16):][:sl_t + 16]
-                assert np.array_equal(sa, sb[:sl_t]), (b, pid, j)
+                if _permuted(Hq, Hkv, d, 32, 0):
+                    sa = _logical(sa, b, code_bytes)
+                assert np.array_equal(sa, _logical(sb[:sl_t], b, code_bytes)), (b, pid, j)
                 masks.append(int(sb[sl_t:sl_t + 8].view(np.uint64)[0]))
                 assert not sb[sl_t + 8:].any()
             fill = bin(masks[0]).count("1")
