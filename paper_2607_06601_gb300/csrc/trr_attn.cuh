@@ -1046,7 +1046,7 @@ struct CtaRing {
 // by the previous kernel) are in.  Before the wait the producer takes ring space only
 // where it is free, never waiting for consumers.  Nothing is written to global memory
 // before the wait.
-template <int D, bool STEP>
+template <int D, bool STEP, bool HM>
 __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, int NQB, const int* pre, int* ent,
                                              const CtaRing& cr, int lane) {
   const LayerArgs& a = ka.a;
@@ -1216,15 +1216,39 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
     // per-head modes those read by a full head of the block (pages before the local
     // window) and those read by any head of the block (the other pages)
     unsigned need_full = (1u << nkv) - 1u, need_any = need_full;
-    if (a.head_modes && !err) {
-      const int hm = lane < nh ? ka.modes[static_cast<int64_t>(q) * a.Hq + h0 + lane] : 0;
+    // per-head modes: the block's heads, slot s (a consumer warp) taking head hsel byte s.
+    // With up to 32 query heads a query's heads are ranked by mode (full, local, skip;
+    // by index within a mode) and block qb takes ranks qb * hpu .. + nh - 1, so that the
+    // full heads share as few blocks as possible (a block reads the pages of its widest
+    // mode); else (-1) slot s takes head h0 + s.  need_full / need_any are then masks of
+    // slots, and a page brings one KV slice per slot that needs it.
+    int hsel = -1;
+    if (HM && !err) {
+      if (a.Hq <= 32) {
+        const int ml = lane < a.Hq ? ka.modes[static_cast<int64_t>(q) * a.Hq + lane] : TRR_MODE_FULL + 1;
+        const int cl = ml == TRR_MODE_FULL ? 0 : ml == TRR_MODE_LOCAL ? 1 : ml == TRR_MODE_SKIP ? 2 : 3;
+        const unsigned b0 = __ballot_sync(0xffffffffu, cl == 0), b1 = __ballot_sync(0xffffffffu, cl == 1);
+        const unsigned b2 = __ballot_sync(0xffffffffu, cl == 2), lt = (1u << lane) - 1u;
+        const int rank = cl == 0 ? __popc(b0 & lt)
+                         : cl == 1 ? __popc(b0) + __popc(b1 & lt)
+                         : cl == 2 ? __popc(b0) + __popc(b1) + __popc(b2 & lt) : 255;
+        hsel = 0;
+#pragma unroll
+        for (int sl = 0; sl < kNcw; ++sl) {
+          const unsigned hit = __ballot_sync(0xffffffffu, rank == h0 + sl);
+          hsel |= (hit ? __ffs(hit) - 1 : 0) << (8 * sl);
+        }
+      }
+      const int hs = hsel >= 0 ? (hsel >> (8 * (lane & 3))) & 255 : h0 + lane;  // lane < nh: slot lane's head
+      const int hm = lane < nh ? ka.modes[static_cast<int64_t>(q) * a.Hq + hs] : 0;
       bmode = static_cast<int>(__reduce_max_sync(0xffffffffu, static_cast<unsigned>(hm)));
       hpack = static_cast<int>(__reduce_or_sync(0xffffffffu, static_cast<unsigned>(hm) << (2 * (lane & 15))));
-      const unsigned kbit = 1u << (((h0 + (lane & 15)) / g - kv0) & 31);
-      need_full = __reduce_or_sync(0xffffffffu, (lane < nh && hm == TRR_MODE_FULL) ? kbit : 0u);
-      need_any = __reduce_or_sync(0xffffffffu, (lane < nh && hm != TRR_MODE_SKIP) ? kbit : 0u);
+      need_full = __ballot_sync(0xffffffffu, lane < nh && hm == TRR_MODE_FULL);
+      need_any = __ballot_sync(0xffffffffu, lane < nh && hm != TRR_MODE_SKIP);
     }
-    if (a.head_modes && !err && bmode == TRR_MODE_LOCAL) {
+    // the query head of slot s (per-head modes; s < nh)
+    auto slot_head = [&](int sl) -> int { return hsel >= 0 ? (hsel >> (8 * sl)) & 255 : h0 + sl; };
+    if (HM && !err && bmode == TRR_MODE_LOCAL) {
       // per-head modes, a block of local and skip heads in a query whose widest head is
       // full: the block's own split count, from its window; its splits past that have
       // nothing to do, and its heads merge that many partials
@@ -1244,15 +1268,18 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
     const int lo = bmode == TRR_MODE_FULL ? 0 : max(0, t - w + 1);
     int wid = -1, wmeta = 0, wfirst = 0, wlast = INT_MAX, T = 0;
     if (!err && bmode != TRR_MODE_SKIP)
-      T = plan_split(a, P, seq, lo, t, sp, ns, lane, wid, wmeta, a.head_modes ? &wfirst : nullptr,
-                     a.head_modes ? &wlast : nullptr);
+      T = plan_split(a, P, seq, lo, t, sp, ns, lane, wid, wmeta, HM ? &wfirst : nullptr,
+                     HM ? &wlast : nullptr);
     if (err || bmode == TRR_MODE_SKIP) {
       // zero rows (once per block); the error of the lowest query; a skip token that
       // stores KV has its rows written here
       ensure_waited();
       if (sp == 0) {
-        uint4* o = reinterpret_cast<uint4*>(ka.out + (static_cast<int64_t>(q) * a.Hq + h0) * D);
-        for (int i = lane; i < nh * D / 8; i += 32) o[i] = make_uint4(0, 0, 0, 0);
+        for (int i = lane; i < nh * D / 8; i += 32) {  // slot i / (D / 8)'s row
+          const int h = HM ? slot_head(i / (D / 8)) : h0 + i / (D / 8);
+          reinterpret_cast<uint4*>(ka.out + (static_cast<int64_t>(q) * a.Hq + h) * D)[i % (D / 8)] =
+              make_uint4(0, 0, 0, 0);
+        }
       }
       if (!STEP && err && qb == 0 && lane == 0) atomicMin(&a.lctl[kFirstBadQuery], (ka.q0 + q) * 16 + err);
       if (STEP && !call_failed() && sp == 0 && ent[2 * q] >= 0) {
@@ -1272,7 +1299,7 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
       const int lo_local = max(0, t - w + 1);
       // per-head modes: a page before the local window is read by the block's full heads
       // only; a page across the window's start brings its slot positions
-      if (a.head_modes && lane < T) {
+      if (HM && lane < T) {
         if (wlast < lo_local) wmeta |= kEarly;
         else if (wfirst < lo_local) wmeta |= kMask;
       }
@@ -1291,9 +1318,15 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
         }
         const bool only = T == 0 && !has_new;
         const int meta = kQRows | kFirst | (only ? (kLast | kNoPage) : 0) | (qb << 16);
-        const int4 ra = make_int4(meta, off, q, lo), rc = make_int4(hpack, max(0, t - w + 1), -1, 0);
+        const int4 ra = make_int4(meta, off, q, lo), rc = make_int4(hpack, max(0, t - w + 1), -1, hsel);
         const uint16_t* src = ka.q + (static_cast<int64_t>(q) * a.Hq + h0) * D;
-        if (waited) {
+        if (HM) {  // the slots' rows, each from its head (no early mode with head modes)
+          const uint32_t slot = push(ra, rb, rc, taken, need);
+          if (lane == 0)
+            for (int sl = 0; sl < nh; ++sl)
+              bulk_g2s(cr.ring + off + sl * D * 2, ka.q + (static_cast<int64_t>(q) * a.Hq + slot_head(sl)) * D, D * 2,
+                       &cr.full[slot]);
+        } else if (waited) {
           const uint32_t slot = push(ra, rb, rc, taken, need);
           if (lane == 0) bulk_g2s(cr.ring + off, src, need, &cr.full[slot]);
         } else {  // its slot now, its record and copy after the wait
@@ -1371,7 +1404,7 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
         const unsigned needed = __shfl_sync(0xffffffffu, pg_need, j);
         const int slice = geo & 0xfffff, maxk = geo >> 20;
         const unsigned all = (1u << nkv) - 1u;
-        if (!a.head_modes && !(pm & kMask) && needed == all && nkv <= maxk) {
+        if (!HM && !(pm & kMask) && needed == all && nkv <= maxk) {
           // a run of full pages of this class, every KV head of the block: one stage
           // holding up to R/2 bytes of them (a page's slices after the other), one copy
           // per page; only the run's last page may hold fewer than P tokens
@@ -1398,6 +1431,41 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
             if (lane == 0) bulk_g2s(cr.ring + off + r * pb, pg + a.hdr + static_cast<int64_t>(kv0) * slice, pb, &cr.full[slot]);
           }
           j += run - 1;
+          continue;
+        }
+        if (HM) {  // per-head modes: the needed slots' slices, at most maxk a stage
+          unsigned rest = needed;
+          while (rest && ok) {
+            unsigned chunk = 0;
+            int nk = 0;
+            while (rest && nk < maxk) {
+              chunk |= rest & (0u - rest);
+              rest &= rest - 1u;
+              ++nk;
+            }
+            const int posb = (pm & kMask) ? 4 * P : 0;
+            const int need = nk * slice + posb;
+            int taken = 0;
+            const int off = reserve_any(need, taken);
+            if (off < 0) {
+              ok = false;
+              break;
+            }
+            const bool last = j == T - 1 && rest == 0 && new_done;
+            const int meta = pm | (last ? kLast : 0) | (qb << 16);
+            const uint32_t slot = push(make_int4(meta, off, q, lo), rb,
+                                       make_int4(static_cast<int>(chunk), nk | (1 << 8), posb ? off + nk * slice : -1, slice),
+                                       taken, need);
+            if (lane == 0) {
+              int pos = 0;
+              for (unsigned m = chunk; m; m &= m - 1u, ++pos) {
+                const int kvh = slot_head(__ffs(m) - 1) / g;
+                bulk_g2s(cr.ring + off + pos * slice, page + a.hdr + static_cast<int64_t>(kvh) * slice, slice,
+                         &cr.full[slot]);
+              }
+              if (posb) bulk_g2s(cr.ring + off + nk * slice, page, posb, &cr.full[slot]);
+            }
+          }
           continue;
         }
         // one stage per run of consecutive needed KV heads, at most maxk slices each
@@ -1659,6 +1727,10 @@ __device__ __forceinline__ void run_consumer_cc(const AttnKernelArgs& ka, const 
       const int qb = (meta >> 16) & 0x7fff;
       u_h = qb * kNcw + cw;
       active = u_h < a.Hq;
+      if (HM && active) {  // the head of this warp's slot (ranked by mode; or h0 + slot)
+        const int hsel = lds128i(rec + 32).w;
+        if (hsel >= 0) u_h = (hsel >> (8 * cw)) & 255;
+      }
       u_kvi = u_h / g - (qb * kNcw) / g;
       u_q = ra.z;
       u_lo = ra.w;
@@ -1708,7 +1780,10 @@ __device__ __forceinline__ void run_consumer_cc(const AttnKernelArgs& ka, const 
     } else if (active) {
       const int4 rc = lds128i(rec + 32);
       const int nks = rc.y & 255, npg = rc.y >> 8;  // KV slices per page, pages of the stage
-      if (u_kvi >= rc.x && u_kvi < rc.x + nks && !(HM && u_local && (meta & kEarly))) {
+      // per-head modes: the stage brings one slice per slot of its mask (rc.x), in slot
+      // order; otherwise KV slices rc.x .. rc.x + nks - 1 of the block
+      const bool mine = HM ? ((static_cast<unsigned>(rc.x) >> cw) & 1u) != 0 : (u_kvi >= rc.x && u_kvi < rc.x + nks);
+      if (mine && !(HM && u_local && (meta & kEarly))) {
         const int cls = meta & 3, fill = (meta >> 2) & 127;  // the last page's fill; the others are full
         if (STEP && rc.z == kNewRows) {  // the query's own token: this warp's KV head (warps that
                                          // share a KV head write the same bytes); the keys past
@@ -1722,7 +1797,8 @@ __device__ __forceinline__ void run_consumer_cc(const AttnKernelArgs& ka, const 
         }
         const bool masked = meta & kMask;
         for (int pg = 0; pg < npg; ++pg) {
-          const uint32_t s0 = smem_u32(cr.ring + ra.y + (pg * nks + u_kvi - rc.x) * rc.w);
+          const int idx = HM ? __popc(static_cast<unsigned>(rc.x) & ((1u << cw) - 1u)) : u_kvi - rc.x;
+          const uint32_t s0 = smem_u32(cr.ring + ra.y + (pg * nks + idx) * rc.w);
           const int f = pg == npg - 1 ? fill : P;
           const uint32_t sp = masked ? smem_u32(cr.ring + rc.z) : s0;
           uint64_t pm = ~0ull;  // per-head modes: this KV head's presence mask, which ends
@@ -2375,7 +2451,7 @@ __global__ void __launch_bounds__(32 * (kNcw + 1), cc_ctas_per_sm(D))
   const int NQB = (ka.a.Hq + ka.hpu - 1) / ka.hpu;
   int *pre, *ent;
   const CtaRing cr = attn_prologue<STEP>(ka, smem, P, NQB, pre, ent);
-  if (warp == 0) run_producer<D, STEP>(ka, P, NQB, pre, ent, cr, lane);
+  if (warp == 0) run_producer<D, STEP, HM>(ka, P, NQB, pre, ent, cr, lane);
   else run_consumer_cc<D, P, cc_elems(D), HM, STEP>(ka, cr, ent, warp - 1, lane);
   attn_epilogue<STEP>(ka, ent);
 }
@@ -2390,7 +2466,7 @@ __global__ void __launch_bounds__(32 * (kNcw + 1), kMmaCtasPerSm) attn_mma_kerne
   int *pre, *ent;
   const CtaRing cr = attn_prologue<STEP>(ka, smem, P, NQB, pre, ent);
   if (warp == 0) {
-    run_producer<D, STEP>(ka, P, NQB, pre, ent, cr, lane);
+    run_producer<D, STEP, false>(ka, P, NQB, pre, ent, cr, lane);
   } else {
     const AttnSmem lay(ka.ring_bytes, ka.n, ka.scr_floats, STEP);
     float* scr = reinterpret_cast<float*>(smem + lay.scr) + (warp - 1) * ka.scr_floats;
