@@ -678,6 +678,35 @@ __device__ __forceinline__ int plan_split(const LayerArgs& a, int P, int seq, in
   return T;
 }
 
+// Key positions that query q's head blocks read in all (r: its widest head's range):
+// NQB times r, or with per-head modes each block its own widest head's range, the heads
+// assigned to blocks as the producer assigns them (ranked by mode when Hq <= 32, in index
+// order otherwise).  It sizes the splits only.
+__device__ __forceinline__ long long query_block_work(const AttnKernelArgs& ka, int q, int t, int w, int r,
+                                                      int NQB) {
+  const LayerArgs& a = ka.a;
+  if (!a.head_modes || ka.mode_logits || r == 0) return static_cast<long long>(r) * NQB;
+  const uint8_t* row = ka.modes + static_cast<int64_t>(q) * a.Hq;
+  if (a.Hq <= 32) {
+    int nf = 0, nl = 0;
+    for (int h = 0; h < a.Hq; ++h) {
+      nf += row[h] == TRR_MODE_FULL;
+      nl += row[h] == TRR_MODE_LOCAL;
+    }
+    const int bf = (nf + ka.hpu - 1) / ka.hpu;               // blocks holding a full head
+    const int bl = (nf + nl + ka.hpu - 1) / ka.hpu - bf;     // blocks led by a local head
+    return static_cast<long long>(bf) * query_range(t, TRR_MODE_FULL, w) +
+           (bl > 0 ? static_cast<long long>(bl) * query_range(t, TRR_MODE_LOCAL, w) : 0ll);
+  }
+  long long s = 0;
+  for (int h0 = 0; h0 < a.Hq; h0 += ka.hpu) {
+    int m = 0;
+    for (int h = h0; h < min(a.Hq, h0 + ka.hpu); ++h) m = max(m, static_cast<int>(row[h]));
+    s += query_range(t, m, w);
+  }
+  return s;
+}
+
 // The work units of a call, computed the same way by every CTA: query q gets ns_q
 // splits from its key range (per-head modes: its widest head's); pre[q] numbers its
 // first split, pre[n] counts them all, pre[n + 1] is the call's key positions per split.
@@ -691,7 +720,7 @@ __device__ __forceinline__ void plan_units(const AttnKernelArgs& ka, int P, int 
     const int w = ka.windows ? ka.windows[q] : ka.window_scalar;
     const int r = query_error(a, seq, t, mode, any_local, w) ? 0 : query_range(t, mode, w);
     pre[q] = r;
-    rsum += r;
+    rsum += query_block_work(ka, q, t, w, r, NQB);
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) rsum += __shfl_xor_sync(0xffffffffu, rsum, o);
@@ -703,10 +732,12 @@ __device__ __forceinline__ void plan_units(const AttnKernelArgs& ka, int P, int 
   // chains, and a second unit on a CTA doubles the call); a large one up to
   // kUnitsPerCta per CTA, each of at least kMinUnitPositions positions per head block
   // (the producer plans the next unit while the consumers work on this one); never
-  // below pos_split.  Binary32 arithmetic: the same result in every CTA, and it only
+  // below pos_split.  The work counts each head block's own range, so that per-head
+  // modes, whose blocks past the full heads read only a window or nothing, size their
+  // units by the blocks that read pages.  Binary32 arithmetic: the same result in every CTA, and it only
   // sizes the splits.
   const float ctas = static_cast<float>(gridDim.x);
-  const float rs = static_cast<float>(rsum) * static_cast<float>(NQB);
+  const float rs = static_cast<float>(rsum);
   const float want = fmaxf(0.8f * ctas, fminf(static_cast<float>(kUnitsPerCta) * ctas, rs / kMinUnitPositions));
   const float by_work = ceilf(rs / want);
   const int pos_split = by_work > static_cast<float>(a.pos_split) ? static_cast<int>(fminf(by_work, 1073741824.f))
@@ -1183,8 +1214,11 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
   // counter: a CTA takes its first unit as it starts and another only once its consumers
   // are done with the current one.  The CTAs that start last (on SM slots the previous
   // kernel frees as it ends) then get the last units, or none.  A larger call gives each
-  // CTA its own first unit and lets the producer take the next from the counter while
-  // the consumers work on the current one.
+  // CTA its own first unit and lets the producer take the next from the counter once it
+  // has pushed every stage of the current one, while the consumers still work on it: a
+  // CTA whose unit turns out empty (a block of local or skip heads past its own splits)
+  // or short asks again before the busy CTAs do, and takes the units they would have
+  // queued.
   const bool on_demand = total <= static_cast<int>(gridDim.x);
   int u = static_cast<int>(blockIdx.x);
   if (on_demand) {
@@ -1193,7 +1227,9 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
   }
   while (u < total) {
     int u_next = 0;
-    if (!on_demand && lane == 0) u_next = static_cast<int>(gridDim.x) + atomicAdd(&a.lctl[kNextUnit], 1);  // used last
+    auto take_next = [&]() {
+      if (lane == 0) u_next = (on_demand ? 0 : static_cast<int>(gridDim.x)) + atomicAdd(&a.lctl[kNextUnit], 1);
+    };
     const int un = u / NQB, qb = u - un * NQB;
     int lo_q = 0, hi_q = n;  // the query of split un: pre[q] <= un < pre[q + 1]
     while (hi_q - lo_q > 1) {
@@ -1255,7 +1291,7 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
       ns = min(ns, splits_of(query_range(t, TRR_MODE_LOCAL, w), pre[n + 1], P, a.s_cap));
       if (sp >= ns) {
         __syncwarp();
-        if (on_demand && lane == 0) u_next = atomicAdd(&a.lctl[kNextUnit], 1);
+        take_next();
         u = __shfl_sync(0xffffffffu, u_next, 0);
         continue;
       }
@@ -1500,8 +1536,8 @@ __device__ __forceinline__ void run_producer(const AttnKernelArgs& ka, int P, in
     if (on_demand) {  // the consumers first finish this unit
       while (ok && released < pushed) ok = release_one();
       if (!ok) break;
-      if (lane == 0) u_next = atomicAdd(&a.lctl[kNextUnit], 1);
     }
+    take_next();
     u = __shfl_sync(0xffffffffu, u_next, 0);
   }
   if (ok) {
