@@ -734,8 +734,8 @@ __device__ __forceinline__ void plan_units(const AttnKernelArgs& ka, int P, int 
   // (the producer plans the next unit while the consumers work on this one); never
   // below pos_split.  The work counts each head block's own range, so that per-head
   // modes, whose blocks past the full heads read only a window or nothing, size their
-  // units by the blocks that read pages.  Binary32 arithmetic: the same result in every CTA, and it only
-  // sizes the splits.
+  // units by the blocks that read pages.  Binary32 arithmetic: the same result in every
+  // CTA, and it only sizes the splits.
   const float ctas = static_cast<float>(gridDim.x);
   const float rs = static_cast<float>(rsum);
   const float want = fmaxf(0.8f * ctas, fminf(static_cast<float>(kUnitsPerCta) * ctas, rs / kMinUnitPositions));
